@@ -1,0 +1,162 @@
+/*
+ * tq.h - C ABI of the packed ternary (W1.58A16) linear layer.
+ *
+ * What is computed (paper: "Model and Representation", eq. for W-hat):
+ * every targeted projection W (N rows = outputs, K columns = inputs) is a
+ * ternary reconstruction offset + alpha0*T0 + alpha1*T1, the second plane
+ * only on salience-selected parts.  This library uses the per-group reading:
+ * with g = floor(k / 128),
+ *
+ *     W[n][k] = s1[n][g] * T1[n][k] + off[n][g] + sal[n][g] * s2[n][g] * T2[n][k]
+ *
+ * T1, T2 in {-1, 0, +1}; s1, off, s2 fp16; sal a 1-bit salience map.
+ * Activations x and outputs y stay fp16 (weight-only A16, paper
+ * "Model and Representation").  The layer computes y[m][n] = sum_k x[m][k] W[n][k]
+ * with fp32 accumulation, directly from the packed bytes (paper
+ * "Direct Packed Execution").
+ *
+ * Packed ("lattice-aware") format (paper "Packing: From Quantization to
+ * Serialization"; the byte layout itself is not printed there, this is the
+ * library's definition):
+ *   - one byte holds five trits as a base-3 numeral, digit d = t + 1, first
+ *     trit least significant: byte = sum_{i<5} d_i * 3^i  (0..242; 243..255
+ *     are invalid).  3^5 = 243 <= 256 gives 1.6 bits per trit against the
+ *     log2(3) = 1.585-bit bound of the paper's eq. b_T.
+ *   - a 128-trit group is 26 bytes: bytes 0..24 hold trits 5j..5j+4, byte 25
+ *     holds trits 125..127 in digits 0..2 and pad digits 3,4 = 1 (t = 0).
+ *   - plane 1 rows are TQ_GROUP_BYTES * G bytes padded with 0x00 to a
+ *     multiple of 16 (tq_row_bytes).
+ *   - plane 2 stores only the salient groups, 26 bytes each, in (n, g) order;
+ *     rowptr[n] is the number of salient groups in rows 0..n-1.
+ *
+ * Conventions (all entry points):
+ *   - every pointer argument except the tq_weight / tq_problem structs
+ *     themselves refers to DEVICE memory owned by the caller;
+ *   - every call is asynchronous on `stream` (a cudaStream_t passed as void*,
+ *     NULL = legacy default stream); the library never allocates device
+ *     memory, never synchronizes and never throws across the ABI;
+ *   - argument errors (null pointers, shapes, alignment) are returned
+ *     synchronously and nothing is launched;
+ *   - data errors found by the codec kernels are OR-ed into the caller's
+ *     device word *d_status (TQ_DATA_* bits); the caller zeroes it before the
+ *     call and reads it after synchronizing;
+ *   - TQ_ERR_CUDA means a launch failed (cudaGetLastError after launch).
+ */
+#ifndef TQ_H_
+#define TQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TQ_GROUP 128        /* trits per group along K                       */
+#define TQ_GROUP_BYTES 26   /* bytes per packed 128-trit group                */
+#define TQ_TRITS_PER_BYTE 5 /* 3^5 = 243 <= 256                               */
+#define TQ_MAX_SKINNY_M 16  /* M <= this runs the decode (GEMV / skinny) path */
+
+typedef enum {
+  TQ_OK = 0,
+  TQ_ERR_NULL = -1,     /* a required pointer is NULL                     */
+  TQ_ERR_SHAPE = -2,    /* M, N or K out of range, K % 128 != 0, group != 128 */
+  TQ_ERR_ALIGN = -3,    /* a pointer is not 16-byte aligned               */
+  TQ_ERR_CODE = -4,     /* reserved: invalid trit code (reported in d_status) */
+  TQ_ERR_BYTE = -5,     /* reserved: invalid packed byte (d_status)       */
+  TQ_ERR_SALIENCE = -6, /* descriptor nnz / salience inconsistent          */
+  TQ_ERR_CUDA = -7,     /* a CUDA launch or query failed                  */
+  TQ_ERR_TIMEOUT = -8   /* a bounded device wait ran out                  */
+} tq_status;
+
+/* Bits OR-ed into *d_status by the codec kernels. */
+#define TQ_DATA_BAD_CODE 1u     /* a trit code not in {-1, 0, +1}                */
+#define TQ_DATA_T2_OUTSIDE 2u   /* T2 != 0 in a group whose salience bit is 0    */
+#define TQ_DATA_BAD_BYTE 4u     /* a packed byte > 242                           */
+#define TQ_DATA_BAD_PAD 8u      /* a nonzero pad digit (tail byte) or pad byte   */
+#define TQ_DATA_BAD_ROWPTR 16u  /* rowptr disagrees with the salience map        */
+
+/* A packed projection.  All pointers: device memory owned by the caller. */
+typedef struct {
+  int32_t N, K;             /* rows (outputs), columns (inputs); K % 128 == 0  */
+  int32_t group;            /* must be TQ_GROUP                                */
+  const uint8_t *plane1;    /* [N][tq_row_bytes(K)], 16-byte aligned           */
+  const uint32_t *salience; /* [N][tq_sal_words(K)], bit g%32 of word g/32     */
+  const int32_t *rowptr;    /* [N+1], exclusive prefix count of salient groups */
+  const uint8_t *plane2;    /* [nnz][26]; may be NULL when nnz == 0            */
+  const uint16_t *scale1;   /* fp16 bits [N][G]                                */
+  const uint16_t *offset;   /* fp16 bits [N][G]                                */
+  const uint16_t *scale2;   /* fp16 bits [nnz]; may be NULL when nnz == 0      */
+  int64_t nnz;              /* number of salient groups = rowptr[N]            */
+} tq_weight;
+
+/* Bytes of one packed plane-1 row: roundup(26 * K / 128, 16).  0 if K is not
+ * a positive multiple of 128. */
+size_t tq_row_bytes(int32_t K);
+/* 32-bit words of one salience row: ceil((K / 128) / 32). */
+size_t tq_sal_words(int32_t K);
+
+/* rowptr[n] = number of set salience bits in rows 0..n-1, for n = 0..N
+ * (so rowptr[N] = nnz).  sal: [N][tq_sal_words(K)].  Bits at g >= K/128 in
+ * the last word of a row must be 0, else TQ_DATA_BAD_PAD is OR-ed into
+ * *d_status and those bits are not counted. */
+tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t *rowptr,
+                             uint32_t *d_status, void *stream);
+
+/* Pack int8 trit codes into the lattice format (paper "Packing").
+ *   T1: int8 [N][K] in {-1,0,+1};  T2: int8 [N][K], nonzero only where the
+ *   group is salient (NULL means "no second plane": sal must then be all 0);
+ *   sal: [N][tq_sal_words(K)];  rowptr: [N+1] as from tq_salience_rowptr;
+ *   plane1: out [N][tq_row_bytes(K)] (pad bytes written as 0);
+ *   plane2: out [rowptr[N]][26] (NULL iff T2 is NULL).
+ * Invalid codes set TQ_DATA_BAD_CODE (the digit is clamped into the byte),
+ * T2 != 0 outside salience sets TQ_DATA_T2_OUTSIDE, a rowptr that disagrees
+ * with sal sets TQ_DATA_BAD_ROWPTR. */
+tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+                  const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *d_status,
+                  void *stream);
+
+/* Inverse of tq_pack: T1 [N][K] and (unless NULL) T2 [N][K] int8, T2 = 0 in
+ * non-salient groups.  Validates every byte: > 242 -> TQ_DATA_BAD_BYTE (the
+ * trits are written as 0), tail pad digit != 1 or row pad byte != 0 ->
+ * TQ_DATA_BAD_PAD, rowptr disagreeing with sal -> TQ_DATA_BAD_ROWPTR. */
+tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *plane2,
+                    const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                    uint32_t *d_status, void *stream);
+
+/* y = x W^T for one packed projection (paper "Direct Packed Execution").
+ *   x: fp16 [M][K] row-major, 16-byte aligned; y: fp16 [M][N] (rounded to
+ *   nearest even from the fp32 accumulator).  M >= 1.  M <= TQ_MAX_SKINNY_M
+ *   runs the decode kernel (GEMV / skinny GEMM); larger M runs the prefill
+ *   kernel (dequantized tile -> tensor-core MMA, fp32 accumulation).
+ * The packed bytes are trusted (produced by tq_pack): no per-byte
+ * validation on this path. */
+tq_status tq_linear(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
+                    uint16_t *y, void *stream);
+
+/* As tq_linear but y is fp32 [M][N] (the accumulator before rounding). */
+tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weight *w,
+                           const uint16_t *x, float *y, void *stream);
+
+/* Many independent projections in one launch (one decode step of a model:
+ * every targeted projection of every layer).  Each problem has its own
+ * weight, input and output; all share M (<= TQ_MAX_SKINNY_M).  `problems`
+ * is a HOST array read during the call (validated, then passed to the kernel
+ * by value in its launch parameters, at most TQ_MAX_BATCH entries). */
+#define TQ_MAX_BATCH 256
+typedef struct {
+  tq_weight w;
+  const uint16_t *x; /* fp16 [M][w.K] */
+  uint16_t *y;       /* fp16 [M][w.N] */
+} tq_problem;
+
+tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *stream);
+
+/* Human-readable name of a status code (static string). */
+const char *tq_status_str(tq_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TQ_H_ */
