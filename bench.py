@@ -1,0 +1,363 @@
+"""Benchmark of the packed ternary linear layer on GB300.
+
+Default workload: one Qwen3-8B decode step, linear layers only, batch M = 1
+(36 layers x {q, k, v, o, gate, up, down} = 252 packed projections, 10 % of
+groups salient), seeded synthetic weights and activations resident in HBM.
+One step = one pass over all 252 projections (tq_linear_batched: one kernel
+launch).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tq|reference]
+
+--impl reference times the CPU oracle on the host cores (the reference arm
+of this project: a plain fp64 implementation of the same layer) on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Qwen3-8B W1.58A16 GEMV: packed GB/s vs HBM peak; linear-layer tokens/s"
+HBM_FALLBACK_GBS = 6800.0
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return HBM_FALLBACK_GBS, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- workload
+def build_step(M, device, seed0=0, layers=None):
+    """Pack the 252 projections of the Qwen3-8B step on the device.  Every
+    projection's activations and outputs are views of one contiguous x / y
+    buffer (so a step's inputs move host<->device in one copy each).
+    Returns (items, x_all, y_all, packed_bytes, weights)."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    projs = wl.config_projections(2)
+    if layers is not None:
+        projs = [p for p in projs if p.layer < layers]
+    x_all = torch.empty(sum(M * p.K for p in projs), dtype=torch.float16, device=device)
+    y_all = torch.empty(sum(M * p.N for p in projs), dtype=torch.float16, device=device)
+    items, total_bytes, total_w, xo, yo = [], 0, 0, 0, 0
+    for p in projs:
+        seed = seed0 * 100003 + p.layer * 16 + p.proj
+        g = wl.gen_weights_torch(p.N, p.K, 0.1, device, seed)
+        pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+        del g
+        x = x_all[xo:xo + M * p.K].view(M, p.K)
+        x.copy_(wl.gen_x_torch(M, p.K, device, seed + 7))
+        y = y_all[yo:yo + M * p.N].view(M, p.N)
+        xo += M * p.K
+        yo += M * p.N
+        items.append((pw, x, y))
+        total_bytes += pw.packed_bytes()
+        total_w += p.N * p.K
+    torch.cuda.synchronize()
+    return items, x_all, y_all, total_bytes, total_w
+
+
+def kernel_hash():
+    import hashlib
+
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_09240_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh")):
+            h.update(open(os.path.join(csrc, f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic():
+    """dram bytes per launch of the decode kernel from the committed ncu
+    summary, or None if the kernel changed since it was captured."""
+    p = os.path.join(ROOT, "profiles", "gemv_qwen3_8b_step_traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p))
+    if d.get("kernel_hash") != kernel_hash():
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------ cpu baseline
+def oracle_sample(target_rows=None, seconds=None):
+    """Times the CPU oracle on a bounded sample of the same workload: the
+    first rows of every projection of one Qwen3-8B layer (same shapes and
+    distributions, numpy-drawn).  Returns (GB/s of packed bytes, cores,
+    description, seconds)."""
+    import oracle
+    import workloads as wl
+
+    cores = os.cpu_count() or 1
+    rows_per = target_rows or 64
+    tot_bytes, tot_time = 0, 0.0
+    for p in wl.config_projections(4):  # the seven shapes of one Qwen3-8B layer
+        Nr = rows_per
+        w = wl.gen_weights(Nr, p.K, 0.1, config=2, layer=0, proj=p.proj)
+        x = wl.gen_x(1, p.K, config=2, layer=0, proj=p.proj)
+        rp, _ = oracle.rowptr(Nr, p.K, w.sal)
+        p1, p2, _ = oracle.pack(Nr, p.K, w.T1, w.T2, w.sal, rp)
+        t0 = time.perf_counter()
+        oracle.linear(1, Nr, p.K, p1, p2, w.sal, w.s1, w.off, w.s2, x, nthreads=cores)
+        tot_time += time.perf_counter() - t0
+        G = p.K // 128
+        tot_bytes += (p1.nbytes + w.s1.nbytes + w.off.nbytes + w.sal.nbytes + p2.nbytes + w.s2.nbytes
+                      + rp.nbytes)
+    desc = f"first {rows_per} rows of each of the 7 Qwen3-8B projection shapes (M=1, 10% salient)"
+    return tot_bytes / tot_time / 1e9, cores, desc, tot_time
+
+
+def calibrate_oracle_rows(budget_s):
+    gbs, cores, _, t = oracle_sample(16)
+    rows = int(16 * budget_s / max(t, 1e-3))
+    return max(16, min(rows, 4096))
+
+
+# ------------------------------------------------------------------- main
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return 0
+    import oracle
+
+    oracle.build()
+    rows = calibrate_oracle_rows(budget_s=20.0 / max(args.steps + args.warmup, 1))
+    vals = []
+    for i in range(args.warmup + args.steps):
+        gbs, cores, desc, t = oracle_sample(rows)
+        if i >= args.warmup:
+            vals.append(gbs)
+    value = float(np.median(vals))
+    bytes_step = 1_792_241_424
+    out = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": bytes_step / (value * 1e9) * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "impl": "reference",
+        "config": {"workload": "qwen3-8b decode step, linear layers only, M=1 (252 packed projections)",
+                   "global_batch": 1, "seq_len": 1, "parallelism": "none (host CPU)"},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "tokens_per_s": value * 1e9 / bytes_step,
+    }
+    print(json.dumps(out), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
+    ap.add_argument("--M", type=int, default=1, help="tokens per step (1 = batch-1 decode)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None, help="profile a smaller step (first L layers)")
+    args = ap.parse_args()
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, ws, rank)
+
+    import torch
+
+    assert torch.cuda.is_available(), "bench.py needs a GPU"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    from paper_2609_09240_gb300 import tq
+
+    tq.lib()
+    items, x_all, y_all, packed_bytes, n_weights = build_step(args.M, dev, seed0=0, layers=args.layers)
+    batch = tq.Batch(args.M, items)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        tq.tq_linear_batched(batch, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+
+    # device-timed region: inputs resident in HBM (1.79 GB of packed weights
+    # per step, larger than the 129 MB L2, so no flush is needed)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+        t1.record(stream)
+        barrier()
+    total_ms = t0.elapsed_time(t1)
+    launch_ms = [a.elapsed_time(b) for a, b in ev]
+    if pg:
+        t = torch.tensor([total_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = ws * packed_bytes / (ms_per_step * 1e-3) / 1e9
+    launch_avg = float(np.mean(launch_ms))
+
+    # end to end through the C ABI with host buffers: per step, H2D of every
+    # projection's activations from pinned memory, the step, D2H of outputs
+    x_host = x_all.cpu().pin_memory()
+    y_host = torch.empty(y_all.shape, dtype=y_all.dtype).pin_memory()
+    h2d = x_host.numel() * x_host.element_size()
+    d2h = y_host.numel() * y_host.element_size()
+
+    def e2e_step():
+        x_all.copy_(x_host, non_blocking=True)
+        step()
+        y_host.copy_(y_all, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    if pg:
+        t = torch.tensor([e2e_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = ws * packed_bytes / (e2e_ms * 1e-3) / 1e9
+
+    peak, peak_kind = measured_peaks()
+    achieved = packed_bytes / (launch_avg * 1e-3) / 1e9
+    out = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"qwen3-8b decode step, linear layers only, M={args.M} (252 packed projections)",
+                   "model": "Qwen3-8B projection shapes, random ternary weights", "global_batch": args.M * ws,
+                   "seq_len": 1, "parallelism": f"replicas x{ws}" if ws > 1 else "none",
+                   "packed_bytes_per_step": packed_bytes, "weights_per_step": n_weights,
+                   "l2": "no flush: 1.79 GB of packed weights per step > 129 MB L2"},
+        "tokens_per_s": ws * args.M / (ms_per_step * 1e-3),
+        "us_per_step": ms_per_step * 1e3,
+        "frac_of_8TBps_nominal": value / ws / 8000.0,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
+                     "traffic": ncu_traffic(), "kernel": "tq decode kernel (one launch per step)",
+                     "launch_ms_avg": launch_avg},
+        "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms},
+        "gpu_launches": args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        oracle.build()
+        rows = calibrate_oracle_rows(budget_s=15.0)
+        gbs, cores, desc, t = oracle_sample(rows)
+        out["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                               "sample": desc, "seconds": t}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if pg:
+        pg.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -48,6 +48,12 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#if defined(__GNUC__)
+#define TQ_API __attribute__((visibility("default")))
+#else
+#define TQ_API
+#endif
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -92,15 +98,15 @@ typedef struct {
 
 /* Bytes of one packed plane-1 row: roundup(26 * K / 128, 16).  0 if K is not
  * a positive multiple of 128. */
-size_t tq_row_bytes(int32_t K);
+TQ_API size_t tq_row_bytes(int32_t K);
 /* 32-bit words of one salience row: ceil((K / 128) / 32). */
-size_t tq_sal_words(int32_t K);
+TQ_API size_t tq_sal_words(int32_t K);
 
 /* rowptr[n] = number of set salience bits in rows 0..n-1, for n = 0..N
  * (so rowptr[N] = nnz).  sal: [N][tq_sal_words(K)].  Bits at g >= K/128 in
  * the last word of a row must be 0, else TQ_DATA_BAD_PAD is OR-ed into
  * *d_status and those bits are not counted. */
-tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t *rowptr,
+TQ_API tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t *rowptr,
                              uint32_t *d_status, void *stream);
 
 /* Pack int8 trit codes into the lattice format (paper "Packing").
@@ -112,7 +118,7 @@ tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t 
  * Invalid codes set TQ_DATA_BAD_CODE (the digit is clamped into the byte),
  * T2 != 0 outside salience sets TQ_DATA_T2_OUTSIDE, a rowptr that disagrees
  * with sal sets TQ_DATA_BAD_ROWPTR. */
-tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+TQ_API tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                   const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *d_status,
                   void *stream);
 
@@ -120,23 +126,34 @@ tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T2, cons
  * non-salient groups.  Validates every byte: > 242 -> TQ_DATA_BAD_BYTE (the
  * trits are written as 0), tail pad digit != 1 or row pad byte != 0 ->
  * TQ_DATA_BAD_PAD, rowptr disagreeing with sal -> TQ_DATA_BAD_ROWPTR. */
-tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *plane2,
+TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *plane2,
                     const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                     uint32_t *d_status, void *stream);
 
+/* Device workspace of the decode path (M <= TQ_MAX_SKINNY_M): the
+ * activations of every call are first rearranged into the tensor-core
+ * operand order of the packed weights (with the per-group correction terms).
+ * The caller provides this scratch memory (the library never allocates).
+ * Bytes needed for one projection with K inputs and M tokens (M > 16 needs
+ * the M = 16 amount); 0 if K is invalid. */
+TQ_API size_t tq_workspace_bytes(int32_t M, int32_t K);
+
 /* y = x W^T for one packed projection (paper "Direct Packed Execution").
  *   x: fp16 [M][K] row-major, 16-byte aligned; y: fp16 [M][N] (rounded to
- *   nearest even from the fp32 accumulator).  M >= 1.  M <= TQ_MAX_SKINNY_M
- *   runs the decode kernel (GEMV / skinny GEMM); larger M runs the prefill
- *   kernel (dequantized tile -> tensor-core MMA, fp32 accumulation).
+ *   nearest even from the fp32 accumulator).  M >= 1; M is processed in
+ *   chunks of TQ_MAX_SKINNY_M tokens on the decode path.
+ *   workspace: device scratch of at least tq_workspace_bytes(M, K) bytes,
+ *   256-byte aligned; its contents are overwritten; calls that share a
+ *   workspace must not overlap in time.
  * The packed bytes are trusted (produced by tq_pack): no per-byte
  * validation on this path. */
-tq_status tq_linear(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
-                    uint16_t *y, void *stream);
+TQ_API tq_status tq_linear(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
+                           uint16_t *y, void *workspace, size_t workspace_bytes, void *stream);
 
 /* As tq_linear but y is fp32 [M][N] (the accumulator before rounding). */
-tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weight *w,
-                           const uint16_t *x, float *y, void *stream);
+TQ_API tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weight *w,
+                                  const uint16_t *x, float *y, void *workspace, size_t workspace_bytes,
+                                  void *stream);
 
 /* Many independent projections in one launch (one decode step of a model:
  * every targeted projection of every layer).  Each problem has its own
@@ -150,10 +167,21 @@ typedef struct {
   uint16_t *y;       /* fp16 [M][w.N] */
 } tq_problem;
 
-tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *stream);
+/* Workspace bytes of a batched call (sum over problems, 256-byte padded). */
+TQ_API size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_problem *problems);
+
+TQ_API tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
+                                   size_t workspace_bytes, void *stream);
+
+/* Device status word of the library's linear kernels, OR of:
+ *   1 = a bounded device-side wait ran out (the kernel stopped early and its
+ *       outputs are incomplete), 2 = shared-memory placement failed.
+ * SYNCHRONOUS (unlike every other entry point): copies the word from the
+ * device of the current context; clear != 0 resets it to 0 afterwards. */
+TQ_API tq_status tq_get_device_status(uint32_t *status_host, int clear);
 
 /* Human-readable name of a status code (static string). */
-const char *tq_status_str(tq_status s);
+TQ_API const char *tq_status_str(tq_status s);
 
 #ifdef __cplusplus
 }

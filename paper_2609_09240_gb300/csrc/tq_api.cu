@@ -1,0 +1,234 @@
+// tq_api.cu - the C ABI (include/tq.h): argument validation and dispatch.
+//
+// Nothing here allocates device memory or synchronizes; every launch goes to
+// the caller's stream.  Shape / null / alignment errors return before any
+// launch.
+#include <string.h>
+
+#include "tq_common.cuh"
+
+namespace tq {
+cudaError_t launch_rowptr(int N, int K, const uint32_t *sal, int32_t *rowptr, uint32_t *status,
+                          cudaStream_t s);
+cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t *rowptr,
+                                uint32_t *status, cudaStream_t s);
+cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+                        const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
+                        cudaStream_t s);
+cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
+                          const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                          uint32_t *status, cudaStream_t s);
+cudaError_t launch_gemv_tc(const BatchParams &p, cudaStream_t s);
+int tc_rows_per_tile();
+size_t tc_workspace_bytes(int M, int K);
+size_t tc_workspace_b_bytes(int M, int K);
+cudaError_t read_status_gemv_tc(uint32_t *out, bool clear);
+}  // namespace tq
+
+using namespace tq;
+
+namespace {
+
+constexpr int kMaxK = 1 << 20;  // 1 Mi inputs per row: far above any projection here
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+bool aligned2(const void *p) { return ((uintptr_t)p & 1u) == 0; }
+
+tq_status check_shape(int32_t N, int32_t K) {
+  if (N < 1 || K < TQ_GROUP || K % TQ_GROUP != 0 || K > kMaxK) return TQ_ERR_SHAPE;
+  return TQ_OK;
+}
+
+tq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? TQ_OK : TQ_ERR_CUDA; }
+
+tq_status check_weight(const tq_weight *w, int32_t N, int32_t K) {
+  if (!w) return TQ_ERR_NULL;
+  if (w->group != TQ_GROUP) return TQ_ERR_SHAPE;
+  if (w->N != N || w->K != K) return TQ_ERR_SHAPE;
+  if (tq_status s = check_shape(N, K)) return s;
+  if (!w->plane1 || !w->salience || !w->rowptr || !w->scale1 || !w->offset) return TQ_ERR_NULL;
+  if (w->nnz < 0 || w->nnz > (int64_t)N * (K / TQ_GROUP)) return TQ_ERR_SALIENCE;
+  if (w->nnz > 0 && (!w->plane2 || !w->scale2)) return TQ_ERR_NULL;
+  if (!aligned16(w->plane1)) return TQ_ERR_ALIGN;
+  if (!aligned2(w->scale1) || !aligned2(w->offset) || (w->plane2 && !aligned2(w->plane2)) ||
+      (w->scale2 && !aligned2(w->scale2)) || ((uintptr_t)w->salience & 3u) ||
+      ((uintptr_t)w->rowptr & 3u))
+    return TQ_ERR_ALIGN;
+  return TQ_OK;
+}
+
+Problem to_problem(const tq_weight *w, const uint16_t *x, void *y) {
+  Problem P;
+  memset(&P, 0, sizeof(P));
+  P.plane1 = w->plane1;
+  P.sal = w->salience;
+  P.rowptr = w->rowptr;
+  P.plane2 = w->plane2;
+  P.s1 = reinterpret_cast<const __half *>(w->scale1);
+  P.off = reinterpret_cast<const __half *>(w->offset);
+  P.s2 = reinterpret_cast<const __half *>(w->scale2);
+  P.x = reinterpret_cast<const __half *>(x);
+  P.y = y;
+  P.N = w->N;
+  P.K = w->K;
+  P.nnz = (int32_t)w->nnz;
+  return P;
+}
+
+size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
+
+// Places every problem's workspace (activation slots, then C/S) and runs the
+// decode kernel.  Returns TQ_ERR_SHAPE when the workspace is too small.
+tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
+  const int rows = tc_rows_per_tile();
+  const int mw = bp.M <= 8 ? 8 : 16;  // workspace sizing uses the padded token count
+  int tiles = 0;
+  size_t off = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    Problem &P = bp.prob[i];
+    P.tile_begin = tiles;
+    tiles += (P.N + rows - 1) / rows;
+    const size_t bb = tc_workspace_b_bytes(mw, P.K), tot = tc_workspace_bytes(mw, P.K);
+    if (off + pad256(tot) > ws_bytes) return TQ_ERR_SHAPE;
+    P.wsB = ws + off;
+    P.wsCS = reinterpret_cast<float *>(ws + off + bb);
+    off += pad256(tot);
+  }
+  bp.total_tiles = tiles;
+  return from_cuda(launch_gemv_tc(bp, s));
+}
+
+tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
+                      void *y, bool f32, void *ws, size_t ws_bytes, cudaStream_t s) {
+  if (M < 1) return TQ_ERR_SHAPE;
+  if (tq_status st = check_weight(w, N, K)) return st;
+  if (!x || !y || !ws) return TQ_ERR_NULL;
+  if (!aligned16(x) || ((uintptr_t)ws & 255u)) return TQ_ERR_ALIGN;
+  if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
+  if (ws_bytes < tc_workspace_bytes(M, K)) return TQ_ERR_SHAPE;
+  static BatchParams bp;  // large; filled per call (host-side, not thread-safe across calls)
+  // Tokens are processed in chunks of TQ_MAX_SKINNY_M.
+  for (int32_t m0 = 0; m0 < M; m0 += TQ_MAX_SKINNY_M) {
+    const int32_t mc = M - m0 < TQ_MAX_SKINNY_M ? M - m0 : TQ_MAX_SKINNY_M;
+    bp.count = 1;
+    bp.M = mc;
+    bp.out_f32 = f32 ? 1 : 0;
+    char *yb = static_cast<char *>(y) + (int64_t)m0 * N * (f32 ? 4 : 2);
+    bp.prob[0] = to_problem(w, x + (int64_t)m0 * K, yb);
+    if (tq_status st = run_batch(bp, static_cast<unsigned char *>(ws), ws_bytes, s)) return st;
+  }
+  return TQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t tq_row_bytes(int32_t K) {
+  if (check_shape(1, K) != TQ_OK) return 0;
+  return (size_t)row_bytes_of(K);
+}
+
+size_t tq_sal_words(int32_t K) {
+  if (check_shape(1, K) != TQ_OK) return 0;
+  return (size_t)sal_words_of(K);
+}
+
+tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t *rowptr,
+                             uint32_t *d_status, void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!sal || !rowptr || !d_status) return TQ_ERR_NULL;
+  return from_cuda(launch_rowptr(N, K, sal, rowptr, d_status, (cudaStream_t)stream));
+}
+
+tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+                  const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *d_status,
+                  void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!T1 || !sal || !rowptr || !plane1 || !d_status) return TQ_ERR_NULL;
+  if ((T2 == nullptr) != (plane2 == nullptr)) return TQ_ERR_NULL;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (tq_status st = from_cuda(launch_check_rowptr(N, K, sal, rowptr, d_status, s))) return st;
+  return from_cuda(launch_pack(N, K, T1, T2, sal, rowptr, plane1, plane2, d_status, s));
+}
+
+tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *plane2,
+                    const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                    uint32_t *d_status, void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!plane1 || !sal || !rowptr || !T1 || !d_status) return TQ_ERR_NULL;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (tq_status st = from_cuda(launch_check_rowptr(N, K, sal, rowptr, d_status, s))) return st;
+  return from_cuda(launch_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, s));
+}
+
+size_t tq_workspace_bytes(int32_t M, int32_t K) {
+  if (M < 1 || check_shape(1, K) != TQ_OK) return 0;
+  return pad256(tc_workspace_bytes(M <= 8 ? 8 : 16, K));
+}
+
+size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_problem *problems) {
+  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH || !problems) return 0;
+  size_t tot = 0;
+  for (int i = 0; i < count; ++i) {
+    if (check_shape(1, problems[i].w.K) != TQ_OK) return 0;
+    tot += pad256(tc_workspace_bytes(M <= 8 ? 8 : 16, problems[i].w.K));
+  }
+  return tot;
+}
+
+tq_status tq_linear(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
+                    uint16_t *y, void *workspace, size_t workspace_bytes, void *stream) {
+  return linear_impl(M, N, K, w, x, y, false, workspace, workspace_bytes, (cudaStream_t)stream);
+}
+
+tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weight *w,
+                           const uint16_t *x, float *y, void *workspace, size_t workspace_bytes,
+                           void *stream) {
+  return linear_impl(M, N, K, w, x, y, true, workspace, workspace_bytes, (cudaStream_t)stream);
+}
+
+tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
+                            size_t workspace_bytes, void *stream) {
+  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
+  if (!problems || !workspace) return TQ_ERR_NULL;
+  if ((uintptr_t)workspace & 255u) return TQ_ERR_ALIGN;
+  static BatchParams bp;
+  bp.count = count;
+  bp.M = M;
+  bp.out_f32 = 0;
+  for (int i = 0; i < count; ++i) {
+    const tq_problem &q = problems[i];
+    if (tq_status st = check_weight(&q.w, q.w.N, q.w.K)) return st;
+    if (!q.x || !q.y) return TQ_ERR_NULL;
+    if (!aligned16(q.x)) return TQ_ERR_ALIGN;
+    if (!aligned2(q.y)) return TQ_ERR_ALIGN;
+    bp.prob[i] = to_problem(&q.w, q.x, q.y);
+  }
+  return run_batch(bp, static_cast<unsigned char *>(workspace), workspace_bytes, (cudaStream_t)stream);
+}
+
+tq_status tq_get_device_status(uint32_t *status_host, int clear) {
+  if (!status_host) return TQ_ERR_NULL;
+  uint32_t a = 0;
+  if (read_status_gemv_tc(&a, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  *status_host = a;
+  return TQ_OK;
+}
+
+const char *tq_status_str(tq_status s) {
+  switch (s) {
+    case TQ_OK: return "TQ_OK";
+    case TQ_ERR_NULL: return "TQ_ERR_NULL: a required pointer is NULL";
+    case TQ_ERR_SHAPE: return "TQ_ERR_SHAPE: M, N or K out of range, or K not a multiple of 128";
+    case TQ_ERR_ALIGN: return "TQ_ERR_ALIGN: a pointer is not aligned (plane1 and x need 16 bytes)";
+    case TQ_ERR_CODE: return "TQ_ERR_CODE: invalid trit code";
+    case TQ_ERR_BYTE: return "TQ_ERR_BYTE: invalid packed byte";
+    case TQ_ERR_SALIENCE: return "TQ_ERR_SALIENCE: nnz inconsistent with the salience map";
+    case TQ_ERR_CUDA: return "TQ_ERR_CUDA: a CUDA launch failed";
+    case TQ_ERR_TIMEOUT: return "TQ_ERR_TIMEOUT: a bounded device wait ran out";
+  }
+  return "unknown tq_status";
+}
+
+}  // extern "C"

@@ -1,0 +1,256 @@
+// tq_codec.cu - pack / unpack / salience row-prefix kernels.
+//
+// The lattice-aware serialization of the paper ("Packing: From Quantization
+// to Serialization") stores the discrete supports (trit codes) and their
+// parameters instead of fp16 values.  Byte layout (library definition, the
+// paper prints none): five trits per byte as a base-3 numeral, digit =
+// trit + 1, first trit least significant; a 128-trit group is 26 bytes
+// (25 full bytes, then a tail byte with trits 125..127 and pad digits 1);
+// plane-1 rows are padded with 0x00 to a multiple of 16 bytes.  Plane 2
+// holds only salient groups in (row, group) order.
+//
+// Every kernel validates what it reads and ORs TQ_DATA_* bits into the
+// caller's status word; no kernel traps, and every plane-2 index is checked
+// against rowptr[N] before it is used.
+#include "tq_common.cuh"
+
+namespace tq {
+
+__device__ __forceinline__ int sal_bit(const uint32_t *sal, int W, int n, int g) {
+  return (int)((sal[(int64_t)n * W + (g >> 5)] >> (g & 31)) & 1u);
+}
+
+// Number of salient groups of row n before group g.
+__device__ __forceinline__ int sal_rank(const uint32_t *sal, int W, int n, int g) {
+  const uint32_t *row = sal + (int64_t)n * W;
+  int r = 0;
+  for (int w = 0; w < (g >> 5); ++w) r += __popc(row[w]);
+  uint32_t part = row[g >> 5] & ((1u << (g & 31)) - 1u);
+  return r + __popc(part);
+}
+
+// Set bits of row n at valid group positions, and whether pad bits are set.
+__device__ __forceinline__ int row_popc(const uint32_t *sal, int W, int G, int n, bool *pad_bad) {
+  const uint32_t *row = sal + (int64_t)n * W;
+  int r = 0;
+  for (int w = 0; w < W; ++w) {
+    uint32_t v = row[w];
+    int valid = G - 32 * w;  // valid bits in this word
+    if (valid < 32) {
+      uint32_t mask = valid > 0 ? ((1u << valid) - 1u) : 0u;
+      if (v & ~mask) *pad_bad = true;
+      v &= mask;
+    }
+    r += __popc(v);
+  }
+  return r;
+}
+
+// ---------------------------------------------------------------- rowptr
+// One block: each thread sums a contiguous run of rows, then a block scan.
+__global__ void __launch_bounds__(1024) rowptr_kernel(int N, int K, const uint32_t *sal,
+                                                      int32_t *rowptr, uint32_t *status) {
+  const int G = K / kGroup, W = sal_words_of(K);
+  const int per = (N + blockDim.x - 1) / blockDim.x;
+  const int r0 = threadIdx.x * per;
+  const int r1 = min(N, r0 + per);
+  bool pad_bad = false;
+  int local = 0;
+  for (int n = r0; n < r1; ++n) local += row_popc(sal, W, G, n, &pad_bad);
+  // inclusive warp scan, then scan of warp totals
+  __shared__ int warp_tot[32];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int incl = local;
+  for (int o = 1; o < 32; o <<= 1) {
+    int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) warp_tot[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    int nw = blockDim.x >> 5;
+    int v = lane < nw ? warp_tot[lane] : 0;
+    for (int o = 1; o < 32; o <<= 1) {
+      int u = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += u;
+    }
+    if (lane < nw) warp_tot[lane] = v;  // inclusive over warps
+  }
+  __syncthreads();
+  int base = (wid > 0 ? warp_tot[wid - 1] : 0) + incl - local;
+  for (int n = r0; n < r1; ++n) {
+    rowptr[n] = base;
+    bool dummy = false;
+    base += row_popc(sal, W, G, n, &dummy);
+  }
+  if (threadIdx.x == blockDim.x - 1) rowptr[N] = warp_tot[(blockDim.x >> 5) - 1];
+  if (pad_bad) atomicOr(status, TQ_DATA_BAD_PAD);
+}
+
+// Thread per row: rowptr[0] == 0 and rowptr[n+1] - rowptr[n] == popcount.
+__global__ void check_rowptr_kernel(int N, int K, const uint32_t *sal, const int32_t *rowptr,
+                                    uint32_t *status) {
+  const int G = K / kGroup, W = sal_words_of(K);
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= N) return;
+  bool pad_bad = false;
+  int c = row_popc(sal, W, G, n, &pad_bad);
+  uint32_t st = 0;
+  if (pad_bad) st |= TQ_DATA_BAD_PAD;
+  if (rowptr[n + 1] - rowptr[n] != c) st |= TQ_DATA_BAD_ROWPTR;
+  if (n == 0 && rowptr[0] != 0) st |= TQ_DATA_BAD_ROWPTR;
+  if (st) atomicOr(status, st);
+}
+
+// ------------------------------------------------------------------- pack
+__device__ __forceinline__ uint8_t encode_codes(const int8_t *t, int ntr, uint32_t *st) {
+  int v = 0, p = 1;
+  for (int i = 0; i < 5; ++i) {
+    int d = 1;  // pad digit (trit 0)
+    if (i < ntr) {
+      int c = t[i];
+      if (c < -1 || c > 1) {
+        *st |= TQ_DATA_BAD_CODE;
+        c = c < -1 ? -1 : 1;
+      }
+      d = c + 1;
+    }
+    v += d * p;
+    p *= 3;
+  }
+  return (uint8_t)v;
+}
+
+// Thread per plane-1 byte (n, b).
+__global__ void pack_kernel(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+                            const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2,
+                            uint32_t *status) {
+  const int G = K / kGroup, W = sal_words_of(K);
+  const int64_t RB = row_bytes_of(K);
+  const int64_t total = (int64_t)N * RB;
+  const int32_t nnz = rowptr[N];
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int n = (int)(idx / RB);
+    const int b = (int)(idx - (int64_t)n * RB);
+    uint32_t st = 0;
+    if (b >= G * kGroupBytes) {
+      plane1[idx] = 0;
+      continue;
+    }
+    const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+    const int ntr = pos < kFullBytes ? 5 : kTailTrits;
+    const int64_t k0 = (int64_t)n * K + (int64_t)g * kGroup + 5 * pos;
+    plane1[idx] = encode_codes(T1 + k0, ntr, &st);
+    const int s = sal_bit(sal, W, n, g);
+    if (T2) {
+      if (s) {
+        int64_t j = (int64_t)rowptr[n] + sal_rank(sal, W, n, g);
+        if (j >= 0 && j < nnz)
+          plane2[j * kGroupBytes + pos] = encode_codes(T2 + k0, ntr, &st);
+        else
+          st |= TQ_DATA_BAD_ROWPTR;
+      } else {
+        for (int i = 0; i < ntr; ++i)
+          if (T2[k0 + i] != 0) st |= TQ_DATA_T2_OUTSIDE;
+      }
+    } else if (s) {
+      st |= TQ_DATA_T2_OUTSIDE;
+    }
+    if (st) atomicOr(status, st);
+  }
+}
+
+// ----------------------------------------------------------------- unpack
+__device__ __forceinline__ void decode_to(uint8_t v, int ntr, int8_t *t, uint32_t *st) {
+  if (v > 242) {
+    *st |= TQ_DATA_BAD_BYTE;
+    for (int i = 0; i < ntr; ++i) t[i] = 0;
+    return;
+  }
+  int q = v;
+  for (int i = 0; i < 5; ++i) {
+    int d = q % 3;
+    q /= 3;
+    if (i < ntr)
+      t[i] = (int8_t)(d - 1);
+    else if (d != 1)
+      *st |= TQ_DATA_BAD_PAD;
+  }
+}
+
+__global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
+                              const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                              uint32_t *status) {
+  const int G = K / kGroup, W = sal_words_of(K);
+  const int64_t RB = row_bytes_of(K);
+  const int64_t total = (int64_t)N * RB;
+  const int32_t nnz = rowptr[N];
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int n = (int)(idx / RB);
+    const int b = (int)(idx - (int64_t)n * RB);
+    uint32_t st = 0;
+    const uint8_t v = plane1[idx];
+    if (b >= G * kGroupBytes) {
+      if (v != 0) atomicOr(status, TQ_DATA_BAD_PAD);
+      continue;
+    }
+    const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+    const int ntr = pos < kFullBytes ? 5 : kTailTrits;
+    const int64_t k0 = (int64_t)n * K + (int64_t)g * kGroup + 5 * pos;
+    decode_to(v, ntr, T1 + k0, &st);
+    if (T2) {
+      if (sal_bit(sal, W, n, g)) {
+        int64_t j = (int64_t)rowptr[n] + sal_rank(sal, W, n, g);
+        if (plane2 && j >= 0 && j < nnz) {
+          decode_to(plane2[j * kGroupBytes + pos], ntr, T2 + k0, &st);
+        } else {
+          st |= TQ_DATA_BAD_ROWPTR;
+          for (int i = 0; i < ntr; ++i) T2[k0 + i] = 0;
+        }
+      } else {
+        for (int i = 0; i < ntr; ++i) T2[k0 + i] = 0;
+      }
+    }
+    if (st) atomicOr(status, st);
+  }
+}
+
+// ------------------------------------------------------------- launchers
+static int grid_for(int64_t work, int block) {
+  int64_t g = (work + block - 1) / block;
+  if (g > 152 * 32) g = 152 * 32;
+  return (int)(g < 1 ? 1 : g);
+}
+
+cudaError_t launch_rowptr(int N, int K, const uint32_t *sal, int32_t *rowptr, uint32_t *status,
+                          cudaStream_t s) {
+  rowptr_kernel<<<1, 1024, 0, s>>>(N, K, sal, rowptr, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t *rowptr,
+                                uint32_t *status, cudaStream_t s) {
+  check_rowptr_kernel<<<(N + 255) / 256, 256, 0, s>>>(N, K, sal, rowptr, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
+                        const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
+                        cudaStream_t s) {
+  int64_t total = (int64_t)N * row_bytes_of(K);
+  pack_kernel<<<grid_for(total, 256), 256, 0, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
+                          const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                          uint32_t *status, cudaStream_t s) {
+  int64_t total = (int64_t)N * row_bytes_of(K);
+  unpack_kernel<<<grid_for(total, 256), 256, 0, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
+                                                     status);
+  return cudaGetLastError();
+}
+
+}  // namespace tq

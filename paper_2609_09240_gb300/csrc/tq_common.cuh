@@ -1,0 +1,54 @@
+// tq_common.cuh - device-side helpers shared by the CUDA kernels of the
+// packed ternary linear layer (format constants, fp16 bit helpers, the
+// kernel-side problem descriptor).
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "tq.h"
+
+namespace tq {
+
+constexpr int kGroup = TQ_GROUP;            // trits per group along K
+constexpr int kGroupBytes = TQ_GROUP_BYTES;  // 25 full bytes + 1 tail byte
+constexpr int kFullBytes = 25;
+constexpr int kTailTrits = 3;
+// Tail byte of an all-zero group: digits (1,1,1) plus the two pad digits 1.
+constexpr int kZeroByte = 121;  // 1 + 3 + 9 + 27 + 81
+
+__host__ __device__ inline int64_t row_bytes_of(int K) {
+  int64_t raw = (int64_t)(K / kGroup) * kGroupBytes;
+  return (raw + 15) / 16 * 16;
+}
+__host__ __device__ inline int sal_words_of(int K) { return (K / kGroup + 31) / 32; }
+
+// Kernel-side descriptor of one projection (copied by value into launch
+// parameters; all pointers are device pointers).
+struct Problem {
+  const uint8_t *plane1;
+  const uint32_t *sal;
+  const int32_t *rowptr;
+  const uint8_t *plane2;
+  const __half *s1;
+  const __half *off;
+  const __half *s2;
+  const __half *x;  // [M][K]
+  void *y;          // [M][N] fp16 or fp32
+  unsigned char *wsB;  // workspace: activation slots of this problem
+  float *wsCS;         // workspace: per-group C and S of this problem
+  int32_t N, K;
+  int32_t tile_begin;  // first global tile index of this problem
+  int32_t nnz;         // plane-2 records (rowptr[N]); indices are clamped below it
+};
+
+struct BatchParams {
+  int32_t count;        // problems in prob[]
+  int32_t M;            // tokens (rows of every x)
+  int32_t total_tiles;  // sum of tiles over problems
+  int32_t out_f32;      // y is fp32 (else fp16)
+  Problem prob[TQ_MAX_BATCH];
+};
+
+}  // namespace tq

@@ -1,0 +1,264 @@
+"""Thin ctypes binding of the C ABI in include/tq.h.
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of libtq.so.  Tensors are torch CUDA tensors (torch supplies device
+memory and streams); there is no CPU fallback and a missing library raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+
+import torch
+
+from . import build as _build
+
+TQ_GROUP = 128
+TQ_GROUP_BYTES = 26
+TQ_MAX_SKINNY_M = 16
+TQ_MAX_BATCH = 256
+
+TQ_OK = 0
+STATUS_NAMES = {0: "TQ_OK", -1: "TQ_ERR_NULL", -2: "TQ_ERR_SHAPE", -3: "TQ_ERR_ALIGN", -4: "TQ_ERR_CODE",
+                -5: "TQ_ERR_BYTE", -6: "TQ_ERR_SALIENCE", -7: "TQ_ERR_CUDA", -8: "TQ_ERR_TIMEOUT"}
+DATA_BAD_CODE, DATA_T2_OUTSIDE, DATA_BAD_BYTE, DATA_BAD_PAD, DATA_BAD_ROWPTR = 1, 2, 4, 8, 16
+
+_lock = threading.Lock()
+_lib = None
+
+
+class TQError(RuntimeError):
+    def __init__(self, code, where):
+        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)}")
+        self.code = code
+
+
+class tq_weight(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int32), ("K", ctypes.c_int32), ("group", ctypes.c_int32),
+                ("plane1", ctypes.c_void_p), ("salience", ctypes.c_void_p), ("rowptr", ctypes.c_void_p),
+                ("plane2", ctypes.c_void_p), ("scale1", ctypes.c_void_p), ("offset", ctypes.c_void_p),
+                ("scale2", ctypes.c_void_p), ("nnz", ctypes.c_int64)]
+
+
+class tq_problem(ctypes.Structure):
+    _fields_ = [("w", tq_weight), ("x", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load libtq.so (building it first if stale).  Raises if unavailable."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build()
+            if not os.path.exists(path):
+                raise RuntimeError(f"CUDA library missing: {path}")
+            L = ctypes.CDLL(path)
+            vp, i32 = ctypes.c_void_p, ctypes.c_int32
+            L.tq_row_bytes.restype = ctypes.c_size_t
+            L.tq_row_bytes.argtypes = [i32]
+            L.tq_sal_words.restype = ctypes.c_size_t
+            L.tq_sal_words.argtypes = [i32]
+            L.tq_salience_rowptr.restype = ctypes.c_int
+            L.tq_salience_rowptr.argtypes = [i32, i32, vp, vp, vp, vp]
+            L.tq_pack.restype = ctypes.c_int
+            L.tq_pack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.tq_unpack.restype = ctypes.c_int
+            L.tq_unpack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+            sz = ctypes.c_size_t
+            L.tq_workspace_bytes.restype = sz
+            L.tq_workspace_bytes.argtypes = [i32, i32]
+            L.tq_batched_workspace_bytes.restype = sz
+            L.tq_batched_workspace_bytes.argtypes = [i32, i32, ctypes.POINTER(tq_problem)]
+            L.tq_linear.restype = ctypes.c_int
+            L.tq_linear.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp, sz, vp]
+            L.tq_linear_f32out.restype = ctypes.c_int
+            L.tq_linear_f32out.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp, sz, vp]
+            L.tq_linear_batched.restype = ctypes.c_int
+            L.tq_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
+            L.tq_get_device_status.restype = ctypes.c_int
+            L.tq_get_device_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int]
+            L.tq_status_str.restype = ctypes.c_char_p
+            L.tq_status_str.argtypes = [ctypes.c_int]
+            _lib = L
+    return _lib
+
+
+def _p(t):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch tensor")
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor (device memory)")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code, where):
+    if code != TQ_OK:
+        raise TQError(code, where)
+
+
+def tq_row_bytes(K: int) -> int:
+    return int(lib().tq_row_bytes(K))
+
+
+def tq_sal_words(K: int) -> int:
+    return int(lib().tq_sal_words(K))
+
+
+def tq_get_device_status(clear: bool = True) -> int:
+    """Synchronous read of the library's device status word (0 = no bounded
+    wait ran out)."""
+    v = ctypes.c_uint32(0)
+    _check(lib().tq_get_device_status(ctypes.byref(v), 1 if clear else 0), "tq_get_device_status")
+    return int(v.value)
+
+
+def tq_status_str(code: int) -> str:
+    return lib().tq_status_str(code).decode()
+
+
+def tq_salience_rowptr(N, K, sal, rowptr, d_status, stream=None):
+    _check(lib().tq_salience_rowptr(N, K, _p(sal), _p(rowptr), _p(d_status), _stream(stream)), "tq_salience_rowptr")
+
+
+def tq_pack(N, K, T1, T2, sal, rowptr, plane1, plane2, d_status, stream=None):
+    _check(lib().tq_pack(N, K, _p(T1), _p(T2), _p(sal), _p(rowptr), _p(plane1), _p(plane2), _p(d_status),
+                         _stream(stream)), "tq_pack")
+
+
+def tq_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, stream=None):
+    _check(lib().tq_unpack(N, K, _p(plane1), _p(plane2), _p(sal), _p(rowptr), _p(T1), _p(T2), _p(d_status),
+                           _stream(stream)), "tq_unpack")
+
+
+@dataclass
+class PackedWeight:
+    """Device tensors of one packed projection (the fields of tq_weight)."""
+    N: int
+    K: int
+    plane1: torch.Tensor   # uint8 [N][row_bytes]
+    salience: torch.Tensor  # int32 (uint32 bits) [N][sal_words]
+    rowptr: torch.Tensor   # int32 [N+1]
+    plane2: torch.Tensor | None   # uint8 [nnz][26]
+    scale1: torch.Tensor   # fp16 [N][G]
+    offset: torch.Tensor   # fp16 [N][G]
+    scale2: torch.Tensor | None   # fp16 [nnz]
+    nnz: int
+
+    def struct(self) -> tq_weight:
+        w = tq_weight()
+        w.N, w.K, w.group = self.N, self.K, TQ_GROUP
+        w.plane1 = self.plane1.data_ptr()
+        w.salience = self.salience.data_ptr()
+        w.rowptr = self.rowptr.data_ptr()
+        w.plane2 = self.plane2.data_ptr() if self.plane2 is not None and self.nnz > 0 else None
+        w.scale1 = self.scale1.data_ptr()
+        w.offset = self.offset.data_ptr()
+        w.scale2 = self.scale2.data_ptr() if self.scale2 is not None and self.nnz > 0 else None
+        w.nnz = self.nnz
+        return w
+
+    def packed_bytes(self) -> int:
+        """Bytes of the packed representation read by the linear kernels."""
+        t = [self.plane1, self.salience, self.rowptr, self.scale1, self.offset]
+        if self.nnz:
+            t += [self.plane2, self.scale2]
+        return sum(x.numel() * x.element_size() for x in t)
+
+
+def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True) -> PackedWeight:
+    """Pack device int8 codes + fp16 params with tq_salience_rowptr + tq_pack.
+
+    Reads nnz back to the host (one synchronization) to size plane 2."""
+    N, K = T1.shape
+    dev = T1.device
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    rowptr = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    tq_salience_rowptr(N, K, sal, rowptr, status, stream)
+    nnz = int(rowptr[N].item())
+    plane1 = torch.empty((N, tq_row_bytes(K)), dtype=torch.uint8, device=dev)
+    plane2 = torch.empty((max(nnz, 1), TQ_GROUP_BYTES), dtype=torch.uint8, device=dev)
+    tq_pack(N, K, T1, T2 if nnz > 0 else None, sal, rowptr, plane1, plane2 if nnz > 0 else None, status, stream)
+    if check:
+        st = int(status.item())
+        if st:
+            raise TQError(-4, f"tq_pack data status {st:#x}")
+    if s2 is None or nnz == 0:
+        s2 = torch.zeros(1, dtype=torch.float16, device=dev)
+    return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz)
+
+
+def tq_workspace_bytes(M: int, K: int) -> int:
+    return int(lib().tq_workspace_bytes(M, K))
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """Device scratch for the decode path (torch allocations are 256-byte aligned)."""
+    t = torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+    assert t.data_ptr() % 256 == 0
+    return t
+
+
+def tq_linear(x, w: PackedWeight, y=None, ws=None, stream=None):
+    """y = x W^T, fp16.  x: fp16 [M][K] on the device; ws: optional workspace."""
+    M, K = x.shape
+    assert K == w.K and x.dtype == torch.float16
+    if y is None:
+        y = torch.empty((M, w.N), dtype=torch.float16, device=x.device)
+    if ws is None:
+        ws = workspace(tq_workspace_bytes(M, K), x.device)
+    ws_ = w.struct()
+    _check(lib().tq_linear(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _p(ws), ws.numel(), _stream(stream)),
+           "tq_linear")
+    return y
+
+
+def tq_linear_f32out(x, w: PackedWeight, y=None, ws=None, stream=None):
+    M, K = x.shape
+    assert K == w.K and x.dtype == torch.float16
+    if y is None:
+        y = torch.empty((M, w.N), dtype=torch.float32, device=x.device)
+    if ws is None:
+        ws = workspace(tq_workspace_bytes(M, K), x.device)
+    ws_ = w.struct()
+    _check(lib().tq_linear_f32out(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _p(ws), ws.numel(),
+                                  _stream(stream)), "tq_linear_f32out")
+    return y
+
+
+class Batch:
+    """A prepared tq_problem array (host memory) and its device workspace."""
+
+    def __init__(self, M, items, device=None):
+        self.M = M
+        self.items = list(items)  # (PackedWeight, x, y); keeps tensors alive
+        self.arr = (tq_problem * len(self.items))()
+        for i, (w, x, y) in enumerate(self.items):
+            self.arr[i].w = w.struct()
+            self.arr[i].x = x.data_ptr()
+            self.arr[i].y = y.data_ptr()
+        nbytes = int(lib().tq_batched_workspace_bytes(M, len(self.items), self.arr))
+        if nbytes == 0:
+            raise TQError(-2, "tq_batched_workspace_bytes")
+        dev = device if device is not None else self.items[0][1].device
+        self.ws = workspace(nbytes, dev)
+
+
+def tq_linear_batched(batch: Batch, stream=None):
+    _check(lib().tq_linear_batched(batch.M, len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(),
+                                   _stream(stream)), "tq_linear_batched")

@@ -1,0 +1,52 @@
+"""CPU checks of the C-ABI library: it builds for sm_103a, loads, and exports
+every entry point declared in include/tq.h (no compute calls without a GPU)."""
+import ctypes
+import os
+import re
+import subprocess
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, "include", "tq.h")).read()
+    return sorted(set(re.findall(r"TQ_API\s+[\w\s\*]*?\b(tq_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_abi():
+    names = declared_symbols()
+    for want in ("tq_pack", "tq_unpack", "tq_linear", "tq_linear_f32out", "tq_linear_batched",
+                 "tq_salience_rowptr", "tq_row_bytes", "tq_sal_words", "tq_status_str",
+                 "tq_workspace_bytes", "tq_batched_workspace_bytes", "tq_get_device_status"):
+        assert want in names
+
+
+def test_library_loads_and_exports_every_symbol():
+    from paper_2609_09240_gb300 import build, tq
+    path = build.build()
+    L = ctypes.CDLL(path)
+    for name in declared_symbols():
+        assert hasattr(L, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (tq_\w+)", out))
+    assert set(declared_symbols()) <= exported
+    assert tq.tq_row_bytes(2560) == 528 and tq.tq_row_bytes(100) == 0
+    assert tq.tq_sal_words(4224) == 2
+    assert "ALIGN" in tq.tq_status_str(-3)
+
+
+def test_host_side_argument_errors_without_gpu():
+    """Shape and null checks return before any CUDA call."""
+    from paper_2609_09240_gb300 import tq
+    L = tq.lib()
+    assert L.tq_salience_rowptr(0, 128, None, None, None, None) == -2
+    assert L.tq_salience_rowptr(4, 100, None, None, None, None) == -2
+    assert L.tq_salience_rowptr(4, 128, None, None, None, None) == -1
+    assert L.tq_pack(4, 128, None, None, None, None, None, None, None, None) == -1
+    assert L.tq_unpack(4, 130, None, None, None, None, None, None, None, None) == -2
+    assert L.tq_linear(1, 4, 128, None, None, None, None, 0, None) == -1
+    assert L.tq_linear_batched(17, 1, None, None, 0, None) == -2
+    assert L.tq_linear_batched(1, 0, None, None, 0, None) == -2
+    assert tq.tq_workspace_bytes(1, 4096) == 32 * (2560 + 64)
+    assert tq.tq_workspace_bytes(16, 4096) == 32 * (5120 + 128)
+    assert tq.tq_workspace_bytes(1, 100) == 0

@@ -1,0 +1,107 @@
+"""GPU linear parity: tq_linear / tq_linear_f32out / tq_linear_batched
+against the fp64 CPU oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element."""
+import numpy as np
+import pytest
+import torch
+
+import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def H():
+    import gpu_helpers
+    return gpu_helpers
+
+
+def run_case(H, N, K, frac, M, f32, proj=0, config=6):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, frac, config=config, proj=proj)
+    x = wl.gen_x(M, K, config=config, proj=proj)
+    y_ref, a_ref = H.oracle_ref(w, x)
+    pw = H.pack_on_gpu(w)
+    xd = H.dev(x)
+    y = (tq.tq_linear_f32out if f32 else tq.tq_linear)(xd, pw)
+    H.device_status_ok()
+    yg = y.float().cpu().numpy().astype(np.float64)
+    return H.assert_close(yg, y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 16])
+@pytest.mark.parametrize("f32", [False, True])
+def test_config0_single_linear(H, M, f32):
+    run_case(H, 512, 1024, 0.0, M, f32)
+
+
+@pytest.mark.parametrize("N,K,frac", [(1, 128, 0.0), (1, 128, 1.0), (129, 256, 0.5), (200, 2560, 0.1),
+                                      (77, 4224, 0.1), (300, 9728, 0.1), (128, 12288, 0.1)])
+@pytest.mark.parametrize("M", [1, 5, 16])
+def test_ragged_shapes(H, N, K, frac, M):
+    run_case(H, N, K, frac, M, f32=False, proj=N)
+
+
+@pytest.mark.parametrize("M", [17, 40])
+def test_m_above_skinny(H, M):
+    run_case(H, 130, 1024, 0.1, M, f32=True, proj=3)
+
+
+@pytest.mark.parametrize("idx", range(7))
+def test_config1_qwen3_4b_layer(H, idx):
+    name, N, K = wl.QWEN3_4B[idx]
+    run_case(H, N, K, 0.1, 1, f32=False, proj=idx, config=1)
+
+
+def test_zero_codes_offset_only(H):
+    """All-zero codes: the output is the offset term alone (zero trits still
+    carry the offset, paper "E2M-ATQ" on mu != 0)."""
+    from paper_2609_09240_gb300 import tq
+    N, K, M = 256, 1024, 2
+    w = wl.gen_weights(N, K, 0.1, config=6, proj=9)
+    w.T1[:] = 0
+    w.T2[:] = 0
+    x = wl.gen_x(M, K, config=6, proj=9)
+    y_ref, a_ref = H.oracle_ref(w, x)
+    y = tq.tq_linear_f32out(H.dev(x), H.pack_on_gpu(w))
+    H.assert_close(y.cpu().numpy(), y_ref, a_ref)
+
+
+def test_batched_layer(H):
+    from paper_2609_09240_gb300 import tq
+    items, refs = [], []
+    for i, (name, N, K) in enumerate(wl.QWEN3_4B):
+        w = wl.gen_weights(N, K, 0.1, config=1, proj=i)
+        x = wl.gen_x(1, K, config=1, proj=i)
+        refs.append(H.oracle_ref(w, x))
+        items.append((H.pack_on_gpu(w), H.dev(x), torch.empty((1, N), dtype=torch.float16, device="cuda")))
+    b = tq.Batch(1, items)
+    tq.tq_linear_batched(b)
+    H.device_status_ok()
+    for (pw, xd, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+
+
+def test_argument_errors(H):
+    from paper_2609_09240_gb300 import tq
+    import ctypes
+    w = wl.gen_weights(64, 256, 0.0, config=6, proj=11)
+    pw = H.pack_on_gpu(w)
+    x = torch.zeros((1, 256), dtype=torch.float16, device="cuda")
+    y = torch.empty((1, 64), dtype=torch.float16, device="cuda")
+    ws = tq.workspace(tq.tq_workspace_bytes(1, 256), "cuda")
+    L = tq.lib()
+    s = tq._stream(None)
+    ws_ = pw.struct()
+    P = lambda t: ctypes.c_void_p(t.data_ptr())
+    n = ws.numel()
+    assert L.tq_linear(0, 64, 256, ctypes.byref(ws_), P(x), P(y), P(ws), n, s) == -2
+    assert L.tq_linear(1, 64, 200, ctypes.byref(ws_), P(x), P(y), P(ws), n, s) == -2
+    assert L.tq_linear(1, 64, 256, None, P(x), P(y), P(ws), n, s) == -1
+    assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), None, n, s) == -1
+    assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), P(ws), 16, s) == -2  # workspace too small
+    xb = torch.zeros(300, dtype=torch.float16, device="cuda")[1:257]
+    assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), ctypes.c_void_p(xb.data_ptr()), P(y), P(ws), n, s) == -3
+    wb = torch.empty(n + 256, dtype=torch.uint8, device="cuda")[16:]
+    assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), ctypes.c_void_p(wb.data_ptr()), n, s) == -3
+    ws_.group = 64
+    assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), P(ws), n, s) == -2
