@@ -20,24 +20,41 @@
 // y, C and S per (group, token) are prepared once per call by
 // gemv_prep_kernel into the caller's workspace.
 //
-// Schedule (one persistent CTA per SM, a contiguous cost-balanced range of
-// 128-row tiles): every 8-group stage of a tile is handled by one of two
-// decode quads (warps 0-3, 4-7; stages alternate), thread r = row r.  Warp 8
-// streams each stage's packed rows (1-D bulk copies, 208 B per row), its
-// activation slots and C/S into a shared-memory slot ring; warp 9 issues the
-// MMAs (lane 0 for quad 0, lane 1 for quad 1): 10 MMAs (M=128, N=16, K=16)
-// per group, A from tensor memory, B from shared memory, one fp32 column
-// block per group.  After a stage the quad reads the block back once and
-// applies s1 / off.  Plane 2: the stage's salient (row, group) pairs are
-// compacted one per thread, decoded into the quad's A slot, multiplied by the
-// stage's B blocks stacked along N (each record reads its own group's
-// columns), scaled by s2 and added into the row accumulator in shared
-// memory.  The last quad to finish a tile's row writes y.
+// Roles (one persistent CTA per SM over a contiguous, cost-balanced range of
+// 128-row tiles; every tile is walked in 8-group stages):
+//  * warp 12 (producer): per stage, 1-D bulk copies of the 128 rows' packed
+//    bytes (208 B each), the stage's activation slots and C/S into a ring of
+//    shared-memory stage slots;
+//  * warps 0-3 and 4-7 (decode quads, thread r = row r): even / odd groups;
+//    each group's 26 bytes become 80 tensor-memory columns of the MMA's A
+//    operand in a 3-slot ring; decoders wait for MMAs only to reuse a slot;
+//  * warp 13 (one thread): 10 MMAs (M=128, N=16, K=16) per group into a
+//    per-group fp32 accumulator slot; the chunks of two groups are
+//    interleaved so that two accumulation chains are in flight (MMAs on one
+//    accumulator serialize), and plane-2 batches are issued as they arrive;
+//  * warps 8-11 (epilogue quad, thread r = row r): applies s1 / off per
+//    group, and runs plane 2: the stage's salient (row, group) pairs are
+//    compacted one per thread, decoded into a tensor-memory A slot and
+//    multiplied by the stage's B blocks stacked along N (each record reads
+//    its own group's columns); s2 * P2 goes to the row's shared-memory
+//    accumulator; a stage's plane-2 result is collected one stage later.
+//    The epilogue quad writes y.
 // Every wait is bounded (tq_sm100.cuh); a timeout raises a CTA-wide abort.
 #include "tq_common.cuh"
 #include "tq_sm100.cuh"
 
 namespace tq {
+
+#ifdef TQ_CHECKS
+// debugging aid (check builds only): first failed check id and its value
+static __device__ uint32_t g_check[2];
+#define TQ_CHK(cond, id, val)                                   \
+  ((cond) ? true                                                \
+          : (atomicOr(&g_tq_device_status, 8u), atomicCAS(&g_check[0], 0u, (uint32_t)(id)), \
+             atomicCAS(&g_check[1], 0u, (uint32_t)(val)), false))
+#else
+#define TQ_CHK(cond, id, val) true
+#endif
 
 namespace tc {
 
@@ -46,8 +63,9 @@ constexpr int kStageG = 8;        // groups per stage
 constexpr int kStageBytes = 208;  // plane-1 bytes per row per stage (13 x 16)
 constexpr int kACols = 80;        // tensor-memory columns of A per group (160 K slots)
 constexpr int kMmaPerGroup = 10;  // K = 16 each
-constexpr int kQuad = 128;        // threads per decode quad
-constexpr int kThreads = 320;     // 2 quads + producer warp + MMA warp
+constexpr int kQuad = 128;        // threads per quad
+constexpr int kWarpEpi = 8, kWarpProd = 12, kWarpMma = 13;
+constexpr int kThreads = 14 * 32;
 constexpr int kBHalf = 2560;      // one 8-row x 160-slot activation block
 constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
 constexpr uint32_t kDynShared = 1024;  // shared-window offset of dynamic smem
@@ -55,36 +73,37 @@ constexpr int kDynBytes = 232448;      // whole opt-in shared memory of a CTA
 constexpr int kArena1 = 65536 - (int)kDynShared;          // below the table
 constexpr int kArena2 = kDynBytes - kArena1 - kLutBytes;  // above the table
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kQuadTmem = 256;  // tensor-memory columns per quad
+constexpr int kRA = 3;  // A slots
 
 template <int MP>
 struct Cfg {
   static constexpr int NS = MP == 8 ? 3 : 2;        // stage slots
-  static constexpr int DEPTH = MP == 8 ? 2 : 1;     // A slots per quad
+  static constexpr int RD = MP == 8 ? 8 : 4;        // accumulator slots (16 columns)
   static constexpr int BGroup = (MP / 8) * kBHalf;  // activation block of one group
-  // MP = 8: group g's N=16 MMA reads rows 8..15 from group g+1's block (its
-  // columns 8..15 are overwritten by group g+1 later), so one extra block.
+  // MP = 8: an N=16 MMA of group g reads rows 8..15 from the next block
+  // (harmless: those accumulator columns are never read), hence one extra.
   static constexpr int BStage = kStageG * BGroup + (MP == 8 ? kBHalf : 0);
   static constexpr int CSGroup = 2 * MP * 4;  // C[MP], S[MP] floats
   static constexpr int CSStage = kStageG * CSGroup;
-  static constexpr int DStep = MP == 8 ? 8 : 16;    // accumulator columns per group
-  static constexpr uint32_t ColD = DEPTH * kACols;  // accumulator block offset in a quad
   static constexpr int StageBuf = kRows * kStageBytes;
-  // arena 1 (below the table): two byte buffers, record lists, barriers and,
-  // for MP = 8, the shared row accumulators
+  // tensor-memory columns
+  static constexpr uint32_t ColA = 0;
+  static constexpr uint32_t ColD = kRA * kACols;
+  static constexpr uint32_t ColA2 = ColD + RD * 16;
+  static constexpr uint32_t ColD2 = ColA2 + kACols;
+  static_assert(ColD2 + 8 * MP <= kTmemCols, "tensor memory overflow");
+  // shared memory
   static constexpr int AccBytes = 2 * kRows * MP * 4;  // 2 tile parities x 128 rows x MP
   static constexpr bool AccIn1 = MP == 8;
   static constexpr int oBytes1 = 0;
-  static constexpr int oList = oBytes1 + 2 * StageBuf;  // 2 quads x 128 x int2
-  static constexpr int oBar = oList + 2 * kRows * 8;
+  static constexpr int oList = oBytes1 + 2 * StageBuf;  // 128 x int2
+  static constexpr int oBar = oList + kRows * 8;
   static constexpr int oAcc1 = oBar + 512;
   static constexpr int kArena1Used = oAcc1 + (AccIn1 ? AccBytes : 0);
-  // arena 2 (above the table): third byte buffer, B, C/S, counters (and acc)
   static constexpr int oBytes2 = 0;
   static constexpr int oB = oBytes2 + (NS - 2) * StageBuf;
   static constexpr int oCS = oB + NS * BStage;
-  static constexpr int oCnt = oCS + NS * CSStage;  // 2 tile parities x 128 int
-  static constexpr int oAcc2 = oCnt + 2 * kRows * 4;
+  static constexpr int oAcc2 = oCS + NS * CSStage;
   static constexpr int kArena2Used = oAcc2 + (AccIn1 ? 0 : AccBytes);
   static_assert(kArena1Used <= kArena1, "arena 1 overflow");
   static_assert(kArena2Used <= kArena2, "arena 2 overflow");
@@ -92,10 +111,15 @@ struct Cfg {
 
 struct Bars {
   uint64_t full[3], empty[3];
-  uint64_t a1_full[2][2], mma_done[2][2], d1_done[2], a2_full[2], mma2_done[2];
+  uint64_t a_full[kRA], a_free[kRA];
+  uint64_t d_full[8], d_free[8];
+  uint64_t a2_full, g2_done;
   uint32_t tmem_slot;
-  uint32_t nrec[2];
-  int32_t wtot[2][4];
+  // plane-2 batch handed from the epilogue quad to the MMA thread
+  uint32_t p2_rows;   // records in the batch (0: nothing to multiply)
+  uint32_t p2_buf;    // stage slot whose activation blocks it uses
+  uint32_t p2_last;   // 1 if it is the last batch of its stage
+  int32_t wtot[4];
   int32_t abort_;
 };
 
@@ -194,6 +218,50 @@ __device__ __forceinline__ void decode_stage_group_rt(int g, const unsigned char
   }
 }
 
+// Loads the 26-byte plane-2 record j without reading past the end of plane 2
+// and returns it as 7 words (bytes 0..25, little-endian).
+__device__ __forceinline__ void load_record(const uint8_t *plane2, int64_t j, uint32_t *rw) {
+  const int64_t off0 = j * kGroupBytes;
+  const int64_t base4 = off0 & ~(int64_t)3;
+  const int sh = (int)(off0 - base4);  // 0 or 2
+  const uint32_t *src = reinterpret_cast<const uint32_t *>(plane2 + base4);
+  uint32_t r8[8];
+#pragma unroll
+  for (int i = 0; i < 6; ++i) r8[i] = __ldg(src + i);
+  r8[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
+  r8[7] = 0u;
+#pragma unroll
+  for (int i = 0; i < 7; ++i) rw[i] = sh ? __funnelshift_r(r8[i], r8[i + 1], 16) : r8[i];
+}
+
+// Iterates (tile, stage) in the CTA's order; every role walks the same list.
+struct Walk {
+  int tile, t_end, pi, s, nstages, gs;
+  const BatchParams *bp;
+  __device__ void set_tile() {
+    while (pi + 1 < bp->count && bp->prob[pi + 1].tile_begin <= tile) ++pi;
+    const int G = bp->prob[pi].K / kGroup;
+    nstages = (G + kStageG - 1) / kStageG;
+    s = 0;
+    gs = min(kStageG, G);
+  }
+  __device__ Walk(const BatchParams *b, int t0, int t1)
+      : tile(t0), t_end(t1), pi(0), s(0), nstages(0), gs(0), bp(b) {
+    if (tile < t_end) set_tile();
+  }
+  __device__ bool valid() const { return tile < t_end; }
+  __device__ const Problem &P() const { return bp->prob[pi]; }
+  __device__ bool last_stage() const { return s + 1 == nstages; }
+  __device__ void next() {
+    if (++s < nstages) {
+      const int G = bp->prob[pi].K / kGroup;
+      gs = min(kStageG, G - s * kStageG);
+    } else if (++tile < t_end) {
+      set_tile();
+    }
+  }
+};
+
 // ------------------------------------------------------------------ prep
 // Activation slots y, C (the all-zero-trit MMA value) and S = sum x for every
 // (problem, group, token); rows m in [M, MP) are zero.  Layout per problem:
@@ -253,12 +321,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   unsigned char *ar1 = dyn, *lut_p = dyn + kArena1, *ar2 = dyn + kArena1 + kLutBytes;
   const uint32_t lut_s = kDynShared + kArena1;  // 65536
-  // stage byte buffers: two below the table, the third (MP = 8) above it
   auto bytes_buf = [&](int b) -> unsigned char * {
     return b < 2 ? ar1 + C_::oBytes1 + b * C_::StageBuf : ar2 + C_::oBytes2;
   };
-  int2 *lists = reinterpret_cast<int2 *>(ar1 + C_::oList);
-  int32_t *cnt = reinterpret_cast<int32_t *>(ar2 + C_::oCnt);
+  int2 *list = reinterpret_cast<int2 *>(ar1 + C_::oList);
   Bars *bars = reinterpret_cast<Bars *>(ar1 + C_::oBar);
   unsigned char *B_p = ar2 + C_::oB;
   float *CS_p = reinterpret_cast<float *>(ar2 + C_::oCS);
@@ -272,24 +338,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t *bz = reinterpret_cast<uint32_t *>(B_p);
     for (int i = tid; i < C_::NS * C_::BStage / 4; i += kThreads) bz[i] = 0u;
     for (int i = tid; i < 2 * kRows * MP; i += kThreads) acc_s[i] = 0.f;
-    for (int i = tid; i < 2 * kRows; i += kThreads) cnt[i] = 0;
   }
   if (tid == 0) {
     for (int i = 0; i < C_::NS; ++i) {
       mbar_init(&bars->full[i], 1);
-      mbar_init(&bars->empty[i], kQuad);
+      mbar_init(&bars->empty[i], 2 * kQuad + 1);
     }
-    for (int q = 0; q < 2; ++q) {
-      for (int i = 0; i < 2; ++i) {
-        mbar_init(&bars->a1_full[q][i], kQuad);
-        mbar_init(&bars->mma_done[q][i], 1);
-      }
-      mbar_init(&bars->d1_done[q], 1);
-      mbar_init(&bars->a2_full[q], kQuad);
-      mbar_init(&bars->mma2_done[q], 1);
-      bars->nrec[q] = 0;
+    for (int i = 0; i < kRA; ++i) {
+      mbar_init(&bars->a_full[i], kQuad);
+      mbar_init(&bars->a_free[i], 1);
     }
+    for (int i = 0; i < C_::RD; ++i) {
+      mbar_init(&bars->d_full[i], 1);
+      mbar_init(&bars->d_free[i], kQuad);
+    }
+    mbar_init(&bars->a2_full, kQuad);
+    mbar_init(&bars->g2_done, 1);
     bars->abort_ = 0;
+    bars->p2_rows = 0;
+    bars->p2_buf = 0;
+    bars->p2_last = 0;
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(&bars->tmem_slot, kTmemCols);
@@ -299,261 +367,299 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_slot;
   const int t_begin = sc.cta_tile[blockIdx.x], t_end = sc.cta_tile[blockIdx.x + 1];
+  const uint32_t lane_tm = (uint32_t)((warp & 3) * 32) << 16;  // this warp's tensor-memory lanes
 
-  if (warp < 8) {
-    // =============================================================== decode
-    const int qd = warp >> 2;           // quad
-    const int r = tid & (kQuad - 1);    // row within the tile
-    const uint32_t lane_tm = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t qt = tmem + lane_tm + qd * kQuadTmem;  // this quad's tensor-memory base
+  if (warp < kWarpEpi) {
+    // ================================================================ decode
+    const int qd = warp >> 2;
+    const int r = tid & (kQuad - 1);
     const uint32_t lanebase = lut_s | ((uint32_t)lane << 2);
-    const uint32_t barid = 1 + qd;
-    int2 *list = lists + qd * kRows;
     {
       uint32_t z[16];
 #pragma unroll
       for (int i = 0; i < 16; ++i) z[i] = 0u;
-      for (int c = 0; c < C_::DEPTH * kACols; c += 16) tmem_st16(qt + c, z);
+      for (int c = qd * 16; c < kRA * kACols; c += 32) tmem_st16(tmem + lane_tm + C_::ColA + c, z);
+      tmem_wait_st();
+    }
+    uint32_t q = 0, G = 0;  // global stage and group counters
+    // the abort test is a warp vote: tcgen05.st / wait are warp-collective
+    for (Walk w(&bp, t_begin, t_end); w.valid() && !__any_sync(0xffffffffu, *abort_ != 0); w.next(), ++q) {
+      const int buf = (int)(q % C_::NS);
+      bool have_bytes = false;
+      const unsigned char *rowp = bytes_buf(buf) + r * kStageBytes;
+#pragma unroll 1
+      for (int g = 0; g < w.gs; ++g, ++G) {
+        if ((int)(G & 1u) != qd) continue;
+        if (!have_bytes) {
+          wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
+          have_bytes = true;
+        }
+        const uint32_t slot = G % kRA;
+        if (G >= (uint32_t)kRA) wait_or_abort(&bars->a_free[slot], (G / kRA - 1) & 1u, abort_);
+        uint32_t a[kACols];
+        decode_stage_group_rt(g, rowp, lanebase, a);
+        store_a(tmem + lane_tm + C_::ColA + slot * kACols, a);
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&bars->a_full[slot]);
+      }
+      // this quad is done with the stage's bytes; a quad without a group in a
+      // (partial) stage still waits for the stage to land first, so that its
+      // arrival counts toward this stage's phase of the slot
+      if (!have_bytes) wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
+      mbar_arrive(&bars->empty[buf]);
+    }
+  } else if (warp < kWarpProd) {
+    // ============================================================== epilogue
+    const int r = tid - kWarpEpi * 32;
+    const uint32_t lanebase = lut_s | ((uint32_t)lane << 2);
+    const uint32_t a2 = tmem + lane_tm + C_::ColA2;
+    {
+      uint32_t z[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) z[i] = 0u;
+      for (int c = 0; c < kACols; c += 16) tmem_st16(a2 + c, z);
       tmem_wait_st();
     }
     float acc[MP];
 #pragma unroll
     for (int m = 0; m < MP; ++m) acc[m] = 0.f;
-    uint32_t q = 0, gcount = 0, own = 0, bcount = 0;  // global stage, own groups, own stages, plane-2 batches
-    bool dec_abort = false;
-    int pi = 0;
-    for (int tile = t_begin; tile < t_end && !dec_abort; ++tile) {
-      while (pi + 1 < bp.count && bp.prob[pi + 1].tile_begin <= tile) ++pi;
-      const Problem &P = bp.prob[pi];
-      const int K = P.K, G = K / kGroup, W = sal_words_of(K);
-      const int n0 = (tile - P.tile_begin) * kRows;
-      const int n = n0 + r;
-      const bool valid = n < P.N;
-      const int nstages = (G + kStageG - 1) / kStageG;
-      const int tpar = tile & 1;
-      for (int s = 0; s < nstages && !dec_abort; ++s, ++q) {
-        if ((int)(q & 1u) != qd) continue;
-        const int gs = min(kStageG, G - s * kStageG);
-        const int g0 = s * kStageG;
-        const int buf = (int)(q % C_::NS);
-        // ---- per-row data of the stage, loaded early
-        float s1v[kStageG], offv[kStageG];
-        uint32_t bits = 0;
-        int j0 = 0;
+    uint32_t q = 0, G = 0, bc = 0;
+    // the plane-2 batch whose MMA is in flight
+    bool pend = false;
+    int pend_buf = 0, pend_gs = 0, pend_rows = 0;
+    int2 pend_rec = make_int2(-1, 0);
+    float pend_s2 = 0.f;
+    // the tile whose y is written when its last stage's plane 2 is collected
+    bool fin = false, fin_valid = false;
+    int fin_par = 0, fin_n = 0, fin_N = 0;
+    void *fin_y = nullptr;
+
+    // collects the batch in flight: s2 * P2 of every record into acc_s
+    auto collect = [&](bool release_stage) {
+      wait_or_abort(&bars->g2_done, bc & 1u, abort_);
+      ++bc;
+      tc_fence_after();
+      if (pend_rows > 0) {
+        const int g = pend_rec.x >= 0 ? ((pend_rec.x >> 8) & 0xff) : 0;  // bits 8..15: group
+        uint32_t d[16];
 #pragma unroll
-        for (int g = 0; g < kStageG; ++g) {
-          s1v[g] = (valid && g < gs) ? __half2float(P.s1[(int64_t)n * G + g0 + g]) : 0.f;
-          offv[g] = (valid && g < gs) ? __half2float(P.off[(int64_t)n * G + g0 + g]) : 0.f;
-        }
-        if (valid) {
-          const uint32_t *srow = P.sal + (int64_t)n * W;
-          const uint32_t word = srow[g0 >> 5];
-          bits = (word >> (g0 & 31)) & ((1u << gs) - 1u);
-          if (bits) {
-            int before = 0;
-            for (int w = 0; w < (g0 >> 5); ++w) before += __popc(srow[w]);
-            before += __popc(word & ((1u << (g0 & 31)) - 1u));
-            j0 = P.rowptr[n] + before;
-          }
-        }
-        // ---- plane 1
-        wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
-        const unsigned char *rowp = bytes_buf(buf) + r * kStageBytes;
+        for (int i = 0; i < 16; ++i) d[i] = 0u;
+        // one column address per warp-collective load: walk the groups
 #pragma unroll 1
-        for (int g = 0; g < gs; ++g, ++gcount) {
-          const uint32_t slot = gcount % C_::DEPTH;
-          const uint32_t use = gcount / C_::DEPTH;
-          if (use > 0) wait_or_abort(&bars->mma_done[qd][slot], (use - 1) & 1u, abort_);
-          uint32_t a[kACols];
-          decode_stage_group_rt(g, rowp, lanebase, a);
-          store_a(qt + slot * kACols, a);
-          tmem_wait_st();
-          tc_fence_before();
-          mbar_arrive(&bars->a1_full[qd][slot]);
-        }
-        // ---- compact this stage's plane-2 records (one per thread)
-        const int c = __popc(bits);
-        int incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int v = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += v;
-        }
-        if (lane == 31) bars->wtot[qd][warp & 3] = incl;
-        named_bar(barid, kQuad);
-        int wbase = 0, total = 0;
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const int t = bars->wtot[qd][w];
-          wbase += w < (warp & 3) ? t : 0;
-          total += t;
-        }
-        const int my0 = wbase + incl - c;
-        // ---- epilogue of plane 1 (one accumulator column block per group)
-        wait_or_abort(&bars->d1_done[qd], own & 1u, abort_);
-        tc_fence_after();
-        const float *cs = CS_p + buf * (C_::CSStage / 4);
-#pragma unroll 1
-        for (int g = 0; g < gs; ++g) {
-          uint32_t d[16];
-          tmem_ld_cols<MP>(qt + C_::ColD + g * C_::DStep, d);
+        for (int gg = 0; gg < pend_gs; ++gg) {
+          uint32_t t[16];
+          tmem_ld_cols<MP>(tmem + lane_tm + C_::ColD2 + gg * MP, t);
           tmem_wait_ld();
-          const float *Cg = cs + g * 2 * MP, *Sg = Cg + MP;
-          float s1g = 0.f, offg = 0.f;
+          if (gg == g) {
 #pragma unroll
-          for (int gg = 0; gg < kStageG; ++gg)
-            if (gg == g) {
-              s1g = s1v[gg];
-              offg = offv[gg];
-            }
-#pragma unroll
-          for (int m = 0; m < MP; ++m) acc[m] = fmaf(s1g, __uint_as_float(d[m]) - Cg[m], fmaf(offg, Sg[m], acc[m]));
+            for (int i = 0; i < MP; ++i) d[i] = t[i];
+          }
         }
-        // ---- plane 2 of the stage, in batches of 128 records
-        for (int b0 = 0;; b0 += kRows) {
-          named_bar(barid, kQuad);  // earlier readers of the list are done
-          {
-            int o = my0, jj = j0;
-            uint32_t bb = bits;
-            while (bb) {
-              const int g = __ffs(bb) - 1;
-              bb &= bb - 1;
-              if (o >= b0 && o < b0 + kRows) list[o - b0] = make_int2(r | (g << 8), jj);
-              ++o;
-              ++jj;
-            }
-          }
-          if (r == 0) bars->nrec[qd] = (uint32_t)total;
-          named_bar(barid, kQuad);
-          const int rows_here = min(total - b0, kRows);
-          int2 rec = make_int2(-1, 0);
-          uint32_t a[kACols];
-          if (r < rows_here && P.nnz > 0) {
-            rec = list[r];
-            const int64_t jj = min(max((int64_t)rec.y, (int64_t)0), (int64_t)P.nnz - 1);
-            const int64_t off0 = jj * kGroupBytes;
-            const int64_t base4 = off0 & ~(int64_t)3;
-            const int sh = (int)(off0 - base4);  // 0 or 2
-            const uint32_t *src = reinterpret_cast<const uint32_t *>(P.plane2 + base4);
-            uint32_t r8[8];
-#pragma unroll
-            for (int i = 0; i < 6; ++i) r8[i] = __ldg(src + i);
-            // the record's last bytes without reading past the end of plane 2
-            r8[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
-            r8[7] = 0u;
-            uint32_t rw[7];
-#pragma unroll
-            for (int i = 0; i < 7; ++i) rw[i] = sh ? __funnelshift_r(r8[i], r8[i + 1], 16) : r8[i];
-            decode_group<0>(rw, lanebase, a);
-          } else {
-#pragma unroll
-            for (int i = 0; i < kACols; ++i) a[i] = 0u;
-          }
-          store_a(qt, a);  // A slot 0 is free: every plane-1 MMA of the stage is done
-          tmem_wait_st();
-          tc_fence_before();
-          mbar_arrive(&bars->a2_full[qd]);
-          wait_or_abort(&bars->mma2_done[qd], bcount & 1u, abort_);
-          ++bcount;
-          tc_fence_after();
-          if (rows_here > 0) {
-            const int g = rec.x >= 0 ? (rec.x >> 8) : 0;
-            uint32_t d[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) d[i] = 0u;
-            // one column address per warp-collective load: walk the groups
-#pragma unroll 1
-            for (int gg = 0; gg < gs; ++gg) {
-              uint32_t t[16];
-              tmem_ld_cols<MP>(qt + C_::ColD + gg * MP, t);
-              tmem_wait_ld();
-              if (gg == g) {
-#pragma unroll
-                for (int i = 0; i < MP; ++i) d[i] = t[i];
-              }
-            }
-            if (rec.x >= 0) {
-              const float s2 = __half2float(P.s2[min(max(rec.y, 0), P.nnz - 1)]);
-              const float *Cg = cs + g * 2 * MP;
-              float *dst = acc_s + (tpar * kRows + (rec.x & 0xff)) * MP;
-#pragma unroll
-              for (int m = 0; m < MP; ++m)
-                if (m < M) atomicAdd(dst + m, s2 * (__uint_as_float(d[m]) - Cg[m]));
-            }
-          }
-          if (b0 + kRows >= total) break;
-        }
-        named_bar(barid, kQuad);  // the stage's plane-2 atomics are complete
-        mbar_arrive(&bars->empty[buf]);
-        ++own;
-        // ---- this quad's last stage of the tile: hand the row over
-        if (s + 2 >= nstages) {
-          const int quads = nstages >= 2 ? 2 : 1;
-          float *dst = acc_s + (tpar * kRows + r) * MP;
+        if (pend_rec.x >= 0 && TQ_CHK(g < kStageG && pend_buf < C_::NS && (pend_rec.x & 0xff) < kRows, 1, pend_rec.x)) {
+          const float *Cg = CS_p + pend_buf * (C_::CSStage / 4) + g * 2 * MP;
+          const int par = (pend_rec.x >> 16) & 1;  // bit 16: tile parity
+          float *dst = acc_s + (par * kRows + (pend_rec.x & 0xff)) * MP;
 #pragma unroll
           for (int m = 0; m < MP; ++m)
-            if (m < M) atomicAdd(dst + m, acc[m]);
-          __threadfence_block();
-          const int prev = atomicAdd(cnt + tpar * kRows + r, 1);
-          if (prev == quads - 1) {
-            __threadfence_block();
-            if (valid) {
+            if (m < M) atomicAdd(dst + m, pend_s2 * (__uint_as_float(d[m]) - Cg[m]));
+        }
+      }
+      tc_fence_before();
+      named_bar(1, kQuad);  // the batch's contributions are in acc_s; A2 / D2 are free
+      pend = false;
+      if (release_stage && r == 0) mbar_arrive(&bars->empty[pend_buf]);
+      if (release_stage && fin) {
+        float *src = acc_s + (fin_par * kRows + r) * MP;
+        if (fin_valid) {
 #pragma unroll
-              for (int m = 0; m < MP; ++m) {
-                if (m < M) {
-                  const float v = atomicAdd(dst + m, 0.f);
-                  if (F32)
-                    static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
-                  else
-                    static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
-                }
-              }
+          for (int m = 0; m < MP; ++m) {
+            if (m < M) {
+              const float v = src[m];
+              if (F32)
+                static_cast<float *>(fin_y)[(int64_t)m * fin_N + fin_n] = v;
+              else
+                static_cast<__half *>(fin_y)[(int64_t)m * fin_N + fin_n] = __float2half_rn(v);
             }
+          }
+        }
 #pragma unroll
-            for (int m = 0; m < MP; ++m) dst[m] = 0.f;
-            cnt[tpar * kRows + r] = 0;
+        for (int m = 0; m < MP; ++m) src[m] = 0.f;
+        fin = false;
+      }
+    };
+
+    bool eq_abort = false;  // uniform across the quad (decided at a barrier)
+    for (Walk w(&bp, t_begin, t_end); w.valid() && !eq_abort; w.next(), ++q) {
+      const Problem &P = w.P();
+      const int K = P.K, Gk = K / kGroup, W = sal_words_of(K);
+      const int n = (w.tile - P.tile_begin) * kRows + r;
+      const bool valid = n < P.N;
+      const int g0 = w.s * kStageG, gs = w.gs;
+      const int buf = (int)(q % C_::NS);
+      const int tpar = w.tile & 1;
+      // ---- per-row data of the stage
+      float s1v[kStageG], offv[kStageG];
+#pragma unroll
+      for (int g = 0; g < kStageG; ++g) {
+        s1v[g] = (valid && g < gs) ? __half2float(P.s1[(int64_t)n * Gk + g0 + g]) : 0.f;
+        offv[g] = (valid && g < gs) ? __half2float(P.off[(int64_t)n * Gk + g0 + g]) : 0.f;
+      }
+      uint32_t bits = 0;
+      int j0 = 0;
+      if (valid) {
+        const uint32_t *srow = P.sal + (int64_t)n * W;
+        const uint32_t word = srow[g0 >> 5];
+        bits = (word >> (g0 & 31)) & ((1u << gs) - 1u);
+        if (bits) {
+          int before = 0;
+          for (int ww = 0; ww < (g0 >> 5); ++ww) before += __popc(srow[ww]);
+          before += __popc(word & ((1u << (g0 & 31)) - 1u));
+          j0 = P.rowptr[n] + before;
+        }
+      }
+      // ---- plane 1: one accumulator slot per group
+      wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
+      const float *cs = CS_p + buf * (C_::CSStage / 4);
+#pragma unroll 1
+      for (int g = 0; g < gs; ++g, ++G) {
+        const uint32_t ds = G % C_::RD;
+        wait_or_abort(&bars->d_full[ds], (G / C_::RD) & 1u, abort_);
+        tc_fence_after();
+        uint32_t d[16];
+        tmem_ld_cols<MP>(tmem + lane_tm + C_::ColD + ds * 16, d);
+        tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(&bars->d_free[ds]);
+        const float *Cg = cs + g * 2 * MP, *Sg = Cg + MP;
+        float s1g = 0.f, offg = 0.f;
+#pragma unroll
+        for (int gg = 0; gg < kStageG; ++gg)
+          if (gg == g) {
+            s1g = s1v[gg];
+            offg = offv[gg];
           }
 #pragma unroll
-          for (int m = 0; m < MP; ++m) acc[m] = 0.f;
-        }
-        dec_abort = named_bar_any(barid, kQuad, *abort_ != 0);
+        for (int m = 0; m < MP; ++m) acc[m] = fmaf(s1g, __uint_as_float(d[m]) - Cg[m], fmaf(offg, Sg[m], acc[m]));
       }
+      if (w.last_stage()) {
+        // the row's plane-1 part is complete: park it in the tile's slot
+        float *dst = acc_s + (tpar * kRows + r) * MP;
+#pragma unroll
+        for (int m = 0; m < MP; ++m) {
+          if (m < M) atomicAdd(dst + m, acc[m]);
+          acc[m] = 0.f;
+        }
+      }
+      // ---- plane 2 of the previous stage
+      if (pend) collect(true);
+      // ---- plane 2 of this stage: compact the salient (row, group) pairs
+      const int c = __popc(bits);
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      if (lane == 31) bars->wtot[warp & 3] = incl;
+      named_bar(1, kQuad);
+      int wbase = 0, total = 0;
+#pragma unroll
+      for (int ww = 0; ww < 4; ++ww) {
+        const int t = bars->wtot[ww];
+        wbase += ww < (warp & 3) ? t : 0;
+        total += t;
+      }
+      const int my0 = wbase + incl - c;
+      const int nb = total > kRows ? (total + kRows - 1) / kRows : 1;
+      for (int b = 0; b < nb; ++b) {
+        const int b0 = b * kRows;
+        // more than 128 pairs in one stage (rare): the earlier batch is
+        // collected first, its A / D slots are reused
+        if (b > 0) collect(false);
+        {
+          int o = my0, jj = j0;
+          uint32_t bb = bits;
+          while (bb) {
+            const int g = __ffs(bb) - 1;
+            bb &= bb - 1;
+            if (o >= b0 && o < b0 + kRows && TQ_CHK(g < gs, 2, g)) list[o - b0] = make_int2(r | (g << 8) | (tpar << 16), jj);
+            ++o;
+            ++jj;
+          }
+        }
+        const int rows_here = min(total - b0, kRows);
+        if (r == 0) {
+          bars->p2_rows = (uint32_t)rows_here;
+          bars->p2_buf = (uint32_t)buf;
+          bars->p2_last = b + 1 == nb ? 1u : 0u;
+        }
+        named_bar(1, kQuad);
+        int2 rec = make_int2(-1, 0);
+        float s2v = 0.f;
+        uint32_t a[kACols];
+        if (r < rows_here && P.nnz > 0 && TQ_CHK(rows_here <= kRows, 3, rows_here)) {
+          rec = list[r];
+          TQ_CHK(rec.y >= 0 && rec.y < P.nnz, 4, rec.y);
+          const int jj = min(max(rec.y, 0), P.nnz - 1);
+          s2v = __half2float(P.s2[jj]);
+          uint32_t rw[7];
+          load_record(P.plane2, jj, rw);
+          decode_group<0>(rw, lanebase, a);
+        } else {
+#pragma unroll
+          for (int i = 0; i < kACols; ++i) a[i] = 0u;
+        }
+        store_a(a2, a);
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&bars->a2_full);
+        pend = true;
+        pend_buf = buf;
+        pend_gs = gs;
+        pend_rows = rows_here;
+        pend_rec = rec;
+        pend_s2 = s2v;
+      }
+      if (w.last_stage()) {
+        fin = true;
+        fin_valid = valid;
+        fin_par = tpar;
+        fin_n = n;
+        fin_N = P.N;
+        fin_y = P.y;
+      }
+      eq_abort = named_bar_any(1, kQuad, *abort_ != 0);
     }
-  } else if (warp == 8) {
-    // ============================================================ producer
+    if (pend && !eq_abort) collect(true);
+  } else if (warp == kWarpProd) {
+    // ============================================================== producer
     uint32_t q = 0;
-    int pi = 0;
-    bool stop = false;
-    for (int tile = t_begin; tile < t_end && !stop; ++tile) {
-      while (pi + 1 < bp.count && bp.prob[pi + 1].tile_begin <= tile) ++pi;
-      const Problem &P = bp.prob[pi];
-      const int K = P.K, G = K / kGroup;
-      const int64_t RB = row_bytes_of(K);
-      const int n0 = (tile - P.tile_begin) * kRows;
+    for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
+      const Problem &P = w.P();
+      const int64_t RB = row_bytes_of(P.K);
+      const int n0 = (w.tile - P.tile_begin) * kRows;
       const int rows = min(kRows, P.N - n0);
-      const int nstages = (G + kStageG - 1) / kStageG;
-      for (int s = 0; s < nstages; ++s, ++q) {
-        const int gs = min(kStageG, G - s * kStageG);
-        const uint32_t rb = (uint32_t)((gs * kGroupBytes + 15) / 16 * 16);
-        const uint32_t bb = (uint32_t)(gs * C_::BGroup);
-        const uint32_t cb = (uint32_t)(gs * C_::CSGroup);
-        const int buf = (int)(q % C_::NS);
-        if (!wait_or_abort(&bars->empty[buf], ((q / C_::NS) & 1u) ^ 1u, abort_)) {
-          stop = true;
-          break;
-        }
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&bars->full[buf], rb * (uint32_t)rows + bb + cb);
-          bulk_g2s(B_p + buf * C_::BStage, P.wsB + (int64_t)s * kStageG * C_::BGroup, bb, &bars->full[buf]);
-          bulk_g2s(reinterpret_cast<unsigned char *>(CS_p) + buf * C_::CSStage,
-                   reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)s * kStageG * C_::CSGroup, cb,
-                   &bars->full[buf]);
-        }
-        __syncwarp();
-        for (int rr = lane; rr < rows; rr += 32)
-          bulk_g2s(bytes_buf(buf) + rr * kStageBytes,
-                   P.plane1 + (int64_t)(n0 + rr) * RB + (int64_t)s * kStageBytes, rb, &bars->full[buf]);
+      const int s = w.s, gs = w.gs;
+      const uint32_t rb = (uint32_t)((gs * kGroupBytes + 15) / 16 * 16);
+      const uint32_t bb = (uint32_t)(gs * C_::BGroup);
+      const uint32_t cb = (uint32_t)(gs * C_::CSGroup);
+      const int buf = (int)(q % C_::NS);
+      int ok = 1;
+      if (lane == 0) ok = wait_or_abort(&bars->empty[buf], ((q / C_::NS) & 1u) ^ 1u, abort_) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars->full[buf], rb * (uint32_t)rows + bb + cb);
+        bulk_g2s(B_p + buf * C_::BStage, P.wsB + (int64_t)s * kStageG * C_::BGroup, bb, &bars->full[buf]);
+        bulk_g2s(reinterpret_cast<unsigned char *>(CS_p) + buf * C_::CSStage,
+                 reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)s * kStageG * C_::CSGroup, cb,
+                 &bars->full[buf]);
       }
+      __syncwarp();
+      TQ_CHK((int64_t)s * kStageBytes + rb <= RB && rows >= 1 && rows <= kRows, 7, s * 1000 + rows);
+      for (int rr = lane; rr < rows; rr += 32)
+        bulk_g2s(bytes_buf(buf) + rr * kStageBytes, P.plane1 + (int64_t)(n0 + rr) * RB + (int64_t)s * kStageBytes,
+                 rb, &bars->full[buf]);
     }
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
@@ -561,64 +667,92 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (uint32_t k = (q > (uint32_t)C_::NS ? q - C_::NS : 0); k < q; ++k)
         mbar_wait(&bars->full[k % C_::NS], (k / C_::NS) & 1u);
     }
-  } else if (lane < 2) {
-    // ================================================================= MMA
-    const int qd = lane;  // lane 0 serves quad 0, lane 1 quad 1
-    const uint32_t qt = tmem + qd * kQuadTmem;
+  } else if (warp == kWarpMma && lane == 0) {
+    // =================================================================== MMA
     const uint32_t idesc1 = idesc_f16_f32(128, 16);
     const uint32_t idesc2 = idesc_f16_f32(128, 8 * MP);
-    uint32_t q = 0, gcount = 0, bcount = 0;
-    int pi = 0;
+    uint32_t q = 0, G = 0, bc = 0;
+    uint32_t p2_stages_done = 0;
     bool stop = false;
-    for (int tile = t_begin; tile < t_end && !stop; ++tile) {
-      while (pi + 1 < bp.count && bp.prob[pi + 1].tile_begin <= tile) ++pi;
-      const Problem &P = bp.prob[pi];
-      const int G = P.K / kGroup;
-      const int nstages = (G + kStageG - 1) / kStageG;
-      for (int s = 0; s < nstages && !stop; ++s, ++q) {
-        if ((int)(q & 1u) != qd) continue;
-        const int gs = min(kStageG, G - s * kStageG);
-        const int buf = (int)(q % C_::NS);
-        const uint32_t Bst = smem_u32(B_p + buf * C_::BStage);
-        for (int g = 0; g < gs; ++g, ++gcount) {
-          const uint32_t slot = gcount % C_::DEPTH;
-          if (!wait_or_abort(&bars->a1_full[qd][slot], (gcount / C_::DEPTH) & 1u, abort_)) {
-            stop = true;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t bg = Bst + g * C_::BGroup;
-#pragma unroll
-          for (int i = 0; i < kMmaPerGroup; ++i)
-            mma_tmemA(qt + C_::ColD + g * C_::DStep, qt + slot * kACols + 8 * i,
-                      smem_desc(bg + 2 * i * 128, 128, kBHalf), idesc1, i > 0 ? 1u : 0u);
-          mma_commit(&bars->mma_done[qd][slot]);
+    // issues the next plane-2 batch if the epilogue has handed one over
+    auto try_plane2 = [&](bool block) -> bool {
+      if (block) {
+        if (!wait_or_abort(&bars->a2_full, bc & 1u, abort_)) {
+          stop = true;
+          return false;
         }
-        if (stop) break;
-        mma_commit(&bars->d1_done[qd]);
-        // plane-2 batches of the stage (at least one, possibly empty)
-        uint32_t nb = 1;
-        for (uint32_t b = 0; b < nb; ++b) {
-          if (!wait_or_abort(&bars->a2_full[qd], bcount & 1u, abort_)) {
-            stop = true;
-            break;
-          }
-          ++bcount;
-          tc_fence_after();
-          const uint32_t total = bars->nrec[qd];
-          nb = total > (uint32_t)kRows ? (total + kRows - 1) / kRows : 1u;
-          if (total > b * (uint32_t)kRows) {
+      } else if (!mbar_try_wait(&bars->a2_full, bc & 1u)) {
+        return false;
+      }
+      ++bc;
+      tc_fence_after();
+      const uint32_t rows = bars->p2_rows, buf = bars->p2_buf, last = bars->p2_last;
+      if (rows > 0 && TQ_CHK(buf < (uint32_t)C_::NS && rows <= (uint32_t)kRows, 5, buf * 1000 + rows)) {
+        const uint32_t Bst = smem_u32(B_p + buf * C_::BStage);
 #pragma unroll
-            for (int i = 0; i < kMmaPerGroup; ++i)
-              mma_tmemA(qt + C_::ColD, qt + 8 * i, smem_desc(Bst + 2 * i * 128, 128, kBHalf), idesc2,
-                        i > 0 ? 1u : 0u);
-            mma_commit(&bars->mma2_done[qd]);
-          } else {
-            mbar_arrive(&bars->mma2_done[qd]);
+        for (int i = 0; i < kMmaPerGroup; ++i)
+          mma_tmemA(tmem + C_::ColD2, tmem + C_::ColA2 + 8 * i, smem_desc(Bst + 2 * i * 128, 128, kBHalf), idesc2,
+                    i > 0 ? 1u : 0u);
+        mma_commit(&bars->g2_done);
+      } else {
+        mbar_arrive(&bars->g2_done);
+      }
+      p2_stages_done += last;
+      return true;
+    };
+    // waits for `bar`, issuing plane-2 batches while it is not ready
+    auto wait_serving = [&](uint64_t *bar, uint32_t parity) -> bool {
+      const uint64_t t0 = global_ns();
+      for (uint32_t i = 0;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        try_plane2(false);
+        if ((i & 63u) == 63u) {
+          if (*abort_) return false;
+          if (global_ns() - t0 > kWaitLimitNs) {
+            atomicOr(&g_tq_device_status, kStatusTimeout);
+            *abort_ = 1;
+            return false;
           }
         }
       }
+    };
+    for (Walk w(&bp, t_begin, t_end); w.valid() && !stop; w.next(), ++q) {
+      const int buf = (int)(q % C_::NS);
+      const uint32_t Bst = smem_u32(B_p + buf * C_::BStage);
+      // plane 1: groups in pairs, chunks interleaved (two accumulation chains)
+      for (int g = 0; g < w.gs && !stop; g += 2) {
+        const int ng = min(2, w.gs - g);
+        for (int k = 0; k < ng && !stop; ++k) {
+          const uint32_t Gk = G + k;
+          if (!wait_serving(&bars->a_full[Gk % kRA], (Gk / kRA) & 1u)) stop = true;
+          if (!stop && Gk >= (uint32_t)C_::RD && !wait_serving(&bars->d_free[Gk % C_::RD], (Gk / C_::RD - 1) & 1u))
+            stop = true;
+        }
+        if (stop) break;
+        tc_fence_after();
+        if (!TQ_CHK(g + ng <= kStageG && buf < C_::NS, 6, g * 100 + ng)) {
+          stop = true;
+          break;
+        }
+#pragma unroll 1
+        for (int i = 0; i < kMmaPerGroup; ++i) {
+          for (int k = 0; k < ng; ++k) {
+            const uint32_t Gk = G + k;
+            const uint32_t bg = Bst + (g + k) * C_::BGroup;
+            mma_tmemA(tmem + C_::ColD + (Gk % C_::RD) * 16, tmem + C_::ColA + (Gk % kRA) * kACols + 8 * i,
+                      smem_desc(bg + 2 * i * 128, 128, kBHalf), idesc1, i > 0 ? 1u : 0u);
+          }
+        }
+        for (int k = 0; k < ng; ++k) {
+          const uint32_t Gk = G + k;
+          mma_commit(&bars->a_free[Gk % kRA]);
+          mma_commit(&bars->d_full[Gk % C_::RD]);
+        }
+        G += ng;
+      }
     }
+    // the remaining plane-2 batches: one stage's last batch per stage
+    while (!stop && p2_stages_done < q) try_plane2(true);
   }
 
   tc_fence_before();
@@ -658,6 +792,12 @@ size_t tc_workspace_b_bytes(int M, int K) {
 }
 
 TQ_STATUS_ACCESSOR(read_status_gemv_tc)
+
+#ifdef TQ_CHECKS
+extern "C" __attribute__((visibility("default"))) int tq_debug_checks(uint32_t *out) {
+  return (int)cudaMemcpyFromSymbol(out, g_check, sizeof(uint32_t) * 2);
+}
+#endif
 
 template <int MP, bool F32>
 static cudaError_t launch_tc(const BatchParams &bp, cudaStream_t s) {
