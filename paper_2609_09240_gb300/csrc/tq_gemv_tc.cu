@@ -45,6 +45,19 @@
 
 namespace tq {
 
+#ifdef TQ_TRACE
+// debugging aid (trace builds only): clock64 stamps from CTA 0
+static __device__ unsigned long long g_trace[4096];
+#define TQ_STAMP(idx)                                                        \
+  do {                                                                       \
+    if (blockIdx.x == 0 && (idx) < 4096) g_trace[(idx)] = clock64();         \
+  } while (0)
+#else
+#define TQ_STAMP(idx) \
+  do {                \
+  } while (0)
+#endif
+
 #ifdef TQ_CHECKS
 // debugging aid (check builds only): first failed check id and its value
 static __device__ uint32_t g_check[2];
@@ -390,18 +403,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
       for (int g = 0; g < w.gs; ++g, ++G) {
         if ((int)(G & 1u) != qd) continue;
+        const bool st0 = (tid == 0 && G < 512);
+        if (st0) TQ_STAMP((G / 2) * 4 + 0);
         if (!have_bytes) {
           wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
           have_bytes = true;
         }
         const uint32_t slot = G % kRA;
         if (G >= (uint32_t)kRA) wait_or_abort(&bars->a_free[slot], (G / kRA - 1) & 1u, abort_);
+        if (st0) TQ_STAMP((G / 2) * 4 + 1);
         uint32_t a[kACols];
         decode_stage_group_rt(g, rowp, lanebase, a);
+        if (st0) TQ_STAMP((G / 2) * 4 + 2);
         store_a(tmem + lane_tm + C_::ColA + slot * kACols, a);
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&bars->a_full[slot]);
+        if (st0) TQ_STAMP((G / 2) * 4 + 3);
       }
       // this quad is done with the stage's bytes; a quad without a group in a
       // (partial) stage still waits for the stage to land first, so that its
@@ -518,8 +536,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           j0 = P.rowptr[n] + before;
         }
       }
+      const bool se = (r == 0 && q < 128);
+      if (se) TQ_STAMP(1024 + q * 8 + 0);
       // ---- plane 1: one accumulator slot per group
       wait_or_abort(&bars->full[buf], (q / C_::NS) & 1u, abort_);
+      if (se) TQ_STAMP(1024 + q * 8 + 1);
       const float *cs = CS_p + buf * (C_::CSStage / 4);
 #pragma unroll 1
       for (int g = 0; g < gs; ++g, ++G) {
@@ -542,6 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int m = 0; m < MP; ++m) acc[m] = fmaf(s1g, __uint_as_float(d[m]) - Cg[m], fmaf(offg, Sg[m], acc[m]));
       }
+      if (se) TQ_STAMP(1024 + q * 8 + 2);
       if (w.last_stage()) {
         // the row's plane-1 part is complete: park it in the tile's slot
         float *dst = acc_s + (tpar * kRows + r) * MP;
@@ -553,6 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // ---- plane 2 of the previous stage
       if (pend) collect(true);
+      if (se) TQ_STAMP(1024 + q * 8 + 3);
       // ---- plane 2 of this stage: compact the salient (row, group) pairs
       const int c = __popc(bits);
       int incl = c;
@@ -610,10 +633,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int i = 0; i < kACols; ++i) a[i] = 0u;
         }
+        if (se) TQ_STAMP(1024 + q * 8 + 4);
         store_a(a2, a);
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&bars->a2_full);
+        if (se) TQ_STAMP(1024 + q * 8 + 5);
         pend = true;
         pend_buf = buf;
         pend_gs = gs;
@@ -630,6 +655,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         fin_y = P.y;
       }
       eq_abort = named_bar_any(1, kQuad, *abort_ != 0);
+      if (se) TQ_STAMP(1024 + q * 8 + 6);
     }
     if (pend && !eq_abort) collect(true);
   } else if (warp == kWarpProd) {
@@ -729,6 +755,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             stop = true;
         }
         if (stop) break;
+        if (G / 2 < 512) TQ_STAMP(2048 + (G / 2) * 2);
         tc_fence_after();
         if (!TQ_CHK(g + ng <= kStageG && buf < C_::NS, 6, g * 100 + ng)) {
           stop = true;
@@ -748,6 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(&bars->a_free[Gk % kRA]);
           mma_commit(&bars->d_full[Gk % C_::RD]);
         }
+        if (G / 2 < 512) TQ_STAMP(2048 + (G / 2) * 2 + 1);
         G += ng;
       }
     }
@@ -792,6 +820,12 @@ size_t tc_workspace_b_bytes(int M, int K) {
 }
 
 TQ_STATUS_ACCESSOR(read_status_gemv_tc)
+
+#ifdef TQ_TRACE
+extern "C" __attribute__((visibility("default"))) int tq_debug_trace(unsigned long long *out, int n) {
+  return (int)cudaMemcpyFromSymbol(out, g_trace, sizeof(unsigned long long) * (n < 4096 ? n : 4096));
+}
+#endif
 
 #ifdef TQ_CHECKS
 extern "C" __attribute__((visibility("default"))) int tq_debug_checks(uint32_t *out) {
