@@ -89,7 +89,7 @@ typedef struct {
   const uint8_t *plane1;    /* [N][tq_row_bytes(K)], 16-byte aligned           */
   const uint32_t *salience; /* [N][tq_sal_words(K)], bit g%32 of word g/32     */
   const int32_t *rowptr;    /* [N+1], exclusive prefix count of salient groups */
-  const uint8_t *plane2;    /* [nnz][26]; may be NULL when nnz == 0            */
+  const uint8_t *plane2;    /* [nnz][26], 16-byte aligned; NULL when nnz == 0  */
   const uint16_t *scale1;   /* fp16 bits [N][G]                                */
   const uint16_t *offset;   /* fp16 bits [N][G]                                */
   const uint16_t *scale2;   /* fp16 bits [nnz]; may be NULL when nnz == 0      */
@@ -132,17 +132,20 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
 
 /* Device workspace of the decode path (M <= TQ_MAX_SKINNY_M): the
  * activations of every call are first rearranged into the tensor-core
- * operand order of the packed weights (with the per-group correction terms).
- * The caller provides this scratch memory (the library never allocates).
- * Bytes needed for one projection with K inputs and M tokens (M > 16 needs
- * the M = 16 amount); 0 if K is invalid. */
-TQ_API size_t tq_workspace_bytes(int32_t M, int32_t K);
+ * operand order of the packed weights (with the per-group correction terms),
+ * and for M <= 8 the second plane's fp32 partial sums of every row are
+ * staged there before the first plane is streamed.  The caller provides this
+ * scratch memory (the library never allocates).  Bytes needed for one
+ * projection of N rows, K inputs and M tokens (a call with M > 16 runs in
+ * chunks of 16 and needs the amount returned for its M); 0 if M, N or K is
+ * invalid. */
+TQ_API size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K);
 
 /* y = x W^T for one packed projection (paper "Direct Packed Execution").
  *   x: fp16 [M][K] row-major, 16-byte aligned; y: fp16 [M][N] (rounded to
  *   nearest even from the fp32 accumulator).  M >= 1; M is processed in
  *   chunks of TQ_MAX_SKINNY_M tokens on the decode path.
- *   workspace: device scratch of at least tq_workspace_bytes(M, K) bytes,
+ *   workspace: device scratch of at least tq_workspace_bytes(M, N, K) bytes,
  *   256-byte aligned; its contents are overwritten; calls that share a
  *   workspace must not overlap in time.
  * The packed bytes are trusted (produced by tq_pack): no per-byte

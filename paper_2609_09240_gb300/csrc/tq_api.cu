@@ -23,6 +23,10 @@ int tc_rows_per_tile();
 size_t tc_workspace_bytes(int M, int K);
 size_t tc_workspace_b_bytes(int M, int K);
 cudaError_t read_status_gemv_tc(uint32_t *out, bool clear);
+cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
+int mma_rows_per_tile();
+void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
+cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
 }  // namespace tq
 
 using namespace tq;
@@ -50,7 +54,8 @@ tq_status check_weight(const tq_weight *w, int32_t N, int32_t K) {
   if (w->nnz < 0 || w->nnz > (int64_t)N * (K / TQ_GROUP)) return TQ_ERR_SALIENCE;
   if (w->nnz > 0 && (!w->plane2 || !w->scale2)) return TQ_ERR_NULL;
   if (!aligned16(w->plane1)) return TQ_ERR_ALIGN;
-  if (!aligned2(w->scale1) || !aligned2(w->offset) || (w->plane2 && !aligned2(w->plane2)) ||
+  if (w->plane2 && !aligned16(w->plane2)) return TQ_ERR_ALIGN;
+  if (!aligned2(w->scale1) || !aligned2(w->offset) ||
       (w->scale2 && !aligned2(w->scale2)) || ((uintptr_t)w->salience & 3u) ||
       ((uintptr_t)w->rowptr & 3u))
     return TQ_ERR_ALIGN;
@@ -77,25 +82,53 @@ Problem to_problem(const tq_weight *w, const uint16_t *x, void *y) {
 
 size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
 
-// Places every problem's workspace (activation slots, then C/S) and runs the
-// decode kernel.  Returns TQ_ERR_SHAPE when the workspace is too small.
+// Workspace bytes of one problem for a launch over M tokens (M <= 16).
+size_t problem_ws_bytes(int M, int N, int K) {
+  if (M <= 8) {
+    size_t b, cs, y2;
+    mma_workspace_parts(M, N, K, &b, &cs, &y2);
+    return pad256(b) + pad256(cs) + pad256(y2);
+  }
+  return pad256(tc_workspace_bytes(16, K));
+}
+
+// Workspace bytes that cover every chunk of a call over M tokens (chunks of
+// TQ_MAX_SKINNY_M; a remainder of at most 8 tokens takes the M <= 8 path).
+size_t call_ws_bytes(int M, int N, int K) {
+  if (M <= 8) return problem_ws_bytes(M, N, K);
+  const size_t a = problem_ws_bytes(16, N, K), b = problem_ws_bytes(8, N, K);
+  return a > b ? a : b;
+}
+
+// Places every problem's workspace and runs the decode path for bp.M tokens
+// (M <= 8: warp-level MMA kernels; 8 < M <= 16: the tensor-memory kernel).
+// Returns TQ_ERR_SHAPE when the workspace is too small.
 tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
-  const int rows = tc_rows_per_tile();
-  const int mw = bp.M <= 8 ? 8 : 16;  // workspace sizing uses the padded token count
+  const bool small = bp.M <= 8;
+  const int rows = small ? mma_rows_per_tile() : tc_rows_per_tile();
   int tiles = 0;
   size_t off = 0;
   for (int i = 0; i < bp.count; ++i) {
     Problem &P = bp.prob[i];
     P.tile_begin = tiles;
     tiles += (P.N + rows - 1) / rows;
-    const size_t bb = tc_workspace_b_bytes(mw, P.K), tot = tc_workspace_bytes(mw, P.K);
-    if (off + pad256(tot) > ws_bytes) return TQ_ERR_SHAPE;
-    P.wsB = ws + off;
-    P.wsCS = reinterpret_cast<float *>(ws + off + bb);
-    off += pad256(tot);
+    const size_t tot = problem_ws_bytes(bp.M, P.N, P.K);
+    if (off + tot > ws_bytes) return TQ_ERR_SHAPE;
+    if (small) {
+      size_t b, cs, y2;
+      mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
+      P.wsB = ws + off;
+      P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
+      P.wsY2 = reinterpret_cast<float *>(ws + off + pad256(b) + pad256(cs));
+    } else {
+      P.wsB = ws + off;
+      P.wsCS = reinterpret_cast<float *>(ws + off + tc_workspace_b_bytes(16, P.K));
+      P.wsY2 = nullptr;
+    }
+    off += tot;
   }
   bp.total_tiles = tiles;
-  return from_cuda(launch_gemv_tc(bp, s));
+  return from_cuda(small ? launch_gemv_mma(bp, s) : launch_gemv_tc(bp, s));
 }
 
 tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
@@ -105,7 +138,7 @@ tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const
   if (!x || !y || !ws) return TQ_ERR_NULL;
   if (!aligned16(x) || ((uintptr_t)ws & 255u)) return TQ_ERR_ALIGN;
   if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
-  if (ws_bytes < tc_workspace_bytes(M, K)) return TQ_ERR_SHAPE;
+  if (ws_bytes < call_ws_bytes(M, N, K)) return TQ_ERR_SHAPE;
   static BatchParams bp;  // large; filled per call (host-side, not thread-safe across calls)
   // Tokens are processed in chunks of TQ_MAX_SKINNY_M.
   for (int32_t m0 = 0; m0 < M; m0 += TQ_MAX_SKINNY_M) {
@@ -162,17 +195,17 @@ tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *
   return from_cuda(launch_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, s));
 }
 
-size_t tq_workspace_bytes(int32_t M, int32_t K) {
-  if (M < 1 || check_shape(1, K) != TQ_OK) return 0;
-  return pad256(tc_workspace_bytes(M <= 8 ? 8 : 16, K));
+size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K) {
+  if (M < 1 || check_shape(N, K) != TQ_OK) return 0;
+  return call_ws_bytes(M, N, K);
 }
 
 size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_problem *problems) {
   if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH || !problems) return 0;
   size_t tot = 0;
   for (int i = 0; i < count; ++i) {
-    if (check_shape(1, problems[i].w.K) != TQ_OK) return 0;
-    tot += pad256(tc_workspace_bytes(M <= 8 ? 8 : 16, problems[i].w.K));
+    if (check_shape(problems[i].w.N, problems[i].w.K) != TQ_OK) return 0;
+    tot += problem_ws_bytes(M, problems[i].w.N, problems[i].w.K);
   }
   return tot;
 }
@@ -210,9 +243,10 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {
   if (!status_host) return TQ_ERR_NULL;
-  uint32_t a = 0;
+  uint32_t a = 0, b = 0;
   if (read_status_gemv_tc(&a, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
-  *status_host = a;
+  if (read_status_gemv_mma(&b, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  *status_host = a | b;
   return TQ_OK;
 }
 
@@ -221,7 +255,7 @@ const char *tq_status_str(tq_status s) {
     case TQ_OK: return "TQ_OK";
     case TQ_ERR_NULL: return "TQ_ERR_NULL: a required pointer is NULL";
     case TQ_ERR_SHAPE: return "TQ_ERR_SHAPE: M, N or K out of range, or K not a multiple of 128";
-    case TQ_ERR_ALIGN: return "TQ_ERR_ALIGN: a pointer is not aligned (plane1 and x need 16 bytes)";
+    case TQ_ERR_ALIGN: return "TQ_ERR_ALIGN: a pointer is not aligned (plane1, plane2 and x need 16 bytes)";
     case TQ_ERR_CODE: return "TQ_ERR_CODE: invalid trit code";
     case TQ_ERR_BYTE: return "TQ_ERR_BYTE: invalid packed byte";
     case TQ_ERR_SALIENCE: return "TQ_ERR_SALIENCE: nnz inconsistent with the salience map";

@@ -1,0 +1,712 @@
+// tq_gemv_mma.cu - decode-path linear for M <= 8 tokens: packed bytes are
+// streamed from HBM into shared memory by bulk copies, decoded in registers
+// and contracted on the tensor cores with warp-level m16n8k16 MMAs (fp16
+// operands, fp32 accumulators).
+//
+// What is computed (per-group reading of the paper's eq. W-hat, "Model and
+// Representation"; packed execution as in "Direct Packed Execution"):
+//   y[m][n] = sum_g ( s1[n,g] * P1[n,g,m] + off[n,g] * S[g,m]
+//                   + sal[n,g] * s2[j(n,g)] * P2[n,g,m] )
+//   P1 = sum_{k in g} T1[n,k] x[m,k],  P2 likewise with T2,  S = sum_{k in g} x[m,k].
+//
+// Operand encoding (five MMA slots per packed byte, the minimum: the five
+// digits d0..d4 of a byte, digit = trit + 1, are five independent linear
+// functions of the byte value v = sum_i d_i 3^i).  A lane-replicated table
+// maps v to the fp16x2 word
+//   W  = (4 + d0 + d2/4, 4 + d1 + d3/4)
+// and one LOP3 gives W' = (16 + d2, 16 + d3).  The fifth slot is the byte
+// value itself, 4 + v/256, read straight off the table address (two bytes
+// share one PRMT).  With z_i = x_i - 3^i x4 / 81 the activation slots
+//   y_a = z0, y_b = z1, y_c = z2 - z0/4, y_d = z3 - z1/4, y_e = 256 x4 / 81
+// make the MMA return  const + sum_i d_i x_i  (exact up to the rounding of
+// the slots to fp16); subtracting C, the same MMA for all digits 1 (all
+// trits 0), leaves sum_i t_i x_i.  Slots, C and S per (group, token) come
+// from gemv_mma_prep_kernel into the caller's workspace.
+//
+// Fragment layout.  In an m16n8k16 MMA, lane (g, c) (g = lane / 4,
+// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  Here
+// lane c of a row decodes the bytes in byte position c of the 7 words of
+// the group's window (the aligned words covering the group's 26 bytes,
+// starting 0 or 2 bytes before it); its 18 A words per group are
+// W, W' of each of its 7 bytes and 4 V words, in that order, and chunk j
+// of the group's 9 MMAs takes words 2j and 2j + 1.  Bytes of a window that
+// do not belong to the group get zero activations, so every lane runs the
+// same code.  The prep kernel writes B (the activation slots) in exactly
+// this order, per group parity.
+//
+// Kernels (one step = three launches):
+//  * gemv_mma_prep_kernel: B fragments, C and S per (problem, group, token);
+//  * gemv_mma_p2_kernel: the second plane.  One CTA per 128-row tile
+//    compacts the tile's salient (row, group) pairs per group, decodes their
+//    records with the same encoding and runs m16n8k16 MMAs over 16 records
+//    at a time; s2 * P2 per row goes to the workspace (y2, fp32);
+//  * gemv_mma_kernel (one persistent CTA per SM over a cost-balanced range
+//    of 128-row tiles, 8-group stages): warp 8 stages each stage's packed
+//    rows, B fragments, C/S and s1/off into a ring of shared-memory slots;
+//    warps 0..7 each own 16 rows, decode and multiply, apply s1 / off per
+//    group, and at the tile's end add y2 and write y.
+// Every wait is bounded (tq_sm100.cuh); a timeout raises a CTA-wide abort.
+#include "tq_common.cuh"
+#include "tq_sm100.cuh"
+
+namespace tq {
+namespace mm {
+
+constexpr int kRows = 128;        // tile rows (8 m16 tiles)
+constexpr int kStageG = 8;        // groups per stage
+constexpr int kStageBytes = 208;  // plane-1 bytes per row per stage (13 x 16)
+constexpr int kChunks = 9;        // k16 chunks per group (144 K slots)
+constexpr int kCP = 5;            // chunk pairs (the fifth: chunk 8 and zeros)
+constexpr int kBLane = 16;        // B bytes per (chunk pair, token, lane position)
+constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
+constexpr int kCSGroup = 64;             // C[8], S[8] floats per group
+constexpr int kWarpsP1 = 8, kWarpProd = 8;
+constexpr int kThreads = 9 * 32;
+constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
+constexpr uint32_t kLutShared = 65536;  // shared-window address of the table
+constexpr uint32_t kDynShared = 1024;   // shared-window offset of dynamic smem
+constexpr int kDynBytes = 232448;       // whole opt-in shared memory of a CTA
+constexpr int kArena1 = (int)(kLutShared - kDynShared);   // below the table
+constexpr int kArena2 = kDynBytes - kArena1 - kLutBytes;  // above the table
+constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
+constexpr int kSOSlot = 2 * kRows * 16;                   // s1 then off, 16 B per row
+constexpr int kCSSlot = kStageG * kCSGroup;               // 512
+constexpr int kBarOff = 2 * kBytesSlot;                   // barriers in arena 1
+// The table address PRMT: byte 0 = lane * 4, byte 1 = the packed byte,
+// byte 2 = 0x44 (the fp16 exponent of the fifth slot), byte 3 = 0.  The
+// 0x44 is removed again by the load's immediate offset.
+constexpr uint32_t kLaneTag = 0x00440000u;
+constexpr int kLutImm = (int)kLutShared - (int)kLaneTag;
+
+__host__ __device__ constexpr int num_slots(int MB) { return MB <= 2 ? 4 : 3; }
+__host__ __device__ constexpr int b_stage_bytes(int MB) { return kStageG * kBTok * MB; }
+
+// Stage-slot layout for MB tokens: plane-1 slots 0, 1 in arena 1, the rest
+// in arena 2 followed by the B, s1/off and C/S slots.
+struct Layout {
+  int NS, BStage;
+  int oBytes2, oB, oSO, oCS, used2;
+  __host__ __device__ explicit Layout(int MB) {
+    NS = num_slots(MB);
+    BStage = b_stage_bytes(MB);
+    oBytes2 = 0;
+    oB = oBytes2 + (NS - 2) * kBytesSlot;
+    oSO = oB + NS * BStage;
+    oCS = oSO + NS * kSOSlot;
+    used2 = oCS + NS * kCSSlot;
+  }
+};
+
+struct Bars {
+  uint64_t full[4], empty[4];
+  int32_t abort_;
+};
+
+// Schedule: CTA c processes global tiles [cta_tile[c], cta_tile[c+1]).
+struct Sched {
+  int32_t cta_tile[257];
+};
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, volatile int32_t *abort_) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0) {
+      if (*abort_) return false;
+      if (global_ns() - t0 > kWaitLimitNs) break;
+    }
+  }
+  atomicOr(&g_tq_device_status, kStatusTimeout);
+  *abort_ = 1;
+  return false;
+}
+
+// Table word of a byte value (see the file comment); invalid bytes
+// (243..255) map to the exponent pattern alone.
+__host__ __device__ __forceinline__ uint32_t lut_word(int v) {
+  uint32_t w = 0x44004400u;
+  if (v <= 242) {
+    const uint32_t d0 = v % 3, d1 = (v / 3) % 3, d2 = (v / 9) % 3, d3 = (v / 27) % 3;
+    w |= (d0 << 8) | (d2 << 6) | (d1 << 24) | (d3 << 22);
+  }
+  return w;
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t s) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(s));
+  return d;
+}
+__device__ __forceinline__ uint32_t lut_load(uint32_t tagged_addr) {
+  uint32_t w;
+  asm volatile("ld.shared.u32 %0, [%1+%2];" : "=r"(w) : "r"(tagged_addr), "n"(kLutImm) : "memory");
+  return w;
+}
+__device__ __forceinline__ uint32_t w_prime(uint32_t w) {
+  uint32_t d;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(d) : "r"(w), "n"(0x00C000C0), "n"(0x4C004C00));
+  return d;
+}
+
+// The 18 A words of one row and group from the 7 window words (lane-replicated
+// table; `tag` = kLaneTag | lane * 4, `sel` = 0x7604 | c << 4).
+__device__ __forceinline__ void decode_window(const uint32_t *win, uint32_t tag, uint32_t sel, uint32_t *a) {
+  uint32_t r[7];
+#pragma unroll
+  for (int i = 0; i < 7; ++i) r[i] = prmt(win[i], tag, sel);
+#pragma unroll
+  for (int i = 0; i < 7; ++i) {
+    const uint32_t w = lut_load(r[i]);
+    a[2 * i] = w;
+    a[2 * i + 1] = w_prime(w);
+  }
+  a[14] = prmt(r[0], r[1], 0x6521u);
+  a[15] = prmt(r[2], r[3], 0x6521u);
+  a[16] = prmt(r[4], r[5], 0x6521u);
+  a[17] = prmt(r[6], r[6], 0x6521u);
+}
+
+// The same from a compact (not replicated) 256-word table at `lut`.
+__device__ __forceinline__ void decode_window_compact(const uint32_t *win, const uint32_t *lut, int c,
+                                                      uint32_t *a) {
+  uint32_t v[7];
+#pragma unroll
+  for (int i = 0; i < 7; ++i) v[i] = (win[i] >> (8 * c)) & 0xffu;
+#pragma unroll
+  for (int i = 0; i < 7; ++i) {
+    const uint32_t w = lut[v[i]];
+    a[2 * i] = w;
+    a[2 * i + 1] = w_prime(w);
+  }
+  a[14] = 0x44004400u | v[0] | (v[1] << 16);
+  a[15] = 0x44004400u | v[2] | (v[3] << 16);
+  a[16] = 0x44004400u | v[4] | (v[5] << 16);
+  a[17] = 0x44004400u | v[6] | (v[6] << 16);
+}
+
+// D += A * B, m16n8k16, fp16 in, fp32 accumulate.
+__device__ __forceinline__ void mma16816(float *d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// The 9 MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
+// (b[2j], b[2j+1] for chunk j).  Two accumulation chains, summed into d.
+__device__ __forceinline__ void group_mma(const uint32_t *aL, const uint32_t *aH, const uint32_t *b, float *d) {
+  float e[4] = {0.f, 0.f, 0.f, 0.f}, o[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < kChunks; ++j) {
+    float *acc = (j & 1) ? o : e;
+    mma16816(acc, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) d[i] = e[i] + o[i];
+}
+
+// Iterates (tile, stage) in the CTA's order.
+struct Walk {
+  int tile, t_end, pi, s, nstages, gs;
+  const BatchParams *bp;
+  __device__ void set_tile() {
+    while (pi + 1 < bp->count && bp->prob[pi + 1].tile_begin <= tile) ++pi;
+    const int G = bp->prob[pi].K / kGroup;
+    nstages = (G + kStageG - 1) / kStageG;
+    s = 0;
+    gs = min(kStageG, G);
+  }
+  __device__ Walk(const BatchParams *b, int t0, int t1)
+      : tile(t0), t_end(t1), pi(0), s(0), nstages(0), gs(0), bp(b) {
+    if (tile < t_end) set_tile();
+  }
+  __device__ bool valid() const { return tile < t_end; }
+  __device__ const Problem &P() const { return bp->prob[pi]; }
+  __device__ bool last_stage() const { return s + 1 == nstages; }
+  __device__ void next() {
+    if (++s < nstages) {
+      const int G = bp->prob[pi].K / kGroup;
+      gs = min(kStageG, G - s * kStageG);
+    } else if (++tile < t_end) {
+      set_tile();
+    }
+  }
+};
+
+// ------------------------------------------------------------------ prep
+// B fragments, C and S for every (problem, group, token).  B layout of a
+// group: [chunk pair cp][token m][lane position c] x 16 B, each 16 B being
+// (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
+__global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp) {
+  const int p = blockIdx.y;
+  if (p >= bp.count) return;
+  const Problem &P = bp.prob[p];
+  const int MB = bp.M;
+  const int G = P.K / kGroup;
+  const int task = blockIdx.x * blockDim.x + threadIdx.x;
+  if (task >= G * MB) return;
+  const int g = task / MB, m = task % MB;
+  const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
+  // activation slots of the 26 bytes, rounded to fp16
+  __half ya[26], yb[26], yc[26], yd[26], ye[26];
+  float C = 0.f, S = 0.f;
+  for (int b = 0; b < 26; ++b) {
+    const int ntr = b < 25 ? 5 : 3;
+    float x[5];
+#pragma unroll
+    for (int i = 0; i < 5; ++i) x[i] = i < ntr ? __half2float(xr[5 * b + i]) : 0.f;
+    const float z0 = x[0] - x[4] * (1.f / 81.f), z1 = x[1] - x[4] * (3.f / 81.f);
+    const float z2 = x[2] - x[4] * (9.f / 81.f), z3 = x[3] - x[4] * (27.f / 81.f);
+    ya[b] = __float2half_rn(z0);
+    yb[b] = __float2half_rn(z1);
+    const float fa = __half2float(ya[b]), fb = __half2float(yb[b]);
+    yc[b] = __float2half_rn(z2 - 0.25f * fa);
+    yd[b] = __float2half_rn(z3 - 0.25f * fb);
+    ye[b] = __float2half_rn(x[4] * (256.f / 81.f));
+    // all digits 1: slots 4 + 1 + 1/4, 16 + 1, 4 + 121/256
+    C += 5.25f * (fa + fb) + 17.f * (__half2float(yc[b]) + __half2float(yd[b])) +
+         (4.f + 121.f / 256.f) * __half2float(ye[b]);
+    S += x[0] + x[1] + x[2] + x[3] + x[4];
+  }
+  const int o = (g & 1) ? 2 : 0;  // window offset: stage-relative parity of the group
+  unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
+  const __half z = __float2half_rn(0.f);
+  for (int c = 0; c < 4; ++c) {
+    // byte of window word jw in lane position c, or -1 if not in the group
+    auto byte_of = [&](int jw) -> int {
+      const int b = 4 * jw + c - o;
+      return (b >= 0 && b < 26) ? b : -1;
+    };
+    uint32_t words[20];
+    for (int j = 0; j < 7; ++j) {
+      const int b = byte_of(j);
+      __half2 w0 = __halves2half2(z, z), w1 = __halves2half2(z, z);
+      if (b >= 0) {
+        w0 = __halves2half2(ya[b], yb[b]);
+        w1 = __halves2half2(yc[b], yd[b]);
+      }
+      words[2 * j] = *reinterpret_cast<uint32_t *>(&w0);
+      words[2 * j + 1] = *reinterpret_cast<uint32_t *>(&w1);
+    }
+    for (int k = 0; k < 4; ++k) {
+      const int b0 = byte_of(2 * k), b1 = k < 3 ? byte_of(2 * k + 1) : -1;
+      __half2 v = __halves2half2(b0 >= 0 ? ye[b0] : z, b1 >= 0 ? ye[b1] : z);
+      words[14 + k] = *reinterpret_cast<uint32_t *>(&v);
+    }
+    words[18] = 0u;
+    words[19] = 0u;
+    for (int cp = 0; cp < kCP; ++cp) {
+      uint4 q = make_uint4(words[4 * cp], words[4 * cp + 1], words[4 * cp + 2], words[4 * cp + 3]);
+      *reinterpret_cast<uint4 *>(Bg + ((cp * MB + m) * 4 + c) * kBLane) = q;
+    }
+  }
+  float *cs = P.wsCS + (int64_t)g * (kCSGroup / 4);
+  cs[m] = C;
+  cs[8 + m] = S;
+  if (m == 0)
+    for (int mm = MB; mm < 8; ++mm) cs[mm] = cs[8 + mm] = 0.f;
+}
+
+// ------------------------------------------------------------ plane 2
+// One CTA (4 warps) per 128-row tile of one problem.  Thread t = row t
+// compacts the tile's salient pairs of each 32-group salience word into
+// per-group lists; each warp then takes 16-record items of one group.
+constexpr int kP2Threads = 128;
+__global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_constant__ BatchParams bp) {
+  const int p = blockIdx.y;
+  if (p >= bp.count) return;
+  const Problem &P = bp.prob[p];
+  const int n0 = blockIdx.x * kRows;
+  if (n0 >= P.N) return;
+  const int MB = bp.M;
+  __shared__ uint32_t lut[256];
+  __shared__ int2 list[32][kRows];  // (row, record index)
+  __shared__ int cnt[4][32], base[4][32], tot[32];
+  __shared__ float acc[kRows][8];
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  for (int i = t; i < 256; i += kP2Threads) lut[i] = lut_word(i);
+  for (int i = t; i < kRows * 8; i += kP2Threads) (&acc[0][0])[i] = 0.f;
+  const int n = n0 + t;
+  const bool valid = n < P.N;
+  const int G = P.K / kGroup, W = sal_words_of(P.K);
+  int j = (valid && P.nnz > 0) ? P.rowptr[n] : 0;
+  const uint32_t lt = (1u << lane) - 1u;
+  const int gq = lane >> 2, c = lane & 3;
+  __syncthreads();
+  for (int w = 0; w < W && P.nnz > 0; ++w) {
+    const int gbase = 32 * w, gw = min(32, G - gbase);
+    uint32_t bits = valid ? P.sal[(int64_t)n * W + w] : 0u;
+    if (gw < 32) bits &= (1u << gw) - 1u;
+    for (int gl = 0; gl < 32; ++gl) {
+      const uint32_t m = __ballot_sync(0xffffffffu, (bits >> gl) & 1u);
+      if (lane == 0) cnt[warp][gl] = __popc(m);
+    }
+    __syncthreads();
+    if (t < 32) {
+      int s = 0;
+      for (int ww = 0; ww < 4; ++ww) {
+        base[ww][t] = s;
+        s += cnt[ww][t];
+      }
+      tot[t] = s;
+    }
+    __syncthreads();
+    for (int gl = 0; gl < 32; ++gl) {
+      const uint32_t m = __ballot_sync(0xffffffffu, (bits >> gl) & 1u);
+      if ((bits >> gl) & 1u)
+        list[gl][base[warp][gl] + __popc(m & lt)] = make_int2(t, j + __popc(bits & ((1u << gl) - 1u)));
+    }
+    j += __popc(bits);
+    __syncthreads();
+    // items: (group, first record) in order; item k goes to warp k % 4
+    int k = 0;
+    for (int gl = 0; gl < gw; ++gl) {
+      const int tg = tot[gl];
+      for (int e0 = 0; e0 < tg; e0 += 16, ++k) {
+        if ((k & 3) != warp) continue;
+        const int g = gbase + gl;
+        const int o = (g & 1) ? 2 : 0;
+        uint32_t aL[18], aH[18];
+        int rows[2] = {-1, -1};
+        float s2v[2] = {0.f, 0.f};
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int e = e0 + gq + 8 * h;
+          uint32_t win[7];
+#pragma unroll
+          for (int i = 0; i < 7; ++i) win[i] = 0u;
+          if (e < tg) {
+            const int2 rec = list[gl][e];
+            rows[h] = rec.x;
+            const int64_t jj = min(max((int64_t)rec.y, (int64_t)0), (int64_t)P.nnz - 1);
+            s2v[h] = __half2float(P.s2[jj]);
+            // 7 aligned words covering the record (plane 2 is 16-byte aligned,
+            // so the record starts 0 or 2 bytes into a word)
+            const uint8_t *A = P.plane2 + jj * kGroupBytes;
+            const int sh = (int)(jj & 1) * 2;
+            const uint32_t *src = reinterpret_cast<const uint32_t *>(A - sh);
+            uint32_t wv[8];
+#pragma unroll
+            for (int i = 0; i < 6; ++i) wv[i] = __ldg(src + i);
+            wv[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
+            wv[7] = 0u;
+            if (sh == o) {
+#pragma unroll
+              for (int i = 0; i < 7; ++i) win[i] = wv[i];
+            } else if (o == 2) {  // record 4-aligned, window starts 2 bytes before it
+#pragma unroll
+              for (int i = 0; i < 7; ++i) win[i] = __funnelshift_l(i ? wv[i - 1] : 0u, wv[i], 16);
+            } else {  // record starts 2 bytes into a word, window at the record
+#pragma unroll
+              for (int i = 0; i < 7; ++i) win[i] = __funnelshift_r(wv[i], wv[i + 1], 16);
+            }
+          }
+          decode_window_compact(win, lut, c, h ? aH : aL);
+        }
+        uint32_t b[20];
+        const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
+#pragma unroll
+        for (int cp = 0; cp < kCP; ++cp) {
+          uint4 q = make_uint4(0u, 0u, 0u, 0u);
+          if (gq < MB) q = __ldg(reinterpret_cast<const uint4 *>(Bg + ((cp * MB + gq) * 4 + c) * kBLane));
+          b[4 * cp] = q.x;
+          b[4 * cp + 1] = q.y;
+          b[4 * cp + 2] = q.z;
+          b[4 * cp + 3] = q.w;
+        }
+        float d[4];
+        group_mma(aL, aH, b, d);
+        const float *cs = P.wsCS + (int64_t)g * (kCSGroup / 4);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (rows[h] < 0) continue;
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            const int m = 2 * c + i;
+            if (m < MB) atomicAdd(&acc[rows[h]][m], s2v[h] * (d[2 * h + i] - __ldg(cs + m)));
+          }
+        }
+      }
+    }
+    __syncthreads();
+  }
+  if (valid) {
+    float *y2 = P.wsY2 + (int64_t)n * MB;
+    for (int m = 0; m < MB; ++m) y2[m] = acc[t][m];
+  }
+}
+
+// ------------------------------------------------------------------ main
+template <bool F32>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemv_mma_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
+  extern __shared__ __align__(1024) unsigned char dyn[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int M = bp.M, MB = bp.M;
+  if (smem_u32(dyn) != kDynShared) {
+    // the table address trick needs the dynamic window right after the
+    // reserved 1 KiB of shared memory; anything else is reported
+    if (tid == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  const Layout L(MB);
+  const int NS = L.NS;
+  unsigned char *ar1 = dyn, *ar2 = dyn + kArena1 + kLutBytes;
+  auto bytes_buf = [&](int b) -> unsigned char * {
+    return b < 2 ? ar1 + b * kBytesSlot : ar2 + L.oBytes2 + (b - 2) * kBytesSlot;
+  };
+  Bars *bars = reinterpret_cast<Bars *>(ar1 + kBarOff);
+  volatile int32_t *abort_ = &bars->abort_;
+
+  // ---- one-time set-up: the lane-replicated table, barriers
+  {
+    uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
+    for (int i = tid; i < 256 * 32; i += kThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+  }
+  if (tid == 0) {
+    for (int i = 0; i < NS; ++i) {
+      mbar_init(&bars->full[i], 1 + 32);  // producer's expect-tx arrival + one per producer lane
+      mbar_init(&bars->empty[i], kWarpsP1);
+    }
+    bars->abort_ = 0;
+    mbar_fence_init();
+  }
+  __syncthreads();
+  const int t_begin = sc.cta_tile[blockIdx.x], t_end = sc.cta_tile[blockIdx.x + 1];
+
+  if (warp < kWarpsP1) {
+    // ============================================================ decode
+    const int g = lane >> 2, c = lane & 3;
+    const int R0 = warp * 16 + g, R1 = R0 + 8;
+    const uint32_t tag = kLaneTag | ((uint32_t)lane << 2);
+    const uint32_t sel = 0x7604u | ((uint32_t)c << 4);
+    float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
+    uint32_t q = 0;
+    for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
+      const int buf = (int)(q % (uint32_t)NS);
+      const bool ok = wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      const unsigned char *rp0 = bytes_buf(buf) + R0 * kStageBytes;
+      const unsigned char *rp1 = bytes_buf(buf) + R1 * kStageBytes;
+      const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
+      const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * kCSSlot);
+      const unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
+      const uint4 s1a = *reinterpret_cast<const uint4 *>(SO + R0 * 16);
+      const uint4 s1b = *reinterpret_cast<const uint4 *>(SO + R1 * 16);
+      const uint4 ofa = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R0 * 16);
+      const uint4 ofb = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R1 * 16);
+      const uint32_t s1w[2][4] = {{s1a.x, s1a.y, s1a.z, s1a.w}, {s1b.x, s1b.y, s1b.z, s1b.w}};
+      const uint32_t ofw[2][4] = {{ofa.x, ofa.y, ofa.z, ofa.w}, {ofb.x, ofb.y, ofb.z, ofb.w}};
+      const int gs = w.gs;
+#pragma unroll
+      for (int GL = 0; GL < kStageG; ++GL) {
+        if (GL < gs) {
+          // window words of this group in rows R0 / R1
+          const int c0 = (26 * GL) / 16, c1 = (26 * GL + 25) / 16;
+          const int wstart = (26 * GL) / 4 - 4 * c0;
+          uint32_t u0[12], u1[12];
+#pragma unroll
+          for (int cc = 0; cc < 3; ++cc) {
+            if (c0 + cc <= c1) {
+              const uint4 v0 = *reinterpret_cast<const uint4 *>(rp0 + 16 * (c0 + cc));
+              const uint4 v1 = *reinterpret_cast<const uint4 *>(rp1 + 16 * (c0 + cc));
+              u0[4 * cc] = v0.x; u0[4 * cc + 1] = v0.y; u0[4 * cc + 2] = v0.z; u0[4 * cc + 3] = v0.w;
+              u1[4 * cc] = v1.x; u1[4 * cc + 1] = v1.y; u1[4 * cc + 2] = v1.z; u1[4 * cc + 3] = v1.w;
+            }
+          }
+          uint32_t aL[18], aH[18];
+          decode_window(u0 + wstart, tag, sel, aL);
+          decode_window(u1 + wstart, tag, sel, aH);
+          uint32_t b[20];
+#pragma unroll
+          for (int cp = 0; cp < kCP; ++cp) {
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (g < MB) v = *reinterpret_cast<const uint4 *>(Bst + GL * kBTok * MB + ((cp * MB + g) * 4 + c) * kBLane);
+            b[4 * cp] = v.x;
+            b[4 * cp + 1] = v.y;
+            b[4 * cp + 2] = v.z;
+            b[4 * cp + 3] = v.w;
+          }
+          float d[4];
+          group_mma(aL, aH, b, d);
+          const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
+          const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
+            const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
+            const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+            y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
+            y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->empty[buf]);
+      if (w.last_stage()) {
+        const Problem &P = w.P();
+        const int nb = (w.tile - P.tile_begin) * kRows;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int n = nb + (h ? R1 : R0);
+          if (n < P.N) {
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+              const int m = 2 * c + i;
+              if (m < M) {
+                float v = y[2 * h + i];
+                if (P.nnz > 0) v += P.wsY2[(int64_t)n * MB + m];
+                if (F32)
+                  static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
+                else
+                  static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
+              }
+            }
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) y[i] = 0.f;
+      }
+    }
+  } else if (warp == kWarpProd) {
+    // ========================================================== producer
+    uint32_t q = 0;
+    for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
+      const Problem &P = w.P();
+      const int G = P.K / kGroup;
+      const int64_t RB = row_bytes_of(P.K);
+      const int n0 = (w.tile - P.tile_begin) * kRows;
+      const int rows = min(kRows, P.N - n0);
+      const int s = w.s, gs = w.gs, g0 = s * kStageG;
+      const uint32_t rb = (uint32_t)((gs * kGroupBytes + 15) / 16 * 16);
+      const uint32_t bb = (uint32_t)(gs * kBTok * MB);
+      const uint32_t cb = (uint32_t)(gs * kCSGroup);
+      const int buf = (int)(q % (uint32_t)NS);
+      int ok = 1;
+      if (lane == 0) ok = wait_or_abort(&bars->empty[buf], ((q / NS) & 1u) ^ 1u, abort_) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
+      unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars->full[buf], rb * (uint32_t)rows + bb + cb);
+        bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, &bars->full[buf]);
+        bulk_g2s(ar2 + L.oCS + buf * kCSSlot, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * kCSGroup,
+                 cb, &bars->full[buf]);
+      }
+      __syncwarp();
+      for (int rr = lane; rr < rows; rr += 32)
+        bulk_g2s(bytes_buf(buf) + rr * kStageBytes, P.plane1 + (int64_t)(n0 + rr) * RB + (int64_t)s * kStageBytes, rb,
+                 &bars->full[buf]);
+      // s1 / off of the stage: 8 halves per row
+      const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+      if (vec) {
+        for (int rr = lane; rr < rows; rr += 32) {
+          const int64_t o = ((int64_t)(n0 + rr) * G + g0) * 2;
+          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(SO + rr * 16)),
+                       "l"(reinterpret_cast<const unsigned char *>(P.s1) + o)
+                       : "memory");
+          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(SO + kRows * 16 + rr * 16)),
+                       "l"(reinterpret_cast<const unsigned char *>(P.off) + o)
+                       : "memory");
+        }
+        asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&bars->full[buf]))
+                     : "memory");
+      } else {
+        for (int rr = lane; rr < rows; rr += 32) {
+          __half *d1 = reinterpret_cast<__half *>(SO + rr * 16);
+          __half *d2 = reinterpret_cast<__half *>(SO + kRows * 16 + rr * 16);
+          const int64_t o = (int64_t)(n0 + rr) * G + g0;
+          for (int gg = 0; gg < kStageG; ++gg) {
+            d1[gg] = gg < gs ? P.s1[o + gg] : __float2half_rn(0.f);
+            d2[gg] = gg < gs ? P.off[o + gg] : __float2half_rn(0.f);
+          }
+        }
+        mbar_arrive(&bars->full[buf]);
+      }
+    }
+    // drain: every issued copy lands before the CTA exits (waited on even
+    // after an abort; bounded by the wall-time limit)
+    if (lane == 0) {
+      for (uint32_t k = (q > (uint32_t)NS ? q - NS : 0); k < q; ++k) mbar_wait(&bars->full[k % NS], (k / NS) & 1u);
+    }
+  }
+  __syncthreads();
+}
+
+}  // namespace mm
+
+// -------------------------------------------------------------- launcher
+static int num_sms_mm() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+int mma_rows_per_tile() { return mm::kRows; }
+
+// Workspace bytes of one problem for M <= 8 tokens: B fragments, C/S, y2.
+void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2) {
+  const size_t G = (size_t)(K / kGroup);
+  *b = G * (size_t)mm::kBTok * (size_t)M;
+  *cs = G * (size_t)mm::kCSGroup;
+  *y2 = (size_t)N * (size_t)M * 4;
+}
+
+TQ_STATUS_ACCESSOR(read_status_gemv_mma)
+
+template <bool F32>
+static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
+  static mm::Sched sc;
+  if (bp.M < 1 || bp.M > 8 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
+  const int ctas = min(num_sms_mm(), 256);
+  int64_t total_cost = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    const int tiles_i = (bp.prob[i].N + mm::kRows - 1) / mm::kRows;
+    total_cost += (int64_t)tiles_i * (bp.prob[i].K / kGroup);
+  }
+  int c = 0, tile = 0;
+  int64_t run = 0;
+  sc.cta_tile[0] = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    const int tiles_i = (bp.prob[i].N + mm::kRows - 1) / mm::kRows;
+    const int64_t cost = bp.prob[i].K / kGroup;
+    for (int t = 0; t < tiles_i; ++t, ++tile) {
+      const int64_t mid2 = 2 * run + cost;
+      while (c < ctas - 1 && mid2 * ctas >= 2 * total_cost * (int64_t)(c + 1)) sc.cta_tile[++c] = tile;
+      run += cost;
+    }
+  }
+  while (c < ctas) sc.cta_tile[++c] = tile;
+  int gmax = 0, tmax = 0;
+  bool any2 = false;
+  for (int i = 0; i < bp.count; ++i) {
+    gmax = max(gmax, bp.prob[i].K / kGroup);
+    tmax = max(tmax, (bp.prob[i].N + mm::kRows - 1) / mm::kRows);
+    any2 = any2 || bp.prob[i].nnz > 0;
+  }
+  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (any2) {
+    mm::gemv_mma_p2_kernel<<<dim3(tmax, bp.count), mm::kP2Threads, 0, s>>>(bp);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  e = cudaFuncSetAttribute(mm::gemv_mma_kernel<F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kDynBytes);
+  if (e != cudaSuccess) return e;
+  mm::gemv_mma_kernel<F32><<<ctas, mm::kThreads, mm::kDynBytes, s>>>(bp, sc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv_mma(const BatchParams &bp, cudaStream_t s) {
+  return bp.out_f32 ? launch_mm<true>(bp, s) : launch_mm<false>(bp, s);
+}
+
+}  // namespace tq

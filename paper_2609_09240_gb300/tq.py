@@ -72,7 +72,7 @@ def lib():
             L.tq_unpack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             sz = ctypes.c_size_t
             L.tq_workspace_bytes.restype = sz
-            L.tq_workspace_bytes.argtypes = [i32, i32]
+            L.tq_workspace_bytes.argtypes = [i32, i32, i32]
             L.tq_batched_workspace_bytes.restype = sz
             L.tq_batched_workspace_bytes.argtypes = [i32, i32, ctypes.POINTER(tq_problem)]
             L.tq_linear.restype = ctypes.c_int
@@ -203,8 +203,8 @@ def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True) -> PackedWeig
     return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz)
 
 
-def tq_workspace_bytes(M: int, K: int) -> int:
-    return int(lib().tq_workspace_bytes(M, K))
+def tq_workspace_bytes(M: int, N: int, K: int) -> int:
+    return int(lib().tq_workspace_bytes(M, N, K))
 
 
 def workspace(nbytes: int, device) -> torch.Tensor:
@@ -221,7 +221,7 @@ def tq_linear(x, w: PackedWeight, y=None, ws=None, stream=None):
     if y is None:
         y = torch.empty((M, w.N), dtype=torch.float16, device=x.device)
     if ws is None:
-        ws = workspace(tq_workspace_bytes(M, K), x.device)
+        ws = workspace(tq_workspace_bytes(M, w.N, K), x.device)
     ws_ = w.struct()
     _check(lib().tq_linear(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _p(ws), ws.numel(), _stream(stream)),
            "tq_linear")
@@ -234,7 +234,7 @@ def tq_linear_f32out(x, w: PackedWeight, y=None, ws=None, stream=None):
     if y is None:
         y = torch.empty((M, w.N), dtype=torch.float32, device=x.device)
     if ws is None:
-        ws = workspace(tq_workspace_bytes(M, K), x.device)
+        ws = workspace(tq_workspace_bytes(M, w.N, K), x.device)
     ws_ = w.struct()
     _check(lib().tq_linear_f32out(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _p(ws), ws.numel(),
                                   _stream(stream)), "tq_linear_f32out")

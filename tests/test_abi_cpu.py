@@ -47,6 +47,15 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_linear(1, 4, 128, None, None, None, None, 0, None) == -1
     assert L.tq_linear_batched(17, 1, None, None, 0, None) == -2
     assert L.tq_linear_batched(1, 0, None, None, 0, None) == -2
-    assert tq.tq_workspace_bytes(1, 4096) == 32 * (2560 + 64)
-    assert tq.tq_workspace_bytes(16, 4096) == 32 * (5120 + 128)
-    assert tq.tq_workspace_bytes(1, 100) == 0
+    # M <= 8: activation fragments (320 B per group and token), C/S (64 B per
+    # group), second-plane partials (4 B per row and token), each 256-padded
+    pad = lambda b: (b + 255) // 256 * 256
+    mma = lambda M, N, K: pad(K // 128 * 320 * M) + pad(K // 128 * 64) + pad(N * M * 4)
+    assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) == 28672
+    assert tq.tq_workspace_bytes(5, 100, 1024) == mma(5, 100, 1024)
+    # 8 < M <= 16: tensor-memory path (2 x 2560 B of slots + 128 B C/S per group);
+    # larger M runs in chunks of 16 and may end on a chunk of <= 8 tokens
+    assert tq.tq_workspace_bytes(16, 4096, 4096) == max(32 * (5120 + 128), mma(8, 4096, 4096))
+    assert tq.tq_workspace_bytes(40, 64, 4096) == max(32 * (5120 + 128), mma(8, 64, 4096))
+    assert tq.tq_workspace_bytes(1, 4096, 100) == 0
+    assert tq.tq_workspace_bytes(1, 0, 4096) == 0

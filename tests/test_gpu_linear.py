@@ -88,7 +88,7 @@ def test_argument_errors(H):
     pw = H.pack_on_gpu(w)
     x = torch.zeros((1, 256), dtype=torch.float16, device="cuda")
     y = torch.empty((1, 64), dtype=torch.float16, device="cuda")
-    ws = tq.workspace(tq.tq_workspace_bytes(1, 256), "cuda")
+    ws = tq.workspace(tq.tq_workspace_bytes(1, 64, 256), "cuda")
     L = tq.lib()
     s = tq._stream(None)
     ws_ = pw.struct()
