@@ -24,15 +24,15 @@
 // from gemv_mma_prep_kernel into the caller's workspace.
 //
 // Fragment layout.  In an m16n8k16 MMA, lane (g, c) (g = lane / 4,
-// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  Here
-// lane c of a row decodes the bytes in byte position c of the 7 words of
-// the group's window (the aligned words covering the group's 26 bytes,
-// starting 0 or 2 bytes before it); its 18 A words per group are
-// W, W' of each of its 7 bytes and 4 V words, in that order, and chunk j
-// of the group's 9 MMAs takes words 2j and 2j + 1.  Bytes of a window that
-// do not belong to the group get zero activations, so every lane runs the
-// same code.  The prep kernel writes B (the activation slots) in exactly
-// this order, per group parity.
+// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  The
+// packed rows reach the registers by ldmatrix, which gives lane c word c of
+// every 16-byte chunk; so lane c of a row decodes two whole words of the
+// group's window (the aligned words covering its 26 bytes): 8 bytes, whose
+// 20 A words (W, W' of each byte, then 4 V words) feed the group's 10 MMAs,
+// chunk j taking words 2j and 2j + 1.  Window bytes outside the group get
+// zero activations, so every lane runs the same code.  The prep kernel
+// writes B (the activation slots) in exactly this order for each of the 8
+// positions a group can take in its stage.
 //
 // Kernels (one step = three launches):
 //  * gemv_mma_prep_kernel: B fragments, C and S per (problem, group, token);
@@ -41,11 +41,15 @@
 //    records with the same encoding and runs m16n8k16 MMAs over 16 records
 //    at a time; s2 * P2 per row goes to the workspace (y2, fp32);
 //  * gemv_mma_kernel (one persistent CTA per SM over a cost-balanced range
-//    of 128-row tiles, 8-group stages): warp 8 stages each stage's packed
-//    rows, B fragments, C/S and s1/off into a ring of shared-memory slots;
-//    warps 0..7 each own 16 rows, decode and multiply, apply s1 / off per
-//    group, and at the tile's end add y2 and write y.
+//    of 128-row tiles, 8-group stages): warps 0..7 each own 16 rows of the
+//    tile, fetch those rows' packed bytes and s1 / off with 16-byte
+//    asynchronous copies a few stages ahead into a ring of shared-memory
+//    slots, decode and multiply, apply s1 / off per group, and at the tile's
+//    end add y2 and write y; warp 8 bulk-copies each stage's B fragments and
+//    C/S into the same ring.
 // Every wait is bounded (tq_sm100.cuh); a timeout raises a CTA-wide abort.
+#include <type_traits>
+
 #include "tq_common.cuh"
 #include "tq_sm100.cuh"
 
@@ -55,13 +59,13 @@ namespace mm {
 constexpr int kRows = 128;        // tile rows (8 m16 tiles)
 constexpr int kStageG = 8;        // groups per stage
 constexpr int kStageBytes = 208;  // plane-1 bytes per row per stage (13 x 16)
-constexpr int kChunks = 9;        // k16 chunks per group (144 K slots)
-constexpr int kCP = 5;            // chunk pairs (the fifth: chunk 8 and zeros)
+constexpr int kChunks = 10;       // k16 chunks per group (160 K slots)
+constexpr int kCP = 5;            // chunk pairs
 constexpr int kBLane = 16;        // B bytes per (chunk pair, token, lane position)
 constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
 constexpr int kCSGroup = 64;             // C[8], S[8] floats per group
-constexpr int kWarpsP1 = 8, kWarpProd = 8;
-constexpr int kThreads = 9 * 32;
+constexpr int kWarpsP1 = 16, kWarpProd = 16;
+constexpr int kThreads = 17 * 32;
 constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
 constexpr uint32_t kLutShared = 65536;  // shared-window address of the table
 constexpr uint32_t kDynShared = 1024;   // shared-window offset of dynamic smem
@@ -72,6 +76,8 @@ constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
 constexpr int kSOSlot = 2 * kRows * 16;                   // s1 then off, 16 B per row
 constexpr int kCSSlot = kStageG * kCSGroup;               // 512
 constexpr int kBarOff = 2 * kBytesSlot;                   // barriers in arena 1
+constexpr int kYPartOff = kBarOff + 512;                  // 8 x 32 float4: pair hand-off at tile end
+static_assert(kYPartOff + 8 * 32 * 16 <= kArena1, "arena 1 overflow");
 // The table address PRMT: byte 0 = lane * 4, byte 1 = the packed byte,
 // byte 2 = 0x44 (the fp16 exponent of the fifth slot), byte 3 = 0.  The
 // 0x44 is removed again by the load's immediate offset.
@@ -149,40 +155,81 @@ __device__ __forceinline__ uint32_t w_prime(uint32_t w) {
   return d;
 }
 
-// The 18 A words of one row and group from the 7 window words (lane-replicated
-// table; `tag` = kLaneTag | lane * 4, `sel` = 0x7604 | c << 4).
-__device__ __forceinline__ void decode_window(const uint32_t *win, uint32_t tag, uint32_t sel, uint32_t *a) {
-  uint32_t r[7];
+// Window of a group: the aligned words of the stage row that cover its 26
+// bytes, words wstart .. wstart + 6 with wstart = 26 GL / 4 (GL = the
+// group's index in its stage); the group starts o = 26 GL % 4 bytes into
+// the first.  Lane c of a row owns the window words whose stage-row index
+// is c mod 4 (two words: the first at or after wstart, and the one four
+// words later; bytes outside the group get zero activations), which is how
+// ldmatrix hands out 16-byte rows: lane c receives word c of each.
+__host__ __device__ constexpr int win_start(int GL) { return (26 * GL) / 4; }
+// Stage-row word index of lane c's first window word.
+__host__ __device__ constexpr int first_word(int GL, int c) {
+  return win_start(GL) + ((c - win_start(GL)) % 4 + 4) % 4;
+}
+
+// The 20 A words of one row and group from the lane's two window words
+// (lane-replicated table; `tag` = kLaneTag | lane * 4): W, W' of bytes 0..3
+// of the first word, then of the second, then the four V words.
+__device__ __forceinline__ void decode_words(uint32_t w0, uint32_t w1, uint32_t tag, uint32_t *a) {
+  uint32_t r[8];
 #pragma unroll
-  for (int i = 0; i < 7; ++i) r[i] = prmt(win[i], tag, sel);
+  for (int k = 0; k < 4; ++k) {
+    r[k] = prmt(w0, tag, 0x7604u | (k << 4));
+    r[4 + k] = prmt(w1, tag, 0x7604u | (k << 4));
+  }
 #pragma unroll
-  for (int i = 0; i < 7; ++i) {
+  for (int i = 0; i < 8; ++i) {
     const uint32_t w = lut_load(r[i]);
     a[2 * i] = w;
     a[2 * i + 1] = w_prime(w);
   }
-  a[14] = prmt(r[0], r[1], 0x6521u);
-  a[15] = prmt(r[2], r[3], 0x6521u);
-  a[16] = prmt(r[4], r[5], 0x6521u);
-  a[17] = prmt(r[6], r[6], 0x6521u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) a[16 + i] = prmt(r[2 * i], r[2 * i + 1], 0x6521u);
 }
 
 // The same from a compact (not replicated) 256-word table at `lut`.
-__device__ __forceinline__ void decode_window_compact(const uint32_t *win, const uint32_t *lut, int c,
-                                                      uint32_t *a) {
-  uint32_t v[7];
+__device__ __forceinline__ void decode_words_compact(uint32_t w0, uint32_t w1, const uint32_t *lut, uint32_t *a) {
+  uint32_t v[8];
 #pragma unroll
-  for (int i = 0; i < 7; ++i) v[i] = (win[i] >> (8 * c)) & 0xffu;
+  for (int k = 0; k < 4; ++k) {
+    v[k] = (w0 >> (8 * k)) & 0xffu;
+    v[4 + k] = (w1 >> (8 * k)) & 0xffu;
+  }
 #pragma unroll
-  for (int i = 0; i < 7; ++i) {
+  for (int i = 0; i < 8; ++i) {
     const uint32_t w = lut[v[i]];
     a[2 * i] = w;
     a[2 * i + 1] = w_prime(w);
   }
-  a[14] = 0x44004400u | v[0] | (v[1] << 16);
-  a[15] = 0x44004400u | v[2] | (v[3] << 16);
-  a[16] = 0x44004400u | v[4] | (v[5] << 16);
-  a[17] = 0x44004400u | v[6] | (v[6] << 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) a[16 + i] = 0x44004400u | v[2 * i] | (v[2 * i + 1] << 16);
+}
+
+// ldmatrix: four (x4) or two (x2) 8 x 16-byte rows; lane (g, c) receives
+// word c of row g of each.
+__device__ __forceinline__ void ldsm_x4(const void *p, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(smem_u32(p))
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x2(const void *p, uint32_t &r0, uint32_t &r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(smem_u32(p))
+               : "memory");
+}
+
+// 16-byte asynchronous global -> shared copies (completion tracked per
+// thread in commit groups).
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // D += A * B, m16n8k16, fp16 in, fp32 accumulate.
@@ -238,7 +285,7 @@ struct Walk {
 
 // ------------------------------------------------------------------ prep
 // B fragments, C and S for every (problem, group, token).  B layout of a
-// group: [chunk pair cp][token m][lane position c] x 16 B, each 16 B being
+// group: [token m][chunk pair cp][lane position c] x 16 B, each 16 B being
 // (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
 __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp) {
   const int p = blockIdx.y;
@@ -271,36 +318,36 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp) {
          (4.f + 121.f / 256.f) * __half2float(ye[b]);
     S += x[0] + x[1] + x[2] + x[3] + x[4];
   }
-  const int o = (g & 1) ? 2 : 0;  // window offset: stage-relative parity of the group
+  const int GL = g % kStageG;  // the group's index in its stage fixes its window
   unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
   const __half z = __float2half_rn(0.f);
   for (int c = 0; c < 4; ++c) {
-    // byte of window word jw in lane position c, or -1 if not in the group
-    auto byte_of = [&](int jw) -> int {
-      const int b = 4 * jw + c - o;
+    // group byte of byte k of lane c's word i (0: first, 1: second), or -1
+    auto byte_of = [&](int i, int k) -> int {
+      const int b = 4 * (first_word(GL, c) + 4 * i) + k - 26 * GL;
       return (b >= 0 && b < 26) ? b : -1;
     };
     uint32_t words[20];
-    for (int j = 0; j < 7; ++j) {
-      const int b = byte_of(j);
-      __half2 w0 = __halves2half2(z, z), w1 = __halves2half2(z, z);
-      if (b >= 0) {
-        w0 = __halves2half2(ya[b], yb[b]);
-        w1 = __halves2half2(yc[b], yd[b]);
+    for (int i = 0; i < 2; ++i) {
+      for (int k = 0; k < 4; ++k) {
+        const int b = byte_of(i, k);
+        __half2 w0 = __halves2half2(z, z), w1 = __halves2half2(z, z);
+        if (b >= 0) {
+          w0 = __halves2half2(ya[b], yb[b]);
+          w1 = __halves2half2(yc[b], yd[b]);
+        }
+        words[2 * (4 * i + k)] = *reinterpret_cast<uint32_t *>(&w0);
+        words[2 * (4 * i + k) + 1] = *reinterpret_cast<uint32_t *>(&w1);
       }
-      words[2 * j] = *reinterpret_cast<uint32_t *>(&w0);
-      words[2 * j + 1] = *reinterpret_cast<uint32_t *>(&w1);
     }
-    for (int k = 0; k < 4; ++k) {
-      const int b0 = byte_of(2 * k), b1 = k < 3 ? byte_of(2 * k + 1) : -1;
+    for (int i = 0; i < 4; ++i) {
+      const int b0 = byte_of(i >> 1, 2 * (i & 1)), b1 = byte_of(i >> 1, 2 * (i & 1) + 1);
       __half2 v = __halves2half2(b0 >= 0 ? ye[b0] : z, b1 >= 0 ? ye[b1] : z);
-      words[14 + k] = *reinterpret_cast<uint32_t *>(&v);
+      words[16 + i] = *reinterpret_cast<uint32_t *>(&v);
     }
-    words[18] = 0u;
-    words[19] = 0u;
     for (int cp = 0; cp < kCP; ++cp) {
       uint4 q = make_uint4(words[4 * cp], words[4 * cp + 1], words[4 * cp + 2], words[4 * cp + 3]);
-      *reinterpret_cast<uint4 *>(Bg + ((cp * MB + m) * 4 + c) * kBLane) = q;
+      *reinterpret_cast<uint4 *>(Bg + ((m * kCP + cp) * 4 + c) * kBLane) = q;
     }
   }
   float *cs = P.wsCS + (int64_t)g * (kCSGroup / 4);
@@ -368,25 +415,29 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
       for (int e0 = 0; e0 < tg; e0 += 16, ++k) {
         if ((k & 3) != warp) continue;
         const int g = gbase + gl;
-        const int o = (g & 1) ? 2 : 0;
-        uint32_t aL[18], aH[18];
+        uint32_t aL[20], aH[20];
         int rows[2] = {-1, -1};
         float s2v[2] = {0.f, 0.f};
+        // lane c's window words: (c - wstart) mod 4 and 4 words later
+        const int GL = g % kStageG;
+        const int jw1 = ((c - win_start(GL)) % 4 + 4) % 4;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int e = e0 + gq + 8 * h;
-          uint32_t win[7];
+          uint32_t win[8];
 #pragma unroll
-          for (int i = 0; i < 7; ++i) win[i] = 0u;
+          for (int i = 0; i < 8; ++i) win[i] = 0u;
           if (e < tg) {
             const int2 rec = list[gl][e];
             rows[h] = rec.x;
             const int64_t jj = min(max((int64_t)rec.y, (int64_t)0), (int64_t)P.nnz - 1);
             s2v[h] = __half2float(P.s2[jj]);
             // 7 aligned words covering the record (plane 2 is 16-byte aligned,
-            // so the record starts 0 or 2 bytes into a word)
+            // so the record starts 0 or 2 bytes into a word), then shifted so
+            // that the record sits o = 26 GL % 4 bytes into its window
             const uint8_t *A = P.plane2 + jj * kGroupBytes;
             const int sh = (int)(jj & 1) * 2;
+            const int o = (GL & 1) * 2;
             const uint32_t *src = reinterpret_cast<const uint32_t *>(A - sh);
             uint32_t wv[8];
 #pragma unroll
@@ -404,14 +455,21 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
               for (int i = 0; i < 7; ++i) win[i] = __funnelshift_r(wv[i], wv[i + 1], 16);
             }
           }
-          decode_window_compact(win, lut, c, h ? aH : aL);
+          uint32_t w0 = win[0], w1 = win[4];
+#pragma unroll
+          for (int i = 1; i < 4; ++i)
+            if (jw1 == i) {
+              w0 = win[i];
+              w1 = win[i + 4];
+            }
+          decode_words_compact(w0, w1, lut, h ? aH : aL);
         }
         uint32_t b[20];
         const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
 #pragma unroll
         for (int cp = 0; cp < kCP; ++cp) {
           uint4 q = make_uint4(0u, 0u, 0u, 0u);
-          if (gq < MB) q = __ldg(reinterpret_cast<const uint4 *>(Bg + ((cp * MB + gq) * 4 + c) * kBLane));
+          if (gq < MB) q = __ldg(reinterpret_cast<const uint4 *>(Bg + ((gq * kCP + cp) * 4 + c) * kBLane));
           b[4 * cp] = q.x;
           b[4 * cp + 1] = q.y;
           b[4 * cp + 2] = q.z;
@@ -459,6 +517,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     return b < 2 ? ar1 + b * kBytesSlot : ar2 + L.oBytes2 + (b - 2) * kBytesSlot;
   };
   Bars *bars = reinterpret_cast<Bars *>(ar1 + kBarOff);
+  float4 *ypart = reinterpret_cast<float4 *>(ar1 + kYPartOff);
   volatile int32_t *abort_ = &bars->abort_;
 
   // ---- one-time set-up: the lane-replicated table, barriers
@@ -468,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (tid == 0) {
     for (int i = 0; i < NS; ++i) {
-      mbar_init(&bars->full[i], 1 + 32);  // producer's expect-tx arrival + one per producer lane
+      mbar_init(&bars->full[i], 1);  // the producer's expect-tx arrival
       mbar_init(&bars->empty[i], kWarpsP1);
     }
     bars->abort_ = 0;
@@ -479,152 +538,203 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp < kWarpsP1) {
     // ============================================================ decode
-    const int g = lane >> 2, c = lane & 3;
-    const int R0 = warp * 16 + g, R1 = R0 + 8;
-    const uint32_t tag = kLaneTag | ((uint32_t)lane << 2);
-    const uint32_t sel = 0x7604u | ((uint32_t)c << 4);
-    float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
-    uint32_t q = 0;
-    for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
-      const int buf = (int)(q % (uint32_t)NS);
-      const bool ok = wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_);
-      if (!__all_sync(0xffffffffu, ok)) break;
-      const unsigned char *rp0 = bytes_buf(buf) + R0 * kStageBytes;
-      const unsigned char *rp1 = bytes_buf(buf) + R1 * kStageBytes;
-      const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
-      const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * kCSSlot);
-      const unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
-      const uint4 s1a = *reinterpret_cast<const uint4 *>(SO + R0 * 16);
-      const uint4 s1b = *reinterpret_cast<const uint4 *>(SO + R1 * 16);
-      const uint4 ofa = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R0 * 16);
-      const uint4 ofb = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R1 * 16);
-      const uint32_t s1w[2][4] = {{s1a.x, s1a.y, s1a.z, s1a.w}, {s1b.x, s1b.y, s1b.z, s1b.w}};
-      const uint32_t ofw[2][4] = {{ofa.x, ofa.y, ofa.z, ofa.w}, {ofb.x, ofb.y, ofb.z, ofb.w}};
-      const int gs = w.gs;
+    // Warps mt and mt + 8 share the 16 rows of m16 tile mt: the first takes
+    // the stage's even groups, the second the odd ones.  Both fetch half of
+    // the rows' bytes and meet at named barrier 1 + mt once per stage.
+    auto body = [&](auto par_c) {
+      constexpr int PAR = decltype(par_c)::value;
+      const int mt = warp & 7;
+      const uint32_t bar_id = 1u + (uint32_t)mt;
+      const int g = lane >> 2, c = lane & 3;
+      const int R0 = mt * 16 + g, R1 = R0 + 8;
+      const uint32_t tag = kLaneTag | ((uint32_t)lane << 2);
+      const bool breal = g < MB;  // lanes of absent tokens keep zero B operands
+      uint32_t b[20];
 #pragma unroll
-      for (int GL = 0; GL < kStageG; ++GL) {
-        if (GL < gs) {
-          // window words of this group in rows R0 / R1
-          const int c0 = (26 * GL) / 16, c1 = (26 * GL + 25) / 16;
-          const int wstart = (26 * GL) / 4 - 4 * c0;
-          uint32_t u0[12], u1[12];
-#pragma unroll
-          for (int cc = 0; cc < 3; ++cc) {
-            if (c0 + cc <= c1) {
-              const uint4 v0 = *reinterpret_cast<const uint4 *>(rp0 + 16 * (c0 + cc));
-              const uint4 v1 = *reinterpret_cast<const uint4 *>(rp1 + 16 * (c0 + cc));
-              u0[4 * cc] = v0.x; u0[4 * cc + 1] = v0.y; u0[4 * cc + 2] = v0.z; u0[4 * cc + 3] = v0.w;
-              u1[4 * cc] = v1.x; u1[4 * cc + 1] = v1.y; u1[4 * cc + 2] = v1.z; u1[4 * cc + 3] = v1.w;
-            }
+      for (int i = 0; i < 20; ++i) b[i] = 0u;
+      float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
+      // The tile's 16 rows of a stage (packed bytes, s1 and off), fetched with
+      // 16-byte asynchronous copies NS - 1 stages ahead; one commit group per
+      // stage and warp.
+      auto fetch_rows = [&](const Walk &a, int slot) {
+        const Problem &P = a.P();
+        const int64_t RB = row_bytes_of(P.K);
+        const int n0 = (a.tile - P.tile_begin) * kRows + mt * 16;
+        const int rows = min(16, P.N - n0);
+        const int nch = (a.gs * kGroupBytes + 15) / 16;  // 16-byte chunks per row
+        unsigned char *dst = bytes_buf(slot) + mt * 16 * kStageBytes;
+        const unsigned char *src = P.plane1 + (int64_t)n0 * RB + (int64_t)a.s * kStageBytes;
+        if (nch == kStageBytes / 16) {
+          for (int i = 2 * lane + PAR; i < rows * (kStageBytes / 16); i += 64) {
+            const int r = i / (kStageBytes / 16), ch = i - r * (kStageBytes / 16);
+            cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
           }
-          uint32_t aL[18], aH[18];
-          decode_window(u0 + wstart, tag, sel, aL);
-          decode_window(u1 + wstart, tag, sel, aH);
-          uint32_t b[20];
-#pragma unroll
-          for (int cp = 0; cp < kCP; ++cp) {
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (g < MB) v = *reinterpret_cast<const uint4 *>(Bst + GL * kBTok * MB + ((cp * MB + g) * 4 + c) * kBLane);
-            b[4 * cp] = v.x;
-            b[4 * cp + 1] = v.y;
-            b[4 * cp + 2] = v.z;
-            b[4 * cp + 3] = v.w;
-          }
-          float d[4];
-          group_mma(aL, aH, b, d);
-          const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
-          const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
-            const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
-            const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
-            y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
-            y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
+        } else {
+          for (int i = 2 * lane + PAR; i < rows * nch; i += 64) {
+            const int r = i / nch, ch = i - r * nch;
+            cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
           }
         }
+        const int G = P.K / kGroup, g0 = a.s * kStageG;
+        const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+        const __half *arr = PAR ? P.off : P.s1;  // the even-group warp fetches s1, the other off
+        unsigned char *d = ar2 + L.oSO + slot * kSOSlot + PAR * kRows * 16 + (mt * 16 + lane) * 16;
+        if (lane < rows) {
+          const int64_t o = (int64_t)(n0 + lane) * G + g0;
+          if (vec) {
+            cp_async16(d, arr + o);
+          } else {
+            __half *dh = reinterpret_cast<__half *>(d);
+            for (int gg = 0; gg < kStageG; ++gg) dh[gg] = gg < a.gs ? arr[o + gg] : __float2half_rn(0.f);
+          }
+        }
+        cp_async_commit();
+      };
+      Walk ahead(&bp, t_begin, t_end);
+      for (int k = 0; k < NS - 1; ++k) {
+        if (ahead.valid()) {
+          fetch_rows(ahead, k);
+          ahead.next();
+        } else {
+          cp_async_commit();
+        }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->empty[buf]);
-      if (w.last_stage()) {
-        const Problem &P = w.P();
-        const int nb = (w.tile - P.tile_begin) * kRows;
+      uint32_t q = 0;
+      for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
+        const int buf = (int)(q % (uint32_t)NS);
+        // refill the slot the previous stage used, then wait for this stage
+        if (ahead.valid()) {
+          fetch_rows(ahead, (int)((q + NS - 1) % (uint32_t)NS));
+          ahead.next();
+        } else {
+          cp_async_commit();
+        }
+        if (NS == 4)
+          cp_async_wait<3>();
+        else
+          cp_async_wait<2>();
+        const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_));
+        // both warps of the pair see each other's copies and take the same decision
+        if (named_bar_any(bar_id, 64, !ok || *abort_ != 0)) break;
+        // this lane's ldmatrix row: row (lane % 16) of the m16 tile
+        const unsigned char *mrow = bytes_buf(buf) + (mt * 16 + (lane & 15)) * kStageBytes;
+        const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
+        const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * kCSSlot);
+        const unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
+        const uint4 s1a = *reinterpret_cast<const uint4 *>(SO + R0 * 16);
+        const uint4 s1b = *reinterpret_cast<const uint4 *>(SO + R1 * 16);
+        const uint4 ofa = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R0 * 16);
+        const uint4 ofb = *reinterpret_cast<const uint4 *>(SO + kRows * 16 + R1 * 16);
+        const uint32_t s1w[2][4] = {{s1a.x, s1a.y, s1a.z, s1a.w}, {s1b.x, s1b.y, s1b.z, s1b.w}};
+        const uint32_t ofw[2][4] = {{ofa.x, ofa.y, ofa.z, ofa.w}, {ofb.x, ofb.y, ofb.z, ofb.w}};
+        const int gs = w.gs;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int n = nb + (h ? R1 : R0);
-          if (n < P.N) {
+        for (int GL = PAR; GL < kStageG; GL += 2) {
+          if (GL < gs) {
+            // the group's 16-byte chunks of rows R0 / R1 (2 or 3), one ldmatrix
+            const int k0 = win_start(GL) / 4, kl = (win_start(GL) + 6) / 4, sft = win_start(GL) % 4;
+            uint32_t x0[3], x1[3];
+            ldsm_x4(mrow + 16 * (lane < 16 ? k0 : k0 + 1), x0[0], x1[0], x0[1], x1[1]);
+            if (kl == k0 + 2) {
+              ldsm_x2(mrow + 16 * (k0 + 2), x0[2], x1[2]);
+            } else {
+              x0[2] = x0[1];
+              x1[2] = x1[1];
+            }
+            // lane c's two words: chunks k0, k0 + 1, or k0 + 1, k0 + 2 when c < wstart % 4
+            const bool up = c < sft;
+            uint32_t aL[20], aH[20];
+            decode_words(up ? x0[1] : x0[0], up ? x0[2] : x0[1], tag, aL);
+            decode_words(up ? x1[1] : x1[0], up ? x1[2] : x1[1], tag, aH);
+            if (breal) {
+              const unsigned char *bsrc = Bst + GL * kBTok * MB + g * kBTok + c * kBLane;
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-              const int m = 2 * c + i;
-              if (m < M) {
-                float v = y[2 * h + i];
-                if (P.nnz > 0) v += P.wsY2[(int64_t)n * MB + m];
-                if (F32)
-                  static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
-                else
-                  static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
+              for (int cp = 0; cp < kCP; ++cp) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(bsrc + cp * 4 * kBLane);
+                b[4 * cp] = v.x;
+                b[4 * cp + 1] = v.y;
+                b[4 * cp + 2] = v.z;
+                b[4 * cp + 3] = v.w;
+              }
+            }
+            float d[4];
+            group_mma(aL, aH, b, d);
+            const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
+            const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
+              const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
+              const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+              y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
+              y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
+            }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->empty[buf]);
+        if (w.last_stage()) {
+          // the odd-group warp hands its partial sums to the even-group warp,
+          // which adds the second plane and writes y
+          float4 *yp = ypart + mt * 32 + lane;
+          if (PAR == 1) *yp = make_float4(y[0], y[1], y[2], y[3]);
+          named_bar(bar_id, 64);
+          if (PAR == 0) {
+            const float4 o = *yp;
+            y[0] += o.x;
+            y[1] += o.y;
+            y[2] += o.z;
+            y[3] += o.w;
+            const Problem &P = w.P();
+            const int nb = (w.tile - P.tile_begin) * kRows;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int n = nb + (h ? R1 : R0);
+              if (n < P.N) {
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                  const int m = 2 * c + i;
+                  if (m < M) {
+                    float v = y[2 * h + i];
+                    if (P.nnz > 0) v += P.wsY2[(int64_t)n * MB + m];
+                    if (F32)
+                      static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
+                    else
+                      static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
+                  }
+                }
               }
             }
           }
-        }
 #pragma unroll
-        for (int i = 0; i < 4; ++i) y[i] = 0.f;
+          for (int i = 0; i < 4; ++i) y[i] = 0.f;
+        }
       }
-    }
+    };
+    if (warp >= 8)
+      body(std::integral_constant<int, 1>{});
+    else
+      body(std::integral_constant<int, 0>{});
+    cp_async_wait<0>();  // nothing in flight into shared memory at exit
   } else if (warp == kWarpProd) {
     // ========================================================== producer
     uint32_t q = 0;
     for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
       const Problem &P = w.P();
-      const int G = P.K / kGroup;
-      const int64_t RB = row_bytes_of(P.K);
-      const int n0 = (w.tile - P.tile_begin) * kRows;
-      const int rows = min(kRows, P.N - n0);
-      const int s = w.s, gs = w.gs, g0 = s * kStageG;
-      const uint32_t rb = (uint32_t)((gs * kGroupBytes + 15) / 16 * 16);
+      const int gs = w.gs, g0 = w.s * kStageG;
       const uint32_t bb = (uint32_t)(gs * kBTok * MB);
       const uint32_t cb = (uint32_t)(gs * kCSGroup);
       const int buf = (int)(q % (uint32_t)NS);
       int ok = 1;
       if (lane == 0) ok = wait_or_abort(&bars->empty[buf], ((q / NS) & 1u) ^ 1u, abort_) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
-      unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
       if (lane == 0) {
-        mbar_arrive_expect_tx(&bars->full[buf], rb * (uint32_t)rows + bb + cb);
+        mbar_arrive_expect_tx(&bars->full[buf], bb + cb);
         bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, &bars->full[buf]);
         bulk_g2s(ar2 + L.oCS + buf * kCSSlot, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * kCSGroup,
                  cb, &bars->full[buf]);
       }
       __syncwarp();
-      for (int rr = lane; rr < rows; rr += 32)
-        bulk_g2s(bytes_buf(buf) + rr * kStageBytes, P.plane1 + (int64_t)(n0 + rr) * RB + (int64_t)s * kStageBytes, rb,
-                 &bars->full[buf]);
-      // s1 / off of the stage: 8 halves per row
-      const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
-      if (vec) {
-        for (int rr = lane; rr < rows; rr += 32) {
-          const int64_t o = ((int64_t)(n0 + rr) * G + g0) * 2;
-          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(SO + rr * 16)),
-                       "l"(reinterpret_cast<const unsigned char *>(P.s1) + o)
-                       : "memory");
-          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(SO + kRows * 16 + rr * 16)),
-                       "l"(reinterpret_cast<const unsigned char *>(P.off) + o)
-                       : "memory");
-        }
-        asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&bars->full[buf]))
-                     : "memory");
-      } else {
-        for (int rr = lane; rr < rows; rr += 32) {
-          __half *d1 = reinterpret_cast<__half *>(SO + rr * 16);
-          __half *d2 = reinterpret_cast<__half *>(SO + kRows * 16 + rr * 16);
-          const int64_t o = (int64_t)(n0 + rr) * G + g0;
-          for (int gg = 0; gg < kStageG; ++gg) {
-            d1[gg] = gg < gs ? P.s1[o + gg] : __float2half_rn(0.f);
-            d2[gg] = gg < gs ? P.off[o + gg] : __float2half_rn(0.f);
-          }
-        }
-        mbar_arrive(&bars->full[buf]);
-      }
     }
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
