@@ -72,7 +72,9 @@ typedef enum {
   TQ_ERR_BYTE = -5,     /* reserved: invalid packed byte (d_status)       */
   TQ_ERR_SALIENCE = -6, /* descriptor nnz / salience inconsistent          */
   TQ_ERR_CUDA = -7,     /* a CUDA launch or query failed                  */
-  TQ_ERR_TIMEOUT = -8   /* a bounded device wait ran out                  */
+  TQ_ERR_TIMEOUT = -8,  /* a bounded device wait ran out                  */
+  TQ_ERR_SCRATCH = -9   /* tq_linear_static: the call needs more scratch than
+                           TQ_STATIC_SCRATCH_BYTES                         */
 } tq_status;
 
 /* Bits OR-ed into *d_status by the codec kernels. */
@@ -175,6 +177,38 @@ TQ_API size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_prob
 
 TQ_API tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
                                    size_t workspace_bytes, void *stream);
+
+/* ---------------------------------------------------------------------
+ * Allocation-free variant (no counterpart in the paper; an integration aid).
+ *
+ * tq_linear_static is tq_linear with its workspace taken from a scratch
+ * array that the library itself holds in device memory (a file-scope
+ * __device__ array of TQ_STATIC_SCRATCH_BYTES, reserved when the module
+ * loads), so the caller passes no workspace and nothing is allocated at
+ * call time.  It is for callers that cannot allocate or own device memory:
+ * code inside a region where allocation is not allowed (a stream being
+ * captured, where cudaMalloc / cudaFree would invalidate the capture, or a
+ * serving loop that forbids allocator calls and their implicit
+ * synchronization), and hosts that have no allocator to hand (plain C
+ * callers of the library).
+ *
+ *   - Limit: the call's need, tq_workspace_bytes(M, N, K), must not exceed
+ *     TQ_STATIC_SCRATCH_BYTES (1 MiB: every Qwen3-8B projection up to
+ *     M = 16); otherwise TQ_ERR_SCRATCH is returned before anything runs.
+ *   - Set-up: the first call on a device looks up the scratch array's device
+ *     address once (cudaGetSymbolAddress) and caches it for that device; make
+ *     that first call before any stream capture on the device.  A failed
+ *     lookup returns TQ_ERR_CUDA.
+ *   - Nothing in the scratch has to start at zero: every call writes all of
+ *     the scratch it reads before reading it.
+ *   - There is ONE scratch array per device: calls on the same device that
+ *     may overlap in time (different streams, different host threads without
+ *     ordering) race on it and produce wrong results.  Serialize them.
+ * Arguments, layouts and other errors as tq_linear.
+ */
+#define TQ_STATIC_SCRATCH_BYTES ((size_t)1 << 20)
+TQ_API tq_status tq_linear_static(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
+                                  uint16_t *y, void *stream);
 
 /* Device status word of the library's linear kernels, OR of:
  *   1 = a bounded device-side wait ran out (the kernel stopped early and its

@@ -92,6 +92,9 @@ size_t problem_ws_bytes(int M, int N, int K) {
   return pad256(tc_workspace_bytes(16, K));
 }
 
+}  // namespace
+
+namespace tq {
 // Workspace bytes that cover every chunk of a call over M tokens (chunks of
 // TQ_MAX_SKINNY_M; a remainder of at most 8 tokens takes the M <= 8 path).
 size_t call_ws_bytes(int M, int N, int K) {
@@ -99,6 +102,9 @@ size_t call_ws_bytes(int M, int N, int K) {
   const size_t a = problem_ws_bytes(16, N, K), b = problem_ws_bytes(8, N, K);
   return a > b ? a : b;
 }
+}  // namespace tq
+
+namespace {
 
 // Places every problem's workspace and runs the decode path for bp.M tokens
 // (M <= 8: warp-level MMA kernels; 8 < M <= 16: the tensor-memory kernel).
@@ -261,6 +267,8 @@ const char *tq_status_str(tq_status s) {
     case TQ_ERR_SALIENCE: return "TQ_ERR_SALIENCE: nnz inconsistent with the salience map";
     case TQ_ERR_CUDA: return "TQ_ERR_CUDA: a CUDA launch failed";
     case TQ_ERR_TIMEOUT: return "TQ_ERR_TIMEOUT: a bounded device wait ran out";
+    case TQ_ERR_SCRATCH:
+      return "TQ_ERR_SCRATCH: the call needs more workspace than the static scratch of tq_linear_static (1 MiB)";
   }
   return "unknown tq_status";
 }

@@ -79,6 +79,8 @@ def lib():
             L.tq_linear.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp, sz, vp]
             L.tq_linear_f32out.restype = ctypes.c_int
             L.tq_linear_f32out.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp, sz, vp]
+            L.tq_linear_static.restype = ctypes.c_int
+            L.tq_linear_static.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp]
             L.tq_linear_batched.restype = ctypes.c_int
             L.tq_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
             L.tq_get_device_status.restype = ctypes.c_int
@@ -238,6 +240,21 @@ def tq_linear_f32out(x, w: PackedWeight, y=None, ws=None, stream=None):
     ws_ = w.struct()
     _check(lib().tq_linear_f32out(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _p(ws), ws.numel(),
                                   _stream(stream)), "tq_linear_f32out")
+    return y
+
+
+STATIC_SCRATCH_BYTES = 1 << 20  # TQ_STATIC_SCRATCH_BYTES
+
+
+def tq_linear_static(x, w: PackedWeight, y=None, stream=None):
+    """y = x W^T, fp16, with the library's own device scratch (no workspace
+    argument, nothing allocated by the call except y when y is None)."""
+    M, K = x.shape
+    assert K == w.K and x.dtype == torch.float16
+    if y is None:
+        y = torch.empty((M, w.N), dtype=torch.float16, device=x.device)
+    ws_ = w.struct()
+    _check(lib().tq_linear_static(M, w.N, K, ctypes.byref(ws_), _p(x), _p(y), _stream(stream)), "tq_linear_static")
     return y
 
 
