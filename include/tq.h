@@ -61,7 +61,8 @@ extern "C" {
 #define TQ_GROUP 128        /* trits per group along K                       */
 #define TQ_GROUP_BYTES 26   /* bytes per packed 128-trit group                */
 #define TQ_TRITS_PER_BYTE 5 /* 3^5 = 243 <= 256                               */
-#define TQ_MAX_SKINNY_M 16  /* M <= this runs the decode (GEMV / skinny) path */
+#define TQ_MAX_SKINNY_M 16  /* M <= this runs the decode (GEMV / skinny) path,
+                               larger M the prefill tile path               */
 
 typedef enum {
   TQ_OK = 0,
@@ -138,15 +139,18 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
  * and for M <= 8 the second plane's fp32 partial sums of every row are
  * staged there before the first plane is streamed.  The caller provides this
  * scratch memory (the library never allocates).  Bytes needed for one
- * projection of N rows, K inputs and M tokens (a call with M > 16 runs in
- * chunks of 16 and needs the amount returned for its M); 0 if M, N or K is
- * invalid. */
+ * projection of N rows, K inputs and M tokens; a call with M > 16 (the
+ * prefill tile path) uses none and the function returns 256 for it; 0 if M,
+ * N or K is invalid. */
 TQ_API size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K);
 
 /* y = x W^T for one packed projection (paper "Direct Packed Execution").
  *   x: fp16 [M][K] row-major, 16-byte aligned; y: fp16 [M][N] (rounded to
- *   nearest even from the fp32 accumulator).  M >= 1; M is processed in
- *   chunks of TQ_MAX_SKINNY_M tokens on the decode path.
+ *   nearest even from the fp32 accumulator).  M >= 1.  M <= 16 runs the
+ *   decode path straight from the packed bytes; M > 16 runs the prefill
+ *   path, which dequantizes each 256-row x 128-column weight tile to fp16
+ *   (w = s1 t1 + off + s2 t2, rounded once) and multiplies it by 128-token
+ *   activation tiles on the tensor cores.
  *   workspace: device scratch of at least tq_workspace_bytes(M, N, K) bytes,
  *   256-byte aligned; its contents are overwritten; calls that share a
  *   workspace must not overlap in time.

@@ -27,6 +27,8 @@ cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
+cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
+cudaError_t read_status_prefill(uint32_t *out, bool clear);
 }  // namespace tq
 
 using namespace tq;
@@ -95,12 +97,11 @@ size_t problem_ws_bytes(int M, int N, int K) {
 }  // namespace
 
 namespace tq {
-// Workspace bytes that cover every chunk of a call over M tokens (chunks of
-// TQ_MAX_SKINNY_M; a remainder of at most 8 tokens takes the M <= 8 path).
+// Workspace bytes of a call over M tokens (M > TQ_MAX_SKINNY_M runs the
+// prefill tile path, which needs none: 256 bytes keep the argument uniform).
 size_t call_ws_bytes(int M, int N, int K) {
-  if (M <= 8) return problem_ws_bytes(M, N, K);
-  const size_t a = problem_ws_bytes(16, N, K), b = problem_ws_bytes(8, N, K);
-  return a > b ? a : b;
+  if (M > TQ_MAX_SKINNY_M) return 256;
+  return problem_ws_bytes(M, N, K);
 }
 }  // namespace tq
 
@@ -145,17 +146,17 @@ tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const
   if (!aligned16(x) || ((uintptr_t)ws & 255u)) return TQ_ERR_ALIGN;
   if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
   if (ws_bytes < call_ws_bytes(M, N, K)) return TQ_ERR_SHAPE;
-  static BatchParams bp;  // large; filled per call (host-side, not thread-safe across calls)
-  // Tokens are processed in chunks of TQ_MAX_SKINNY_M.
-  for (int32_t m0 = 0; m0 < M; m0 += TQ_MAX_SKINNY_M) {
-    const int32_t mc = M - m0 < TQ_MAX_SKINNY_M ? M - m0 : TQ_MAX_SKINNY_M;
-    bp.count = 1;
-    bp.M = mc;
-    bp.out_f32 = f32 ? 1 : 0;
-    char *yb = static_cast<char *>(y) + (int64_t)m0 * N * (f32 ? 4 : 2);
-    bp.prob[0] = to_problem(w, x + (int64_t)m0 * K, yb);
-    if (tq_status st = run_batch(bp, static_cast<unsigned char *>(ws), ws_bytes, s)) return st;
+  if (M > TQ_MAX_SKINNY_M) {
+    // prefill: dequantized weight tiles x activation tiles on the tensor cores
+    const Problem P = to_problem(w, x, y);
+    return from_cuda(launch_prefill(P, M, f32, s));
   }
+  static BatchParams bp;  // large; filled per call (host-side, not thread-safe across calls)
+  bp.count = 1;
+  bp.M = M;
+  bp.out_f32 = f32 ? 1 : 0;
+  bp.prob[0] = to_problem(w, x, y);
+  if (tq_status st = run_batch(bp, static_cast<unsigned char *>(ws), ws_bytes, s)) return st;
   return TQ_OK;
 }
 
@@ -249,10 +250,11 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {
   if (!status_host) return TQ_ERR_NULL;
-  uint32_t a = 0, b = 0;
+  uint32_t a = 0, b = 0, c = 0;
   if (read_status_gemv_tc(&a, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
   if (read_status_gemv_mma(&b, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
-  *status_host = a | b;
+  if (read_status_prefill(&c, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  *status_host = a | b | c;
   return TQ_OK;
 }
 

@@ -15,8 +15,8 @@
 // maps v to the fp16x2 word
 //   W  = (4 + d0 + d2/4, 4 + d1 + d3/4)
 // and one LOP3 gives W' = (16 + d2, 16 + d3).  The fifth slot is the byte
-// value itself, 4 + v/256, read straight off the table address (two bytes
-// share one PRMT).  With z_i = x_i - 3^i x4 / 81 the activation slots
+// value itself, 4 + v/256: one PRMT puts two bytes of a packed word under
+// the exponent byte 0x44.  With z_i = x_i - 3^i x4 / 81 the activation slots
 //   y_a = z0, y_b = z1, y_c = z2 - z0/4, y_d = z3 - z1/4, y_e = 256 x4 / 81
 // make the MMA return  const + sum_i d_i x_i  (exact up to the rounding of
 // the slots to fp16); subtracting C, the same MMA for all digits 1 (all
@@ -64,8 +64,8 @@ constexpr int kCP = 5;            // chunk pairs
 constexpr int kBLane = 16;        // B bytes per (chunk pair, token, lane position)
 constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
 constexpr int kCSGroup = 64;             // C[8], S[8] floats per group
-constexpr int kWarpsP1 = 16, kWarpProd = 16;
-constexpr int kThreads = 17 * 32;
+constexpr int kWarpsP1 = 8, kWarpProd = 8;
+constexpr int kThreads = 9 * 32;
 constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
 constexpr uint32_t kLutShared = 65536;  // shared-window address of the table
 constexpr uint32_t kDynShared = 1024;   // shared-window offset of dynamic smem
@@ -76,13 +76,7 @@ constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
 constexpr int kSOSlot = 2 * kRows * 16;                   // s1 then off, 16 B per row
 constexpr int kCSSlot = kStageG * kCSGroup;               // 512
 constexpr int kBarOff = 2 * kBytesSlot;                   // barriers in arena 1
-constexpr int kYPartOff = kBarOff + 512;                  // 8 x 32 float4: pair hand-off at tile end
-static_assert(kYPartOff + 8 * 32 * 16 <= kArena1, "arena 1 overflow");
-// The table address PRMT: byte 0 = lane * 4, byte 1 = the packed byte,
-// byte 2 = 0x44 (the fp16 exponent of the fifth slot), byte 3 = 0.  The
-// 0x44 is removed again by the load's immediate offset.
-constexpr uint32_t kLaneTag = 0x00440000u;
-constexpr int kLutImm = (int)kLutShared - (int)kLaneTag;
+static_assert(kBarOff + 512 <= kArena1, "arena 1 overflow");
 
 __host__ __device__ constexpr int num_slots(int MB) { return MB <= 2 ? 4 : 3; }
 __host__ __device__ constexpr int b_stage_bytes(int MB) { return kStageG * kBTok * MB; }
@@ -117,8 +111,10 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, vo
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 0) {
+    // sleep in the wait rather than spin: the waiting warps share the
+    // issue slots with the decoding warps
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if ((i & 7u) == 0) {
       if (*abort_) return false;
       if (global_ns() - t0 > kWaitLimitNs) break;
     }
@@ -144,9 +140,10 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t s) {
   asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(s));
   return d;
 }
-__device__ __forceinline__ uint32_t lut_load(uint32_t tagged_addr) {
+// The table is constant after set-up: an ordinary (reorderable) load.
+__device__ __forceinline__ uint32_t lut_load(uint32_t addr) {
   uint32_t w;
-  asm volatile("ld.shared.u32 %0, [%1+%2];" : "=r"(w) : "r"(tagged_addr), "n"(kLutImm) : "memory");
+  asm("ld.shared.u32 %0, [%1];" : "=r"(w) : "r"(addr));
   return w;
 }
 __device__ __forceinline__ uint32_t w_prime(uint32_t w) {
@@ -169,8 +166,10 @@ __host__ __device__ constexpr int first_word(int GL, int c) {
 }
 
 // The 20 A words of one row and group from the lane's two window words
-// (lane-replicated table; `tag` = kLaneTag | lane * 4): W, W' of bytes 0..3
-// of the first word, then of the second, then the four V words.
+// (lane-replicated table; `tag` = table base | lane * 4, so that one PRMT
+// yields the entry's address): W, W' of bytes 0..3 of the first word, then
+// of the second, then the four V words, each made by one PRMT of a word's
+// byte pair with the fifth slot's exponent byte 0x44.
 __device__ __forceinline__ void decode_words(uint32_t w0, uint32_t w1, uint32_t tag, uint32_t *a) {
   uint32_t r[8];
 #pragma unroll
@@ -184,8 +183,11 @@ __device__ __forceinline__ void decode_words(uint32_t w0, uint32_t w1, uint32_t 
     a[2 * i] = w;
     a[2 * i + 1] = w_prime(w);
   }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) a[16 + i] = prmt(r[2 * i], r[2 * i + 1], 0x6521u);
+  const uint32_t e44 = 0x44444444u;
+  a[16] = prmt(w0, e44, 0x4140u);
+  a[17] = prmt(w0, e44, 0x4342u);
+  a[18] = prmt(w1, e44, 0x4140u);
+  a[19] = prmt(w1, e44, 0x4342u);
 }
 
 // The same from a compact (not replicated) 256-word table at `lut`.
@@ -242,12 +244,24 @@ __device__ __forceinline__ void mma16816(float *d, uint32_t a0, uint32_t a1, uin
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// The 9 MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
+// D = A * B (zero accumulator in).
+__device__ __forceinline__ void mma16816_z(float *d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                           uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%10,%10,%10,%10};"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.f));
+}
+
+// The MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
 // (b[2j], b[2j+1] for chunk j).  Two accumulation chains, summed into d.
 __device__ __forceinline__ void group_mma(const uint32_t *aL, const uint32_t *aH, const uint32_t *b, float *d) {
-  float e[4] = {0.f, 0.f, 0.f, 0.f}, o[4] = {0.f, 0.f, 0.f, 0.f};
+  float e[4], o[4];
+  mma16816_z(e, aL[0], aH[0], aL[1], aH[1], b[0], b[1]);
+  mma16816_z(o, aL[2], aH[2], aL[3], aH[3], b[2], b[3]);
 #pragma unroll
-  for (int j = 0; j < kChunks; ++j) {
+  for (int j = 2; j < kChunks; ++j) {
     float *acc = (j & 1) ? o : e;
     mma16816(acc, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
   }
@@ -358,10 +372,37 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp) {
 }
 
 // ------------------------------------------------------------ plane 2
-// One CTA (4 warps) per 128-row tile of one problem.  Thread t = row t
-// compacts the tile's salient pairs of each 32-group salience word into
-// per-group lists; each warp then takes 16-record items of one group.
+// One CTA (4 warps) per 128-row tile of one problem.  For each 32-group
+// salience word, thread t = row t compacts the tile's salient pairs into
+// per-group row lists; then the records (the 28 aligned bytes around each)
+// and their s2 are staged in shared memory with asynchronous copies, one
+// round of at most kRecCap records at a time, and each warp multiplies
+// 16-record items of one group like the first plane (the activation
+// fragments of the next item are loaded while the current one computes).
+// s2 * P2 per row accumulates in shared memory and goes to the workspace
+// (y2, fp32) at the end.
 constexpr int kP2Threads = 128;
+constexpr int kRecCap = 512;
+constexpr int kMaxItems = kRecCap / 16 + 32;
+
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void load_b_frag(const Problem &P, int g, int MB, int gq, int c, uint32_t *b, float2 &Cv) {
+  const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
+#pragma unroll
+  for (int cp = 0; cp < kCP; ++cp) {
+    uint4 q = make_uint4(0u, 0u, 0u, 0u);
+    if (gq < MB) q = __ldg(reinterpret_cast<const uint4 *>(Bg + ((gq * kCP + cp) * 4 + c) * kBLane));
+    b[4 * cp] = q.x;
+    b[4 * cp + 1] = q.y;
+    b[4 * cp + 2] = q.z;
+    b[4 * cp + 3] = q.w;
+  }
+  Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + 2 * c));
+}
+
 __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_constant__ BatchParams bp) {
   const int p = blockIdx.y;
   if (p >= bp.count) return;
@@ -370,8 +411,15 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
   if (n0 >= P.N) return;
   const int MB = bp.M;
   __shared__ uint32_t lut[256];
-  __shared__ int2 list[32][kRows];  // (row, record index)
-  __shared__ int cnt[4][32], base[4][32], tot[32];
+  __shared__ uint8_t rowl[32][kRows];  // row of each salient pair, per group
+  __shared__ int jbase[kRows];         // record index of the row's first pair in this word
+  __shared__ uint32_t bitsv[kRows];    // the row's salience bits of this word
+  __shared__ int cnt[4][32];
+  __shared__ int eoff[33];             // per-group offsets in the flat (group-major) pair order
+  __shared__ int itm[kMaxItems];       // item: group << 16 | first flat pair
+  __shared__ int nitm;
+  __shared__ __align__(16) uint32_t rec[kRecCap][8];  // 28 record bytes + the record's word offset
+  __shared__ float s2s[kRecCap];
   __shared__ float acc[kRows][8];
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   for (int i = t; i < 256; i += kP2Threads) lut[i] = lut_word(i);
@@ -387,6 +435,8 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
     const int gbase = 32 * w, gw = min(32, G - gbase);
     uint32_t bits = valid ? P.sal[(int64_t)n * W + w] : 0u;
     if (gw < 32) bits &= (1u << gw) - 1u;
+    jbase[t] = j;
+    bitsv[t] = bits;
     for (int gl = 0; gl < 32; ++gl) {
       const uint32_t m = __ballot_sync(0xffffffffu, (bits >> gl) & 1u);
       if (lane == 0) cnt[warp][gl] = __popc(m);
@@ -395,62 +445,99 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
     if (t < 32) {
       int s = 0;
       for (int ww = 0; ww < 4; ++ww) {
-        base[ww][t] = s;
-        s += cnt[ww][t];
+        const int v = cnt[ww][t];
+        cnt[ww][t] = s;  // becomes the warp's base within the group
+        s += v;
       }
-      tot[t] = s;
+      // exclusive scan of the group totals across the warp
+      int incl = s;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      eoff[t] = incl - s;
+      if (t == 31) eoff[32] = incl;
     }
     __syncthreads();
     for (int gl = 0; gl < 32; ++gl) {
       const uint32_t m = __ballot_sync(0xffffffffu, (bits >> gl) & 1u);
-      if ((bits >> gl) & 1u)
-        list[gl][base[warp][gl] + __popc(m & lt)] = make_int2(t, j + __popc(bits & ((1u << gl) - 1u)));
+      if ((bits >> gl) & 1u) rowl[gl][cnt[warp][gl] + __popc(m & lt)] = (uint8_t)t;
     }
     j += __popc(bits);
     __syncthreads();
-    // items: (group, first record) in order; item k goes to warp k % 4
-    int k = 0;
-    for (int gl = 0; gl < gw; ++gl) {
-      const int tg = tot[gl];
-      for (int e0 = 0; e0 < tg; e0 += 16, ++k) {
-        if ((k & 3) != warp) continue;
-        const int g = gbase + gl;
+    const int E = eoff[32];
+    for (int r0 = 0; r0 < E; r0 += kRecCap) {
+      const int r1 = min(E, r0 + kRecCap);
+      // ---- stage the round's records and s2
+      for (int e = r0 + t; e < r1; e += kP2Threads) {
+        int gl = 0;
+#pragma unroll
+        for (int step = 16; step >= 1; step >>= 1)
+          if (gl + step < 32 && eoff[gl + step] <= e) gl += step;
+        const int row = rowl[gl][e - eoff[gl]];
+        const int64_t jj = min(max((int64_t)jbase[row] + __popc(bitsv[row] & ((1u << gl) - 1u)), (int64_t)0),
+                               (int64_t)P.nnz - 1);
+        const uint8_t *A = P.plane2 + jj * kGroupBytes;
+        const int sh = (int)(jj & 1) * 2;  // plane 2 is 16-byte aligned: the record starts 0 or 2 bytes into a word
+        const uint32_t *src = reinterpret_cast<const uint32_t *>(A - sh);
+        uint32_t *dst = rec[e - r0];
+#pragma unroll
+        for (int i = 0; i < 6; ++i) cp_async4(dst + i, src + i);
+        if (sh) {
+          cp_async4(dst + 6, src + 6);
+        } else {  // bytes 24, 25 only: the word after them may lie past the end of plane 2
+          dst[6] = (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
+        }
+        dst[7] = (uint32_t)sh;
+        s2s[e - r0] = __half2float(P.s2[jj]);
+      }
+      asm volatile("cp.async.wait_all;" ::: "memory");
+      if (t == 0) {
+        int k = 0;
+        for (int gl = 0; gl < gw; ++gl) {
+          const int a = max(eoff[gl], r0), b = min(eoff[gl + 1], r1);
+          for (int e = a; e < b; e += 16) itm[k++] = (gl << 16) | e;
+        }
+        nitm = k;
+      }
+      __syncthreads();
+      // ---- items
+      const int ni = nitm;
+      uint32_t b[20], bn[20];
+      float2 Cv = make_float2(0.f, 0.f), Cn = Cv;
+      if (warp < ni) load_b_frag(P, gbase + (itm[warp] >> 16), MB, gq, c, b, Cv);
+      for (int k = warp; k < ni; k += 4) {
+        if (k + 4 < ni) load_b_frag(P, gbase + (itm[k + 4] >> 16), MB, gq, c, bn, Cn);
+        const int gl = itm[k] >> 16, e0 = itm[k] & 0xffff;
+        const int seg_end = min(eoff[gl + 1], r1);
+        const int g = gbase + gl, GL = g % kStageG;
+        const int o = (GL & 1) * 2;
+        const int jw1 = ((c - win_start(GL)) % 4 + 4) % 4;
         uint32_t aL[20], aH[20];
         int rows[2] = {-1, -1};
         float s2v[2] = {0.f, 0.f};
-        // lane c's window words: (c - wstart) mod 4 and 4 words later
-        const int GL = g % kStageG;
-        const int jw1 = ((c - win_start(GL)) % 4 + 4) % 4;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int e = e0 + gq + 8 * h;
           uint32_t win[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) win[i] = 0u;
-          if (e < tg) {
-            const int2 rec = list[gl][e];
-            rows[h] = rec.x;
-            const int64_t jj = min(max((int64_t)rec.y, (int64_t)0), (int64_t)P.nnz - 1);
-            s2v[h] = __half2float(P.s2[jj]);
-            // 7 aligned words covering the record (plane 2 is 16-byte aligned,
-            // so the record starts 0 or 2 bytes into a word), then shifted so
-            // that the record sits o = 26 GL % 4 bytes into its window
-            const uint8_t *A = P.plane2 + jj * kGroupBytes;
-            const int sh = (int)(jj & 1) * 2;
-            const int o = (GL & 1) * 2;
-            const uint32_t *src = reinterpret_cast<const uint32_t *>(A - sh);
-            uint32_t wv[8];
-#pragma unroll
-            for (int i = 0; i < 6; ++i) wv[i] = __ldg(src + i);
-            wv[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
-            wv[7] = 0u;
+          if (e < seg_end) {
+            rows[h] = rowl[gl][e - eoff[gl]];
+            s2v[h] = s2s[e - r0];
+            const uint4 q0 = *reinterpret_cast<const uint4 *>(rec[e - r0]);
+            const uint4 q1 = *reinterpret_cast<const uint4 *>(rec[e - r0] + 4);
+            const uint32_t wv[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, 0u};
+            const int sh = (int)q1.w;
+            // place the record o = 26 GL % 4 bytes into its window
             if (sh == o) {
 #pragma unroll
               for (int i = 0; i < 7; ++i) win[i] = wv[i];
-            } else if (o == 2) {  // record 4-aligned, window starts 2 bytes before it
+            } else if (o == 2) {
 #pragma unroll
               for (int i = 0; i < 7; ++i) win[i] = __funnelshift_l(i ? wv[i - 1] : 0u, wv[i], 16);
-            } else {  // record starts 2 bytes into a word, window at the record
+            } else {
 #pragma unroll
               for (int i = 0; i < 7; ++i) win[i] = __funnelshift_r(wv[i], wv[i + 1], 16);
             }
@@ -464,33 +551,26 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
             }
           decode_words_compact(w0, w1, lut, h ? aH : aL);
         }
-        uint32_t b[20];
-        const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
-#pragma unroll
-        for (int cp = 0; cp < kCP; ++cp) {
-          uint4 q = make_uint4(0u, 0u, 0u, 0u);
-          if (gq < MB) q = __ldg(reinterpret_cast<const uint4 *>(Bg + ((gq * kCP + cp) * 4 + c) * kBLane));
-          b[4 * cp] = q.x;
-          b[4 * cp + 1] = q.y;
-          b[4 * cp + 2] = q.z;
-          b[4 * cp + 3] = q.w;
-        }
         float d[4];
         group_mma(aL, aH, b, d);
-        const float *cs = P.wsCS + (int64_t)g * (kCSGroup / 4);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (rows[h] < 0) continue;
+          const float cc[2] = {Cv.x, Cv.y};
 #pragma unroll
           for (int i = 0; i < 2; ++i) {
             const int m = 2 * c + i;
-            if (m < MB) atomicAdd(&acc[rows[h]][m], s2v[h] * (d[2 * h + i] - __ldg(cs + m)));
+            if (m < MB) atomicAdd(&acc[rows[h]][m], s2v[h] * (d[2 * h + i] - cc[i]));
           }
         }
+#pragma unroll
+        for (int i = 0; i < 20; ++i) b[i] = bn[i];
+        Cv = Cn;
       }
+      __syncthreads();  // the round's buffers are free again
     }
-    __syncthreads();
   }
+  __syncthreads();
   if (valid) {
     float *y2 = P.wsY2 + (int64_t)n * MB;
     for (int m = 0; m < MB; ++m) y2[m] = acc[t][m];
@@ -517,7 +597,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     return b < 2 ? ar1 + b * kBytesSlot : ar2 + L.oBytes2 + (b - 2) * kBytesSlot;
   };
   Bars *bars = reinterpret_cast<Bars *>(ar1 + kBarOff);
-  float4 *ypart = reinterpret_cast<float4 *>(ar1 + kYPartOff);
   volatile int32_t *abort_ = &bars->abort_;
 
   // ---- one-time set-up: the lane-replicated table, barriers
@@ -538,16 +617,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp < kWarpsP1) {
     // ============================================================ decode
-    // Warps mt and mt + 8 share the 16 rows of m16 tile mt: the first takes
-    // the stage's even groups, the second the odd ones.  Both fetch half of
-    // the rows' bytes and meet at named barrier 1 + mt once per stage.
-    auto body = [&](auto par_c) {
-      constexpr int PAR = decltype(par_c)::value;
-      const int mt = warp & 7;
-      const uint32_t bar_id = 1u + (uint32_t)mt;
+    // Warp mt owns the 16 rows of m16 tile mt and every group of a stage.
+    {
+      const int mt = warp;
       const int g = lane >> 2, c = lane & 3;
       const int R0 = mt * 16 + g, R1 = R0 + 8;
-      const uint32_t tag = kLaneTag | ((uint32_t)lane << 2);
+      const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
       const bool breal = g < MB;  // lanes of absent tokens keep zero B operands
       uint32_t b[20];
 #pragma unroll
@@ -565,22 +640,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         unsigned char *dst = bytes_buf(slot) + mt * 16 * kStageBytes;
         const unsigned char *src = P.plane1 + (int64_t)n0 * RB + (int64_t)a.s * kStageBytes;
         if (nch == kStageBytes / 16) {
-          for (int i = 2 * lane + PAR; i < rows * (kStageBytes / 16); i += 64) {
+          for (int i = lane; i < rows * (kStageBytes / 16); i += 32) {
             const int r = i / (kStageBytes / 16), ch = i - r * (kStageBytes / 16);
             cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
           }
         } else {
-          for (int i = 2 * lane + PAR; i < rows * nch; i += 64) {
+          for (int i = lane; i < rows * nch; i += 32) {
             const int r = i / nch, ch = i - r * nch;
             cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
           }
         }
         const int G = P.K / kGroup, g0 = a.s * kStageG;
         const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
-        const __half *arr = PAR ? P.off : P.s1;  // the even-group warp fetches s1, the other off
-        unsigned char *d = ar2 + L.oSO + slot * kSOSlot + PAR * kRows * 16 + (mt * 16 + lane) * 16;
-        if (lane < rows) {
-          const int64_t o = (int64_t)(n0 + lane) * G + g0;
+        const int rs = lane & 15;  // lanes 0-15 fetch s1, lanes 16-31 off
+        const __half *arr = (lane >> 4) ? P.off : P.s1;
+        unsigned char *d = ar2 + L.oSO + slot * kSOSlot + (lane >> 4) * kRows * 16 + (mt * 16 + rs) * 16;
+        if (rs < rows) {
+          const int64_t o = (int64_t)(n0 + rs) * G + g0;
           if (vec) {
             cp_async16(d, arr + o);
           } else {
@@ -614,8 +690,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         else
           cp_async_wait<2>();
         const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_));
-        // both warps of the pair see each other's copies and take the same decision
-        if (named_bar_any(bar_id, 64, !ok || *abort_ != 0)) break;
+        if (!ok) break;
+        __syncwarp();  // every lane's copies are visible to the warp
         // this lane's ldmatrix row: row (lane % 16) of the m16 tile
         const unsigned char *mrow = bytes_buf(buf) + (mt * 16 + (lane & 15)) * kStageBytes;
         const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
@@ -628,11 +704,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t s1w[2][4] = {{s1a.x, s1a.y, s1a.z, s1a.w}, {s1b.x, s1b.y, s1b.z, s1b.w}};
         const uint32_t ofw[2][4] = {{ofa.x, ofa.y, ofa.z, ofa.w}, {ofb.x, ofb.y, ofb.z, ofb.w}};
         const int gs = w.gs;
+        // s1 / off / C / S of group GL applied to its accumulators d
+        auto epilogue = [&](auto glc, const float *d) {
+          constexpr int GL = decltype(glc)::value;
+          const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
+          const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
 #pragma unroll
-        for (int GL = PAR; GL < kStageG; GL += 2) {
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
+            const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
+            const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+            y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
+            y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
+          }
+        };
+        // Software pipeline over the stage's groups: the MMAs of group GL run
+        // while group GL + 1 is decoded; GL's epilogue comes after that.
+        float dp[4] = {0.f, 0.f, 0.f, 0.f};
+        auto group = [&](auto glc) {
+          constexpr int GL = decltype(glc)::value;
           if (GL < gs) {
             // the group's 16-byte chunks of rows R0 / R1 (2 or 3), one ldmatrix
-            const int k0 = win_start(GL) / 4, kl = (win_start(GL) + 6) / 4, sft = win_start(GL) % 4;
+            constexpr int k0 = win_start(GL) / 4, kl = (win_start(GL) + 6) / 4, sft = win_start(GL) % 4;
             uint32_t x0[3], x1[3];
             ldsm_x4(mrow + 16 * (lane < 16 ? k0 : k0 + 1), x0[0], x1[0], x0[1], x1[1]);
             if (kl == k0 + 2) {
@@ -646,45 +739,49 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t aL[20], aH[20];
             decode_words(up ? x0[1] : x0[0], up ? x0[2] : x0[1], tag, aL);
             decode_words(up ? x1[1] : x1[0], up ? x1[2] : x1[1], tag, aH);
-            if (breal) {
-              const unsigned char *bsrc = Bst + GL * kBTok * MB + g * kBTok + c * kBLane;
+            {
+              // lanes of absent tokens keep their zero operands (predicated, no branch)
+              const uint32_t bsrc = smem_u32(Bst + GL * kBTok * MB + g * kBTok + c * kBLane);
 #pragma unroll
-              for (int cp = 0; cp < kCP; ++cp) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(bsrc + cp * 4 * kBLane);
-                b[4 * cp] = v.x;
-                b[4 * cp + 1] = v.y;
-                b[4 * cp + 2] = v.z;
-                b[4 * cp + 3] = v.w;
-              }
+              for (int cp = 0; cp < kCP; ++cp)
+                asm volatile(
+                    "{\n.reg .pred p;\nsetp.ne.b32 p, %5, 0;\n@p ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];\n}"
+                    : "+r"(b[4 * cp]), "+r"(b[4 * cp + 1]), "+r"(b[4 * cp + 2]), "+r"(b[4 * cp + 3])
+                    : "r"(bsrc + cp * 4 * kBLane), "r"((uint32_t)breal));
             }
             float d[4];
             group_mma(aL, aH, b, d);
-            const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
-            const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
+            if constexpr (GL >= 1) epilogue(std::integral_constant<int, GL - 1>{}, dp);
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
-              const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
-              const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
-              y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
-              y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
-            }
+            for (int i = 0; i < 4; ++i) dp[i] = d[i];
           }
-        }
+        };
+        group(std::integral_constant<int, 0>{});
+        group(std::integral_constant<int, 1>{});
+        group(std::integral_constant<int, 2>{});
+        group(std::integral_constant<int, 3>{});
+        group(std::integral_constant<int, 4>{});
+        group(std::integral_constant<int, 5>{});
+        group(std::integral_constant<int, 6>{});
+        group(std::integral_constant<int, 7>{});
+        // the epilogue of the stage's last group
+        auto last = [&](auto glc) {
+          constexpr int GL = decltype(glc)::value;
+          if (GL < gs && GL + 1 >= gs) epilogue(glc, dp);
+        };
+        last(std::integral_constant<int, 0>{});
+        last(std::integral_constant<int, 1>{});
+        last(std::integral_constant<int, 2>{});
+        last(std::integral_constant<int, 3>{});
+        last(std::integral_constant<int, 4>{});
+        last(std::integral_constant<int, 5>{});
+        last(std::integral_constant<int, 6>{});
+        last(std::integral_constant<int, 7>{});
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->empty[buf]);
         if (w.last_stage()) {
-          // the odd-group warp hands its partial sums to the even-group warp,
-          // which adds the second plane and writes y
-          float4 *yp = ypart + mt * 32 + lane;
-          if (PAR == 1) *yp = make_float4(y[0], y[1], y[2], y[3]);
-          named_bar(bar_id, 64);
-          if (PAR == 0) {
-            const float4 o = *yp;
-            y[0] += o.x;
-            y[1] += o.y;
-            y[2] += o.z;
-            y[3] += o.w;
+          // add the second plane and write y
+          {
             const Problem &P = w.P();
             const int nb = (w.tile - P.tile_begin) * kRows;
 #pragma unroll
@@ -710,11 +807,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = 0; i < 4; ++i) y[i] = 0.f;
         }
       }
-    };
-    if (warp >= 8)
-      body(std::integral_constant<int, 1>{});
-    else
-      body(std::integral_constant<int, 0>{});
+    }
     cp_async_wait<0>();  // nothing in flight into shared memory at exit
   } else if (warp == kWarpProd) {
     // ========================================================== producer

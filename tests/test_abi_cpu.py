@@ -54,8 +54,8 @@ def test_host_side_argument_errors_without_gpu():
     assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) == 28672
     assert tq.tq_workspace_bytes(5, 100, 1024) == mma(5, 100, 1024)
     # 8 < M <= 16: tensor-memory path (2 x 2560 B of slots + 128 B C/S per group);
-    # larger M runs in chunks of 16 and may end on a chunk of <= 8 tokens
-    assert tq.tq_workspace_bytes(16, 4096, 4096) == max(32 * (5120 + 128), mma(8, 4096, 4096))
-    assert tq.tq_workspace_bytes(40, 64, 4096) == max(32 * (5120 + 128), mma(8, 64, 4096))
+    # M > 16: the prefill tile path needs no workspace (256 bytes are asked for)
+    assert tq.tq_workspace_bytes(16, 4096, 4096) == 32 * (5120 + 128)
+    assert tq.tq_workspace_bytes(40, 64, 4096) == 256
     assert tq.tq_workspace_bytes(1, 4096, 100) == 0
     assert tq.tq_workspace_bytes(1, 0, 4096) == 0

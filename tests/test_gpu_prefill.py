@@ -1,0 +1,52 @@
+"""GPU parity of the prefill tile path (M > 16 tokens: weight tiles
+dequantized to fp16 and multiplied on the tensor cores) against the fp64 CPU
+oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element.  The full-size case
+is the Qwen3-8B prefill shape (M = 2048 tokens) checked on sampled rows."""
+import numpy as np
+import pytest
+import torch
+
+import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def H():
+    import gpu_helpers
+    return gpu_helpers
+
+
+@pytest.mark.parametrize("M,N,K,frac,f32", [
+    (17, 512, 1024, 0.0, False),    # barely past the decode path, one ragged token tile
+    (129, 256, 1024, 0.1, True),    # two token tiles, the second with one token
+    (200, 300, 4224, 0.1, False),   # odd group count, ragged rows and tokens
+    (256, 520, 2560, 1.0, False),   # every group salient
+    (64, 1, 128, 0.5, True),        # one row, one group
+])
+def test_prefill_small(H, M, N, K, frac, f32):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, frac, config=4, proj=(M * 7 + N) % 97)
+    xb = wl.gen_x(M, K, config=4, proj=(M * 7 + N) % 97)
+    y_ref, a_ref = H.oracle_ref(w, xb)
+    pw = H.pack_on_gpu(w)
+    x = H.dev(xb)
+    y = (tq.tq_linear_f32out(x, pw) if f32 else tq.tq_linear(x, pw)).float().cpu().numpy()
+    H.device_status_ok()
+    H.assert_close(y, y_ref, a_ref)
+
+
+@pytest.mark.parametrize("name,N,K,nrows", [("k", 1024, 4096, 48), ("down", 4096, 12288, 24)])
+def test_prefill_qwen3_8b_shape_sampled_rows(H, name, N, K, nrows):
+    """M = 2048 tokens through one Qwen3-8B projection shape; the oracle
+    checks a seeded sample of rows (every token) across all row tiles."""
+    from paper_2609_09240_gb300 import tq
+    M = 2048
+    w = wl.gen_weights(N, K, 0.1, config=4, layer=0, proj=3 if name == "k" else 6)
+    xb = wl.gen_x(M, K, config=4, layer=0, proj=3 if name == "k" else 6)
+    pw = H.pack_on_gpu(w)
+    y = tq.tq_linear(H.dev(xb), pw).float().cpu().numpy()
+    H.device_status_ok()
+    rows = np.sort(np.random.default_rng(4).choice(N, size=nrows, replace=False)).astype(np.int32)
+    y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
+    H.assert_close(y[:, rows], y_ref, a_ref)

@@ -21,10 +21,10 @@ def H():
 def test_oversize_call_is_rejected_without_gpu():
     from paper_2609_09240_gb300 import tq
     L = tq.lib()
-    # M = 8, N = 1 Mi rows needs far more than the 1 MiB scratch; rejected
+    # K = 512 Ki inputs needs far more than the 1 MiB scratch; rejected
     # before any pointer is looked at or any CUDA call is made
-    assert tq.tq_workspace_bytes(8, 1 << 20, 4096) > tq.STATIC_SCRATCH_BYTES
-    assert L.tq_linear_static(8, 1 << 20, 4096, None, None, None, None) == -9
+    assert tq.tq_workspace_bytes(8, 64, 1 << 19) > tq.STATIC_SCRATCH_BYTES
+    assert L.tq_linear_static(8, 64, 1 << 19, None, None, None, None) == -9
     assert L.tq_linear_static(0, 64, 4096, None, None, None, None) == -2
     assert b"SCRATCH" in L.tq_status_str(-9)
 
