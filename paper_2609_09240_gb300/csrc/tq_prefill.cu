@@ -104,20 +104,6 @@ __device__ __forceinline__ void decode_weights(const uint32_t *rw, uint32_t v01,
   }
 }
 
-// The 26-byte record j of plane 2 as 7 words (plane 2 is 16-byte aligned).
-__device__ __forceinline__ void load_record(const uint8_t *plane2, int64_t j, uint32_t *rw) {
-  const int64_t off0 = j * kGroupBytes;
-  const int sh = (int)(off0 & 3);
-  const uint32_t *src = reinterpret_cast<const uint32_t *>(plane2 + off0 - sh);
-  uint32_t r8[8];
-#pragma unroll
-  for (int i = 0; i < 6; ++i) r8[i] = __ldg(src + i);
-  r8[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
-  r8[7] = 0u;
-#pragma unroll
-  for (int i = 0; i < 7; ++i) rw[i] = sh ? __funnelshift_r(r8[i], r8[i + 1], 16) : r8[i];
-}
-
 // Core-matrix offset of (row, K element e) in a tile of 8-row groups x 16
 // core matrices along K.
 __device__ __forceinline__ int cm_off(int row, int e) { return ((row >> 3) * 16 + (e >> 3)) * 128 + (row & 7) * 16; }
@@ -158,36 +144,47 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
     // its 26 bytes, s1, off, whether it is salient and then its plane-2
     // record and s2.
     struct Next {
-      uint32_t rw[7], rec[7];
-      float s1, of, s2;
-      bool salient;
+      uint32_t r8[7], q8[7];  // raw aligned words of the group and of its record
+      unsigned short s1, of, s2;
+      bool odd, rodd, salient;
     };
     int64_t j = (valid && P.nnz > 0) ? P.rowptr[n] : 0;  // record index of the row's next salient group
     uint32_t salw = (valid && P.nnz > 0) ? __ldg(salrow) : 0u;
+    // issues the loads only: nothing here waits for them (they are used one
+    // group later)
     auto fetch = [&](int g, Next &nx) {
       // plane-1 rows are 16-byte aligned and groups are 26 bytes, so group g
       // starts 0 or 2 bytes into a word; 7 aligned words cover it
-      const int sh = (g & 1) ? 2 : 0;
-      const uint32_t *src = reinterpret_cast<const uint32_t *>(row + (int64_t)g * kGroupBytes - sh);
-      uint32_t r8[8];
+      nx.odd = g & 1;
+      const uint32_t *src = reinterpret_cast<const uint32_t *>(row + (int64_t)g * kGroupBytes - (nx.odd ? 2 : 0));
 #pragma unroll
-      for (int i = 0; i < 7; ++i) r8[i] = valid ? __ldg(src + i) : 0x79797979u;  // 121: all-zero trits
-      r8[7] = 0u;
-#pragma unroll
-      for (int i = 0; i < 7; ++i) nx.rw[i] = sh ? __funnelshift_r(r8[i], r8[i + 1], 16) : r8[i];
-      nx.s1 = valid ? __half2float(P.s1[(int64_t)n * G + g]) : 0.f;
-      nx.of = valid ? __half2float(P.off[(int64_t)n * G + g]) : 0.f;
+      for (int i = 0; i < 7; ++i) nx.r8[i] = valid ? __ldg(src + i) : 0x79797979u;  // 121: all-zero trits
+      const unsigned short *s1h = reinterpret_cast<const unsigned short *>(P.s1);
+      const unsigned short *ofh = reinterpret_cast<const unsigned short *>(P.off);
+      nx.s1 = valid ? __ldg(s1h + (int64_t)n * G + g) : (unsigned short)0;
+      nx.of = valid ? __ldg(ofh + (int64_t)n * G + g) : (unsigned short)0;
       if ((g & 31) == 0 && g > 0 && valid && P.nnz > 0) salw = __ldg(salrow + (g >> 5));
       nx.salient = (salw >> (g & 31)) & 1u;
-      nx.s2 = 0.f;
+      nx.s2 = 0;
+      nx.rodd = false;
 #pragma unroll
-      for (int i = 0; i < 7; ++i) nx.rec[i] = 0x79797979u;
+      for (int i = 0; i < 7; ++i) nx.q8[i] = 0x79797979u;
       if (nx.salient) {
         const int64_t jj = j < P.nnz ? j : P.nnz - 1;
-        load_record(P.plane2, jj, nx.rec);
-        nx.s2 = __half2float(P.s2[jj]);
+        const int64_t off0 = jj * kGroupBytes;
+        nx.rodd = (off0 & 3) != 0;  // plane 2 is 16-byte aligned: records start 0 or 2 bytes into a word
+        const uint32_t *rs = reinterpret_cast<const uint32_t *>(P.plane2 + off0 - (nx.rodd ? 2 : 0));
+#pragma unroll
+        for (int i = 0; i < 6; ++i) nx.q8[i] = __ldg(rs + i);
+        nx.q8[6] = nx.rodd ? __ldg(rs + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(rs + 6));
+        nx.s2 = __ldg(reinterpret_cast<const unsigned short *>(P.s2) + jj);
         ++j;
       }
+    };
+    // the 7 words of a 26-byte run, byte 0 first, from its raw aligned words
+    auto realign = [](const uint32_t *r8, bool odd, uint32_t *rw) {
+#pragma unroll
+      for (int i = 0; i < 7; ++i) rw[i] = odd ? __funnelshift_r(r8[i], i < 6 ? r8[i + 1] : 0u, 16) : r8[i];
     };
     Next nx;
     fetch(0, nx);
@@ -213,21 +210,25 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
       asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&bars->full[s])) : "memory");
       const Next cur = nx;
       if (g + 1 < G) fetch(g + 1, nx);
-      const float s1 = cur.s1, of = cur.of;
+      const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
       const bool salient = cur.salient;
+      uint32_t rw[7];
+      realign(cur.r8, cur.odd, rw);
       const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
       const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
       const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
       uint32_t wv[64];
-      decode_weights(cur.rw, v01, v22, sel, wv);
+      decode_weights(rw, v01, v22, sel, wv);
       if (__any_sync(0xffffffffu, salient)) {
         // second plane: + s2 t2 on salient groups (other rows add zeros)
-        const float s2 = cur.s2;
+        const float s2 = __half2float(__ushort_as_half(cur.s2));
+        uint32_t rec[7];
+        realign(cur.q8, cur.rodd, rec);
         const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
         const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
         const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
         uint32_t w2[64];
-        decode_weights(cur.rec, u01, u22, sel, w2);
+        decode_weights(rec, u01, u22, sel, w2);
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
           const __half2 a = *reinterpret_cast<const __half2 *>(&wv[i]);
