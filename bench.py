@@ -7,10 +7,13 @@ One step = one pass over all 252 projections (tq_linear_batched: one kernel
 launch).  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tq|reference]
+  python bench.py --prefill      (one Qwen3-8B layer at M = 2048 tokens)
 
 --impl reference times the CPU oracle on the host cores (the reference arm
 of this project: a plain fp64 implementation of the same layer) on a
-bounded sample of the same workload.
+bounded sample of the same workload.  --prefill measures the prefill tile
+path (tensor-core bound) and times dense fp16 cuBLAS on the same shapes as
+context.
 """
 from __future__ import annotations
 
@@ -38,6 +41,17 @@ def measured_peaks():
             d = json.load(f)
         return float(d["hbm_gbs"]), "measured"
     return HBM_FALLBACK_GBS, "fallback"
+
+
+def measured_tensor_peak():
+    """fp16 dense tensor peak (TFLOP/s): the measured sustained bf16 cuBLAS
+    rate (fp16 and bf16 share the nominal rate), else the fallback."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured sustained bf16 (= fp16 rate)"
+    return 1700.0, "fallback sustained"
 
 
 def dist_env():
@@ -218,6 +232,85 @@ def cpu_baseline(budget_s):
     return nbytes / t / 1e9, L.cores, desc, t
 
 
+# ------------------------------------------------------------------- prefill
+def run_prefill(args, ws, rank, local):
+    """One Qwen3-8B layer (its seven projections) at M = 2048 tokens through
+    the prefill tile path, one tq_linear per projection; dense fp16 cuBLAS on
+    the same shapes is timed beside it as context."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    M = 2048
+    items, flops, packed = [], 0, 0
+    for p in wl.config_projections(4):
+        g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 500 + p.proj)
+        pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+        del g
+        x = wl.gen_x_torch(M, p.K, dev, 600 + p.proj)
+        y = torch.empty((M, p.N), dtype=torch.float16, device=dev)
+        wsb = tq.workspace(tq.tq_workspace_bytes(M, p.N, p.K), dev)
+        items.append((pw, x, y, wsb))
+        flops += 2 * M * p.N * p.K
+        packed += pw.packed_bytes()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for pw, x, y, wsb in items:
+            tq.tq_linear(x, pw, y=y, ws=wsb, stream=stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, 20))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        e0.record(stream)
+        for _ in range(steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    # context: dense fp16 matmul (cuBLAS) with a dense W of the same shapes
+    dense = [torch.randn((pw.N, pw.K), device=dev, dtype=torch.float16) for pw, _, _, _ in items]
+
+    def dstep():
+        for (pw, x, y, _), W in zip(items, dense):
+            torch.matmul(x, W.t(), out=y)
+
+    for _ in range(3):
+        dstep()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(steps):
+        dstep()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms_dense = e0.elapsed_time(e1) / steps
+    peak, kind = measured_tensor_peak()
+    tflops = flops / (ms * 1e-3) / 1e12
+    out = {
+        "metric": "Qwen3-8B W1.58A16 prefill: TFLOP/s of one layer at M=2048", "value": tflops,
+        "unit": "TFLOP/s", "n_gpus": 1, "steps": steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "config": {"workload": "qwen3-8b prefill, one layer's 7 projections, M=2048 tokens",
+                   "flops_per_step": flops, "packed_bytes_per_step": packed,
+                   "l2": "no flush: 2048-token activations and outputs of a layer exceed L2 per step"},
+        "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
+                     "peak_kind": kind, "traffic": None,
+                     "kernel": "prefill tile kernel (one launch per projection, 7 per step)"},
+        "dense_fp16_cublas": {"ms_per_step": ms_dense, "tflops": flops / (ms_dense * 1e-3) / 1e12},
+        "gpu_launches": 7 * steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    return 0
+
+
 # ------------------------------------------------------------------- main
 def run_reference(args, ws, rank):
     """The oracle timed on the host cores: each step is one pass over a
@@ -263,10 +356,13 @@ def main():
     ap.add_argument("--M", type=int, default=1, help="tokens per step (1 = batch-1 decode)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="profile a smaller step (first L layers)")
+    ap.add_argument("--prefill", action="store_true", help="one Qwen3-8B layer at M = 2048 tokens")
     args = ap.parse_args()
     ws, rank, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, ws, rank)
+    if args.prefill:
+        return run_prefill(args, ws, rank, local)
 
     import torch
 
@@ -285,6 +381,8 @@ def main():
     items, x_all, y_all, packed_bytes, n_weights = build_step(args.M, dev, seed0=0, layers=args.layers)
     batch = tq.Batch(args.M, items)
     stream = torch.cuda.current_stream()
+    # activation prep, second plane (when any projection has one), first plane
+    launches_per_step = 3 if any(pw.nnz > 0 for pw, _, _ in items) else 2
 
     def step():
         tq.tq_linear_batched(batch, stream)
@@ -367,11 +465,13 @@ def main():
         "frac_of_8TBps_nominal": value / ws / 8000.0,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
-                     "traffic": ncu_traffic(), "kernel": "tq decode kernel (one launch per step)",
+                     "traffic": ncu_traffic(),
+                     "kernel": "decode step: activation prep + second plane + first plane "
+                               "(3 launches per step, timed together; the first-plane kernel is ~70 % of it)",
                      "launch_ms_avg": launch_avg},
         "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * launches_per_step,
         "clocks": clk.summary(),
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
