@@ -24,22 +24,24 @@
 // from gemv_mma_prep_kernel into the caller's workspace.
 //
 // Fragment layout.  In an m16n8k16 MMA, lane (g, c) (g = lane / 4,
-// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  The
-// packed rows reach the registers by ldmatrix, which gives lane c word c of
-// every 16-byte chunk; so lane c of a row decodes two whole words of the
-// group's window (the aligned words covering its 26 bytes): 8 bytes, whose
-// 20 A words (W, W' of each byte, then 4 V words) feed the group's 10 MMAs,
-// chunk j taking words 2j and 2j + 1.  Window bytes outside the group get
-// zero activations, so every lane runs the same code.  The prep kernel
+// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  Lane c
+// of a row decodes the two words of the group's window (the aligned words
+// covering its 26 bytes) whose index is c mod 4, loaded straight from the
+// stage row in shared memory (the 32 lanes hit 32 different banks): 8 bytes,
+// whose 20 A words (W, W' of each byte, then 4 V words) feed the group's 10
+// MMAs, chunk j taking words 2j and 2j + 1.  Window bytes outside the group
+// get zero activations, so every lane runs the same code.  The prep kernel
 // writes B (the activation slots) in exactly this order for each of the 8
 // positions a group can take in its stage.
 //
 // Kernels (one step = three launches):
 //  * gemv_mma_prep_kernel: B fragments, C and S per (problem, group, token);
-//  * gemv_mma_p2_kernel: the second plane.  One CTA per 128-row tile
+//  * the second plane, s2 * P2 per row into the workspace (y2, fp32):
+//    gemv_mma_p2_one_kernel for one token (a thread per record on the CUDA
+//    cores), gemv_mma_p2_kernel for 2..8 tokens (one CTA per 128-row tile
 //    compacts the tile's salient (row, group) pairs per group, decodes their
 //    records with the same encoding and runs m16n8k16 MMAs over 16 records
-//    at a time; s2 * P2 per row goes to the workspace (y2, fp32);
+//    at a time);
 //  * gemv_mma_kernel (one persistent CTA per SM over a cost-balanced range
 //    of 128-row tiles, 8-group stages): warps 0..7 each own 16 rows of the
 //    tile, fetch those rows' packed bytes and s1 / off with 16-byte
@@ -157,8 +159,7 @@ __device__ __forceinline__ uint32_t w_prime(uint32_t w) {
 // group's index in its stage); the group starts o = 26 GL % 4 bytes into
 // the first.  Lane c of a row owns the window words whose stage-row index
 // is c mod 4 (two words: the first at or after wstart, and the one four
-// words later; bytes outside the group get zero activations), which is how
-// ldmatrix hands out 16-byte rows: lane c receives word c of each.
+// words later; bytes outside the group get zero activations).
 __host__ __device__ constexpr int win_start(int GL) { return (26 * GL) / 4; }
 // Stage-row word index of lane c's first window word.
 __host__ __device__ constexpr int first_word(int GL, int c) {
@@ -206,21 +207,6 @@ __device__ __forceinline__ void decode_words_compact(uint32_t w0, uint32_t w1, c
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) a[16 + i] = 0x44004400u | v[2 * i] | (v[2 * i + 1] << 16);
-}
-
-// ldmatrix: four (x4) or two (x2) 8 x 16-byte rows; lane (g, c) receives
-// word c of row g of each.
-__device__ __forceinline__ void ldsm_x4(const void *p, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(smem_u32(p))
-               : "memory");
-}
-__device__ __forceinline__ void ldsm_x2(const void *p, uint32_t &r0, uint32_t &r1) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];"
-               : "=r"(r0), "=r"(r1)
-               : "r"(smem_u32(p))
-               : "memory");
 }
 
 // 16-byte asynchronous global -> shared copies (completion tracked per
@@ -577,6 +563,151 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
   }
 }
 
+// Second plane for a single token (M = 1) on the CUDA cores, one thread per
+// record, persistent over the main kernel's tile ranges.  A span of up to
+// kP1SpanRows consecutive rows of one problem owns one contiguous range of
+// plane-2 records; a record's row is a binary search over the span's rowptr
+// and its group the rank-th set bit of that row's salience words.  Each of
+// the record's four lane positions is decoded into the same five-slot words
+// as the first plane (same lane-replicated table at the same address) and
+// dotted with that position's activation words of the group, staged in
+// shared memory per problem, by fp16 x fp16 -> fp32 fused multiply-adds.
+// s2 * (dot - C) per row accumulates in shared memory and goes to y2.
+constexpr int kP1Threads = 512;
+constexpr int kP1SpanRows = 1024;
+constexpr int kP1ActStride = 84;  // words per group: 4 lane positions x 20, padded for the banks
+constexpr int kP1MaxG = (kDynBytes - kArena1 - kLutBytes) / (kP1ActStride * 4);
+
+__host__ __device__ constexpr int p1_dyn_bytes(int G) { return kArena1 + kLutBytes + G * kP1ActStride * 4; }
+static_assert((2 * kP1SpanRows + 1 + kP1MaxG + kP1SpanRows * ((kP1MaxG + 31) / 32)) * 4 <= kArena1,
+              "plane-2 span arrays overflow the region below the table");
+
+// d + lo(a) lo(b) + hi(a) hi(b), fp16 operands, fp32 accumulation
+__device__ __forceinline__ float fma_h2(uint32_t a, uint32_t b, float d) {
+  float r;
+  asm("{ .reg .f16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\t"
+      "mov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.f16 %0, al, bl, %3;\n\t"
+      "fma.rn.f32.f16 %0, ah, bh, %0; }"
+      : "=f"(r)
+      : "r"(a), "r"(b), "f"(d));
+  return r;
+}
+
+__global__ void __launch_bounds__(kP1Threads, 1)
+    gemv_mma_p2_one_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
+  extern __shared__ __align__(1024) unsigned char dyn[];
+  const int t = threadIdx.x, lane = t & 31;
+  if (smem_u32(dyn) != kDynShared) {
+    if (t == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  int *rp = reinterpret_cast<int *>(dyn);                     // [kP1SpanRows + 1]
+  float *acc = reinterpret_cast<float *>(rp + kP1SpanRows + 1);  // [kP1SpanRows]
+  float *cg = acc + kP1SpanRows;                              // [kP1MaxG]
+  uint32_t *sw = reinterpret_cast<uint32_t *>(cg + kP1MaxG);  // [span rows][W]
+  uint32_t *act = reinterpret_cast<uint32_t *>(dyn + kArena1 + kLutBytes);
+  {
+    uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
+    for (int i = t; i < 256 * 32; i += kP1Threads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+  }
+  const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
+  const int t1 = sc.cta_tile[blockIdx.x + 1];
+  int tile = sc.cta_tile[blockIdx.x], q = 0, staged = -1;
+  while (tile < t1) {
+    while (q + 1 < bp.count && bp.prob[q + 1].tile_begin <= tile) ++q;
+    const Problem &P = bp.prob[q];
+    const int tend = min(min(t1, P.tile_begin + (P.N + kRows - 1) / kRows), tile + kP1SpanRows / kRows);
+    const int n0 = (tile - P.tile_begin) * kRows, n1 = min(P.N, (tend - P.tile_begin) * kRows);
+    tile = tend;
+    if (P.nnz <= 0) continue;  // the main kernel adds no y2 for this problem
+    const int G = P.K / kGroup, W = sal_words_of(P.K), rows = n1 - n0;
+    __syncthreads();  // the previous span's arrays are free
+    if (q != staged) {
+      staged = q;
+      for (int i = t; i < G * 20; i += kP1Threads) {
+        const int g = i / 20, r = i - g * 20, c = r / 5, cp = r - c * 5;
+        *reinterpret_cast<uint4 *>(act + g * kP1ActStride + c * 20 + cp * 4) =
+            __ldg(reinterpret_cast<const uint4 *>(P.wsB + (int64_t)g * kBTok + (cp * 4 + c) * kBLane));
+      }
+      for (int g = t; g < G; g += kP1Threads) cg[g] = P.wsCS[(int64_t)g * (kCSGroup / 4)];
+    }
+    for (int i = t; i <= rows; i += kP1Threads) rp[i] = P.rowptr[n0 + i];
+    for (int i = t; i < rows * W; i += kP1Threads) {
+      const int w = i % W, gw = G - 32 * w;
+      const uint32_t bits = P.sal[(int64_t)n0 * W + i];
+      sw[i] = gw < 32 ? bits & ((1u << gw) - 1u) : bits;
+    }
+    for (int i = t; i < rows; i += kP1Threads) acc[i] = 0.f;
+    __syncthreads();
+    const int J0 = max(rp[0], 0), J1 = min(rp[rows], P.nnz);
+    for (int j = J0 + t; j < J1; j += kP1Threads) {
+      int r = 0;  // the record's row in the span: the last r with rp[r] <= j
+#pragma unroll
+      for (int step = kP1SpanRows / 2; step >= 1; step >>= 1)
+        if (r + step < rows && rp[r + step] <= j) r += step;
+      int rank = j - rp[r], g = 0;
+      for (int w = 0; w < W; ++w) {
+        const uint32_t word = sw[r * W + w];
+        const int cnt = __popc(word);
+        if (rank < cnt) {
+          g = 32 * w + (int)__fns(word, 0u, rank + 1);
+          break;
+        }
+        rank -= cnt;
+      }
+      const int GL = g % kStageG;
+      // the record's 26 bytes, placed o = 26 GL % 4 bytes into its window
+      const int64_t off0 = (int64_t)j * kGroupBytes;
+      const int sh = (int)(j & 1) * 2;  // plane 2 is 16-byte aligned: the record starts 0 or 2 bytes into a word
+      const uint32_t *src = reinterpret_cast<const uint32_t *>(P.plane2 + off0 - sh);
+      uint32_t wv[8];
+#pragma unroll
+      for (int i = 0; i < 6; ++i) wv[i] = __ldg(src + i);
+      // bytes 24, 25 only when the record is word-aligned: the word after them may lie past the end of plane 2
+      wv[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
+      wv[7] = 0u;
+      const float s2 = __half2float(P.s2[j]);
+      const int o = (GL & 1) * 2;
+      uint32_t win[8];
+      if (o == sh) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) win[i] = wv[i];
+      } else if (o == 2) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) win[i] = __funnelshift_l(i ? wv[i - 1] : 0u, wv[i], 16);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) win[i] = __funnelshift_r(wv[i], i < 7 ? wv[i + 1] : 0u, 16);
+      }
+      // window word i belongs to lane position c = (win_start + i) mod 4
+      const int ws = win_start(GL);
+      const uint32_t *ag = act + g * kP1ActStride;
+      float d[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        uint32_t a[20];
+        decode_words(win[i], win[i + 4], tag, a);
+        const uint4 *bq = reinterpret_cast<const uint4 *>(ag + ((ws + i) & 3) * 20);
+        float e = 0.f;
+#pragma unroll
+        for (int cp = 0; cp < kCP; ++cp) {
+          const uint4 b = bq[cp];
+          e = fma_h2(a[4 * cp], b.x, e);
+          e = fma_h2(a[4 * cp + 1], b.y, e);
+          e = fma_h2(a[4 * cp + 2], b.z, e);
+          e = fma_h2(a[4 * cp + 3], b.w, e);
+        }
+        d[i] = e;
+      }
+      atomicAdd(&acc[r], s2 * (((d[0] + d[1]) + (d[2] + d[3])) - cg[g]));
+    }
+    __syncthreads();
+    for (int i = t; i < rows; i += kP1Threads) P.wsY2[n0 + i] = acc[i];
+  }
+}
+
 // ------------------------------------------------------------------ main
 template <bool F32>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -623,10 +754,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int g = lane >> 2, c = lane & 3;
       const int R0 = mt * 16 + g, R1 = R0 + 8;
       const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
-      const bool breal = g < MB;  // lanes of absent tokens keep zero B operands
       uint32_t b[20];
-#pragma unroll
-      for (int i = 0; i < 20; ++i) b[i] = 0u;
       float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
       // The tile's 16 rows of a stage (packed bytes, s1 and off), fetched with
       // 16-byte asynchronous copies NS - 1 stages ahead; one commit group per
@@ -639,7 +767,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nch = (a.gs * kGroupBytes + 15) / 16;  // 16-byte chunks per row
         unsigned char *dst = bytes_buf(slot) + mt * 16 * kStageBytes;
         const unsigned char *src = P.plane1 + (int64_t)n0 * RB + (int64_t)a.s * kStageBytes;
-        if (nch == kStageBytes / 16) {
+        if (nch == kStageBytes / 16 && rows == 16) {
+          // 208 chunks; lane takes chunk i = lane + 32 k, i.e. row r = i / 13,
+          // chunk ch = i % 13, advanced incrementally (32 = 2 x 13 + 6)
+          static_assert(kStageBytes == 13 * 16, "a stage row is 13 chunks");
+          const int r = lane / 13, ch0 = lane - 13 * r;
+          int ch = ch0;
+          unsigned char *dptr = dst + r * kStageBytes + 16 * ch0;
+          const unsigned char *sptr = src + r * RB + 16 * ch0;
+#pragma unroll
+          for (int k = 0; k < 7; ++k) {
+            if (k < 6 || lane < 16) cp_async16(dptr, sptr);
+            ch += 6;
+            dptr += 2 * kStageBytes + 96;
+            sptr += 2 * RB + 96;
+            if (ch >= 13) {  // one more row, 13 chunks back: the slot's rows are contiguous
+              ch -= 13;
+              sptr += RB - kStageBytes;
+            }
+          }
+        } else if (nch == kStageBytes / 16) {
           for (int i = lane; i < rows * (kStageBytes / 16); i += 32) {
             const int r = i / (kStageBytes / 16), ch = i - r * (kStageBytes / 16);
             cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
@@ -692,9 +839,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_));
         if (!ok) break;
         __syncwarp();  // every lane's copies are visible to the warp
-        // this lane's ldmatrix row: row (lane % 16) of the m16 tile
-        const unsigned char *mrow = bytes_buf(buf) + (mt * 16 + (lane & 15)) * kStageBytes;
         const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
+        // this lane's B words (lanes of absent tokens load the last token's:
+        // their output columns are never written)
+        const unsigned char *Bl = Bst + min(g, MB - 1) * kBTok + c * kBLane;
         const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * kCSSlot);
         const unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
         const uint4 s1a = *reinterpret_cast<const uint4 *>(SO + R0 * 16);
@@ -721,33 +869,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Software pipeline over the stage's groups: the MMAs of group GL run
         // while group GL + 1 is decoded; GL's epilogue comes after that.
         float dp[4] = {0.f, 0.f, 0.f, 0.f};
-        auto group = [&](auto glc) {
+        // lane (g, c)'s window words of a group at shift k = win_start % 4:
+        // stage-row words win_start + ((c - k) & 3) (+ 4) of rows R0, R1
+        const unsigned char *rowp = bytes_buf(buf) + R0 * kStageBytes;
+        const unsigned char *wb[4] = {rowp + 4 * (c & 3), rowp + 4 * ((c - 1) & 3), rowp + 4 * ((c - 2) & 3),
+                                      rowp + 4 * ((c - 3) & 3)};
+        auto group = [&](auto glc, auto fullc) {
           constexpr int GL = decltype(glc)::value;
-          if (GL < gs) {
-            // the group's 16-byte chunks of rows R0 / R1 (2 or 3), one ldmatrix
-            constexpr int k0 = win_start(GL) / 4, kl = (win_start(GL) + 6) / 4, sft = win_start(GL) % 4;
-            uint32_t x0[3], x1[3];
-            ldsm_x4(mrow + 16 * (lane < 16 ? k0 : k0 + 1), x0[0], x1[0], x0[1], x1[1]);
-            if (kl == k0 + 2) {
-              ldsm_x2(mrow + 16 * (k0 + 2), x0[2], x1[2]);
-            } else {
-              x0[2] = x0[1];
-              x1[2] = x1[1];
-            }
-            // lane c's two words: chunks k0, k0 + 1, or k0 + 1, k0 + 2 when c < wstart % 4
-            const bool up = c < sft;
+          constexpr bool FULL = decltype(fullc)::value;
+          if (FULL || GL < gs) {
+            constexpr int ws = win_start(GL);
+            const unsigned char *src = wb[ws % 4] + 4 * ws;
+            const uint32_t x00 = *reinterpret_cast<const uint32_t *>(src);
+            const uint32_t x01 = *reinterpret_cast<const uint32_t *>(src + 16);
+            const uint32_t x10 = *reinterpret_cast<const uint32_t *>(src + 8 * kStageBytes);
+            const uint32_t x11 = *reinterpret_cast<const uint32_t *>(src + 8 * kStageBytes + 16);
             uint32_t aL[20], aH[20];
-            decode_words(up ? x0[1] : x0[0], up ? x0[2] : x0[1], tag, aL);
-            decode_words(up ? x1[1] : x1[0], up ? x1[2] : x1[1], tag, aH);
+            decode_words(x00, x01, tag, aL);
+            decode_words(x10, x11, tag, aH);
             {
-              // lanes of absent tokens keep their zero operands (predicated, no branch)
-              const uint32_t bsrc = smem_u32(Bst + GL * kBTok * MB + g * kBTok + c * kBLane);
+              const uint4 *bq = reinterpret_cast<const uint4 *>(Bl + GL * kBTok * MB);
 #pragma unroll
-              for (int cp = 0; cp < kCP; ++cp)
-                asm volatile(
-                    "{\n.reg .pred p;\nsetp.ne.b32 p, %5, 0;\n@p ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];\n}"
-                    : "+r"(b[4 * cp]), "+r"(b[4 * cp + 1]), "+r"(b[4 * cp + 2]), "+r"(b[4 * cp + 3])
-                    : "r"(bsrc + cp * 4 * kBLane), "r"((uint32_t)breal));
+              for (int cp = 0; cp < kCP; ++cp) {
+                const uint4 v = bq[cp * 4];
+                b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
+              }
             }
             float d[4];
             group_mma(aL, aH, b, d);
@@ -756,27 +902,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 4; ++i) dp[i] = d[i];
           }
         };
-        group(std::integral_constant<int, 0>{});
-        group(std::integral_constant<int, 1>{});
-        group(std::integral_constant<int, 2>{});
-        group(std::integral_constant<int, 3>{});
-        group(std::integral_constant<int, 4>{});
-        group(std::integral_constant<int, 5>{});
-        group(std::integral_constant<int, 6>{});
-        group(std::integral_constant<int, 7>{});
-        // the epilogue of the stage's last group
-        auto last = [&](auto glc) {
-          constexpr int GL = decltype(glc)::value;
-          if (GL < gs && GL + 1 >= gs) epilogue(glc, dp);
+        auto stage = [&](auto fullc) {
+          group(std::integral_constant<int, 0>{}, fullc);
+          group(std::integral_constant<int, 1>{}, fullc);
+          group(std::integral_constant<int, 2>{}, fullc);
+          group(std::integral_constant<int, 3>{}, fullc);
+          group(std::integral_constant<int, 4>{}, fullc);
+          group(std::integral_constant<int, 5>{}, fullc);
+          group(std::integral_constant<int, 6>{}, fullc);
+          group(std::integral_constant<int, 7>{}, fullc);
         };
-        last(std::integral_constant<int, 0>{});
-        last(std::integral_constant<int, 1>{});
-        last(std::integral_constant<int, 2>{});
-        last(std::integral_constant<int, 3>{});
-        last(std::integral_constant<int, 4>{});
-        last(std::integral_constant<int, 5>{});
-        last(std::integral_constant<int, 6>{});
-        last(std::integral_constant<int, 7>{});
+        if (gs == kStageG) {
+          // a full stage: straight-line code
+          stage(std::true_type{});
+          epilogue(std::integral_constant<int, kStageG - 1>{}, dp);
+        } else {
+          stage(std::false_type{});
+          // the epilogue of the stage's last group
+          auto last = [&](auto glc) {
+            constexpr int GL = decltype(glc)::value;
+            if (GL < gs && GL + 1 >= gs) epilogue(glc, dp);
+          };
+          last(std::integral_constant<int, 0>{});
+          last(std::integral_constant<int, 1>{});
+          last(std::integral_constant<int, 2>{});
+          last(std::integral_constant<int, 3>{});
+          last(std::integral_constant<int, 4>{});
+          last(std::integral_constant<int, 5>{});
+          last(std::integral_constant<int, 6>{});
+        }
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->empty[buf]);
         if (w.last_stage()) {
@@ -897,7 +1051,14 @@ static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
   mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (any2) {
+  if (any2 && bp.M == 1 && gmax <= mm::kP1MaxG) {
+    const int sm = mm::p1_dyn_bytes(gmax);
+    e = cudaFuncSetAttribute(mm::gemv_mma_p2_one_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+    if (e != cudaSuccess) return e;
+    mm::gemv_mma_p2_one_kernel<<<ctas, mm::kP1Threads, sm, s>>>(bp, sc);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  } else if (any2) {
     mm::gemv_mma_p2_kernel<<<dim3(tmax, bp.count), mm::kP2Threads, 0, s>>>(bp);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
