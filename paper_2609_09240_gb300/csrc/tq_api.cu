@@ -89,7 +89,7 @@ size_t problem_ws_bytes(int M, int N, int K) {
   if (M <= 8) {
     size_t b, cs, y2;
     mma_workspace_parts(M, N, K, &b, &cs, &y2);
-    return pad256(b) + pad256(cs) + pad256(y2);
+    return pad256(b) + pad256(cs) + pad256(y2) + 256;  // + the plane-1 tensor map
   }
   return pad256(tc_workspace_bytes(16, K));
 }
@@ -127,6 +127,7 @@ tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStr
       P.wsB = ws + off;
       P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
       P.wsY2 = reinterpret_cast<float *>(ws + off + pad256(b) + pad256(cs));
+      P.wsMap = ws + off + pad256(b) + pad256(cs) + pad256(y2);
     } else {
       P.wsB = ws + off;
       P.wsCS = reinterpret_cast<float *>(ws + off + tc_workspace_b_bytes(16, P.K));

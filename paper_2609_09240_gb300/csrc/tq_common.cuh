@@ -39,6 +39,7 @@ struct Problem {
   unsigned char *wsB;  // workspace: activation slots of this problem
   float *wsCS;         // workspace: per-group C and S of this problem
   float *wsY2;         // workspace: second-plane partial sums [N][M] (M <= 8 path)
+  void *wsMap;         // workspace: 128-byte tensor map of plane 1 (M <= 8 path)
   int32_t N, K;
   int32_t tile_begin;  // first global tile index of this problem
   int32_t nnz;         // plane-2 records (rowptr[N]); indices are clamped below it

@@ -50,6 +50,10 @@
 //    end add y2 and write y; warp 8 bulk-copies each stage's B fragments and
 //    C/S into the same ring.
 // Every wait is bounded (tq_sm100.cuh); a timeout raises a CTA-wide abort.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
 #include <type_traits>
 
 #include "tq_common.cuh"
@@ -283,14 +287,37 @@ struct Walk {
   }
 };
 
+// Tensor-map templates of plane 1, one per distinct row length in a batch
+// (encoded on the host for that row length and stride); idx[p] picks
+// problem p's.
+constexpr int kMaxMapTemplates = 8;
+struct MapTemplates {
+  CUtensorMap t[kMaxMapTemplates];
+  uint8_t idx[TQ_MAX_BATCH];
+};
+
 // ------------------------------------------------------------------ prep
 // B fragments, C and S for every (problem, group, token).  B layout of a
 // group: [token m][chunk pair cp][lane position c] x 16 B, each 16 B being
 // (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
-__global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp) {
+__global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ MapTemplates mt) {
   const int p = blockIdx.y;
   if (p >= bp.count) return;
   const Problem &P = bp.prob[p];
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    // plane 1 as a 2-D byte tensor (row_bytes x N) for the main kernel's
+    // stage copies: the template of its row length with this problem's
+    // address and row count
+    const uint4 *src = reinterpret_cast<const uint4 *>(&mt.t[mt.idx[p]]);
+    uint4 *dst = reinterpret_cast<uint4 *>(P.wsMap);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) dst[i] = src[i];
+    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(P.wsMap), "l"(P.plane1)
+                 : "memory");
+    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(P.wsMap), "r"((uint32_t)P.N)
+                 : "memory");
+    asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
+  }
   const int MB = bp.M;
   const int G = P.K / kGroup;
   const int task = blockIdx.x * blockDim.x + threadIdx.x;
@@ -708,6 +735,332 @@ __global__ void __launch_bounds__(kP1Threads, 1)
   }
 }
 
+// Second plane, tensor-core version (1..8 tokens).  Persistent over the
+// main kernel's tile ranges, in spans of 1..4 consecutive tiles of one
+// problem (as many as keep the span's expected records within the record
+// buffer).  For each span the CTA stages the rows' rowptr and salience words
+// and the span's contiguous range of plane-2 records and s2 in shared
+// memory, one span ahead (asynchronous copies; each span's metadata carries
+// the next span's record bounds, so the next records can be requested at
+// once; a span whose records exceed the buffer is done in several record
+// ranges).  Warp w takes groups g = w, w + 16, ...: per 128 rows a ballot
+// gives the rows whose bit g is set, compacted into a per-warp list with
+// their records' places; 16 list entries form one m16 tile whose rows are
+// records, decoded with the same encoding as the first plane and multiplied
+// by group g's B fragment.  s2 * (D - C) per record accumulates per row in
+// shared memory and goes to the workspace (y2) at the span's end.
+constexpr int kQThreads = 512, kQWarps = 16;
+constexpr int kQMaxSpanTiles = 4, kQMaxSpanRows = kQMaxSpanTiles * kRows;
+constexpr int kQRecBuf = 47104;                                   // record bytes per buffer
+constexpr int kQRecCap = (kQRecBuf - 16) / kGroupBytes;           // records per range
+constexpr int kQRecPerThread = (kQRecCap + kQThreads - 1) / kQThreads;
+constexpr int kQMaxW = 10;                                        // salience words per row
+constexpr int kQMaxG = kQMaxW * 32;
+constexpr int kQS2Buf = ((2 * kQRecCap + 8 + 15) / 16) * 16;      // s2 bytes per buffer
+constexpr int kQMetaSal = 2304;                                   // salience words per span
+struct QMeta {
+  int32_t rp[kQMaxSpanRows + 4];  // rowptr of the span's rows (rows + 1 used)
+  int32_t next[4];                // record bounds of the next span
+  uint32_t sal[kQMetaSal];        // salience words, [row][W]
+};
+constexpr int kQMetaOff = 0;                                          // QMeta[2]
+constexpr int kQListOff = kQMetaOff + 2 * (int)sizeof(QMeta);         // records by group: entry, s2
+constexpr int kQCntOff = kQListOff + kQRecCap * 8;                    // per group: count, first entry
+constexpr int kQAccOff = kQCntOff + 2 * kQMaxG * 4;                   // float [span row][8]
+constexpr int kQS2Off = kQAccOff + kQMaxSpanRows * 8 * 4;             // s2 buffers
+constexpr int kQEndA = kQS2Off + 2 * kQS2Buf;
+static_assert(kQEndA <= kArena1, "plane-2 arrays overflow the region below the table");
+constexpr int kQRecOff = kArena1 + kLutBytes;                         // record buffers, above the table
+constexpr int kQRecStride = kQRecBuf + 64;
+constexpr int kQDynBytes = kQRecOff + 2 * kQRecStride;
+static_assert(kQDynBytes <= kDynBytes, "plane-2 shared memory");
+static_assert(kQMetaSal >= kRows * kQMaxW, "one tile's salience words fit a span");
+
+__device__ __forceinline__ void cp_async16_zfill(void *dst, const void *src, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async4_zfill(void *dst, const void *src, int src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+
+// Tiles per span of a problem: the expected records of a span (the mean
+// per row, nnz / N) stay below 85 % of the buffer, the salience words fit.
+__device__ __forceinline__ int q_span_tiles(const Problem &P) {
+  const int W = sal_words_of(P.K);
+  const int by_meta = kQMetaSal / (kRows * W);
+  const int64_t per_tile = ((int64_t)kRows * P.nnz + P.N - 1) / P.N;
+  const int by_rec = (int)min((int64_t)kQMaxSpanTiles, (int64_t)(kQRecCap * 85 / 100) / max(per_tile, (int64_t)1));
+  return max(1, min(by_meta, by_rec));
+}
+
+// The span starting at the first tile at or after `tile` (below t_end) of
+// a problem with a second plane; q is the problem to start the search from.
+struct QSpan {
+  int tile, ntiles, q, n0, rows;
+  bool valid;
+};
+__device__ __forceinline__ QSpan q_span(const BatchParams &bp, int tile, int q, int t_end) {
+  QSpan S{0, 0, 0, 0, 0, false};
+  while (tile < t_end) {
+    while (q + 1 < bp.count && bp.prob[q + 1].tile_begin <= tile) ++q;
+    const Problem &P = bp.prob[q];
+    const int p_end = P.tile_begin + (P.N + kRows - 1) / kRows;
+    if (P.nnz > 0) {
+      S.tile = tile, S.q = q;
+      S.ntiles = min(q_span_tiles(P), min(p_end, t_end) - tile);
+      S.n0 = (tile - P.tile_begin) * kRows;
+      S.rows = min(S.ntiles * kRows, P.N - S.n0);
+      S.valid = true;
+      return S;
+    }
+    tile = p_end;  // skip the problem
+  }
+  return S;
+}
+
+// A record range: records [lo, hi) of plane 2 (of the span's [r0, end)),
+// staged from the 16-byte boundary at or below byte 26 lo (delta bytes
+// earlier); s2 from the 4-byte boundary at or below s2 + lo (ds bytes earlier).
+struct QRange {
+  int64_t lo, hi, end;
+  int delta, ds;
+};
+__device__ __forceinline__ QRange q_range(const Problem &P, int32_t first, int32_t last, int64_t lo) {
+  QRange R;
+  const int64_t nnz = P.nnz;
+  const int64_t r0 = min(max((int64_t)first, (int64_t)0), nnz);
+  R.end = min(max((int64_t)last, r0), nnz);
+  R.lo = lo < 0 ? r0 : lo;
+  R.hi = min(R.end, R.lo + kQRecCap);
+  R.delta = (int)((R.lo * kGroupBytes) & 15);
+  R.ds = (int)(((uintptr_t)(P.s2 + R.lo)) & 3u);
+  return R;
+}
+
+// The span's rowptr and salience words, and the next span's record bounds.
+__device__ __forceinline__ void q_issue_meta(const BatchParams &bp, const QSpan &S, const QSpan &Sn, QMeta *M) {
+  const Problem &P = bp.prob[S.q];
+  const int W = sal_words_of(P.K);
+  for (int i = threadIdx.x; i <= S.rows; i += kQThreads) cp_async4(&M->rp[i], P.rowptr + S.n0 + i);
+  for (int i = threadIdx.x; i < S.rows * W; i += kQThreads) cp_async4(&M->sal[i], P.sal + (int64_t)S.n0 * W + i);
+  if (Sn.valid && threadIdx.x < 2) {
+    const Problem &Pn = bp.prob[Sn.q];
+    cp_async4(&M->next[threadIdx.x], Pn.rowptr + Sn.n0 + (threadIdx.x ? Sn.rows : 0));
+  }
+}
+
+__device__ __forceinline__ void q_issue_records(const Problem &P, const QRange &R, unsigned char *rec,
+                                                unsigned char *s2b) {
+  const int64_t a0 = R.lo * kGroupBytes - R.delta, end = R.hi * kGroupBytes, lim = P.nnz * kGroupBytes;
+  const int nch = (int)((end - a0 + 15) / 16);
+  for (int k = threadIdx.x; k < nch; k += kQThreads) {
+    const int64_t off = a0 + 16 * (int64_t)k;
+    cp_async16_zfill(rec + 16 * k, P.plane2 + off, (int)min((int64_t)16, lim - off));
+  }
+  const unsigned char *b0 = reinterpret_cast<const unsigned char *>(P.s2 + R.lo) - R.ds;
+  const unsigned char *bend = reinterpret_cast<const unsigned char *>(P.s2 + R.hi);
+  const unsigned char *blim = reinterpret_cast<const unsigned char *>(P.s2 + P.nnz);
+  const int nw = (int)((bend - b0 + 3) / 4);
+  for (int k = threadIdx.x; k < nw; k += kQThreads)
+    cp_async4_zfill(s2b + 4 * k, b0 + 4 * k, (int)min((ptrdiff_t)4, blim - (b0 + 4 * k)));
+}
+
+template <bool ONE>
+__global__ void __launch_bounds__(kQThreads, 1)
+    gemv_mma_p2v3_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
+  extern __shared__ __align__(1024) unsigned char dynq[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (smem_u32(dynq) != kDynShared) {
+    if (tid == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  const int t_end = sc.cta_tile[blockIdx.x + 1];
+  QSpan S = q_span(bp, sc.cta_tile[blockIdx.x], 0, t_end);
+  if (!S.valid) return;
+  QMeta *meta = reinterpret_cast<QMeta *>(dynq + kQMetaOff);
+  uint32_t *list = reinterpret_cast<uint32_t *>(dynq + kQListOff);
+  float *lists2 = reinterpret_cast<float *>(list + kQRecCap);
+  int *gcnt = reinterpret_cast<int *>(dynq + kQCntOff);
+  int *goff = gcnt + kQMaxG;
+  float *acc = reinterpret_cast<float *>(dynq + kQAccOff);
+  unsigned char *s2buf = dynq + kQS2Off;
+  unsigned char *recbuf = dynq + kQRecOff;
+  {
+    uint32_t *lut = reinterpret_cast<uint32_t *>(dynq + kArena1);
+    for (int i = tid; i < 256 * 32; i += kQThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+    for (int i = tid; i < kQMaxSpanRows * 8; i += kQThreads) acc[i] = 0.f;
+    for (int i = tid; i < kQMaxG; i += kQThreads) gcnt[i] = 0;
+  }
+  const int MB = ONE ? 1 : bp.M;
+  const int g16 = lane >> 2, c = lane & 3;
+  const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
+
+  // prologue: the first span's metadata (with the next span's record bounds), then its records
+  QSpan S1 = q_span(bp, S.tile + S.ntiles, S.q, t_end);
+  q_issue_meta(bp, S, S1, &meta[0]);
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+  q_issue_records(bp.prob[S.q], q_range(bp.prob[S.q], meta[0].rp[0], meta[0].rp[S.rows], -1), recbuf, s2buf);
+  cp_async_commit();
+
+  for (int k = 0; S.valid; ++k) {
+    const int cur = k & 1, nxt = cur ^ 1;
+    QMeta &M = meta[cur];
+    cp_async_wait<0>();
+    __syncthreads();  // this span's records and metadata are in; the previous span is done
+    // request the next span's records (bounds from this span's metadata) and
+    // its metadata (with the record bounds of the one after)
+    QSpan S2{0, 0, 0, 0, 0, false};
+    if (S1.valid) {
+      S2 = q_span(bp, S1.tile + S1.ntiles, S1.q, t_end);
+      q_issue_records(bp.prob[S1.q], q_range(bp.prob[S1.q], M.next[0], M.next[1], -1), recbuf + nxt * kQRecStride,
+                      s2buf + nxt * kQS2Buf);
+      q_issue_meta(bp, S1, S2, &meta[nxt]);
+      cp_async_commit();
+    }
+    const Problem &P = bp.prob[S.q];
+    const int G = P.K / kGroup, W = sal_words_of(P.K), rows = S.rows;
+    unsigned char *rec = recbuf + cur * kQRecStride;
+    unsigned char *s2b = s2buf + cur * kQS2Buf;
+    const int rp0 = M.rp[0];
+    QRange R = q_range(P, M.rp[0], M.rp[rows], -1);
+    for (;;) {
+      const int n_rel = (int)(R.hi - R.lo);
+      // records of the range by group (counting sort): a record's row is the
+      // last r with rp[r] <= j, its group the rank-th set bit of that row
+      int rj[kQRecPerThread], gj[kQRecPerThread], pj[kQRecPerThread];
+#pragma unroll
+      for (int u = 0; u < kQRecPerThread; ++u) {
+        const int jr = tid + u * kQThreads;
+        gj[u] = -1;
+        if (jr < n_rel) {
+          const int j = (int)(R.lo - rp0) + jr;  // relative to the span's first record
+          int r = 0;
+#pragma unroll
+          for (int step = kQMaxSpanRows / 2; step >= 1; step >>= 1)
+            if (r + step < rows && M.rp[r + step] - rp0 <= j) r += step;
+          int rank = j - (M.rp[r] - rp0), g = -1;
+          for (int w = 0; w < W; ++w) {
+            const uint32_t word = M.sal[r * W + w];
+            const int cnt = __popc(word);
+            if (rank < cnt) {
+              g = 32 * w + (int)__fns(word, 0u, rank + 1);
+              break;
+            }
+            rank -= cnt;
+          }
+          if (g >= 0 && g < G) {
+            rj[u] = r;
+            gj[u] = g;
+            pj[u] = atomicAdd(&gcnt[g], 1);
+          }
+        }
+      }
+      __syncthreads();
+      if (warp == 0) {
+        // exclusive scan of the group counts (each lane a run of groups)
+        const int per = (G + 31) / 32, g0 = lane * per;
+        int run = 0;
+        for (int i = 0; i < per; ++i)
+          if (g0 + i < G) run += gcnt[g0 + i];
+        int incl = run;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int v = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += v;
+        }
+        int base = incl - run;
+        for (int i = 0; i < per; ++i)
+          if (g0 + i < G) {
+            goff[g0 + i] = base;
+            base += gcnt[g0 + i];
+          }
+      }
+      __syncthreads();
+      // entry = span row | (4 + byte offset of the record's window in the buffer) << 9
+#pragma unroll
+      for (int u = 0; u < kQRecPerThread; ++u) {
+        if (gj[u] < 0) continue;
+        const int jr = tid + u * kQThreads, g = gj[u], GL = g % kStageG;
+        const int pos = goff[g] + pj[u];
+        list[pos] = (uint32_t)rj[u] | ((uint32_t)(R.delta + kGroupBytes * jr - 2 * (GL & 1) + 4) << 9);
+        lists2[pos] = __half2float(*reinterpret_cast<const __half *>(s2b + R.ds + 2 * jr));
+      }
+      __syncthreads();
+      for (int g = warp; g < G; g += kQWarps) {
+        const int count = gcnt[g];
+        if (count == 0) continue;
+        const uint32_t *lg = list + goff[g];
+        const float *sg = lists2 + goff[g];
+        const int GL = g % kStageG;
+        // the group's B fragment (lanes of absent tokens repeat the last token) and C
+        const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB + min(g16, MB - 1) * kBTok + c * kBLane;
+        uint32_t b[20];
+#pragma unroll
+        for (int cp = 0; cp < kCP; ++cp) {
+          const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg + cp * 4 * kBLane));
+          b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
+        }
+        const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + 2 * c));
+        // lane c's window words: win_start + jw and + 4 (the record starts o bytes in)
+        const int jw = (c - win_start(GL)) & 3;
+        for (int e0 = 0; e0 < count; e0 += 16) {
+          uint32_t aL[20], aH[20];
+          int rowv[2];
+          float s2v[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int s = e0 + g16 + 8 * h;
+            const uint32_t e = s < count ? lg[s] : 4u << 9;
+            rowv[h] = s < count ? (int)(e & 511u) : -1;
+            s2v[h] = sg[s < count ? s : 0];
+            const uint32_t a = (e >> 9) + 4 * jw, sh = (a & 3u) * 8u;
+            const uint32_t *wp = reinterpret_cast<const uint32_t *>(rec - 4 + (a & ~3u));
+            decode_words(__funnelshift_r(wp[0], wp[1], sh), __funnelshift_r(wp[4], wp[5], sh), tag, h ? aH : aL);
+          }
+          float d[4];
+          group_mma(aL, aH, b, d);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            if (rowv[h] < 0) continue;
+            if (ONE) {
+              if (c == 0) atomicAdd(&acc[rowv[h] * 8], s2v[h] * (d[2 * h] - Cv.x));
+            } else {
+#pragma unroll
+              for (int i = 0; i < 2; ++i) {
+                const int m = 2 * c + i;
+                if (m < MB) atomicAdd(&acc[rowv[h] * 8 + m], s2v[h] * (d[2 * h + i] - (i ? Cv.y : Cv.x)));
+              }
+            }
+          }
+        }
+      }
+      __syncthreads();
+      for (int i = tid; i < G; i += kQThreads) gcnt[i] = 0;
+      if (R.hi >= R.end) break;
+      // a further record range of this span (the buffer holds kQRecCap records)
+      __syncthreads();
+      R = q_range(P, M.rp[0], M.rp[rows], R.hi);
+      q_issue_records(P, R, rec, s2b);
+      cp_async_commit();
+      cp_async_wait<0>();
+      __syncthreads();
+    }
+    __syncthreads();
+    for (int i = tid; i < rows * MB; i += kQThreads) {
+      const int r = ONE ? i : i / MB, m = ONE ? 0 : i - r * MB;
+      P.wsY2[(int64_t)(S.n0 + r) * MB + m] = acc[r * 8 + m];
+      acc[r * 8 + m] = 0.f;
+    }
+    S = S1;
+    S1 = S2;
+  }
+  cp_async_wait<0>();
+}
+
 // ------------------------------------------------------------------ main
 template <bool F32>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -737,7 +1090,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (tid == 0) {
     for (int i = 0; i < NS; ++i) {
-      mbar_init(&bars->full[i], 1);  // the producer's expect-tx arrival
+      mbar_init(&bars->full[i], 1 + 32);  // the producer's expect-tx arrival + its lanes' s1/off arrivals
       mbar_init(&bars->empty[i], kWarpsP1);
     }
     bars->abort_ = 0;
@@ -756,89 +1109,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
       uint32_t b[20];
       float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
-      // The tile's 16 rows of a stage (packed bytes, s1 and off), fetched with
-      // 16-byte asynchronous copies NS - 1 stages ahead; one commit group per
-      // stage and warp.
-      auto fetch_rows = [&](const Walk &a, int slot) {
-        const Problem &P = a.P();
-        const int64_t RB = row_bytes_of(P.K);
-        const int n0 = (a.tile - P.tile_begin) * kRows + mt * 16;
-        const int rows = min(16, P.N - n0);
-        const int nch = (a.gs * kGroupBytes + 15) / 16;  // 16-byte chunks per row
-        unsigned char *dst = bytes_buf(slot) + mt * 16 * kStageBytes;
-        const unsigned char *src = P.plane1 + (int64_t)n0 * RB + (int64_t)a.s * kStageBytes;
-        if (nch == kStageBytes / 16 && rows == 16) {
-          // 208 chunks; lane takes chunk i = lane + 32 k, i.e. row r = i / 13,
-          // chunk ch = i % 13, advanced incrementally (32 = 2 x 13 + 6)
-          static_assert(kStageBytes == 13 * 16, "a stage row is 13 chunks");
-          const int r = lane / 13, ch0 = lane - 13 * r;
-          int ch = ch0;
-          unsigned char *dptr = dst + r * kStageBytes + 16 * ch0;
-          const unsigned char *sptr = src + r * RB + 16 * ch0;
-#pragma unroll
-          for (int k = 0; k < 7; ++k) {
-            if (k < 6 || lane < 16) cp_async16(dptr, sptr);
-            ch += 6;
-            dptr += 2 * kStageBytes + 96;
-            sptr += 2 * RB + 96;
-            if (ch >= 13) {  // one more row, 13 chunks back: the slot's rows are contiguous
-              ch -= 13;
-              sptr += RB - kStageBytes;
-            }
-          }
-        } else if (nch == kStageBytes / 16) {
-          for (int i = lane; i < rows * (kStageBytes / 16); i += 32) {
-            const int r = i / (kStageBytes / 16), ch = i - r * (kStageBytes / 16);
-            cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
-          }
-        } else {
-          for (int i = lane; i < rows * nch; i += 32) {
-            const int r = i / nch, ch = i - r * nch;
-            cp_async16(dst + r * kStageBytes + 16 * ch, src + r * RB + 16 * ch);
-          }
-        }
-        const int G = P.K / kGroup, g0 = a.s * kStageG;
-        const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
-        const int rs = lane & 15;  // lanes 0-15 fetch s1, lanes 16-31 off
-        const __half *arr = (lane >> 4) ? P.off : P.s1;
-        unsigned char *d = ar2 + L.oSO + slot * kSOSlot + (lane >> 4) * kRows * 16 + (mt * 16 + rs) * 16;
-        if (rs < rows) {
-          const int64_t o = (int64_t)(n0 + rs) * G + g0;
-          if (vec) {
-            cp_async16(d, arr + o);
-          } else {
-            __half *dh = reinterpret_cast<__half *>(d);
-            for (int gg = 0; gg < kStageG; ++gg) dh[gg] = gg < a.gs ? arr[o + gg] : __float2half_rn(0.f);
-          }
-        }
-        cp_async_commit();
-      };
-      Walk ahead(&bp, t_begin, t_end);
-      for (int k = 0; k < NS - 1; ++k) {
-        if (ahead.valid()) {
-          fetch_rows(ahead, k);
-          ahead.next();
-        } else {
-          cp_async_commit();
-        }
-      }
-      uint32_t q = 0;
-      for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
-        const int buf = (int)(q % (uint32_t)NS);
-        // refill the slot the previous stage used, then wait for this stage
-        if (ahead.valid()) {
-          fetch_rows(ahead, (int)((q + NS - 1) % (uint32_t)NS));
-          ahead.next();
-        } else {
-          cp_async_commit();
-        }
-        if (NS == 4)
-          cp_async_wait<3>();
-        else
-          cp_async_wait<2>();
-        const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->full[buf], (q / NS) & 1u, abort_));
+      uint32_t buf = 0, phase = 0;
+      for (Walk w(&bp, t_begin, t_end); w.valid(); w.next()) {
+        // the stage's rows, s1 / off, B and C / S are in slot buf
+        const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->full[buf], phase, abort_));
         if (!ok) break;
-        __syncwarp();  // every lane's copies are visible to the warp
         const unsigned char *Bst = ar2 + L.oB + buf * L.BStage;
         // this lane's B words (lanes of absent tokens load the last token's:
         // their output columns are never written)
@@ -960,29 +1235,77 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int i = 0; i < 4; ++i) y[i] = 0.f;
         }
+        if (++buf == (uint32_t)NS) buf = 0, phase ^= 1u;
       }
     }
-    cp_async_wait<0>();  // nothing in flight into shared memory at exit
   } else if (warp == kWarpProd) {
     // ========================================================== producer
-    uint32_t q = 0;
+    // Per stage: the tile's plane-1 bytes (one 2-D tensor copy), B and C / S
+    // (bulk copies), counted in bytes on full[buf]; s1 / off (16-byte
+    // asynchronous copies spread over the lanes), each lane arriving on
+    // full[buf] once its copies landed.
+    uint32_t buf = 0, phase = 0, q = 0;
+    int map_pi = -1;
     for (Walk w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
       const Problem &P = w.P();
       const int gs = w.gs, g0 = w.s * kStageG;
+      const int n0 = (w.tile - P.tile_begin) * kRows, rows = min(kRows, P.N - n0);
       const uint32_t bb = (uint32_t)(gs * kBTok * MB);
       const uint32_t cb = (uint32_t)(gs * kCSGroup);
-      const int buf = (int)(q % (uint32_t)NS);
       int ok = 1;
-      if (lane == 0) ok = wait_or_abort(&bars->empty[buf], ((q / NS) & 1u) ^ 1u, abort_) ? 1 : 0;
+      if (lane == 0) ok = wait_or_abort(&bars->empty[buf], phase ^ 1u, abort_) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
+      uint64_t *full = &bars->full[buf];
       if (lane == 0) {
-        mbar_arrive_expect_tx(&bars->full[buf], bb + cb);
-        bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, &bars->full[buf]);
+        if (w.pi != map_pi) {
+          // the problem's tensor map, written by the prep kernel
+          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(P.wsMap) : "memory");
+          map_pi = w.pi;
+        }
+        mbar_arrive_expect_tx(full, bb + cb + (uint32_t)kBytesSlot);
+        bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, full);
         bulk_g2s(ar2 + L.oCS + buf * kCSSlot, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * kCSGroup,
-                 cb, &bars->full[buf]);
+                 cb, full);
+        // the stage's 208 bytes of the tile's 128 rows (rows past N and bytes
+        // past the row's end arrive as zeros)
+        asm volatile(
+            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+                smem_u32(bytes_buf((int)buf))),
+            "l"(P.wsMap), "r"(w.s * kStageBytes), "r"(n0), "r"(smem_u32(full))
+            : "memory");
       }
       __syncwarp();
+      {
+        const int G = P.K / kGroup;
+        const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+        unsigned char *so = ar2 + L.oSO + buf * kSOSlot;
+        if (vec) {
+#pragma unroll
+          for (int k = 0; k < kRows / 32; ++k) {
+            const int r = lane + 32 * k;
+            if (r < rows) {
+              const int64_t o = (int64_t)(n0 + r) * G + g0;
+              cp_async16(so + r * 16, P.s1 + o);
+              cp_async16(so + kRows * 16 + r * 16, P.off + o);
+            }
+          }
+          cp_async_mbar_arrive_noinc(full);
+        } else {
+          for (int r = lane; r < rows; r += 32) {
+            const int64_t o = (int64_t)(n0 + r) * G + g0;
+            __half *d1 = reinterpret_cast<__half *>(so + r * 16);
+            __half *d2 = reinterpret_cast<__half *>(so + kRows * 16 + r * 16);
+            for (int gg = 0; gg < kStageG; ++gg) {
+              d1[gg] = gg < gs ? P.s1[o + gg] : __float2half_rn(0.f);
+              d2[gg] = gg < gs ? P.off[o + gg] : __float2half_rn(0.f);
+            }
+          }
+          mbar_arrive(full);
+        }
+      }
+      if (++buf == (uint32_t)NS) buf = 0, phase ^= 1u;
     }
+    cp_async_wait<0>();  // the lanes' s1 / off copies have landed
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
     if (lane == 0) {
@@ -1018,9 +1341,94 @@ void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2)
 
 TQ_STATUS_ACCESSOR(read_status_gemv_mma)
 
+// Tensor map of plane 1 as a 2-D byte tensor of rows of `rb` bytes (box
+// 208 x 128 bytes, no swizzle, zero fill), encoded once per row length;
+// the prep kernel puts in each problem's address and row count.
+static bool plane1_template(int64_t rb, const void *plane1, int N, CUtensorMap *out) {
+  // the driver's encoder, looked up through the runtime (no link-time
+  // dependence on the driver library)
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      fn = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }();
+  if (!encode) return false;
+  static std::mutex mu;
+  static int64_t keys[64];
+  static CUtensorMap maps[64];
+  static int n = 0;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < n; ++i)
+    if (keys[i] == rb) {
+      *out = maps[i];
+      return true;
+    }
+  CUtensorMap m;
+  cuuint64_t dims[2] = {(cuuint64_t)rb, (cuuint64_t)N};
+  cuuint64_t strides[1] = {(cuuint64_t)rb};
+  cuuint32_t box[2] = {(cuuint32_t)mm::kStageBytes, (cuuint32_t)mm::kRows};
+  cuuint32_t estr[2] = {1, 1};
+  if (encode(&m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(plane1), dims, strides, box, estr,
+                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return false;
+  if (n < 64) keys[n] = rb, maps[n] = m, ++n;
+  *out = m;
+  return true;
+}
+
+static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) <= 32764, "prep kernel parameters");
+static_assert(sizeof(BatchParams) + sizeof(mm::Sched) <= 32764, "main kernel parameters");
+
+// Distinct plane-1 row lengths of a batch (up to `cap` + 1 are counted).
+static int distinct_row_lengths(const BatchParams &bp, int first, int last, int cap) {
+  int64_t seen[mm::kMaxMapTemplates + 1];
+  int n = 0;
+  for (int i = first; i < last && n <= cap; ++i) {
+    const int64_t rb = row_bytes_of(bp.prob[i].K);
+    int k = 0;
+    while (k < n && seen[k] != rb) ++k;
+    if (k == n) seen[n++] = rb;
+  }
+  return n;
+}
+
+template <bool F32>
+static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s);
+
+// A batch with more distinct row lengths than tensor-map templates runs as
+// consecutive sub-batches (in order, same stream).
 template <bool F32>
 static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
-  static mm::Sched sc;
+  if (distinct_row_lengths(bp, 0, bp.count, mm::kMaxMapTemplates) <= mm::kMaxMapTemplates) return launch_mm_one<F32>(bp, s);
+  thread_local BatchParams sub;
+  int i = 0;
+  while (i < bp.count) {
+    int j = i + 1;
+    while (j < bp.count && distinct_row_lengths(bp, i, j + 1, mm::kMaxMapTemplates) <= mm::kMaxMapTemplates) ++j;
+    sub.count = j - i;
+    sub.M = bp.M;
+    sub.out_f32 = bp.out_f32;
+    int tiles = 0;
+    for (int k = 0; k < sub.count; ++k) {
+      sub.prob[k] = bp.prob[i + k];
+      sub.prob[k].tile_begin = tiles;
+      tiles += (sub.prob[k].N + mm::kRows - 1) / mm::kRows;
+    }
+    sub.total_tiles = tiles;
+    const cudaError_t e = launch_mm_one<F32>(sub, s);
+    if (e != cudaSuccess) return e;
+    i = j;
+  }
+  return cudaSuccess;
+}
+
+template <bool F32>
+static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
+  thread_local mm::Sched sc;
   if (bp.M < 1 || bp.M > 8 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
   const int ctas = min(num_sms_mm(), 256);
   int64_t total_cost = 0;
@@ -1048,14 +1456,30 @@ static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
     tmax = max(tmax, (bp.prob[i].N + mm::kRows - 1) / mm::kRows);
     any2 = any2 || bp.prob[i].nnz > 0;
   }
-  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp);
+  thread_local mm::MapTemplates mt;
+  {
+    int64_t rbs[mm::kMaxMapTemplates];
+    int nt = 0;
+    for (int i = 0; i < bp.count; ++i) {
+      const int64_t rb = row_bytes_of(bp.prob[i].K);
+      int k = 0;
+      while (k < nt && rbs[k] != rb) ++k;
+      if (k == nt) {
+        if (nt == mm::kMaxMapTemplates) return cudaErrorNotSupported;  // launch_mm splits such batches
+        if (!plane1_template(rb, bp.prob[i].plane1, bp.prob[i].N, &mt.t[nt])) return cudaErrorInvalidValue;
+        rbs[nt++] = rb;
+      }
+      mt.idx[i] = (uint8_t)k;
+    }
+  }
+  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (any2 && bp.M == 1 && gmax <= mm::kP1MaxG) {
-    const int sm = mm::p1_dyn_bytes(gmax);
-    e = cudaFuncSetAttribute(mm::gemv_mma_p2_one_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (any2 && gmax <= mm::kQMaxG) {
+    auto kern = bp.M == 1 ? mm::gemv_mma_p2v3_kernel<true> : mm::gemv_mma_p2v3_kernel<false>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kQDynBytes);
     if (e != cudaSuccess) return e;
-    mm::gemv_mma_p2_one_kernel<<<ctas, mm::kP1Threads, sm, s>>>(bp, sc);
+    kern<<<ctas, mm::kQThreads, mm::kQDynBytes, s>>>(bp, sc);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   } else if (any2) {

@@ -83,6 +83,12 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
   return false;
 }
 
+// Arrive on `bar` once the executing thread's earlier cp.async copies have
+// completed (the arrival is one of the barrier's expected arrivals).
+__device__ __forceinline__ void cp_async_mbar_arrive_noinc(uint64_t *bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 // ---------------------------------------------------------- bulk copies
 // 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
 // src, dst 16-byte aligned; bytes a multiple of 16.
