@@ -37,18 +37,18 @@
 // Kernels (one step = three launches):
 //  * gemv_mma_prep_kernel: B fragments, C and S per (problem, group, token);
 //  * the second plane, s2 * P2 per row into the workspace (y2, fp32):
-//    gemv_mma_p2_one_kernel for one token (a thread per record on the CUDA
-//    cores), gemv_mma_p2_kernel for 2..8 tokens (one CTA per 128-row tile
-//    compacts the tile's salient (row, group) pairs per group, decodes their
-//    records with the same encoding and runs m16n8k16 MMAs over 16 records
-//    at a time);
+//    gemv_mma_p2v3_kernel (persistent over row spans: a counting sort of the
+//    span's records by group, then m16n8k16 MMAs over 16 records of one group
+//    at a time); gemv_mma_p2_kernel, one CTA per 128-row tile, when a row has
+//    more salience words than the former's staging holds;
 //  * gemv_mma_kernel (one persistent CTA per SM over a cost-balanced range
-//    of 128-row tiles, 8-group stages): warps 0..7 each own 16 rows of the
-//    tile, fetch those rows' packed bytes and s1 / off with 16-byte
-//    asynchronous copies a few stages ahead into a ring of shared-memory
-//    slots, decode and multiply, apply s1 / off per group, and at the tile's
-//    end add y2 and write y; warp 8 bulk-copies each stage's B fragments and
-//    C/S into the same ring.
+//    of 128-row tiles, 8-group stages): warp 8 fills a ring of shared-memory
+//    slots, per stage the tile's 208 bytes of 128 rows (one 2-D tensor copy
+//    through the problem's tensor map, which the prep kernel writes into
+//    the workspace), the B fragments and C/S (bulk copies) and s1 / off
+//    (16-byte asynchronous copies); warps 0..7 each own 16 rows of the tile,
+//    decode and multiply, apply s1 / off per group, and at the tile's end
+//    add y2 and write y.
 // Every wait is bounded (tq_sm100.cuh); a timeout raises a CTA-wide abort.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -587,151 +587,6 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
   if (valid) {
     float *y2 = P.wsY2 + (int64_t)n * MB;
     for (int m = 0; m < MB; ++m) y2[m] = acc[t][m];
-  }
-}
-
-// Second plane for a single token (M = 1) on the CUDA cores, one thread per
-// record, persistent over the main kernel's tile ranges.  A span of up to
-// kP1SpanRows consecutive rows of one problem owns one contiguous range of
-// plane-2 records; a record's row is a binary search over the span's rowptr
-// and its group the rank-th set bit of that row's salience words.  Each of
-// the record's four lane positions is decoded into the same five-slot words
-// as the first plane (same lane-replicated table at the same address) and
-// dotted with that position's activation words of the group, staged in
-// shared memory per problem, by fp16 x fp16 -> fp32 fused multiply-adds.
-// s2 * (dot - C) per row accumulates in shared memory and goes to y2.
-constexpr int kP1Threads = 512;
-constexpr int kP1SpanRows = 1024;
-constexpr int kP1ActStride = 84;  // words per group: 4 lane positions x 20, padded for the banks
-constexpr int kP1MaxG = (kDynBytes - kArena1 - kLutBytes) / (kP1ActStride * 4);
-
-__host__ __device__ constexpr int p1_dyn_bytes(int G) { return kArena1 + kLutBytes + G * kP1ActStride * 4; }
-static_assert((2 * kP1SpanRows + 1 + kP1MaxG + kP1SpanRows * ((kP1MaxG + 31) / 32)) * 4 <= kArena1,
-              "plane-2 span arrays overflow the region below the table");
-
-// d + lo(a) lo(b) + hi(a) hi(b), fp16 operands, fp32 accumulation
-__device__ __forceinline__ float fma_h2(uint32_t a, uint32_t b, float d) {
-  float r;
-  asm("{ .reg .f16 al, ah, bl, bh;\n\t"
-      "mov.b32 {al, ah}, %1;\n\t"
-      "mov.b32 {bl, bh}, %2;\n\t"
-      "fma.rn.f32.f16 %0, al, bl, %3;\n\t"
-      "fma.rn.f32.f16 %0, ah, bh, %0; }"
-      : "=f"(r)
-      : "r"(a), "r"(b), "f"(d));
-  return r;
-}
-
-__global__ void __launch_bounds__(kP1Threads, 1)
-    gemv_mma_p2_one_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
-  extern __shared__ __align__(1024) unsigned char dyn[];
-  const int t = threadIdx.x, lane = t & 31;
-  if (smem_u32(dyn) != kDynShared) {
-    if (t == 0) atomicOr(&g_tq_device_status, 2u);
-    return;
-  }
-  int *rp = reinterpret_cast<int *>(dyn);                     // [kP1SpanRows + 1]
-  float *acc = reinterpret_cast<float *>(rp + kP1SpanRows + 1);  // [kP1SpanRows]
-  float *cg = acc + kP1SpanRows;                              // [kP1MaxG]
-  uint32_t *sw = reinterpret_cast<uint32_t *>(cg + kP1MaxG);  // [span rows][W]
-  uint32_t *act = reinterpret_cast<uint32_t *>(dyn + kArena1 + kLutBytes);
-  {
-    uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
-    for (int i = t; i < 256 * 32; i += kP1Threads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
-  }
-  const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
-  const int t1 = sc.cta_tile[blockIdx.x + 1];
-  int tile = sc.cta_tile[blockIdx.x], q = 0, staged = -1;
-  while (tile < t1) {
-    while (q + 1 < bp.count && bp.prob[q + 1].tile_begin <= tile) ++q;
-    const Problem &P = bp.prob[q];
-    const int tend = min(min(t1, P.tile_begin + (P.N + kRows - 1) / kRows), tile + kP1SpanRows / kRows);
-    const int n0 = (tile - P.tile_begin) * kRows, n1 = min(P.N, (tend - P.tile_begin) * kRows);
-    tile = tend;
-    if (P.nnz <= 0) continue;  // the main kernel adds no y2 for this problem
-    const int G = P.K / kGroup, W = sal_words_of(P.K), rows = n1 - n0;
-    __syncthreads();  // the previous span's arrays are free
-    if (q != staged) {
-      staged = q;
-      for (int i = t; i < G * 20; i += kP1Threads) {
-        const int g = i / 20, r = i - g * 20, c = r / 5, cp = r - c * 5;
-        *reinterpret_cast<uint4 *>(act + g * kP1ActStride + c * 20 + cp * 4) =
-            __ldg(reinterpret_cast<const uint4 *>(P.wsB + (int64_t)g * kBTok + (cp * 4 + c) * kBLane));
-      }
-      for (int g = t; g < G; g += kP1Threads) cg[g] = P.wsCS[(int64_t)g * (kCSGroup / 4)];
-    }
-    for (int i = t; i <= rows; i += kP1Threads) rp[i] = P.rowptr[n0 + i];
-    for (int i = t; i < rows * W; i += kP1Threads) {
-      const int w = i % W, gw = G - 32 * w;
-      const uint32_t bits = P.sal[(int64_t)n0 * W + i];
-      sw[i] = gw < 32 ? bits & ((1u << gw) - 1u) : bits;
-    }
-    for (int i = t; i < rows; i += kP1Threads) acc[i] = 0.f;
-    __syncthreads();
-    const int J0 = max(rp[0], 0), J1 = min(rp[rows], P.nnz);
-    for (int j = J0 + t; j < J1; j += kP1Threads) {
-      int r = 0;  // the record's row in the span: the last r with rp[r] <= j
-#pragma unroll
-      for (int step = kP1SpanRows / 2; step >= 1; step >>= 1)
-        if (r + step < rows && rp[r + step] <= j) r += step;
-      int rank = j - rp[r], g = 0;
-      for (int w = 0; w < W; ++w) {
-        const uint32_t word = sw[r * W + w];
-        const int cnt = __popc(word);
-        if (rank < cnt) {
-          g = 32 * w + (int)__fns(word, 0u, rank + 1);
-          break;
-        }
-        rank -= cnt;
-      }
-      const int GL = g % kStageG;
-      // the record's 26 bytes, placed o = 26 GL % 4 bytes into its window
-      const int64_t off0 = (int64_t)j * kGroupBytes;
-      const int sh = (int)(j & 1) * 2;  // plane 2 is 16-byte aligned: the record starts 0 or 2 bytes into a word
-      const uint32_t *src = reinterpret_cast<const uint32_t *>(P.plane2 + off0 - sh);
-      uint32_t wv[8];
-#pragma unroll
-      for (int i = 0; i < 6; ++i) wv[i] = __ldg(src + i);
-      // bytes 24, 25 only when the record is word-aligned: the word after them may lie past the end of plane 2
-      wv[6] = sh ? __ldg(src + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(src + 6));
-      wv[7] = 0u;
-      const float s2 = __half2float(P.s2[j]);
-      const int o = (GL & 1) * 2;
-      uint32_t win[8];
-      if (o == sh) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) win[i] = wv[i];
-      } else if (o == 2) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) win[i] = __funnelshift_l(i ? wv[i - 1] : 0u, wv[i], 16);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) win[i] = __funnelshift_r(wv[i], i < 7 ? wv[i + 1] : 0u, 16);
-      }
-      // window word i belongs to lane position c = (win_start + i) mod 4
-      const int ws = win_start(GL);
-      const uint32_t *ag = act + g * kP1ActStride;
-      float d[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        uint32_t a[20];
-        decode_words(win[i], win[i + 4], tag, a);
-        const uint4 *bq = reinterpret_cast<const uint4 *>(ag + ((ws + i) & 3) * 20);
-        float e = 0.f;
-#pragma unroll
-        for (int cp = 0; cp < kCP; ++cp) {
-          const uint4 b = bq[cp];
-          e = fma_h2(a[4 * cp], b.x, e);
-          e = fma_h2(a[4 * cp + 1], b.y, e);
-          e = fma_h2(a[4 * cp + 2], b.z, e);
-          e = fma_h2(a[4 * cp + 3], b.w, e);
-        }
-        d[i] = e;
-      }
-      atomicAdd(&acc[r], s2 * (((d[0] + d[1]) + (d[2] + d[3])) - cg[g]));
-    }
-    __syncthreads();
-    for (int i = t; i < rows; i += kP1Threads) P.wsY2[n0 + i] = acc[i];
   }
 }
 

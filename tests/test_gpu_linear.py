@@ -105,3 +105,28 @@ def test_argument_errors(H):
     assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), ctypes.c_void_p(wb.data_ptr()), n, s) == -3
     ws_.group = 64
     assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), P(ws), n, s) == -2
+
+
+@pytest.mark.parametrize("M", [1, 3])
+def test_long_rows_second_plane(H, M):
+    """321 groups per row: more salience words than the span kernel of the
+    second plane stages, so the per-tile kernel runs it."""
+    run_case(H, 96, 321 * 128, 0.1, M, f32=True, proj=21)
+
+
+def test_batched_many_row_lengths(H):
+    """A batch with more distinct plane-1 row lengths than tensor-map
+    templates per launch runs as consecutive sub-batches."""
+    from paper_2609_09240_gb300 import tq
+    items, refs = [], []
+    for i in range(11):
+        N, K = 64 + 32 * i, 128 * (i + 1)
+        w = wl.gen_weights(N, K, 0.2, config=6, proj=30 + i)
+        x = wl.gen_x(1, K, config=6, proj=30 + i)
+        refs.append(H.oracle_ref(w, x))
+        items.append((H.pack_on_gpu(w), H.dev(x), torch.empty((1, N), dtype=torch.float16, device="cuda")))
+    b = tq.Batch(1, items)
+    tq.tq_linear_batched(b)
+    H.device_status_ok()
+    for (pw, xd, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
