@@ -97,6 +97,9 @@ typedef struct {
   const uint16_t *offset;   /* fp16 bits [N][G]                                */
   const uint16_t *scale2;   /* fp16 bits [nnz]; may be NULL when nnz == 0      */
   int64_t nnz;              /* number of salient groups = rowptr[N]            */
+  const int32_t *p2index;   /* optional: tq_plane2_index of this weight, or
+                               NULL (the decode path then groups the second
+                               plane itself on every call)                     */
 } tq_weight;
 
 /* Bytes of one packed plane-1 row: roundup(26 * K / 128, 16).  0 if K is not
@@ -111,6 +114,25 @@ TQ_API size_t tq_sal_words(int32_t K);
  * *d_status and those bits are not counted. */
 TQ_API tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, int32_t *rowptr,
                              uint32_t *d_status, void *stream);
+
+/* Second-plane index (no counterpart in the paper; a layout aid for the
+ * decode path, M <= 8).  The salient (row, group) pairs of a weight listed
+ * group by group: int32 colptr[G + 1] (group g's entries are colptr[g] ..
+ * colptr[g+1] - 1), then, from int32 offset tq_plane2_index_rec_offset(K),
+ * rec[nnz] (each entry's plane-2 record index j = rowptr[n] + rank of g
+ * among row n's salient groups), then, from offset
+ * tq_plane2_index_row_offset(K, nnz), row[nnz] (its row n); within a group
+ * the entries follow increasing n.  It depends on the salience map only, so
+ * it is built once per weight; with it tq_linear runs the second plane one
+ * group at a time without grouping the records first.
+ *   index: device, tq_plane2_index_bytes(N, K, nnz) bytes, 16-byte aligned.
+ *   sal, rowptr as for tq_pack (rowptr[N] == nnz); bits at g >= K/128 are
+ *   ignored.  Asynchronous on stream. */
+TQ_API size_t tq_plane2_index_bytes(int32_t N, int32_t K, int64_t nnz);
+TQ_API size_t tq_plane2_index_rec_offset(int32_t K);
+TQ_API size_t tq_plane2_index_row_offset(int32_t K, int64_t nnz);
+TQ_API tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
+                                 int32_t *index, void *stream);
 
 /* Pack int8 trit codes into the lattice format (paper "Packing").
  *   T1: int8 [N][K] in {-1,0,+1};  T2: int8 [N][K], nonzero only where the

@@ -15,6 +15,8 @@ cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t
 cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                         const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
                         cudaStream_t s);
+cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
+                                cudaStream_t s);
 cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s);
@@ -57,6 +59,7 @@ tq_status check_weight(const tq_weight *w, int32_t N, int32_t K) {
   if (w->nnz > 0 && (!w->plane2 || !w->scale2)) return TQ_ERR_NULL;
   if (!aligned16(w->plane1)) return TQ_ERR_ALIGN;
   if (w->plane2 && !aligned16(w->plane2)) return TQ_ERR_ALIGN;
+  if (w->p2index && !aligned16(w->p2index)) return TQ_ERR_ALIGN;
   if (!aligned2(w->scale1) || !aligned2(w->offset) ||
       (w->scale2 && !aligned2(w->scale2)) || ((uintptr_t)w->salience & 3u) ||
       ((uintptr_t)w->rowptr & 3u))
@@ -71,6 +74,7 @@ Problem to_problem(const tq_weight *w, const uint16_t *x, void *y) {
   P.sal = w->salience;
   P.rowptr = w->rowptr;
   P.plane2 = w->plane2;
+  P.p2idx = w->nnz > 0 ? w->p2index : nullptr;
   P.s1 = reinterpret_cast<const __half *>(w->scale1);
   P.off = reinterpret_cast<const __half *>(w->offset);
   P.s2 = reinterpret_cast<const __half *>(w->scale2);
@@ -126,12 +130,12 @@ tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStr
       mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
       P.wsB = ws + off;
       P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
-      P.wsY2 = reinterpret_cast<float *>(ws + off + pad256(b) + pad256(cs));
-      P.wsMap = ws + off + pad256(b) + pad256(cs) + pad256(y2);
+      P.y2_off = (int32_t)(pad256(b) + pad256(cs));
+      P.map_off = (int32_t)(pad256(b) + pad256(cs) + pad256(y2));
     } else {
       P.wsB = ws + off;
       P.wsCS = reinterpret_cast<float *>(ws + off + tc_workspace_b_bytes(16, P.K));
-      P.wsY2 = nullptr;
+      P.y2_off = P.map_off = 0;
     }
     off += tot;
   }
@@ -201,6 +205,30 @@ tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *
   cudaStream_t s = (cudaStream_t)stream;
   if (tq_status st = from_cuda(launch_check_rowptr(N, K, sal, rowptr, d_status, s))) return st;
   return from_cuda(launch_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, s));
+}
+
+size_t tq_plane2_index_rec_offset(int32_t K) {
+  if (K < TQ_GROUP || K % TQ_GROUP) return 0;
+  return ((size_t)(K / TQ_GROUP) + 1 + 3) & ~(size_t)3;
+}
+
+size_t tq_plane2_index_row_offset(int32_t K, int64_t nnz) {
+  if (K < TQ_GROUP || K % TQ_GROUP || nnz < 0) return 0;
+  return tq_plane2_index_rec_offset(K) + (((size_t)nnz + 3) & ~(size_t)3);
+}
+
+size_t tq_plane2_index_bytes(int32_t N, int32_t K, int64_t nnz) {
+  if (check_shape(N, K) != TQ_OK || nnz < 0 || nnz > (int64_t)N * (K / TQ_GROUP)) return 0;
+  return 4 * (tq_plane2_index_row_offset(K, nnz) + (((size_t)nnz + 3) & ~(size_t)3));
+}
+
+tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
+                          void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!sal || !rowptr || !index) return TQ_ERR_NULL;
+  if (nnz < 0 || nnz > (int64_t)N * (K / TQ_GROUP)) return TQ_ERR_SALIENCE;
+  if ((uintptr_t)index & 15u) return TQ_ERR_ALIGN;
+  return from_cuda(launch_plane2_index(N, K, sal, rowptr, nnz, index, (cudaStream_t)stream));
 }
 
 size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K) {

@@ -217,6 +217,69 @@ __global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t
   }
 }
 
+// ------------------------------------------------------ second-plane index
+// One block per group g walks the rows in chunks of blockDim.x, in order;
+// a block-wide count (and, for the fill, an exclusive scan of the row bits)
+// gives each salient row its place in group g's list.
+constexpr int kIdxThreads = 256;
+
+__device__ __forceinline__ size_t p2index_rec_off(int K) { return ((size_t)(K / kGroup) + 1 + 3) & ~(size_t)3; }
+
+__global__ void __launch_bounds__(kIdxThreads) p2index_count_kernel(int N, int K, const uint32_t *sal,
+                                                                     int32_t *colptr) {
+  const int g = blockIdx.x, W = sal_words_of(K);
+  int total = 0;
+  for (int n0 = 0; n0 < N; n0 += kIdxThreads) {
+    const int n = n0 + threadIdx.x;
+    total += __syncthreads_count(n < N && sal_bit(sal, W, n, g));
+  }
+  if (threadIdx.x == 0) colptr[g + 1] = total;
+}
+
+__global__ void p2index_scan_kernel(int G, int32_t *colptr) {
+  if (threadIdx.x != 0) return;
+  colptr[0] = 0;
+  for (int g = 0; g < G; ++g) colptr[g + 1] += colptr[g];
+}
+
+__global__ void __launch_bounds__(kIdxThreads) p2index_fill_kernel(int N, int K, const uint32_t *sal,
+                                                                    const int32_t *rowptr, int64_t nnz,
+                                                                    int32_t *index) {
+  __shared__ int warp_base[kIdxThreads / 32 + 1];
+  const int g = blockIdx.x, W = sal_words_of(K);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int32_t *rec = index + p2index_rec_off(K);
+  int32_t *row = rec + ((nnz + 3) & ~(int64_t)3);
+  int base = index[g];
+  for (int n0 = 0; n0 < N; n0 += kIdxThreads) {
+    const int n = n0 + threadIdx.x;
+    const bool bit = n < N && sal_bit(sal, W, n, g);
+    const uint32_t m = __ballot_sync(0xffffffffu, bit);
+    if (lane == 0) warp_base[warp] = __popc(m);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int run = 0;
+      for (int w = 0; w < kIdxThreads / 32; ++w) {
+        const int c = warp_base[w];
+        warp_base[w] = run;
+        run += c;
+      }
+      warp_base[kIdxThreads / 32] = run;
+    }
+    __syncthreads();
+    if (bit) {
+      const int pos = base + warp_base[warp] + __popc(m & ((1u << lane) - 1u));
+      const int64_t j = (int64_t)rowptr[n] + sal_rank(sal, W, n, g);
+      if (pos < nnz) {  // within the index (entries beyond nnz, from a rowptr that disagrees, are dropped)
+        rec[pos] = (int32_t)min(max(j, (int64_t)0), nnz > 0 ? nnz - 1 : (int64_t)0);
+        row[pos] = n;
+      }
+    }
+    base += warp_base[kIdxThreads / 32];
+    __syncthreads();
+  }
+}
+
 // ------------------------------------------------------------- launchers
 static int grid_for(int64_t work, int block) {
   int64_t g = (work + block - 1) / block;
@@ -250,6 +313,15 @@ cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *pl
   int64_t total = (int64_t)N * row_bytes_of(K);
   unpack_kernel<<<grid_for(total, 256), 256, 0, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
                                                      status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
+                                cudaStream_t s) {
+  const int G = K / kGroup;
+  p2index_count_kernel<<<G, kIdxThreads, 0, s>>>(N, K, sal, index);
+  p2index_scan_kernel<<<1, 32, 0, s>>>(G, index);
+  p2index_fill_kernel<<<G, kIdxThreads, 0, s>>>(N, K, sal, rowptr, nnz, index);
   return cudaGetLastError();
 }
 

@@ -38,11 +38,14 @@ struct Problem {
   void *y;          // [M][N] fp16 or fp32
   unsigned char *wsB;  // workspace: activation slots of this problem
   float *wsCS;         // workspace: per-group C and S of this problem
-  float *wsY2;         // workspace: second-plane partial sums [N][M] (M <= 8 path)
-  void *wsMap;         // workspace: 128-byte tensor map of plane 1 (M <= 8 path)
+  const int32_t *p2idx;  // optional second-plane index (tq_plane2_index), or null
+  int32_t y2_off;      // workspace bytes from wsB: second-plane partial sums [N][M] (M <= 8 path)
+  int32_t map_off;     // workspace bytes from wsB: 128-byte tensor map of plane 1 (M <= 8 path)
   int32_t N, K;
   int32_t tile_begin;  // first global tile index of this problem
   int32_t nnz;         // plane-2 records (rowptr[N]); indices are clamped below it
+  __host__ __device__ float *y2() const { return reinterpret_cast<float *>(wsB + y2_off); }
+  __host__ __device__ void *map() const { return wsB + map_off; }
 };
 
 struct BatchParams {

@@ -300,21 +300,30 @@ struct MapTemplates {
 // B fragments, C and S for every (problem, group, token).  B layout of a
 // group: [token m][chunk pair cp][lane position c] x 16 B, each 16 B being
 // (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
-__global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ MapTemplates mt) {
+__global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ MapTemplates mt,
+                                     int32_t *unit_counter) {
   const int p = blockIdx.y;
   if (p >= bp.count) return;
   const Problem &P = bp.prob[p];
+  if (P.nnz > 0) {
+    // y2 starts at zero (the indexed second-plane kernel adds into it)
+    float *y2 = P.y2();
+    const int64_t n = (int64_t)P.N * bp.M;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+      y2[i] = 0.f;
+  }
+  if (p == 0 && blockIdx.x == 0 && threadIdx.x == 0 && unit_counter) *unit_counter = 0;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     // plane 1 as a 2-D byte tensor (row_bytes x N) for the main kernel's
     // stage copies: the template of its row length with this problem's
     // address and row count
     const uint4 *src = reinterpret_cast<const uint4 *>(&mt.t[mt.idx[p]]);
-    uint4 *dst = reinterpret_cast<uint4 *>(P.wsMap);
+    uint4 *dst = reinterpret_cast<uint4 *>(P.map());
 #pragma unroll
     for (int i = 0; i < 8; ++i) dst[i] = src[i];
-    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(P.wsMap), "l"(P.plane1)
+    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(P.map()), "l"(P.plane1)
                  : "memory");
-    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(P.wsMap), "r"((uint32_t)P.N)
+    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(P.map()), "r"((uint32_t)P.N)
                  : "memory");
     asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
   }
@@ -585,7 +594,7 @@ __global__ void __launch_bounds__(kP2Threads) gemv_mma_p2_kernel(const __grid_co
   }
   __syncthreads();
   if (valid) {
-    float *y2 = P.wsY2 + (int64_t)n * MB;
+    float *y2 = P.y2() + (int64_t)n * MB;
     for (int m = 0; m < MB; ++m) y2[m] = acc[t][m];
   }
 }
@@ -907,13 +916,123 @@ __global__ void __launch_bounds__(kQThreads, 1)
     __syncthreads();
     for (int i = tid; i < rows * MB; i += kQThreads) {
       const int r = ONE ? i : i / MB, m = ONE ? 0 : i - r * MB;
-      P.wsY2[(int64_t)(S.n0 + r) * MB + m] = acc[r * 8 + m];
+      P.y2()[(int64_t)(S.n0 + r) * MB + m] = acc[r * 8 + m];
       acc[r * 8 + m] = 0.f;
     }
     S = S1;
     S1 = S2;
   }
   cp_async_wait<0>();
+}
+
+// Second plane with the per-weight index (1..8 tokens).  Persistent warps
+// take (problem, group) units from a counter in the workspace (problems with
+// more records per group first); for its unit a warp loads group g's B
+// fragment and C once and runs the group's records in the index's order, 16
+// at a time as the rows of an m16 tile: each lane reads its two window words
+// of its two records straight from plane 2, decodes them with the
+// lane-replicated table, and s2 * (D - C) per record is added to y2 of the
+// record's row with a global atomic (the prep kernel zeroes y2).
+constexpr int kCThreads = 512;
+constexpr int kCDynBytes = kArena1 + kLutBytes;  // the table at its fixed address, nothing else
+struct CUnits {
+  int32_t base[TQ_MAX_BATCH + 1];  // units of order[0..i) (a unit per group)
+  uint8_t order[TQ_MAX_BATCH];     // problems with a second plane, most records per group first
+  int32_t count;                   // entries of order[]
+  int32_t *counter;                // the next unit (zeroed by the prep kernel)
+};
+
+// The 4 bytes at record-relative offset q (even, -2 <= q <= 28) of the record
+// starting at byte r0 of plane 2 (lim = its byte size).  Bytes outside the
+// record's 26 may be anything: the aligned words read are clamped to the
+// record's own, and the last word of plane 2 is read as 2 bytes when the
+// array ends inside it.
+__device__ __forceinline__ uint32_t rec_word(const uint8_t *plane2, int64_t r0, int q, int64_t lim) {
+  const int64_t a = r0 + q;
+  const int64_t lo = r0 & ~(int64_t)3, hi = (r0 + kGroupBytes - 1) & ~(int64_t)3;
+  const int64_t a0 = a & ~(int64_t)3;
+  const int64_t x0 = min(max(a0, lo), hi), x1 = min(max(a0 + 4, lo), hi);
+  const uint32_t w0 = x0 + 4 <= lim ? __ldg(reinterpret_cast<const uint32_t *>(plane2 + x0))
+                                    : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(plane2 + x0));
+  const uint32_t w1 = x1 + 4 <= lim ? __ldg(reinterpret_cast<const uint32_t *>(plane2 + x1))
+                                    : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(plane2 + x1));
+  return __funnelshift_r(w0, w1, (uint32_t)(a & 3) * 8u);
+}
+
+__global__ void __launch_bounds__(kCThreads, 1)
+    gemv_mma_p2c_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ CUnits un) {
+  extern __shared__ __align__(1024) unsigned char dync[];
+  const int tid = threadIdx.x, lane = tid & 31;
+  if (smem_u32(dync) != kDynShared) {
+    if (tid == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  {
+    uint32_t *lut = reinterpret_cast<uint32_t *>(dync + kArena1);
+    for (int i = tid; i < 256 * 32; i += kCThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+  }
+  __syncthreads();
+  const int MB = bp.M, g16 = lane >> 2, c = lane & 3;
+  const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
+  const int total = un.base[un.count];
+  for (;;) {
+    int u = 0;
+    if (lane == 0) u = atomicAdd(un.counter, 1);
+    u = __shfl_sync(0xffffffffu, u, 0);
+    if (u >= total) break;
+    int i = 0;  // the unit's entry: the last i with base[i] <= u
+    for (int step = 128; step >= 1; step >>= 1)
+      if (i + step < un.count && un.base[i + step] <= u) i += step;
+    const Problem &P = bp.prob[un.order[i]];
+    const int g = u - un.base[i], GL = g % kStageG;
+    const int G = P.K / kGroup;
+    const int64_t nnz = P.nnz;
+    const int32_t *colptr = P.p2idx;
+    const int32_t *recj = P.p2idx + ((G + 1 + 3) & ~3);
+    const int32_t *rown = recj + ((nnz + 3) & ~(int64_t)3);
+    const int k0 = (int)min(max((int64_t)__ldg(colptr + g), (int64_t)0), nnz);
+    const int k1 = (int)min(max((int64_t)__ldg(colptr + g + 1), (int64_t)k0), nnz);
+    if (k0 >= k1) continue;
+    // the group's B fragment (lanes of absent tokens repeat the last token) and C
+    const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB + min(g16, MB - 1) * kBTok + c * kBLane;
+    uint32_t b[20];
+#pragma unroll
+    for (int cp = 0; cp < kCP; ++cp) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg + cp * 4 * kBLane));
+      b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
+    }
+    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + 2 * c));
+    // lane c's window words: win_start + jw and + 4; the record starts o bytes into the window
+    const int q = 4 * ((c - win_start(GL)) & 3) - 2 * (GL & 1);
+    const int64_t lim = nnz * kGroupBytes;
+    float *y2 = P.y2();
+    for (int e0 = k0; e0 < k1; e0 += 16) {
+      uint32_t aL[20], aH[20];
+      int rowv[2];
+      float s2v[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int s = e0 + g16 + 8 * h;
+        const bool ok = s < k1;
+        const int64_t j = min(max((int64_t)__ldg(recj + (ok ? s : k0)), (int64_t)0), nnz - 1);
+        rowv[h] = ok ? __ldg(rown + s) : -1;
+        s2v[h] = __half2float(P.s2[j]);
+        const int64_t r0 = j * kGroupBytes;
+        decode_words(rec_word(P.plane2, r0, q, lim), rec_word(P.plane2, r0, q + 16, lim), tag, h ? aH : aL);
+      }
+      float d[4];
+      group_mma(aL, aH, b, d);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (rowv[h] < 0 || rowv[h] >= P.N) continue;
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+          const int m = 2 * c + ii;
+          if (m < MB) atomicAdd(&y2[(int64_t)rowv[h] * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+        }
+      }
+    }
+  }
 }
 
 // ------------------------------------------------------------------ main
@@ -1077,7 +1196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const int m = 2 * c + i;
                   if (m < M) {
                     float v = y[2 * h + i];
-                    if (P.nnz > 0) v += P.wsY2[(int64_t)n * MB + m];
+                    if (P.nnz > 0) v += P.y2()[(int64_t)n * MB + m];
                     if (F32)
                       static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
                     else
@@ -1114,7 +1233,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) {
         if (w.pi != map_pi) {
           // the problem's tensor map, written by the prep kernel
-          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(P.wsMap) : "memory");
+          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(P.map()) : "memory");
           map_pi = w.pi;
         }
         mbar_arrive_expect_tx(full, bb + cb + (uint32_t)kBytesSlot);
@@ -1126,7 +1245,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile(
             "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
                 smem_u32(bytes_buf((int)buf))),
-            "l"(P.wsMap), "r"(w.s * kStageBytes), "r"(n0), "r"(smem_u32(full))
+            "l"(P.map()), "r"(w.s * kStageBytes), "r"(n0), "r"(smem_u32(full))
             : "memory");
       }
       __syncwarp();
@@ -1235,7 +1354,8 @@ static bool plane1_template(int64_t rb, const void *plane1, int N, CUtensorMap *
   return true;
 }
 
-static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) <= 32764, "prep kernel parameters");
+static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) + 8 <= 32764, "prep kernel parameters");
+static_assert(sizeof(BatchParams) + sizeof(mm::CUnits) <= 32764, "indexed second-plane kernel parameters");
 static_assert(sizeof(BatchParams) + sizeof(mm::Sched) <= 32764, "main kernel parameters");
 
 // Distinct plane-1 row lengths of a batch (up to `cap` + 1 are counted).
@@ -1327,10 +1447,42 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
       mt.idx[i] = (uint8_t)k;
     }
   }
-  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt);
+  // second plane: the indexed kernel when every weight with a second plane
+  // has its index, else the span kernel (or, for rows of more than
+  // kQMaxW salience words, the per-tile one)
+  bool all_idx = true;
+  for (int i = 0; i < bp.count; ++i)
+    if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx) all_idx = false;
+  thread_local mm::CUnits un;
+  int32_t *counter = nullptr;
+  if (any2 && all_idx) {
+    // units (one per group) of the problems with a second plane, most records per group first
+    int n = 0;
+    for (int i = 0; i < bp.count; ++i)
+      if (bp.prob[i].nnz > 0) un.order[n++] = (uint8_t)i;
+    auto density = [&](int i) { return (double)bp.prob[i].nnz / (double)(bp.prob[i].K / kGroup); };
+    for (int a = 1; a < n; ++a)  // insertion sort by density, descending (stable)
+      for (int b2 = a; b2 > 0 && density(un.order[b2]) > density(un.order[b2 - 1]); --b2) {
+        const uint8_t t = un.order[b2];
+        un.order[b2] = un.order[b2 - 1];
+        un.order[b2 - 1] = t;
+      }
+    un.count = n;
+    un.base[0] = 0;
+    for (int a = 0; a < n; ++a) un.base[a + 1] = un.base[a] + bp.prob[un.order[a]].K / kGroup;
+    counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + 128);
+    un.counter = counter;
+  }
+  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (any2 && gmax <= mm::kQMaxG) {
+  if (any2 && all_idx) {
+    e = cudaFuncSetAttribute(mm::gemv_mma_p2c_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes);
+    if (e != cudaSuccess) return e;
+    mm::gemv_mma_p2c_kernel<<<ctas, mm::kCThreads, mm::kCDynBytes, s>>>(bp, un);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  } else if (any2 && gmax <= mm::kQMaxG) {
     auto kern = bp.M == 1 ? mm::gemv_mma_p2v3_kernel<true> : mm::gemv_mma_p2v3_kernel<false>;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kQDynBytes);
     if (e != cudaSuccess) return e;

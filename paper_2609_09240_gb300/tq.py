@@ -39,7 +39,7 @@ class tq_weight(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int32), ("K", ctypes.c_int32), ("group", ctypes.c_int32),
                 ("plane1", ctypes.c_void_p), ("salience", ctypes.c_void_p), ("rowptr", ctypes.c_void_p),
                 ("plane2", ctypes.c_void_p), ("scale1", ctypes.c_void_p), ("offset", ctypes.c_void_p),
-                ("scale2", ctypes.c_void_p), ("nnz", ctypes.c_int64)]
+                ("scale2", ctypes.c_void_p), ("nnz", ctypes.c_int64), ("p2index", ctypes.c_void_p)]
 
 
 class tq_problem(ctypes.Structure):
@@ -68,6 +68,15 @@ def lib():
             L.tq_salience_rowptr.argtypes = [i32, i32, vp, vp, vp, vp]
             L.tq_pack.restype = ctypes.c_int
             L.tq_pack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+            i64 = ctypes.c_int64
+            L.tq_plane2_index_bytes.restype = ctypes.c_size_t
+            L.tq_plane2_index_bytes.argtypes = [i32, i32, i64]
+            L.tq_plane2_index_rec_offset.restype = ctypes.c_size_t
+            L.tq_plane2_index_rec_offset.argtypes = [i32]
+            L.tq_plane2_index_row_offset.restype = ctypes.c_size_t
+            L.tq_plane2_index_row_offset.argtypes = [i32, i64]
+            L.tq_plane2_index.restype = ctypes.c_int
+            L.tq_plane2_index.argtypes = [i32, i32, vp, vp, i64, vp, vp]
             L.tq_unpack.restype = ctypes.c_int
             L.tq_unpack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             sz = ctypes.c_size_t
@@ -148,6 +157,16 @@ def tq_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, stream=None):
                            _stream(stream)), "tq_unpack")
 
 
+def tq_plane2_index(N, K, sal, rowptr, nnz, stream=None):
+    """The second-plane index of a weight (int32 device tensor), see tq.h."""
+    nbytes = int(lib().tq_plane2_index_bytes(N, K, nnz))
+    if nbytes == 0:
+        raise TQError(-2, "tq_plane2_index_bytes")
+    idx = torch.empty(nbytes // 4, dtype=torch.int32, device=sal.device)
+    _check(lib().tq_plane2_index(N, K, _p(sal), _p(rowptr), nnz, _p(idx), _stream(stream)), "tq_plane2_index")
+    return idx
+
+
 @dataclass
 class PackedWeight:
     """Device tensors of one packed projection (the fields of tq_weight)."""
@@ -161,6 +180,7 @@ class PackedWeight:
     offset: torch.Tensor   # fp16 [N][G]
     scale2: torch.Tensor | None   # fp16 [nnz]
     nnz: int
+    p2index: torch.Tensor | None = None  # int32, tq_plane2_index (optional)
 
     def struct(self) -> tq_weight:
         w = tq_weight()
@@ -173,6 +193,7 @@ class PackedWeight:
         w.offset = self.offset.data_ptr()
         w.scale2 = self.scale2.data_ptr() if self.scale2 is not None and self.nnz > 0 else None
         w.nnz = self.nnz
+        w.p2index = self.p2index.data_ptr() if self.p2index is not None and self.nnz > 0 else None
         return w
 
     def packed_bytes(self) -> int:
@@ -183,8 +204,9 @@ class PackedWeight:
         return sum(x.numel() * x.element_size() for x in t)
 
 
-def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True) -> PackedWeight:
-    """Pack device int8 codes + fp16 params with tq_salience_rowptr + tq_pack.
+def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True, index=True) -> PackedWeight:
+    """Pack device int8 codes + fp16 params with tq_salience_rowptr + tq_pack
+    (and, unless index=False, the second-plane index).
 
     Reads nnz back to the host (one synchronization) to size plane 2."""
     N, K = T1.shape
@@ -202,7 +224,8 @@ def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True) -> PackedWeig
             raise TQError(-4, f"tq_pack data status {st:#x}")
     if s2 is None or nnz == 0:
         s2 = torch.zeros(1, dtype=torch.float16, device=dev)
-    return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz)
+    p2index = tq_plane2_index(N, K, sal, rowptr, nnz, stream) if index and nnz > 0 else None
+    return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz, p2index)
 
 
 def tq_workspace_bytes(M: int, N: int, K: int) -> int:

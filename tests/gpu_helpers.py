@@ -19,9 +19,9 @@ def dev(a: np.ndarray, dtype=None):
     return t if dtype is None else t.to(dtype)
 
 
-def pack_on_gpu(w: wl.Weights) -> tq.PackedWeight:
+def pack_on_gpu(w: wl.Weights, index=True) -> tq.PackedWeight:
     return tq.pack_weight(dev(w.T1), dev(w.T2), dev(w.sal), dev(w.s1), dev(w.off),
-                          dev(w.s2) if w.nnz else None)
+                          dev(w.s2) if w.nnz else None, index=index)
 
 
 def oracle_ref(w: wl.Weights, x_bits: np.ndarray, rows=None, nthreads=None):

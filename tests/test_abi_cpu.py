@@ -59,4 +59,10 @@ def test_host_side_argument_errors_without_gpu():
     assert tq.tq_workspace_bytes(16, 4096, 4096) == 32 * (5120 + 128)
     assert tq.tq_workspace_bytes(40, 64, 4096) == 256
     assert tq.tq_workspace_bytes(1, 4096, 100) == 0
+    # second-plane index: colptr (G + 1, padded to 4), rec and row (each nnz, padded to 4), int32
+    L = tq.lib()
+    assert L.tq_plane2_index_rec_offset(4096) == 36
+    assert L.tq_plane2_index_row_offset(4096, 13) == 36 + 16
+    assert L.tq_plane2_index_bytes(100, 4096, 13) == 4 * (36 + 16 + 16)
+    assert L.tq_plane2_index_bytes(100, 4096, 100 * 32 + 1) == 0  # more records than groups
     assert tq.tq_workspace_bytes(1, 0, 4096) == 0

@@ -120,3 +120,28 @@ def test_large_rowptr(H):
     rp = torch.empty(N + 1, dtype=torch.int32, device="cuda")
     tq.tq_salience_rowptr(N, K, H.dev(sal), rp, status)
     assert np.array_equal(rp.cpu().numpy(), rp_o)
+
+
+@pytest.mark.parametrize("N,K,frac", [s for s in SHAPES if s[2] > 0] + [(1000, 41088, 0.05)])
+def test_plane2_index_bit_exact(H, N, K, frac):
+    """The second-plane index lists, group by group and in row order, each
+    salient (row, group) pair's record j = rowptr[n] + rank and its row n."""
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, frac, config=7, proj=3 * N + K)
+    G = K // 128
+    rp, st = oracle.rowptr(N, K, w.sal)
+    assert st == 0
+    nnz = int(rp[N])
+    idx = tq.tq_plane2_index(N, K, H.dev(w.sal), H.dev(rp), nnz).cpu().numpy()
+    bits = ((w.sal[:, np.arange(G) // 32] >> (np.arange(G) % 32)) & 1).astype(bool)  # [N][G]
+    rank = np.cumsum(bits, axis=1) - bits  # salient groups of the row before g
+    colptr = np.concatenate([[0], np.cumsum(bits.sum(axis=0))]).astype(np.int64)
+    ro = int(tq.lib().tq_plane2_index_rec_offset(K))
+    wo = int(tq.lib().tq_plane2_index_row_offset(K, nnz))
+    assert ro >= G + 1 and ro % 4 == 0 and wo >= ro + nnz and wo % 4 == 0
+    np.testing.assert_array_equal(idx[:G + 1], colptr)
+    rows = np.concatenate([np.nonzero(bits[:, g])[0] for g in range(G)]) if nnz else np.zeros(0, np.int64)
+    recs = np.concatenate([rp[np.nonzero(bits[:, g])[0]] + rank[bits[:, g], g] for g in range(G)]) if nnz \
+        else np.zeros(0, np.int64)
+    np.testing.assert_array_equal(idx[wo:wo + nnz], rows)
+    np.testing.assert_array_equal(idx[ro:ro + nnz], recs)

@@ -15,12 +15,12 @@ def H():
     return gpu_helpers
 
 
-def run_case(H, N, K, frac, M, f32, proj=0, config=6):
+def run_case(H, N, K, frac, M, f32, proj=0, config=6, index=True):
     from paper_2609_09240_gb300 import tq
     w = wl.gen_weights(N, K, frac, config=config, proj=proj)
     x = wl.gen_x(M, K, config=config, proj=proj)
     y_ref, a_ref = H.oracle_ref(w, x)
-    pw = H.pack_on_gpu(w)
+    pw = H.pack_on_gpu(w, index=index)
     xd = H.dev(x)
     y = (tq.tq_linear_f32out if f32 else tq.tq_linear)(xd, pw)
     H.device_status_ok()
@@ -130,3 +130,11 @@ def test_batched_many_row_lengths(H):
     H.device_status_ok()
     for (pw, xd, y), (y_ref, a_ref) in zip(items, refs):
         H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("N,K,frac", [(1, 128, 1.0), (129, 256, 0.5), (300, 9728, 0.1), (700, 4096, 0.3)])
+@pytest.mark.parametrize("M", [1, 3, 8])
+def test_second_plane_without_index(H, N, K, frac, M):
+    """Weights packed without the second-plane index: the span kernel groups
+    the records itself."""
+    run_case(H, N, K, frac, M, f32=True, proj=40 + N, index=False)
