@@ -934,7 +934,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
 // lane-replicated table, and s2 * (D - C) per record is added to y2 of the
 // record's row with a global atomic (the prep kernel zeroes y2).
 constexpr int kCThreads = 512;
-constexpr int kCDynBytes = kArena1 + kLutBytes;  // the table at its fixed address, nothing else
+
 struct CUnits {
   int32_t base[TQ_MAX_BATCH + 1];  // units of order[0..i) (a unit per group)
   uint8_t order[TQ_MAX_BATCH];     // problems with a second plane, most records per group first
@@ -942,23 +942,28 @@ struct CUnits {
   int32_t *counter;                // the next unit (zeroed by the prep kernel)
 };
 
-// The 4 bytes at record-relative offset q (even, -2 <= q <= 28) of the record
-// starting at byte r0 of plane 2 (lim = its byte size).  Bytes outside the
-// record's 26 may be anything: the aligned words read are clamped to the
-// record's own, and the last word of plane 2 is read as 2 bytes when the
-// array ends inside it.
-__device__ __forceinline__ uint32_t rec_word(const uint8_t *plane2, int64_t r0, int q, int64_t lim) {
-  const int64_t a = r0 + q;
-  const int64_t lo = r0 & ~(int64_t)3, hi = (r0 + kGroupBytes - 1) & ~(int64_t)3;
-  const int64_t a0 = a & ~(int64_t)3;
-  const int64_t x0 = min(max(a0, lo), hi), x1 = min(max(a0 + 4, lo), hi);
-  const uint32_t w0 = x0 + 4 <= lim ? __ldg(reinterpret_cast<const uint32_t *>(plane2 + x0))
-                                    : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(plane2 + x0));
-  const uint32_t w1 = x1 + 4 <= lim ? __ldg(reinterpret_cast<const uint32_t *>(plane2 + x1))
-                                    : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(plane2 + x1));
-  return __funnelshift_r(w0, w1, (uint32_t)(a & 3) * 8u);
+// Per-warp staging in shared memory: a chunk of the group's index entries
+// (record index j, row n), and a ring of kCDepth tiles of record words: for
+// each lane its two records' aligned words around its two window words and
+// the 4-byte word holding each record's s2 (10 words).
+constexpr int kCWarps = kCThreads / 32;
+constexpr int kCChunk = 256;                        // index entries per chunk
+constexpr int kCIdxWords = kCChunk + 4;             // + the start rounded down to 4 entries
+constexpr int kCDepth = 3;                          // m16 tiles in flight per warp
+constexpr int kCRing = kCDepth * 32 * 10;           // words
+constexpr int kCIdxOff = 0;                         // per warp: j[kCIdxWords], n[kCIdxWords] (below the table)
+constexpr int kCRingOff = kArena1 + kLutBytes;      // per warp: the ring (above the table)
+static_assert(kCIdxOff + kCWarps * 2 * kCIdxWords * 4 <= kArena1, "index chunks overflow");
+constexpr int kCDynBytes2 = kCRingOff + kCWarps * kCRing * 4;
+static_assert(kCDynBytes2 <= kDynBytes, "record rings overflow");
+
+// One aligned 4-byte word of plane 2 into the ring (`bytes` = 2 for the last
+// word of plane 2 when the array ends inside it).
+__device__ __forceinline__ void c_copy_word(uint32_t *dst, const uint8_t *src, int bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(bytes) : "memory");
 }
 
+template <bool ONE>
 __global__ void __launch_bounds__(kCThreads, 1)
     gemv_mma_p2c_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ CUnits un) {
   extern __shared__ __align__(1024) unsigned char dync[];
@@ -972,9 +977,12 @@ __global__ void __launch_bounds__(kCThreads, 1)
     for (int i = tid; i < 256 * 32; i += kCThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
   }
   __syncthreads();
-  const int MB = bp.M, g16 = lane >> 2, c = lane & 3;
+  const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, warp = tid >> 5;
   const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
   const int total = un.base[un.count];
+  int32_t *idx_j = reinterpret_cast<int32_t *>(dync + kCIdxOff) + warp * 2 * kCIdxWords;
+  int32_t *idx_n = idx_j + kCIdxWords;
+  uint32_t *ring = reinterpret_cast<uint32_t *>(dync + kCRingOff) + warp * kCRing;
   for (;;) {
     int u = 0;
     if (lane == 0) u = atomicAdd(un.counter, 1);
@@ -1004,33 +1012,106 @@ __global__ void __launch_bounds__(kCThreads, 1)
     const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + 2 * c));
     // lane c's window words: win_start + jw and + 4; the record starts o bytes into the window
     const int q = 4 * ((c - win_start(GL)) & 3) - 2 * (GL & 1);
-    const int64_t lim = nnz * kGroupBytes;
     float *y2 = P.y2();
-    for (int e0 = k0; e0 < k1; e0 += 16) {
-      uint32_t aL[20], aH[20];
-      int rowv[2];
-      float s2v[2];
+    const int64_t nidx4 = (nnz + 3) & ~(int64_t)3;  // entries of each index array, as allocated
+    const bool s2_al = (reinterpret_cast<uintptr_t>(P.s2) & 3u) == 0;
+    const int nnz32 = (int)nnz;  // plane 2 of this path is below 2^31 bytes (the launcher checks)
+    // record j starts d = 2 (j & 1) bytes into a word (plane 2 is 16-byte aligned); the
+    // aligned words around the lane's window words, at record-relative offsets x .. x + 20,
+    // clamped onto the words holding the record's bytes (the others meet zero
+    // activations, so the copies stay inside the record): per parity of j
+    int xo[2][4];
+    uint32_t shp[2];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int s = e0 + g16 + 8 * h;
-        const bool ok = s < k1;
-        const int64_t j = min(max((int64_t)__ldg(recj + (ok ? s : k0)), (int64_t)0), nnz - 1);
-        rowv[h] = ok ? __ldg(rown + s) : -1;
-        s2v[h] = __half2float(P.s2[j]);
-        const int64_t r0 = j * kGroupBytes;
-        decode_words(rec_word(P.plane2, r0, q, lim), rec_word(P.plane2, r0, q + 16, lim), tag, h ? aH : aL);
+    for (int par = 0; par < 2; ++par) {
+      const int d = 2 * par, x = q - ((q + d) & 3);
+      shp[par] = (uint32_t)((q + d) & 3) * 8u;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) xo[par][k] = min(max(x + 4 * (k & 1) + 16 * (k >> 1), -d), 24 - d);
+    }
+    for (int c0 = k0; c0 < k1; c0 += kCChunk) {
+      const int c1 = min(c0 + kCChunk, k1);
+      // the chunk's entries, from the 4-entry boundary at or below c0
+      const int a0 = c0 & ~3;
+      const int nch = (int)min((int64_t)(c1 - a0 + 3) / 4, (nidx4 - a0) / 4);
+      for (int k = lane; k < nch; k += 32) {
+        cp_async16(idx_j + 4 * k, recj + a0 + 4 * k);
+        cp_async16(idx_n + 4 * k, rown + a0 + 4 * k);
       }
-      float d[4];
-      group_mma(aL, aH, b, d);
+      cp_async_commit();
+      cp_async_wait<0>();
+      __syncwarp();
+      // tile t of the chunk covers entries c0 + 16 t .. + 15; lane slots g16, g16 + 8
+      const int ntiles = (c1 - c0 + 15) / 16;
+      auto issue = [&](int t) {
+        if (t < ntiles) {
+          uint32_t *dst = ring + ((t % kCDepth) * 32 + lane) * 10;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (rowv[h] < 0 || rowv[h] >= P.N) continue;
+          for (int h = 0; h < 2; ++h) {
+            const int e = c0 + 16 * t + g16 + 8 * h;
+            const int j = min(max(idx_j[(e < c1 ? e : c0) - a0], 0), nnz32 - 1);
+            const uint8_t *rec = P.plane2 + (uint32_t)j * (uint32_t)kGroupBytes;
+            const int par = j & 1;
+            const bool tail = par == 0 && j == nnz32 - 1;  // its last aligned word ends 2 bytes past plane 2
 #pragma unroll
-        for (int ii = 0; ii < 2; ++ii) {
-          const int m = 2 * c + ii;
-          if (m < MB) atomicAdd(&y2[(int64_t)rowv[h] * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+            for (int k = 0; k < 4; ++k) {
+              const int x = par ? xo[1][k] : xo[0][k];
+              c_copy_word(dst + 5 * h + k, rec + x, (tail && x == 24) ? 2 : 4);
+            }
+            if (s2_al) {
+              // the 4-byte word holding s2[j] (2 bytes of it past the end of s2 when j is the last, even)
+              asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst + 5 * h + 4)),
+                           "l"(P.s2 + (j & ~1)), "r"((j | 1) < nnz32 ? 4 : 2)
+                           : "memory");
+            }
+          }
+        }
+        cp_async_commit();
+      };
+#pragma unroll
+      for (int t = 0; t < kCDepth - 1; ++t) issue(t);
+      for (int t = 0; t < ntiles; ++t) {
+        issue(t + kCDepth - 1);
+        cp_async_wait<kCDepth - 1>();  // this lane's copies of tile t
+        const uint32_t *src = ring + ((t % kCDepth) * 32 + lane) * 10;
+        uint32_t aL[20], aH[20];
+        int rowv[2];
+        float s2v[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int e = c0 + 16 * t + g16 + 8 * h;
+          const int j = min(max(idx_j[(e < c1 ? e : c0) - a0], 0), nnz32 - 1);
+          rowv[h] = e < c1 ? idx_n[e - a0] : -1;
+          const uint32_t sh = (j & 1) ? shp[1] : shp[0];
+          const uint32_t w0 = __funnelshift_r(src[5 * h], src[5 * h + 1], sh);
+          const uint32_t w1 = __funnelshift_r(src[5 * h + 2], src[5 * h + 3], sh);
+          if (s2_al) {
+            const uint32_t s2w = src[5 * h + 4];
+            s2v[h] = __half2float(__ushort_as_half((unsigned short)((j & 1) ? s2w >> 16 : s2w & 0xffffu)));
+          } else {
+            s2v[h] = __half2float(P.s2[j]);  // s2 not 4-byte aligned: read in place
+          }
+          decode_words(w0, w1, tag, h ? aH : aL);
+        }
+        float d[4];
+        group_mma(aL, aH, b, d);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int n = rowv[h];
+          if (n < 0 || n >= P.N) continue;
+          if (ONE) {
+            if (c == 0) atomicAdd(&y2[n], s2v[h] * (d[2 * h] - Cv.x));
+          } else {
+#pragma unroll
+            for (int ii = 0; ii < 2; ++ii) {
+              const int m = 2 * c + ii;
+              if (m < MB) atomicAdd(&y2[(int64_t)n * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+            }
+          }
         }
       }
+      cp_async_wait<0>();
+      __syncwarp();  // the chunk's entries are read before the next chunk is staged
     }
   }
 }
@@ -1452,7 +1533,8 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   // kQMaxW salience words, the per-tile one)
   bool all_idx = true;
   for (int i = 0; i < bp.count; ++i)
-    if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx) all_idx = false;
+    if (bp.prob[i].nnz > 0 && (!bp.prob[i].p2idx || bp.prob[i].nnz * (int64_t)kGroupBytes >= ((int64_t)1 << 31)))
+      all_idx = false;
   thread_local mm::CUnits un;
   int32_t *counter = nullptr;
   if (any2 && all_idx) {
@@ -1477,9 +1559,10 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (any2 && all_idx) {
-    e = cudaFuncSetAttribute(mm::gemv_mma_p2c_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes);
+    auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true> : mm::gemv_mma_p2c_kernel<false>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
-    mm::gemv_mma_p2c_kernel<<<ctas, mm::kCThreads, mm::kCDynBytes, s>>>(bp, un);
+    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(bp, un);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   } else if (any2 && gmax <= mm::kQMaxG) {

@@ -138,3 +138,22 @@ def test_second_plane_without_index(H, N, K, frac, M):
     """Weights packed without the second-plane index: the span kernel groups
     the records itself."""
     run_case(H, N, K, frac, M, f32=True, proj=40 + N, index=False)
+
+
+@pytest.mark.parametrize("M", [1, 4])
+def test_second_plane_scale2_two_byte_aligned(H, M):
+    """s2 is only required to be 2-byte aligned: a view starting 2 bytes
+    into an allocation takes the in-place read of the indexed kernel."""
+    from paper_2609_09240_gb300 import tq
+    N, K = 300, 4096
+    w = wl.gen_weights(N, K, 0.2, config=6, proj=77)
+    x = wl.gen_x(M, K, config=6, proj=77)
+    y_ref, a_ref = H.oracle_ref(w, x)
+    pw = H.pack_on_gpu(w)
+    buf = torch.empty(pw.nnz + 1, dtype=torch.float16, device="cuda")
+    buf[1:] = pw.scale2[:pw.nnz]
+    pw.scale2 = buf[1:]
+    assert pw.scale2.data_ptr() % 4 == 2
+    y = tq.tq_linear_f32out(H.dev(x), pw)
+    H.device_status_ok()
+    H.assert_close(y.cpu().numpy(), y_ref, a_ref)
