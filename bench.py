@@ -459,6 +459,8 @@ def main():
                    "model": "Qwen3-8B projection shapes, random ternary weights", "global_batch": args.M * ws,
                    "seq_len": 1, "parallelism": f"replicas x{ws}" if ws > 1 else "none",
                    "packed_bytes_per_step": packed_bytes, "weights_per_step": n_weights,
+                   "p2index_bytes_per_step": sum(pw.p2index.numel() * 4 for pw, _, _ in items
+                                                 if pw.p2index is not None),
                    "l2": "no flush: 1.79 GB of packed weights per step > 129 MB L2"},
         "tokens_per_s": ws * args.M / (ms_per_step * 1e-3),
         "us_per_step": ms_per_step * 1e3,
@@ -466,8 +468,8 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
                      "traffic": ncu_traffic(),
-                     "kernel": "decode step: activation prep + second plane + first plane "
-                               "(3 launches per step, timed together; the first-plane kernel is ~70 % of it)",
+                     "kernel": "decode step: activation prep + second plane (per-weight index) + first plane "
+                               "(3 launches per step, timed together; the first-plane kernel is ~75 % of it)",
                      "launch_ms_avg": launch_avg},
         "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},
