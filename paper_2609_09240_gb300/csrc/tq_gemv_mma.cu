@@ -950,7 +950,8 @@ constexpr int kCWarps = kCThreads / 32;
 constexpr int kCChunk = 256;                        // index entries per chunk
 constexpr int kCIdxWords = kCChunk + 4;             // + the start rounded down to 4 entries
 constexpr int kCDepth = 3;                          // m16 tiles in flight per warp
-constexpr int kCRing = kCDepth * 32 * 10;           // words
+constexpr int kCLaneWords = 11;                     // 10 used; odd, so the lanes' reads hit 32 banks
+constexpr int kCRing = kCDepth * 32 * kCLaneWords;  // words
 constexpr int kCIdxOff = 0;                         // per warp: j[kCIdxWords], n[kCIdxWords] (below the table)
 constexpr int kCRingOff = kArena1 + kLutBytes;      // per warp: the ring (above the table)
 static_assert(kCIdxOff + kCWarps * 2 * kCIdxWords * 4 <= kArena1, "index chunks overflow");
@@ -1045,7 +1046,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
       const int ntiles = (c1 - c0 + 15) / 16;
       auto issue = [&](int t) {
         if (t < ntiles) {
-          uint32_t *dst = ring + ((t % kCDepth) * 32 + lane) * 10;
+          uint32_t *dst = ring + ((t % kCDepth) * 32 + lane) * kCLaneWords;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int e = c0 + 16 * t + g16 + 8 * h;
@@ -1073,7 +1074,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
       for (int t = 0; t < ntiles; ++t) {
         issue(t + kCDepth - 1);
         cp_async_wait<kCDepth - 1>();  // this lane's copies of tile t
-        const uint32_t *src = ring + ((t % kCDepth) * 32 + lane) * 10;
+        const uint32_t *src = ring + ((t % kCDepth) * 32 + lane) * kCLaneWords;
         uint32_t aL[20], aH[20];
         int rowv[2];
         float s2v[2];
@@ -1117,12 +1118,12 @@ __global__ void __launch_bounds__(kCThreads, 1)
 }
 
 // ------------------------------------------------------------------ main
-template <bool F32>
+template <bool F32, bool ONE>
 __global__ void __launch_bounds__(kThreads, 1)
     gemv_mma_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
   extern __shared__ __align__(1024) unsigned char dyn[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int M = bp.M, MB = bp.M;
+  const int M = ONE ? 1 : bp.M, MB = M;
   if (smem_u32(dyn) != kDynShared) {
     // the table address trick needs the dynamic window right after the
     // reserved 1 KiB of shared memory; anything else is reported
@@ -1185,6 +1186,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         // s1 / off / C / S of group GL applied to its accumulators d
         auto epilogue = [&](auto glc, const float *d) {
           constexpr int GL = decltype(glc)::value;
+          if (ONE) {
+            // one token: only column 0 (lanes c = 0) is ever written
+            const float Cx = CSst[GL * 16 + 2 * c], Sx = CSst[GL * 16 + 8 + 2 * c];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
+              const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
+              const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+              y[2 * h] = fmaf(s1, d[2 * h] - Cx, fmaf(of, Sx, y[2 * h]));
+            }
+            return;
+          }
           const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
           const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
 #pragma unroll
@@ -1577,9 +1590,10 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  e = cudaFuncSetAttribute(mm::gemv_mma_kernel<F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kDynBytes);
+  auto main_kern = bp.M == 1 ? mm::gemv_mma_kernel<F32, true> : mm::gemv_mma_kernel<F32, false>;
+  e = cudaFuncSetAttribute(main_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kDynBytes);
   if (e != cudaSuccess) return e;
-  mm::gemv_mma_kernel<F32><<<ctas, mm::kThreads, mm::kDynBytes, s>>>(bp, sc);
+  main_kern<<<ctas, mm::kThreads, mm::kDynBytes, s>>>(bp, sc);
   return cudaGetLastError();
 }
 
