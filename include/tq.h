@@ -159,9 +159,9 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
  * activations of every call are first rearranged into the tensor-core
  * operand order of the packed weights (with the per-group correction terms),
  * and for M <= 8 the second plane's fp32 partial sums of every row are
- * staged there before the first plane is streamed, next to a 128-byte
- * descriptor through which the first plane is copied into shared memory
- * (one per projection, written by the same call).  The caller provides this
+ * staged there before the first plane is streamed, next to the 128-byte
+ * descriptors through which the first plane, s1 and off are copied into
+ * shared memory (written by the same call).  The caller provides this
  * scratch memory (the library never allocates).  Bytes needed for one
  * projection of N rows, K inputs and M tokens; a call with M > 16 (the
  * prefill tile path) uses none and the function returns 256 for it; 0 if M,

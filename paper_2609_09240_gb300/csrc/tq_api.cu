@@ -93,7 +93,7 @@ size_t problem_ws_bytes(int M, int N, int K) {
   if (M <= 8) {
     size_t b, cs, y2;
     mma_workspace_parts(M, N, K, &b, &cs, &y2);
-    return pad256(b) + pad256(cs) + pad256(y2) + 256;  // + the plane-1 tensor map
+    return pad256(b) + pad256(cs) + pad256(y2) + 512;  // + the tensor maps of plane 1, s1, off
   }
   return pad256(tc_workspace_bytes(16, K));
 }

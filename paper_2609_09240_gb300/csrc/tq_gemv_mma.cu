@@ -287,14 +287,22 @@ struct Walk {
   }
 };
 
-// Tensor-map templates of plane 1, one per distinct row length in a batch
-// (encoded on the host for that row length and stride); idx[p] picks
-// problem p's.
-constexpr int kMaxMapTemplates = 8;
+// Tensor-map templates, one per distinct (tensor kind, row length, row
+// count) in a batch, encoded on the host; idx[p] / idx_so[p] pick problem
+// p's.  The prep kernel only puts in the problem's address: a template
+// encoded for the same sizes then equals the host encoding byte for byte.
+constexpr int kMaxMapTemplates = 10;
+constexpr uint8_t kNoMap = 255;
 struct MapTemplates {
   CUtensorMap t[kMaxMapTemplates];
-  uint8_t idx[TQ_MAX_BATCH];
+  uint8_t idx[TQ_MAX_BATCH];    // plane 1's template
+  uint8_t idx_so[TQ_MAX_BATCH];  // s1's and off's template, or kNoMap (then asynchronous copies)
 };
+// Workspace slot of a problem's tensor maps: plane 1, s1, off, then the
+// indexed second-plane kernel's unit counter.
+constexpr int kMapSlotBytes = 512;
+constexpr int kMapS1 = 128, kMapOff = 256, kCounterOff = 384;
+static_assert(kCounterOff + 4 <= kMapSlotBytes, "map slot");
 
 // ------------------------------------------------------------------ prep
 // B fragments, C and S for every (problem, group, token).  B layout of a
@@ -315,16 +323,21 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   if (p == 0 && blockIdx.x == 0 && threadIdx.x == 0 && unit_counter) *unit_counter = 0;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     // plane 1 as a 2-D byte tensor (row_bytes x N) for the main kernel's
-    // stage copies: the template of its row length with this problem's
-    // address and row count
-    const uint4 *src = reinterpret_cast<const uint4 *>(&mt.t[mt.idx[p]]);
-    uint4 *dst = reinterpret_cast<uint4 *>(P.map());
+    // stage copies: the template of its sizes with this problem's address
+    auto build = [&](unsigned char *m, int t, const void *addr) {
+      const uint4 *src = reinterpret_cast<const uint4 *>(&mt.t[t]);
+      uint4 *dst = reinterpret_cast<uint4 *>(m);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) dst[i] = src[i];
-    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(P.map()), "l"(P.plane1)
-                 : "memory");
-    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(P.map()), "r"((uint32_t)P.N)
-                 : "memory");
+      for (int i = 0; i < 8; ++i) dst[i] = src[i];
+      asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(m), "l"(addr) : "memory");
+    };
+    unsigned char *m = static_cast<unsigned char *>(P.map());
+    build(m, mt.idx[p], P.plane1);
+    if (mt.idx_so[p] != kNoMap) {
+      // s1 and off as 2-D fp16 tensors (G x N), for the stage copies of their 8 groups
+      build(m + kMapS1, mt.idx_so[p], P.s1);
+      build(m + kMapOff, mt.idx_so[p], P.off);
+    }
     asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
   }
   const int MB = bp.M;
@@ -1324,13 +1337,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) ok = wait_or_abort(&bars->empty[buf], phase ^ 1u, abort_) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
       uint64_t *full = &bars->full[buf];
+      // s1 / off go by tensor copies when their rows are whole 16-byte units
+      // (the prep kernel then built their maps), else by asynchronous copies
+      const int G = P.K / kGroup;
+      const bool so_map = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+      unsigned char *so = ar2 + L.oSO + buf * kSOSlot;
+      const unsigned char *maps = static_cast<const unsigned char *>(P.map());
       if (lane == 0) {
         if (w.pi != map_pi) {
-          // the problem's tensor map, written by the prep kernel
-          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(P.map()) : "memory");
+          // the problem's tensor maps, written by the prep kernel
+          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps) : "memory");
+          if (so_map) {
+            asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + kMapS1) : "memory");
+            asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + kMapOff) : "memory");
+          }
           map_pi = w.pi;
         }
-        mbar_arrive_expect_tx(full, bb + cb + (uint32_t)kBytesSlot);
+        mbar_arrive_expect_tx(full, bb + cb + (uint32_t)kBytesSlot + (so_map ? (uint32_t)kSOSlot : 0u));
         bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, full);
         bulk_g2s(ar2 + L.oCS + buf * kCSSlot, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * kCSGroup,
                  cb, full);
@@ -1339,26 +1362,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile(
             "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
                 smem_u32(bytes_buf((int)buf))),
-            "l"(P.map()), "r"(w.s * kStageBytes), "r"(n0), "r"(smem_u32(full))
+            "l"(maps), "r"(w.s * kStageBytes), "r"(n0), "r"(smem_u32(full))
             : "memory");
+        if (so_map) {
+          // the stage's 8 groups of s1 and of off for the 128 rows (16 bytes a row)
+          asm volatile(
+              "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+                  smem_u32(so)),
+              "l"(maps + kMapS1), "r"(g0), "r"(n0), "r"(smem_u32(full))
+              : "memory");
+          asm volatile(
+              "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+                  smem_u32(so + kRows * 16)),
+              "l"(maps + kMapOff), "r"(g0), "r"(n0), "r"(smem_u32(full))
+              : "memory");
+        }
       }
       __syncwarp();
-      {
-        const int G = P.K / kGroup;
-        const bool vec = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
-        unsigned char *so = ar2 + L.oSO + buf * kSOSlot;
-        if (vec) {
-#pragma unroll
-          for (int k = 0; k < kRows / 32; ++k) {
-            const int r = lane + 32 * k;
-            if (r < rows) {
-              const int64_t o = (int64_t)(n0 + r) * G + g0;
-              cp_async16(so + r * 16, P.s1 + o);
-              cp_async16(so + kRows * 16 + r * 16, P.off + o);
-            }
-          }
-          cp_async_mbar_arrive_noinc(full);
-        } else {
+      if (so_map) {
+        mbar_arrive(full);  // the lanes' arrivals (the barrier counts 1 + 32)
+      } else {
+        {
           for (int r = lane; r < rows; r += 32) {
             const int64_t o = (int64_t)(n0 + r) * G + g0;
             __half *d1 = reinterpret_cast<__half *>(so + r * 16);
@@ -1373,7 +1397,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (++buf == (uint32_t)NS) buf = 0, phase ^= 1u;
     }
-    cp_async_wait<0>();  // the lanes' s1 / off copies have landed
+    cp_async_wait<0>();  // nothing of this warp in flight at exit
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
     if (lane == 0) {
@@ -1409,10 +1433,12 @@ void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2)
 
 TQ_STATUS_ACCESSOR(read_status_gemv_mma)
 
-// Tensor map of plane 1 as a 2-D byte tensor of rows of `rb` bytes (box
-// 208 x 128 bytes, no swizzle, zero fill), encoded once per row length;
-// the prep kernel puts in each problem's address and row count.
-static bool plane1_template(int64_t rb, const void *plane1, int N, CUtensorMap *out) {
+// Template tensor maps, encoded once per (kind, row length, rows) and cached:
+// kind 0 = plane 1 as a 2-D byte tensor of rows of `len` bytes (box 208 x 128
+// bytes); kind 1 = s1 / off as a 2-D fp16 tensor of rows of `len` halves (box
+// 8 x 128).  No swizzle, zero fill.  The prep kernel puts in each problem's
+// address.
+static bool map_template(int kind, int64_t len, const void *addr, int N, CUtensorMap *out) {
   // the driver's encoder, looked up through the runtime (no link-time
   // dependence on the driver library)
   static PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
@@ -1428,39 +1454,51 @@ static bool plane1_template(int64_t rb, const void *plane1, int N, CUtensorMap *
   static int64_t keys[64];
   static CUtensorMap maps[64];
   static int n = 0;
+  const int64_t key = ((int64_t)N << 32) | (len << 1) | kind;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n; ++i)
-    if (keys[i] == rb) {
+    if (keys[i] == key) {
       *out = maps[i];
       return true;
     }
   CUtensorMap m;
-  cuuint64_t dims[2] = {(cuuint64_t)rb, (cuuint64_t)N};
-  cuuint64_t strides[1] = {(cuuint64_t)rb};
-  cuuint32_t box[2] = {(cuuint32_t)mm::kStageBytes, (cuuint32_t)mm::kRows};
+  const int esz = kind == 0 ? 1 : 2;
+  cuuint64_t dims[2] = {(cuuint64_t)len, (cuuint64_t)N};
+  cuuint64_t strides[1] = {(cuuint64_t)(len * esz)};
+  cuuint32_t box[2] = {kind == 0 ? (cuuint32_t)mm::kStageBytes : (cuuint32_t)mm::kStageG, (cuuint32_t)mm::kRows};
   cuuint32_t estr[2] = {1, 1};
-  if (encode(&m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(plane1), dims, strides, box, estr,
-                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+  if (encode(&m, kind == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(addr),
+             dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return false;
-  if (n < 64) keys[n] = rb, maps[n] = m, ++n;
+  if (n < 64) keys[n] = key, maps[n] = m, ++n;
   *out = m;
   return true;
+}
+
+// s1 / off of a problem go by tensor copies (rows of whole 16-byte units)
+static bool scales_by_map(const Problem &P) {
+  return (P.K / kGroup) % 8 == 0 && (((uintptr_t)P.s1 | (uintptr_t)P.off) & 15u) == 0;
 }
 
 static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) + 8 <= 32764, "prep kernel parameters");
 static_assert(sizeof(BatchParams) + sizeof(mm::CUnits) <= 32764, "indexed second-plane kernel parameters");
 static_assert(sizeof(BatchParams) + sizeof(mm::Sched) <= 32764, "main kernel parameters");
 
-// Distinct plane-1 row lengths of a batch (up to `cap` + 1 are counted).
+// Distinct tensor-map templates of a batch's problems (up to `cap` + 1 are
+// counted): (row length, rows) of plane 1, and (groups, rows) of scales by map.
 static int distinct_row_lengths(const BatchParams &bp, int first, int last, int cap) {
-  int64_t seen[mm::kMaxMapTemplates + 1];
+  int64_t seen[mm::kMaxMapTemplates + 2] = {};
   int n = 0;
-  for (int i = first; i < last && n <= cap; ++i) {
-    const int64_t rb = row_bytes_of(bp.prob[i].K);
+  auto add = [&](int64_t key) {
     int k = 0;
-    while (k < n && seen[k] != rb) ++k;
-    if (k == n) seen[n++] = rb;
+    while (k < n && seen[k] != key) ++k;
+    if (k == n) seen[n++] = key;
+  };
+  for (int i = first; i < last && n <= cap; ++i) {
+    const int64_t rows = (int64_t)bp.prob[i].N << 32;
+    add(rows | (row_bytes_of(bp.prob[i].K) << 1));
+    if (scales_by_map(bp.prob[i])) add(rows | ((int64_t)(bp.prob[i].K / kGroup) << 1) | 1);
   }
   return n;
 }
@@ -1527,18 +1565,30 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   }
   thread_local mm::MapTemplates mt;
   {
-    int64_t rbs[mm::kMaxMapTemplates];
+    int64_t keys[mm::kMaxMapTemplates] = {};
     int nt = 0;
-    for (int i = 0; i < bp.count; ++i) {
-      const int64_t rb = row_bytes_of(bp.prob[i].K);
+    auto slot = [&](int kind, int64_t len, const void *addr, int N) -> int {
+      const int64_t key = ((int64_t)N << 32) | (len << 1) | kind;
       int k = 0;
-      while (k < nt && rbs[k] != rb) ++k;
+      while (k < nt && keys[k] != key) ++k;
       if (k == nt) {
-        if (nt == mm::kMaxMapTemplates) return cudaErrorNotSupported;  // launch_mm splits such batches
-        if (!plane1_template(rb, bp.prob[i].plane1, bp.prob[i].N, &mt.t[nt])) return cudaErrorInvalidValue;
-        rbs[nt++] = rb;
+        if (nt == mm::kMaxMapTemplates) return -1;  // launch_mm splits such batches
+        if (!map_template(kind, len, addr, N, &mt.t[nt])) return -2;
+        keys[nt++] = key;
       }
-      mt.idx[i] = (uint8_t)k;
+      return k;
+    };
+    for (int i = 0; i < bp.count; ++i) {
+      const Problem &P = bp.prob[i];
+      const int k1 = slot(0, row_bytes_of(P.K), P.plane1, P.N);
+      if (k1 < 0) return k1 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
+      mt.idx[i] = (uint8_t)k1;
+      mt.idx_so[i] = mm::kNoMap;
+      if (scales_by_map(P)) {
+        const int k2 = slot(1, P.K / kGroup, P.s1, P.N);
+        if (k2 < 0) return k2 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
+        mt.idx_so[i] = (uint8_t)k2;
+      }
     }
   }
   // second plane: the indexed kernel when every weight with a second plane
@@ -1565,7 +1615,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     un.count = n;
     un.base[0] = 0;
     for (int a = 0; a < n; ++a) un.base[a + 1] = un.base[a] + bp.prob[un.order[a]].K / kGroup;
-    counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + 128);
+    counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + mm::kCounterOff);
     un.counter = counter;
   }
   mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);

@@ -49,10 +49,10 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_linear_batched(1, 0, None, None, 0, None) == -2
     # M <= 8: activation fragments (320 B per group and token), C/S (64 B per
     # group), second-plane partials (4 B per row and token), each 256-padded,
-    # and a 256-byte slot for the plane-1 tensor map
+    # and a 512-byte slot for the tensor maps of plane 1, s1 and off
     pad = lambda b: (b + 255) // 256 * 256
-    mma = lambda M, N, K: pad(K // 128 * 320 * M) + pad(K // 128 * 64) + pad(N * M * 4) + 256
-    assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) == 28928
+    mma = lambda M, N, K: pad(K // 128 * 320 * M) + pad(K // 128 * 64) + pad(N * M * 4) + 512
+    assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) == 29184
     assert tq.tq_workspace_bytes(5, 100, 1024) == mma(5, 100, 1024)
     # 8 < M <= 16: tensor-memory path (2 x 2560 B of slots + 128 B C/S per group);
     # M > 16: the prefill tile path needs no workspace (256 bytes are asked for)
