@@ -141,6 +141,13 @@ __host__ __device__ __forceinline__ uint32_t lut_word(int v) {
   return w;
 }
 
+// The low (hi = false) or high fp16 of a word, as float.
+template <bool HI>
+__device__ __forceinline__ float half_of(uint32_t w) {
+  const __half2 h = *reinterpret_cast<const __half2 *>(&w);
+  return HI ? __high2float(h) : __low2float(h);
+}
+
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t s) {
   uint32_t d;
   asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(s));
@@ -245,18 +252,12 @@ __device__ __forceinline__ void mma16816_z(float *d, uint32_t a0, uint32_t a1, u
 }
 
 // The MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
-// (b[2j], b[2j+1] for chunk j).  Two accumulation chains, summed into d.
+// (b[2j], b[2j+1] for chunk j), one accumulation chain (measured faster than
+// two or four chains summed at the end: the adds cost more than the latency).
 __device__ __forceinline__ void group_mma(const uint32_t *aL, const uint32_t *aH, const uint32_t *b, float *d) {
-  float e[4], o[4];
-  mma16816_z(e, aL[0], aH[0], aL[1], aH[1], b[0], b[1]);
-  mma16816_z(o, aL[2], aH[2], aL[3], aH[3], b[2], b[3]);
+  mma16816_z(d, aL[0], aH[0], aL[1], aH[1], b[0], b[1]);
 #pragma unroll
-  for (int j = 2; j < kChunks; ++j) {
-    float *acc = (j & 1) ? o : e;
-    mma16816(acc, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) d[i] = e[i] + o[i];
+  for (int j = 1; j < kChunks; ++j) mma16816(d, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
 }
 
 // Iterates (tile, stage) in the CTA's order.
@@ -1204,9 +1205,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float Cx = CSst[GL * 16 + 2 * c], Sx = CSst[GL * 16 + 8 + 2 * c];
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-              const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
-              const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
-              const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+              const float s1 = half_of<(GL & 1) != 0>(s1w[h][GL >> 1]);
+              const float of = half_of<(GL & 1) != 0>(ofw[h][GL >> 1]);
               y[2 * h] = fmaf(s1, d[2 * h] - Cx, fmaf(of, Sx, y[2 * h]));
             }
             return;
@@ -1215,9 +1215,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
-            const uint32_t sw = s1w[h][GL >> 1], ow = ofw[h][GL >> 1];
-            const float s1 = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? sw >> 16 : sw & 0xffffu)));
-            const float of = __half2float(__ushort_as_half((unsigned short)((GL & 1) ? ow >> 16 : ow & 0xffffu)));
+            const float s1 = half_of<(GL & 1) != 0>(s1w[h][GL >> 1]);
+            const float of = half_of<(GL & 1) != 0>(ofw[h][GL >> 1]);
             y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
             y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
           }
