@@ -468,8 +468,8 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
                      "traffic": ncu_traffic(),
-                     "kernel": "decode step: activation prep + second plane (per-weight index) + first plane "
-                               "(3 launches per step, timed together; the first-plane kernel is ~75 % of it)",
+                     "kernel": "decode step: activation prep + second plane (group-ordered index) + first plane "
+                               "(3 launches per step, timed together; the first-plane kernel is ~80 % of it)",
                      "launch_ms_avg": launch_avg},
         "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},

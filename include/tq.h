@@ -116,23 +116,35 @@ TQ_API tq_status tq_salience_rowptr(int32_t N, int32_t K, const uint32_t *sal, i
                              uint32_t *d_status, void *stream);
 
 /* Second-plane index (no counterpart in the paper; a layout aid for the
- * decode path, M <= 8).  The salient (row, group) pairs of a weight listed
- * group by group: int32 colptr[G + 1] (group g's entries are colptr[g] ..
- * colptr[g+1] - 1), then, from int32 offset tq_plane2_index_rec_offset(K),
- * rec[nnz] (each entry's plane-2 record index j = rowptr[n] + rank of g
- * among row n's salient groups), then, from offset
- * tq_plane2_index_row_offset(K, nnz), row[nnz] (its row n); within a group
- * the entries follow increasing n.  It depends on the salience map only, so
- * it is built once per weight; with it tq_linear runs the second plane one
- * group at a time without grouping the records first.
+ * decode path, M <= 8): plane 2 re-laid out group by group.  The salient
+ * (row, group) pairs of each group g, in increasing row order, padded with
+ * empty entries to a multiple of 16, each entry a 32-byte slot that holds
+ * the pair's plane-2 record, its s2 and its row.  It depends on the weight
+ * alone, so it is built once; with it tq_linear runs the second plane one
+ * group at a time, 16 entries per tensor-core tile, and reads this copy
+ * instead of plane 2 and s2.
+ * Layout, with C = tq_plane2_index_capacity(K, nnz) (a multiple of 16):
+ *   int32 colptr[G + 1] at byte 0: group g's entries are colptr[g] ..
+ *     colptr[g+1] - 1, multiples of 16 (colptr[G] <= C);
+ *   slot[C][32] at byte tq_plane2_index_slot_offset(K) (128-byte aligned).
+ * A slot's 32 bytes, in logical order L[0..31], o = 2 * ((g % 8) & 1),
+ * the decode kernels' window alignment of group g):
+ *   L[o .. o+25]  the pair's 26-byte plane-2 record,
+ *   L[o ? 0 : 26] the pair's s2 (fp16, two bytes),
+ *   L[28 .. 31]   the row n (int32; -1 for an empty entry, whose other bytes
+ *                 are zero),
+ * stored as 4-byte words in the order of logical words 0, 4, 1, 5, 2, 6, 3,
+ * 7 (so logical words i and i + 4, which one lane decodes, are adjacent).
+ * Entries from colptr[G] to C are empty too.
  *   index: device, tq_plane2_index_bytes(N, K, nnz) bytes, 16-byte aligned.
- *   sal, rowptr as for tq_pack (rowptr[N] == nnz); bits at g >= K/128 are
- *   ignored.  Asynchronous on stream. */
+ *   sal, rowptr, plane2, scale2 as for tq_linear (rowptr[N] == nnz; bits at
+ *   g >= K/128 are ignored; a pair whose record index falls outside
+ *   [0, nnz) becomes an empty entry).  Asynchronous on stream. */
+TQ_API size_t tq_plane2_index_capacity(int32_t K, int64_t nnz);
+TQ_API size_t tq_plane2_index_slot_offset(int32_t K);
 TQ_API size_t tq_plane2_index_bytes(int32_t N, int32_t K, int64_t nnz);
-TQ_API size_t tq_plane2_index_rec_offset(int32_t K);
-TQ_API size_t tq_plane2_index_row_offset(int32_t K, int64_t nnz);
 TQ_API tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
-                                 int32_t *index, void *stream);
+                                 const uint8_t *plane2, const uint16_t *scale2, int32_t *index, void *stream);
 
 /* Pack int8 trit codes into the lattice format (paper "Packing").
  *   T1: int8 [N][K] in {-1,0,+1};  T2: int8 [N][K], nonzero only where the

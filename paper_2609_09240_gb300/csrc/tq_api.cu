@@ -15,8 +15,8 @@ cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t
 cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                         const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
                         cudaStream_t s);
-cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
-                                cudaStream_t s);
+cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
+                                const uint8_t *plane2, const uint16_t *scale2, int32_t *index, cudaStream_t s);
 cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s);
@@ -207,28 +207,31 @@ tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *
   return from_cuda(launch_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, s));
 }
 
-size_t tq_plane2_index_rec_offset(int32_t K) {
-  if (K < TQ_GROUP || K % TQ_GROUP) return 0;
-  return ((size_t)(K / TQ_GROUP) + 1 + 3) & ~(size_t)3;
+size_t tq_plane2_index_capacity(int32_t K, int64_t nnz) {
+  if (K < TQ_GROUP || K % TQ_GROUP || nnz < 0) return 0;
+  return (((size_t)nnz + 15 * (size_t)(K / TQ_GROUP)) + 15) & ~(size_t)15;
 }
 
-size_t tq_plane2_index_row_offset(int32_t K, int64_t nnz) {
-  if (K < TQ_GROUP || K % TQ_GROUP || nnz < 0) return 0;
-  return tq_plane2_index_rec_offset(K) + (((size_t)nnz + 3) & ~(size_t)3);
+size_t tq_plane2_index_slot_offset(int32_t K) {
+  if (K < TQ_GROUP || K % TQ_GROUP) return 0;
+  return ((size_t)(K / TQ_GROUP + 1) * 4 + 127) & ~(size_t)127;
 }
 
 size_t tq_plane2_index_bytes(int32_t N, int32_t K, int64_t nnz) {
   if (check_shape(N, K) != TQ_OK || nnz < 0 || nnz > (int64_t)N * (K / TQ_GROUP)) return 0;
-  return 4 * (tq_plane2_index_row_offset(K, nnz) + (((size_t)nnz + 3) & ~(size_t)3));
+  if (tq_plane2_index_capacity(K, nnz) > (size_t)INT32_MAX) return 0;  // colptr is int32
+  return tq_plane2_index_slot_offset(K) + 32 * tq_plane2_index_capacity(K, nnz);
 }
 
-tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
-                          void *stream) {
+tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
+                          const uint8_t *plane2, const uint16_t *scale2, int32_t *index, void *stream) {
   if (tq_status st = check_shape(N, K)) return st;
   if (!sal || !rowptr || !index) return TQ_ERR_NULL;
+  if (nnz > 0 && (!plane2 || !scale2)) return TQ_ERR_NULL;
   if (nnz < 0 || nnz > (int64_t)N * (K / TQ_GROUP)) return TQ_ERR_SALIENCE;
-  if ((uintptr_t)index & 15u) return TQ_ERR_ALIGN;
-  return from_cuda(launch_plane2_index(N, K, sal, rowptr, nnz, index, (cudaStream_t)stream));
+  if (tq_plane2_index_bytes(N, K, nnz) == 0) return TQ_ERR_SHAPE;
+  if (((uintptr_t)index & 15u) || (plane2 && !aligned16(plane2)) || (scale2 && !aligned2(scale2))) return TQ_ERR_ALIGN;
+  return from_cuda(launch_plane2_index(N, K, sal, rowptr, nnz, plane2, scale2, index, (cudaStream_t)stream));
 }
 
 size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K) {

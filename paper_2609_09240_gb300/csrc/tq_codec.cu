@@ -220,10 +220,17 @@ __global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t
 // ------------------------------------------------------ second-plane index
 // One block per group g walks the rows in chunks of blockDim.x, in order;
 // a block-wide count (and, for the fill, an exclusive scan of the row bits)
-// gives each salient row its place in group g's list.
+// gives each salient row its place in group g's list.  Group lists start at
+// multiples of 16; the entries after a group's last pair, up to the next
+// start, are empty.
 constexpr int kIdxThreads = 256;
 
-__device__ __forceinline__ size_t p2index_rec_off(int K) { return ((size_t)(K / kGroup) + 1 + 3) & ~(size_t)3; }
+__host__ __device__ __forceinline__ int64_t p2index_capacity(int K, int64_t nnz) {
+  return (nnz + 15 * (int64_t)(K / kGroup) + 15) & ~(int64_t)15;
+}
+__host__ __device__ __forceinline__ int64_t p2index_slot_off(int K) {
+  return ((int64_t)(K / kGroup + 1) * 4 + 127) & ~(int64_t)127;
+}
 
 __global__ void __launch_bounds__(kIdxThreads) p2index_count_kernel(int N, int K, const uint32_t *sal,
                                                                      int32_t *colptr) {
@@ -236,21 +243,68 @@ __global__ void __launch_bounds__(kIdxThreads) p2index_count_kernel(int N, int K
   if (threadIdx.x == 0) colptr[g + 1] = total;
 }
 
-__global__ void p2index_scan_kernel(int G, int32_t *colptr) {
+// colptr[g+1] = colptr[g] + count rounded up to 16, at most the capacity
+// (which the counts of a consistent salience map never reach).
+__global__ void p2index_scan_kernel(int G, int64_t cap, int32_t *colptr) {
   if (threadIdx.x != 0) return;
   colptr[0] = 0;
-  for (int g = 0; g < G; ++g) colptr[g + 1] += colptr[g];
+  int64_t run = 0;
+  for (int g = 0; g < G; ++g) {
+    run = min(run + (((int64_t)colptr[g + 1] + 15) & ~(int64_t)15), cap);
+    colptr[g + 1] = (int32_t)run;
+  }
 }
 
+// One slot: 8 words in the order of logical words 0, 4, 1, 5, 2, 6, 3, 7.
+__device__ __forceinline__ void p2index_store_slot(uint8_t *slot, const uint32_t *L) {
+  uint4 *d = reinterpret_cast<uint4 *>(slot);
+  d[0] = make_uint4(L[0], L[4], L[1], L[5]);
+  d[1] = make_uint4(L[2], L[6], L[3], L[7]);
+}
+
+__device__ __forceinline__ void p2index_empty_slot(uint8_t *slot) {
+  const uint32_t L[8] = {0, 0, 0, 0, 0, 0, 0, 0xffffffffu};
+  p2index_store_slot(slot, L);
+}
+
+// Entry e of group g: the record j of row n (plane 2 and s2 are 2-byte
+// aligned at a record, so the record is read as 13 halves).
+__device__ __forceinline__ void p2index_fill_slot(uint8_t *slot, int g, int n, int64_t j, int64_t nnz,
+                                                  const uint8_t *plane2, const uint16_t *scale2) {
+  if (j < 0 || j >= nnz) {
+    p2index_empty_slot(slot);
+    return;
+  }
+  uint32_t L[8] = {0, 0, 0, 0, 0, 0, 0, (uint32_t)n};
+  const int h0 = (g % 8) & 1;  // the record starts at logical half h0 (byte o = 2 h0)
+  const uint16_t *rec = reinterpret_cast<const uint16_t *>(plane2 + j * kGroupBytes);
+#pragma unroll
+  for (int i = 0; i < kGroupBytes / 2; ++i) {
+    const int h = h0 + i;
+    L[h >> 1] |= (uint32_t)rec[i] << (16 * (h & 1));
+  }
+  const int hs = h0 ? 0 : kGroupBytes / 2;  // s2 in the free half next to the record
+  L[hs >> 1] |= (uint32_t)scale2[j] << (16 * (hs & 1));
+  p2index_store_slot(slot, L);
+}
+
+// Blocks 0 .. G-1 fill group g's entries; block G empties the slots from
+// colptr[G] to the capacity.
 __global__ void __launch_bounds__(kIdxThreads) p2index_fill_kernel(int N, int K, const uint32_t *sal,
                                                                     const int32_t *rowptr, int64_t nnz,
+                                                                    const uint8_t *plane2, const uint16_t *scale2,
                                                                     int32_t *index) {
   __shared__ int warp_base[kIdxThreads / 32 + 1];
-  const int g = blockIdx.x, W = sal_words_of(K);
+  const int G = K / kGroup, g = blockIdx.x, W = sal_words_of(K);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int32_t *rec = index + p2index_rec_off(K);
-  int32_t *row = rec + ((nnz + 3) & ~(int64_t)3);
-  int base = index[g];
+  uint8_t *slots = reinterpret_cast<uint8_t *>(index) + p2index_slot_off(K);
+  if (g == G) {
+    const int64_t cap = p2index_capacity(K, nnz);
+    for (int64_t e = index[G] + threadIdx.x; e < cap; e += kIdxThreads) p2index_empty_slot(slots + 32 * e);
+    return;
+  }
+  const int64_t lim = index[g + 1];
+  int64_t base = index[g];
   for (int n0 = 0; n0 < N; n0 += kIdxThreads) {
     const int n = n0 + threadIdx.x;
     const bool bit = n < N && sal_bit(sal, W, n, g);
@@ -268,16 +322,16 @@ __global__ void __launch_bounds__(kIdxThreads) p2index_fill_kernel(int N, int K,
     }
     __syncthreads();
     if (bit) {
-      const int pos = base + warp_base[warp] + __popc(m & ((1u << lane) - 1u));
-      const int64_t j = (int64_t)rowptr[n] + sal_rank(sal, W, n, g);
-      if (pos < nnz) {  // within the index (entries beyond nnz, from a rowptr that disagrees, are dropped)
-        rec[pos] = (int32_t)min(max(j, (int64_t)0), nnz > 0 ? nnz - 1 : (int64_t)0);
-        row[pos] = n;
+      const int64_t pos = base + warp_base[warp] + __popc(m & ((1u << lane) - 1u));
+      if (pos < lim) {  // within the group's entries (the capacity cuts an inconsistent map short)
+        const int64_t j = (int64_t)rowptr[n] + sal_rank(sal, W, n, g);
+        p2index_fill_slot(slots + 32 * pos, g, n, j, nnz, plane2, scale2);
       }
     }
     base += warp_base[kIdxThreads / 32];
     __syncthreads();
   }
+  for (int64_t e = base + threadIdx.x; e < lim; e += kIdxThreads) p2index_empty_slot(slots + 32 * e);
 }
 
 // ------------------------------------------------------------- launchers
@@ -316,12 +370,12 @@ cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *pl
   return cudaGetLastError();
 }
 
-cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz, int32_t *index,
-                                cudaStream_t s) {
+cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
+                                const uint8_t *plane2, const uint16_t *scale2, int32_t *index, cudaStream_t s) {
   const int G = K / kGroup;
   p2index_count_kernel<<<G, kIdxThreads, 0, s>>>(N, K, sal, index);
-  p2index_scan_kernel<<<1, 32, 0, s>>>(G, index);
-  p2index_fill_kernel<<<G, kIdxThreads, 0, s>>>(N, K, sal, rowptr, nnz, index);
+  p2index_scan_kernel<<<1, 32, 0, s>>>(G, p2index_capacity(K, nnz), index);
+  p2index_fill_kernel<<<G + 1, kIdxThreads, 0, s>>>(N, K, sal, rowptr, nnz, plane2, scale2, index);
   return cudaGetLastError();
 }
 

@@ -53,6 +53,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 #include <type_traits>
 
@@ -939,48 +940,36 @@ __global__ void __launch_bounds__(kQThreads, 1)
   cp_async_wait<0>();
 }
 
-// Second plane with the per-weight index (1..8 tokens).  Persistent warps
-// take (problem, group) units from a counter in the workspace (problems with
-// more records per group first); for its unit a warp loads group g's B
-// fragment and C once and runs the group's records in the index's order, 16
-// at a time as the rows of an m16 tile: each lane reads its two window words
-// of its two records straight from plane 2, decodes them with the
-// lane-replicated table, and s2 * (D - C) per record is added to y2 of the
-// record's row with a global atomic (the prep kernel zeroes y2).
+// Second plane with the group-ordered index (1..8 tokens).  Persistent
+// warps take units from a counter in the workspace: a unit is one of the
+// c_parts contiguous shares of one group's 16-entry tiles, numbered problem
+// by problem (each CTA builds the table of first units per problem in shared
+// memory).  For its unit a warp loads group g's B fragment and C once and
+// runs the tiles as m16 tiles: lane (r, c) loads slot words 2 jw, 2 jw + 1
+// of entries r and r + 8 (its two window words, one 8-byte load per entry;
+// a quad's loads cover the slot), decodes them with the lane-replicated
+// table and, after the MMAs, takes the entries' rows and s2 from the quad's
+// lanes that hold them; s2 (D - C) per entry is added to y2 of the entry's
+// row with a global atomic (the prep kernel zeroes y2).
 constexpr int kCThreads = 512;
+constexpr int kCDepth = 4;                        // tiles in flight per warp (in registers)
+constexpr int kCDynBytes2 = kArena1 + kLutBytes;  // unit table below the table of codes
+constexpr int kCUnitTiles = 24;                   // target tiles per unit
+static_assert((TQ_MAX_BATCH + 8 + kCThreads / 32) * 4 <= kArena1, "unit table");
 
-struct CUnits {
-  int32_t base[TQ_MAX_BATCH + 1];  // units of order[0..i) (a unit per group)
-  uint8_t order[TQ_MAX_BATCH];     // problems with a second plane, most records per group first
-  int32_t count;                   // entries of order[]
-  int32_t *counter;                // the next unit (zeroed by the prep kernel)
-};
-
-// Per-warp staging in shared memory: a chunk of the group's index entries
-// (record index j, row n), and a ring of kCDepth tiles of record words: for
-// each lane its two records' aligned words around its two window words and
-// the 4-byte word holding each record's s2 (10 words).
-constexpr int kCWarps = kCThreads / 32;
-constexpr int kCChunk = 256;                        // index entries per chunk
-constexpr int kCIdxWords = kCChunk + 4;             // + the start rounded down to 4 entries
-constexpr int kCDepth = 3;                          // m16 tiles in flight per warp
-constexpr int kCLaneWords = 11;                     // 10 used; odd, so the lanes' reads hit 32 banks
-constexpr int kCRing = kCDepth * 32 * kCLaneWords;  // words
-constexpr int kCIdxOff = 0;                         // per warp: j[kCIdxWords], n[kCIdxWords] (below the table)
-constexpr int kCRingOff = kArena1 + kLutBytes;      // per warp: the ring (above the table)
-static_assert(kCIdxOff + kCWarps * 2 * kCIdxWords * 4 <= kArena1, "index chunks overflow");
-constexpr int kCDynBytes2 = kCRingOff + kCWarps * kCRing * 4;
-static_assert(kCDynBytes2 <= kDynBytes, "record rings overflow");
-
-// One aligned 4-byte word of plane 2 into the ring (`bytes` = 2 for the last
-// word of plane 2 when the array ends inside it).
-__device__ __forceinline__ void c_copy_word(uint32_t *dst, const uint8_t *src, int bytes) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(bytes) : "memory");
+__device__ __forceinline__ int64_t c_capacity(int K, int64_t nnz) {
+  return (nnz + 15 * (int64_t)(K / kGroup) + 15) & ~(int64_t)15;
+}
+__device__ __forceinline__ int64_t c_slot_off(int K) { return ((int64_t)(K / kGroup + 1) * 4 + 127) & ~(int64_t)127; }
+// Units per group: the mean tiles per group over kCUnitTiles, rounded up, 1 .. 32.
+__device__ __forceinline__ int c_parts(const Problem &P) {
+  const int64_t per = (int64_t)(P.K / kGroup) * 16 * kCUnitTiles;
+  return (int)min(max((P.nnz + per - 1) / per, (int64_t)1), (int64_t)32);
 }
 
 template <bool ONE>
 __global__ void __launch_bounds__(kCThreads, 1)
-    gemv_mma_p2c_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ CUnits un) {
+    gemv_mma_p2c_kernel(const __grid_constant__ BatchParams bp, int32_t *counter) {
   extern __shared__ __align__(1024) unsigned char dync[];
   const int tid = threadIdx.x, lane = tid & 31;
   if (smem_u32(dync) != kDynShared) {
@@ -991,31 +980,50 @@ __global__ void __launch_bounds__(kCThreads, 1)
     uint32_t *lut = reinterpret_cast<uint32_t *>(dync + kArena1);
     for (int i = tid; i < 256 * 32; i += kCThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
   }
+  // first unit of each problem: base[p] = sum over q < p of G_q * parts_q (problems without a
+  // second plane have none); an inclusive scan of one value per thread
+  int32_t *base = reinterpret_cast<int32_t *>(dync);
+  int32_t *warp_sum = base + TQ_MAX_BATCH + 8;  // (no static shared memory: it would move the window)
+  {
+    static_assert(kCThreads >= TQ_MAX_BATCH, "one problem per thread");
+    int v = 0;
+    if (tid < bp.count) {
+      const Problem &Q = bp.prob[tid];
+      if (Q.nnz > 0 && Q.p2idx) v = (Q.K / kGroup) * c_parts(Q);
+    }
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += t;
+    }
+    if (lane == 31) warp_sum[tid >> 5] = v;
+    __syncthreads();
+    for (int w = 0; w < (tid >> 5); ++w) v += warp_sum[w];
+    if (tid == 0) base[0] = 0;
+    if (tid < TQ_MAX_BATCH) base[tid + 1] = v;
+  }
   __syncthreads();
-  const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, warp = tid >> 5;
+  const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, quad = lane & ~3;
   const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
-  const int total = un.base[un.count];
-  int32_t *idx_j = reinterpret_cast<int32_t *>(dync + kCIdxOff) + warp * 2 * kCIdxWords;
-  int32_t *idx_n = idx_j + kCIdxWords;
-  uint32_t *ring = reinterpret_cast<uint32_t *>(dync + kCRingOff) + warp * kCRing;
+  const int count = bp.count, total = base[count];
   for (;;) {
     int u = 0;
-    if (lane == 0) u = atomicAdd(un.counter, 1);
+    if (lane == 0) u = atomicAdd(counter, 1);
     u = __shfl_sync(0xffffffffu, u, 0);
     if (u >= total) break;
-    int i = 0;  // the unit's entry: the last i with base[i] <= u
+    int i = 0;  // the unit's problem: the last i with base[i] <= u
     for (int step = 128; step >= 1; step >>= 1)
-      if (i + step < un.count && un.base[i + step] <= u) i += step;
-    const Problem &P = bp.prob[un.order[i]];
-    const int g = u - un.base[i], GL = g % kStageG;
-    const int G = P.K / kGroup;
-    const int64_t nnz = P.nnz;
-    const int32_t *colptr = P.p2idx;
-    const int32_t *recj = P.p2idx + ((G + 1 + 3) & ~3);
-    const int32_t *rown = recj + ((nnz + 3) & ~(int64_t)3);
-    const int k0 = (int)min(max((int64_t)__ldg(colptr + g), (int64_t)0), nnz);
-    const int k1 = (int)min(max((int64_t)__ldg(colptr + g + 1), (int64_t)k0), nnz);
-    if (k0 >= k1) continue;
+      if (i + step < count && base[i + step] <= u) i += step;
+    const Problem &P = bp.prob[i];
+    const int S = c_parts(P), local = u - base[i];
+    const int g = local / S, part = local - g * S, GL = g % kStageG;
+    // the group's entries, clamped into the index (whole tiles)
+    const int64_t cap = c_capacity(P.K, P.nnz);
+    const int64_t e0 = min(max((int64_t)__ldg(P.p2idx + g), (int64_t)0), cap) & ~(int64_t)15;
+    const int64_t e1 = min(max((int64_t)__ldg(P.p2idx + g + 1), e0), cap) & ~(int64_t)15;
+    const int nt = (int)((e1 - e0) >> 4);
+    const int t0 = (int)((int64_t)nt * part / S), n = (int)((int64_t)nt * (part + 1) / S) - t0;
+    if (n <= 0) continue;
     // the group's B fragment (lanes of absent tokens repeat the last token) and C
     const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB + min(g16, MB - 1) * kBTok + c * kBLane;
     uint32_t b[20];
@@ -1024,109 +1032,67 @@ __global__ void __launch_bounds__(kCThreads, 1)
       const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg + cp * 4 * kBLane));
       b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
     }
-    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + 2 * c));
-    // lane c's window words: win_start + jw and + 4; the record starts o bytes into the window
-    const int q = 4 * ((c - win_start(GL)) & 3) - 2 * (GL & 1);
+    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + (ONE ? 0 : 2 * c)));
+    // lane c's window words jw and jw + 4 are slot words 2 jw, 2 jw + 1; the row is the second
+    // word of the lane with jw = 3, s2 a half of the first word of jw = 0 (record at byte 2)
+    // or of the second word of jw = 2 (record at byte 0)
+    const int ws = win_start(GL), jw = (c - ws) & 3, odd = GL & 1;
+    const int c_row = quad + ((3 + ws) & 3), c_s2 = quad + (((odd ? 0 : 2) + ws) & 3);
+    const unsigned char *src = reinterpret_cast<const unsigned char *>(P.p2idx) + c_slot_off(P.K) +
+                               (e0 + 16 * (int64_t)t0 + g16) * 32 + jw * 8;
     float *y2 = P.y2();
-    const int64_t nidx4 = (nnz + 3) & ~(int64_t)3;  // entries of each index array, as allocated
-    const bool s2_al = (reinterpret_cast<uintptr_t>(P.s2) & 3u) == 0;
-    const int nnz32 = (int)nnz;  // plane 2 of this path is below 2^31 bytes (the launcher checks)
-    // record j starts d = 2 (j & 1) bytes into a word (plane 2 is 16-byte aligned); the
-    // aligned words around the lane's window words, at record-relative offsets x .. x + 20,
-    // clamped onto the words holding the record's bytes (the others meet zero
-    // activations, so the copies stay inside the record): per parity of j
-    int xo[2][4];
-    uint32_t shp[2];
+    uint2 pre[kCDepth][2];
 #pragma unroll
-    for (int par = 0; par < 2; ++par) {
-      const int d = 2 * par, x = q - ((q + d) & 3);
-      shp[par] = (uint32_t)((q + d) & 3) * 8u;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) xo[par][k] = min(max(x + 4 * (k & 1) + 16 * (k >> 1), -d), 24 - d);
+    for (int k = 0; k < kCDepth; ++k) {
+      pre[k][0] = pre[k][1] = make_uint2(0u, 0u);
+      if (k < n) {
+        pre[k][0] = __ldg(reinterpret_cast<const uint2 *>(src + k * 512));
+        pre[k][1] = __ldg(reinterpret_cast<const uint2 *>(src + k * 512 + 256));
+      }
     }
-    for (int c0 = k0; c0 < k1; c0 += kCChunk) {
-      const int c1 = min(c0 + kCChunk, k1);
-      // the chunk's entries, from the 4-entry boundary at or below c0
-      const int a0 = c0 & ~3;
-      const int nch = (int)min((int64_t)(c1 - a0 + 3) / 4, (nidx4 - a0) / 4);
-      for (int k = lane; k < nch; k += 32) {
-        cp_async16(idx_j + 4 * k, recj + a0 + 4 * k);
-        cp_async16(idx_n + 4 * k, rown + a0 + 4 * k);
-      }
-      cp_async_commit();
-      cp_async_wait<0>();
-      __syncwarp();
-      // tile t of the chunk covers entries c0 + 16 t .. + 15; lane slots g16, g16 + 8
-      const int ntiles = (c1 - c0 + 15) / 16;
-      auto issue = [&](int t) {
-        if (t < ntiles) {
-          uint32_t *dst = ring + ((t % kCDepth) * 32 + lane) * kCLaneWords;
+    for (int t = 0; t < n; t += kCDepth) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int e = c0 + 16 * t + g16 + 8 * h;
-            const int j = min(max(idx_j[(e < c1 ? e : c0) - a0], 0), nnz32 - 1);
-            const uint8_t *rec = P.plane2 + (uint32_t)j * (uint32_t)kGroupBytes;
-            const int par = j & 1;
-            const bool tail = par == 0 && j == nnz32 - 1;  // its last aligned word ends 2 bytes past plane 2
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const int x = par ? xo[1][k] : xo[0][k];
-              c_copy_word(dst + 5 * h + k, rec + x, (tail && x == 24) ? 2 : 4);
-            }
-            if (s2_al) {
-              // the 4-byte word holding s2[j] (2 bytes of it past the end of s2 when j is the last, even)
-              asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst + 5 * h + 4)),
-                           "l"(P.s2 + (j & ~1)), "r"((j | 1) < nnz32 ? 4 : 2)
-                           : "memory");
-            }
+      for (int k = 0; k < kCDepth; ++k) {
+        if (t + k < n) {
+          const uint2 r0 = pre[k][0], r1 = pre[k][1];
+          if (t + k + kCDepth < n) {
+            const unsigned char *p = src + (int64_t)(t + k + kCDepth) * 512;
+            pre[k][0] = __ldg(reinterpret_cast<const uint2 *>(p));
+            pre[k][1] = __ldg(reinterpret_cast<const uint2 *>(p + 256));
           }
-        }
-        cp_async_commit();
-      };
-#pragma unroll
-      for (int t = 0; t < kCDepth - 1; ++t) issue(t);
-      for (int t = 0; t < ntiles; ++t) {
-        issue(t + kCDepth - 1);
-        cp_async_wait<kCDepth - 1>();  // this lane's copies of tile t
-        const uint32_t *src = ring + ((t % kCDepth) * 32 + lane) * kCLaneWords;
-        uint32_t aL[20], aH[20];
-        int rowv[2];
-        float s2v[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int e = c0 + 16 * t + g16 + 8 * h;
-          const int j = min(max(idx_j[(e < c1 ? e : c0) - a0], 0), nnz32 - 1);
-          rowv[h] = e < c1 ? idx_n[e - a0] : -1;
-          const uint32_t sh = (j & 1) ? shp[1] : shp[0];
-          const uint32_t w0 = __funnelshift_r(src[5 * h], src[5 * h + 1], sh);
-          const uint32_t w1 = __funnelshift_r(src[5 * h + 2], src[5 * h + 3], sh);
-          if (s2_al) {
-            const uint32_t s2w = src[5 * h + 4];
-            s2v[h] = __half2float(__ushort_as_half((unsigned short)((j & 1) ? s2w >> 16 : s2w & 0xffffu)));
-          } else {
-            s2v[h] = __half2float(P.s2[j]);  // s2 not 4-byte aligned: read in place
-          }
-          decode_words(w0, w1, tag, h ? aH : aL);
-        }
-        float d[4];
-        group_mma(aL, aH, b, d);
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int n = rowv[h];
-          if (n < 0 || n >= P.N) continue;
+          uint32_t aL[20], aH[20];
+          decode_words(r0.x, r0.y, tag, aL);
+          decode_words(r1.x, r1.y, tag, aH);
+          float d[4];
+          group_mma(aL, aH, b, d);
+          const uint32_t sw0 = __shfl_sync(0xffffffffu, odd ? r0.x : r0.y, c_s2);
+          const uint32_t sw1 = __shfl_sync(0xffffffffu, odd ? r1.x : r1.y, c_s2);
+          const float s2v0 = odd ? half_of<false>(sw0) : half_of<true>(sw0);
+          const float s2v1 = odd ? half_of<false>(sw1) : half_of<true>(sw1);
           if (ONE) {
-            if (c == 0) atomicAdd(&y2[n], s2v[h] * (d[2 * h] - Cv.x));
+            // every column of D is token 0: the lane holding the rows adds
+            if (lane == c_row) {
+              const int n0 = (int)r0.y, n1 = (int)r1.y;
+              if (n0 >= 0 && n0 < P.N) atomicAdd(&y2[n0], s2v0 * (d[0] - Cv.x));
+              if (n1 >= 0 && n1 < P.N) atomicAdd(&y2[n1], s2v1 * (d[2] - Cv.x));
+            }
           } else {
+            const int rows[2] = {__shfl_sync(0xffffffffu, (int)r0.y, c_row),
+                                 __shfl_sync(0xffffffffu, (int)r1.y, c_row)};
+            const float s2v[2] = {s2v0, s2v1};
 #pragma unroll
-            for (int ii = 0; ii < 2; ++ii) {
-              const int m = 2 * c + ii;
-              if (m < MB) atomicAdd(&y2[(int64_t)n * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+            for (int h = 0; h < 2; ++h) {
+              const int nr = rows[h];
+              if (nr < 0 || nr >= P.N) continue;
+#pragma unroll
+              for (int ii = 0; ii < 2; ++ii) {
+                const int m = 2 * c + ii;
+                if (m < MB) atomicAdd(&y2[(int64_t)nr * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+              }
             }
           }
         }
       }
-      cp_async_wait<0>();
-      __syncwarp();  // the chunk's entries are read before the next chunk is staged
     }
   }
 }
@@ -1481,7 +1447,7 @@ static bool scales_by_map(const Problem &P) {
 }
 
 static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) + 8 <= 32764, "prep kernel parameters");
-static_assert(sizeof(BatchParams) + sizeof(mm::CUnits) <= 32764, "indexed second-plane kernel parameters");
+static_assert(sizeof(BatchParams) + 8 <= 32764, "indexed second-plane kernel parameters");
 static_assert(sizeof(BatchParams) + sizeof(mm::Sched) <= 32764, "main kernel parameters");
 
 // Distinct tensor-map templates of a batch's problems (up to `cap` + 1 are
@@ -1595,28 +1561,11 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   // kQMaxW salience words, the per-tile one)
   bool all_idx = true;
   for (int i = 0; i < bp.count; ++i)
-    if (bp.prob[i].nnz > 0 && (!bp.prob[i].p2idx || bp.prob[i].nnz * (int64_t)kGroupBytes >= ((int64_t)1 << 31)))
+    if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx)
       all_idx = false;
-  thread_local mm::CUnits un;
   int32_t *counter = nullptr;
-  if (any2 && all_idx) {
-    // units (one per group) of the problems with a second plane, most records per group first
-    int n = 0;
-    for (int i = 0; i < bp.count; ++i)
-      if (bp.prob[i].nnz > 0) un.order[n++] = (uint8_t)i;
-    auto density = [&](int i) { return (double)bp.prob[i].nnz / (double)(bp.prob[i].K / kGroup); };
-    for (int a = 1; a < n; ++a)  // insertion sort by density, descending (stable)
-      for (int b2 = a; b2 > 0 && density(un.order[b2]) > density(un.order[b2 - 1]); --b2) {
-        const uint8_t t = un.order[b2];
-        un.order[b2] = un.order[b2 - 1];
-        un.order[b2 - 1] = t;
-      }
-    un.count = n;
-    un.base[0] = 0;
-    for (int a = 0; a < n; ++a) un.base[a + 1] = un.base[a] + bp.prob[un.order[a]].K / kGroup;
+  if (any2 && all_idx)
     counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + mm::kCounterOff);
-    un.counter = counter;
-  }
   mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -1624,7 +1573,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true> : mm::gemv_mma_p2c_kernel<false>;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
-    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(bp, un);
+    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(bp, counter);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   } else if (any2 && gmax <= mm::kQMaxG) {

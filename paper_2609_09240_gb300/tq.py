@@ -71,12 +71,12 @@ def lib():
             i64 = ctypes.c_int64
             L.tq_plane2_index_bytes.restype = ctypes.c_size_t
             L.tq_plane2_index_bytes.argtypes = [i32, i32, i64]
-            L.tq_plane2_index_rec_offset.restype = ctypes.c_size_t
-            L.tq_plane2_index_rec_offset.argtypes = [i32]
-            L.tq_plane2_index_row_offset.restype = ctypes.c_size_t
-            L.tq_plane2_index_row_offset.argtypes = [i32, i64]
+            L.tq_plane2_index_capacity.restype = ctypes.c_size_t
+            L.tq_plane2_index_capacity.argtypes = [i32, i64]
+            L.tq_plane2_index_slot_offset.restype = ctypes.c_size_t
+            L.tq_plane2_index_slot_offset.argtypes = [i32]
             L.tq_plane2_index.restype = ctypes.c_int
-            L.tq_plane2_index.argtypes = [i32, i32, vp, vp, i64, vp, vp]
+            L.tq_plane2_index.argtypes = [i32, i32, vp, vp, i64, vp, vp, vp, vp]
             L.tq_unpack.restype = ctypes.c_int
             L.tq_unpack.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             sz = ctypes.c_size_t
@@ -157,13 +157,14 @@ def tq_unpack(N, K, plane1, plane2, sal, rowptr, T1, T2, d_status, stream=None):
                            _stream(stream)), "tq_unpack")
 
 
-def tq_plane2_index(N, K, sal, rowptr, nnz, stream=None):
-    """The second-plane index of a weight (int32 device tensor), see tq.h."""
+def tq_plane2_index(N, K, sal, rowptr, nnz, plane2, scale2, stream=None):
+    """The group-ordered second-plane index of a weight (int32 device tensor), see tq.h."""
     nbytes = int(lib().tq_plane2_index_bytes(N, K, nnz))
     if nbytes == 0:
         raise TQError(-2, "tq_plane2_index_bytes")
     idx = torch.empty(nbytes // 4, dtype=torch.int32, device=sal.device)
-    _check(lib().tq_plane2_index(N, K, _p(sal), _p(rowptr), nnz, _p(idx), _stream(stream)), "tq_plane2_index")
+    _check(lib().tq_plane2_index(N, K, _p(sal), _p(rowptr), nnz, _p(plane2), _p(scale2), _p(idx), _stream(stream)),
+           "tq_plane2_index")
     return idx
 
 
@@ -224,7 +225,7 @@ def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True, index=True) -
             raise TQError(-4, f"tq_pack data status {st:#x}")
     if s2 is None or nnz == 0:
         s2 = torch.zeros(1, dtype=torch.float16, device=dev)
-    p2index = tq_plane2_index(N, K, sal, rowptr, nnz, stream) if index and nnz > 0 else None
+    p2index = tq_plane2_index(N, K, sal, rowptr, nnz, plane2, s2, stream) if index and nnz > 0 else None
     return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz, p2index)
 
 

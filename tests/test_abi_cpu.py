@@ -59,10 +59,14 @@ def test_host_side_argument_errors_without_gpu():
     assert tq.tq_workspace_bytes(16, 4096, 4096) == 32 * (5120 + 128)
     assert tq.tq_workspace_bytes(40, 64, 4096) == 256
     assert tq.tq_workspace_bytes(1, 4096, 100) == 0
-    # second-plane index: colptr (G + 1, padded to 4), rec and row (each nnz, padded to 4), int32
+    # second-plane index: int32 colptr[G + 1] padded to 128 bytes, then 32-byte slots for
+    # up to nnz + 15 G entries (each group padded to 16), rounded up to 16 entries
     L = tq.lib()
-    assert L.tq_plane2_index_rec_offset(4096) == 36
-    assert L.tq_plane2_index_row_offset(4096, 13) == 36 + 16
-    assert L.tq_plane2_index_bytes(100, 4096, 13) == 4 * (36 + 16 + 16)
+    assert L.tq_plane2_index_slot_offset(4096) == 256  # 33 x 4 = 132 -> 256
+    assert L.tq_plane2_index_slot_offset(128) == 128
+    assert L.tq_plane2_index_capacity(4096, 13) == 496  # 13 + 15 x 32 = 493 -> 496
+    assert L.tq_plane2_index_capacity(4096, 0) == 480
+    assert L.tq_plane2_index_bytes(100, 4096, 13) == 256 + 32 * 496
     assert L.tq_plane2_index_bytes(100, 4096, 100 * 32 + 1) == 0  # more records than groups
+    assert L.tq_plane2_index_bytes(100, 4000, 13) == 0  # K not a multiple of 128
     assert tq.tq_workspace_bytes(1, 0, 4096) == 0

@@ -122,26 +122,52 @@ def test_large_rowptr(H):
     assert np.array_equal(rp.cpu().numpy(), rp_o)
 
 
-@pytest.mark.parametrize("N,K,frac", [s for s in SHAPES if s[2] > 0] + [(1000, 41088, 0.05)])
+def plane2_index_model(N, K, sal, rp, p2, s2_bits, cap, slot_off):
+    """The index's bytes as tq.h lays them out, built with numpy from the
+    oracle's plane 2: (colptr int32 [G + 1], slots uint8 [cap][32])."""
+    G = K // 128
+    bits = ((sal[:, np.arange(G) // 32] >> (np.arange(G) % 32)) & 1).astype(bool)  # [N][G]
+    rank = np.cumsum(bits, axis=1) - bits  # salient groups of the row before g
+    counts = bits.sum(axis=0)
+    colptr = np.concatenate([[0], np.cumsum((counts + 15) // 16 * 16)]).astype(np.int64)
+    logical = np.zeros((cap, 32), np.uint8)
+    logical[:, 28:32] = 0xFF  # row -1 in the empty entries
+    for g in range(G):
+        rows = np.nonzero(bits[:, g])[0]
+        j = rp[rows].astype(np.int64) + rank[rows, g]
+        e = colptr[g] + np.arange(rows.size)
+        o = 2 * ((g % 8) & 1)
+        logical[e, :] = 0
+        logical[e, o:o + 26] = p2[j]
+        s2b = s2_bits[j].astype("<u2").view(np.uint8).reshape(-1, 2)
+        so = 0 if o else 26
+        logical[e, so:so + 2] = s2b
+        logical[e, 28:32] = rows.astype("<i4").view(np.uint8).reshape(-1, 4)
+    words = logical.reshape(cap, 8, 4)
+    slots = words[:, [0, 4, 1, 5, 2, 6, 3, 7], :].reshape(cap, 32)
+    return colptr, slots
+
+
+@pytest.mark.parametrize("N,K,frac", [s for s in SHAPES if s[2] > 0] + [(1000, 41088, 0.05), (37, 1152, 1.0)])
 def test_plane2_index_bit_exact(H, N, K, frac):
-    """The second-plane index lists, group by group and in row order, each
-    salient (row, group) pair's record j = rowptr[n] + rank and its row n."""
+    """The group-ordered second-plane index: per group, its salient rows in
+    order, each with its record (at the group's window alignment), s2 and row;
+    groups padded to 16 entries with empty slots; bit for bit."""
     from paper_2609_09240_gb300 import tq
     w = wl.gen_weights(N, K, frac, config=7, proj=3 * N + K)
-    G = K // 128
     rp, st = oracle.rowptr(N, K, w.sal)
     assert st == 0
+    _, p2, st = oracle.pack(N, K, w.T1, w.T2, w.sal, rp)
+    assert st == 0
     nnz = int(rp[N])
-    idx = tq.tq_plane2_index(N, K, H.dev(w.sal), H.dev(rp), nnz).cpu().numpy()
-    bits = ((w.sal[:, np.arange(G) // 32] >> (np.arange(G) % 32)) & 1).astype(bool)  # [N][G]
-    rank = np.cumsum(bits, axis=1) - bits  # salient groups of the row before g
-    colptr = np.concatenate([[0], np.cumsum(bits.sum(axis=0))]).astype(np.int64)
-    ro = int(tq.lib().tq_plane2_index_rec_offset(K))
-    wo = int(tq.lib().tq_plane2_index_row_offset(K, nnz))
-    assert ro >= G + 1 and ro % 4 == 0 and wo >= ro + nnz and wo % 4 == 0
-    np.testing.assert_array_equal(idx[:G + 1], colptr)
-    rows = np.concatenate([np.nonzero(bits[:, g])[0] for g in range(G)]) if nnz else np.zeros(0, np.int64)
-    recs = np.concatenate([rp[np.nonzero(bits[:, g])[0]] + rank[bits[:, g], g] for g in range(G)]) if nnz \
-        else np.zeros(0, np.int64)
-    np.testing.assert_array_equal(idx[wo:wo + nnz], rows)
-    np.testing.assert_array_equal(idx[ro:ro + nnz], recs)
+    s2_bits = np.ascontiguousarray(w.s2).view(np.uint16)
+    idx = tq.tq_plane2_index(N, K, H.dev(w.sal), H.dev(rp), nnz, H.dev(p2), H.dev(s2_bits)).cpu().numpy()
+    L = tq.lib()
+    cap = int(L.tq_plane2_index_capacity(K, nnz))
+    so = int(L.tq_plane2_index_slot_offset(K))
+    assert idx.size * 4 == so + 32 * cap
+    colptr, slots = plane2_index_model(N, K, w.sal, rp, p2, s2_bits, cap, so)
+    np.testing.assert_array_equal(idx[:K // 128 + 1], colptr)
+    got = idx.view(np.uint8)[so:].reshape(cap, 32)
+    bad = np.nonzero((got != slots).any(axis=1))[0]
+    assert bad.size == 0, f"{bad.size} slots differ; first {bad[0]}: {got[bad[0]]} vs {slots[bad[0]]}"
