@@ -943,33 +943,40 @@ __global__ void __launch_bounds__(kQThreads, 1)
 // Second plane with the group-ordered index (1..8 tokens).  Persistent
 // warps take units from a counter in the workspace: a unit is one of the
 // c_parts contiguous shares of one group's 16-entry tiles, numbered problem
-// by problem (each CTA builds the table of first units per problem in shared
-// memory).  For its unit a warp loads group g's B fragment and C once and
-// runs the tiles as m16 tiles: lane (r, c) loads slot words 2 jw, 2 jw + 1
-// of entries r and r + 8 (its two window words, one 8-byte load per entry;
-// a quad's loads cover the slot), decodes them with the lane-replicated
-// table and, after the MMAs, takes the entries' rows and s2 from the quad's
-// lanes that hold them; s2 (D - C) per entry is added to y2 of the entry's
-// row with a global atomic (the prep kernel zeroes y2).
-constexpr int kCThreads = 512;
+// by problem (CBase: the first unit of each problem).  For its unit a warp
+// loads group g's B fragment and C once and runs the tiles as m16 tiles:
+// lane (r, c) loads slot words 2 jw, 2 jw + 1 of entries r and r + 8 (its
+// two window words, one 8-byte load per entry; a quad's loads cover the
+// slot), decodes them with the lane-replicated table and, after the MMAs,
+// takes the entries' rows and s2 from the quad's lanes that hold them;
+// s2 (D - C) per entry is added to y2 of the entry's row with a global
+// atomic (the prep kernel zeroes y2).
+constexpr int kCThreads = 768;
 constexpr int kCDepth = 4;                        // tiles in flight per warp (in registers)
-constexpr int kCDynBytes2 = kArena1 + kLutBytes;  // unit table below the table of codes
-constexpr int kCUnitTiles = 24;                   // target tiles per unit
-static_assert((TQ_MAX_BATCH + 8 + kCThreads / 32) * 4 <= kArena1, "unit table");
+constexpr int kCDynBytes2 = kArena1 + kLutBytes;  // the table of codes at its fixed address
+constexpr int kCUnitTiles = 32;                   // target tiles per unit
+
+// The kernel's first parameter, so that the loop's indexed reads of it stay
+// at the low offsets of the parameter space.
+struct CBase {
+  int32_t count;                   // problems
+  int32_t base[TQ_MAX_BATCH + 1];  // first unit of problem p (base[count]: all units)
+};
 
 __device__ __forceinline__ int64_t c_capacity(int K, int64_t nnz) {
   return (nnz + 15 * (int64_t)(K / kGroup) + 15) & ~(int64_t)15;
 }
 __device__ __forceinline__ int64_t c_slot_off(int K) { return ((int64_t)(K / kGroup + 1) * 4 + 127) & ~(int64_t)127; }
 // Units per group: the mean tiles per group over kCUnitTiles, rounded up, 1 .. 32.
-__device__ __forceinline__ int c_parts(const Problem &P) {
-  const int64_t per = (int64_t)(P.K / kGroup) * 16 * kCUnitTiles;
-  return (int)min(max((P.nnz + per - 1) / per, (int64_t)1), (int64_t)32);
+__host__ __device__ __forceinline__ int c_parts(int K, int64_t nnz) {
+  const int64_t per = (int64_t)(K / kGroup) * 16 * kCUnitTiles;
+  const int64_t q = (nnz + per - 1) / per;
+  return (int)(q < 1 ? 1 : q > 32 ? 32 : q);
 }
 
 template <bool ONE>
 __global__ void __launch_bounds__(kCThreads, 1)
-    gemv_mma_p2c_kernel(const __grid_constant__ BatchParams bp, int32_t *counter) {
+    gemv_mma_p2c_kernel(const __grid_constant__ CBase cb, const __grid_constant__ BatchParams bp, int32_t *counter) {
   extern __shared__ __align__(1024) unsigned char dync[];
   const int tid = threadIdx.x, lane = tid & 31;
   if (smem_u32(dync) != kDynShared) {
@@ -980,32 +987,10 @@ __global__ void __launch_bounds__(kCThreads, 1)
     uint32_t *lut = reinterpret_cast<uint32_t *>(dync + kArena1);
     for (int i = tid; i < 256 * 32; i += kCThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
   }
-  // first unit of each problem: base[p] = sum over q < p of G_q * parts_q (problems without a
-  // second plane have none); an inclusive scan of one value per thread
-  int32_t *base = reinterpret_cast<int32_t *>(dync);
-  int32_t *warp_sum = base + TQ_MAX_BATCH + 8;  // (no static shared memory: it would move the window)
-  {
-    static_assert(kCThreads >= TQ_MAX_BATCH, "one problem per thread");
-    int v = 0;
-    if (tid < bp.count) {
-      const Problem &Q = bp.prob[tid];
-      if (Q.nnz > 0 && Q.p2idx) v = (Q.K / kGroup) * c_parts(Q);
-    }
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int t = __shfl_up_sync(0xffffffffu, v, o);
-      if (lane >= o) v += t;
-    }
-    if (lane == 31) warp_sum[tid >> 5] = v;
-    __syncthreads();
-    for (int w = 0; w < (tid >> 5); ++w) v += warp_sum[w];
-    if (tid == 0) base[0] = 0;
-    if (tid < TQ_MAX_BATCH) base[tid + 1] = v;
-  }
   __syncthreads();
   const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, quad = lane & ~3;
   const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
-  const int count = bp.count, total = base[count];
+  const int count = cb.count, total = cb.base[count];
   for (;;) {
     int u = 0;
     if (lane == 0) u = atomicAdd(counter, 1);
@@ -1013,16 +998,17 @@ __global__ void __launch_bounds__(kCThreads, 1)
     if (u >= total) break;
     int i = 0;  // the unit's problem: the last i with base[i] <= u
     for (int step = 128; step >= 1; step >>= 1)
-      if (i + step < count && base[i + step] <= u) i += step;
+      if (i + step < count && cb.base[i + step] <= u) i += step;
     const Problem &P = bp.prob[i];
-    const int S = c_parts(P), local = u - base[i];
+    const int S = c_parts(P.K, P.nnz), local = u - cb.base[i];
     const int g = local / S, part = local - g * S, GL = g % kStageG;
     // the group's entries, clamped into the index (whole tiles)
     const int64_t cap = c_capacity(P.K, P.nnz);
     const int64_t e0 = min(max((int64_t)__ldg(P.p2idx + g), (int64_t)0), cap) & ~(int64_t)15;
     const int64_t e1 = min(max((int64_t)__ldg(P.p2idx + g + 1), e0), cap) & ~(int64_t)15;
-    const int nt = (int)((e1 - e0) >> 4);
-    const int t0 = (int)((int64_t)nt * part / S), n = (int)((int64_t)nt * (part + 1) / S) - t0;
+    const uint32_t nt = (uint32_t)((e1 - e0) >> 4);  // below 2^27: nt * 32 fits 32 bits
+    const int t0 = (int)(nt * (uint32_t)part / (uint32_t)S);
+    const int n = (int)(nt * (uint32_t)(part + 1) / (uint32_t)S) - t0;
     if (n <= 0) continue;
     // the group's B fragment (lanes of absent tokens repeat the last token) and C
     const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB + min(g16, MB - 1) * kBTok + c * kBLane;
@@ -1447,7 +1433,7 @@ static bool scales_by_map(const Problem &P) {
 }
 
 static_assert(sizeof(BatchParams) + sizeof(mm::MapTemplates) + 8 <= 32764, "prep kernel parameters");
-static_assert(sizeof(BatchParams) + 8 <= 32764, "indexed second-plane kernel parameters");
+static_assert(sizeof(mm::CBase) + sizeof(BatchParams) + 8 <= 32764, "indexed second-plane kernel parameters");
 static_assert(sizeof(BatchParams) + sizeof(mm::Sched) <= 32764, "main kernel parameters");
 
 // Distinct tensor-map templates of a batch's problems (up to `cap` + 1 are
@@ -1564,8 +1550,16 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx)
       all_idx = false;
   int32_t *counter = nullptr;
-  if (any2 && all_idx)
+  thread_local mm::CBase cb;
+  if (any2 && all_idx) {
+    cb.count = bp.count;
+    cb.base[0] = 0;
+    for (int p = 0; p < bp.count; ++p) {
+      const Problem &P = bp.prob[p];
+      cb.base[p + 1] = cb.base[p] + (P.nnz > 0 ? P.K / kGroup * mm::c_parts(P.K, P.nnz) : 0);
+    }
     counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + mm::kCounterOff);
+  }
   mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -1573,7 +1567,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true> : mm::gemv_mma_p2c_kernel<false>;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
-    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(bp, counter);
+    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(cb, bp, counter);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   } else if (any2 && gmax <= mm::kQMaxG) {

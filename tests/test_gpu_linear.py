@@ -132,6 +132,31 @@ def test_batched_many_row_lengths(H):
         H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
 
 
+@pytest.mark.parametrize("index", [True, False])
+@pytest.mark.parametrize("M", [1, 3])
+def test_batched_max_problems(H, M, index):
+    """A batch of TQ_MAX_BATCH problems, all with a second plane: the last
+    problems' descriptors sit at the far end of the kernels' parameter
+    space, which every per-problem read has to reach."""
+    from paper_2609_09240_gb300 import tq
+    shapes = [(48, 256), (80, 640), (48, 640), (80, 256)]
+    items, refs = [], []
+    for i in range(tq.TQ_MAX_BATCH):
+        N, K = shapes[i % 4]
+        w = wl.gen_weights(N, K, 0.3, config=8, proj=i)
+        x = wl.gen_x(M, K, config=8, proj=i)
+        refs.append(H.oracle_ref(w, x))
+        items.append((H.pack_on_gpu(w, index=index), H.dev(x), torch.empty((M, N), dtype=torch.float16, device="cuda")))
+    b = tq.Batch(M, items)
+    tq.tq_linear_batched(b)
+    H.device_status_ok()
+    for i, ((pw, xd, y), (y_ref, a_ref)) in enumerate(zip(items, refs)):
+        try:
+            H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+        except AssertionError as e:
+            raise AssertionError(f"problem {i}: {e}") from None
+
+
 @pytest.mark.parametrize("N,K,frac", [(1, 128, 1.0), (129, 256, 0.5), (300, 9728, 0.1), (700, 4096, 0.3)])
 @pytest.mark.parametrize("M", [1, 3, 8])
 def test_second_plane_without_index(H, N, K, frac, M):
