@@ -23,6 +23,9 @@
 // three fp16 values off - s1, off, off + s1 held in two registers; a
 // 243-entry table gives, per digit, the PRMT selector nibbles of its value,
 // so two weights cost one PRMT.  Every wait is bounded.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "tq_common.cuh"
 #include "tq_sm100.cuh"
 
@@ -104,6 +107,100 @@ __device__ __forceinline__ void decode_weights(const uint32_t *rw, uint32_t v01,
   }
 }
 
+// One weight row's data for one group, loaded a group ahead of its decode:
+// the raw aligned words of its 26 bytes and of its plane-2 record, s1, off,
+// s2, and whether the group is salient.
+struct RowGroup {
+  uint32_t r8[7], q8[7];
+  unsigned short s1, of, s2;
+  bool odd, rodd, salient;
+};
+
+// Walks one weight row group by group (thread = row): fetch() issues the
+// loads of group g (nothing waits for them until the group is decoded).
+struct RowWalker {
+  const Problem *P;
+  const uint8_t *row;
+  const uint32_t *salrow;
+  int64_t j;      // record index of the row's next salient group
+  uint32_t salw;  // the row's current salience word
+  int G, n;
+  bool valid;
+  __device__ RowWalker(const Problem &p, int n_) : P(&p), n(n_) {
+    const int K = p.K, W = sal_words_of(K);
+    G = K / kGroup;
+    valid = n < p.N;
+    row = p.plane1 + (int64_t)(valid ? n : 0) * row_bytes_of(K);
+    salrow = p.sal + (int64_t)(valid ? n : 0) * W;
+    j = (valid && p.nnz > 0) ? p.rowptr[n] : 0;
+    salw = (valid && p.nnz > 0) ? __ldg(salrow) : 0u;
+  }
+  __device__ void fetch(int g, RowGroup &nx) {
+    // plane-1 rows are 16-byte aligned and groups are 26 bytes, so group g
+    // starts 0 or 2 bytes into a word; 7 aligned words cover it
+    nx.odd = g & 1;
+    const uint32_t *src = reinterpret_cast<const uint32_t *>(row + (int64_t)g * kGroupBytes - (nx.odd ? 2 : 0));
+#pragma unroll
+    for (int i = 0; i < 7; ++i) nx.r8[i] = valid ? __ldg(src + i) : 0x79797979u;  // 121: all-zero trits
+    const unsigned short *s1h = reinterpret_cast<const unsigned short *>(P->s1);
+    const unsigned short *ofh = reinterpret_cast<const unsigned short *>(P->off);
+    nx.s1 = valid ? __ldg(s1h + (int64_t)n * G + g) : (unsigned short)0;
+    nx.of = valid ? __ldg(ofh + (int64_t)n * G + g) : (unsigned short)0;
+    if ((g & 31) == 0 && g > 0 && valid && P->nnz > 0) salw = __ldg(salrow + (g >> 5));
+    nx.salient = (salw >> (g & 31)) & 1u;
+    nx.s2 = 0;
+    nx.rodd = false;
+#pragma unroll
+    for (int i = 0; i < 7; ++i) nx.q8[i] = 0x79797979u;
+    if (nx.salient) {
+      const int64_t jj = j < P->nnz ? j : P->nnz - 1;
+      const int64_t off0 = jj * kGroupBytes;
+      nx.rodd = (off0 & 3) != 0;  // plane 2 is 16-byte aligned: records start 0 or 2 bytes into a word
+      const uint32_t *rs = reinterpret_cast<const uint32_t *>(P->plane2 + off0 - (nx.rodd ? 2 : 0));
+#pragma unroll
+      for (int i = 0; i < 6; ++i) nx.q8[i] = __ldg(rs + i);
+      nx.q8[6] = nx.rodd ? __ldg(rs + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(rs + 6));
+      nx.s2 = __ldg(reinterpret_cast<const unsigned short *>(P->s2) + jj);
+      ++j;
+    }
+  }
+};
+
+// the 7 words of a 26-byte run, byte 0 first, from its raw aligned words
+__device__ __forceinline__ void realign(const uint32_t *r8, bool odd, uint32_t *rw) {
+#pragma unroll
+  for (int i = 0; i < 7; ++i) rw[i] = odd ? __funnelshift_r(r8[i], i < 6 ? r8[i + 1] : 0u, 16) : r8[i];
+}
+
+// The group's 128 fp16 weights of one row (64 words): s1 t1 + off, plus
+// s2 t2 when any row of the warp is salient (other rows add zeros).
+__device__ __forceinline__ void decode_row_group(const RowGroup &cur, const uint64_t *sel, uint32_t *wv) {
+  const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
+  uint32_t rw[7];
+  realign(cur.r8, cur.odd, rw);
+  const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
+  const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+  const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
+  decode_weights(rw, v01, v22, sel, wv);
+  if (__any_sync(0xffffffffu, cur.salient)) {
+    const float s2 = __half2float(__ushort_as_half(cur.s2));
+    uint32_t rec[7];
+    realign(cur.q8, cur.rodd, rec);
+    const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
+    const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
+    const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
+    uint32_t w2[64];
+    decode_weights(rec, u01, u22, sel, w2);
+#pragma unroll
+    for (int i = 0; i < 64; ++i) {
+      const __half2 a = *reinterpret_cast<const __half2 *>(&wv[i]);
+      const __half2 b = *reinterpret_cast<const __half2 *>(&w2[i]);
+      const __half2 c = __hadd2(a, b);
+      wv[i] = *reinterpret_cast<const uint32_t *>(&c);
+    }
+  }
+}
+
 // Core-matrix offset of (row, K element e) in a tile of 8-row groups x 16
 // core matrices along K.
 __device__ __forceinline__ int cm_off(int row, int e) { return ((row >> 3) * 16 + (e >> 3)) * 128 + (row & 7) * 16; }
@@ -113,8 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
-  const int K = P.K, N = P.N, G = K / kGroup, W = sal_words_of(K);
-  const int64_t RB = row_bytes_of(K);
+  const int K = P.K, N = P.N, G = K / kGroup;
   uint64_t *sel = reinterpret_cast<uint64_t *>(smem + oSel);
   Bars *bars = reinterpret_cast<Bars *>(smem + oBar);
   volatile int32_t *abort_ = &bars->abort_;
@@ -136,58 +232,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
 
   if (tid < kDecThreads) {
     // ============================================= x copies + weight decode
-    const int r = tid, n = n0 + r;
-    const bool valid = n < N;
-    const uint8_t *row = P.plane1 + (int64_t)(valid ? n : 0) * RB;
-    const uint32_t *salrow = P.sal + (int64_t)(valid ? n : 0) * W;
-    // Everything a group needs from global memory is loaded one group ahead:
-    // its 26 bytes, s1, off, whether it is salient and then its plane-2
-    // record and s2.
-    struct Next {
-      uint32_t r8[7], q8[7];  // raw aligned words of the group and of its record
-      unsigned short s1, of, s2;
-      bool odd, rodd, salient;
-    };
-    int64_t j = (valid && P.nnz > 0) ? P.rowptr[n] : 0;  // record index of the row's next salient group
-    uint32_t salw = (valid && P.nnz > 0) ? __ldg(salrow) : 0u;
-    // issues the loads only: nothing here waits for them (they are used one
-    // group later)
-    auto fetch = [&](int g, Next &nx) {
-      // plane-1 rows are 16-byte aligned and groups are 26 bytes, so group g
-      // starts 0 or 2 bytes into a word; 7 aligned words cover it
-      nx.odd = g & 1;
-      const uint32_t *src = reinterpret_cast<const uint32_t *>(row + (int64_t)g * kGroupBytes - (nx.odd ? 2 : 0));
-#pragma unroll
-      for (int i = 0; i < 7; ++i) nx.r8[i] = valid ? __ldg(src + i) : 0x79797979u;  // 121: all-zero trits
-      const unsigned short *s1h = reinterpret_cast<const unsigned short *>(P.s1);
-      const unsigned short *ofh = reinterpret_cast<const unsigned short *>(P.off);
-      nx.s1 = valid ? __ldg(s1h + (int64_t)n * G + g) : (unsigned short)0;
-      nx.of = valid ? __ldg(ofh + (int64_t)n * G + g) : (unsigned short)0;
-      if ((g & 31) == 0 && g > 0 && valid && P.nnz > 0) salw = __ldg(salrow + (g >> 5));
-      nx.salient = (salw >> (g & 31)) & 1u;
-      nx.s2 = 0;
-      nx.rodd = false;
-#pragma unroll
-      for (int i = 0; i < 7; ++i) nx.q8[i] = 0x79797979u;
-      if (nx.salient) {
-        const int64_t jj = j < P.nnz ? j : P.nnz - 1;
-        const int64_t off0 = jj * kGroupBytes;
-        nx.rodd = (off0 & 3) != 0;  // plane 2 is 16-byte aligned: records start 0 or 2 bytes into a word
-        const uint32_t *rs = reinterpret_cast<const uint32_t *>(P.plane2 + off0 - (nx.rodd ? 2 : 0));
-#pragma unroll
-        for (int i = 0; i < 6; ++i) nx.q8[i] = __ldg(rs + i);
-        nx.q8[6] = nx.rodd ? __ldg(rs + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(rs + 6));
-        nx.s2 = __ldg(reinterpret_cast<const unsigned short *>(P.s2) + jj);
-        ++j;
-      }
-    };
-    // the 7 words of a 26-byte run, byte 0 first, from its raw aligned words
-    auto realign = [](const uint32_t *r8, bool odd, uint32_t *rw) {
-#pragma unroll
-      for (int i = 0; i < 7; ++i) rw[i] = odd ? __funnelshift_r(r8[i], i < 6 ? r8[i + 1] : 0u, 16) : r8[i];
-    };
-    Next nx;
-    fetch(0, nx);
+    const int r = tid;
+    RowWalker rwk(P, n0 + r);
+    RowGroup nx;
+    rwk.fetch(0, nx);
     bool ok = true;
     for (int g = 0; g < G && ok; ++g) {
       const int s = g % NS;
@@ -208,35 +256,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
                      : "memory");
       }
       asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&bars->full[s])) : "memory");
-      const Next cur = nx;
-      if (g + 1 < G) fetch(g + 1, nx);
-      const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
-      const bool salient = cur.salient;
-      uint32_t rw[7];
-      realign(cur.r8, cur.odd, rw);
-      const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
-      const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-      const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
+      const RowGroup cur = nx;
+      if (g + 1 < G) rwk.fetch(g + 1, nx);
       uint32_t wv[64];
-      decode_weights(rw, v01, v22, sel, wv);
-      if (__any_sync(0xffffffffu, salient)) {
-        // second plane: + s2 t2 on salient groups (other rows add zeros)
-        const float s2 = __half2float(__ushort_as_half(cur.s2));
-        uint32_t rec[7];
-        realign(cur.q8, cur.rodd, rec);
-        const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
-        const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
-        const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
-        uint32_t w2[64];
-        decode_weights(rec, u01, u22, sel, w2);
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          const __half2 a = *reinterpret_cast<const __half2 *>(&wv[i]);
-          const __half2 b = *reinterpret_cast<const __half2 *>(&w2[i]);
-          const __half2 c = __hadd2(a, b);
-          wv[i] = *reinterpret_cast<const uint32_t *>(&c);
-        }
-      }
+      decode_row_group(cur, sel, wv);
       // 16 core-matrix rows of 8 weights
 #pragma unroll
       for (int kc = 0; kc < 16; ++kc)
@@ -314,13 +337,228 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
   }
 }
 
+// ------------------------------------------------------------------------
+// prefill2_kernel: a 256-row x 256-token output tile per CTA, weights as the
+// MMA's M operand (two halves of 128 rows), tokens as N = 256.
+//  * warps 0..7 (thread r = weight row n0 + r): decode each group's 128
+//    weights of their row into a 2-slot ring of weight tiles (64 KiB, the
+//    no-swizzle K-major core-matrix layout, 16 core matrices along K);
+//  * warp 8 (one thread): the x tiles, 256 tokens x 64 K (32 KiB) per stage,
+//    one 4-D tensor copy each (element, token in group of 8, 8-element
+//    chunk, token group: the box lands in exactly the core-matrix layout),
+//    into a 3-slot ring, two stages per group;
+//  * warp 9 (one thread): per stage 8 MMAs (M = 128 rows, N = 256 tokens,
+//    K = 16; rows 0..127 into tensor-memory columns 0..255, rows 128..255
+//    into 256..511);
+//  * at the end warps 0..7 read the accumulators and write y.
+// A decoded weight tile serves 256 tokens and 16 MMAs.  Needs M % 8 == 0
+// (the token-group view of x) and a tensor map that the host encodes.
+constexpr int BR2 = 256;                 // weight rows per CTA
+constexpr int BT2 = 256;                 // tokens per CTA (MMA N)
+constexpr int XK2 = 64;                  // K per x stage
+constexpr int kXStage2 = BT2 * XK2 * 2;  // 32 KiB
+constexpr int kWTile2 = BR2 * BK * 2;    // 64 KiB
+constexpr int NW2 = 2, NX2 = 3;
+constexpr int oW2 = 0;
+constexpr int oX2 = NW2 * kWTile2;
+constexpr int oSel2 = oX2 + NX2 * kXStage2;
+constexpr int oBar2 = oSel2 + 256 * 8;
+constexpr int kSmem2 = oBar2 + 256;
+static_assert(kSmem2 <= 232448, "prefill2 shared memory");
+constexpr int kDecWarps2 = 8, kWarpProd2 = 8, kWarpMma2 = 9;
+constexpr int kThreads2 = 10 * 32;
+constexpr uint32_t kTmemCols2 = 512;
+
+struct Bars2 {
+  uint64_t xfull[NX2], xempty[NX2], wfull[NW2], wempty[NW2], done;
+  uint32_t tmem_slot;
+  int32_t abort_;
+};
+static_assert(sizeof(Bars2) <= 256, "prefill2 barriers");
+
+template <bool F32>
+__global__ void __launch_bounds__(kThreads2, 1)
+    prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap, int M) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int m0 = blockIdx.x * BT2, n0 = blockIdx.y * BR2;
+  const int N = P.N, G = P.K / kGroup;
+  uint64_t *sel = reinterpret_cast<uint64_t *>(smem + oSel2);
+  Bars2 *bars = reinterpret_cast<Bars2 *>(smem + oBar2);
+  volatile int32_t *abort_ = &bars->abort_;
+  for (int i = tid; i < 256; i += kThreads2) sel[i] = sel_entry(i);
+  if (tid == 0) {
+    for (int i = 0; i < NX2; ++i) {
+      mbar_init(&bars->xfull[i], 1);  // the producer's expect-tx arrival
+      mbar_init(&bars->xempty[i], 1);
+    }
+    for (int i = 0; i < NW2; ++i) {
+      mbar_init(&bars->wfull[i], kDecWarps2 * 32);
+      mbar_init(&bars->wempty[i], 1);
+    }
+    mbar_init(&bars->done, 1);
+    bars->abort_ = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(&bars->tmem_slot, kTmemCols2);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_slot;
+
+  if (warp < kDecWarps2) {
+    // ======================================================= weight decode
+    const int r = tid;
+    RowWalker rwk(P, n0 + r);
+    RowGroup nx;
+    rwk.fetch(0, nx);
+    for (int g = 0; g < G; ++g) {
+      const int s = g % NW2;
+      if (g >= NW2 && !__all_sync(0xffffffffu, wait_or_abort(&bars->wempty[s], ((uint32_t)(g / NW2) & 1u) ^ 1u, abort_)))
+        break;
+      const RowGroup cur = nx;
+      if (g + 1 < G) rwk.fetch(g + 1, nx);
+      uint32_t wv[64];
+      decode_row_group(cur, sel, wv);
+      unsigned char *Wt = smem + oW2 + s * kWTile2;
+#pragma unroll
+      for (int kc = 0; kc < 16; ++kc)
+        *reinterpret_cast<uint4 *>(Wt + cm_off(r, kc * 8)) =
+            make_uint4(wv[4 * kc], wv[4 * kc + 1], wv[4 * kc + 2], wv[4 * kc + 3]);
+      fence_proxy_async_smem();  // the MMA reads these stores through the async proxy
+      mbar_arrive(&bars->wfull[s]);
+    }
+  } else if (warp == kWarpProd2) {
+    // ============================================================ x tiles
+    if (lane == 0) {
+      uint32_t issued = 0;
+      for (int xs = 0; xs < 2 * G; ++xs) {
+        const int sl = xs % NX2;
+        if (xs >= NX2 && !wait_or_abort(&bars->xempty[sl], ((uint32_t)(xs / NX2) & 1u) ^ 1u, abort_)) break;
+        mbar_arrive_expect_tx(&bars->xfull[sl], (uint32_t)kXStage2);
+        // element 0, token 0 of the group, chunk (K / 8), token group
+        asm volatile(
+            "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(
+                smem_u32(smem + oX2 + sl * kXStage2)),
+            "l"(&xmap), "r"(0), "r"(0), "r"(xs * (XK2 / 8)), "r"(m0 / 8), "r"(smem_u32(&bars->xfull[sl]))
+            : "memory");
+        ++issued;
+      }
+      // every issued copy lands before the CTA exits (bounded)
+      for (uint32_t k = (issued > (uint32_t)NX2 ? issued - NX2 : 0); k < issued; ++k)
+        mbar_wait(&bars->xfull[k % NX2], (k / NX2) & 1u);
+    }
+  } else if (lane == 0) {
+    // ================================================================= MMA
+    const uint32_t idesc = idesc_f16_f32(128, BT2);
+    bool ok = true;
+    for (int g = 0; g < G && ok; ++g) {
+      const int s = g % NW2;
+      if (!wait_or_abort(&bars->wfull[s], (uint32_t)(g / NW2) & 1u, abort_)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t Wb = smem_u32(smem + oW2 + s * kWTile2);
+      for (int h = 0; h < 2; ++h) {
+        const int xs = 2 * g + h, sl = xs % NX2;
+        if (!wait_or_abort(&bars->xfull[sl], (uint32_t)(xs / NX2) & 1u, abort_)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t Xb = smem_u32(smem + oX2 + sl * kXStage2);
+#pragma unroll
+        for (int kk = 0; kk < XK2 / 16; ++kk) {
+          const uint64_t bdesc = smem_desc(Xb + kk * 256, 128, 1024);
+          const uint32_t acc = (g > 0 || h > 0 || kk > 0) ? 1u : 0u;
+#pragma unroll
+          for (int half = 0; half < 2; ++half)
+            mma_smemA(tmem + (uint32_t)(half * BT2), smem_desc(Wb + half * (kWTile2 / 2) + (4 * h + kk) * 256, 128, 2048),
+                      bdesc, idesc, acc);
+        }
+        mma_commit(&bars->xempty[sl]);
+      }
+      if (ok) mma_commit(&bars->wempty[s]);
+    }
+    if (ok) mma_commit(&bars->done);
+  }
+
+  // ================================================================ epilogue
+  __syncwarp();
+  if (warp < kDecWarps2) {
+    const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->done, 0u, abort_));
+    tc_fence_after();
+    if (ok) {
+      const int q = warp & 3, half = warp >> 2;  // tensor-memory lanes 32q.., rows 128 half..
+      const int n = n0 + half * 128 + 32 * q + lane;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BT2; c0 += 8) {
+        uint32_t v[8];
+        tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * BT2 + c0), v);
+        tmem_wait_ld();
+        if (n < N) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int m = m0 + c0 + i;
+            if (m < M) {
+              if (F32)
+                static_cast<float *>(P.y)[(int64_t)m * N + n] = __uint_as_float(v[i]);
+              else
+                static_cast<__half *>(P.y)[(int64_t)m * N + n] = __float2half_rn(__uint_as_float(v[i]));
+            }
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols2);
+  }
+}
+
 }  // namespace pf
 
 TQ_STATUS_ACCESSOR(read_status_prefill)
 
+// x [M][K] fp16 as a 4-D tensor (element, token within a group of 8, 8-element
+// chunk, token group) whose box (8, 8, 8, 32) lands in shared memory in the
+// no-swizzle K-major core-matrix layout.  false when the driver's encoder is
+// unavailable or refuses.
+static bool encode_x_map(const void *x, int M, int K, CUtensorMap *out) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      fn = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }();
+  if (!encode) return false;
+  cuuint64_t dims[4] = {8, 8, (cuuint64_t)(K / 8), (cuuint64_t)(M / 8)};
+  cuuint64_t strides[3] = {(cuuint64_t)K * 2, 16, (cuuint64_t)K * 16};
+  cuuint32_t box[4] = {8, 8, (cuuint32_t)(pf::XK2 / 8), (cuuint32_t)(pf::BT2 / 8)};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
-  const dim3 grid((M + pf::BM - 1) / pf::BM, (P.N + pf::BN - 1) / pf::BN);
   cudaError_t e;
+  CUtensorMap xmap;
+  if (M % 8 == 0 && encode_x_map(P.x, M, P.K, &xmap)) {
+    const dim3 grid((M + pf::BT2 - 1) / pf::BT2, (P.N + pf::BR2 - 1) / pf::BR2);
+    auto kern = f32 ? pf::prefill2_kernel<true> : pf::prefill2_kernel<false>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem2);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, M);
+    return cudaGetLastError();
+  }
+  const dim3 grid((M + pf::BM - 1) / pf::BM, (P.N + pf::BN - 1) / pf::BN);
   if (f32) {
     e = cudaFuncSetAttribute(pf::prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem);
     if (e != cudaSuccess) return e;

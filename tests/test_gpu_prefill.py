@@ -1,6 +1,8 @@
 """GPU parity of the prefill tile path (M > 16 tokens: weight tiles
 dequantized to fp16 and multiplied on the tensor cores) against the fp64 CPU
-oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element.  The full-size case
+oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element.  Token counts that are
+multiples of 8 take the kernel fed by tensor copies of x, the others the
+per-thread-copy kernel; both appear below.  The full-size case
 is the Qwen3-8B prefill shape (M = 2048 tokens) checked on sampled rows."""
 import numpy as np
 import pytest
@@ -23,6 +25,8 @@ def H():
     (200, 300, 4224, 0.1, False),   # odd group count, ragged rows and tokens
     (256, 520, 2560, 1.0, False),   # every group salient
     (64, 1, 128, 0.5, True),        # one row, one group
+    (24, 257, 640, 0.3, True),      # smallest token multiple of 8 past the decode path; a one-row second row tile
+    (264, 384, 1152, 0.2, False),   # a second token tile of 8 tokens; odd group count
 ])
 def test_prefill_small(H, M, N, K, frac, f32):
     from paper_2609_09240_gb300 import tq
