@@ -376,12 +376,12 @@ struct Bars2 {
 };
 static_assert(sizeof(Bars2) <= 256, "prefill2 barriers");
 
-template <bool F32>
+template <bool F32, int NH>
 __global__ void __launch_bounds__(kThreads2, 1)
     prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap, int M) {
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * BT2, n0 = blockIdx.y * BR2;
+  const int m0 = blockIdx.x * BT2, n0 = blockIdx.y * (NH * 128);
   const int N = P.N, G = P.K / kGroup;
   uint64_t *sel = reinterpret_cast<uint64_t *>(smem + oSel2);
   Bars2 *bars = reinterpret_cast<Bars2 *>(smem + oBar2);
@@ -393,7 +393,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
       mbar_init(&bars->xempty[i], 1);
     }
     for (int i = 0; i < NW2; ++i) {
-      mbar_init(&bars->wfull[i], kDecWarps2 * 32);
+      mbar_init(&bars->wfull[i], NH * 128);
       mbar_init(&bars->wempty[i], 1);
     }
     mbar_init(&bars->done, 1);
@@ -406,7 +406,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_slot;
 
-  if (warp < kDecWarps2) {
+  if (warp < NH * 4) {
     // ======================================================= weight decode
     const int r = tid;
     RowWalker rwk(P, n0 + r);
@@ -448,7 +448,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
       for (uint32_t k = (issued > (uint32_t)NX2 ? issued - NX2 : 0); k < issued; ++k)
         mbar_wait(&bars->xfull[k % NX2], (k / NX2) & 1u);
     }
-  } else if (lane == 0) {
+  } else if (warp == kWarpMma2 && lane == 0) {
     // ================================================================= MMA
     const uint32_t idesc = idesc_f16_f32(128, BT2);
     bool ok = true;
@@ -473,7 +473,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
           const uint64_t bdesc = smem_desc(Xb + kk * 256, 128, 1024);
           const uint32_t acc = (g > 0 || h > 0 || kk > 0) ? 1u : 0u;
 #pragma unroll
-          for (int half = 0; half < 2; ++half)
+          for (int half = 0; half < NH; ++half)
             mma_smemA(tmem + (uint32_t)(half * BT2), smem_desc(Wb + half * (kWTile2 / 2) + (4 * h + kk) * 256, 128, 2048),
                       bdesc, idesc, acc);
         }
@@ -490,10 +490,14 @@ __global__ void __launch_bounds__(kThreads2, 1)
     const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->done, 0u, abort_));
     tc_fence_after();
     if (ok) {
-      const int q = warp & 3, half = warp >> 2;  // tensor-memory lanes 32q.., rows 128 half..
+      // tensor-memory lanes 32 q..; two row halves (all tokens each), or for
+      // 128-row tiles two token halves of the one accumulator
+      const int q = warp & 3, sel2 = warp >> 2;
+      const int half = NH == 2 ? sel2 : 0;
+      const int cb = NH == 2 ? 0 : sel2 * (BT2 / 2), ce = NH == 2 ? BT2 : cb + BT2 / 2;
       const int n = n0 + half * 128 + 32 * q + lane;
 #pragma unroll 1
-      for (int c0 = 0; c0 < BT2; c0 += 8) {
+      for (int c0 = cb; c0 < ce; c0 += 8) {
         uint32_t v[8];
         tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * BT2 + c0), v);
         tmem_wait_ld();
@@ -551,8 +555,12 @@ cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
   cudaError_t e;
   CUtensorMap xmap;
   if (M % 8 == 0 && encode_x_map(P.x, M, P.K, &xmap)) {
-    const dim3 grid((M + pf::BT2 - 1) / pf::BT2, (P.N + pf::BR2 - 1) / pf::BR2);
-    auto kern = f32 ? pf::prefill2_kernel<true> : pf::prefill2_kernel<false>;
+    // 128-row tiles when 256-row tiles would leave more than half of the SMs idle
+    const int mt = (M + pf::BT2 - 1) / pf::BT2;
+    const bool narrow = (int64_t)mt * ((P.N + pf::BR2 - 1) / pf::BR2) * 2 <= 152;
+    const dim3 grid(mt, narrow ? (P.N + 127) / 128 : (P.N + pf::BR2 - 1) / pf::BR2);
+    auto kern = narrow ? (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>)
+                       : (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem2);
     if (e != cudaSuccess) return e;
     kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, M);

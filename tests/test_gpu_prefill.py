@@ -54,3 +54,22 @@ def test_prefill_qwen3_8b_shape_sampled_rows(H, name, N, K, nrows):
     rows = np.sort(np.random.default_rng(4).choice(N, size=nrows, replace=False)).astype(np.int32)
     y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
     H.assert_close(y[:, rows], y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M,N,K,narrow", [(2048, 2560, 640, False), (2048, 1024, 640, True)])
+def test_prefill_tile_heights_sampled_rows(H, M, N, K, narrow):
+    """Both row-tile heights of the tensor-copy kernel at M = 2048: 256-row
+    tiles when they fill the GPU (2560 rows), 128-row tiles when 256-row
+    ones would leave most SMs idle (1024 rows); sampled rows of every tile."""
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, 0.2, config=4, layer=1, proj=N % 89)
+    xb = wl.gen_x(M, K, config=4, layer=1, proj=N % 89)
+    pw = H.pack_on_gpu(w)
+    y = tq.tq_linear(H.dev(xb), pw).float().cpu().numpy()
+    H.device_status_ok()
+    tile = 128 if narrow else 256
+    rng = np.random.default_rng(N)
+    rows = np.sort(np.concatenate([t * tile + rng.choice(tile, size=2, replace=False)
+                                   for t in range(N // tile)])).astype(np.int32)
+    y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
+    H.assert_close(y[:, rows], y_ref, a_ref)
