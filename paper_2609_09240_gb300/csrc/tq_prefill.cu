@@ -344,15 +344,15 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
 //    weights of their row into a 2-slot ring of weight tiles (64 KiB, the
 //    no-swizzle K-major core-matrix layout, 16 core matrices along K);
 //  * warp 8 (one thread): the x tiles, 256 tokens x 64 K (32 KiB) per stage,
-//    one 4-D tensor copy each (element, token in group of 8, 8-element
-//    chunk, token group: the box lands in exactly the core-matrix layout),
-//    into a 3-slot ring, two stages per group;
+//    one 2-D tensor copy each with 128-byte swizzling (the K-major layout
+//    the MMA reads through a swizzled descriptor), into a 3-slot ring, two
+//    stages per group;
 //  * warp 9 (one thread): per stage 8 MMAs (M = 128 rows, N = 256 tokens,
 //    K = 16; rows 0..127 into tensor-memory columns 0..255, rows 128..255
 //    into 256..511);
 //  * at the end warps 0..7 read the accumulators and write y.
-// A decoded weight tile serves 256 tokens and 16 MMAs.  Needs M % 8 == 0
-// (the token-group view of x) and a tensor map that the host encodes.
+// A decoded weight tile serves 256 tokens and 16 MMAs.  Needs a tensor map
+// of x that the host encodes (x 16-byte aligned, K a multiple of 128).
 constexpr int BR2 = 256;                 // weight rows per CTA
 constexpr int BT2 = 256;                 // tokens per CTA (MMA N)
 constexpr int XK2 = 64;                  // K per x stage
@@ -436,11 +436,11 @@ __global__ void __launch_bounds__(kThreads2, 1)
         const int sl = xs % NX2;
         if (xs >= NX2 && !wait_or_abort(&bars->xempty[sl], ((uint32_t)(xs / NX2) & 1u) ^ 1u, abort_)) break;
         mbar_arrive_expect_tx(&bars->xfull[sl], (uint32_t)kXStage2);
-        // element 0, token 0 of the group, chunk (K / 8), token group
+        // K = 64 xs .., tokens m0 .. (tokens past M arrive as zeros)
         asm volatile(
-            "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(
+            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
                 smem_u32(smem + oX2 + sl * kXStage2)),
-            "l"(&xmap), "r"(0), "r"(0), "r"(xs * (XK2 / 8)), "r"(m0 / 8), "r"(smem_u32(&bars->xfull[sl]))
+            "l"(&xmap), "r"(xs * XK2), "r"(m0), "r"(smem_u32(&bars->xfull[sl]))
             : "memory");
         ++issued;
       }
@@ -470,7 +470,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
         const uint32_t Xb = smem_u32(smem + oX2 + sl * kXStage2);
 #pragma unroll
         for (int kk = 0; kk < XK2 / 16; ++kk) {
-          const uint64_t bdesc = smem_desc(Xb + kk * 256, 128, 1024);
+          const uint64_t bdesc = smem_desc_sw128(Xb + kk * 32);
           const uint32_t acc = (g > 0 || h > 0 || kk > 0) ? 1u : 0u;
 #pragma unroll
           for (int half = 0; half < NH; ++half)
@@ -528,10 +528,8 @@ __global__ void __launch_bounds__(kThreads2, 1)
 
 TQ_STATUS_ACCESSOR(read_status_prefill)
 
-// x [M][K] fp16 as a 4-D tensor (element, token within a group of 8, 8-element
-// chunk, token group) whose box (8, 8, 8, 32) lands in shared memory in the
-// no-swizzle K-major core-matrix layout.  false when the driver's encoder is
-// unavailable or refuses.
+// x [M][K] fp16 as a 2-D tensor, box 64 (K) x 256 (tokens), 128-byte
+// swizzling.  false when the driver's encoder is unavailable or refuses.
 static bool encode_x_map(const void *x, int M, int K, CUtensorMap *out) {
   static PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
     void *fn = nullptr;
@@ -542,19 +540,19 @@ static bool encode_x_map(const void *x, int M, int K, CUtensorMap *out) {
     return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }();
   if (!encode) return false;
-  cuuint64_t dims[4] = {8, 8, (cuuint64_t)(K / 8), (cuuint64_t)(M / 8)};
-  cuuint64_t strides[3] = {(cuuint64_t)K * 2, 16, (cuuint64_t)K * 16};
-  cuuint32_t box[4] = {8, 8, (cuuint32_t)(pf::XK2 / 8), (cuuint32_t)(pf::BT2 / 8)};
-  cuuint32_t estr[4] = {1, 1, 1, 1};
-  return encode(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x), dims, strides, box, estr,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)M};
+  cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+  cuuint32_t box[2] = {(cuuint32_t)pf::XK2, (cuuint32_t)pf::BT2};
+  cuuint32_t estr[2] = {1, 1};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(x), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
   cudaError_t e;
   CUtensorMap xmap;
-  if (M % 8 == 0 && encode_x_map(P.x, M, P.K, &xmap)) {
+  if (encode_x_map(P.x, M, P.K, &xmap)) {
     // 128-row tiles when 256-row tiles would leave more than half of the SMs idle
     const int mt = (M + pf::BT2 - 1) / pf::BT2;
     const bool narrow = (int64_t)mt * ((P.N + pf::BR2 - 1) / pf::BR2) * 2 <= 152;

@@ -189,6 +189,21 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
   return d;
 }
 
+// Shared-memory matrix descriptor of a K-major tile in the 128-byte swizzle
+// layout that a tensor copy with 128-byte swizzling writes: rows of 128
+// bytes (64 fp16 along K), 8-row groups 1024 bytes apart, the tile
+// 1024-byte aligned.  A K step inside the 128-byte row advances saddr by the
+// step's bytes.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1 << 16;              // leading-byte offset: unused within one 128-byte row
+  d |= (uint64_t)(1024 >> 4) << 32;    // 8-row groups
+  d |= (uint64_t)1 << 46;              // descriptor version field of the sm_100 family
+  d |= (uint64_t)2 << 61;              // 128-byte swizzling
+  return d;
+}
+
 // Instruction descriptor of kind::f16: fp16 A and B, fp32 accumulator,
 // both K-major, shape M x N.
 __host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {

@@ -1,8 +1,8 @@
 """GPU parity of the prefill tile path (M > 16 tokens: weight tiles
 dequantized to fp16 and multiplied on the tensor cores) against the fp64 CPU
-oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element.  Token counts that are
-multiples of 8 take the kernel fed by tensor copies of x, the others the
-per-thread-copy kernel; both appear below.  The full-size case
+oracle, |y - y_ref| <= 2e-3 * sum_k |W x| per element.  Every token count
+takes the kernel fed by tensor copies of x (ragged counts included).  The
+full-size case
 is the Qwen3-8B prefill shape (M = 2048 tokens) checked on sampled rows."""
 import numpy as np
 import pytest
