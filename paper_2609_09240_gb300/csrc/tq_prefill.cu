@@ -358,10 +358,13 @@ constexpr int BT2 = 256;                 // tokens per CTA (MMA N)
 constexpr int XK2 = 64;                  // K per x stage
 constexpr int kXStage2 = BT2 * XK2 * 2;  // 32 KiB
 constexpr int kWTile2 = BR2 * BK * 2;    // 64 KiB
-constexpr int NW2 = 2, NX2 = 3;
+constexpr int kPRow2 = 48;                 // plane-1 window per row: the 16-byte units covering a group
+constexpr int kPSlot2 = BR2 * kPRow2;      // 12 KiB
+constexpr int NW2 = 2, NX2 = 2, NP2 = 2;
 constexpr int oW2 = 0;
 constexpr int oX2 = NW2 * kWTile2;
-constexpr int oSel2 = oX2 + NX2 * kXStage2;
+constexpr int oP2 = oX2 + NX2 * kXStage2;
+constexpr int oSel2 = oP2 + NP2 * kPSlot2;
 constexpr int oBar2 = oSel2 + 256 * 8;
 constexpr int kSmem2 = oBar2 + 256;
 static_assert(kSmem2 <= 232448, "prefill2 shared memory");
@@ -370,7 +373,7 @@ constexpr int kThreads2 = 10 * 32;
 constexpr uint32_t kTmemCols2 = 512;
 
 struct Bars2 {
-  uint64_t xfull[NX2], xempty[NX2], wfull[NW2], wempty[NW2], done;
+  uint64_t xfull[NX2], xempty[NX2], wfull[NW2], wempty[NW2], pfull[NP2], pempty[NP2], done;
   uint32_t tmem_slot;
   int32_t abort_;
 };
@@ -378,7 +381,8 @@ static_assert(sizeof(Bars2) <= 256, "prefill2 barriers");
 
 template <bool F32, int NH>
 __global__ void __launch_bounds__(kThreads2, 1)
-    prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap, int M) {
+    prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap,
+                    const __grid_constant__ CUtensorMap pmap, int M) {
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.x * BT2, n0 = blockIdx.y * (NH * 128);
@@ -396,6 +400,10 @@ __global__ void __launch_bounds__(kThreads2, 1)
       mbar_init(&bars->wfull[i], NH * 128);
       mbar_init(&bars->wempty[i], 1);
     }
+    for (int i = 0; i < NP2; ++i) {
+      mbar_init(&bars->pfull[i], 1);          // the producer's expect-tx arrival
+      mbar_init(&bars->pempty[i], NH * 4);    // one arrival per decoder warp
+    }
     mbar_init(&bars->done, 1);
     bars->abort_ = 0;
     mbar_fence_init();
@@ -408,16 +416,80 @@ __global__ void __launch_bounds__(kThreads2, 1)
 
   if (warp < NH * 4) {
     // ======================================================= weight decode
+    // Thread r = row n0 + r.  The group's packed bytes come from the plane-1
+    // window ring (one tensor copy per group: 48 bytes of each row, from the
+    // 16-byte unit that holds the group's first byte); s1 / off (8 groups
+    // per load where rows allow), salience and the plane-2 record are
+    // loaded by the thread one group ahead.
     const int r = tid;
-    RowWalker rwk(P, n0 + r);
+    const int n = n0 + r;
+    const bool valid = n < N;
+    const int W = sal_words_of(P.K);
+    const uint32_t *salrow = P.sal + (int64_t)(valid ? n : 0) * W;
+    int64_t j = (valid && P.nnz > 0) ? P.rowptr[n] : 0;
+    uint32_t salw = (valid && P.nnz > 0) ? __ldg(salrow) : 0u;
+    const bool vec8 = (G % 8) == 0 && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+    const unsigned short *s1h = reinterpret_cast<const unsigned short *>(P.s1) + (int64_t)(valid ? n : 0) * G;
+    const unsigned short *ofh = reinterpret_cast<const unsigned short *>(P.off) + (int64_t)(valid ? n : 0) * G;
+    uint4 s1v = make_uint4(0u, 0u, 0u, 0u), ofv = make_uint4(0u, 0u, 0u, 0u);
+    // everything of group g but its plane-1 bytes
+    auto fetch = [&](int g, RowGroup &nx) {
+      if (vec8) {
+        if ((g & 7) == 0 && valid) {
+          s1v = __ldg(reinterpret_cast<const uint4 *>(s1h + g));
+          ofv = __ldg(reinterpret_cast<const uint4 *>(ofh + g));
+        }
+        const int k = g & 7;
+        const uint32_t ws1 = k < 2 ? s1v.x : k < 4 ? s1v.y : k < 6 ? s1v.z : s1v.w;
+        const uint32_t wof = k < 2 ? ofv.x : k < 4 ? ofv.y : k < 6 ? ofv.z : ofv.w;
+        nx.s1 = (unsigned short)((k & 1) ? ws1 >> 16 : ws1);
+        nx.of = (unsigned short)((k & 1) ? wof >> 16 : wof);
+      } else {
+        nx.s1 = valid ? __ldg(s1h + g) : (unsigned short)0;
+        nx.of = valid ? __ldg(ofh + g) : (unsigned short)0;
+      }
+      if ((g & 31) == 0 && g > 0 && valid && P.nnz > 0) salw = __ldg(salrow + (g >> 5));
+      nx.salient = (salw >> (g & 31)) & 1u;
+      nx.s2 = 0;
+      nx.rodd = false;
+#pragma unroll
+      for (int i = 0; i < 7; ++i) nx.q8[i] = 0x79797979u;
+      if (nx.salient) {
+        const int64_t jj = j < P.nnz ? j : P.nnz - 1;
+        const int64_t off0 = jj * kGroupBytes;
+        nx.rodd = (off0 & 3) != 0;  // plane 2 is 16-byte aligned: records start 0 or 2 bytes into a word
+        const uint32_t *rs = reinterpret_cast<const uint32_t *>(P.plane2 + off0 - (nx.rodd ? 2 : 0));
+#pragma unroll
+        for (int i = 0; i < 6; ++i) nx.q8[i] = __ldg(rs + i);
+        nx.q8[6] = nx.rodd ? __ldg(rs + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(rs + 6));
+        nx.s2 = __ldg(reinterpret_cast<const unsigned short *>(P.s2) + jj);
+        ++j;
+      }
+    };
     RowGroup nx;
-    rwk.fetch(0, nx);
+    fetch(0, nx);
     for (int g = 0; g < G; ++g) {
-      const int s = g % NW2;
+      const int s = g % NW2, ps = g % NP2;
       if (g >= NW2 && !__all_sync(0xffffffffu, wait_or_abort(&bars->wempty[s], ((uint32_t)(g / NW2) & 1u) ^ 1u, abort_)))
         break;
-      const RowGroup cur = nx;
-      if (g + 1 < G) rwk.fetch(g + 1, nx);
+      if (!__all_sync(0xffffffffu, wait_or_abort(&bars->pfull[ps], (uint32_t)(g / NP2) & 1u, abort_))) break;
+      RowGroup cur = nx;
+      {
+        // the row's 7 words of group g: the window's words from (26 g mod 16) / 4 on
+        const uint4 *pw = reinterpret_cast<const uint4 *>(smem + oP2 + ps * kPSlot2 + r * kPRow2);
+        const uint4 a0 = pw[0], a1 = pw[1], a2 = pw[2];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->pempty[ps]);
+        const uint32_t w[12] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w, a2.x, a2.y, a2.z, a2.w};
+        const int q = ((kGroupBytes * g) & 15) >> 2;
+        uint32_t t[10];
+#pragma unroll
+        for (int i = 0; i < 10; ++i) t[i] = (q & 2) ? w[i + 2] : w[i];
+#pragma unroll
+        for (int i = 0; i < 7; ++i) cur.r8[i] = (q & 1) ? t[i + 1] : t[i];
+        cur.odd = g & 1;  // the group starts 2 bytes into its first word
+      }
+      if (g + 1 < G) fetch(g + 1, nx);
       uint32_t wv[64];
       decode_row_group(cur, sel, wv);
       unsigned char *Wt = smem + oW2 + s * kWTile2;
@@ -429,7 +501,24 @@ __global__ void __launch_bounds__(kThreads2, 1)
       mbar_arrive(&bars->wfull[s]);
     }
   } else if (warp == kWarpProd2) {
-    // ============================================================ x tiles
+    // ===================================== x tiles (lane 0), plane-1 windows (lane 1)
+    if (lane == 1) {
+      uint32_t issued = 0;
+      for (int g = 0; g < G; ++g) {
+        const int sl = g % NP2;
+        if (g >= NP2 && !wait_or_abort(&bars->pempty[sl], ((uint32_t)(g / NP2) & 1u) ^ 1u, abort_)) break;
+        mbar_arrive_expect_tx(&bars->pfull[sl], (uint32_t)(NH * 128 * kPRow2));
+        // bytes from the 16-byte unit holding the group's first byte; rows n0 ..
+        asm volatile(
+            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+                smem_u32(smem + oP2 + sl * kPSlot2)),
+            "l"(&pmap), "r"((kGroupBytes * g) & ~15), "r"(n0), "r"(smem_u32(&bars->pfull[sl]))
+            : "memory");
+        ++issued;
+      }
+      for (uint32_t k = (issued > (uint32_t)NP2 ? issued - NP2 : 0); k < issued; ++k)
+        mbar_wait(&bars->pfull[k % NP2], (k / NP2) & 1u);
+    }
     if (lane == 0) {
       uint32_t issued = 0;
       for (int xs = 0; xs < 2 * G; ++xs) {
@@ -549,19 +638,40 @@ static bool encode_x_map(const void *x, int M, int K, CUtensorMap *out) {
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// plane 1 [N][row bytes] as a 2-D byte tensor, box 48 bytes x `rows` rows.
+static bool encode_p_map(const void *plane1, int N, int K, int rows, CUtensorMap *out) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      fn = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }();
+  if (!encode) return false;
+  const int64_t rb = row_bytes_of(K);
+  cuuint64_t dims[2] = {(cuuint64_t)rb, (cuuint64_t)N};
+  cuuint64_t strides[1] = {(cuuint64_t)rb};
+  cuuint32_t box[2] = {(cuuint32_t)pf::kPRow2, (cuuint32_t)rows};
+  cuuint32_t estr[2] = {1, 1};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(plane1), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
   cudaError_t e;
-  CUtensorMap xmap;
-  if (encode_x_map(P.x, M, P.K, &xmap)) {
+  CUtensorMap xmap, pmap;
+  const int mt = (M + pf::BT2 - 1) / pf::BT2;
+  const bool narrow = (int64_t)mt * ((P.N + pf::BR2 - 1) / pf::BR2) * 2 <= 152;
+  if (encode_x_map(P.x, M, P.K, &xmap) && encode_p_map(P.plane1, P.N, P.K, narrow ? 128 : 256, &pmap)) {
     // 128-row tiles when 256-row tiles would leave more than half of the SMs idle
-    const int mt = (M + pf::BT2 - 1) / pf::BT2;
-    const bool narrow = (int64_t)mt * ((P.N + pf::BR2 - 1) / pf::BR2) * 2 <= 152;
     const dim3 grid(mt, narrow ? (P.N + 127) / 128 : (P.N + pf::BR2 - 1) / pf::BR2);
     auto kern = narrow ? (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>)
                        : (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem2);
     if (e != cudaSuccess) return e;
-    kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, M);
+    kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, pmap, M);
     return cudaGetLastError();
   }
   const dim3 grid((M + pf::BM - 1) / pf::BM, (P.N + pf::BN - 1) / pf::BN);
