@@ -201,6 +201,64 @@ __device__ __forceinline__ void decode_row_group(const RowGroup &cur, const uint
   }
 }
 
+// 35 fp16x2 words from byte pairs P0 .. P0 + 6 of a 26-byte run (word i =
+// trits 10 P0 + 2i, + 1), as decode_weights does for all 13 pairs.
+template <int P0>
+__device__ __forceinline__ void decode_pairs7(const uint32_t *rw, uint32_t v01, uint32_t v22, const uint64_t *sel,
+                                              uint32_t *out) {
+#pragma unroll
+  for (int q = 0; q < 7; ++q) {
+    const int p = P0 + q;
+    const int ba = 2 * p, bb = 2 * p + 1;
+    const uint32_t va = (rw[ba >> 2] >> (8 * (ba & 3))) & 0xffu;
+    const uint32_t vb = (rw[bb >> 2] >> (8 * (bb & 3))) & 0xffu;
+    const uint64_t ta = sel[va], tb = sel[vb];
+    const uint32_t ta_lo = (uint32_t)ta, ta_hi = (uint32_t)(ta >> 32);
+    const uint32_t tb_lo = (uint32_t)tb, tb_hi = (uint32_t)(tb >> 32);
+    out[5 * q] = prmt(v01, v22, ta_lo);
+    out[5 * q + 1] = prmt(v01, v22, ta_lo >> 16);
+    out[5 * q + 2] = prmt(v01, v22, prmt(ta_hi, tb_lo, 0x0040u));
+    out[5 * q + 3] = prmt(v01, v22, tb_lo >> 8);
+    out[5 * q + 4] = prmt(v01, v22, prmt(tb_lo, tb_hi, 0x0043u));
+  }
+}
+
+// Half H of a group's 128 weights of one row (32 words, K = 64 H .. 64 H +
+// 63): s1 t1 + off, plus s2 t2 when any row of the warp is salient.  Half 0
+// decodes pairs 0..6 (trits 0..69, keeps words 0..31), half 1 pairs 6..12
+// (trits 60..129, keeps words 2..33).
+template <int H>
+__device__ __forceinline__ void decode_row_half(const RowGroup &cur, const uint64_t *sel, uint32_t *wv) {
+  constexpr int P0 = H ? 6 : 0, W0 = H ? 2 : 0;
+  const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
+  uint32_t rw[7];
+  realign(cur.r8, cur.odd, rw);
+  const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
+  const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+  const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
+  uint32_t w1[35];
+  decode_pairs7<P0>(rw, v01, v22, sel, w1);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) wv[i] = w1[W0 + i];
+  if (__any_sync(0xffffffffu, cur.salient)) {
+    const float s2 = __half2float(__ushort_as_half(cur.s2));
+    uint32_t rec[7];
+    realign(cur.q8, cur.rodd, rec);
+    const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
+    const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
+    const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
+    uint32_t w2[35];
+    decode_pairs7<P0>(rec, u01, u22, sel, w2);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const __half2 x = *reinterpret_cast<const __half2 *>(&wv[i]);
+      const __half2 y = *reinterpret_cast<const __half2 *>(&w2[W0 + i]);
+      const __half2 z = __hadd2(x, y);
+      wv[i] = *reinterpret_cast<const uint32_t *>(&z);
+    }
+  }
+}
+
 // Core-matrix offset of (row, K element e) in a tile of 8-row groups x 16
 // core matrices along K.
 __device__ __forceinline__ int cm_off(int row, int e) { return ((row >> 3) * 16 + (e >> 3)) * 128 + (row & 7) * 16; }
@@ -340,17 +398,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_const
 // ------------------------------------------------------------------------
 // prefill2_kernel: a 256-row x 256-token output tile per CTA, weights as the
 // MMA's M operand (two halves of 128 rows), tokens as N = 256.
-//  * warps 0..7 (thread r = weight row n0 + r): decode each group's 128
-//    weights of their row into a 2-slot ring of weight tiles (64 KiB, the
-//    no-swizzle K-major core-matrix layout, 16 core matrices along K);
-//  * warp 8 (one thread): the x tiles, 256 tokens x 64 K (32 KiB) per stage,
+//  * warps 0..15 (thread r + 256 h = half h of weight row n0 + r): decode
+//    each group's 64 weights of their half row into a 2-slot ring of weight
+//    tiles (64 KiB, the no-swizzle K-major core-matrix layout, 16 core
+//    matrices along K), from the group's plane-1 window (a tensor copy of
+//    48 bytes per row by warp 16's lane 1, 2-slot ring);
+//  * warp 16 (lane 0): the x tiles, 256 tokens x 64 K (32 KiB) per stage,
 //    one 2-D tensor copy each with 128-byte swizzling (the K-major layout
 //    the MMA reads through a swizzled descriptor), into a 3-slot ring, two
 //    stages per group;
-//  * warp 9 (one thread): per stage 8 MMAs (M = 128 rows, N = 256 tokens,
+//  * warp 17 (one thread): per stage 8 MMAs (M = 128 rows, N = 256 tokens,
 //    K = 16; rows 0..127 into tensor-memory columns 0..255, rows 128..255
 //    into 256..511);
-//  * at the end warps 0..7 read the accumulators and write y.
+//  * at the end warps 0..15 read the accumulators and write y.
 // A decoded weight tile serves 256 tokens and 16 MMAs.  Needs a tensor map
 // of x that the host encodes (x 16-byte aligned, K a multiple of 128).
 constexpr int BR2 = 256;                 // weight rows per CTA
@@ -368,8 +428,8 @@ constexpr int oSel2 = oP2 + NP2 * kPSlot2;
 constexpr int oBar2 = oSel2 + 256 * 8;
 constexpr int kSmem2 = oBar2 + 256;
 static_assert(kSmem2 <= 232448, "prefill2 shared memory");
-constexpr int kDecWarps2 = 8, kWarpProd2 = 8, kWarpMma2 = 9;
-constexpr int kThreads2 = 10 * 32;
+constexpr int kDecWarps2 = 16, kWarpProd2 = 16, kWarpMma2 = 17;
+constexpr int kThreads2 = 18 * 32;
 constexpr uint32_t kTmemCols2 = 512;
 
 struct Bars2 {
@@ -397,12 +457,12 @@ __global__ void __launch_bounds__(kThreads2, 1)
       mbar_init(&bars->xempty[i], 1);
     }
     for (int i = 0; i < NW2; ++i) {
-      mbar_init(&bars->wfull[i], NH * 128);
+      mbar_init(&bars->wfull[i], NH * 256);
       mbar_init(&bars->wempty[i], 1);
     }
     for (int i = 0; i < NP2; ++i) {
       mbar_init(&bars->pfull[i], 1);          // the producer's expect-tx arrival
-      mbar_init(&bars->pempty[i], NH * 4);    // one arrival per decoder warp
+      mbar_init(&bars->pempty[i], NH * 8);    // one arrival per decoder warp
     }
     mbar_init(&bars->done, 1);
     bars->abort_ = 0;
@@ -414,14 +474,14 @@ __global__ void __launch_bounds__(kThreads2, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_slot;
 
-  if (warp < NH * 4) {
+  if (warp < kDecWarps2 && (warp & 7) < NH * 4) {
     // ======================================================= weight decode
     // Thread r = row n0 + r.  The group's packed bytes come from the plane-1
     // window ring (one tensor copy per group: 48 bytes of each row, from the
     // 16-byte unit that holds the group's first byte); s1 / off (8 groups
     // per load where rows allow), salience and the plane-2 record are
     // loaded by the thread one group ahead.
-    const int r = tid;
+    const int r = tid & 255, hh = tid >> 8;  // half hh of row r (warp-uniform)
     const int n = n0 + r;
     const bool valid = n < N;
     const int W = sal_words_of(P.K);
@@ -478,8 +538,6 @@ __global__ void __launch_bounds__(kThreads2, 1)
         // the row's 7 words of group g: the window's words from (26 g mod 16) / 4 on
         const uint4 *pw = reinterpret_cast<const uint4 *>(smem + oP2 + ps * kPSlot2 + r * kPRow2);
         const uint4 a0 = pw[0], a1 = pw[1], a2 = pw[2];
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->pempty[ps]);
         const uint32_t w[12] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w, a2.x, a2.y, a2.z, a2.w};
         const int q = ((kGroupBytes * g) & 15) >> 2;
         uint32_t t[10];
@@ -490,15 +548,23 @@ __global__ void __launch_bounds__(kThreads2, 1)
         cur.odd = g & 1;  // the group starts 2 bytes into its first word
       }
       if (g + 1 < G) fetch(g + 1, nx);
-      uint32_t wv[64];
-      decode_row_group(cur, sel, wv);
+      uint32_t wv[32];
+      if (hh == 0)
+        decode_row_half<0>(cur, sel, wv);
+      else
+        decode_row_half<1>(cur, sel, wv);
       unsigned char *Wt = smem + oW2 + s * kWTile2;
 #pragma unroll
-      for (int kc = 0; kc < 16; ++kc)
-        *reinterpret_cast<uint4 *>(Wt + cm_off(r, kc * 8)) =
+      for (int kc = 0; kc < 8; ++kc)
+        *reinterpret_cast<uint4 *>(Wt + cm_off(r, (8 * hh + kc) * 8)) =
             make_uint4(wv[4 * kc], wv[4 * kc + 1], wv[4 * kc + 2], wv[4 * kc + 3]);
       fence_proxy_async_smem();  // the MMA reads these stores through the async proxy
       mbar_arrive(&bars->wfull[s]);
+      // the window is released once the stores that depend on its words have
+      // issued (releasing right after the loads would let the next tensor copy
+      // overwrite words a lane has not received yet)
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->pempty[ps]);
     }
   } else if (warp == kWarpProd2) {
     // ===================================== x tiles (lane 0), plane-1 windows (lane 1)
@@ -581,9 +647,11 @@ __global__ void __launch_bounds__(kThreads2, 1)
     if (ok) {
       // tensor-memory lanes 32 q..; two row halves (all tokens each), or for
       // 128-row tiles two token halves of the one accumulator
-      const int q = warp & 3, sel2 = warp >> 2;
-      const int half = NH == 2 ? sel2 : 0;
-      const int cb = NH == 2 ? 0 : sel2 * (BT2 / 2), ce = NH == 2 ? BT2 : cb + BT2 / 2;
+      // 16 warps: lane quarter q, then row half (two accumulators) and token quarter or half
+      const int q = warp & 3, sel2 = warp >> 2;  // 0..3
+      const int half = NH == 2 ? (sel2 & 1) : 0;
+      const int parts = NH == 2 ? 2 : 4, part = NH == 2 ? (sel2 >> 1) : sel2;
+      const int cb = part * (BT2 / parts), ce = cb + BT2 / parts;
       const int n = n0 + half * 128 + 32 * q + lane;
 #pragma unroll 1
       for (int c0 = cb; c0 < ce; c0 += 8) {
