@@ -7,18 +7,10 @@
 //   W[n][k] = s1[n,g] t1[n,k] + off[n,g] + sal[n,g] s2[j(n,g)] t2[n,k],  g = k / 128,
 // each W element rounded once to fp16 (x is fp16), fp32 accumulation.
 //
-// One CTA computes a 128-token x 256-row output tile.  K is walked one
-// 128-wide group per stage through a 2-slot shared-memory ring:
-//  * threads 0..255 (thread r = weight row n0 + r) copy their share of the
-//    stage's x tile (128 tokens x 128, fp16) with 16-byte asynchronous
-//    copies, then decode their row's 26 packed bytes (and, on a salient
-//    group, the plane-2 record) into 128 fp16 weights;
-//  * one thread issues the stage's 8 MMAs (M = 128 tokens, N = 256 rows,
-//    K = 16), A = the x tile, B = the weight tile, both in the no-swizzle
-//    K-major core-matrix layout (core matrix = 8 rows x 8 K elements =
-//    128 bytes; consecutive along K, 16 core matrices per 8-row group);
-//  * at the end every warp reads its quarter of the tensor-memory lanes and
-//    half of the 256 columns and writes y.
+// prefill2_kernel: a 256-row x 256-token output tile per CTA (or 128 rows
+// for narrow grids), weights as the MMA's M operand; x tiles and per-group
+// plane-1 windows arrive by tensor copies, 16 warps decode the weight tiles
+// into shared memory, one thread issues the MMAs (see its comment).
 // Weight decode: a byte's five digits d (trit + 1) select among the row's
 // three fp16 values off - s1, off, off + s1 held in two registers; a
 // 243-entry table gives, per digit, the PRMT selector nibbles of its value,
@@ -32,25 +24,7 @@
 namespace tq {
 namespace pf {
 
-constexpr int BM = 128;          // tokens per tile (MMA M)
-constexpr int BN = 256;          // weight rows per tile (MMA N)
-constexpr int BK = 128;          // K per stage (one group)
-constexpr int kDecThreads = 256;
-constexpr int kThreads = kDecThreads + 32;  // + the MMA warp
-constexpr int kATile = BM * BK * 2;         // 32 KiB
-constexpr int kBTile = BN * BK * 2;         // 64 KiB
-constexpr int kStage = kATile + kBTile;
-constexpr int NS = 2;
-constexpr int oSel = NS * kStage;           // 243 x 8-byte selector entries
-constexpr int oBar = oSel + 256 * 8;
-constexpr int kSmem = oBar + 128;
-constexpr uint32_t kTmemCols = 256;
-
-struct Bars {
-  uint64_t full[NS], empty[NS], done;
-  uint32_t tmem_slot;
-  int32_t abort_;
-};
+constexpr int BK = 128;          // K per group
 
 __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, volatile int32_t *abort_) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -86,27 +60,6 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t s) {
   return d;
 }
 
-// 64 fp16x2 words of a group's 128 weights from its 26 bytes (7 words, byte
-// 0 first) and the three values v01 = (v0, v1), v22 = (v2, v2).
-__device__ __forceinline__ void decode_weights(const uint32_t *rw, uint32_t v01, uint32_t v22, const uint64_t *sel,
-                                               uint32_t *out) {
-#pragma unroll
-  for (int p = 0; p < 13; ++p) {
-    const int ba = 2 * p, bb = 2 * p + 1;
-    const uint32_t va = (rw[ba >> 2] >> (8 * (ba & 3))) & 0xffu;
-    const uint32_t vb = (rw[bb >> 2] >> (8 * (bb & 3))) & 0xffu;
-    const uint64_t ta = sel[va], tb = sel[vb];
-    const uint32_t ta_lo = (uint32_t)ta, ta_hi = (uint32_t)(ta >> 32);
-    const uint32_t tb_lo = (uint32_t)tb, tb_hi = (uint32_t)(tb >> 32);
-    // weights 10p .. 10p + 9: (a0 a1) (a2 a3) (a4 b0) (b1 b2) (b3 b4)
-    out[5 * p] = prmt(v01, v22, ta_lo);
-    out[5 * p + 1] = prmt(v01, v22, ta_lo >> 16);
-    if (5 * p + 2 < 64) out[5 * p + 2] = prmt(v01, v22, prmt(ta_hi, tb_lo, 0x0040u));
-    if (5 * p + 3 < 64) out[5 * p + 3] = prmt(v01, v22, tb_lo >> 8);
-    if (5 * p + 4 < 64) out[5 * p + 4] = prmt(v01, v22, prmt(tb_lo, tb_hi, 0x0043u));
-  }
-}
-
 // One weight row's data for one group, loaded a group ahead of its decode:
 // the raw aligned words of its 26 bytes and of its plane-2 record, s1, off,
 // s2, and whether the group is salient.
@@ -116,89 +69,10 @@ struct RowGroup {
   bool odd, rodd, salient;
 };
 
-// Walks one weight row group by group (thread = row): fetch() issues the
-// loads of group g (nothing waits for them until the group is decoded).
-struct RowWalker {
-  const Problem *P;
-  const uint8_t *row;
-  const uint32_t *salrow;
-  int64_t j;      // record index of the row's next salient group
-  uint32_t salw;  // the row's current salience word
-  int G, n;
-  bool valid;
-  __device__ RowWalker(const Problem &p, int n_) : P(&p), n(n_) {
-    const int K = p.K, W = sal_words_of(K);
-    G = K / kGroup;
-    valid = n < p.N;
-    row = p.plane1 + (int64_t)(valid ? n : 0) * row_bytes_of(K);
-    salrow = p.sal + (int64_t)(valid ? n : 0) * W;
-    j = (valid && p.nnz > 0) ? p.rowptr[n] : 0;
-    salw = (valid && p.nnz > 0) ? __ldg(salrow) : 0u;
-  }
-  __device__ void fetch(int g, RowGroup &nx) {
-    // plane-1 rows are 16-byte aligned and groups are 26 bytes, so group g
-    // starts 0 or 2 bytes into a word; 7 aligned words cover it
-    nx.odd = g & 1;
-    const uint32_t *src = reinterpret_cast<const uint32_t *>(row + (int64_t)g * kGroupBytes - (nx.odd ? 2 : 0));
-#pragma unroll
-    for (int i = 0; i < 7; ++i) nx.r8[i] = valid ? __ldg(src + i) : 0x79797979u;  // 121: all-zero trits
-    const unsigned short *s1h = reinterpret_cast<const unsigned short *>(P->s1);
-    const unsigned short *ofh = reinterpret_cast<const unsigned short *>(P->off);
-    nx.s1 = valid ? __ldg(s1h + (int64_t)n * G + g) : (unsigned short)0;
-    nx.of = valid ? __ldg(ofh + (int64_t)n * G + g) : (unsigned short)0;
-    if ((g & 31) == 0 && g > 0 && valid && P->nnz > 0) salw = __ldg(salrow + (g >> 5));
-    nx.salient = (salw >> (g & 31)) & 1u;
-    nx.s2 = 0;
-    nx.rodd = false;
-#pragma unroll
-    for (int i = 0; i < 7; ++i) nx.q8[i] = 0x79797979u;
-    if (nx.salient) {
-      const int64_t jj = j < P->nnz ? j : P->nnz - 1;
-      const int64_t off0 = jj * kGroupBytes;
-      nx.rodd = (off0 & 3) != 0;  // plane 2 is 16-byte aligned: records start 0 or 2 bytes into a word
-      const uint32_t *rs = reinterpret_cast<const uint32_t *>(P->plane2 + off0 - (nx.rodd ? 2 : 0));
-#pragma unroll
-      for (int i = 0; i < 6; ++i) nx.q8[i] = __ldg(rs + i);
-      nx.q8[6] = nx.rodd ? __ldg(rs + 6) : (uint32_t)__ldg(reinterpret_cast<const uint16_t *>(rs + 6));
-      nx.s2 = __ldg(reinterpret_cast<const unsigned short *>(P->s2) + jj);
-      ++j;
-    }
-  }
-};
-
 // the 7 words of a 26-byte run, byte 0 first, from its raw aligned words
 __device__ __forceinline__ void realign(const uint32_t *r8, bool odd, uint32_t *rw) {
 #pragma unroll
   for (int i = 0; i < 7; ++i) rw[i] = odd ? __funnelshift_r(r8[i], i < 6 ? r8[i + 1] : 0u, 16) : r8[i];
-}
-
-// The group's 128 fp16 weights of one row (64 words): s1 t1 + off, plus
-// s2 t2 when any row of the warp is salient (other rows add zeros).
-__device__ __forceinline__ void decode_row_group(const RowGroup &cur, const uint64_t *sel, uint32_t *wv) {
-  const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
-  uint32_t rw[7];
-  realign(cur.r8, cur.odd, rw);
-  const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
-  const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-  const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
-  decode_weights(rw, v01, v22, sel, wv);
-  if (__any_sync(0xffffffffu, cur.salient)) {
-    const float s2 = __half2float(__ushort_as_half(cur.s2));
-    uint32_t rec[7];
-    realign(cur.q8, cur.rodd, rec);
-    const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
-    const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
-    const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
-    uint32_t w2[64];
-    decode_weights(rec, u01, u22, sel, w2);
-#pragma unroll
-    for (int i = 0; i < 64; ++i) {
-      const __half2 a = *reinterpret_cast<const __half2 *>(&wv[i]);
-      const __half2 b = *reinterpret_cast<const __half2 *>(&w2[i]);
-      const __half2 c = __hadd2(a, b);
-      wv[i] = *reinterpret_cast<const uint32_t *>(&c);
-    }
-  }
 }
 
 // 35 fp16x2 words from byte pairs P0 .. P0 + 6 of a 26-byte run (word i =
@@ -262,138 +136,6 @@ __device__ __forceinline__ void decode_row_half(const RowGroup &cur, const uint6
 // Core-matrix offset of (row, K element e) in a tile of 8-row groups x 16
 // core matrices along K.
 __device__ __forceinline__ int cm_off(int row, int e) { return ((row >> 3) * 16 + (e >> 3)) * 128 + (row & 7) * 16; }
-
-template <bool F32>
-__global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const __grid_constant__ Problem P, int M) {
-  extern __shared__ __align__(1024) unsigned char smem[];
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
-  const int K = P.K, N = P.N, G = K / kGroup;
-  uint64_t *sel = reinterpret_cast<uint64_t *>(smem + oSel);
-  Bars *bars = reinterpret_cast<Bars *>(smem + oBar);
-  volatile int32_t *abort_ = &bars->abort_;
-  for (int i = tid; i < 256; i += kThreads) sel[i] = sel_entry(i);
-  if (tid == 0) {
-    for (int s = 0; s < NS; ++s) {
-      mbar_init(&bars->full[s], 2 * kDecThreads);  // one async (x copies) + one decode arrival per thread
-      mbar_init(&bars->empty[s], 1);
-    }
-    mbar_init(&bars->done, 1);
-    bars->abort_ = 0;
-    mbar_fence_init();
-  }
-  if (warp == 0) tmem_alloc(&bars->tmem_slot, kTmemCols);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = bars->tmem_slot;
-
-  if (tid < kDecThreads) {
-    // ============================================= x copies + weight decode
-    const int r = tid;
-    RowWalker rwk(P, n0 + r);
-    RowGroup nx;
-    rwk.fetch(0, nx);
-    bool ok = true;
-    for (int g = 0; g < G && ok; ++g) {
-      const int s = g % NS;
-      const uint32_t ph = (uint32_t)(g / NS) & 1u;
-      if (g >= NS) ok = __all_sync(0xffffffffu, wait_or_abort(&bars->empty[s], ph ^ 1u, abort_));
-      if (!ok) break;
-      unsigned char *At = smem + s * kStage, *Bt = At + kATile;
-      // x tile: 128 tokens x 16 chunks of 16 bytes; thread tid takes 8
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const int i = tid + kDecThreads * k;
-        const int t = i >> 4, kc = i & 15;
-        const int m = m0 + t;
-        const __half *src = P.x + (int64_t)(m < M ? m : 0) * K + (int64_t)g * BK + kc * 8;
-        const uint32_t bytes = m < M ? 16u : 0u;  // tokens past M read as zeros
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(At + cm_off(t, kc * 8))),
-                     "l"(src), "r"(bytes)
-                     : "memory");
-      }
-      asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&bars->full[s])) : "memory");
-      const RowGroup cur = nx;
-      if (g + 1 < G) rwk.fetch(g + 1, nx);
-      uint32_t wv[64];
-      decode_row_group(cur, sel, wv);
-      // 16 core-matrix rows of 8 weights
-#pragma unroll
-      for (int kc = 0; kc < 16; ++kc)
-        *reinterpret_cast<uint4 *>(Bt + cm_off(r, kc * 8)) =
-            make_uint4(wv[4 * kc], wv[4 * kc + 1], wv[4 * kc + 2], wv[4 * kc + 3]);
-      fence_proxy_async_smem();  // the MMA reads these stores through the async proxy
-      mbar_arrive(&bars->full[s]);
-    }
-    asm volatile("cp.async.wait_all;" ::: "memory");
-  } else if (lane == 0) {
-    // ================================================================= MMA
-    const uint32_t idesc = idesc_f16_f32(BM, BN);
-    bool ok = true;
-    for (int g = 0; g < G && ok; ++g) {
-      const int s = g % NS;
-      if (!wait_or_abort(&bars->full[s], (uint32_t)(g / NS) & 1u, abort_)) {
-        ok = false;
-        break;
-      }
-      fence_proxy_async_smem();  // x tile written by asynchronous copies in the generic proxy
-      tc_fence_after();
-      const uint32_t A = smem_u32(smem + s * kStage), B = A + kATile;
-#pragma unroll
-      for (int kk = 0; kk < BK / 16; ++kk)
-        mma_smemA(tmem, smem_desc(A + kk * 256, 128, 2048), smem_desc(B + kk * 256, 128, 2048), idesc,
-                  (g > 0 || kk > 0) ? 1u : 0u);
-      mma_commit(&bars->empty[s]);
-    }
-    if (ok) mma_commit(&bars->done);
-  }
-
-  // ================================================================ epilogue
-  __syncwarp();
-  if (tid < kDecThreads) {
-    const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->done, 0u, abort_));
-    tc_fence_after();
-    if (ok) {
-      const int q = warp & 3, half = warp >> 2;  // tensor-memory lanes 32q.., columns 128 half..
-      const int m = m0 + 32 * q + lane;
-#pragma unroll 1
-      for (int c0 = 0; c0 < 128; c0 += 8) {
-        uint32_t v[8];
-        tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * 128 + c0), v);
-        tmem_wait_ld();
-        const int nb = n0 + half * 128 + c0;
-        if (m < M) {
-          if (F32) {
-            float *yr = static_cast<float *>(P.y) + (int64_t)m * N;
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-              if (nb + i < N) yr[nb + i] = __uint_as_float(v[i]);
-          } else {
-            __half *yr = static_cast<__half *>(P.y) + (int64_t)m * N;
-            if (nb + 8 <= N && (N & 7) == 0 && ((uintptr_t)P.y & 15u) == 0) {
-              uint4 o;
-              __half2 *oh = reinterpret_cast<__half2 *>(&o);
-#pragma unroll
-              for (int i = 0; i < 4; ++i) oh[i] = __floats2half2_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-              *reinterpret_cast<uint4 *>(yr + nb) = o;
-            } else {
-#pragma unroll
-              for (int i = 0; i < 8; ++i)
-                if (nb + i < N) yr[nb + i] = __float2half_rn(__uint_as_float(v[i]));
-            }
-          }
-        }
-      }
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) {
-    tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
-  }
-}
 
 // ------------------------------------------------------------------------
 // prefill2_kernel: a 256-row x 256-token output tile per CTA, weights as the
@@ -742,17 +484,8 @@ cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
     kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, pmap, M);
     return cudaGetLastError();
   }
-  const dim3 grid((M + pf::BM - 1) / pf::BM, (P.N + pf::BN - 1) / pf::BN);
-  if (f32) {
-    e = cudaFuncSetAttribute(pf::prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem);
-    if (e != cudaSuccess) return e;
-    pf::prefill_kernel<true><<<grid, pf::kThreads, pf::kSmem, s>>>(P, M);
-  } else {
-    e = cudaFuncSetAttribute(pf::prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem);
-    if (e != cudaSuccess) return e;
-    pf::prefill_kernel<false><<<grid, pf::kThreads, pf::kSmem, s>>>(P, M);
-  }
-  return cudaGetLastError();
+  // the driver's tensor-map encoder is unavailable or refused the shapes
+  return cudaErrorNotSupported;
 }
 
 }  // namespace tq
