@@ -170,10 +170,11 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
 /* Device workspace of the decode path (M <= TQ_MAX_SKINNY_M): the
  * activations of every call are first rearranged into the tensor-core
  * operand order of the packed weights (with the per-group correction terms),
- * and for M <= 8 the second plane's fp32 partial sums of every row are
- * staged there before the first plane is streamed, next to the 128-byte
- * descriptors through which the first plane, s1 and off are copied into
- * shared memory (written by the same call).  The caller provides this
+ * and the second plane's fp32 partial sums of every row are staged there
+ * before the first plane is streamed, next to the 128-byte descriptors
+ * through which the first plane, s1 and off are copied into shared memory
+ * (written by the same call).  A call with 8 < M <= 16 runs tokens 0..7 and
+ * then the rest over the same workspace, sized for 8 tokens.  The caller provides this
  * scratch memory (the library never allocates).  Bytes needed for one
  * projection of N rows, K inputs and M tokens; a call with M > 16 (the
  * prefill tile path) uses none and the function returns 256 for it; 0 if M,
@@ -184,9 +185,9 @@ TQ_API size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K);
  *   x: fp16 [M][K] row-major, 16-byte aligned; y: fp16 [M][N] (rounded to
  *   nearest even from the fp32 accumulator).  M >= 1.  M <= 16 runs the
  *   decode path straight from the packed bytes; M > 16 runs the prefill
- *   path, which dequantizes each 256-row x 128-column weight tile to fp16
- *   (w = s1 t1 + off + s2 t2, rounded once) and multiplies it by 128-token
- *   activation tiles on the tensor cores.
+ *   path, which dequantizes each 256-row (or 128-row) x 128-column weight
+ *   tile to fp16 (w = s1 t1 + off + s2 t2, rounded once) and multiplies it
+ *   by 256-token activation tiles on the tensor cores.
  *   workspace: device scratch of at least tq_workspace_bytes(M, N, K) bytes,
  *   256-byte aligned; its contents are overwritten; calls that share a
  *   workspace must not overlap in time.

@@ -20,11 +20,6 @@ cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t
 cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s);
-cudaError_t launch_gemv_tc(const BatchParams &p, cudaStream_t s);
-int tc_rows_per_tile();
-size_t tc_workspace_bytes(int M, int K);
-size_t tc_workspace_b_bytes(int M, int K);
-cudaError_t read_status_gemv_tc(uint32_t *out, bool clear);
 cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
@@ -88,14 +83,12 @@ Problem to_problem(const tq_weight *w, const uint16_t *x, void *y) {
 
 size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
 
-// Workspace bytes of one problem for a launch over M tokens (M <= 16).
+// Workspace bytes of one problem for a call over M tokens (M <= 16; more than
+// 8 tokens run as two passes of at most 8 over the same workspace).
 size_t problem_ws_bytes(int M, int N, int K) {
-  if (M <= 8) {
-    size_t b, cs, y2;
-    mma_workspace_parts(M, N, K, &b, &cs, &y2);
-    return pad256(b) + pad256(cs) + pad256(y2) + 512;  // + the tensor maps of plane 1, s1, off
-  }
-  return pad256(tc_workspace_bytes(16, K));
+  size_t b, cs, y2;
+  mma_workspace_parts(M <= 8 ? M : 8, N, K, &b, &cs, &y2);
+  return pad256(b) + pad256(cs) + pad256(y2) + 512;  // + the tensor maps of plane 1, s1, off
 }
 
 }  // namespace
@@ -111,12 +104,11 @@ size_t call_ws_bytes(int M, int N, int K) {
 
 namespace {
 
-// Places every problem's workspace and runs the decode path for bp.M tokens
-// (M <= 8: warp-level MMA kernels; 8 < M <= 16: the tensor-memory kernel).
-// Returns TQ_ERR_SHAPE when the workspace is too small.
-tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
-  const bool small = bp.M <= 8;
-  const int rows = small ? mma_rows_per_tile() : tc_rows_per_tile();
+// Places every problem's workspace and runs the decode path for bp.M <= 8
+// tokens (warp-level MMA kernels).  Returns TQ_ERR_SHAPE when the workspace
+// is too small.
+tq_status run_pass(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
+  const int rows = mma_rows_per_tile();
   int tiles = 0;
   size_t off = 0;
   for (int i = 0; i < bp.count; ++i) {
@@ -125,22 +117,38 @@ tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStr
     tiles += (P.N + rows - 1) / rows;
     const size_t tot = problem_ws_bytes(bp.M, P.N, P.K);
     if (off + tot > ws_bytes) return TQ_ERR_SHAPE;
-    if (small) {
-      size_t b, cs, y2;
-      mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
-      P.wsB = ws + off;
-      P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
-      P.y2_off = (int32_t)(pad256(b) + pad256(cs));
-      P.map_off = (int32_t)(pad256(b) + pad256(cs) + pad256(y2));
-    } else {
-      P.wsB = ws + off;
-      P.wsCS = reinterpret_cast<float *>(ws + off + tc_workspace_b_bytes(16, P.K));
-      P.y2_off = P.map_off = 0;
-    }
+    size_t b, cs, y2;
+    mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
+    P.wsB = ws + off;
+    P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
+    P.y2_off = (int32_t)(pad256(b) + pad256(cs));
+    P.map_off = (int32_t)(pad256(b) + pad256(cs) + pad256(y2));
     off += tot;
   }
   bp.total_tiles = tiles;
-  return from_cuda(small ? launch_gemv_mma(bp, s) : launch_gemv_tc(bp, s));
+  return from_cuda(launch_gemv_mma(bp, s));
+}
+
+// The decode path for bp.M <= 16 tokens: 8 < M runs tokens 0..7 and then
+// 8..M-1 (x and y are token-major, so each pass reads and writes one
+// contiguous block of rows) over the same workspace, one pass after the other
+// on the stream.
+tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
+  if (bp.M <= 8) return run_pass(bp, ws, ws_bytes, s);
+  thread_local BatchParams hi;  // large: kept off the stack
+  hi = bp;
+  hi.M = bp.M - 8;
+  for (int i = 0; i < hi.count; ++i) {
+    Problem &P = hi.prob[i];
+    P.x += (int64_t)8 * P.K;
+    P.y = static_cast<unsigned char *>(P.y) + (int64_t)8 * P.N * (hi.out_f32 ? 4 : 2);
+  }
+  const int M = bp.M;
+  bp.M = 8;
+  const tq_status st = run_pass(bp, ws, ws_bytes, s);
+  bp.M = M;
+  if (st != TQ_OK) return st;
+  return run_pass(hi, ws, ws_bytes, s);
 }
 
 tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
@@ -282,11 +290,10 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {
   if (!status_host) return TQ_ERR_NULL;
-  uint32_t a = 0, b = 0, c = 0;
-  if (read_status_gemv_tc(&a, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  uint32_t b = 0, c = 0;
   if (read_status_gemv_mma(&b, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
   if (read_status_prefill(&c, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
-  *status_host = a | b | c;
+  *status_host = b | c;
   return TQ_OK;
 }
 
