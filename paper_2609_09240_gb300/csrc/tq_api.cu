@@ -83,11 +83,12 @@ Problem to_problem(const tq_weight *w, const uint16_t *x, void *y) {
 
 size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
 
-// Workspace bytes of one problem for a call over M tokens (M <= 16; more than
-// 8 tokens run as two passes of at most 8 over the same workspace).
+// Workspace bytes of one problem for a pass over M <= 16 tokens.  (A call
+// whose more than 8 tokens have to run as two passes of at most 8 places the
+// smaller 8-token layout in the same space.)
 size_t problem_ws_bytes(int M, int N, int K) {
   size_t b, cs, y2;
-  mma_workspace_parts(M <= 8 ? M : 8, N, K, &b, &cs, &y2);
+  mma_workspace_parts(M, N, K, &b, &cs, &y2);
   return pad256(b) + pad256(cs) + pad256(y2) + 512;  // + the tensor maps of plane 1, s1, off
 }
 
@@ -104,9 +105,9 @@ size_t call_ws_bytes(int M, int N, int K) {
 
 namespace {
 
-// Places every problem's workspace and runs the decode path for bp.M <= 8
-// tokens (warp-level MMA kernels).  Returns TQ_ERR_SHAPE when the workspace
-// is too small.
+// Places every problem's workspace and runs the decode path for bp.M <= 16
+// tokens in one pass (warp-level MMA kernels).  Returns TQ_ERR_SHAPE when the
+// workspace is too small.
 tq_status run_pass(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
   const int rows = mma_rows_per_tile();
   int tiles = 0;
@@ -129,12 +130,16 @@ tq_status run_pass(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStre
   return from_cuda(launch_gemv_mma(bp, s));
 }
 
-// The decode path for bp.M <= 16 tokens: 8 < M runs tokens 0..7 and then
-// 8..M-1 (x and y are token-major, so each pass reads and writes one
-// contiguous block of rows) over the same workspace, one pass after the other
-// on the stream.
+// The decode path for bp.M <= 16 tokens.  One pass, unless more than 8
+// tokens meet a second plane without its index (the span kernels take 8
+// tokens at most): then tokens 0..7 and 8..M-1 run one after the other over
+// the same workspace (x and y are token-major, so each pass reads and writes
+// one contiguous block of rows).
 tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
-  if (bp.M <= 8) return run_pass(bp, ws, ws_bytes, s);
+  bool indexed = true;
+  for (int i = 0; i < bp.count; ++i)
+    if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx) indexed = false;
+  if (bp.M <= 8 || indexed) return run_pass(bp, ws, ws_bytes, s);
   thread_local BatchParams hi;  // large: kept off the stack
   hi = bp;
   hi.M = bp.M - 8;

@@ -1,4 +1,4 @@
-// tq_gemv_mma.cu - decode-path linear for M <= 8 tokens: packed bytes are
+// tq_gemv_mma.cu - decode-path linear for M <= 16 tokens: packed bytes are
 // streamed from HBM into shared memory by bulk copies, decoded in registers
 // and contracted on the tensor cores with warp-level m16n8k16 MMAs (fp16
 // operands, fp32 accumulators).
@@ -24,7 +24,9 @@
 // from gemv_mma_prep_kernel into the caller's workspace.
 //
 // Fragment layout.  In an m16n8k16 MMA, lane (g, c) (g = lane / 4,
-// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8.  Lane c
+// c = lane % 4) holds A's k-pairs c and c + 4 of rows g and g + 8; B's
+// column g is token g (with more than 8 tokens a second MMA on the same A
+// takes tokens 8 + g, and C/S come in one block per 8-token tile).  Lane c
 // of a row decodes the two words of the group's window (the aligned words
 // covering its 26 bytes) whose index is c mod 4, loaded straight from the
 // stage row in shared memory (the 32 lanes hit 32 different banks): 8 bytes,
@@ -70,7 +72,7 @@ constexpr int kChunks = 10;       // k16 chunks per group (160 K slots)
 constexpr int kCP = 5;            // chunk pairs
 constexpr int kBLane = 16;        // B bytes per (chunk pair, token, lane position)
 constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
-constexpr int kCSGroup = 64;             // C[8], S[8] floats per group
+constexpr int kCSGroup = 64;             // C[8], S[8] floats per group and 8-token tile
 constexpr int kWarpsP1 = 8, kWarpProd = 8;
 constexpr int kThreads = 9 * 32;
 constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
@@ -81,26 +83,30 @@ constexpr int kArena1 = (int)(kLutShared - kDynShared);   // below the table
 constexpr int kArena2 = kDynBytes - kArena1 - kLutBytes;  // above the table
 constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
 constexpr int kSOSlot = 2 * kRows * 16;                   // s1 then off, 16 B per row
-constexpr int kCSSlot = kStageG * kCSGroup;               // 512
+
 constexpr int kBarOff = 2 * kBytesSlot;                   // barriers in arena 1
 static_assert(kBarOff + 512 <= kArena1, "arena 1 overflow");
 
-__host__ __device__ constexpr int num_slots(int MB) { return MB <= 2 ? 4 : 3; }
+__host__ __device__ constexpr int num_slots(int MB) { return MB <= 2 ? 4 : MB <= 8 ? 3 : 2; }
 __host__ __device__ constexpr int b_stage_bytes(int MB) { return kStageG * kBTok * MB; }
+// C/S bytes per group: C[8], S[8] of tokens 0..7, then (more than 8 tokens)
+// the same for tokens 8..15
+__host__ __device__ constexpr int cs_group_bytes(int MB) { return MB > 8 ? 2 * kCSGroup : kCSGroup; }
 
 // Stage-slot layout for MB tokens: plane-1 slots 0, 1 in arena 1, the rest
 // in arena 2 followed by the B, s1/off and C/S slots.
 struct Layout {
-  int NS, BStage;
+  int NS, BStage, CSStage;
   int oBytes2, oB, oSO, oCS, used2;
   __host__ __device__ explicit Layout(int MB) {
     NS = num_slots(MB);
     BStage = b_stage_bytes(MB);
+    CSStage = kStageG * cs_group_bytes(MB);
     oBytes2 = 0;
     oB = oBytes2 + (NS - 2) * kBytesSlot;
     oSO = oB + NS * BStage;
     oCS = oSO + NS * kSOSlot;
-    used2 = oCS + NS * kCSSlot;
+    used2 = oCS + NS * CSStage;
   }
 };
 
@@ -401,11 +407,12 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
       *reinterpret_cast<uint4 *>(Bg + ((m * kCP + cp) * 4 + c) * kBLane) = q;
     }
   }
-  float *cs = P.wsCS + (int64_t)g * (kCSGroup / 4);
-  cs[m] = C;
-  cs[8 + m] = S;
+  // C, S of token m in its 8-token tile's block; unused tokens' entries zero
+  float *cs = P.wsCS + (int64_t)g * (cs_group_bytes(MB) / 4);
+  cs[(m >> 3) * 16 + (m & 7)] = C;
+  cs[(m >> 3) * 16 + 8 + (m & 7)] = S;
   if (m == 0)
-    for (int mm = MB; mm < 8; ++mm) cs[mm] = cs[8 + mm] = 0.f;
+    for (int mm = MB; mm < (MB > 8 ? 16 : 8); ++mm) cs[(mm >> 3) * 16 + (mm & 7)] = cs[(mm >> 3) * 16 + 8 + (mm & 7)] = 0.f;
 }
 
 // ------------------------------------------------------------ plane 2
@@ -974,7 +981,7 @@ __host__ __device__ __forceinline__ int c_parts(int K, int64_t nnz) {
   return (int)(q < 1 ? 1 : q > 32 ? 32 : q);
 }
 
-template <bool ONE>
+template <bool ONE, bool TWO>
 __global__ void __launch_bounds__(kCThreads, 1)
     gemv_mma_p2c_kernel(const __grid_constant__ CBase cb, const __grid_constant__ BatchParams bp, int32_t *counter) {
   extern __shared__ __align__(1024) unsigned char dync[];
@@ -1012,13 +1019,24 @@ __global__ void __launch_bounds__(kCThreads, 1)
     if (n <= 0) continue;
     // the group's B fragment (lanes of absent tokens repeat the last token) and C
     const unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB + min(g16, MB - 1) * kBTok + c * kBLane;
-    uint32_t b[20];
+    uint32_t b[20], b2[20];  // tokens g16 and (more than 8 tokens) 8 + g16 as MMA columns
 #pragma unroll
     for (int cp = 0; cp < kCP; ++cp) {
       const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg + cp * 4 * kBLane));
       b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
     }
-    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (kCSGroup / 4) + (ONE ? 0 : 2 * c)));
+    const float *csg = P.wsCS + (int64_t)g * (cs_group_bytes(MB) / 4);
+    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(csg + (ONE ? 0 : 2 * c)));
+    float2 Cv2 = make_float2(0.f, 0.f);
+    if (TWO) {
+      const unsigned char *Bg2 = P.wsB + (int64_t)g * kBTok * MB + min(8 + g16, MB - 1) * kBTok + c * kBLane;
+#pragma unroll
+      for (int cp = 0; cp < kCP; ++cp) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg2 + cp * 4 * kBLane));
+        b2[4 * cp] = v.x, b2[4 * cp + 1] = v.y, b2[4 * cp + 2] = v.z, b2[4 * cp + 3] = v.w;
+      }
+      Cv2 = __ldg(reinterpret_cast<const float2 *>(csg + 16 + 2 * c));
+    }
     // lane c's window words jw and jw + 4 are slot words 2 jw, 2 jw + 1; the row is the second
     // word of the lane with jw = 3, s2 a half of the first word of jw = 0 (record at byte 2)
     // or of the second word of jw = 2 (record at byte 0)
@@ -1049,8 +1067,9 @@ __global__ void __launch_bounds__(kCThreads, 1)
           uint32_t aL[20], aH[20];
           decode_words(r0.x, r0.y, tag, aL);
           decode_words(r1.x, r1.y, tag, aH);
-          float d[4];
+          float d[4], d2[4] = {0.f, 0.f, 0.f, 0.f};
           group_mma(aL, aH, b, d);
+          if (TWO) group_mma(aL, aH, b2, d2);
           const uint32_t sw0 = __shfl_sync(0xffffffffu, odd ? r0.x : r0.y, c_s2);
           const uint32_t sw1 = __shfl_sync(0xffffffffu, odd ? r1.x : r1.y, c_s2);
           const float s2v0 = odd ? half_of<false>(sw0) : half_of<true>(sw0);
@@ -1074,6 +1093,8 @@ __global__ void __launch_bounds__(kCThreads, 1)
               for (int ii = 0; ii < 2; ++ii) {
                 const int m = 2 * c + ii;
                 if (m < MB) atomicAdd(&y2[(int64_t)nr * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
+                if (TWO && 8 + m < MB)
+                  atomicAdd(&y2[(int64_t)nr * MB + 8 + m], s2v[h] * (d2[2 * h + ii] - (ii ? Cv2.y : Cv2.x)));
               }
             }
           }
@@ -1084,7 +1105,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
 }
 
 // ------------------------------------------------------------------ main
-template <bool F32, bool ONE>
+template <bool F32, bool ONE, bool TWO>
 __global__ void __launch_bounds__(kThreads, 1)
     gemv_mma_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
   extern __shared__ __align__(1024) unsigned char dyn[];
@@ -1129,8 +1150,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int g = lane >> 2, c = lane & 3;
       const int R0 = mt * 16 + g, R1 = R0 + 8;
       const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
-      uint32_t b[20];
+      uint32_t b[20], b2[20];  // tokens g, and (more than 8 tokens) 8 + g, as MMA columns
       float y[4] = {0.f, 0.f, 0.f, 0.f};  // (R0, 2c), (R0, 2c+1), (R1, 2c), (R1, 2c+1)
+      float y2t[4] = {0.f, 0.f, 0.f, 0.f};  // the same for tokens 8 + 2c, 8 + 2c + 1
+      constexpr int CSF = (TWO ? 2 : 1) * kCSGroup / 4;  // C/S floats per group
       uint32_t buf = 0, phase = 0;
       for (Walk w(&bp, t_begin, t_end); w.valid(); w.next()) {
         // the stage's rows, s1 / off, B and C / S are in slot buf
@@ -1140,7 +1163,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // this lane's B words (lanes of absent tokens load the last token's:
         // their output columns are never written)
         const unsigned char *Bl = Bst + min(g, MB - 1) * kBTok + c * kBLane;
-        const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * kCSSlot);
+        const unsigned char *Bl2 = Bst + min(8 + g, MB - 1) * kBTok + c * kBLane;
+        const float *CSst = reinterpret_cast<const float *>(ar2 + L.oCS + buf * L.CSStage);
         const unsigned char *SO = ar2 + L.oSO + buf * kSOSlot;
         const uint4 s1a = *reinterpret_cast<const uint4 *>(SO + R0 * 16);
         const uint4 s1b = *reinterpret_cast<const uint4 *>(SO + R1 * 16);
@@ -1150,11 +1174,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ofw[2][4] = {{ofa.x, ofa.y, ofa.z, ofa.w}, {ofb.x, ofb.y, ofb.z, ofb.w}};
         const int gs = w.gs;
         // s1 / off / C / S of group GL applied to its accumulators d
-        auto epilogue = [&](auto glc, const float *d) {
+        auto epilogue = [&](auto glc, const float *d, const float *d2) {
           constexpr int GL = decltype(glc)::value;
           if (ONE) {
             // one token: only column 0 (lanes c = 0) is ever written
-            const float Cx = CSst[GL * 16 + 2 * c], Sx = CSst[GL * 16 + 8 + 2 * c];
+            const float Cx = CSst[GL * CSF + 2 * c], Sx = CSst[GL * CSF + 8 + 2 * c];
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
               const float s1 = half_of<(GL & 1) != 0>(s1w[h][GL >> 1]);
@@ -1163,8 +1187,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             return;
           }
-          const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 2 * c);
-          const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * 16 + 8 + 2 * c);
+          const float2 Cv = *reinterpret_cast<const float2 *>(CSst + GL * CSF + 2 * c);
+          const float2 Sv = *reinterpret_cast<const float2 *>(CSst + GL * CSF + 8 + 2 * c);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const float s1 = half_of<(GL & 1) != 0>(s1w[h][GL >> 1]);
@@ -1172,10 +1196,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             y[2 * h] = fmaf(s1, d[2 * h] - Cv.x, fmaf(of, Sv.x, y[2 * h]));
             y[2 * h + 1] = fmaf(s1, d[2 * h + 1] - Cv.y, fmaf(of, Sv.y, y[2 * h + 1]));
           }
+          if (TWO) {
+            // tokens 8 + 2c, 8 + 2c + 1: the second C/S block
+            const float2 Cw = *reinterpret_cast<const float2 *>(CSst + GL * CSF + 16 + 2 * c);
+            const float2 Sw = *reinterpret_cast<const float2 *>(CSst + GL * CSF + 24 + 2 * c);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const float s1 = half_of<(GL & 1) != 0>(s1w[h][GL >> 1]);
+              const float of = half_of<(GL & 1) != 0>(ofw[h][GL >> 1]);
+              y2t[2 * h] = fmaf(s1, d2[2 * h] - Cw.x, fmaf(of, Sw.x, y2t[2 * h]));
+              y2t[2 * h + 1] = fmaf(s1, d2[2 * h + 1] - Cw.y, fmaf(of, Sw.y, y2t[2 * h + 1]));
+            }
+          }
         };
         // Software pipeline over the stage's groups: the MMAs of group GL run
         // while group GL + 1 is decoded; GL's epilogue comes after that.
-        float dp[4] = {0.f, 0.f, 0.f, 0.f};
+        float dp[4] = {0.f, 0.f, 0.f, 0.f}, dp2[4] = {0.f, 0.f, 0.f, 0.f};
         // lane (g, c)'s window words of a group at shift k = win_start % 4:
         // stage-row words win_start + ((c - k) & 3) (+ 4) of rows R0, R1
         const unsigned char *rowp = bytes_buf(buf) + R0 * kStageBytes;
@@ -1201,12 +1237,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint4 v = bq[cp * 4];
                 b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
               }
-            }
-            float d[4];
-            group_mma(aL, aH, b, d);
-            if constexpr (GL >= 1) epilogue(std::integral_constant<int, GL - 1>{}, dp);
+              if (TWO) {
+                const uint4 *bq2 = reinterpret_cast<const uint4 *>(Bl2 + GL * kBTok * MB);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) dp[i] = d[i];
+                for (int cp = 0; cp < kCP; ++cp) {
+                  const uint4 v = bq2[cp * 4];
+                  b2[4 * cp] = v.x, b2[4 * cp + 1] = v.y, b2[4 * cp + 2] = v.z, b2[4 * cp + 3] = v.w;
+                }
+              }
+            }
+            float d[4], d2[4] = {0.f, 0.f, 0.f, 0.f};
+            group_mma(aL, aH, b, d);
+            if (TWO) group_mma(aL, aH, b2, d2);
+            if constexpr (GL >= 1) epilogue(std::integral_constant<int, GL - 1>{}, dp, dp2);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) dp[i] = d[i], dp2[i] = d2[i];
           }
         };
         auto stage = [&](auto fullc) {
@@ -1222,13 +1267,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (gs == kStageG) {
           // a full stage: straight-line code
           stage(std::true_type{});
-          epilogue(std::integral_constant<int, kStageG - 1>{}, dp);
+          epilogue(std::integral_constant<int, kStageG - 1>{}, dp, dp2);
         } else {
           stage(std::false_type{});
           // the epilogue of the stage's last group
           auto last = [&](auto glc) {
             constexpr int GL = decltype(glc)::value;
-            if (GL < gs && GL + 1 >= gs) epilogue(glc, dp);
+            if (GL < gs && GL + 1 >= gs) epilogue(glc, dp, dp2);
           };
           last(std::integral_constant<int, 0>{});
           last(std::integral_constant<int, 1>{});
@@ -1250,22 +1295,24 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int n = nb + (h ? R1 : R0);
               if (n < P.N) {
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                  const int m = 2 * c + i;
-                  if (m < M) {
-                    float v = y[2 * h + i];
-                    if (P.nnz > 0) v += P.y2()[(int64_t)n * MB + m];
-                    if (F32)
-                      static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
-                    else
-                      static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
+                for (int t2 = 0; t2 < (TWO ? 2 : 1); ++t2)
+#pragma unroll
+                  for (int i = 0; i < 2; ++i) {
+                    const int m = 8 * t2 + 2 * c + i;
+                    if (m < M) {
+                      float v = t2 ? y2t[2 * h + i] : y[2 * h + i];
+                      if (P.nnz > 0) v += P.y2()[(int64_t)n * MB + m];
+                      if (F32)
+                        static_cast<float *>(P.y)[(int64_t)m * P.N + n] = v;
+                      else
+                        static_cast<__half *>(P.y)[(int64_t)m * P.N + n] = __float2half_rn(v);
+                    }
                   }
-                }
               }
             }
           }
 #pragma unroll
-          for (int i = 0; i < 4; ++i) y[i] = 0.f;
+          for (int i = 0; i < 4; ++i) y[i] = 0.f, y2t[i] = 0.f;
         }
         if (++buf == (uint32_t)NS) buf = 0, phase ^= 1u;
       }
@@ -1283,7 +1330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int gs = w.gs, g0 = w.s * kStageG;
       const int n0 = (w.tile - P.tile_begin) * kRows, rows = min(kRows, P.N - n0);
       const uint32_t bb = (uint32_t)(gs * kBTok * MB);
-      const uint32_t cb = (uint32_t)(gs * kCSGroup);
+      const uint32_t cb = (uint32_t)(gs * cs_group_bytes(MB));
       int ok = 1;
       if (lane == 0) ok = wait_or_abort(&bars->empty[buf], phase ^ 1u, abort_) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
@@ -1306,7 +1353,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_arrive_expect_tx(full, bb + cb + (uint32_t)kBytesSlot + (so_map ? (uint32_t)kSOSlot : 0u));
         bulk_g2s(ar2 + L.oB + buf * L.BStage, P.wsB + (int64_t)g0 * kBTok * MB, bb, full);
-        bulk_g2s(ar2 + L.oCS + buf * kCSSlot, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * kCSGroup,
+        bulk_g2s(ar2 + L.oCS + buf * L.CSStage, reinterpret_cast<const unsigned char *>(P.wsCS) + (int64_t)g0 * cs_group_bytes(MB),
                  cb, full);
         // the stage's 208 bytes of the tile's 128 rows (rows past N and bytes
         // past the row's end arrive as zeros)
@@ -1374,11 +1421,11 @@ static int num_sms_mm() {
 
 int mma_rows_per_tile() { return mm::kRows; }
 
-// Workspace bytes of one problem for M <= 8 tokens: B fragments, C/S, y2.
+// Workspace bytes of one problem for M <= 16 tokens: B fragments, C/S, y2.
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2) {
   const size_t G = (size_t)(K / kGroup);
   *b = G * (size_t)mm::kBTok * (size_t)M;
-  *cs = G * (size_t)mm::kCSGroup;
+  *cs = G * (size_t)mm::cs_group_bytes(M);
   *y2 = (size_t)N * (size_t)M * 4;
 }
 
@@ -1487,7 +1534,7 @@ static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
 template <bool F32>
 static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   thread_local mm::Sched sc;
-  if (bp.M < 1 || bp.M > 8 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
+  if (bp.M < 1 || bp.M > 16 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
   const int ctas = min(num_sms_mm(), 256);
   int64_t total_cost = 0;
   for (int i = 0; i < bp.count; ++i) {
@@ -1563,8 +1610,12 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
   mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  // more than 8 tokens in one pass needs every second plane indexed (the
+  // other plane-2 kernels take 8 tokens at most)
+  if (bp.M > 8 && any2 && !all_idx) return cudaErrorInvalidValue;
   if (any2 && all_idx) {
-    auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true> : mm::gemv_mma_p2c_kernel<false>;
+    auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true, false>
+                          : (bp.M > 8 ? mm::gemv_mma_p2c_kernel<false, true> : mm::gemv_mma_p2c_kernel<false, false>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
     kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(cb, bp, counter);
@@ -1582,7 +1633,8 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  auto main_kern = bp.M == 1 ? mm::gemv_mma_kernel<F32, true> : mm::gemv_mma_kernel<F32, false>;
+  auto main_kern = bp.M == 1 ? mm::gemv_mma_kernel<F32, true, false>
+                             : (bp.M > 8 ? mm::gemv_mma_kernel<F32, false, true> : mm::gemv_mma_kernel<F32, false, false>);
   e = cudaFuncSetAttribute(main_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kDynBytes);
   if (e != cudaSuccess) return e;
   main_kern<<<ctas, mm::kThreads, mm::kDynBytes, s>>>(bp, sc);

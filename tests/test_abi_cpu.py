@@ -54,9 +54,11 @@ def test_host_side_argument_errors_without_gpu():
     mma = lambda M, N, K: pad(K // 128 * 320 * M) + pad(K // 128 * 64) + pad(N * M * 4) + 512
     assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) == 29184
     assert tq.tq_workspace_bytes(5, 100, 1024) == mma(5, 100, 1024)
-    # 8 < M <= 16: two passes of at most 8 tokens over one M = 8 workspace;
+    # 8 < M <= 16: C/S for two 8-token tiles (128 B per group);
     # M > 16: the prefill tile path needs no workspace (256 bytes are asked for)
-    assert tq.tq_workspace_bytes(16, 4096, 4096) == tq.tq_workspace_bytes(9, 4096, 4096) == mma(8, 4096, 4096)
+    mma16 = lambda M, N, K: pad(K // 128 * 320 * M) + pad(K // 128 * 128) + pad(N * M * 4) + 512
+    assert tq.tq_workspace_bytes(16, 4096, 4096) == mma16(16, 4096, 4096)
+    assert tq.tq_workspace_bytes(9, 300, 1152) == mma16(9, 300, 1152)
     assert tq.tq_workspace_bytes(40, 64, 4096) == 256
     assert tq.tq_workspace_bytes(1, 4096, 100) == 0
     # second-plane index: int32 colptr[G + 1] padded to 128 bytes, then 32-byte slots for
