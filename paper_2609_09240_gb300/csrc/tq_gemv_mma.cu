@@ -56,6 +56,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstring>
 #include <mutex>
 #include <type_traits>
 
@@ -301,11 +302,16 @@ struct Walk {
 // encoded for the same sizes then equals the host encoding byte for byte.
 constexpr int kMaxMapTemplates = 10;
 constexpr uint8_t kNoMap = 255;
+// The prep kernel reads the indices by its problem and the templates only at
+// constant offsets (a loop over the template slots): indexed or
+// address-taken reads of a parameter block this far into the parameter
+// space have returned wrong data.
 struct MapTemplates {
-  CUtensorMap t[kMaxMapTemplates];
-  uint8_t idx[TQ_MAX_BATCH];    // plane 1's template
+  uint8_t idx[TQ_MAX_BATCH];     // plane 1's template
   uint8_t idx_so[TQ_MAX_BATCH];  // s1's and off's template, or kNoMap (then asynchronous copies)
+  uint4 t[kMaxMapTemplates][8];  // the encoded templates (128 bytes each)
 };
+static_assert(sizeof(CUtensorMap) == 8 * sizeof(uint4), "tensor map size");
 // Workspace slot of a problem's tensor maps: plane 1, s1, off, then the
 // indexed second-plane kernel's unit counter.
 constexpr int kMapSlotBytes = 512;
@@ -333,10 +339,13 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
     // plane 1 as a 2-D byte tensor (row_bytes x N) for the main kernel's
     // stage copies: the template of its sizes with this problem's address
     auto build = [&](unsigned char *m, int t, const void *addr) {
-      const uint4 *src = reinterpret_cast<const uint4 *>(&mt.t[t]);
       uint4 *dst = reinterpret_cast<uint4 *>(m);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) dst[i] = src[i];
+      for (int k = 0; k < kMaxMapTemplates; ++k)
+        if (k == t) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) dst[i] = mt.t[k][i];
+        }
       asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(m), "l"(addr) : "memory");
     };
     unsigned char *m = static_cast<unsigned char *>(P.map());
@@ -354,14 +363,26 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   if (task >= G * MB) return;
   const int g = task / MB, m = task % MB;
   const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
+  // the group's 128 activations, all loads issued at once (x rows are
+  // 16-byte aligned and groups are 256 bytes)
+  uint4 xv[kGroup / 8];
+#pragma unroll
+  for (int i = 0; i < kGroup / 8; ++i) xv[i] = __ldg(reinterpret_cast<const uint4 *>(xr) + i);
+  // activation j of the group (j known at compile time once unrolled)
+  auto xg = [&](int j) -> float {
+    const uint4 &v = xv[j >> 3];
+    const uint32_t w = (j & 6) == 0 ? v.x : (j & 6) == 2 ? v.y : (j & 6) == 4 ? v.z : v.w;
+    return __half2float(__ushort_as_half((unsigned short)((j & 1) ? (w >> 16) : (w & 0xffffu))));
+  };
   // activation slots of the 26 bytes, rounded to fp16
   __half ya[26], yb[26], yc[26], yd[26], ye[26];
   float C = 0.f, S = 0.f;
+#pragma unroll
   for (int b = 0; b < 26; ++b) {
     const int ntr = b < 25 ? 5 : 3;
     float x[5];
 #pragma unroll
-    for (int i = 0; i < 5; ++i) x[i] = i < ntr ? __half2float(xr[5 * b + i]) : 0.f;
+    for (int i = 0; i < 5; ++i) x[i] = i < ntr ? xg(5 * b + i) : 0.f;
     const float z0 = x[0] - x[4] * (1.f / 81.f), z1 = x[1] - x[4] * (3.f / 81.f);
     const float z2 = x[2] - x[4] * (9.f / 81.f), z3 = x[3] - x[4] * (27.f / 81.f);
     ya[b] = __float2half_rn(z0);
@@ -1571,7 +1592,9 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
       while (k < nt && keys[k] != key) ++k;
       if (k == nt) {
         if (nt == mm::kMaxMapTemplates) return -1;  // launch_mm splits such batches
-        if (!map_template(kind, len, addr, N, &mt.t[nt])) return -2;
+        CUtensorMap enc;
+        if (!map_template(kind, len, addr, N, &enc)) return -2;
+        std::memcpy(&mt.t[nt][0], &enc, sizeof(enc));
         keys[nt++] = key;
       }
       return k;
