@@ -979,8 +979,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
 // takes the entries' rows and s2 from the quad's lanes that hold them;
 // s2 (D - C) per entry is added to y2 of the entry's row with a global
 // atomic (the prep kernel zeroes y2).
-constexpr int kCThreads = 768;
-constexpr int kCDepth = 4;                        // tiles in flight per warp (in registers)
+// threads per CTA: 1024 (64 registers) for up to 8 tokens, 768 for the
+// second token tile's extra fragment registers
+__host__ __device__ constexpr int c_threads(bool two) { return two ? 768 : 1024; }
+constexpr int kCDepth = 2;                        // tiles in flight per warp (in registers)
 constexpr int kCDynBytes2 = kArena1 + kLutBytes;  // the table of codes at its fixed address
 constexpr int kCUnitTiles = 32;                   // target tiles per unit
 
@@ -1003,7 +1005,7 @@ __host__ __device__ __forceinline__ int c_parts(int K, int64_t nnz) {
 }
 
 template <bool ONE, bool TWO>
-__global__ void __launch_bounds__(kCThreads, 1)
+__global__ void __launch_bounds__(c_threads(TWO), 1)
     gemv_mma_p2c_kernel(const __grid_constant__ CBase cb, const __grid_constant__ BatchParams bp, int32_t *counter) {
   extern __shared__ __align__(1024) unsigned char dync[];
   const int tid = threadIdx.x, lane = tid & 31;
@@ -1013,7 +1015,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
   }
   {
     uint32_t *lut = reinterpret_cast<uint32_t *>(dync + kArena1);
-    for (int i = tid; i < 256 * 32; i += kCThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+    for (int i = tid; i < 256 * 32; i += c_threads(TWO)) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
   }
   __syncthreads();
   const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, quad = lane & ~3;
@@ -1641,7 +1643,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
                           : (bp.M > 8 ? mm::gemv_mma_p2c_kernel<false, true> : mm::gemv_mma_p2c_kernel<false, false>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
-    kern<<<ctas, mm::kCThreads, mm::kCDynBytes2, s>>>(cb, bp, counter);
+    kern<<<ctas, mm::c_threads(bp.M > 8), mm::kCDynBytes2, s>>>(cb, bp, counter);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   } else if (any2 && gmax <= mm::kQMaxG) {
