@@ -63,7 +63,11 @@ def dist_env():
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
-    """nvidia-smi sampling of SM clocks and throttle reasons while running."""
+    """nvidia-smi sampling (every 20 ms) of SM clocks and throttle reasons.
+    Enter it before the warm-up, call ready() before the timed region, and
+    mark() its start and end: summary() then counts the samples read during
+    the timed region (and, when the region is shorter than the interval,
+    the samples of the whole sampled span, saying so)."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -72,13 +76,20 @@ class ClockSampler:
     def __init__(self, gpu_index):
         self.gpu = gpu_index
         self.proc = None
-        self.lines = []
+        self.lines = []  # (host time read, line)
+        self.marks = []
 
     def __enter__(self):
         try:
+            # a pseudo-terminal as stdout, so that nvidia-smi writes each sample
+            # as it takes it (into a pipe it would buffer them until exit)
+            import pty
+
+            self.master, slave = pty.openpty()
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "20"], stdout=slave, stderr=subprocess.DEVNULL, close_fds=True)
+            os.close(slave)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
         except Exception:
@@ -86,8 +97,28 @@ class ClockSampler:
         return self
 
     def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append(line.strip())
+        buf = b""
+        while True:
+            try:
+                chunk = os.read(self.master, 4096)
+            except OSError:
+                break
+            if not chunk:
+                break
+            buf += chunk
+            *full, buf = buf.split(b"\n")
+            now = time.perf_counter()
+            for ln in full:
+                self.lines.append((now, ln.decode(errors="replace").strip()))
+
+    def ready(self, timeout=5.0):
+        """Wait (bounded) until the first sample has arrived."""
+        t = time.perf_counter()
+        while self.proc and not self.lines and time.perf_counter() - t < timeout:
+            time.sleep(0.005)
+
+    def mark(self):
+        self.marks.append(time.perf_counter())
 
     def __exit__(self, *a):
         if self.proc:
@@ -96,11 +127,23 @@ class ClockSampler:
                 self.proc.wait(timeout=5)
             except Exception:
                 self.proc.kill()
+            self.t.join(timeout=2)
+            try:
+                os.close(self.master)
+            except OSError:
+                pass
 
     def summary(self):
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
+        lines = [ln for _, ln in self.lines]
+        window = "whole sampled span"
+        if len(self.marks) >= 2:
+            # a sample is read within a few ms of being taken
+            inside = [ln for t, ln in self.lines if self.marks[0] <= t <= self.marks[-1] + 0.01]
+            if inside:
+                lines, window = inside, "timed region"
+        for line in lines:
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 9:
                 continue
@@ -114,7 +157,8 @@ class ClockSampler:
                     reasons.add(n)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm),
+                "window": window}
 
 
 # ---------------------------------------------------------------- workload
@@ -262,17 +306,20 @@ def run_prefill(args, ws, rank, local):
         for pw, x, y, wsb in items:
             tq.tq_linear(x, pw, y=y, ws=wsb, stream=stream)
 
-    for _ in range(max(args.warmup, 3)):
-        step()
-    torch.cuda.synchronize()
-    steps = max(1, min(args.steps, 20))
+    steps = max(1, min(args.steps, 100))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(torch.cuda.current_device()) as clk:
+        clk.ready()
+        for _ in range(max(args.warmup, 3)):
+            step()
+        torch.cuda.synchronize()
+        clk.mark()
         e0.record(stream)
         for _ in range(steps):
             step()
         e1.record(stream)
         torch.cuda.synchronize()
+        clk.mark()
     ms = e0.elapsed_time(e1) / steps
     # context: dense fp16 matmul (cuBLAS) with a dense W of the same shapes
     dense = [torch.randn((pw.N, pw.K), device=dev, dtype=torch.float16) for pw, _, _, _ in items]
@@ -350,7 +397,7 @@ def run_reference(args, ws, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--M", type=int, default=1, help="tokens per step (1 = batch-1 decode)")
@@ -387,10 +434,6 @@ def main():
     def step():
         tq.tq_linear_batched(batch, stream)
 
-    for _ in range(max(args.warmup, 3)):
-        step()
-    torch.cuda.synchronize()
-
     def barrier():
         if pg:
             pg.barrier()
@@ -399,8 +442,12 @@ def main():
     # device-timed region: inputs resident in HBM (1.79 GB of packed weights
     # per step, larger than the 129 MB L2, so no flush is needed)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    barrier()
     with ClockSampler(torch.cuda.current_device()) as clk:
+        clk.ready()
+        for _ in range(max(args.warmup, 3)):
+            step()
+        barrier()
+        clk.mark()
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
@@ -410,6 +457,7 @@ def main():
             ev[i][1].record(stream)
         t1.record(stream)
         barrier()
+        clk.mark()
     total_ms = t0.elapsed_time(t1)
     launch_ms = [a.elapsed_time(b) for a, b in ev]
     if pg:
@@ -469,7 +517,7 @@ def main():
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
                      "traffic": ncu_traffic(),
                      "kernel": "decode step: activation prep + second plane (group-ordered index) + first plane "
-                               "(3 launches per step, timed together; the first-plane kernel is ~80 % of it)",
+                               "(3 launches per step, timed together; the first-plane kernel is ~88 % of it)",
                      "launch_ms_avg": launch_avg},
         "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},
