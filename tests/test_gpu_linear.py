@@ -107,11 +107,13 @@ def test_argument_errors(H):
     assert L.tq_linear(1, 64, 256, ctypes.byref(ws_), P(x), P(y), P(ws), n, s) == -2
 
 
-@pytest.mark.parametrize("M", [1, 3])
-def test_long_rows_second_plane(H, M):
-    """321 groups per row: more salience words than the span kernel of the
-    second plane stages, so the per-tile kernel runs it."""
-    run_case(H, 96, 321 * 128, 0.1, M, f32=True, proj=21)
+@pytest.mark.parametrize("index", [False, True])
+@pytest.mark.parametrize("M", [1, 3, 12])
+def test_long_rows_second_plane(H, M, index):
+    """321 groups per row: without the index, more salience words than the
+    span kernel of the second plane stages, so the per-tile kernel runs it
+    (12 tokens as two passes); with the index, the indexed kernel."""
+    run_case(H, 96, 321 * 128, 0.1, M, f32=True, proj=21, index=index)
 
 
 def test_batched_many_row_lengths(H):
@@ -166,20 +168,24 @@ def test_second_plane_without_index(H, N, K, frac, M):
     run_case(H, N, K, frac, M, f32=True, proj=40 + N, index=False)
 
 
+@pytest.mark.parametrize("index", [False, True])
 @pytest.mark.parametrize("M", [1, 4])
-def test_second_plane_scale2_two_byte_aligned(H, M):
+def test_second_plane_scale2_two_byte_aligned(H, M, index):
     """s2 is only required to be 2-byte aligned: a view starting 2 bytes
-    into an allocation takes the in-place read of the indexed kernel."""
+    into an allocation, read by the span kernel or copied into the
+    group-ordered index."""
     from paper_2609_09240_gb300 import tq
     N, K = 300, 4096
     w = wl.gen_weights(N, K, 0.2, config=6, proj=77)
     x = wl.gen_x(M, K, config=6, proj=77)
     y_ref, a_ref = H.oracle_ref(w, x)
-    pw = H.pack_on_gpu(w)
+    pw = H.pack_on_gpu(w, index=False)
     buf = torch.empty(pw.nnz + 1, dtype=torch.float16, device="cuda")
     buf[1:] = pw.scale2[:pw.nnz]
     pw.scale2 = buf[1:]
     assert pw.scale2.data_ptr() % 4 == 2
+    if index:
+        pw.p2index = tq.tq_plane2_index(N, K, pw.salience, pw.rowptr, pw.nnz, pw.plane2, pw.scale2)
     y = tq.tq_linear_f32out(H.dev(x), pw)
     H.device_status_ok()
     H.assert_close(y.cpu().numpy(), y_ref, a_ref)
