@@ -37,7 +37,7 @@ QWEN3_8B = [
 ]
 QWEN3_8B_LAYERS = 36
 
-TENSOR_T1, TENSOR_S1, TENSOR_OFF, TENSOR_SAL, TENSOR_T2, TENSOR_S2, TENSOR_X = range(7)
+TENSOR_T1, TENSOR_S1, TENSOR_OFF, TENSOR_SAL, TENSOR_T2, TENSOR_S2, TENSOR_X, TENSOR_DENSE = range(8)
 
 
 @dataclass(frozen=True)
@@ -137,6 +137,36 @@ def gen_weights(N: int, K: int, salient_fraction: float, config: int = 0, layer:
 def gen_x(M: int, K: int, config: int = 0, layer: int = 0, proj: int = 0, seed: int = 0) -> np.ndarray:
     """fp16 bits [M][K]."""
     return _fp16_bits(_rng(seed, config, layer, proj, TENSOR_X).normal(0.0, 1.0, (M, K)))
+
+
+def gen_dense_weights(N: int, K: int, config: int = 0, layer: int = 0, proj: int = 0, seed: int = 0) -> np.ndarray:
+    """fp16 bits [N][K] of a dense projection, the ternarizer's input.
+
+    Stand-in for a rotated Qwen3 projection (the paper ternarizes real
+    weights after an orthogonal rotation, which are not available): row n is
+    Normal(m_n, sd_n) with sd_n ~ lognormal(log 0.02, 0.25) and a small row
+    mean m_n ~ Normal(0, 1e-3); one weight in a thousand is an outlier, its
+    value multiplied by 8."""
+    rng = _rng(seed, config, layer, proj, TENSOR_DENSE)
+    sd = np.exp(rng.normal(np.log(0.02), 0.25, (N, 1)))
+    m = rng.normal(0.0, 1e-3, (N, 1))
+    w = m + sd * rng.standard_normal((N, K))
+    w[rng.random((N, K)) < 1e-3] *= 8.0
+    return _fp16_bits(w)
+
+
+def gen_dense_weights_torch(N: int, K: int, device, seed: int):
+    """Device-side draw of the gen_dense_weights distribution (torch's
+    generator, so values differ from gen_dense_weights): fp16 [N][K]."""
+    import torch
+
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    sd = torch.exp(torch.randn((N, 1), generator=g, device=device) * 0.25 + float(np.log(0.02)))
+    m = torch.randn((N, 1), generator=g, device=device) * 1e-3
+    w = torch.randn((N, K), generator=g, device=device) * sd + m
+    w = torch.where(torch.rand((N, K), generator=g, device=device) < 1e-3, w * 8.0, w)
+    return w.half()
 
 
 def half_bits_to_float(bits: np.ndarray) -> np.ndarray:
