@@ -84,6 +84,7 @@ typedef enum {
 #define TQ_DATA_BAD_BYTE 4u     /* a packed byte > 242                           */
 #define TQ_DATA_BAD_PAD 8u      /* a nonzero pad digit (tail byte) or pad byte   */
 #define TQ_DATA_BAD_ROWPTR 16u  /* rowptr disagrees with the salience map        */
+#define TQ_DATA_BAD_WEIGHT 32u  /* tq_ternarize: an input weight is inf or NaN    */
 
 /* A packed projection.  All pointers: device memory owned by the caller. */
 typedef struct {
@@ -166,6 +167,44 @@ TQ_API tq_status tq_pack(int32_t N, int32_t K, const int8_t *T1, const int8_t *T
 TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const uint8_t *plane2,
                     const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                     uint32_t *d_status, void *stream);
+
+/* E2M-ATQ ternarization (paper "Conversion Pipeline", subsection "E2M-ATQ")
+ * of a dense fp16 projection straight into the packed format above.
+ * Per block of one row and one group of 128 columns, with w its weights:
+ *   mu = mean(w), c = w - mu, Delta0 = 0.75 * mean(|c|),
+ *   T0 = +1 where c > Delta0, -1 where c < -Delta0, else 0,
+ *   alpha0 = sum(c * T0) / sum(T0^2) (0 for an empty support),
+ *   residual r = c - alpha0 * T0, energy E = sum(r^2).
+ * The nnz blocks of largest E (ties: lower block id n * G + g) are salient:
+ * their residual gets a second support T1 by the same rule (threshold
+ * 0.75 * mean(|r|)) and alpha1 = sum(r * T1) / sum(T1^2).  Then `sweeps`
+ * alternating refinements with the supports fixed: mu = mean(w - alpha0 T0
+ * - alpha1 T1), alpha0 = least squares of w - mu - alpha1 T1 on T0, alpha1 =
+ * least squares of w - mu - alpha0 T0 on T1.  Outputs: plane1 = T0, plane2
+ * = T1 of the salient blocks, offset = fp16(mu), scale1 = fp16(alpha0),
+ * scale2 = fp16(alpha1) (round to nearest even), sal and rowptr; together a
+ * complete tq_weight with nnz salient groups.
+ * Arithmetic: IEEE float32, no fused multiply-add, every sum over a block in
+ * index order from +0, means as the sum times 1/128; so the supports and the
+ * salience set are reproducible bit for bit by any implementation that does
+ * the same.
+ *   W: fp16 [N][K], 16-byte aligned;  nnz: 0 <= nnz <= N * K / 128;
+ *   sweeps: 0 .. 64;
+ *   plane1: out [N][tq_row_bytes(K)], 16-byte aligned (pad bytes written 0);
+ *   sal: out [N][tq_sal_words(K)];  rowptr: out [N + 1];
+ *   plane2: out [nnz][26], 16-byte aligned;  scale2: out fp16 [nnz]
+ *     (both may be NULL iff nnz == 0);
+ *   scale1, offset: out fp16 [N][K / 128];
+ *   workspace: tq_ternarize_workspace_bytes(N, K) bytes, 16-byte aligned
+ *     (nothing in it needs to start at zero);
+ *   d_status: TQ_DATA_BAD_WEIGHT for an inf or NaN weight (the outputs are
+ *     then unspecified but written in bounds).
+ * Asynchronous on stream: eight kernel launches and one memset. */
+TQ_API size_t tq_ternarize_workspace_bytes(int32_t N, int32_t K);
+TQ_API tq_status tq_ternarize(int32_t N, int32_t K, const uint16_t *W, int64_t nnz, int32_t sweeps,
+                              uint8_t *plane1, uint32_t *sal, int32_t *rowptr, uint8_t *plane2,
+                              uint16_t *scale1, uint16_t *offset, uint16_t *scale2, void *workspace,
+                              size_t workspace_bytes, uint32_t *d_status, void *stream);
 
 /* Device workspace of the decode path (M <= TQ_MAX_SKINNY_M): the
  * activations of every call are first rearranged into the tensor-core

@@ -25,6 +25,10 @@ int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
+size_t ternarize_ws_bytes(int N, int K);
+cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int sweeps, uint8_t *plane1,
+                             uint32_t *sal, int32_t *rowptr, uint8_t *plane2, uint16_t *scale1, uint16_t *offset,
+                             uint16_t *scale2, unsigned char *ws, uint32_t *status, cudaStream_t s);
 cudaError_t read_status_prefill(uint32_t *out, bool clear);
 }  // namespace tq
 
@@ -245,6 +249,29 @@ tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32
   if (tq_plane2_index_bytes(N, K, nnz) == 0) return TQ_ERR_SHAPE;
   if (((uintptr_t)index & 15u) || (plane2 && !aligned16(plane2)) || (scale2 && !aligned2(scale2))) return TQ_ERR_ALIGN;
   return from_cuda(launch_plane2_index(N, K, sal, rowptr, nnz, plane2, scale2, index, (cudaStream_t)stream));
+}
+
+size_t tq_ternarize_workspace_bytes(int32_t N, int32_t K) {
+  if (check_shape(N, K) != TQ_OK || (int64_t)N * (K / TQ_GROUP) > INT32_MAX) return 0;
+  return ternarize_ws_bytes(N, K);
+}
+
+tq_status tq_ternarize(int32_t N, int32_t K, const uint16_t *W, int64_t nnz, int32_t sweeps, uint8_t *plane1,
+                       uint32_t *sal, int32_t *rowptr, uint8_t *plane2, uint16_t *scale1, uint16_t *offset,
+                       uint16_t *scale2, void *workspace, size_t workspace_bytes, uint32_t *d_status,
+                       void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  const int64_t NB = (int64_t)N * (K / TQ_GROUP);
+  if (NB > INT32_MAX || nnz < 0 || nnz > NB || sweeps < 0 || sweeps > 64) return TQ_ERR_SHAPE;
+  if (!W || !plane1 || !sal || !rowptr || !scale1 || !offset || !workspace || !d_status) return TQ_ERR_NULL;
+  if (nnz > 0 && (!plane2 || !scale2)) return TQ_ERR_NULL;
+  if (workspace_bytes < ternarize_ws_bytes(N, K)) return TQ_ERR_SHAPE;
+  if (!aligned16(W) || !aligned16(plane1) || !aligned16(workspace) || (plane2 && !aligned16(plane2)) ||
+      !aligned2(scale1) || !aligned2(offset) || (scale2 && !aligned2(scale2)) || ((uintptr_t)sal & 3u) ||
+      ((uintptr_t)rowptr & 3u))
+    return TQ_ERR_ALIGN;
+  return from_cuda(launch_ternarize(N, K, W, nnz, sweeps, plane1, sal, rowptr, plane2, scale1, offset, scale2,
+                                    static_cast<unsigned char *>(workspace), d_status, (cudaStream_t)stream));
 }
 
 size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K) {

@@ -92,6 +92,10 @@ def lib():
             L.tq_linear_static.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp]
             L.tq_linear_batched.restype = ctypes.c_int
             L.tq_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
+            L.tq_ternarize_workspace_bytes.restype = sz
+            L.tq_ternarize_workspace_bytes.argtypes = [i32, i32]
+            L.tq_ternarize.restype = ctypes.c_int
+            L.tq_ternarize.argtypes = [i32, i32, vp, i64, i32] + [vp] * 8 + [sz, vp, vp]
             L.tq_get_device_status.restype = ctypes.c_int
             L.tq_get_device_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int]
             L.tq_status_str.restype = ctypes.c_char_p
@@ -225,6 +229,36 @@ def pack_weight(T1, T2, sal, s1, off, s2, stream=None, check=True, index=True) -
             raise TQError(-4, f"tq_pack data status {st:#x}")
     if s2 is None or nnz == 0:
         s2 = torch.zeros(1, dtype=torch.float16, device=dev)
+    p2index = tq_plane2_index(N, K, sal, rowptr, nnz, plane2, s2, stream) if index and nnz > 0 else None
+    return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz, p2index)
+
+
+def tq_ternarize_workspace_bytes(N: int, K: int) -> int:
+    return int(lib().tq_ternarize_workspace_bytes(N, K))
+
+
+def ternarize(W, nnz: int, sweeps: int = 4, d_status=None, ws=None, stream=None, index=True) -> PackedWeight:
+    """E2M-ATQ ternarization (tq_ternarize) of fp16 W [N][K] on the device
+    into a packed weight with nnz salient groups (and, unless index=False,
+    its second-plane index).  d_status: optional int32 device word the data
+    status is OR-ed into (else a fresh one, not read)."""
+    N, K = W.shape
+    dev = W.device
+    G = K // TQ_GROUP
+    plane1 = torch.empty((N, tq_row_bytes(K)), dtype=torch.uint8, device=dev)
+    sal = torch.empty((N, tq_sal_words(K)), dtype=torch.int32, device=dev)
+    rowptr = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    plane2 = torch.empty((max(nnz, 1), TQ_GROUP_BYTES), dtype=torch.uint8, device=dev)
+    s1 = torch.empty((N, G), dtype=torch.float16, device=dev)
+    off = torch.empty((N, G), dtype=torch.float16, device=dev)
+    s2 = torch.empty(max(nnz, 1), dtype=torch.float16, device=dev)
+    if ws is None:
+        ws = workspace(tq_ternarize_workspace_bytes(N, K), dev)
+    if d_status is None:
+        d_status = torch.zeros(1, dtype=torch.int32, device=dev)
+    _check(lib().tq_ternarize(N, K, _p(W), nnz, sweeps, _p(plane1), _p(sal), _p(rowptr),
+                              _p(plane2) if nnz > 0 else None, _p(s1), _p(off), _p(s2) if nnz > 0 else None,
+                              _p(ws), ws.numel(), _p(d_status), _stream(stream)), "tq_ternarize")
     p2index = tq_plane2_index(N, K, sal, rowptr, nnz, plane2, s2, stream) if index and nnz > 0 else None
     return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz, p2index)
 

@@ -47,6 +47,14 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_linear(1, 4, 128, None, None, None, None, 0, None) == -1
     assert L.tq_linear_batched(17, 1, None, None, 0, None) == -2
     assert L.tq_linear_batched(1, 0, None, None, 0, None) == -2
+    # ternarizer: shape, count and null checks come before anything touches the device
+    assert L.tq_ternarize(0, 128, None, 0, 4, *[None] * 8, 0, None, None) == -2
+    assert L.tq_ternarize(4, 128, None, 5, 4, *[None] * 8, 0, None, None) == -2   # nnz > N * G
+    assert L.tq_ternarize(4, 128, None, 1, 65, *[None] * 8, 0, None, None) == -2  # sweeps > 64
+    assert L.tq_ternarize(4, 128, None, 1, 4, *[None] * 8, 0, None, None) == -1
+    assert tq.tq_ternarize_workspace_bytes(0, 128) == 0 and tq.tq_ternarize_workspace_bytes(4, 100) == 0
+    # stats (16 B) and keys (4 B) per block, the select state, one word per 1024 salience words
+    assert tq.tq_ternarize_workspace_bytes(4096, 4096) == 2097152 + 524288 + 4352 + 256
     # M <= 8: activation fragments (320 B per group and token), C/S (64 B per
     # group), second-plane partials (4 B per row and token), each 256-padded,
     # and a 512-byte slot for the tensor maps of plane 1, s1 and off
