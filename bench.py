@@ -8,6 +8,7 @@ launch).  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tq|reference]
   python bench.py --prefill      (one Qwen3-8B layer at M = 2048 tokens)
+  python bench.py --ternarize    (E2M-ATQ ternarization of one Qwen3-8B layer)
 
 --impl reference times the CPU oracle on the host cores (the reference arm
 of this project: a plain fp64 implementation of the same layer) on a
@@ -195,14 +196,17 @@ def build_step(M, device, seed0=0, layers=None):
     return items, x_all, y_all, total_bytes, total_w
 
 
+# the sources the decode-step kernels are compiled from
+DECODE_SOURCES = ("tq_common.cuh", "tq_gemv_mma.cu", "tq_sm100.cuh")
+
+
 def kernel_hash():
     import hashlib
 
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_09240_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh")):
-            h.update(open(os.path.join(csrc, f), "rb").read())
+    for f in DECODE_SOURCES:
+        h.update(open(os.path.join(csrc, f), "rb").read())
     return h.hexdigest()[:16]
 
 
@@ -358,6 +362,146 @@ def run_prefill(args, ws, rank, local):
     return 0
 
 
+# ----------------------------------------------------------------- ternarize
+# fp32 operations of the method per weight (the oracle's operations; a
+# product with a trit counts as one), with 4 refinement sweeps:
+#   statistics 15 (mean 1, mean |c| 3, support 3, first scale 3, energy 5);
+#   planes 27 for a block without second plane (support 3, sweep 6 x 4),
+#   78 for a salient block (supports 3 + 5, residual mean 5, second scale 5,
+#   sweep 15 x 4).
+TERN_OPS_STATS, TERN_OPS_PLAIN, TERN_OPS_SALIENT = 15, 27, 78
+# fp32 lanes x SMs x maximum SM clock: the ALU peak for single fp32 operations
+ALU_PEAK_TOPS = 128 * 152 * 2.07e9 / 1e12
+
+
+def run_ternarize(args, ws, rank, local):
+    """E2M-ATQ ternarization (tq_ternarize) of one Qwen3-8B layer: its seven
+    dense fp16 projections (seeded synthetic weights resident in HBM) into
+    packed weights with 10 % salient groups and 4 refinement sweeps."""
+    import ctypes
+
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    L = tq.lib()
+    stream = torch.cuda.current_stream()
+    P = lambda t: ctypes.c_void_p(t.data_ptr())
+    sweeps, frac = 4, 0.1
+    jobs, n_weights, ops = [], 0, 0.0
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    for i, (nm, N, K) in enumerate(wl.QWEN3_8B):
+        W = wl.gen_dense_weights_torch(N, K, dev, seed=700 + i)
+        G = K // 128
+        nnz = int(round(frac * N * G))
+        out = dict(plane1=torch.empty((N, tq.tq_row_bytes(K)), dtype=torch.uint8, device=dev),
+                   sal=torch.empty((N, tq.tq_sal_words(K)), dtype=torch.int32, device=dev),
+                   rowptr=torch.empty(N + 1, dtype=torch.int32, device=dev),
+                   plane2=torch.empty((nnz, 26), dtype=torch.uint8, device=dev),
+                   s1=torch.empty((N, G), dtype=torch.float16, device=dev),
+                   off=torch.empty((N, G), dtype=torch.float16, device=dev),
+                   s2=torch.empty(nnz, dtype=torch.float16, device=dev))
+        wsb = tq.workspace(tq.tq_ternarize_workspace_bytes(N, K), dev)
+        jobs.append((N, K, nnz, W, out, wsb))
+        n_weights += N * K
+        ops += N * K * (TERN_OPS_STATS + (1 - nnz / (N * G)) * TERN_OPS_PLAIN + nnz / (N * G) * TERN_OPS_SALIENT)
+
+    def call(N, K, nnz, W, o, wsb):
+        rc = L.tq_ternarize(N, K, P(W), nnz, sweeps, P(o["plane1"]), P(o["sal"]), P(o["rowptr"]), P(o["plane2"]),
+                            P(o["s1"]), P(o["off"]), P(o["s2"]), P(wsb), wsb.numel(), P(st),
+                            ctypes.c_void_p(stream.cuda_stream))
+        assert rc == 0, rc
+
+    def step():
+        for j in jobs:
+            call(*j)
+
+    steps = max(1, min(args.steps, 50))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        clk.ready()
+        for _ in range(max(args.warmup, 3)):
+            step()
+        torch.cuda.synchronize()
+        clk.mark()
+        e0.record(stream)
+        for _ in range(steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        clk.mark()
+    ms = e0.elapsed_time(e1) / steps
+    assert int(st.item()) == 0
+    # end to end: fp16 weights from pinned host memory, packed outputs back to pinned host memory
+    hostW = [j[3].cpu().pin_memory() for j in jobs]
+    hostO = [{k: v.cpu().pin_memory() for k, v in j[4].items()} for j in jobs]
+    h2d = sum(h.numel() * 2 for h in hostW)
+    d2h = sum(v.numel() * v.element_size() for o in hostO for v in o.values())
+
+    def e2e_step():
+        for (N, K, nnz, W, o, wsb), hw, ho in zip(jobs, hostW, hostO):
+            W.copy_(hw, non_blocking=True)
+            call(N, K, nnz, W, o, wsb)
+            for k, v in o.items():
+                ho[k].copy_(v, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / steps
+    achieved = ops / (ms * 1e-3) / 1e12
+    out = {
+        "metric": "Qwen3-8B E2M-ATQ ternarization into the packed format: weights/s", "value": n_weights / (ms * 1e-3) / 1e9,
+        "unit": "Gweights/s", "n_gpus": 1, "steps": steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "E2M-ATQ of one Qwen3-8B layer's 7 projections (fp16 in, packed out), "
+                               "10% salient groups, 4 sweeps", "weights_per_step": n_weights,
+                   "l2": "no flush: a layer's 386 MB of fp16 weights exceed L2 per step"},
+        "roofline": {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TOPS, "unit": "Top/s",
+                     "frac": achieved / ALU_PEAK_TOPS, "traffic": None,
+                     "peak_kind": "fp32 lanes x 152 SMs x 2.07 GHz (derived, not measured)",
+                     "kernel": "whole tq_ternarize call (nine launches per projection, 63 per step)",
+                     "ops_per_step": ops},
+        "e2e": {"value": n_weights / (e2e_ms * 1e-3) / 1e9, "unit": "Gweights/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": 9 * 7 * steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = ternarize_cpu_baseline(10.0)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    return 0
+
+
+def ternarize_cpu_baseline(budget_s):
+    """The oracle (numpy float32) on whole projections of the same layer, in
+    order, until `budget_s` seconds have been timed."""
+    import workloads as wl
+    from oracle import ternarize as tz
+
+    n, t, names = 0, 0.0, []
+    for i, (nm, N, K) in enumerate(wl.QWEN3_8B):
+        if t >= budget_s:
+            break
+        W = wl.gen_dense_weights(N, K, config=9, proj=700 + i)
+        t0 = time.perf_counter()
+        tz.ternarize(W, int(round(0.1 * N * K / 128)), sweeps=4)
+        t += time.perf_counter() - t0
+        n += N * K
+        names.append(nm)
+    return {"value": n / t / 1e9, "unit": "Gweights/s", "cores": 1, "kind": "oracle",
+            "sample": f"the oracle on whole projections {', '.join(names)} of one Qwen3-8B layer "
+                      f"({n / 1e6:.1f} M weights, {t:.1f} s, numpy on one core)"}
+
+
 # ------------------------------------------------------------------- main
 def run_reference(args, ws, rank):
     """The oracle timed on the host cores: each step is one pass over a
@@ -404,12 +548,15 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="profile a smaller step (first L layers)")
     ap.add_argument("--prefill", action="store_true", help="one Qwen3-8B layer at M = 2048 tokens")
+    ap.add_argument("--ternarize", action="store_true", help="E2M-ATQ ternarization of one Qwen3-8B layer")
     args = ap.parse_args()
     ws, rank, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, ws, rank)
     if args.prefill:
         return run_prefill(args, ws, rank, local)
+    if args.ternarize:
+        return run_ternarize(args, ws, rank, local)
 
     import torch
 

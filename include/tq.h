@@ -74,8 +74,11 @@ typedef enum {
   TQ_ERR_SALIENCE = -6, /* descriptor nnz / salience inconsistent          */
   TQ_ERR_CUDA = -7,     /* a CUDA launch or query failed                  */
   TQ_ERR_TIMEOUT = -8,  /* a bounded device wait ran out                  */
-  TQ_ERR_SCRATCH = -9   /* tq_linear_static: the call needs more scratch than
+  TQ_ERR_SCRATCH = -9,  /* tq_linear_static: the call needs more scratch than
                            TQ_STATIC_SCRATCH_BYTES                         */
+  TQ_ERR_FORMAT = -10,  /* container: bad magic, version, size or hash     */
+  TQ_ERR_KEY = -11      /* container: missing, unexpected, duplicate or
+                           malformed name                                   */
 } tq_status;
 
 /* Bits OR-ed into *d_status by the codec kernels. */
@@ -199,12 +202,70 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
  *     (nothing in it needs to start at zero);
  *   d_status: TQ_DATA_BAD_WEIGHT for an inf or NaN weight (the outputs are
  *     then unspecified but written in bounds).
- * Asynchronous on stream: eight kernel launches and one memset. */
+ * Asynchronous on stream: at most nine kernel launches and one memset. */
 TQ_API size_t tq_ternarize_workspace_bytes(int32_t N, int32_t K);
 TQ_API tq_status tq_ternarize(int32_t N, int32_t K, const uint16_t *W, int64_t nnz, int32_t sweeps,
                               uint8_t *plane1, uint32_t *sal, int32_t *rowptr, uint8_t *plane2,
                               uint16_t *scale1, uint16_t *offset, uint16_t *scale2, void *workspace,
                               size_t workspace_bytes, uint32_t *d_status, void *stream);
+
+/* W-hat of a packed weight as dense fp16 [N][K] (16-byte aligned):
+ * fp16((s1 * t1 + off) + s2 * t2), the sums in float32, rounded to nearest
+ * even (paper "Model and Representation", eq. for W-hat, per group).  For
+ * provenance checks against the source weights and for export.  Invalid
+ * bytes set TQ_DATA_BAD_BYTE, a record index outside [0, nnz)
+ * TQ_DATA_BAD_ROWPTR (that group's second plane is then left out).
+ * Asynchronous on stream. */
+TQ_API tq_status tq_dequantize(int32_t N, int32_t K, const tq_weight *w, uint16_t *out, uint32_t *d_status,
+                               void *stream);
+
+/* ---- Packed-weight container (HOST memory; no device access, synchronous).
+ * Serialization of packed projections under names (paper "Packing: From
+ * Quantization to Serialization": the discrete supports and their
+ * parameters are what is stored), with the checks of its "Provenance
+ * safeguards": every key present and no unexpected one, every field's hash,
+ * the shapes, rowptr against the salience map and every packed byte
+ * (base-3 numerals <= 242, tail pad digits 1, row pad bytes 0).
+ * Layout: a 64-byte header ("TQPACK01", version, count, offsets, total
+ * size, FNV-1a 64 hashes of the table and of the header), a 384-byte table
+ * entry per projection (name, N, K, group, nnz, the source fingerprint, and
+ * offset / size / FNV-1a 64 of each field), then the fields at 16-byte
+ * aligned offsets in the order plane1, salience, rowptr, plane2, scale1,
+ * offset, scale2, each in the tq_weight layout. */
+typedef struct {
+  const char *name;          /* 1..127 bytes, NUL-terminated, unique        */
+  int32_t N, K;
+  int64_t nnz;
+  const uint8_t *plane1;     /* the tq_weight fields, in HOST memory        */
+  const uint32_t *salience;
+  const int32_t *rowptr;
+  const uint8_t *plane2;     /* NULL allowed when nnz == 0                  */
+  const uint16_t *scale1;
+  const uint16_t *offset;
+  const uint16_t *scale2;    /* NULL allowed when nnz == 0                  */
+  uint64_t source_hash;      /* e.g. tq_fnv1a64 of the source fp16 weights; 0 = none */
+} tq_host_weight;
+
+/* FNV-1a 64 (Fowler-Noll-Vo) of a host byte range. */
+TQ_API uint64_t tq_fnv1a64(const void *data, size_t bytes);
+/* Bytes of a container holding these projections; 0 for an invalid shape. */
+TQ_API size_t tq_container_bytes(int32_t count, const tq_host_weight *w);
+/* Writes the container into buf (16-byte aligned, >= tq_container_bytes).
+ * Fields are copied; hashes computed.  TQ_ERR_KEY: a bad or duplicate name. */
+TQ_API tq_status tq_container_write(int32_t count, const tq_host_weight *w, void *buf, size_t bytes);
+/* Number of entries, after checking the header and table hashes.
+ * `bytes` must be the container's exact size. */
+TQ_API tq_status tq_container_count(const void *buf, size_t bytes, int32_t *count);
+/* Index of the entry named `name` (TQ_ERR_KEY if absent). */
+TQ_API tq_status tq_container_find(const void *buf, size_t bytes, const char *name, int32_t *index);
+/* Entry `index`, fully checked (hashes TQ_ERR_FORMAT, rowptr / salience
+ * TQ_ERR_SALIENCE, packed bytes TQ_ERR_BYTE); on success *out points into
+ * buf (name included).  buf must be 8-byte aligned. */
+TQ_API tq_status tq_container_entry(const void *buf, size_t bytes, int32_t index, tq_host_weight *out);
+/* Keys: *missing = expected names absent from the container, *unexpected =
+ * entries whose name is not expected; TQ_ERR_KEY unless both are 0. */
+TQ_API tq_status tq_container_check_keys(const void *buf, size_t bytes, int32_t n_expected,
+                                         const char *const *expected, int32_t *missing, int32_t *unexpected);
 
 /* Device workspace of the decode path (M <= TQ_MAX_SKINNY_M): the
  * activations of every call are first rearranged into the tensor-core

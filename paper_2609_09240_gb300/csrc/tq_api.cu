@@ -26,6 +26,7 @@ void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2)
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
 size_t ternarize_ws_bytes(int N, int K);
+cudaError_t launch_dequantize(int N, int K, const tq_weight *w, uint16_t *out, uint32_t *status, cudaStream_t s);
 cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int sweeps, uint8_t *plane1,
                              uint32_t *sal, int32_t *rowptr, uint8_t *plane2, uint16_t *scale1, uint16_t *offset,
                              uint16_t *scale2, unsigned char *ws, uint32_t *status, cudaStream_t s);
@@ -251,6 +252,14 @@ tq_status tq_plane2_index(int32_t N, int32_t K, const uint32_t *sal, const int32
   return from_cuda(launch_plane2_index(N, K, sal, rowptr, nnz, plane2, scale2, index, (cudaStream_t)stream));
 }
 
+tq_status tq_dequantize(int32_t N, int32_t K, const tq_weight *w, uint16_t *out, uint32_t *d_status,
+                        void *stream) {
+  if (tq_status st = check_weight(w, N, K)) return st;
+  if (!out || !d_status) return TQ_ERR_NULL;
+  if (!aligned16(out)) return TQ_ERR_ALIGN;
+  return from_cuda(launch_dequantize(N, K, w, out, d_status, (cudaStream_t)stream));
+}
+
 size_t tq_ternarize_workspace_bytes(int32_t N, int32_t K) {
   if (check_shape(N, K) != TQ_OK || (int64_t)N * (K / TQ_GROUP) > INT32_MAX) return 0;
   return ternarize_ws_bytes(N, K);
@@ -342,6 +351,8 @@ const char *tq_status_str(tq_status s) {
     case TQ_ERR_TIMEOUT: return "TQ_ERR_TIMEOUT: a bounded device wait ran out";
     case TQ_ERR_SCRATCH:
       return "TQ_ERR_SCRATCH: the call needs more workspace than the static scratch of tq_linear_static (1 MiB)";
+    case TQ_ERR_FORMAT: return "TQ_ERR_FORMAT: container magic, version, size or hash mismatch";
+    case TQ_ERR_KEY: return "TQ_ERR_KEY: container name missing, unexpected, duplicate or malformed";
   }
   return "unknown tq_status";
 }

@@ -29,8 +29,9 @@
 //   tern_mark_kernel    salience words: keys above the selected key, and the
 //                       first `need` equal keys in block-id order
 //   rowptr (tq_codec.cu), then
-//   tern_pack_kernel    per block: supports, second plane, refinement, and
-//                       the packed bytes and fp16 parameters.
+//   tern_planes_kernel  per block: supports, second plane, refinement, and
+//                       the packed bytes and fp16 parameters (salient blocks
+//                       by record, in CTAs of their own).
 #include "tq_common.cuh"
 
 namespace tq {
@@ -41,7 +42,8 @@ cudaError_t launch_rowptr(int N, int K, const uint32_t *sal, int32_t *rowptr, ui
 namespace tz {
 
 constexpr int kBlockThreads = 128;  // per-block kernels: one thread per (row, group)
-constexpr int kSelThreads = 1024;   // select kernels; one salience word per thread in count / mark
+constexpr int kSelThreads = 1024;   // histogram kernels
+constexpr int kMarkThreads = 128;   // count / mark kernels: one salience word per thread
 constexpr float kInvGroup = 0.0078125f;  // 1 / 128, exact
 constexpr float kThresh = 0.75f;         // E2M-ATQ threshold factor
 
@@ -277,19 +279,29 @@ __global__ void __launch_bounds__(kSelThreads) tern_hist_kernel(int pass, int64_
   }
 }
 
-// Keys of salience word w (row n = w / SW, word j = w % SW) compared with the
-// selected key T: masks of the valid groups above T and equal to T.
-__device__ __forceinline__ void word_masks(const uint32_t *keys, int G, int SW, int64_t w, uint32_t T,
-                                           uint32_t &gt, uint32_t &eq) {
-  const int64_t n = w / SW;
-  const int j = (int)(w - n * SW);
-  const int g0 = 32 * j, cnt = min(32, G - g0);
-  const uint32_t *k = keys + n * G + g0;
+// Masks of the 32 salience words w0 .. w0 + 31 (word w: row w / SW, word
+// w % SW) against the selected key T, built by one warp: per word, lane l
+// reads the key of group 32 (w % SW) + l (one coalesced load) and two
+// ballots give the valid groups above T and equal to T; lane k keeps word
+// w0 + k's masks.
+__device__ __forceinline__ void warp_word_masks(const uint32_t *keys, int G, int SW, int NW, int w0, uint32_t T,
+                                                uint32_t &gt, uint32_t &eq) {
+  const int lane = threadIdx.x & 31;
   gt = 0u, eq = 0u;
-  for (int i = 0; i < cnt; ++i) {
-    const uint32_t v = k[i];
-    gt |= (uint32_t)(v > T) << i;
-    eq |= (uint32_t)(v == T) << i;
+  uint32_t v[32];
+  bool ok[32];
+  // all 32 loads first (in flight together), then the ballots
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    const int w = w0 + k, n = w / SW, j = w - n * SW;
+    ok[k] = w < NW && lane < G - 32 * j;
+    v[k] = ok[k] ? keys[(int64_t)n * G + 32 * j + lane] : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    const uint32_t bg = __ballot_sync(0xffffffffu, ok[k] && v[k] > T);
+    const uint32_t be = __ballot_sync(0xffffffffu, ok[k] && v[k] == T);
+    if (lane == k) gt = bg, eq = be;
   }
 }
 
@@ -301,35 +313,38 @@ __device__ __forceinline__ int block_sum(int v, int *red) {
   if (lane == 0) red[wid] = v;
   __syncthreads();
   int t = 0;
-  for (int i = 0; i < kSelThreads / 32; ++i) t += red[i];
+  for (int i = 0; i < kMarkThreads / 32; ++i) t += red[i];
   return t;
 }
 
-__global__ void __launch_bounds__(kSelThreads) tern_count_kernel(int64_t NW, int G, int SW, const uint32_t *keys,
-                                                                 const SelWork *sw, uint32_t *chunk_eq) {
-  __shared__ int red[kSelThreads / 32];
-  const int64_t w = (int64_t)blockIdx.x * kSelThreads + threadIdx.x;
-  uint32_t gt = 0u, eq = 0u;
-  if (w < NW) word_masks(keys, G, SW, w, sw->st.prefix[4], gt, eq);
+// Keys equal to the selected key, per chunk of kMarkThreads salience words.
+__global__ void __launch_bounds__(kMarkThreads) tern_count_kernel(int NW, int G, int SW, const uint32_t *keys,
+                                                                  const SelWork *sw, uint32_t *chunk_eq) {
+  __shared__ int red[kMarkThreads / 32];
+  const int w0 = (int)blockIdx.x * kMarkThreads + (threadIdx.x & ~31);
+  uint32_t gt, eq;
+  warp_word_masks(keys, G, SW, NW, w0, sw->st.prefix[4], gt, eq);
   const int t = block_sum(__popc(eq), red);
   if (threadIdx.x == 0) chunk_eq[blockIdx.x] = (uint32_t)t;
 }
 
-__global__ void __launch_bounds__(kSelThreads) tern_mark_kernel(int64_t NW, int G, int SW, const uint32_t *keys,
-                                                                const SelWork *sw, const uint32_t *chunk_eq,
-                                                                uint32_t *sal) {
-  __shared__ int red[kSelThreads / 32];
-  __shared__ int wpre[kSelThreads / 32];
+// Salience words of a chunk: groups above the selected key, and equal ones
+// while fewer than `need` equal keys precede them in block-id order.
+__global__ void __launch_bounds__(kMarkThreads) tern_mark_kernel(int NW, int G, int SW, const uint32_t *keys,
+                                                                 const SelWork *sw, const uint32_t *chunk_eq,
+                                                                 uint32_t *sal) {
+  __shared__ int red[kMarkThreads / 32];
+  __shared__ int wpre[kMarkThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const uint32_t T = sw->st.prefix[4];
   const int64_t need = sw->st.need[4];
   // equal keys in earlier chunks
   int before = 0;
-  for (int c = tid; c < (int)blockIdx.x; c += kSelThreads) before += (int)chunk_eq[c];
+  for (int c = tid; c < (int)blockIdx.x; c += kMarkThreads) before += (int)chunk_eq[c];
   const int64_t base = block_sum(before, red);
-  const int64_t w = (int64_t)blockIdx.x * kSelThreads + tid;
-  uint32_t gt = 0u, eq = 0u;
-  if (w < NW) word_masks(keys, G, SW, w, T, gt, eq);
+  const int w0 = (int)blockIdx.x * kMarkThreads + (tid & ~31);
+  uint32_t gt, eq;
+  warp_word_masks(keys, G, SW, NW, w0, T, gt, eq);
   // exclusive scan of the equal counts over the chunk's words (block-id order)
   const int cnt = __popc(eq);
   int incl = cnt;
@@ -345,6 +360,7 @@ __global__ void __launch_bounds__(kSelThreads) tern_mark_kernel(int64_t NW, int 
   int64_t rank = base + wbase + incl - cnt;  // equal keys before this word
   uint32_t take = 0u;
   for (uint32_t m = eq; m && rank < need; m &= m - 1u, ++rank) take |= m & (~m + 1u);
+  const int w = w0 + lane;
   if (w < NW) sal[w] = gt | take;
 }
 
@@ -373,19 +389,18 @@ __device__ __forceinline__ void store_group(const uint32_t (&nz)[4], const uint3
   }
 }
 
-// Blocks without a second plane: the first support from the statistics,
+// Blocks without a second plane (the CTAs from p2_ctas on of
+// tern_planes_kernel): the first support from the statistics,
 // then `sweeps` refinements of mu and alpha0 (alpha1 = 0, T1 = 0: the terms
 // -alpha1 T1 = -(+0) leave every value unchanged, so they are left out).
-// Salient blocks are skipped here; tern_plane2_kernel writes them.  Also
+// Salient blocks are skipped here; plane2_blocks writes them.  Also
 // zeroes each row's pad bytes.
-__global__ void __launch_bounds__(kBlockThreads) tern_plane1_kernel(int N, int K, int sweeps, const uint16_t *W,
-                                                                    const float4 *stats, const uint32_t *sal,
-                                                                    uint8_t *plane1, __half *s1, __half *off) {
-  __shared__ uint32_t sx[64 * kBlockThreads];
+__device__ __forceinline__ void plane1_blocks(int cta, int ctas, uint32_t *sx, int N, int K, int sweeps,
+                                              const uint16_t *W, const float4 *stats, const uint32_t *sal,
+                                              uint8_t *plane1, __half *s1, __half *off) {
   const int G = K / kGroup, SW = sal_words_of(K);
   const int64_t NB = (int64_t)N * G, RB = row_bytes_of(K);
-  for (int64_t b = (int64_t)blockIdx.x * kBlockThreads + threadIdx.x; b < NB;
-       b += (int64_t)gridDim.x * kBlockThreads) {
+  for (int64_t b = (int64_t)cta * kBlockThreads + threadIdx.x; b < NB; b += (int64_t)ctas * kBlockThreads) {
     const int64_t n = b / G;
     const int g = (int)(b - n * G);
     uint8_t *row = plane1 + n * RB;
@@ -411,20 +426,20 @@ __global__ void __launch_bounds__(kBlockThreads) tern_plane1_kernel(int N, int K
   }
 }
 
-// Salient blocks, one thread per plane-2 record j < nnz: the record's row
+// Salient blocks (the first p2_ctas CTAs of tern_planes_kernel, scheduled
+// first because they take longest), one thread per plane-2 record j < nnz:
+// the record's row
 // (the last n with rowptr[n] <= j) and group (the (j - rowptr[n])-th set
 // salience bit of the row), then both supports, the refinement of mu,
 // alpha0 and alpha1, and both planes' bytes and parameters.
-__global__ void __launch_bounds__(kBlockThreads) tern_plane2_kernel(int N, int K, int sweeps, int64_t nnz,
-                                                                    const uint16_t *W, const float4 *stats,
-                                                                    const uint32_t *sal, const int32_t *rowptr,
-                                                                    uint8_t *plane1, uint8_t *plane2, __half *s1,
-                                                                    __half *off, __half *s2, uint32_t *status) {
-  __shared__ uint32_t sx[64 * kBlockThreads];
+__device__ __forceinline__ void plane2_blocks(int cta, int ctas, uint32_t *sx, int N, int K, int sweeps,
+                                              int64_t nnz, const uint16_t *W, const float4 *stats,
+                                              const uint32_t *sal, const int32_t *rowptr, uint8_t *plane1,
+                                              uint8_t *plane2, __half *s1, __half *off, __half *s2,
+                                              uint32_t *status) {
   const int G = K / kGroup, SW = sal_words_of(K);
   const int64_t RB = row_bytes_of(K);
-  for (int64_t j = (int64_t)blockIdx.x * kBlockThreads + threadIdx.x; j < nnz;
-       j += (int64_t)gridDim.x * kBlockThreads) {
+  for (int64_t j = (int64_t)cta * kBlockThreads + threadIdx.x; j < nnz; j += (int64_t)ctas * kBlockThreads) {
     int lo = 0, hi = N;  // rowptr[lo] <= j < rowptr[hi] for a consistent rowptr
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
@@ -495,6 +510,21 @@ __global__ void __launch_bounds__(kBlockThreads) tern_plane2_kernel(int N, int K
   }
 }
 
+// Both kinds of blocks in one launch: CTAs below p2_ctas take the salient
+// records, the rest the other blocks, so the two run side by side.
+__global__ void __launch_bounds__(kBlockThreads) tern_planes_kernel(int N, int K, int sweeps, int64_t nnz, int p2_ctas,
+                                                                   const uint16_t *W, const float4 *stats,
+                                                                   const uint32_t *sal, const int32_t *rowptr,
+                                                                   uint8_t *plane1, uint8_t *plane2, __half *s1,
+                                                                   __half *off, __half *s2, uint32_t *status) {
+  __shared__ uint32_t sx[64 * kBlockThreads];
+  if ((int)blockIdx.x < p2_ctas)
+    plane2_blocks(blockIdx.x, p2_ctas, sx, N, K, sweeps, nnz, W, stats, sal, rowptr, plane1, plane2, s1, off, s2,
+                  status);
+  else
+    plane1_blocks(blockIdx.x - p2_ctas, gridDim.x - p2_ctas, sx, N, K, sweeps, W, stats, sal, plane1, s1, off);
+}
+
 int grid_blocks(int64_t NB) {
   int64_t g = (NB + kBlockThreads - 1) / kBlockThreads;
   return (int)(g < 1 ? 1 : g > 152 * 16 ? 152 * 16 : g);
@@ -505,7 +535,7 @@ int grid_blocks(int64_t NB) {
 size_t ternarize_ws_bytes(int N, int K) {
   const int64_t NB = (int64_t)N * (K / kGroup);
   const int64_t NW = (int64_t)N * sal_words_of(K);
-  const int64_t chunks = (NW + tz::kSelThreads - 1) / tz::kSelThreads;
+  const int64_t chunks = (NW + tz::kMarkThreads - 1) / tz::kMarkThreads;
   auto pad = [](int64_t b) { return (b + 255) / 256 * 256; };
   return (size_t)(pad(NB * 16) + pad(NB * 4) + pad(sizeof(tz::SelWork)) + pad(chunks * 4));
 }
@@ -516,7 +546,7 @@ cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int s
   using namespace tz;
   const int G = K / kGroup, SW = sal_words_of(K);
   const int64_t NB = (int64_t)N * G, NW = (int64_t)N * SW;
-  const int64_t chunks = (NW + kSelThreads - 1) / kSelThreads;
+  const int64_t chunks = (NW + kMarkThreads - 1) / kMarkThreads;
   auto pad = [](int64_t b) { return (b + 255) / 256 * 256; };
   float4 *stats = reinterpret_cast<float4 *>(ws);
   uint32_t *keys = reinterpret_cast<uint32_t *>(ws + pad(NB * 16));
@@ -529,8 +559,8 @@ cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int s
     int hg = (int)((NB + kSelThreads - 1) / kSelThreads);
     if (hg > 152 * 2) hg = 152 * 2;
     for (int p = 0; p < 4; ++p) tern_hist_kernel<<<hg, kSelThreads, 0, s>>>(p, NB, nnz, keys, sw);
-    tern_count_kernel<<<(unsigned)chunks, kSelThreads, 0, s>>>(NW, G, SW, keys, sw, chunk_eq);
-    tern_mark_kernel<<<(unsigned)chunks, kSelThreads, 0, s>>>(NW, G, SW, keys, sw, chunk_eq, sal);
+    tern_count_kernel<<<(unsigned)chunks, kMarkThreads, 0, s>>>((int)NW, G, SW, keys, sw, chunk_eq);
+    tern_mark_kernel<<<(unsigned)chunks, kMarkThreads, 0, s>>>((int)NW, G, SW, keys, sw, chunk_eq, sal);
   } else {
     cudaError_t e = cudaMemsetAsync(sal, 0, (size_t)NW * 4, s);
     if (e != cudaSuccess) return e;
@@ -540,11 +570,10 @@ cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int s
   e = launch_rowptr(N, K, sal, rowptr, status, s);
   if (e != cudaSuccess) return e;
   __half *h1 = reinterpret_cast<__half *>(scale1), *ho = reinterpret_cast<__half *>(offset);
-  tern_plane1_kernel<<<grid_blocks(NB), kBlockThreads, 0, s>>>(N, K, sweeps, W, stats, sal, plane1, h1, ho);
-  if (nnz > 0)
-    tern_plane2_kernel<<<grid_blocks(nnz), kBlockThreads, 0, s>>>(N, K, sweeps, nnz, W, stats, sal, rowptr, plane1,
-                                                                   plane2, h1, ho, reinterpret_cast<__half *>(scale2),
-                                                                   status);
+  const int p2 = nnz > 0 ? grid_blocks(nnz) : 0;
+  tern_planes_kernel<<<p2 + grid_blocks(NB), kBlockThreads, 0, s>>>(N, K, sweeps, nnz, p2, W, stats, sal, rowptr,
+                                                                    plane1, plane2, h1, ho,
+                                                                    reinterpret_cast<__half *>(scale2), status);
   return cudaGetLastError();
 }
 

@@ -11,6 +11,7 @@ import os
 import threading
 from dataclasses import dataclass
 
+import numpy as np
 import torch
 
 from . import build as _build
@@ -22,8 +23,10 @@ TQ_MAX_BATCH = 256
 
 TQ_OK = 0
 STATUS_NAMES = {0: "TQ_OK", -1: "TQ_ERR_NULL", -2: "TQ_ERR_SHAPE", -3: "TQ_ERR_ALIGN", -4: "TQ_ERR_CODE",
-                -5: "TQ_ERR_BYTE", -6: "TQ_ERR_SALIENCE", -7: "TQ_ERR_CUDA", -8: "TQ_ERR_TIMEOUT"}
-DATA_BAD_CODE, DATA_T2_OUTSIDE, DATA_BAD_BYTE, DATA_BAD_PAD, DATA_BAD_ROWPTR = 1, 2, 4, 8, 16
+                -5: "TQ_ERR_BYTE", -6: "TQ_ERR_SALIENCE", -7: "TQ_ERR_CUDA", -8: "TQ_ERR_TIMEOUT",
+                -9: "TQ_ERR_SCRATCH", -10: "TQ_ERR_FORMAT", -11: "TQ_ERR_KEY"}
+TQ_ERR_FORMAT, TQ_ERR_KEY = -10, -11
+DATA_BAD_CODE, DATA_T2_OUTSIDE, DATA_BAD_BYTE, DATA_BAD_PAD, DATA_BAD_ROWPTR, DATA_BAD_WEIGHT = 1, 2, 4, 8, 16, 32
 
 _lock = threading.Lock()
 _lib = None
@@ -44,6 +47,13 @@ class tq_weight(ctypes.Structure):
 
 class tq_problem(ctypes.Structure):
     _fields_ = [("w", tq_weight), ("x", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+class tq_host_weight(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("N", ctypes.c_int32), ("K", ctypes.c_int32), ("nnz", ctypes.c_int64),
+                ("plane1", ctypes.c_void_p), ("salience", ctypes.c_void_p), ("rowptr", ctypes.c_void_p),
+                ("plane2", ctypes.c_void_p), ("scale1", ctypes.c_void_p), ("offset", ctypes.c_void_p),
+                ("scale2", ctypes.c_void_p), ("source_hash", ctypes.c_uint64)]
 
 
 def lib_path() -> str:
@@ -96,6 +106,24 @@ def lib():
             L.tq_ternarize_workspace_bytes.argtypes = [i32, i32]
             L.tq_ternarize.restype = ctypes.c_int
             L.tq_ternarize.argtypes = [i32, i32, vp, i64, i32] + [vp] * 8 + [sz, vp, vp]
+            L.tq_dequantize.restype = ctypes.c_int
+            L.tq_dequantize.argtypes = [i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp]
+            L.tq_fnv1a64.restype = ctypes.c_uint64
+            L.tq_fnv1a64.argtypes = [vp, sz]
+            HW = ctypes.POINTER(tq_host_weight)
+            L.tq_container_bytes.restype = sz
+            L.tq_container_bytes.argtypes = [i32, HW]
+            L.tq_container_write.restype = ctypes.c_int
+            L.tq_container_write.argtypes = [i32, HW, vp, sz]
+            L.tq_container_count.restype = ctypes.c_int
+            L.tq_container_count.argtypes = [vp, sz, ctypes.POINTER(ctypes.c_int32)]
+            L.tq_container_find.restype = ctypes.c_int
+            L.tq_container_find.argtypes = [vp, sz, ctypes.c_char_p, ctypes.POINTER(ctypes.c_int32)]
+            L.tq_container_entry.restype = ctypes.c_int
+            L.tq_container_entry.argtypes = [vp, sz, i32, HW]
+            L.tq_container_check_keys.restype = ctypes.c_int
+            L.tq_container_check_keys.argtypes = [vp, sz, i32, ctypes.POINTER(ctypes.c_char_p),
+                                                  ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32)]
             L.tq_get_device_status.restype = ctypes.c_int
             L.tq_get_device_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int]
             L.tq_status_str.restype = ctypes.c_char_p
@@ -261,6 +289,136 @@ def ternarize(W, nnz: int, sweeps: int = 4, d_status=None, ws=None, stream=None,
                               _p(ws), ws.numel(), _p(d_status), _stream(stream)), "tq_ternarize")
     p2index = tq_plane2_index(N, K, sal, rowptr, nnz, plane2, s2, stream) if index and nnz > 0 else None
     return PackedWeight(N, K, plane1, sal, rowptr, plane2, s1, off, s2, nnz, p2index)
+
+
+def tq_dequantize(w: PackedWeight, out=None, d_status=None, stream=None):
+    """W-hat of a packed weight as dense fp16 [N][K] on the device."""
+    if out is None:
+        out = torch.empty((w.N, w.K), dtype=torch.float16, device=w.plane1.device)
+    if d_status is None:
+        d_status = torch.zeros(1, dtype=torch.int32, device=w.plane1.device)
+    ws_ = w.struct()
+    _check(lib().tq_dequantize(w.N, w.K, ctypes.byref(ws_), _p(out), _p(d_status), _stream(stream)), "tq_dequantize")
+    return out
+
+
+def provenance(W_source, w: PackedWeight, stream=None) -> dict:
+    """The paper's "measurable weight change" check of a packed weight
+    against its fp16 source (both on the device): relative RMSE of W-hat,
+    the fraction of weights whose fp16 value changed, and whether W-hat is
+    bit-identical to the source (which a real ternarization never is)."""
+    Wh = tq_dequantize(w, stream=stream)
+    src = W_source.float()
+    err = (Wh.float() - src).pow(2).sum().sqrt() / src.pow(2).sum().sqrt().clamp_min(1e-30)
+    changed = (Wh.view(torch.int16) != W_source.view(torch.int16)).float().mean()
+    return {"rel_rmse": float(err), "changed_fraction": float(changed), "identical": bool(changed == 0)}
+
+
+# ---------------------------------------------------------------- container
+FIELDS = ("plane1", "salience", "rowptr", "plane2", "scale1", "offset", "scale2")
+
+
+def fnv1a64(a) -> int:
+    """FNV-1a 64 of a host array's bytes (or of a device tensor, copied to the host)."""
+    if isinstance(a, torch.Tensor):
+        a = a.detach().contiguous().cpu().numpy()
+    a = np.ascontiguousarray(a)
+    return int(lib().tq_fnv1a64(a.ctypes.data_as(ctypes.c_void_p), a.nbytes))
+
+
+def _aligned_bytes(n: int, align: int = 16) -> np.ndarray:
+    raw = np.empty(n + align, np.uint8)
+    off = (-raw.ctypes.data) % align
+    return raw[off:off + n]
+
+
+def _host_fields(w) -> dict:
+    """Host numpy copies of a weight's seven fields (PackedWeight or dict of arrays)."""
+    if isinstance(w, PackedWeight):
+        nnz = w.nnz
+        d = {"plane1": w.plane1, "salience": w.salience, "rowptr": w.rowptr, "scale1": w.scale1, "offset": w.offset,
+             "plane2": w.plane2[:nnz] if nnz else None, "scale2": w.scale2[:nnz] if nnz else None}
+        d = {k: (None if v is None else v.detach().contiguous().cpu().numpy()) for k, v in d.items()}
+        return dict(N=w.N, K=w.K, nnz=nnz, **d)
+    return dict(w)
+
+
+def container_write(entries) -> np.ndarray:
+    """Serialize [(name, weight, source_hash), ...] (weight: PackedWeight or a
+    dict with N, K, nnz and the seven host fields) into a 16-byte aligned
+    uint8 array, ready to be written to a file."""
+    hs = (tq_host_weight * max(len(entries), 1))()
+    keep = []
+    for i, (name, w, src_hash) in enumerate(entries):
+        f = _host_fields(w)
+        h = hs[i]
+        nb = name.encode()
+        keep.append(nb)
+        h.name, h.N, h.K, h.nnz, h.source_hash = nb, int(f["N"]), int(f["K"]), int(f["nnz"]), int(src_hash)
+        for k in FIELDS:
+            a = f.get(k)
+            if a is not None and a.size:
+                a = np.ascontiguousarray(a)
+                keep.append(a)
+                setattr(h, k, a.ctypes.data_as(ctypes.c_void_p))
+            else:
+                setattr(h, k, None)
+    n = int(lib().tq_container_bytes(len(entries), hs))
+    if n == 0:
+        raise TQError(-2, "tq_container_bytes")
+    buf = _aligned_bytes(n)
+    _check(lib().tq_container_write(len(entries), hs, buf.ctypes.data_as(ctypes.c_void_p), n), "tq_container_write")
+    return buf
+
+
+def container_read(data, expected=None, device=None, index=True):
+    """Check and unpack a container.  `data`: bytes or a uint8 array.  With
+    `expected` (list of names) the key check runs first and raises on any
+    missing or unexpected name.  Returns {name: (weight, source_hash)}; the
+    weight is a dict of host numpy arrays (device None) or a PackedWeight on
+    `device` (with its second-plane index unless index=False)."""
+    buf = _aligned_bytes(len(data))
+    buf[:] = np.frombuffer(data, np.uint8) if not isinstance(data, np.ndarray) else data.view(np.uint8)
+    p, n = buf.ctypes.data_as(ctypes.c_void_p), buf.nbytes
+    L = lib()
+    if expected is not None:
+        names = (ctypes.c_char_p * max(len(expected), 1))(*[e.encode() for e in expected])
+        miss, extra = ctypes.c_int32(0), ctypes.c_int32(0)
+        rc = L.tq_container_check_keys(p, n, len(expected), names, ctypes.byref(miss), ctypes.byref(extra))
+        if rc == TQ_ERR_KEY:
+            raise TQError(rc, f"container keys: {miss.value} missing, {extra.value} unexpected")
+        _check(rc, "tq_container_check_keys")
+    cnt = ctypes.c_int32(0)
+    _check(L.tq_container_count(p, n, ctypes.byref(cnt)), "tq_container_count")
+    out = {}
+    for i in range(cnt.value):
+        h = tq_host_weight()
+        _check(L.tq_container_entry(p, n, i, ctypes.byref(h)), f"tq_container_entry {i}")
+        N, K, nnz = h.N, h.K, h.nnz
+        G = K // TQ_GROUP
+        shapes = {"plane1": ((N, tq_row_bytes(K)), np.uint8), "salience": ((N, tq_sal_words(K)), np.int32),
+                  "rowptr": ((N + 1,), np.int32), "plane2": ((nnz, TQ_GROUP_BYTES), np.uint8),
+                  "scale1": ((N, G), np.float16), "offset": ((N, G), np.float16), "scale2": ((nnz,), np.float16)}
+        f = {}
+        for k, (shape, dt) in shapes.items():
+            ptr = getattr(h, k)
+            cnt_el = int(np.prod(shape))
+            if not ptr or cnt_el == 0:
+                f[k] = np.zeros(shape, dt)
+                continue
+            off = ptr - buf.ctypes.data
+            f[k] = buf[off:off + cnt_el * np.dtype(dt).itemsize].view(dt).reshape(shape).copy()
+        name = h.name.decode()
+        if device is None:
+            out[name] = (dict(N=N, K=K, nnz=nnz, **f), int(h.source_hash))
+            continue
+        t = {k: torch.from_numpy(v).to(device) for k, v in f.items()}
+        plane2 = t["plane2"] if nnz else torch.zeros((1, TQ_GROUP_BYTES), dtype=torch.uint8, device=device)
+        s2 = t["scale2"] if nnz else torch.zeros(1, dtype=torch.float16, device=device)
+        p2i = tq_plane2_index(N, K, t["salience"], t["rowptr"], nnz, plane2, s2) if index and nnz else None
+        out[name] = (PackedWeight(N, K, t["plane1"], t["salience"], t["rowptr"], plane2, t["scale1"], t["offset"],
+                                  s2, nnz, p2i), int(h.source_hash))
+    return out
 
 
 def tq_workspace_bytes(M: int, N: int, K: int) -> int:

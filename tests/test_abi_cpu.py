@@ -53,6 +53,7 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_ternarize(4, 128, None, 1, 65, *[None] * 8, 0, None, None) == -2  # sweeps > 64
     assert L.tq_ternarize(4, 128, None, 1, 4, *[None] * 8, 0, None, None) == -1
     assert tq.tq_ternarize_workspace_bytes(0, 128) == 0 and tq.tq_ternarize_workspace_bytes(4, 100) == 0
+    assert L.tq_dequantize(4, 128, None, None, None, None) == -1
     # stats (16 B) and keys (4 B) per block, the select state, one word per 1024 salience words
     assert tq.tq_ternarize_workspace_bytes(4096, 4096) == 2097152 + 524288 + 4352 + 256
     # M <= 8: activation fragments (320 B per group and token), C/S (64 B per
