@@ -363,13 +363,13 @@ def run_prefill(args, ws, rank, local):
 
 
 # ----------------------------------------------------------------- ternarize
-# fp32 operations of the method per weight (the oracle's operations; a
-# product with a trit counts as one), with 4 refinement sweeps:
+# fp32 operations per weight that the computation needs (a product with a
+# trit counts as one; the refinement sweeps are scalar work per block):
 #   statistics 15 (mean 1, mean |c| 3, support 3, first scale 3, energy 5);
-#   planes 27 for a block without second plane (support 3, sweep 6 x 4),
-#   78 for a salient block (supports 3 + 5, residual mean 5, second scale 5,
-#   sweep 15 x 4).
-TERN_OPS_STATS, TERN_OPS_PLAIN, TERN_OPS_SALIENT = 15, 27, 78
+#   planes 5 for a block without second plane (support 3, moments 2), 16 for
+#   a salient block (support and moments 5, residual mean 5, second support
+#   and its moment 6).
+TERN_OPS_STATS, TERN_OPS_PLAIN, TERN_OPS_SALIENT = 15, 5, 16
 # fp32 lanes x SMs x maximum SM clock: the ALU peak for single fp32 operations
 ALU_PEAK_TOPS = 128 * 152 * 2.07e9 / 1e12
 

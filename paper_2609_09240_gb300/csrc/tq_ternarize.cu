@@ -134,15 +134,18 @@ __device__ __forceinline__ int popc4(const uint32_t (&m)[4]) {
 }
 
 // Support of v (v(x) per weight) at threshold d (E2M-ATQ, eq. for T0): +1
-// above d, -1 below -d; returns the support's size.
-template <class V>
-__device__ __forceinline__ int support(const Blk &B, V v, float d, uint32_t (&nz)[4], uint32_t (&ng)[4]) {
+// above d, -1 below -d; on(x, t) sees each weight with its trit.  Returns
+// the support's size.
+template <class V, class On>
+__device__ __forceinline__ int support(const Blk &B, V v, float d, uint32_t (&nz)[4], uint32_t (&ng)[4], On on) {
   uint32_t mz = 0u, mg = 0u;
   B.each(
       [&](int q, int bit, float x) {
         const float c = v(q, bit, x);
-        if (c > d) mz |= 1u << bit;
-        if (c < -d) mz |= 1u << bit, mg |= 1u << bit;
+        const int t = c > d ? 1 : (c < -d ? -1 : 0);
+        if (t) mz |= 1u << bit;
+        if (t < 0) mg |= 1u << bit;
+        on(x, t);
       },
       [&](int q) {
         put4(nz, q, mz);
@@ -171,7 +174,7 @@ __device__ __forceinline__ void first_plane(const Blk &B, First &f, bool *bad) {
   float a = 0.f;
   B.each([&](int, int, float x) { a = __fadd_rn(a, fabsf(__fsub_rn(x, mu))); });
   const float d0 = __fmul_rn(kThresh, __fmul_rn(a, kInvGroup));
-  f.n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, d0, f.nz, f.ng);
+  f.n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, d0, f.nz, f.ng, [](float, int) {});
   float p = 0.f;
   B.each([&](int q, int bit, float x) {
     p = __fadd_rn(p, times_bit(__fsub_rn(x, mu), pick4(f.nz, q), pick4(f.ng, q), bit));
@@ -390,9 +393,9 @@ __device__ __forceinline__ void store_group(const uint32_t (&nz)[4], const uint3
 }
 
 // Blocks without a second plane (the CTAs from p2_ctas on of
-// tern_planes_kernel): the first support from the statistics,
-// then `sweeps` refinements of mu and alpha0 (alpha1 = 0, T1 = 0: the terms
-// -alpha1 T1 = -(+0) leave every value unchanged, so they are left out).
+// tern_planes_kernel): the first support from the statistics, then `sweeps`
+// refinements of mu and alpha0 (alpha1 = 0) on the block's moments (see
+// plane2_blocks).
 // Salient blocks are skipped here; plane2_blocks writes them.  Also
 // zeroes each row's pad bytes.
 __device__ __forceinline__ void plane1_blocks(int cta, int ctas, uint32_t *sx, int N, int K, int sweeps,
@@ -411,14 +414,13 @@ __device__ __forceinline__ void plane1_blocks(int cta, int ctas, uint32_t *sx, i
     const float4 st = stats[b];
     float mu = st.x, a0 = st.z;
     uint32_t nz0[4] = {0u, 0u, 0u, 0u}, ng0[4] = {0u, 0u, 0u, 0u};
-    const int n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, st.y, nz0, ng0);
+    float mw = 0.f, mw0 = 0.f;  // sum w, sum w T0
+    const int n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, st.y, nz0, ng0,
+                           [&](float x, int t) { mw += x, mw0 += t > 0 ? x : (t < 0 ? -x : 0.f); });
+    const int z0 = n0 - 2 * popc4(ng0);  // sum T0
     for (int sw = 0; sw < sweeps; ++sw) {
-      float u = 0.f;
-      B.each([&](int q, int bit, float x) { u = __fadd_rn(u, __fsub_rn(x, times_bit(a0, pick4(nz0, q), pick4(ng0, q), bit))); });
-      mu = __fmul_rn(u, kInvGroup);
-      float p = 0.f;
-      B.each([&](int q, int bit, float x) { p = __fadd_rn(p, times_bit(__fsub_rn(x, mu), pick4(nz0, q), pick4(ng0, q), bit)); });
-      a0 = n0 > 0 ? __fdiv_rn(p, (float)n0) : 0.f;
+      mu = (mw - a0 * z0) * kInvGroup;
+      a0 = n0 > 0 ? (mw0 - mu * z0) / n0 : 0.f;
     }
     off[b] = __float2half_rn(mu);
     s1[b] = __float2half_rn(a0);
@@ -432,6 +434,15 @@ __device__ __forceinline__ void plane1_blocks(int cta, int ctas, uint32_t *sx, i
 // (the last n with rowptr[n] <= j) and group (the (j - rowptr[n])-th set
 // salience bit of the row), then both supports, the refinement of mu,
 // alpha0 and alpha1, and both planes' bytes and parameters.
+//
+// The refinement decides nothing (the supports are fixed), so it runs on
+// the block's moments: with n0 = |T0|, n1 = |T1|, s0 = sum T0, s1 = sum T1,
+// s01 = sum T0 T1 and the sums w, w T0, w T1, a sweep is
+//   mu = (sum w - alpha0 s0 - alpha1 s1) / 128,
+//   alpha0 = (sum w T0 - mu s0 - alpha1 s01) / n0,
+//   alpha1 = (sum w T1 - mu s1 - alpha0 s01) / n1,
+// the exact coordinate updates of the least-squares fit, without a pass
+// over the weights.  Supports and thresholds keep the in-order sums.
 __device__ __forceinline__ void plane2_blocks(int cta, int ctas, uint32_t *sx, int N, int K, int sweeps,
                                               int64_t nnz, const uint16_t *W, const float4 *stats,
                                               const uint32_t *sal, const int32_t *rowptr, uint8_t *plane1,
@@ -468,39 +479,30 @@ __device__ __forceinline__ void plane2_blocks(int cta, int ctas, uint32_t *sx, i
     float mu = st.x, a0 = st.z, a1 = 0.f;
     uint32_t nz0[4] = {0u, 0u, 0u, 0u}, ng0[4] = {0u, 0u, 0u, 0u};
     uint32_t nz1[4] = {0u, 0u, 0u, 0u}, ng1[4] = {0u, 0u, 0u, 0u};
-    const int n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, st.y, nz0, ng0);
+    float mw = 0.f, mw0 = 0.f, mw1 = 0.f;  // sum w, sum w T0, sum w T1
+    const int n0 = support(B, [&](int, int, float x) { return __fsub_rn(x, mu); }, st.y, nz0, ng0,
+                           [&](float x, int t) { mw += x, mw0 += t > 0 ? x : (t < 0 ? -x : 0.f); });
     auto t0a = [&](float a, int q, int bit) { return times_bit(a, pick4(nz0, q), pick4(ng0, q), bit); };
-    auto t1a = [&](float a, int q, int bit) { return times_bit(a, pick4(nz1, q), pick4(ng1, q), bit); };
     // second support on the residual r = c - alpha0 T0, same threshold rule
     auto resid = [&](int q, int bit, float x) { return __fsub_rn(__fsub_rn(x, mu), t0a(a0, q, bit)); };
     float bsum = 0.f;
     B.each([&](int q, int bit, float x) { bsum = __fadd_rn(bsum, fabsf(resid(q, bit, x))); });
     const float d1 = __fmul_rn(kThresh, __fmul_rn(bsum, kInvGroup));
-    const int n1 = support(B, resid, d1, nz1, ng1);
-    {
-      float qs = 0.f;
-      B.each([&](int q, int bit, float x) { qs = __fadd_rn(qs, t1a(resid(q, bit, x), q, bit)); });
-      a1 = n1 > 0 ? __fdiv_rn(qs, (float)n1) : 0.f;
+    const int n1 = support(B, resid, d1, nz1, ng1,
+                           [&](float x, int t) { mw1 += t > 0 ? x : (t < 0 ? -x : 0.f); });
+    const int z0 = n0 - 2 * popc4(ng0), z1 = n1 - 2 * popc4(ng1);  // sum T0, sum T1
+    int z01 = 0;  // sum T0 T1: +1 where both are nonzero with equal signs, -1 with opposite signs
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t both = nz0[k] & nz1[k], opp = ng0[k] ^ ng1[k];
+      z01 += __popc(both & ~opp) - __popc(both & opp);
     }
-    // alternating refinement, supports fixed: mu, then alpha0, then alpha1
+    // alpha1 = sum r T1 / n1 with r = w - mu - alpha0 T0
+    a1 = n1 > 0 ? (mw1 - mu * z1 - a0 * z01) / n1 : 0.f;
     for (int sw = 0; sw < sweeps; ++sw) {
-      float u = 0.f;
-      B.each([&](int q, int bit, float x) {
-        u = __fadd_rn(u, __fsub_rn(__fsub_rn(x, t0a(a0, q, bit)), t1a(a1, q, bit)));
-      });
-      mu = __fmul_rn(u, kInvGroup);
-      float p = 0.f;
-      B.each([&](int q, int bit, float x) {
-        p = __fadd_rn(p, t0a(__fsub_rn(__fsub_rn(x, mu), t1a(a1, q, bit)), q, bit));
-      });
-      a0 = n0 > 0 ? __fdiv_rn(p, (float)n0) : 0.f;
-      if (n1 > 0) {
-        float qs = 0.f;
-        B.each([&](int q, int bit, float x) {
-          qs = __fadd_rn(qs, t1a(__fsub_rn(__fsub_rn(x, mu), t0a(a0, q, bit)), q, bit));
-        });
-        a1 = __fdiv_rn(qs, (float)n1);
-      }
+      mu = (mw - a0 * z0 - a1 * z1) * kInvGroup;
+      a0 = n0 > 0 ? (mw0 - mu * z0 - a1 * z01) / n0 : 0.f;
+      if (n1 > 0) a1 = (mw1 - mu * z1 - a0 * z01) / n1;
     }
     off[b] = __float2half_rn(mu);
     s1[b] = __float2half_rn(a0);
