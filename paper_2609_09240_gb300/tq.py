@@ -421,6 +421,30 @@ def container_read(data, expected=None, device=None, index=True):
     return out
 
 
+def convert(weights, salient_fraction: float = 0.1, sweeps: int = 4, stream=None):
+    """The paper's conversion pipeline from E2M-ATQ to serialization, for a
+    dict {name: fp16 [N][K] device tensor}: each projection ternarized
+    (round(salient_fraction * N * K / 128) salient groups), its provenance
+    checked (it must differ from the source), and all of them written into
+    one container, each with its source's FNV-1a 64 fingerprint.  Returns
+    (container bytes as a uint8 array, {name: provenance report})."""
+    entries, reports = [], {}
+    for name, W in weights.items():
+        N, K = W.shape
+        st = torch.zeros(1, dtype=torch.int32, device=W.device)
+        pw = ternarize(W, int(round(salient_fraction * N * K / TQ_GROUP)), sweeps=sweeps, d_status=st,
+                       stream=stream, index=False)
+        rep = provenance(W, pw, stream=stream)
+        status = int(st.item())
+        if status:
+            raise TQError(-4, f"tq_ternarize {name}: data status {status:#x}")
+        if rep["identical"]:
+            raise TQError(-4, f"{name}: the packed weight reproduces its source exactly (not ternarized)")
+        reports[name] = rep
+        entries.append((name, pw, fnv1a64(W)))
+    return container_write(entries), reports
+
+
 def tq_workspace_bytes(M: int, N: int, K: int) -> int:
     return int(lib().tq_workspace_bytes(M, N, K))
 

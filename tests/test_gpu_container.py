@@ -96,3 +96,20 @@ def test_container_round_trip_to_device():
     y2 = tq.tq_linear_f32out(x, pw2)
     H.device_status_ok()
     torch.testing.assert_close(y1, y2, rtol=1e-5, atol=1e-5)
+
+
+def test_convert_pipeline():
+    """tq.convert: ternarize, provenance and container for a small model;
+    reading it back with the expected keys gives the same packed weights."""
+    from paper_2609_09240_gb300 import tq
+    shapes = {"layers.0.q": (256, 512), "layers.0.down": (128, 1024), "layers.1.k": (64, 512)}
+    Ws = {n: torch.from_numpy(wl.gen_dense_weights(N, K, config=10, proj=i).view(np.float16)).cuda()
+          for i, (n, (N, K)) in enumerate(shapes.items())}
+    buf, reps = tq.convert(Ws)
+    assert set(reps) == set(shapes) and all(0.1 < r["rel_rmse"] < 0.9 for r in reps.values())
+    out = tq.container_read(buf.tobytes(), expected=list(shapes), device="cuda", index=False)
+    for n, W in Ws.items():
+        pw, h = out[n]
+        assert h == tq.fnv1a64(W)
+        ref = tq.ternarize(W, pw.nnz, index=False)
+        assert torch.equal(ref.plane1, pw.plane1) and torch.equal(ref.salience, pw.salience)
