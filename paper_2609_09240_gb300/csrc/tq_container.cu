@@ -159,7 +159,8 @@ tq_status open_buf(const void *buf, size_t bytes, Header *hdr, const Entry **tab
 // ------------------------------------------------------------ dequantize
 // W-hat[n][k] = fp16((s1 * t1 + off) + s2 * t2) in float32 (paper "Model and
 // Representation", eq. for W-hat, per group): one thread per (row, group),
-// 128 outputs as 16 16-byte stores.
+// 128 outputs as 16 16-byte stores.  status may be null (the prefill path's
+// trusted weights): nothing is then reported.
 __global__ void __launch_bounds__(128) dequantize_kernel(int N, int K, const uint8_t *plane1, const uint32_t *sal,
                                                          const int32_t *rowptr, const uint8_t *plane2, int64_t nnz,
                                                          const __half *s1, const __half *off, const __half *s2,
@@ -177,7 +178,7 @@ __global__ void __launch_bounds__(128) dequantize_kernel(int N, int K, const uin
       rank += __popc(srow[g >> 5] & ((1u << (g & 31)) - 1u));
       rec = (int64_t)rowptr[n] + rank;
       if (rec < 0 || rec >= nnz) {
-        atomicOr(status, TQ_DATA_BAD_ROWPTR);
+        if (status) atomicOr(status, TQ_DATA_BAD_ROWPTR);
         rec = -1;
       }
     }
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(128) dequantize_kernel(int N, int K, const uin
         const int k = 8 * c + e, j = k / 5, q = k - 5 * (k / 5);
         const uint32_t p3 = q == 0 ? 1u : q == 1 ? 3u : q == 2 ? 9u : q == 3 ? 27u : 81u;
         const uint32_t v1 = g1[j], v2 = g2 ? g2[j] : 121u;  // 121: five digits 1 (zero trits)
-        if (v1 > 242 || v2 > 242) atomicOr(status, TQ_DATA_BAD_BYTE);
+        if (status && (v1 > 242 || v2 > 242)) atomicOr(status, TQ_DATA_BAD_BYTE);
         const int t1 = (int)((v1 / p3) % 3u) - 1, t2 = (int)((v2 / p3) % 3u) - 1;
         float w = __fadd_rn(t1 > 0 ? a1 : (t1 < 0 ? -a1 : 0.f), o);
         w = __fadd_rn(w, t2 > 0 ? a2 : (t2 < 0 ? -a2 : 0.f));
