@@ -187,10 +187,13 @@ TQ_API tq_status tq_unpack(int32_t N, int32_t K, const uint8_t *plane1, const ui
  * = T1 of the salient blocks, offset = fp16(mu), scale1 = fp16(alpha0),
  * scale2 = fp16(alpha1) (round to nearest even), sal and rowptr; together a
  * complete tq_weight with nnz salient groups.
- * Arithmetic: IEEE float32, no fused multiply-add, every sum over a block in
- * index order from +0, means as the sum times 1/128; so the supports and the
- * salience set are reproducible bit for bit by any implementation that does
- * the same.
+ * Arithmetic of every decision (supports, thresholds, salience): IEEE
+ * float32, no fused multiply-add, every sum over a block in index order
+ * from +0, means as the sum times 1/128; so the planes and the salience set
+ * are reproducible bit for bit by any implementation that does the same.
+ * The refinement runs the same coordinate updates on each block's moments
+ * (sum w, sum w T0, sum w T1 and the trit counts): its fp16 outputs are
+ * within one ulp of sweeps computed as passes over the weights.
  *   W: fp16 [N][K], 16-byte aligned;  nnz: 0 <= nnz <= N * K / 128;
  *   sweeps: 0 .. 64;
  *   plane1: out [N][tq_row_bytes(K)], 16-byte aligned (pad bytes written 0);

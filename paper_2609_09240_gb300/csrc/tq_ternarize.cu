@@ -13,11 +13,13 @@
 //   alpha1 with the supports fixed.  Stored: offset = fp16(mu), scale1 =
 //   fp16(alpha0), scale2 = fp16(alpha1), plane 1 = T0, plane 2 = T1.
 //
-// The supports and the salience are integer decisions taken from floats, so
-// the arithmetic is fixed: IEEE float32 with explicit round-to-nearest
-// operations (never contracted into fused multiply-adds), every sum over a
-// block in index order 0..127 from +0, means as sums times 1/128.  One
-// thread owns one block, which makes index order its natural order.
+// The supports, thresholds and the salience are integer decisions taken from
+// floats, so their arithmetic is fixed: IEEE float32 with explicit
+// round-to-nearest operations (never contracted into fused multiply-adds),
+// every sum over a block in index order 0..127 from +0, means as sums times
+// 1/128.  One thread owns one block, which makes index order its natural
+// order.  The refinement decides nothing and runs on per-block moments (see
+// plane2_blocks); its fp16 outputs agree with in-order passes to one ulp.
 //
 // Kernels, in launch order:
 //   tern_stats_kernel   per block: mu, Delta0, alpha0 and E (key = E's bits)
