@@ -55,6 +55,24 @@ def measured_tensor_peak():
     return 1700.0, "fallback sustained"
 
 
+def max_over_ranks(value: float, pg, device) -> float:
+    """The largest of every rank's value (the job's time is its slowest
+    rank's); the value itself without a process group."""
+    if pg is None:
+        return float(value)
+    import torch
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, ms: float, scale: float = 1e9) -> float:
+    """Units all ranks processed per second (divided by `scale`), over the
+    slowest rank's time `ms`: each of `world` replicas does the same work."""
+    return world * units_per_rank / (ms * 1e-3) / scale
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -607,12 +625,9 @@ def main():
         clk.mark()
     total_ms = t0.elapsed_time(t1)
     launch_ms = [a.elapsed_time(b) for a, b in ev]
-    if pg:
-        t = torch.tensor([total_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, pg, dev)
     ms_per_step = total_ms / args.steps
-    value = ws * packed_bytes / (ms_per_step * 1e-3) / 1e9
+    value = whole_job_rate(packed_bytes, ws, ms_per_step)
     launch_avg = float(np.mean(launch_ms))
 
     # end to end through the C ABI with host buffers: per step, H2D of every
@@ -638,11 +653,8 @@ def main():
     e1.record(stream)
     barrier()
     e2e_ms = e0.elapsed_time(e1) / args.steps
-    if pg:
-        t = torch.tensor([e2e_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = ws * packed_bytes / (e2e_ms * 1e-3) / 1e9
+    e2e_ms = max_over_ranks(e2e_ms, pg, dev)
+    e2e_value = whole_job_rate(packed_bytes, ws, e2e_ms)
 
     peak, peak_kind = measured_peaks()
     achieved = packed_bytes / (launch_avg * 1e-3) / 1e9
