@@ -361,6 +361,14 @@ TQ_API tq_status tq_linear_static(int32_t M, int32_t N, int32_t K, const tq_weig
  * device of the current context; clear != 0 resets it to 0 afterwards. */
 TQ_API tq_status tq_get_device_status(uint32_t *status_host, int clear);
 
+/* Self-test of the failure path: one kernel makes a bounded wait on a
+ * barrier phase that nothing completes.  After its limit (about 2 s) the
+ * wait gives up, sets bit 0 of the device status word (as any wait of the
+ * library's kernels would) and the kernel returns, writing 0 to
+ * *result (device int32; 1 would mean the phase completed).  The context
+ * stays usable.  Asynchronous on stream. */
+TQ_API tq_status tq_wait_selftest(int32_t *result, void *stream);
+
 /* Human-readable name of a status code (static string). */
 TQ_API const char *tq_status_str(tq_status s);
 

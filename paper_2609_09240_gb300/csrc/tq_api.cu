@@ -31,6 +31,8 @@ cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int s
                              uint32_t *sal, int32_t *rowptr, uint8_t *plane2, uint16_t *scale1, uint16_t *offset,
                              uint16_t *scale2, unsigned char *ws, uint32_t *status, cudaStream_t s);
 cudaError_t read_status_prefill(uint32_t *out, bool clear);
+cudaError_t read_status_selftest(uint32_t *out, bool clear);
+cudaError_t launch_wait_selftest(int32_t *result, cudaStream_t s);
 }  // namespace tq
 
 using namespace tq;
@@ -331,11 +333,18 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {
   if (!status_host) return TQ_ERR_NULL;
-  uint32_t b = 0, c = 0;
+  uint32_t b = 0, c = 0, d = 0;
   if (read_status_gemv_mma(&b, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
   if (read_status_prefill(&c, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
-  *status_host = b | c;
+  if (read_status_selftest(&d, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  *status_host = b | c | d;
   return TQ_OK;
+}
+
+tq_status tq_wait_selftest(int32_t *result, void *stream) {
+  if (!result) return TQ_ERR_NULL;
+  if ((uintptr_t)result & 3u) return TQ_ERR_ALIGN;
+  return from_cuda(launch_wait_selftest(result, (cudaStream_t)stream));
 }
 
 const char *tq_status_str(tq_status s) {

@@ -124,6 +124,8 @@ def lib():
             L.tq_container_check_keys.restype = ctypes.c_int
             L.tq_container_check_keys.argtypes = [vp, sz, i32, ctypes.POINTER(ctypes.c_char_p),
                                                   ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32)]
+            L.tq_wait_selftest.restype = ctypes.c_int
+            L.tq_wait_selftest.argtypes = [vp, vp]
             L.tq_get_device_status.restype = ctypes.c_int
             L.tq_get_device_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int]
             L.tq_status_str.restype = ctypes.c_char_p
