@@ -265,3 +265,41 @@ def test_threshold_factor_boundary(second):
     for i, (t0, t1) in enumerate(want):
         assert np.array_equal(r["T1"].reshape(8, 128)[i], t0), i
         assert np.array_equal(r["T2"].reshape(8, 128)[i], t1), i
+
+
+def test_moment_form_of_the_sweeps():
+    """The GPU runs each refinement sweep on seven moments of the block (n0,
+    n1, sum T0, sum T1, sum T0 T1, sum w, sum w T0, sum w T1) instead of
+    passes over the weights.  In float64 the two forms are the same
+    coordinate updates: they agree to rounding on every block, salient or not."""
+    W = wl.gen_dense_weights(12, 1024, proj=13)
+    r = tz.ternarize(W, nnz=25, sweeps=0)
+    w = W.view(np.float16).astype(np.float64).reshape(-1, 128)
+    T0 = r["T1"].reshape(-1, 128).astype(np.float64)
+    T1 = r["T2"].reshape(-1, 128).astype(np.float64)
+    mu = r["mu"].ravel().astype(np.float64)
+    a0 = r["alpha0"].ravel().astype(np.float64)
+    a1 = r["alpha1"].ravel().astype(np.float64)
+    n0, n1 = np.abs(T0).sum(1), np.abs(T1).sum(1)
+    safe = lambda v, n: np.where(n > 0, v / np.maximum(n, 1), 0.0)
+    # passes over the weights (the oracle's order of updates)
+    pm, p0, p1 = mu.copy(), a0.copy(), a1.copy()
+    # moments
+    z0, z1, z01 = T0.sum(1), T1.sum(1), (T0 * T1).sum(1)
+    sw, sw0, sw1 = w.sum(1), (w * T0).sum(1), (w * T1).sum(1)
+    mm, m0, m1 = mu.copy(), a0.copy(), a1.copy()
+    # the second plane's first scale: least squares of r = w - mu - alpha0 T0 on T1
+    r_first = safe(((w - mu[:, None] - a0[:, None] * T0) * T1).sum(1), n1)
+    np.testing.assert_allclose(safe(sw1 - mu * z1 - a0 * z01, n1), r_first, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(r_first, a1, rtol=1e-5, atol=1e-9)  # the oracle's float32 value
+    for _ in range(4):
+        pm = (w - p0[:, None] * T0 - p1[:, None] * T1).mean(1)
+        p0 = safe(((w - pm[:, None] - p1[:, None] * T1) * T0).sum(1), n0)
+        p1 = safe(((w - pm[:, None] - p0[:, None] * T0) * T1).sum(1), n1)
+        mm = (sw - m0 * z0 - m1 * z1) / 128
+        m0 = safe(sw0 - mm * z0 - m1 * z01, n0)
+        m1 = safe(sw1 - mm * z1 - m0 * z01, n1)
+    assert r["salient"].sum() == 25
+    np.testing.assert_allclose(mm, pm, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(m0, p0, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(m1, p1, rtol=1e-12, atol=1e-15)
