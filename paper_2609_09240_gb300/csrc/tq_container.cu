@@ -8,7 +8,8 @@
 // no malformed packed tensors.  The container stores each projection's seven
 // packed fields under a name, with a hash per field and an optional
 // fingerprint of the fp16 source weights; reading an entry re-checks the
-// hashes, the shapes, rowptr against the salience map and every packed byte.
+// hashes (and that the fields' alignment padding is zero), the shapes, rowptr
+// against the salience map and every packed byte.
 //
 // Layout (little-endian; offsets from the start of the buffer):
 //   0   char     magic[8] = "TQPACK01"
@@ -331,6 +332,11 @@ tq_status tq_container_entry(const void *buf, size_t bytes, int32_t index, tq_ho
         sz[f] > bytes - e.f[f].off)
       return TQ_ERR_FORMAT;
     if (fnv1a(b + e.f[f].off, sz[f]) != e.f[f].hash) return TQ_ERR_FORMAT;
+    // the field's alignment padding (up to 15 bytes) is zero, so that no
+    // byte of the data region escapes a check
+    const uint64_t end = e.f[f].off + sz[f], pend = up16(end) < bytes ? up16(end) : bytes;
+    for (uint64_t i = end; i < pend; ++i)
+      if (b[i]) return TQ_ERR_FORMAT;
   }
   if (tq_status s = check_content(e, b)) return s;
   out->name = e.name;

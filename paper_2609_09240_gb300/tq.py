@@ -423,6 +423,25 @@ def container_read(data, expected=None, device=None, index=True):
     return out
 
 
+def save_container(path, entries) -> int:
+    """container_write(entries) into the file at `path` (written to a
+    temporary name, then renamed, so a reader never sees a partial file).
+    Returns the bytes written."""
+    buf = container_write(entries)
+    tmp = f"{path}.tmp{os.getpid()}"
+    with open(tmp, "wb") as f:
+        f.write(buf.tobytes())
+    os.replace(tmp, path)
+    return buf.nbytes
+
+
+def load_container(path, expected=None, device=None, index=True):
+    """container_read of the file at `path` (every check of the reader applies)."""
+    with open(path, "rb") as f:
+        data = f.read()
+    return container_read(data, expected=expected, device=device, index=index)
+
+
 def convert(weights, salient_fraction: float = 0.1, sweeps: int = 4, stream=None):
     """The paper's conversion pipeline from E2M-ATQ to serialization, for a
     dict {name: fp16 [N][K] device tensor}: each projection ternarized

@@ -90,8 +90,9 @@ def test_empty_container(tq):
 
 
 def test_every_corrupted_byte_region_is_detected(tq):
-    """A flipped bit in the header, the table or any field of any entry makes
-    reading fail (hash mismatch); a truncated or extended buffer too."""
+    """A flipped bit in the header, the table, any field of any entry or the
+    alignment padding between fields makes reading fail (hash mismatch or
+    nonzero padding); a truncated or extended buffer too."""
     ws, buf = build(tq)
     rng = np.random.default_rng(0)
     # header and table
@@ -111,8 +112,7 @@ def test_every_corrupted_byte_region_is_detected(tq):
         except tq.TQError as e:
             assert e.code == tq.TQ_ERR_FORMAT
         else:
-            # only alignment padding between fields is not covered by a hash
-            assert not _inside_field(buf, pos), pos
+            raise AssertionError(f"a flipped bit at {pos} ({'field' if _inside_field(buf, pos) else 'padding'}) went unnoticed")
     for n in (buf.nbytes - 1, buf.nbytes + 16):
         cut = np.zeros(n, np.uint8)
         cut[:min(n, buf.nbytes)] = buf[:min(n, buf.nbytes)]
@@ -163,3 +163,20 @@ def test_write_rejects_inconsistent_shapes(tq):
     f["nnz"] = 9  # more than N * G
     with pytest.raises(tq.TQError):
         tq.container_write([("w", f, 0)])
+
+
+def test_file_round_trip(tq, tmp_path):
+    """A container saved to a file and loaded back with the key check."""
+    ws, buf = build(tq)
+    path = tmp_path / "model.tqpack"
+    n = tq.save_container(str(path), ws)
+    assert n == buf.nbytes == path.stat().st_size
+    out = tq.load_container(str(path), expected=[e[0] for e in ENTRIES])
+    for name, f, h in ws:
+        g, gh = out[name]
+        assert gh == h and np.array_equal(g["plane1"], f["plane1"])
+    data = bytearray(path.read_bytes())
+    data[-3] ^= 0xFF  # inside the last entry's last field
+    path.write_bytes(bytes(data))
+    with pytest.raises(tq.TQError):
+        tq.load_container(str(path))
