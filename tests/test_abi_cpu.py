@@ -81,3 +81,25 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_plane2_index_bytes(100, 4096, 100 * 32 + 1) == 0  # more records than groups
     assert L.tq_plane2_index_bytes(100, 4000, 13) == 0  # K not a multiple of 128
     assert tq.tq_workspace_bytes(1, 0, 4096) == 0
+
+
+def test_binding_argument_counts_match_the_header():
+    """Every function the ctypes binding declares takes as many arguments as
+    its prototype in include/tq.h."""
+    import os
+    import re
+
+    from paper_2609_09240_gb300 import tq
+    L = tq.lib()
+    text = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "tq.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    protos = dict(re.findall(r"TQ_API\s+[\w\s\*]*?\b(tq_\w+)\s*\(([^)]*)\)", text))
+    checked = 0
+    for name, params in protos.items():
+        fn = getattr(L, name)
+        if fn.argtypes is None:
+            continue
+        n = 0 if params.strip() in ("", "void") else params.count(",") + 1
+        assert len(fn.argtypes) == n, (name, len(fn.argtypes), n)
+        checked += 1
+    assert checked >= 25
