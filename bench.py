@@ -181,10 +181,13 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- workload
-def build_step(M, device, seed0=0, layers=None):
+def build_step(M, device, seed0=0, layers=None, on_codes=None):
     """Pack the 252 projections of the Qwen3-8B step on the device.  Every
     projection's activations and outputs are views of one contiguous x / y
     buffer (so a step's inputs move host<->device in one copy each).
+    on_codes(projection, drawn tensors, packed weight), if given, sees each
+    projection's drawn codes and parameters before they are freed (the
+    full-size parity test packs them again with the oracle).
     Returns (items, x_all, y_all, packed_bytes, weights)."""
     import torch
 
@@ -201,6 +204,8 @@ def build_step(M, device, seed0=0, layers=None):
         seed = seed0 * 100003 + p.layer * 16 + p.proj
         g = wl.gen_weights_torch(p.N, p.K, 0.1, device, seed)
         pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+        if on_codes is not None:
+            on_codes(p, g, pw)
         del g
         x = x_all[xo:xo + M * p.K].view(M, p.K)
         x.copy_(wl.gen_x_torch(M, p.K, device, seed + 7))
@@ -315,6 +320,8 @@ def run_prefill(args, ws, rank, local):
     for p in wl.config_projections(4):
         g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 500 + p.proj)
         pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+        if on_codes is not None:
+            on_codes(p, g, pw)
         del g
         x = wl.gen_x_torch(M, p.K, dev, 600 + p.proj)
         y = torch.empty((M, p.N), dtype=torch.float16, device=dev)

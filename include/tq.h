@@ -295,7 +295,11 @@ TQ_API size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K);
  *   256-byte aligned; its contents are overwritten; calls that share a
  *   workspace must not overlap in time.
  * The packed bytes are trusted (produced by tq_pack): no per-byte
- * validation on this path. */
+ * validation on this path.
+ * Host threads: the linear entry points (tq_linear, tq_linear_f32out,
+ * tq_linear_batched, tq_linear_static) keep their launch parameters per
+ * host thread, so several threads may call them at once (each with its own
+ * workspace; tq_linear_static's one scratch array is the exception). */
 TQ_API tq_status tq_linear(int32_t M, int32_t N, int32_t K, const tq_weight *w, const uint16_t *x,
                            uint16_t *y, void *workspace, size_t workspace_bytes, void *stream);
 
@@ -342,7 +346,10 @@ TQ_API tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *p
  *   - Set-up: the first call on a device looks up the scratch array's device
  *     address once (cudaGetSymbolAddress) and caches it for that device; make
  *     that first call before any stream capture on the device.  A failed
- *     lookup returns TQ_ERR_CUDA.
+ *     lookup returns TQ_ERR_CUDA.  The cached address belongs to the
+ *     device's context at the time of the lookup: after cudaDeviceReset (or
+ *     any other teardown of that context) it is stale, and this entry point
+ *     must not be called on that device again in the same process.
  *   - Nothing in the scratch has to start at zero: every call writes all of
  *     the scratch it reads before reading it.
  *   - There is ONE scratch array per device: calls on the same device that

@@ -176,7 +176,9 @@ tq_status linear_impl(int32_t M, int32_t N, int32_t K, const tq_weight *w, const
     const Problem P = to_problem(w, x, y);
     return from_cuda(launch_prefill(P, M, f32, s));
   }
-  static BatchParams bp;  // large; filled per call (host-side, not thread-safe across calls)
+  // large (kept off the stack) and per host thread, so that calls from
+  // several threads never share launch parameters
+  thread_local BatchParams bp;
   bp.count = 1;
   bp.M = M;
   bp.out_f32 = f32 ? 1 : 0;
@@ -316,7 +318,7 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
   if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
   if (!problems || !workspace) return TQ_ERR_NULL;
   if ((uintptr_t)workspace & 255u) return TQ_ERR_ALIGN;
-  static BatchParams bp;
+  thread_local BatchParams bp;  // per host thread, as in linear_impl
   bp.count = count;
   bp.M = M;
   bp.out_f32 = 0;

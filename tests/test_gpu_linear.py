@@ -189,3 +189,47 @@ def test_second_plane_scale2_two_byte_aligned(H, M, index):
     y = tq.tq_linear_f32out(H.dev(x), pw)
     H.device_status_ok()
     H.assert_close(y.cpu().numpy(), y_ref, a_ref)
+
+
+def test_two_host_threads(H):
+    """tq_linear from two host threads at once, different shapes and token
+    counts, each on its own stream and workspace: launch parameters are kept
+    per host thread, so neither call ever runs with the other's sizes or
+    pointers.  Every result of 40 calls per thread matches the oracle."""
+    import threading
+
+    from paper_2609_09240_gb300 import tq
+    cases = [(1, 1024, 4096, 0.1, 11), (5, 300, 2560, 0.2, 12)]
+    prepared = []
+    for M, N, K, frac, proj in cases:
+        w = wl.gen_weights(N, K, frac, config=6, proj=proj)
+        xb = wl.gen_x(M, K, config=6, proj=proj)
+        y_ref, a_ref = H.oracle_ref(w, xb)
+        prepared.append((H.pack_on_gpu(w), H.dev(xb), y_ref, a_ref))
+    torch.cuda.synchronize()
+    results = [[], []]
+    errors = []
+
+    def worker(i):
+        try:
+            pw, x, _, _ = prepared[i]
+            s = torch.cuda.Stream()
+            ws = tq.workspace(tq.tq_workspace_bytes(x.shape[0], pw.N, pw.K), x.device)
+            with torch.cuda.stream(s):
+                for _ in range(40):
+                    results[i].append(tq.tq_linear(x, pw, ws=ws, stream=s).clone())
+            s.synchronize()
+        except Exception as e:  # reported on the main thread
+            errors.append(e)
+
+    th = [threading.Thread(target=worker, args=(i,)) for i in range(2)]
+    for t in th:
+        t.start()
+    for t in th:
+        t.join()
+    assert not errors, errors
+    H.device_status_ok()
+    for i, (_, _, y_ref, a_ref) in enumerate(prepared):
+        assert len(results[i]) == 40
+        for y in results[i]:
+            H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)

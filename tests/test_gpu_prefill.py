@@ -40,14 +40,20 @@ def test_prefill_small(H, M, N, K, frac, f32):
     H.assert_close(y, y_ref, a_ref)
 
 
-@pytest.mark.parametrize("name,N,K,nrows", [("k", 1024, 4096, 48), ("down", 4096, 12288, 24)])
+PROJ = {"q": 0, "k": 1, "v": 2, "o": 3, "gate": 4, "up": 5, "down": 6}
+
+
+@pytest.mark.parametrize("name,N,K,nrows", [("k", 1024, 4096, 48), ("down", 4096, 12288, 24),
+                                            ("q", 4096, 4096, 32), ("gate", 12288, 4096, 48)])
 def test_prefill_qwen3_8b_shape_sampled_rows(H, name, N, K, nrows):
     """M = 2048 tokens through one Qwen3-8B projection shape; the oracle
-    checks a seeded sample of rows (every token) across all row tiles."""
+    checks a seeded sample of rows (every token) across all row tiles.  q
+    (as o: 4096 x 4096) and gate (as up: 12288 x 4096) run 256-row tiles
+    over more than one wave of SMs; k runs 128-row tiles."""
     from paper_2609_09240_gb300 import tq
     M = 2048
-    w = wl.gen_weights(N, K, 0.1, config=4, layer=0, proj=3 if name == "k" else 6)
-    xb = wl.gen_x(M, K, config=4, layer=0, proj=3 if name == "k" else 6)
+    w = wl.gen_weights(N, K, 0.1, config=4, layer=0, proj=PROJ[name])
+    xb = wl.gen_x(M, K, config=4, layer=0, proj=PROJ[name])
     pw = H.pack_on_gpu(w)
     y = tq.tq_linear(H.dev(xb), pw).float().cpu().numpy()
     H.device_status_ok()
