@@ -24,6 +24,8 @@ cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
+cudaError_t read_status_gemv_g4(uint32_t *out, bool clear);
+int64_t g4_workspace_bytes(int M, int K);
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
 size_t ternarize_ws_bytes(int N, int K);
 cudaError_t launch_dequantize(int N, int K, const tq_weight *w, uint16_t *out, uint32_t *status, cudaStream_t s);
@@ -96,7 +98,10 @@ size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
 size_t problem_ws_bytes(int M, int N, int K) {
   size_t b, cs, y2;
   mma_workspace_parts(M, N, K, &b, &cs, &y2);
-  return pad256(b) + pad256(cs) + pad256(y2) + 512;  // + the tensor maps of plane 1, s1, off
+  // + the tensor maps of plane 1, s1, off; with M <= 2 the operands of the
+  // one-group-per-lane kernel follow
+  const size_t g4 = M <= 2 ? (size_t)g4_workspace_bytes(M, K) : 0;
+  return pad256(b) + pad256(cs) + pad256(y2) + 512 + g4;
 }
 
 }  // namespace
@@ -335,11 +340,12 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {
   if (!status_host) return TQ_ERR_NULL;
-  uint32_t b = 0, c = 0, d = 0;
+  uint32_t b = 0, c = 0, d = 0, e = 0;
   if (read_status_gemv_mma(&b, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
+  if (read_status_gemv_g4(&e, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
   if (read_status_prefill(&c, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
   if (read_status_selftest(&d, clear != 0) != cudaSuccess) return TQ_ERR_CUDA;
-  *status_host = b | c | d;
+  *status_host = b | c | d | e;
   return TQ_OK;
 }
 

@@ -61,6 +61,7 @@
 #include <type_traits>
 
 #include "tq_common.cuh"
+#include "tq_decode_ops.cuh"
 #include "tq_sm100.cuh"
 
 namespace tq {
@@ -76,12 +77,6 @@ constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
 constexpr int kCSGroup = 64;             // C[8], S[8] floats per group and 8-token tile
 constexpr int kWarpsP1 = 8, kWarpProd = 8;
 constexpr int kThreads = 9 * 32;
-constexpr int kLutBytes = 65536;  // 256 byte values x 256 B (32 lanes x 4 B used)
-constexpr uint32_t kLutShared = 65536;  // shared-window address of the table
-constexpr uint32_t kDynShared = 1024;   // shared-window offset of dynamic smem
-constexpr int kDynBytes = 232448;       // whole opt-in shared memory of a CTA
-constexpr int kArena1 = (int)(kLutShared - kDynShared);   // below the table
-constexpr int kArena2 = kDynBytes - kArena1 - kLutBytes;  // above the table
 constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
 constexpr int kSOSlot = 2 * kRows * 16;                   // s1 then off, 16 B per row
 
@@ -120,58 +115,6 @@ struct Bars {
 struct Sched {
   int32_t cta_tile[257];
 };
-
-__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, volatile int32_t *abort_) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = global_ns();
-  for (uint32_t i = 1;; ++i) {
-    // sleep in the wait rather than spin: the waiting warps share the
-    // issue slots with the decoding warps
-    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
-    if ((i & 7u) == 0) {
-      if (*abort_) return false;
-      if (global_ns() - t0 > kWaitLimitNs) break;
-    }
-  }
-  atomicOr(&g_tq_device_status, kStatusTimeout);
-  *abort_ = 1;
-  return false;
-}
-
-// Table word of a byte value (see the file comment); invalid bytes
-// (243..255) map to the exponent pattern alone.
-__host__ __device__ __forceinline__ uint32_t lut_word(int v) {
-  uint32_t w = 0x44004400u;
-  if (v <= 242) {
-    const uint32_t d0 = v % 3, d1 = (v / 3) % 3, d2 = (v / 9) % 3, d3 = (v / 27) % 3;
-    w |= (d0 << 8) | (d2 << 6) | (d1 << 24) | (d3 << 22);
-  }
-  return w;
-}
-
-// The low (hi = false) or high fp16 of a word, as float.
-template <bool HI>
-__device__ __forceinline__ float half_of(uint32_t w) {
-  const __half2 h = *reinterpret_cast<const __half2 *>(&w);
-  return HI ? __high2float(h) : __low2float(h);
-}
-
-__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t s) {
-  uint32_t d;
-  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(s));
-  return d;
-}
-// The table is constant after set-up: an ordinary (reorderable) load.
-__device__ __forceinline__ uint32_t lut_load(uint32_t addr) {
-  uint32_t w;
-  asm("ld.shared.u32 %0, [%1];" : "=r"(w) : "r"(addr));
-  return w;
-}
-__device__ __forceinline__ uint32_t w_prime(uint32_t w) {
-  uint32_t d;
-  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(d) : "r"(w), "n"(0x00C000C0), "n"(0x4C004C00));
-  return d;
-}
 
 // Window of a group: the aligned words of the stage row that cover its 26
 // bytes, words wstart .. wstart + 6 with wstart = 26 GL / 4 (GL = the
@@ -226,37 +169,6 @@ __device__ __forceinline__ void decode_words_compact(uint32_t w0, uint32_t w1, c
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) a[16 + i] = 0x44004400u | v[2 * i] | (v[2 * i + 1] << 16);
-}
-
-// 16-byte asynchronous global -> shared copies (completion tracked per
-// thread in commit groups).
-__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// D += A * B, m16n8k16, fp16 in, fp32 accumulate.
-__device__ __forceinline__ void mma16816(float *d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-// D = A * B (zero accumulator in).
-__device__ __forceinline__ void mma16816_z(float *d, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
-                                           uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%10,%10,%10,%10};"
-      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.f));
 }
 
 // The MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
@@ -319,6 +231,48 @@ constexpr int kMapS1 = 128, kMapOff = 256, kCounterOff = 384;
 static_assert(kCounterOff + 4 <= kMapSlotBytes, "map slot");
 
 // ------------------------------------------------------------------ prep
+// Activation slots of one group for the one-group-per-lane kernel (M <= 2,
+// tq_gemv_g4.cu), for the lane that owns it: MMA j = 5 i + m of the lane's
+// 7 window words takes W, W' of window byte 4 i + m (m < 4) or the
+// fifth-slot words of window bytes 4 i .. 4 i + 3 (m = 4); window byte
+// beta is group byte beta - E (E = 2 for odd stage positions, whose window
+// starts two bytes before the group), and bytes outside the group get zero
+// activations.  dst: this (stage, token, group)'s 18 chunks, 64 B apart.
+template <int E>
+__device__ __forceinline__ void g4_write_slots(unsigned char *dst, const __half *ya, const __half *yb,
+                                               const __half *yc, const __half *yd, const __half *ye) {
+  auto pk = [](__half lo, __half hi) -> uint32_t {
+    __half2 v = __halves2half2(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+  };
+  const __half z = __float2half_rn(0.f);
+  auto yev = [&](int b) -> __half { return (b >= 0 && b < 26) ? ye[b] : z; };
+#pragma unroll
+  for (int jp = 0; jp < g4::kBPairs; ++jp) {
+    uint32_t w[4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int j = 2 * jp + h, i = j / 5, m = j % 5;
+      uint32_t b0 = 0u, b1 = 0u;
+      if (j < 35) {
+        if (m < 4) {
+          const int b = 4 * i + m - E;
+          if (b >= 0 && b < 26) {
+            b0 = pk(ya[b], yb[b]);
+            b1 = pk(yc[b], yd[b]);
+          }
+        } else {
+          b0 = pk(yev(4 * i - E), yev(4 * i + 1 - E));
+          b1 = pk(yev(4 * i + 2 - E), yev(4 * i + 3 - E));
+        }
+      }
+      w[2 * h] = b0;
+      w[2 * h + 1] = b1;
+    }
+    *reinterpret_cast<uint4 *>(dst + jp * 64) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 // B fragments, C and S for every (problem, group, token).  B layout of a
 // group: [token m][chunk pair cp][lane position c] x 16 B, each 16 B being
 // (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
@@ -360,8 +314,21 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   const int MB = bp.M;
   const int G = P.K / kGroup;
   const int task = blockIdx.x * blockDim.x + threadIdx.x;
-  if (task >= G * MB) return;
+  // with M <= 2 the one-group-per-lane kernel runs; its operands cover whole
+  // 4-group stages (groups past G get zero activations and C/S)
+  const int Gx = MB <= 2 ? g4::kStageG * g4::nstages(P.K) : G;
+  if (task >= Gx * MB) return;
   const int g = task / MB, m = task % MB;
+  unsigned char *g4b = P.wsB + P.map_off + kMapSlotBytes;
+  float *g4cs = reinterpret_cast<float *>(g4b + g4::pad256(g4::b_bytes(MB, P.K)));
+  unsigned char *g4dst = g4b + (int64_t)((g / g4::kStageG) * MB + m) * g4::kBTok + (g % g4::kStageG) * 16;
+  float *g4q = g4cs + 4 * g;  // (C0, C1, S0, S1) of group g
+  if (g >= G) {
+    for (int jp = 0; jp < g4::kBPairs; ++jp) *reinterpret_cast<uint4 *>(g4dst + jp * 64) = make_uint4(0u, 0u, 0u, 0u);
+    g4q[m] = g4q[2 + m] = 0.f;
+    if (MB == 1) g4q[1] = g4q[3] = 0.f;
+    return;
+  }
   const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
   // the group's 128 activations, all loads issued at once (x rows are
   // 16-byte aligned and groups are 256 bytes)
@@ -395,6 +362,15 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
     C += 5.25f * (fa + fb) + 17.f * (__half2float(yc[b]) + __half2float(yd[b])) +
          (4.f + 121.f / 256.f) * __half2float(ye[b]);
     S += x[0] + x[1] + x[2] + x[3] + x[4];
+  }
+  if (MB <= 2) {
+    if (g & 1)
+      g4_write_slots<2>(g4dst, ya, yb, yc, yd, ye);
+    else
+      g4_write_slots<0>(g4dst, ya, yb, yc, yd, ye);
+    g4q[m] = C;
+    g4q[2 + m] = S;
+    if (MB == 1) g4q[1] = g4q[3] = 0.f;
   }
   const int GL = g % kStageG;  // the group's index in its stage fixes its window
   unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
@@ -1431,6 +1407,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace mm
 
 // -------------------------------------------------------------- launcher
+cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s);
+
 static int num_sms_mm() {
   static int n = 0;
   if (n == 0) {
@@ -1457,8 +1435,9 @@ TQ_STATUS_ACCESSOR(read_status_gemv_mma)
 // Template tensor maps, encoded once per (kind, row length, rows) and cached:
 // kind 0 = plane 1 as a 2-D byte tensor of rows of `len` bytes (box 208 x 128
 // bytes); kind 1 = s1 / off as a 2-D fp16 tensor of rows of `len` halves (box
-// 8 x 128).  No swizzle, zero fill.  The prep kernel puts in each problem's
-// address.
+// 8 x 128); kinds 2 and 3 the same for the one-group-per-lane kernel of
+// M <= 2 (boxes 112 x 256 bytes and 8 x 256 halves).  No swizzle, zero fill.
+// The prep kernel puts in each problem's address.
 static bool map_template(int kind, int64_t len, const void *addr, int N, CUtensorMap *out) {
   // the driver's encoder, looked up through the runtime (no link-time
   // dependence on the driver library)
@@ -1475,7 +1454,7 @@ static bool map_template(int kind, int64_t len, const void *addr, int N, CUtenso
   static int64_t keys[64];
   static CUtensorMap maps[64];
   static int n = 0;
-  const int64_t key = ((int64_t)N << 32) | (len << 1) | kind;
+  const int64_t key = ((int64_t)N << 32) | (len << 2) | kind;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n; ++i)
     if (keys[i] == key) {
@@ -1483,12 +1462,15 @@ static bool map_template(int kind, int64_t len, const void *addr, int N, CUtenso
       return true;
     }
   CUtensorMap m;
-  const int esz = kind == 0 ? 1 : 2;
+  const bool halves = (kind & 1) != 0;
+  const int esz = halves ? 2 : 1;
   cuuint64_t dims[2] = {(cuuint64_t)len, (cuuint64_t)N};
   cuuint64_t strides[1] = {(cuuint64_t)(len * esz)};
-  cuuint32_t box[2] = {kind == 0 ? (cuuint32_t)mm::kStageBytes : (cuuint32_t)mm::kStageG, (cuuint32_t)mm::kRows};
+  const cuuint32_t box_rows = kind >= 2 ? (cuuint32_t)g4::kRows : (cuuint32_t)mm::kRows;
+  const cuuint32_t box_x = halves ? 8u : kind == 0 ? (cuuint32_t)mm::kStageBytes : 112u;
+  cuuint32_t box[2] = {box_x, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  if (encode(&m, kind == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(addr),
+  if (encode(&m, halves ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(addr),
              dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return false;
@@ -1584,12 +1566,14 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     tmax = max(tmax, (bp.prob[i].N + mm::kRows - 1) / mm::kRows);
     any2 = any2 || bp.prob[i].nnz > 0;
   }
+  // one or two tokens: the one-group-per-lane kernel (tq_gemv_g4.cu)
+  const bool g4path = bp.M <= 2;
   thread_local mm::MapTemplates mt;
   {
     int64_t keys[mm::kMaxMapTemplates] = {};
     int nt = 0;
     auto slot = [&](int kind, int64_t len, const void *addr, int N) -> int {
-      const int64_t key = ((int64_t)N << 32) | (len << 1) | kind;
+      const int64_t key = ((int64_t)N << 32) | (len << 2) | kind;
       int k = 0;
       while (k < nt && keys[k] != key) ++k;
       if (k == nt) {
@@ -1603,12 +1587,12 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     };
     for (int i = 0; i < bp.count; ++i) {
       const Problem &P = bp.prob[i];
-      const int k1 = slot(0, row_bytes_of(P.K), P.plane1, P.N);
+      const int k1 = slot(g4path ? 2 : 0, row_bytes_of(P.K), P.plane1, P.N);
       if (k1 < 0) return k1 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
       mt.idx[i] = (uint8_t)k1;
       mt.idx_so[i] = mm::kNoMap;
       if (scales_by_map(P)) {
-        const int k2 = slot(1, P.K / kGroup, P.s1, P.N);
+        const int k2 = slot(g4path ? 3 : 1, P.K / kGroup, P.s1, P.N);
         if (k2 < 0) return k2 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
         mt.idx_so[i] = (uint8_t)k2;
       }
@@ -1632,7 +1616,8 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     }
     counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + mm::kCounterOff);
   }
-  mm::gemv_mma_prep_kernel<<<dim3((gmax * bp.M + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
+  const int gtasks = (g4path ? g4::kStageG * ((gmax + g4::kStageG - 1) / g4::kStageG) : gmax) * bp.M;
+  mm::gemv_mma_prep_kernel<<<dim3((gtasks + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   // more than 8 tokens in one pass needs every second plane indexed (the
@@ -1658,6 +1643,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
+  if (g4path) return launch_gemv_g4(bp, num_sms_mm(), s);
   auto main_kern = bp.M == 1 ? mm::gemv_mma_kernel<F32, true, false>
                              : (bp.M > 8 ? mm::gemv_mma_kernel<F32, false, true> : mm::gemv_mma_kernel<F32, false, false>);
   e = cudaFuncSetAttribute(main_kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kDynBytes);

@@ -36,7 +36,7 @@ def test_config0_single_linear(H, M, f32):
 
 @pytest.mark.parametrize("N,K,frac", [(1, 128, 0.0), (1, 128, 1.0), (129, 256, 0.5), (200, 2560, 0.1),
                                       (77, 4224, 0.1), (300, 9728, 0.1), (128, 12288, 0.1)])
-@pytest.mark.parametrize("M", [1, 5, 16])
+@pytest.mark.parametrize("M", [1, 2, 5, 16])
 def test_ragged_shapes(H, N, K, frac, M):
     run_case(H, N, K, frac, M, f32=False, proj=N)
 
@@ -233,3 +233,31 @@ def test_two_host_threads(H):
         assert len(results[i]) == 40
         for y in results[i]:
             H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M", [1, 2])
+@pytest.mark.parametrize("f32", [False, True])
+def test_one_group_per_lane_stage_shapes(H, M, f32):
+    """The M <= 2 kernel's 4-group stages and 256-row tiles: group counts of
+    every residue mod 4 and mod 8 (scales by tensor copy only when G % 8 ==
+    0), tiles cut short by N, in one batch whose tiles straddle problems."""
+    from paper_2609_09240_gb300 import tq
+    shapes = [(257, 128 * 9), (511, 128 * 10), (256, 128 * 11), (300, 128 * 12), (1, 128 * 16), (640, 128 * 3),
+              (513, 128 * 6)]
+    items, refs = [], []
+    for i, (N, K) in enumerate(shapes):
+        w = wl.gen_weights(N, K, 0.15, config=6, proj=40 + i)
+        xb = wl.gen_x(M, K, config=6, proj=40 + i)
+        refs.append(H.oracle_ref(w, xb))
+        pw = H.pack_on_gpu(w, index=(i % 2 == 0))
+        x = H.dev(xb)
+        if f32:
+            y = tq.tq_linear_f32out(x, pw)
+            H.device_status_ok()
+            H.assert_close(y.cpu().numpy().astype(np.float64), *refs[-1])
+        items.append((pw, x, torch.full((M, N), float("nan"), dtype=torch.float16, device=x.device)))
+    if not f32:
+        tq.tq_linear_batched(tq.Batch(M, items))
+        H.device_status_ok()
+        for (pw, x, y), (y_ref, a_ref) in zip(items, refs):
+            H.assert_close(y.float().cpu().numpy().astype(np.float64), y_ref, a_ref)
