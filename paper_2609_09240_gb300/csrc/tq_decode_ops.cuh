@@ -113,20 +113,27 @@ __device__ __forceinline__ void mma16816_z(float *d, uint32_t a0, uint32_t a1, u
 }  // namespace mm
 
 // Operand layout of the one-group-per-lane decode kernel for M <= 2 tokens
-// (tq_gemv_g4.cu), written by the prep kernel: per problem, after the
-// general decode path's parts, the activation slots [stage][token][pair
-// jp < 18][group c < 4] x 16 B (MMAs 2 jp and 2 jp + 1 of the lane that
-// owns group c: b0, b1 of each) and then C/S [stage][group] x (C0, C1, S0,
-// S1) floats.  A stage is 4 groups.
+// (tq_gemv_g4.cu), written by the prep kernel.  A stage is SG groups of a
+// 256-row tile: SG = 8 for one token (lane c of a row owns groups 2c and
+// 2c + 1, the MMA's 8 columns are the stage's 8 groups), SG = 4 for two
+// tokens (lane c owns group c, columns 2c + t are its two tokens).  Each
+// stage has two activation-slot slices (the two groups of a lane, or its
+// two tokens): per slice, 16-byte chunks [pair jp][lane position c] holding
+// b0, b1 of the lane's MMAs 2 jp and 2 jp + 1; then per stage the C/S block
+// [c] x (C_a, C_b, S_a, S_b) floats of the two slices.  Per problem the
+// slots of all stages come first, then the C/S blocks.
 namespace g4 {
-constexpr int kRows = 256;       // tile rows
-constexpr int kStageG = 4;       // groups per stage
-constexpr int kBPairs = 18;      // 16-byte activation chunks per (stage, token, group)
-constexpr int kBTok = kBPairs * 64;
+constexpr int kRows = 256;  // tile rows
+__host__ __device__ constexpr int stage_groups(int M) { return M == 1 ? 8 : 4; }
+__host__ __device__ constexpr int words(int SG) { return SG == 8 ? 13 : 7; }  // window words per lane and row
+__host__ __device__ constexpr int pairs(int SG) { return (5 * words(SG) + 1) / 2; }  // 16-byte chunks per slice
+__host__ __device__ constexpr int slice_bytes(int SG) { return pairs(SG) * 64; }
 constexpr int kCSStage = 64;
-__host__ __device__ constexpr int nstages(int K) { return (K / kGroup + kStageG - 1) / kStageG; }
+__host__ __device__ constexpr int nstages(int K, int SG) { return (K / kGroup + SG - 1) / SG; }
 __host__ __device__ inline int64_t pad256(int64_t b) { return (b + 255) / 256 * 256; }
-__host__ __device__ inline int64_t b_bytes(int M, int K) { return (int64_t)nstages(K) * kBTok * M; }
-__host__ __device__ inline int64_t cs_bytes(int K) { return (int64_t)nstages(K) * kCSStage; }
+__host__ __device__ inline int64_t b_bytes(int M, int K) {
+  return (int64_t)nstages(K, stage_groups(M)) * 2 * slice_bytes(stage_groups(M));
+}
+__host__ __device__ inline int64_t cs_bytes(int M, int K) { return (int64_t)nstages(K, stage_groups(M)) * kCSStage; }
 }  // namespace g4
 }  // namespace tq

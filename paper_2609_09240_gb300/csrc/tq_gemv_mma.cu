@@ -232,13 +232,15 @@ static_assert(kCounterOff + 4 <= kMapSlotBytes, "map slot");
 
 // ------------------------------------------------------------------ prep
 // Activation slots of one group for the one-group-per-lane kernel (M <= 2,
-// tq_gemv_g4.cu), for the lane that owns it: MMA j = 5 i + m of the lane's
-// 7 window words takes W, W' of window byte 4 i + m (m < 4) or the
-// fifth-slot words of window bytes 4 i .. 4 i + 3 (m = 4); window byte
-// beta is group byte beta - E (E = 2 for odd stage positions, whose window
-// starts two bytes before the group), and bytes outside the group get zero
-// activations.  dst: this (stage, token, group)'s 18 chunks, 64 B apart.
-template <int E>
+// tq_gemv_g4.cu), in the slice of the lane that owns it: MMA j = 5 i + m of
+// the lane's window words takes W, W' of window byte 4 i + m (m < 4) or the
+// fifth-slot words of window bytes 4 i .. 4 i + 3 (m = 4).  Window byte beta
+// is group byte beta - OFFS (OFFS = 2 for the odd groups of a 4-group stage,
+// whose window starts two bytes before the group; 26 for the second group
+// of a lane in an 8-group stage); bytes outside the group get zero
+// activations.  dst: the slice's chunk of this lane position, chunks 64 B
+// apart.
+template <int SG, int OFFS>
 __device__ __forceinline__ void g4_write_slots(unsigned char *dst, const __half *ya, const __half *yb,
                                                const __half *yc, const __half *yd, const __half *ye) {
   auto pk = [](__half lo, __half hi) -> uint32_t {
@@ -248,22 +250,22 @@ __device__ __forceinline__ void g4_write_slots(unsigned char *dst, const __half 
   const __half z = __float2half_rn(0.f);
   auto yev = [&](int b) -> __half { return (b >= 0 && b < 26) ? ye[b] : z; };
 #pragma unroll
-  for (int jp = 0; jp < g4::kBPairs; ++jp) {
+  for (int jp = 0; jp < g4::pairs(SG); ++jp) {
     uint32_t w[4];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int j = 2 * jp + h, i = j / 5, m = j % 5;
       uint32_t b0 = 0u, b1 = 0u;
-      if (j < 35) {
+      if (j < 5 * g4::words(SG)) {
         if (m < 4) {
-          const int b = 4 * i + m - E;
+          const int b = 4 * i + m - OFFS;
           if (b >= 0 && b < 26) {
             b0 = pk(ya[b], yb[b]);
             b1 = pk(yc[b], yd[b]);
           }
         } else {
-          b0 = pk(yev(4 * i - E), yev(4 * i + 1 - E));
-          b1 = pk(yev(4 * i + 2 - E), yev(4 * i + 3 - E));
+          b0 = pk(yev(4 * i - OFFS), yev(4 * i + 1 - OFFS));
+          b1 = pk(yev(4 * i + 2 - OFFS), yev(4 * i + 3 - OFFS));
         }
       }
       w[2 * h] = b0;
@@ -273,9 +275,6 @@ __device__ __forceinline__ void g4_write_slots(unsigned char *dst, const __half 
   }
 }
 
-// B fragments, C and S for every (problem, group, token).  B layout of a
-// group: [token m][chunk pair cp][lane position c] x 16 B, each 16 B being
-// (B0, B1) of chunk 2cp then of chunk 2cp + 1 for that lane.
 __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ MapTemplates mt,
                                      int32_t *unit_counter) {
   const int p = blockIdx.y;
@@ -315,18 +314,22 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   const int G = P.K / kGroup;
   const int task = blockIdx.x * blockDim.x + threadIdx.x;
   // with M <= 2 the one-group-per-lane kernel runs; its operands cover whole
-  // 4-group stages (groups past G get zero activations and C/S)
-  const int Gx = MB <= 2 ? g4::kStageG * g4::nstages(P.K) : G;
+  // stages of SG groups (groups past G get zero activations and C/S)
+  const int SG = g4::stage_groups(MB);
+  const int Gx = MB <= 2 ? SG * g4::nstages(P.K, SG) : G;
   if (task >= Gx * MB) return;
   const int g = task / MB, m = task % MB;
+  // the group's lane position and slice: 4-group stages, group g % 4 and
+  // token m; 8-group stages, lane (g % 8) / 2 and the lane's group g % 2
+  const int gs = g / SG, gp = g % SG;
+  const int g4c = SG == 8 ? gp >> 1 : gp, g4sl = SG == 8 ? gp & 1 : m;
   unsigned char *g4b = P.wsB + P.map_off + kMapSlotBytes;
   float *g4cs = reinterpret_cast<float *>(g4b + g4::pad256(g4::b_bytes(MB, P.K)));
-  unsigned char *g4dst = g4b + (int64_t)((g / g4::kStageG) * MB + m) * g4::kBTok + (g % g4::kStageG) * 16;
-  float *g4q = g4cs + 4 * g;  // (C0, C1, S0, S1) of group g
-  if (g >= G) {
-    for (int jp = 0; jp < g4::kBPairs; ++jp) *reinterpret_cast<uint4 *>(g4dst + jp * 64) = make_uint4(0u, 0u, 0u, 0u);
-    g4q[m] = g4q[2 + m] = 0.f;
-    if (MB == 1) g4q[1] = g4q[3] = 0.f;
+  unsigned char *g4dst = g4b + (int64_t)(gs * 2 + g4sl) * g4::slice_bytes(SG) + g4c * 16;
+  float *g4q = g4cs + (gs * 4 + g4c) * 4;  // (C_a, C_b, S_a, S_b) of the lane position
+  if (MB <= 2 && g >= G) {
+    for (int jp = 0; jp < g4::pairs(SG); ++jp) *reinterpret_cast<uint4 *>(g4dst + jp * 64) = make_uint4(0u, 0u, 0u, 0u);
+    g4q[g4sl] = g4q[2 + g4sl] = 0.f;
     return;
   }
   const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
@@ -363,14 +366,20 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
          (4.f + 121.f / 256.f) * __half2float(ye[b]);
     S += x[0] + x[1] + x[2] + x[3] + x[4];
   }
-  if (MB <= 2) {
-    if (g & 1)
-      g4_write_slots<2>(g4dst, ya, yb, yc, yd, ye);
+  if (MB == 1) {
+    if (g4sl)
+      g4_write_slots<8, 26>(g4dst, ya, yb, yc, yd, ye);
     else
-      g4_write_slots<0>(g4dst, ya, yb, yc, yd, ye);
-    g4q[m] = C;
-    g4q[2 + m] = S;
-    if (MB == 1) g4q[1] = g4q[3] = 0.f;
+      g4_write_slots<8, 0>(g4dst, ya, yb, yc, yd, ye);
+  } else if (MB == 2) {
+    if (g & 1)
+      g4_write_slots<4, 2>(g4dst, ya, yb, yc, yd, ye);
+    else
+      g4_write_slots<4, 0>(g4dst, ya, yb, yc, yd, ye);
+  }
+  if (MB <= 2) {
+    g4q[g4sl] = C;
+    g4q[2 + g4sl] = S;
   }
   const int GL = g % kStageG;  // the group's index in its stage fixes its window
   unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
@@ -1435,8 +1444,10 @@ TQ_STATUS_ACCESSOR(read_status_gemv_mma)
 // Template tensor maps, encoded once per (kind, row length, rows) and cached:
 // kind 0 = plane 1 as a 2-D byte tensor of rows of `len` bytes (box 208 x 128
 // bytes); kind 1 = s1 / off as a 2-D fp16 tensor of rows of `len` halves (box
-// 8 x 128); kinds 2 and 3 the same for the one-group-per-lane kernel of
-// M <= 2 (boxes 112 x 256 bytes and 8 x 256 halves).  No swizzle, zero fill.
+// 8 x 128); kinds 2, 3 and 4 for the one-group-per-lane kernel of M <= 2:
+// plane 1 in boxes of 112 x 256 bytes (4-group stages, two tokens) or
+// 208 x 256 (8-group stages, one token), s1 / off in boxes of 8 x 256 halves.
+// No swizzle, zero fill.
 // The prep kernel puts in each problem's address.
 static bool map_template(int kind, int64_t len, const void *addr, int N, CUtensorMap *out) {
   // the driver's encoder, looked up through the runtime (no link-time
@@ -1454,7 +1465,7 @@ static bool map_template(int kind, int64_t len, const void *addr, int N, CUtenso
   static int64_t keys[64];
   static CUtensorMap maps[64];
   static int n = 0;
-  const int64_t key = ((int64_t)N << 32) | (len << 2) | kind;
+  const int64_t key = ((int64_t)N << 32) | (len << 3) | kind;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n; ++i)
     if (keys[i] == key) {
@@ -1467,7 +1478,7 @@ static bool map_template(int kind, int64_t len, const void *addr, int N, CUtenso
   cuuint64_t dims[2] = {(cuuint64_t)len, (cuuint64_t)N};
   cuuint64_t strides[1] = {(cuuint64_t)(len * esz)};
   const cuuint32_t box_rows = kind >= 2 ? (cuuint32_t)g4::kRows : (cuuint32_t)mm::kRows;
-  const cuuint32_t box_x = halves ? 8u : kind == 0 ? (cuuint32_t)mm::kStageBytes : 112u;
+  const cuuint32_t box_x = halves ? 8u : (kind == 0 || kind == 4) ? (cuuint32_t)mm::kStageBytes : 112u;
   cuuint32_t box[2] = {box_x, box_rows};
   cuuint32_t estr[2] = {1, 1};
   if (encode(&m, halves ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(addr),
@@ -1573,7 +1584,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     int64_t keys[mm::kMaxMapTemplates] = {};
     int nt = 0;
     auto slot = [&](int kind, int64_t len, const void *addr, int N) -> int {
-      const int64_t key = ((int64_t)N << 32) | (len << 2) | kind;
+      const int64_t key = ((int64_t)N << 32) | (len << 3) | kind;
       int k = 0;
       while (k < nt && keys[k] != key) ++k;
       if (k == nt) {
@@ -1587,7 +1598,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     };
     for (int i = 0; i < bp.count; ++i) {
       const Problem &P = bp.prob[i];
-      const int k1 = slot(g4path ? 2 : 0, row_bytes_of(P.K), P.plane1, P.N);
+      const int k1 = slot(g4path ? (bp.M == 1 ? 4 : 2) : 0, row_bytes_of(P.K), P.plane1, P.N);
       if (k1 < 0) return k1 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
       mt.idx[i] = (uint8_t)k1;
       mt.idx_so[i] = mm::kNoMap;
@@ -1616,7 +1627,8 @@ static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
     }
     counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + mm::kCounterOff);
   }
-  const int gtasks = (g4path ? g4::kStageG * ((gmax + g4::kStageG - 1) / g4::kStageG) : gmax) * bp.M;
+  const int sg = g4::stage_groups(bp.M);
+  const int gtasks = (g4path ? sg * ((gmax + sg - 1) / sg) : gmax) * bp.M;
   mm::gemv_mma_prep_kernel<<<dim3((gtasks + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
