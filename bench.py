@@ -273,7 +273,7 @@ class OracleLayer:
             del w
         self.cores = os.cpu_count() or 1
 
-    def run(self, frac=1.0):
+    def run(self, frac=1.0, nthreads=None):
         """One oracle pass over the first `frac` of every projection's rows;
         returns (packed bytes covered, seconds)."""
         nbytes, t = 0, 0.0
@@ -282,7 +282,7 @@ class OracleLayer:
             rows = None if R >= d["N"] else np.arange(R, dtype=np.int32)
             t0 = time.perf_counter()
             self.oracle.linear(1, d["N"], d["K"], d["p1"], d["p2"], d["sal"], d["s1"], d["off"], d["s2"], d["x"],
-                               rows=rows, nthreads=self.cores)
+                               rows=rows, nthreads=nthreads or self.cores)
             t += time.perf_counter() - t0
             nbytes += int(d["cum"][min(R, d["N"])])
         return nbytes, t
@@ -320,8 +320,6 @@ def run_prefill(args, ws, rank, local):
     for p in wl.config_projections(4):
         g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 500 + p.proj)
         pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
-        if on_codes is not None:
-            on_codes(p, g, pw)
         del g
         x = wl.gen_x_torch(M, p.K, dev, 600 + p.proj)
         y = torch.empty((M, p.N), dtype=torch.float16, device=dev)
@@ -527,37 +525,272 @@ def ternarize_cpu_baseline(budget_s):
                       f"({n / 1e6:.1f} M weights, {t:.1f} s, numpy on one core)"}
 
 
+# ------------------------------------------------- the other configurations
+L2_BYTES = 129 * 2 ** 20
+
+
+def graph_ms(fn, reps, warmup=2):
+    """Device time per replay of a CUDA graph that captured fn() (the calls
+    go to the current stream, which is the capture stream while capturing):
+    launch gaps of the host loop are not part of the number."""
+    import torch
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(warmup):
+            fn()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        fn()
+    for _ in range(warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def _clone_weight(pw):
+    from paper_2609_09240_gb300 import tq
+
+    c = lambda t: None if t is None else t.clone()
+    return tq.PackedWeight(pw.N, pw.K, c(pw.plane1), c(pw.salience), c(pw.rowptr), c(pw.plane2), c(pw.scale1),
+                           c(pw.offset), c(pw.scale2), pw.nnz, c(pw.p2index))
+
+
+def sub_config0(dev, peak):
+    """Config 0: one 512 x 1024 ternary linear at M = 1 (no second plane),
+    one tq_linear call at a time over rotated copies whose bytes total more
+    than 4 x L2, so that every call reads its weight from HBM."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    N, K, M = 512, 1024, 1
+    g = wl.gen_weights_torch(N, K, 0.0, dev, 11)
+    pw0 = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], None)
+    ws_bytes = tq.tq_workspace_bytes(M, N, K)
+    per = pw0.packed_bytes() + ws_bytes + 2 * (K + N)
+    R = -(-4 * L2_BYTES // per)
+    copies = [(_clone_weight(pw0), wl.gen_x_torch(M, K, dev, 100 + r), torch.empty((M, N), dtype=torch.float16,
+                                                                              device=dev),
+               tq.workspace(ws_bytes, dev)) for r in range(R)]
+
+    def calls():
+        for pw, x, y, wsb in copies:
+            tq.tq_linear(x, pw, y=y, ws=wsb)
+
+    ms = graph_ms(calls, reps=5) / R
+    gbs = pw0.packed_bytes() / (ms * 1e-3) / 1e9
+    return {"workload": "single ternary linear 512 x 1024, M=1, no second plane (config 0)",
+            "us_per_call": ms * 1e3, "packed_bytes": pw0.packed_bytes(), "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
+            "tokens_per_s": 1.0 / (ms * 1e-3),
+            "timing": f"{R} rotated copies of weight, x, y and workspace ({R * per / 2 ** 20:.0f} MiB > 4 x L2), "
+                      "one tq_linear call each, replayed as one CUDA graph (2 launches per call)"}
+
+
+def sub_config1(dev, peak):
+    """Config 1: one Qwen3-4B decoder layer's seven projections at M = 1,
+    10 % salient groups; a layer as one batched call and as seven tq_linear
+    calls, over rotated copies of the layer (more than 4 x L2 in total)."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    M = 1
+    base = []
+    for p in wl.config_projections(1):
+        g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 700 + p.proj)
+        base.append(tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None))
+        del g
+    layer_bytes = sum(pw.packed_bytes() for pw in base)
+    R = -(-4 * L2_BYTES // layer_bytes)
+    layers, batches = [], []
+    for r in range(R):
+        items = [(pw if r == 0 else _clone_weight(pw), wl.gen_x_torch(M, pw.K, dev, 800 + 8 * r + i),
+                  torch.empty((M, pw.N), dtype=torch.float16, device=dev)) for i, pw in enumerate(base)]
+        layers.append(items)
+        batches.append(tq.Batch(M, items))
+    wss = [tq.workspace(tq.tq_workspace_bytes(M, pw.N, pw.K), dev) for pw in base]
+
+    def batched():
+        for b in batches:
+            tq.tq_linear_batched(b)
+
+    def unbatched():
+        for items in layers:
+            for (pw, x, y), wsb in zip(items, wss):
+                tq.tq_linear(x, pw, y=y, ws=wsb)
+
+    ms_b = graph_ms(batched, reps=10) / R
+    ms_u = graph_ms(unbatched, reps=10) / R
+    gbs = layer_bytes / (ms_b * 1e-3) / 1e9
+    return {"workload": "qwen3-4b one decoder layer (q, k, v, o, gate, up, down), M=1, 10% salient (config 1)",
+            "us_per_layer": ms_b * 1e3, "packed_bytes": layer_bytes, "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
+            "us_per_layer_unbatched": ms_u * 1e3,
+            "timing": f"{R} rotated copies of the layer ({R * layer_bytes / 2 ** 20:.0f} MiB of packed weights > "
+                      "4 x L2); one tq_linear_batched call per layer (3 launches), or seven tq_linear calls; "
+                      "replayed as CUDA graphs"}
+
+
+def sub_skinny(items, M, dev, peak, packed_bytes, steps):
+    """Config 3: the Qwen3-8B step at M tokens (same packed weights as the
+    M = 1 step, fresh activations)."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    its = [(pw, wl.gen_x_torch(M, pw.K, dev, 900 + i), torch.empty((M, pw.N), dtype=torch.float16, device=dev))
+           for i, (pw, _, _) in enumerate(items)]
+    batch = tq.Batch(M, its)
+    stream = torch.cuda.current_stream()
+    for _ in range(3):
+        tq.tq_linear_batched(batch, stream)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        tq.tq_linear_batched(batch, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    gbs = packed_bytes / (ms * 1e-3) / 1e9
+    return {"M": M, "ms_per_step": ms, "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
+            "tokens_per_s": M / (ms * 1e-3), "steps": steps}
+
+
+def sub_unbatched_8b(items, dev, batched_ms):
+    """The Qwen3-8B step's projections called one tq_linear at a time (M = 1),
+    every layer in turn (the step's 1.79 GB rotate through L2)."""
+    from paper_2609_09240_gb300 import tq
+
+    shapes = {}
+    for pw, _, _ in items:
+        shapes.setdefault((pw.N, pw.K), tq.workspace(tq.tq_workspace_bytes(1, pw.N, pw.K), pw.plane1.device))
+
+    def calls():
+        for pw, x, y in items:
+            tq.tq_linear(x, pw, y=y, ws=shapes[(pw.N, pw.K)])
+
+    ms = graph_ms(calls, reps=5)
+    layers = len(items) // 7
+    return {"workload": "qwen3-8b step, each projection its own tq_linear call, M=1",
+            "us_per_layer": ms * 1e3 / layers, "us_per_layer_batched": batched_ms * 1e3 / layers,
+            "ratio_to_batched": ms / batched_ms,
+            "timing": f"{len(items)} tq_linear calls (3 launches each) replayed as one CUDA graph"}
+
+
+def sub_prefill(dev, steps=20):
+    """Config 4: one Qwen3-8B layer's seven projections at M = 2048 tokens
+    (tensor-core tile path); dense fp16 cuBLAS on the same shapes beside it."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    M = 2048
+    items, flops = [], 0
+    for p in wl.config_projections(4):
+        g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 500 + p.proj)
+        pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+        del g
+        items.append((pw, wl.gen_x_torch(M, p.K, dev, 600 + p.proj), torch.empty((M, p.N), dtype=torch.float16,
+                                                                                  device=dev),
+                      tq.workspace(tq.tq_workspace_bytes(M, p.N, p.K), dev)))
+        flops += 2 * M * p.N * p.K
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for pw, x, y, wsb in items:
+            tq.tq_linear(x, pw, y=y, ws=wsb, stream=stream)
+
+    dense = [torch.randn((pw.N, pw.K), device=dev, dtype=torch.float16) for pw, _, _, _ in items]
+
+    def dstep():
+        for (pw, x, y, _), W in zip(items, dense):
+            torch.matmul(x, W.t(), out=y)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps
+
+    ms, ms_dense = timed(step), timed(dstep)
+    peak, kind = measured_tensor_peak()
+    tflops = flops / (ms * 1e-3) / 1e12
+    return {"workload": "qwen3-8b prefill: one layer's 7 projections at M=2048 tokens (config 4)",
+            "ms_per_layer": ms, "flops_per_layer": flops, "tflops": tflops,
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
+                         "peak_kind": kind},
+            "dense_fp16_cublas": {"ms_per_layer": ms_dense, "tflops": flops / (ms_dense * 1e-3) / 1e12},
+            "l2": "no flush: a layer's 2048-token activations and outputs (~234 MB) exceed L2",
+            "gpu_launches_per_layer": 7, "steps": steps}
+
+
+def cpu_baseline_single(budget_s):
+    """The oracle on one host core over a prefix of layer 0's rows."""
+    L = OracleLayer()
+    frac, nbytes, t = 0.02, 0, 0.0
+    while t < budget_s and frac <= 1.0:
+        b, dt = L.run(frac, nthreads=1)
+        nbytes, t = nbytes + b, t + dt
+        frac *= 2
+    return nbytes / t / 1e9, f"the first rows of layer 0's seven projections on 1 core, {nbytes / 1e6:.1f} MB in {t:.1f} s"
+
+
 # ------------------------------------------------------------------- main
 def run_reference(args, ws, rank):
-    """The oracle timed on the host cores: each step is one pass over a
-    fixed fraction of layer 0's rows, sized so that the whole run stays
-    within about two minutes of CPU work."""
+    """The oracle timed on the host cores.  A step is one pass of the oracle
+    over a fixed sample of the workload (the first rows of each of layer 0's
+    seven projections), sized so that the whole run stays within about two
+    minutes of CPU work; ms_per_step is that pass's measured time and value
+    its packed bytes over that time."""
     if rank != 0:
         return 0
     L = OracleLayer()
     _, t_full = L.run()  # calibration pass (untimed)
     n = args.warmup + args.steps
     frac = min(1.0, 120.0 / max(n, 1) / max(t_full, 1e-6))
-    vals, nbytes_step = [], 0
+    times, nbytes_step = [], 0
     for i in range(n):
         b, t = L.run(frac)
         if i >= args.warmup:
-            vals.append(b / t / 1e9)
+            times.append(t)
             nbytes_step = b
-    value = float(np.median(vals))
-    bytes_step = 1_792_241_424
-    desc = (f"per step one oracle pass over the first {frac:.3f} of every row range of layer 0 of the Qwen3-8B "
-            f"step ({nbytes_step / 1e6:.1f} MB of packed bytes, M=1, 10% salient)")
+    t_step = float(np.median(times))
+    value = nbytes_step / t_step / 1e9
+    bytes_full = 1_792_241_424
+    desc = (f"per step one oracle pass over the first {frac:.3f} of the rows of each projection of layer 0 of the "
+            f"Qwen3-8B step ({nbytes_step / 1e6:.1f} MB of packed bytes, M=1, 10% salient); ms_per_step is "
+            "that pass's measured time")
     out = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": bytes_step / (value * 1e9) * 1e3, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": t_step * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": "qwen3-8b decode step, linear layers only, M=1 (252 packed projections)",
-                   "global_batch": 1, "seq_len": 1, "parallelism": "none (host CPU)"},
+        "config": {"workload": "qwen3-8b decode step, linear layers only, M=1: a fixed row sample of layer 0 per step",
+                   "sample_packed_bytes": nbytes_step, "global_batch": 1, "seq_len": 1,
+                   "parallelism": "none (host CPU)"},
         "cpu_baseline": {"value": value, "unit": "GB/s", "cores": L.cores, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-        "tokens_per_s": value * 1e9 / bytes_step,
+        "tokens_per_s_full_step": value * 1e9 / bytes_full,
     }
     print(json.dumps(out), flush=True)
     return 0
@@ -574,6 +807,8 @@ def main():
     ap.add_argument("--layers", type=int, default=None, help="profile a smaller step (first L layers)")
     ap.add_argument("--prefill", action="store_true", help="one Qwen3-8B layer at M = 2048 tokens")
     ap.add_argument("--ternarize", action="store_true", help="E2M-ATQ ternarization of one Qwen3-8B layer")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="time only the Qwen3-8B M=1 step (skip configs 0, 1, 3, 4 and the unbatched calls)")
     args = ap.parse_args()
     ws, rank, local = dist_env()
     if args.impl == "reference":
@@ -668,7 +903,7 @@ def main():
     out = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "accumulate": "f32", "data": "synthetic",
         "config": {"workload": f"qwen3-8b decode step, linear layers only, M={args.M} (252 packed projections)",
                    "model": "Qwen3-8B projection shapes, random ternary weights", "global_batch": args.M * ws,
                    "seq_len": 1, "parallelism": f"replicas x{ws}" if ws > 1 else "none",
@@ -690,10 +925,25 @@ def main():
         "gpu_launches": args.steps * launches_per_step,
         "clocks": clk.summary(),
     }
+    if not args.no_configs and args.layers is None and args.M == 1:
+        # the other configurations, each with its own timing (after the
+        # headline's timed region)
+        with ClockSampler(torch.cuda.current_device()) as clk2:
+            clk2.ready()
+            clk2.mark()
+            cfg = {"config0": sub_config0(dev, peak), "config1": sub_config1(dev, peak),
+                   "config3": [sub_skinny(items, M, dev, peak, packed_bytes, steps=50) for M in (2, 4, 8, 16)],
+                   "unbatched_calls": sub_unbatched_8b(items, dev, ms_per_step)}
+            cfg["config4"] = sub_prefill(dev)
+            clk2.mark()
+        cfg["clocks"] = clk2.summary()
+        out["configs"] = cfg
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         gbs, cores, desc, t = cpu_baseline(budget_s=15.0)
+        gbs1, desc1 = cpu_baseline_single(budget_s=5.0)
         out["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
-                               "sample": desc, "seconds": t}
+                               "sample": desc, "seconds": t,
+                               "single_core": {"value": gbs1, "unit": "GB/s", "cores": 1, "sample": desc1}}
     if rank == 0:
         print(json.dumps(out), flush=True)
     if pg:

@@ -25,7 +25,7 @@ int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
 cudaError_t read_status_gemv_g4(uint32_t *out, bool clear);
-int64_t g4_workspace_bytes(int M, int K);
+int64_t g4_workspace_bytes(int M, int N, int K);
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
 size_t ternarize_ws_bytes(int N, int K);
 cudaError_t launch_dequantize(int N, int K, const tq_weight *w, uint16_t *out, uint32_t *status, cudaStream_t s);
@@ -100,7 +100,7 @@ size_t problem_ws_bytes(int M, int N, int K) {
   mma_workspace_parts(M, N, K, &b, &cs, &y2);
   // + the tensor maps of plane 1, s1, off; with M <= 2 the operands of the
   // one-group-per-lane kernel follow
-  const size_t g4 = M <= 2 ? (size_t)g4_workspace_bytes(M, K) : 0;
+  const size_t g4 = M <= 2 ? (size_t)g4_workspace_bytes(M, N, K) : 0;
   return pad256(b) + pad256(cs) + pad256(y2) + 512 + g4;
 }
 

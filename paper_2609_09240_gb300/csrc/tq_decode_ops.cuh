@@ -135,5 +135,9 @@ __host__ __device__ inline int64_t b_bytes(int M, int K) {
   return (int64_t)nstages(K, stage_groups(M)) * 2 * slice_bytes(stage_groups(M));
 }
 __host__ __device__ inline int64_t cs_bytes(int M, int K) { return (int64_t)nstages(K, stage_groups(M)) * kCSStage; }
+// Split tiles (several CTAs per tile): one arrival counter per (tile,
+// decode warp), after the C/S blocks.
+constexpr int kMaxWarps = 16;
+__host__ __device__ inline int64_t ticket_bytes(int N) { return (int64_t)((N + kRows - 1) / kRows) * kMaxWarps * 4; }
 }  // namespace g4
 }  // namespace tq

@@ -46,6 +46,8 @@
 // units).  Every wait is bounded (tq_sm100.cuh).
 #include <cuda.h>
 
+#include <algorithm>
+
 #include "tq_common.cuh"
 #include "tq_decode_ops.cuh"
 #include "tq_sm100.cuh"
@@ -112,37 +114,46 @@ struct Bars {
 };
 static_assert(sizeof(Bars) <= 256, "barrier block");
 
-// Schedule: CTA c processes global 256-row tiles [cta_tile[c], cta_tile[c+1]).
+// Schedule: CTA c processes global work units [cta_unit[c], cta_unit[c+1]).
+// A unit is one 256-row tile's stages [k nst / u, (k + 1) nst / u) for
+// u = min(nst, split) parts of the tile (u = 1: the whole tile); units are
+// numbered over the problems in order, tile-major.
 struct Sched {
-  int32_t cta_tile[257];
+  int32_t cta_unit[257];
+  int32_t split;
 };
 
-// Iterates (tile, stage) in the CTA's order; tiles are numbered over the
-// problems in order, ceil(N / 256) each.
 template <int SG>
 struct Walk {
   const BatchParams *bp;
-  int tile, t_end, pi, tb, s, nst;
+  int split, unit, u_end, pi, ub, u, nst, tile, s, s_end;
+  __device__ int parts(int p) const { return min(nstages(bp->prob[p].K, SG), split); }
   __device__ void locate() {
     for (;;) {
-      const int T = (bp->prob[pi].N + kRows - 1) / kRows;
-      if (tile < tb + T) break;
-      tb += T;
+      const int U = (bp->prob[pi].N + kRows - 1) / kRows * parts(pi);
+      if (unit < ub + U) break;
+      ub += U;
       ++pi;
     }
+    u = parts(pi);
     nst = nstages(bp->prob[pi].K, SG);
-    s = 0;
+    const int local = unit - ub, k = local % u;
+    tile = local / u;
+    s = k * nst / u;
+    s_end = (k + 1) * nst / u;
   }
-  __device__ Walk(const BatchParams *b, int t0, int t1) : bp(b), tile(t0), t_end(t1), pi(0), tb(0), s(0), nst(0) {
-    if (tile < t_end) locate();
+  __device__ Walk(const BatchParams *b, int sp, int u0, int u1)
+      : bp(b), split(sp), unit(u0), u_end(u1), pi(0), ub(0), u(1), nst(0), tile(0), s(0), s_end(0) {
+    if (unit < u_end) locate();
   }
-  __device__ bool valid() const { return tile < t_end; }
+  __device__ bool valid() const { return unit < u_end; }
   __device__ const Problem &P() const { return bp->prob[pi]; }
-  __device__ int n0() const { return (tile - tb) * kRows; }
-  __device__ bool last_stage() const { return s + 1 == nst; }
+  __device__ int n0() const { return tile * kRows; }
+  __device__ bool last_stage() const { return s + 1 == s_end; }  // of this unit
+  __device__ bool shared_tile() const { return u > 1; }
   __device__ void next() {
-    if (++s < nst) return;
-    if (++tile < t_end) locate();
+    if (++s < s_end) return;
+    if (++unit < u_end) locate();
   }
 };
 
@@ -165,6 +176,9 @@ __device__ __forceinline__ const unsigned char *ws_b(const Problem &P) { return 
 __device__ __forceinline__ const unsigned char *ws_cs(const Problem &P, int MB) {
   return ws_b(P) + pad256(b_bytes(MB, P.K));
 }
+__device__ __forceinline__ int32_t *ws_tickets(const Problem &P, int MB) {
+  return reinterpret_cast<int32_t *>(const_cast<unsigned char *>(ws_cs(P, MB)) + pad256(cs_bytes(MB, P.K)));
+}
 
 // WD decode warps with TL m16 tiles each (WD x TL x 16 = 256 rows), and one
 // producer warp; SG groups per stage (8 for one token, 4 for two).
@@ -172,7 +186,7 @@ template <bool F32, int MB, int SG, int WD, int TL>
 __global__ void __launch_bounds__((WD + 1) * 32, 1)
     gemv_g4_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ Sched sc) {
   using C = Cfg<SG>;
-  static_assert(WD * TL * 16 == kRows, "decode warps cover the tile");
+  static_assert(WD * TL * 16 == kRows && WD <= kMaxWarps, "decode warps cover the tile");
   static_assert((SG == 8 && MB == 1) || (SG == 4 && MB == 2), "stage shape per token count");
   constexpr int kThreads = (WD + 1) * 32;
   constexpr int kNS = C::kNS;
@@ -204,7 +218,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     mbar_fence_init();
   }
   __syncthreads();
-  const int t_begin = sc.cta_tile[blockIdx.x], t_end = sc.cta_tile[blockIdx.x + 1];
+  const int t_begin = sc.cta_unit[blockIdx.x], t_end = sc.cta_unit[blockIdx.x + 1];
 
   if (warp < WD) {
     // ============================================================ decode
@@ -226,7 +240,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
 #pragma unroll
         for (int k = 0; k < MB; ++k) y[t][h][k] = 0.f;
     uint32_t buf = 0, phase = 0;
-    for (Walk<SG> w(&bp, t_begin, t_end); w.valid(); w.next()) {
+    for (Walk<SG> w(&bp, sc.split, t_begin, t_end); w.valid(); w.next()) {
       const bool ok = __all_sync(0xffffffffu, mm::wait_or_abort(&bars->full[buf], phase, abort_));
       if (!ok) break;
       const int s = w.s;
@@ -302,25 +316,62 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
               y[t][h][k] = v;
             }
         const Problem &P = w.P();
+        auto store = [&](int n, int k, float v) {
+          if (F32)
+            static_cast<float *>(P.y)[(int64_t)k * P.N + n] = v;
+          else
+            static_cast<__half *>(P.y)[(int64_t)k * P.N + n] = __float2half_rn(v);
+        };
+        if (!w.shared_tile()) {
+          // the whole tile was this CTA's: write y (+ the second plane)
+#pragma unroll
+          for (int t = 0; t < TL; ++t)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int n = w.n0() + rA + 16 * t + 8 * h;
+              if (((2 * t + h) & 3) == c && n < P.N) {
+#pragma unroll
+                for (int k = 0; k < MB; ++k) store(n, k, y[t][h][k] + (P.nnz > 0 ? P.y2()[(int64_t)n * MB + k] : 0.f));
+              }
+            }
+        } else {
+          // a share of the tile's stages: add the partial sums into y2 (fp32
+          // atomics, zeroed by the prep kernel); the last of the tile's
+          // units to arrive for this warp's rows writes them
+#pragma unroll
+          for (int t = 0; t < TL; ++t)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int n = w.n0() + rA + 16 * t + 8 * h;
+              if (((2 * t + h) & 3) == c && n < P.N) {
+#pragma unroll
+                for (int k = 0; k < MB; ++k) atomicAdd(P.y2() + (int64_t)n * MB + k, y[t][h][k]);
+              }
+            }
+          __threadfence();
+          __syncwarp();
+          int last = 0;
+          if (lane == 0) last = atomicAdd(ws_tickets(P, MB) + w.tile * kMaxWarps + warp, 1) == w.u - 1;
+          if (__shfl_sync(0xffffffffu, last, 0)) {
+            __threadfence();
+#pragma unroll
+            for (int t = 0; t < TL; ++t)
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const int n = w.n0() + rA + 16 * t + 8 * h;
+                if (((2 * t + h) & 3) == c && n < P.N) {
+#pragma unroll
+                  for (int k = 0; k < MB; ++k) store(n, k, __ldcg(P.y2() + (int64_t)n * MB + k));
+                }
+              }
+          }
+        }
 #pragma unroll
         for (int t = 0; t < TL; ++t)
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int n = w.n0() + rA + 16 * t + 8 * h;
-            if (((2 * t + h) & 3) == c && n < P.N) {
-#pragma unroll
-              for (int k = 0; k < MB; ++k) {
-                float v = y[t][h][k];
-                if (P.nnz > 0) v += P.y2()[(int64_t)n * MB + k];
-                if (F32)
-                  static_cast<float *>(P.y)[(int64_t)k * P.N + n] = v;
-                else
-                  static_cast<__half *>(P.y)[(int64_t)k * P.N + n] = __float2half_rn(v);
-              }
-            }
+          for (int h = 0; h < 2; ++h)
 #pragma unroll
             for (int k = 0; k < MB; ++k) y[t][h][k] = 0.f;
-          }
       }
       if (++buf == (uint32_t)kNS) buf = 0, phase ^= 1u;
     }
@@ -328,7 +379,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     // ========================================================== producer
     uint32_t buf = 0, phase = 0, q = 0;
     int map_pi = -1;
-    for (Walk<SG> w(&bp, t_begin, t_end); w.valid(); w.next(), ++q) {
+    for (Walk<SG> w(&bp, sc.split, t_begin, t_end); w.valid(); w.next(), ++q) {
       const Problem &P = w.P();
       const int s = w.s, n0 = w.n0();
       const int G = P.K / kGroup;
@@ -382,27 +433,50 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
         }
       }
       __syncwarp();
-      if (!so_map) {
-        // the stage's groups of s1 and off (zeros past G or N) at their
-        // place in each row's 8-group slot
+      const int col0 = SG == 8 ? 0 : 4 * (s & 1);  // the stage's first column in the 8-group slot rows
+      if (!so_map && G % 4 == 0 && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 7u) == 0) {
+        // rows of scales in whole 8-byte units (G a multiple of 4): 8-byte
+        // asynchronous copies of each 4-group half of the stage (zero-filled
+        // past G or N); each lane's arrival waits for its own copies
         const int rows = min(kRows, P.N - n0);
-        const int col0 = SG == 8 ? 0 : 4 * (s & 1);
-        __half *d1 = reinterpret_cast<__half *>(so), *d2 = reinterpret_cast<__half *>(so + C::kSOHalf);
-        for (int r = lane; r < rows; r += 32) {
-          const int64_t o = (int64_t)(n0 + r) * G;
+        for (int r = lane; r < kRows; r += 32) {
 #pragma unroll
-          for (int gg = 0; gg < SG; ++gg) {
-            const int gi = SG * s + gg;
-            d1[r * 8 + col0 + gg] = gi < G ? P.s1[o + gi] : __float2half_rn(0.f);
-            d2[r * 8 + col0 + gg] = gi < G ? P.off[o + gi] : __float2half_rn(0.f);
+          for (int hh = 0; hh < SG / 4; ++hh) {
+            const int gi = SG * s + 4 * hh;
+            const bool real = r < rows && gi < G;
+            const int64_t o = real ? (int64_t)(n0 + r) * G + gi : 0;
+            const uint32_t dst = smem_u32(so + r * 16 + 2 * (col0 + 4 * hh));
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(P.s1 + o), "r"(real ? 8 : 0)
+                         : "memory");
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst + C::kSOHalf), "l"(P.off + o),
+                         "r"(real ? 8 : 0)
+                         : "memory");
           }
         }
+        cp_async_mbar_arrive_noinc(full);  // the lane's arrival, once its copies have landed
+      } else {
+        if (!so_map) {
+          // other shapes: the stage's groups of s1 and off one by one (zeros
+          // past G or N) at their place in each row's 8-group slot
+          const int rows = min(kRows, P.N - n0);
+          __half *d1 = reinterpret_cast<__half *>(so), *d2 = reinterpret_cast<__half *>(so + C::kSOHalf);
+          for (int r = lane; r < rows; r += 32) {
+            const int64_t o = (int64_t)(n0 + r) * G;
+#pragma unroll
+            for (int gg = 0; gg < SG; ++gg) {
+              const int gi = SG * s + gg;
+              d1[r * 8 + col0 + gg] = gi < G ? P.s1[o + gi] : __float2half_rn(0.f);
+              d2[r * 8 + col0 + gg] = gi < G ? P.off[o + gi] : __float2half_rn(0.f);
+            }
+          }
+        }
+        mbar_arrive(full);  // the lanes' arrivals (the barrier counts 1 + 32)
       }
-      mbar_arrive(full);  // the lanes' arrivals (the barrier counts 1 + 32)
       if (++buf == (uint32_t)kNS) buf = 0, phase ^= 1u;
     }
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
+    mm::cp_async_wait<0>();
     if (lane == 0) {
       for (uint32_t k = (q > (uint32_t)kNS ? q - kNS : 0); k < q; ++k) mbar_wait(&bars->full[k % kNS], (k / kNS) & 1u);
     }
@@ -414,33 +488,51 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
 
 TQ_STATUS_ACCESSOR(read_status_gemv_g4)
 
-int64_t g4_workspace_bytes(int M, int K) {
-  return g4::pad256(g4::b_bytes(M, K)) + g4::pad256(g4::cs_bytes(M, K));
+static_assert(sizeof(BatchParams) + sizeof(g4::Sched) <= 32764, "one-group-per-lane kernel parameters");
+
+int64_t g4_workspace_bytes(int M, int N, int K) {
+  return g4::pad256(g4::b_bytes(M, K)) + g4::pad256(g4::cs_bytes(M, K)) + g4::pad256(g4::ticket_bytes(N));
+}
+
+// How many CTAs share each 256-row tile's stages for an M <= 2 batch: whole
+// tiles when there are at least as many tiles as CTAs, else about CTAs /
+// tiles parts per tile (at most one per stage).
+int g4_split_for(const BatchParams &bp, int num_sms) {
+  const int ctas = min(num_sms, 256);
+  int64_t tiles = 0;
+  for (int i = 0; i < bp.count; ++i) tiles += (bp.prob[i].N + g4::kRows - 1) / g4::kRows;
+  return tiles >= ctas ? 1 : (int)std::min<int64_t>(64, ctas / tiles);
 }
 
 // The M <= 2 decode kernel over a batch whose prep (activation slots, maps,
-// y2) and second plane have been launched on the same stream.
+// y2, tickets) and second plane have been launched on the same stream.
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   thread_local g4::Sched sc;
-  if (bp.M < 1 || bp.M > 2) return cudaErrorInvalidValue;
+  if (bp.M < 1 || bp.M > 2 || bp.g4_split < 1) return cudaErrorInvalidValue;
   const int ctas = min(num_sms, 256);
+  const int SG = g4::stage_groups(bp.M);
+  sc.split = bp.g4_split;
+  // contiguous unit ranges of about equal cost (groups per unit)
   int64_t total_cost = 0;
-  for (int i = 0; i < bp.count; ++i)
-    total_cost += (int64_t)((bp.prob[i].N + g4::kRows - 1) / g4::kRows) * (bp.prob[i].K / kGroup);
-  // contiguous tile ranges of about equal cost (tiles x groups)
-  int c = 0, tile = 0;
-  int64_t run = 0;
-  sc.cta_tile[0] = 0;
+  for (int i = 0; i < bp.count; ++i) total_cost += (int64_t)((bp.prob[i].N + g4::kRows - 1) / g4::kRows) * (bp.prob[i].K / kGroup);
+  int c = 0, unit = 0;
+  int64_t run2 = 0;  // twice the cost before the current unit
+  sc.cta_unit[0] = 0;
   for (int i = 0; i < bp.count; ++i) {
+    const int nst = g4::nstages(bp.prob[i].K, SG), G = bp.prob[i].K / kGroup;
+    const int u = min(nst, sc.split);
     const int tiles_i = (bp.prob[i].N + g4::kRows - 1) / g4::kRows;
-    const int64_t cost = bp.prob[i].K / kGroup;
-    for (int t = 0; t < tiles_i; ++t, ++tile) {
-      const int64_t mid2 = 2 * run + cost;
-      while (c < ctas - 1 && mid2 * ctas >= 2 * total_cost * (int64_t)(c + 1)) sc.cta_tile[++c] = tile;
-      run += cost;
-    }
+    for (int t = 0; t < tiles_i; ++t)
+      for (int k = 0; k < u; ++k, ++unit) {
+        // the unit's groups: its stages' share of G
+        const int64_t s0 = (int64_t)k * nst / u, s1 = (int64_t)(k + 1) * nst / u;
+        const int64_t cost = std::min<int64_t>(G, s1 * SG) - s0 * SG;
+        const int64_t mid2 = run2 + cost;
+        while (c < ctas - 1 && mid2 * ctas >= 2 * total_cost * (int64_t)(c + 1)) sc.cta_unit[++c] = unit;
+        run2 += 2 * cost;
+      }
   }
-  while (c < ctas) sc.cta_tile[++c] = tile;
+  while (c < ctas) sc.cta_unit[++c] = unit;
   using g4::kTL1;
   using g4::kTL2;
   using g4::kWD1;

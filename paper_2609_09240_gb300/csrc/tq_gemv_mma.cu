@@ -280,12 +280,22 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   const int p = blockIdx.y;
   if (p >= bp.count) return;
   const Problem &P = bp.prob[p];
-  if (P.nnz > 0) {
+  const bool g4_shared = bp.M <= 2 && bp.g4_split > 1;  // split tiles add their partial sums into y2
+  if (P.nnz > 0 || g4_shared) {
     // y2 starts at zero (the indexed second-plane kernel adds into it)
     float *y2 = P.y2();
     const int64_t n = (int64_t)P.N * bp.M;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
       y2[i] = 0.f;
+  }
+  if (g4_shared) {
+    // the arrival counters of split tiles start at zero
+    const int MBx = bp.M;
+    int32_t *tk = reinterpret_cast<int32_t *>(P.wsB + P.map_off + kMapSlotBytes + g4::pad256(g4::b_bytes(MBx, P.K)) +
+                                              g4::pad256(g4::cs_bytes(MBx, P.K)));
+    const int64_t n = g4::ticket_bytes(P.N) / 4;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+      tk[i] = 0;
   }
   if (p == 0 && blockIdx.x == 0 && threadIdx.x == 0 && unit_counter) *unit_counter = 0;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -1417,6 +1427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // -------------------------------------------------------------- launcher
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s);
+int g4_split_for(const BatchParams &bp, int num_sms);
 
 static int num_sms_mm() {
   static int n = 0;
@@ -1548,7 +1559,11 @@ static cudaError_t launch_mm(const BatchParams &bp, cudaStream_t s) {
 }
 
 template <bool F32>
-static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s) {
+static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
+  // the batch with the M <= 2 kernel's tile split filled in
+  thread_local BatchParams bp;
+  bp = bp_in;
+  bp.g4_split = bp.M <= 2 ? g4_split_for(bp, num_sms_mm()) : 1;
   thread_local mm::Sched sc;
   if (bp.M < 1 || bp.M > 16 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
   const int ctas = min(num_sms_mm(), 256);

@@ -64,13 +64,14 @@ def test_host_side_argument_errors_without_gpu():
     # M <= 2 adds the one-group-per-lane kernel's operands: per stage (8
     # groups for one token, 4 for two) two slices of activation slots (33 or
     # 18 chunks of 64 B), then 64 B of C/S
-    def g4(M, K):
+    # and 16 arrival counters per 256-row tile (tiles shared by several CTAs)
+    def g4(M, N, K):
         sg = 8 if M == 1 else 4
         nst = (K // 128 + sg - 1) // sg
-        return pad(nst * 2 * (33 if sg == 8 else 18) * 64) + pad(nst * 64)
-    assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) + g4(1, 4096) == 29184 + 16896 + 256
-    assert tq.tq_workspace_bytes(1, 300, 1152) == mma(1, 300, 1152) + g4(1, 1152)
-    assert tq.tq_workspace_bytes(2, 300, 1152) == mma(2, 300, 1152) + g4(2, 1152)
+        return pad(nst * 2 * (33 if sg == 8 else 18) * 64) + pad(nst * 64) + pad((N + 255) // 256 * 64)
+    assert tq.tq_workspace_bytes(1, 4096, 4096) == mma(1, 4096, 4096) + g4(1, 4096, 4096) == 29184 + 16896 + 256 + 1024
+    assert tq.tq_workspace_bytes(1, 300, 1152) == mma(1, 300, 1152) + g4(1, 300, 1152)
+    assert tq.tq_workspace_bytes(2, 300, 1152) == mma(2, 300, 1152) + g4(2, 300, 1152)
     assert tq.tq_workspace_bytes(5, 100, 1024) == mma(5, 100, 1024)
     # 8 < M <= 16: C/S for two 8-token tiles (128 B per group);
     # M > 16: the prefill tile path needs no workspace (256 bytes are asked for)

@@ -261,3 +261,28 @@ def test_one_group_per_lane_stage_shapes(H, M, f32):
         H.device_status_ok()
         for (pw, x, y), (y_ref, a_ref) in zip(items, refs):
             H.assert_close(y.float().cpu().numpy().astype(np.float64), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M,N,K,frac,index", [
+    (1, 1024, 4096, 0.1, True),    # k/v shape: 4 tiles x 4 stages, every stage its own CTA
+    (1, 4096, 12288, 0.1, True),   # down shape: 16 tiles x 12 stages, 9 CTAs per tile
+    (1, 200, 4224, 0.2, False),    # 1 tile, 5 stages (the last of one group), second plane without index
+    (2, 300, 9728, 0.1, True),     # two tokens: 2 tiles x 19 four-group stages
+    (2, 1, 640, 1.0, True),        # one row, every group salient
+])
+def test_split_tiles_single_call(H, M, N, K, frac, index):
+    """One tq_linear call on a projection with fewer 256-row tiles than SMs:
+    each tile's stages are shared by several CTAs, which add partial sums
+    into the fp32 workspace; the last to arrive writes y.  Checked against the
+    oracle on two calls in a row (the counters restart every call)."""
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, frac, config=6, proj=60 + M + N % 7)
+    xb = wl.gen_x(M, K, config=6, proj=60 + M + N % 7)
+    y_ref, a_ref = H.oracle_ref(w, xb)
+    pw = H.pack_on_gpu(w, index=index)
+    x = H.dev(xb)
+    ws = tq.workspace(tq.tq_workspace_bytes(M, N, K), x.device)
+    for _ in range(2):
+        y = tq.tq_linear_f32out(x, pw, ws=ws)
+        H.device_status_ok()
+        H.assert_close(y.cpu().numpy().astype(np.float64), y_ref, a_ref)
