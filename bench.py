@@ -220,7 +220,7 @@ def build_step(M, device, seed0=0, layers=None, on_codes=None):
 
 
 # the sources the decode-step kernels are compiled from
-DECODE_SOURCES = ("tq_common.cuh", "tq_gemv_mma.cu", "tq_sm100.cuh")
+DECODE_SOURCES = ("tq_common.cuh", "tq_decode_ops.cuh", "tq_gemv_g4.cu", "tq_gemv_mma.cu", "tq_sm100.cuh")
 
 
 def kernel_hash():
@@ -918,7 +918,8 @@ def main():
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
                      "traffic": ncu_traffic(),
                      "kernel": "decode step: activation prep + second plane (group-ordered index) + first plane "
-                               "(3 launches per step, timed together; the first-plane kernel is ~88 % of it)",
+                               "(one-group-per-lane kernel); 3 launches per step, timed together (the first-plane "
+                               "kernel is ~84 % of it)",
                      "launch_ms_avg": launch_avg},
         "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms},

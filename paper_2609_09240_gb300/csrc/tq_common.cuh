@@ -53,7 +53,7 @@ struct BatchParams {
   int32_t M;            // tokens (rows of every x)
   int32_t total_tiles;  // sum of tiles over problems
   int32_t out_f32;      // y is fp32 (else fp16)
-  int32_t g4_split;     // M <= 2: CTAs that share one 256-row tile's stages (1: whole tiles)
+  int32_t g4_split;     // M <= 2: target groups per work unit of a 256-row tile (0: whole tiles)
   int32_t reserved_;
   Problem prob[TQ_MAX_BATCH];
 };

@@ -115,19 +115,24 @@ struct Bars {
 static_assert(sizeof(Bars) <= 256, "barrier block");
 
 // Schedule: CTA c processes global work units [cta_unit[c], cta_unit[c+1]).
-// A unit is one 256-row tile's stages [k nst / u, (k + 1) nst / u) for
-// u = min(nst, split) parts of the tile (u = 1: the whole tile); units are
-// numbered over the problems in order, tile-major.
+// A unit is one 256-row tile's stages [k nst / u, (k + 1) nst / u), the
+// tile cut into u = min(nst, ceil(G / split)) parts for a target of `split`
+// groups per unit (split = 0: u = 1, whole tiles); units are numbered over
+// the problems in order, tile-major.
 struct Sched {
   int32_t cta_unit[257];
   int32_t split;
 };
+__host__ __device__ inline int unit_parts(int K, int SG, int split) {
+  const int G = K / kGroup, nst = nstages(K, SG);
+  return split > 0 ? min(nst, max(1, (G + split - 1) / split)) : 1;
+}
 
 template <int SG>
 struct Walk {
   const BatchParams *bp;
   int split, unit, u_end, pi, ub, u, nst, tile, s, s_end;
-  __device__ int parts(int p) const { return min(nstages(bp->prob[p].K, SG), split); }
+  __device__ int parts(int p) const { return unit_parts(bp->prob[p].K, SG, split); }
   __device__ void locate() {
     for (;;) {
       const int U = (bp->prob[pi].N + kRows - 1) / kRows * parts(pi);
@@ -218,6 +223,8 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     mbar_fence_init();
   }
   __syncthreads();
+  // everything below reads what the prep and second-plane kernels wrote
+  grid_dep_wait();
   const int t_begin = sc.cta_unit[blockIdx.x], t_end = sc.cta_unit[blockIdx.x + 1];
 
   if (warp < WD) {
@@ -494,21 +501,27 @@ int64_t g4_workspace_bytes(int M, int N, int K) {
   return g4::pad256(g4::b_bytes(M, K)) + g4::pad256(g4::cs_bytes(M, K)) + g4::pad256(g4::ticket_bytes(N));
 }
 
-// How many CTAs share each 256-row tile's stages for an M <= 2 batch: whole
-// tiles when there are at least as many tiles as CTAs, else about CTAs /
-// tiles parts per tile (at most one per stage).
+// Target groups per work unit for an M <= 2 batch: 0 (whole tiles) when the
+// largest tile costs no more than a CTA's fair share of the batch, else
+// that share, so that no unit holds up the end of the call.
 int g4_split_for(const BatchParams &bp, int num_sms) {
-  const int ctas = min(num_sms, 256);
-  int64_t tiles = 0;
-  for (int i = 0; i < bp.count; ++i) tiles += (bp.prob[i].N + g4::kRows - 1) / g4::kRows;
-  return tiles >= ctas ? 1 : (int)std::min<int64_t>(64, ctas / tiles);
+  const int ctas = std::min(num_sms, 256);
+  int64_t total = 0;
+  int gmax = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    const int G = bp.prob[i].K / kGroup;
+    total += (int64_t)((bp.prob[i].N + g4::kRows - 1) / g4::kRows) * G;
+    gmax = std::max(gmax, G);
+  }
+  const int64_t share = (total + ctas - 1) / ctas;
+  return share >= gmax ? 0 : (int)std::max<int64_t>(1, share);
 }
 
 // The M <= 2 decode kernel over a batch whose prep (activation slots, maps,
 // y2, tickets) and second plane have been launched on the same stream.
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   thread_local g4::Sched sc;
-  if (bp.M < 1 || bp.M > 2 || bp.g4_split < 1) return cudaErrorInvalidValue;
+  if (bp.M < 1 || bp.M > 2 || bp.g4_split < 0) return cudaErrorInvalidValue;
   const int ctas = min(num_sms, 256);
   const int SG = g4::stage_groups(bp.M);
   sc.split = bp.g4_split;
@@ -520,7 +533,7 @@ cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   sc.cta_unit[0] = 0;
   for (int i = 0; i < bp.count; ++i) {
     const int nst = g4::nstages(bp.prob[i].K, SG), G = bp.prob[i].K / kGroup;
-    const int u = min(nst, sc.split);
+    const int u = g4::unit_parts(bp.prob[i].K, SG, sc.split);
     const int tiles_i = (bp.prob[i].N + g4::kRows - 1) / g4::kRows;
     for (int t = 0; t < tiles_i; ++t)
       for (int k = 0; k < u; ++k, ++unit) {
@@ -542,8 +555,19 @@ cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
                   : (bp.out_f32 ? g4::gemv_g4_kernel<true, 2, 4, kWD2, kTL2> : g4::gemv_g4_kernel<false, 2, 4, kWD2, kTL2>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, g4::kDynBytes);
   if (e != cudaSuccess) return e;
-  kern<<<ctas, ((bp.M == 1 ? kWD1 : kWD2) + 1) * 32, g4::kDynBytes, s>>>(bp, sc);
-  return cudaGetLastError();
+  // launched programmatically: its CTAs set up (table, barriers) while the
+  // second-plane kernel finishes, then wait for it (grid_dep_wait)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(ctas);
+  cfg.blockDim = dim3(((bp.M == 1 ? kWD1 : kWD2) + 1) * 32);
+  cfg.dynamicSmemBytes = g4::kDynBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, bp, sc);
 }
 
 }  // namespace tq

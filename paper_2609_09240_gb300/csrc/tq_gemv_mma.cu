@@ -280,7 +280,9 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   const int p = blockIdx.y;
   if (p >= bp.count) return;
   const Problem &P = bp.prob[p];
-  const bool g4_shared = bp.M <= 2 && bp.g4_split > 1;  // split tiles add their partial sums into y2
+  // the next kernel (second plane or main) may start its own set-up now
+  grid_dep_launch_next();
+  const bool g4_shared = bp.M <= 2 && bp.g4_split > 0;  // split tiles add their partial sums into y2
   if (P.nnz > 0 || g4_shared) {
     // y2 starts at zero (the indexed second-plane kernel adds into it)
     float *y2 = P.y2();
@@ -1013,6 +1015,10 @@ __global__ void __launch_bounds__(c_threads(TWO), 1)
     for (int i = tid; i < 256 * 32; i += c_threads(TWO)) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
   }
   __syncthreads();
+  // the work below reads the prep kernel's output (launched programmatically
+  // after it); the main kernel may start its set-up meanwhile
+  grid_dep_wait();
+  grid_dep_launch_next();
   const int MB = ONE ? 1 : bp.M, g16 = lane >> 2, c = lane & 3, quad = lane & ~3;
   const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
   const int count = cb.count, total = cb.base[count];
@@ -1655,8 +1661,19 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
                           : (bp.M > 8 ? mm::gemv_mma_p2c_kernel<false, true> : mm::gemv_mma_p2c_kernel<false, false>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
     if (e != cudaSuccess) return e;
-    kern<<<ctas, mm::c_threads(bp.M > 8), mm::kCDynBytes2, s>>>(cb, bp, counter);
-    e = cudaGetLastError();
+    // launched programmatically after the prep kernel (it sets up its table,
+    // then waits for the prep kernel's output)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(ctas);
+    cfg.blockDim = dim3(mm::c_threads(bp.M > 8));
+    cfg.dynamicSmemBytes = mm::kCDynBytes2;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, cb, bp, counter);
     if (e != cudaSuccess) return e;
   } else if (any2 && gmax <= mm::kQMaxG) {
     auto kern = bp.M == 1 ? mm::gemv_mma_p2v3_kernel<true> : mm::gemv_mma_p2v3_kernel<false>;

@@ -89,6 +89,15 @@ __device__ __forceinline__ void cp_async_mbar_arrive_noinc(uint64_t *bar) {
   asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// ------------------------------------------ programmatic dependent launch
+// A kernel launched with programmatic stream serialization may start while
+// the previous kernel of its stream still runs: it waits here before it
+// reads anything that kernel wrote (returns at once without such a launch).
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel of the stream (if launched programmatically) start
+// its own set-up; it still waits for this grid's completion before reading.
+__device__ __forceinline__ void grid_dep_launch_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------- bulk copies
 // 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
 // src, dst 16-byte aligned; bytes a multiple of 16.
