@@ -744,6 +744,54 @@ def sub_prefill(dev, steps=20):
             "gpu_launches_per_layer": 7, "steps": steps}
 
 
+def sub_sequence(dev, peak, steps=30):
+    """The dependency-ordered Qwen3-8B step (M = 1): per layer q/k/v fused
+    (6144 x 4096), o, gate/up fused (24576 x 4096), down -- 144 problems run
+    in order by tq_linear_sequence (one persistent launch, a grid barrier
+    between problems) -- beside the same 144 problems as one independent
+    tq_linear_batched call."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    fused = [("qkv", 6144, 4096), ("o", 4096, 4096), ("gate_up", 24576, 4096), ("down", 4096, 12288)]
+    items, packed = [], 0
+    for layer in range(wl.QWEN3_8B_LAYERS):
+        for j, (name, N, K) in enumerate(fused):
+            seed = 7_000_000 + layer * 16 + j
+            g = wl.gen_weights_torch(N, K, 0.1, dev, seed)
+            pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"] if g["nnz"] else None)
+            del g
+            items.append((pw, wl.gen_x_torch(1, K, dev, seed + 7), torch.empty((1, N), dtype=torch.float16,
+                                                                               device=dev)))
+            packed += pw.packed_bytes()
+    batch = tq.Batch(1, items)
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        for _ in range(3):
+            fn(batch, stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            fn(batch, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps
+
+    ms_seq = timed(tq.tq_linear_sequence)
+    ms_ind = timed(tq.tq_linear_batched)
+    st = tq.tq_get_device_status(clear=True)
+    gbs = packed / (ms_seq * 1e-3) / 1e9
+    return {"workload": "qwen3-8b decode step, M=1, q/k/v and gate/up fused: 144 problems in layer order",
+            "ms_per_step": ms_seq, "packed_bytes": packed, "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
+            "tokens_per_s": 1.0 / (ms_seq * 1e-3),
+            "independent_ms_per_step": ms_ind, "ordering_cost_ms": ms_seq - ms_ind,
+            "gpu_launches_per_step": 2, "device_status": st, "steps": steps}
+
+
 def cpu_baseline_single(budget_s):
     """The oracle on one host core over a prefix of layer 0's rows."""
     L = OracleLayer()
@@ -936,6 +984,7 @@ def main():
                    "config3": [sub_skinny(items, M, dev, peak, packed_bytes, steps=50) for M in (2, 4, 8, 16)],
                    "unbatched_calls": sub_unbatched_8b(items, dev, ms_per_step)}
             cfg["config4"] = sub_prefill(dev)
+            cfg["dependency_ordered"] = sub_sequence(dev, peak)
             clk2.mark()
         cfg["clocks"] = clk2.summary()
         out["configs"] = cfg

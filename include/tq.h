@@ -326,6 +326,35 @@ TQ_API size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_prob
 TQ_API tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
                                    size_t workspace_bytes, void *stream);
 
+/* Dependency-ordered sequence (paper "Direct Packed Execution": the packed
+ * runtime runs one token's layers in order).  Like tq_linear_batched, but
+ * problem i + 1 starts only once problem i has completed on every SM, as
+ * the layers of a model need: e.g. per layer q/k/v (rows concatenated into
+ * one weight), o, gate/up (concatenated), down.  The attention, norms and
+ * activation between them are outside this library: every problem's x is
+ * an input of the call.  One persistent launch after the activation prep;
+ * between problems a grid-wide barrier whose wait is bounded by the wall-
+ * time limit (a wait that runs out sets the timeout bit of the device
+ * status word, see tq_get_device_status, and the kernel returns).  The
+ * fp32 sums of each problem's rows are added in a varying order, so
+ * results may differ in the last bits from run to run.
+ *   M must be 1 (TQ_ERR_SHAPE otherwise); count <= TQ_MAX_BATCH; every
+ *   weight with a second plane must carry its index (p2index, else
+ *   TQ_ERR_NULL); the workspace is sized by tq_batched_workspace_bytes;
+ *   a sequence's problems may have at most five distinct (N, K) shapes
+ *   (TQ_ERR_CUDA otherwise). */
+TQ_API tq_status tq_linear_sequence(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
+                                    size_t workspace_bytes, void *stream);
+
+/* Failure-path self-test of tq_linear_sequence (no fault involved): runs
+ * its kernel on the given problems with every problem barrier expecting one
+ * more participant than exists, so that the first barrier's bounded wait
+ * runs out after the wall-time limit (about 2 s); the device status word
+ * then has its timeout bit set and the launch ends normally.  Arguments as
+ * tq_linear_sequence with M = 1. */
+TQ_API tq_status tq_sequence_selftest(int32_t count, const tq_problem *problems, void *workspace,
+                                      size_t workspace_bytes, void *stream);
+
 /* ---------------------------------------------------------------------
  * Allocation-free variant (no counterpart in the paper; an integration aid).
  *

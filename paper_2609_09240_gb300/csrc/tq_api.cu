@@ -21,6 +21,7 @@ cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *pl
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s);
 cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
+cudaError_t launch_gemv_sequence(const BatchParams &bp, int barrier_extra, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
@@ -116,6 +117,29 @@ size_t call_ws_bytes(int M, int N, int K) {
 }  // namespace tq
 
 namespace {
+
+// Places every problem's workspace (TQ_ERR_SHAPE when it is too small).
+tq_status place(BatchParams &bp, unsigned char *ws, size_t ws_bytes) {
+  const int rows = mma_rows_per_tile();
+  int tiles = 0;
+  size_t off = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    Problem &P = bp.prob[i];
+    P.tile_begin = tiles;
+    tiles += (P.N + rows - 1) / rows;
+    const size_t tot = problem_ws_bytes(bp.M, P.N, P.K);
+    if (off + tot > ws_bytes) return TQ_ERR_SHAPE;
+    size_t b, cs, y2;
+    mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
+    P.wsB = ws + off;
+    P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
+    P.y2_off = (int32_t)(pad256(b) + pad256(cs));
+    P.map_off = (int32_t)(pad256(b) + pad256(cs) + pad256(y2));
+    off += tot;
+  }
+  bp.total_tiles = tiles;
+  return TQ_OK;
+}
 
 // Places every problem's workspace and runs the decode path for bp.M <= 16
 // tokens in one pass (warp-level MMA kernels).  Returns TQ_ERR_SHAPE when the
@@ -336,6 +360,51 @@ tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems
     bp.prob[i] = to_problem(&q.w, q.x, q.y);
   }
   return run_batch(bp, static_cast<unsigned char *>(workspace), workspace_bytes, (cudaStream_t)stream);
+}
+
+}  // extern "C"
+
+namespace {
+// Validates a host problem array into the per-thread launch parameters.
+tq_status fill_batch(BatchParams &bp, int32_t M, int32_t count, const tq_problem *problems) {
+  bp.count = count;
+  bp.M = M;
+  bp.out_f32 = 0;
+  for (int i = 0; i < count; ++i) {
+    const tq_problem &q = problems[i];
+    if (tq_status st = check_weight(&q.w, q.w.N, q.w.K)) return st;
+    if (!q.x || !q.y) return TQ_ERR_NULL;
+    if (!aligned16(q.x)) return TQ_ERR_ALIGN;
+    if (!aligned2(q.y)) return TQ_ERR_ALIGN;
+    bp.prob[i] = to_problem(&q.w, q.x, q.y);
+  }
+  return TQ_OK;
+}
+
+tq_status run_sequence(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
+                       size_t workspace_bytes, int barrier_extra, cudaStream_t s) {
+  if (M != 1 || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
+  if (!problems || !workspace) return TQ_ERR_NULL;
+  if ((uintptr_t)workspace & 255u) return TQ_ERR_ALIGN;
+  thread_local BatchParams bp;
+  if (tq_status st = fill_batch(bp, M, count, problems)) return st;
+  for (int i = 0; i < count; ++i)
+    if (problems[i].w.nnz > 0 && !problems[i].w.p2index) return TQ_ERR_NULL;
+  if (tq_status st = place(bp, static_cast<unsigned char *>(workspace), workspace_bytes)) return st;
+  return from_cuda(launch_gemv_sequence(bp, barrier_extra, s));
+}
+}  // namespace
+
+extern "C" {
+
+tq_status tq_linear_sequence(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
+                             size_t workspace_bytes, void *stream) {
+  return run_sequence(M, count, problems, workspace, workspace_bytes, 0, (cudaStream_t)stream);
+}
+
+tq_status tq_sequence_selftest(int32_t count, const tq_problem *problems, void *workspace, size_t workspace_bytes,
+                               void *stream) {
+  return run_sequence(1, count, problems, workspace, workspace_bytes, 1, (cudaStream_t)stream);
 }
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {

@@ -50,6 +50,7 @@
 
 #include "tq_common.cuh"
 #include "tq_decode_ops.cuh"
+#include "tq_p2_tile.cuh"
 #include "tq_sm100.cuh"
 
 namespace tq {
@@ -185,6 +186,206 @@ __device__ __forceinline__ int32_t *ws_tickets(const Problem &P, int MB) {
   return reinterpret_cast<int32_t *>(const_cast<unsigned char *>(ws_cs(P, MB)) + pad256(cs_bytes(MB, P.K)));
 }
 
+// Set-up shared by the kernels below: the lane-replicated table, the zero
+// activation block, the stage barriers.
+template <int SG, int WD>
+__device__ __forceinline__ void setup_cta(unsigned char *dyn, int tid, int nthreads) {
+  using C = Cfg<SG>;
+  Bars *bars = reinterpret_cast<Bars *>(dyn + C::kOffBars);
+  uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
+  for (int i = tid; i < 256 * 32; i += nthreads) lut[(i >> 5) * 64 + (i & 31)] = mm::lut_word(i >> 5);
+  for (int i = tid; i < C::kZeroBytes / 16; i += nthreads)
+    reinterpret_cast<uint4 *>(dyn + C::kOffZero)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (tid == 0) {
+    for (int i = 0; i < C::kNS; ++i) {
+      mbar_init(&bars->full[i], 1 + 32);  // the producer's expect-tx arrival + its 32 lanes' arrivals
+      mbar_init(&bars->empty[i], WD);
+    }
+    bars->abort_ = 0;
+    mbar_fence_init();
+  }
+}
+
+// One stage in slot buf for a decode warp: the MMAs of its TL m16 tiles
+// over the stage's window words, then s1 / off of the lane's groups added to
+// y[tile][half][token].  (rA: the warp's first row of the lane; wb: the
+// lane's first window byte; realB: whether the lane holds real activation
+// slots; tag: table base | lane * 4.)
+template <int MB, int SG, int TL>
+__device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, int s, int rA, int wb, int c, int g,
+                                             bool realB, uint32_t tag, float (&y)[TL][2][MB]) {
+  using C = Cfg<SG>;
+  const int shift = SG == 8 ? 0 : 8 * (s & 1);  // odd 4-group stages are copied from 8 bytes early
+  const unsigned char *p1 = dyn + C::p1_off(buf) + shift + wb + rA * C::kBox;
+  const unsigned char *bq =
+      dyn + (realB ? kA2 + C::kOffB + (buf * 2 + (g & 1)) * C::kSlice + c * 16 : C::kOffZero + 16 * ((g >> 1) + 2));
+  const float4 cs = *reinterpret_cast<const float4 *>(dyn + C::kOffCS + buf * kCSStage + c * 16);
+  // accumulators start at -C (slice 0 in columns 2c, slice 1 in 2c + 1)
+  float d[TL][4];
+#pragma unroll
+  for (int t = 0; t < TL; ++t) d[t][0] = d[t][2] = -cs.x, d[t][1] = d[t][3] = -cs.y;
+#pragma unroll
+  for (int i = 0; i < C::kWords; ++i) {
+    uint32_t a[TL][2][10];
+#pragma unroll
+    for (int t = 0; t < TL; ++t)
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+        decode_word(*reinterpret_cast<const uint32_t *>(p1 + (16 * t + 8 * h) * C::kBox + 4 * i), tag, a[t][h]);
+#pragma unroll
+    for (int m = 0; m < 5; ++m) {
+      const int j = 5 * i + m;
+      const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
+      const uint32_t b0 = (j & 1) ? q.z : q.x, b1 = (j & 1) ? q.w : q.y;
+#pragma unroll
+      for (int t = 0; t < TL; ++t)
+        mm::mma16816(d[t], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
+    }
+  }
+  // s1 / off of (row, the lane's groups): the slot holds 8 groups per row
+  // (both halves of an 8-group stage; an odd 4-group stage's at 4)
+  const unsigned char *so = dyn + kA2 + C::kOffSO + buf * C::kSOSlot;
+#pragma unroll
+  for (int t = 0; t < TL; ++t) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = rA + 16 * t + 8 * h;
+      if (SG == 8) {
+        // groups 2c, 2c + 1 (columns 2c, 2c + 1) of the one token
+        const __half2 s1 = *reinterpret_cast<const __half2 *>(so + r * 16 + 4 * c);
+        const __half2 of = *reinterpret_cast<const __half2 *>(so + C::kSOHalf + r * 16 + 4 * c);
+        float v = fmaf(__low2float(of), cs.z, y[t][h][0]);
+        v = fmaf(__high2float(of), cs.w, v);
+        v = fmaf(__low2float(s1), d[t][2 * h], v);
+        y[t][h][0] = fmaf(__high2float(s1), d[t][2 * h + 1], v);
+      } else {
+        // group c, tokens 0 and 1 (columns 2c, 2c + 1)
+        const int gl = 2 * (4 * (s & 1) + c);
+        const float s1 = __half2float(*reinterpret_cast<const __half *>(so + r * 16 + gl));
+        const float of = __half2float(*reinterpret_cast<const __half *>(so + C::kSOHalf + r * 16 + gl));
+        y[t][h][0] = fmaf(s1, d[t][2 * h], fmaf(of, cs.z, y[t][h][0]));
+        y[t][h][MB - 1] = fmaf(s1, d[t][2 * h + 1], fmaf(of, cs.w, y[t][h][MB - 1]));
+      }
+    }
+  }
+}
+
+// The sum over the four lane positions of each row (every lane of a quad
+// then holds it).
+template <int MB, int TL>
+__device__ __forceinline__ void quad_sum(float (&y)[TL][2][MB]) {
+#pragma unroll
+  for (int t = 0; t < TL; ++t)
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int k = 0; k < MB; ++k) {
+        float v = y[t][h][k];
+        v += __shfl_xor_sync(0xffffffffu, v, 1);
+        v += __shfl_xor_sync(0xffffffffu, v, 2);
+        y[t][h][k] = v;
+      }
+}
+
+// The producer's copies of stage s of the tile at row n0 of problem P into
+// slot buf (after the slot's empty wait), ending with the lanes' arrivals on
+// its full barrier.  map_pi: the problem whose tensor maps were last
+// acquired (the fence is needed once per problem).
+template <int MB, int SG>
+__device__ __forceinline__ void produce_stage(unsigned char *dyn, Bars *bars, int buf, const Problem &P, int pi,
+                                              int &map_pi, int s, int n0, int lane) {
+  using C = Cfg<SG>;
+  constexpr int kNSl = SG == 8 ? 2 : MB;
+  const int G = P.K / kGroup;
+  uint64_t *full = &bars->full[buf];
+  // s1 / off go by tensor copies when their rows are whole 16-byte units
+  // (the prep kernel then built their maps), else by asynchronous copies or
+  // plain loads
+  const bool so_map = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
+  unsigned char *so = dyn + kA2 + C::kOffSO + buf * C::kSOSlot;
+  const unsigned char *maps = static_cast<const unsigned char *>(P.map());
+  const int g8 = SG == 8 ? s : s >> 1;  // the 8-group box holding the stage
+  if (lane == 0) {
+    if (pi != map_pi) {
+      // the problem's tensor maps, written by the prep kernel
+      asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps) : "memory");
+      if (so_map) {
+        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + 128) : "memory");
+        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + 256) : "memory");
+      }
+      map_pi = pi;
+    }
+    mbar_arrive_expect_tx(full, (uint32_t)(C::kP1Slot + kNSl * C::kSliceG + kCSStage) +
+                                    (so_map ? (uint32_t)C::kSOSlot : 0u));
+    // the stage's plane-1 bytes of the tile's 256 rows from the 16-byte
+    // boundary at or before them (rows past N and bytes past the row's end
+    // arrive as zeros)
+    const int x = SG == 8 ? C::kStageBytes * s : C::kStageBytes * s - 8 * (s & 1);
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dyn + C::p1_off(buf))),
+        "l"(maps), "r"(x), "r"(n0), "r"(smem_u32(full))
+        : "memory");
+#pragma unroll
+    for (int sl = 0; sl < kNSl; ++sl)
+      bulk_g2s(dyn + kA2 + C::kOffB + (buf * 2 + sl) * C::kSlice, ws_b(P) + ((int64_t)s * 2 + sl) * C::kSliceG,
+               C::kSliceG, full);
+    bulk_g2s(dyn + C::kOffCS + buf * kCSStage, ws_cs(P, MB) + (int64_t)s * kCSStage, kCSStage, full);
+    if (so_map) {
+      asm volatile(
+          "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+              smem_u32(so)),
+          "l"(maps + 128), "r"(8 * g8), "r"(n0), "r"(smem_u32(full))
+          : "memory");
+      asm volatile(
+          "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+              smem_u32(so + C::kSOHalf)),
+          "l"(maps + 256), "r"(8 * g8), "r"(n0), "r"(smem_u32(full))
+          : "memory");
+    }
+  }
+  __syncwarp();
+  const int col0 = SG == 8 ? 0 : 4 * (s & 1);  // the stage's first column in the 8-group slot rows
+  if (!so_map && G % 4 == 0 && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 7u) == 0) {
+    // rows of scales in whole 8-byte units (G a multiple of 4): 8-byte
+    // asynchronous copies of each 4-group half of the stage (zero-filled
+    // past G or N); each lane's arrival waits for its own copies
+    const int rows = min(kRows, P.N - n0);
+    for (int r = lane; r < kRows; r += 32) {
+#pragma unroll
+      for (int hh = 0; hh < SG / 4; ++hh) {
+        const int gi = SG * s + 4 * hh;
+        const bool real = r < rows && gi < G;
+        const int64_t o = real ? (int64_t)(n0 + r) * G + gi : 0;
+        const uint32_t dst = smem_u32(so + r * 16 + 2 * (col0 + 4 * hh));
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(P.s1 + o), "r"(real ? 8 : 0)
+                     : "memory");
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst + C::kSOHalf), "l"(P.off + o),
+                     "r"(real ? 8 : 0)
+                     : "memory");
+      }
+    }
+    cp_async_mbar_arrive_noinc(full);  // the lane's arrival, once its copies have landed
+  } else {
+    if (!so_map) {
+      // other shapes: the stage's groups of s1 and off one by one (zeros
+      // past G or N) at their place in each row's 8-group slot
+      const int rows = min(kRows, P.N - n0);
+      __half *d1 = reinterpret_cast<__half *>(so), *d2 = reinterpret_cast<__half *>(so + C::kSOHalf);
+      for (int r = lane; r < rows; r += 32) {
+        const int64_t o = (int64_t)(n0 + r) * G;
+#pragma unroll
+        for (int gg = 0; gg < SG; ++gg) {
+          const int gi = SG * s + gg;
+          d1[r * 8 + col0 + gg] = gi < G ? P.s1[o + gi] : __float2half_rn(0.f);
+          d2[r * 8 + col0 + gg] = gi < G ? P.off[o + gi] : __float2half_rn(0.f);
+        }
+      }
+    }
+    mbar_arrive(full);  // the lanes' arrivals (the barrier counts 1 + 32)
+  }
+}
+
 // WD decode warps with TL m16 tiles each (WD x TL x 16 = 256 rows), and one
 // producer warp; SG groups per stage (8 for one token, 4 for two).
 template <bool F32, int MB, int SG, int WD, int TL>
@@ -193,9 +394,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
   using C = Cfg<SG>;
   static_assert(WD * TL * 16 == kRows && WD <= kMaxWarps, "decode warps cover the tile");
   static_assert((SG == 8 && MB == 1) || (SG == 4 && MB == 2), "stage shape per token count");
-  constexpr int kThreads = (WD + 1) * 32;
   constexpr int kNS = C::kNS;
-  constexpr int kNSl = SG == 8 ? 2 : MB;  // activation slices in use
   extern __shared__ __align__(1024) unsigned char dyn[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (smem_u32(dyn) != kDynShared) {
@@ -206,22 +405,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
   }
   Bars *bars = reinterpret_cast<Bars *>(dyn + C::kOffBars);
   volatile int32_t *abort_ = &bars->abort_;
-
-  // ---- one-time set-up: the lane-replicated table, the zero block, barriers
-  {
-    uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
-    for (int i = tid; i < 256 * 32; i += kThreads) lut[(i >> 5) * 64 + (i & 31)] = mm::lut_word(i >> 5);
-    for (int i = tid; i < C::kZeroBytes / 16; i += kThreads)
-      reinterpret_cast<uint4 *>(dyn + C::kOffZero)[i] = make_uint4(0u, 0u, 0u, 0u);
-  }
-  if (tid == 0) {
-    for (int i = 0; i < kNS; ++i) {
-      mbar_init(&bars->full[i], 1 + 32);  // the producer's expect-tx arrival + its 32 lanes' arrivals
-      mbar_init(&bars->empty[i], WD);
-    }
-    bars->abort_ = 0;
-    mbar_fence_init();
-  }
+  setup_cta<SG, WD>(dyn, tid, (WD + 1) * 32);
   __syncthreads();
   // everything below reads what the prep and second-plane kernels wrote
   grid_dep_wait();
@@ -238,7 +422,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     const int wb = SG == 8 ? 52 * c : 4 * ((c * 13) >> 1);
     const int rA = 16 * TL * warp + g;
     // activation slots: this lane's column is slice g & 1 of lane position g >> 1
-    const bool realB = ((g >> 1) == c) && ((g & 1) < kNSl);
+    const bool realB = ((g >> 1) == c) && ((g & 1) < (SG == 8 ? 2 : MB));
     float y[TL][2][MB];
 #pragma unroll
     for (int t = 0; t < TL; ++t)
@@ -250,78 +434,13 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     for (Walk<SG> w(&bp, sc.split, t_begin, t_end); w.valid(); w.next()) {
       const bool ok = __all_sync(0xffffffffu, mm::wait_or_abort(&bars->full[buf], phase, abort_));
       if (!ok) break;
-      const int s = w.s;
-      const int shift = SG == 8 ? 0 : 8 * (s & 1);  // odd 4-group stages are copied from 8 bytes early
-      const unsigned char *p1 = dyn + C::p1_off((int)buf) + shift + wb + rA * C::kBox;
-      const unsigned char *bq =
-          dyn + (realB ? kA2 + C::kOffB + ((int)buf * 2 + (g & 1)) * C::kSlice + c * 16 : C::kOffZero + 16 * ((g >> 1) + 2));
-      const float4 cs = *reinterpret_cast<const float4 *>(dyn + C::kOffCS + (int)buf * kCSStage + c * 16);
-      // accumulators start at -C (slice 0 in columns 2c, slice 1 in 2c + 1)
-      float d[TL][4];
-#pragma unroll
-      for (int t = 0; t < TL; ++t) d[t][0] = d[t][2] = -cs.x, d[t][1] = d[t][3] = -cs.y;
-#pragma unroll
-      for (int i = 0; i < C::kWords; ++i) {
-        uint32_t a[TL][2][10];
-#pragma unroll
-        for (int t = 0; t < TL; ++t)
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-            decode_word(*reinterpret_cast<const uint32_t *>(p1 + (16 * t + 8 * h) * C::kBox + 4 * i), tag, a[t][h]);
-#pragma unroll
-        for (int m = 0; m < 5; ++m) {
-          const int j = 5 * i + m;
-          const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
-          const uint32_t b0 = (j & 1) ? q.z : q.x, b1 = (j & 1) ? q.w : q.y;
-#pragma unroll
-          for (int t = 0; t < TL; ++t)
-            mm::mma16816(d[t], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
-        }
-      }
-      // s1 / off of (row, the lane's groups): the slot holds 8 groups per
-      // row (both halves of an 8-group stage; an odd 4-group stage's at 4)
-      {
-        const unsigned char *so = dyn + kA2 + C::kOffSO + (int)buf * C::kSOSlot;
-#pragma unroll
-        for (int t = 0; t < TL; ++t) {
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int r = rA + 16 * t + 8 * h;
-            if (SG == 8) {
-              // groups 2c, 2c + 1 (columns 2c, 2c + 1) of the one token
-              const __half2 s1 = *reinterpret_cast<const __half2 *>(so + r * 16 + 4 * c);
-              const __half2 of = *reinterpret_cast<const __half2 *>(so + C::kSOHalf + r * 16 + 4 * c);
-              float v = fmaf(__low2float(of), cs.z, y[t][h][0]);
-              v = fmaf(__high2float(of), cs.w, v);
-              v = fmaf(__low2float(s1), d[t][2 * h], v);
-              y[t][h][0] = fmaf(__high2float(s1), d[t][2 * h + 1], v);
-            } else {
-              // group c, tokens 0 and 1 (columns 2c, 2c + 1)
-              const int gl = 2 * (4 * (s & 1) + c);
-              const float s1 = __half2float(*reinterpret_cast<const __half *>(so + r * 16 + gl));
-              const float of = __half2float(*reinterpret_cast<const __half *>(so + C::kSOHalf + r * 16 + gl));
-              y[t][h][0] = fmaf(s1, d[t][2 * h], fmaf(of, cs.z, y[t][h][0]));
-              y[t][h][MB - 1] = fmaf(s1, d[t][2 * h + 1], fmaf(of, cs.w, y[t][h][MB - 1]));
-            }
-          }
-        }
-      }
+      decode_stage<MB, SG, TL>(dyn, (int)buf, w.s, rA, wb, c, g, realB, tag, y);
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->empty[buf]);
       if (w.last_stage()) {
         // sum the four lane positions of each row, add the second plane,
         // write y: the quad's rows (t, h) go to lanes c = (2 t + h) mod 4
-#pragma unroll
-        for (int t = 0; t < TL; ++t)
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int k = 0; k < MB; ++k) {
-              float v = y[t][h][k];
-              v += __shfl_xor_sync(0xffffffffu, v, 1);
-              v += __shfl_xor_sync(0xffffffffu, v, 2);
-              y[t][h][k] = v;
-            }
+        quad_sum<MB, TL>(y);
         const Problem &P = w.P();
         auto store = [&](int n, int k, float v) {
           if (F32)
@@ -387,102 +506,213 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
     uint32_t buf = 0, phase = 0, q = 0;
     int map_pi = -1;
     for (Walk<SG> w(&bp, sc.split, t_begin, t_end); w.valid(); w.next(), ++q) {
-      const Problem &P = w.P();
-      const int s = w.s, n0 = w.n0();
-      const int G = P.K / kGroup;
       int ok = 1;
       if (lane == 0) ok = mm::wait_or_abort(&bars->empty[buf], phase ^ 1u, abort_) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;  // uniform across the warp
-      uint64_t *full = &bars->full[buf];
-      // s1 / off go by tensor copies when their rows are whole 16-byte units
-      // (the prep kernel then built their maps), else by plain loads
-      const bool so_map = (G % 8 == 0) && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 15u) == 0;
-      unsigned char *so = dyn + kA2 + C::kOffSO + (int)buf * C::kSOSlot;
-      const unsigned char *maps = static_cast<const unsigned char *>(P.map());
-      const int g8 = SG == 8 ? s : s >> 1;  // the 8-group box holding the stage
-      if (lane == 0) {
-        if (w.pi != map_pi) {
-          // the problem's tensor maps, written by the prep kernel
-          asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps) : "memory");
-          if (so_map) {
-            asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + 128) : "memory");
-            asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(maps + 256) : "memory");
-          }
-          map_pi = w.pi;
-        }
-        mbar_arrive_expect_tx(full, (uint32_t)(C::kP1Slot + kNSl * C::kSliceG + kCSStage) +
-                                        (so_map ? (uint32_t)C::kSOSlot : 0u));
-        // the stage's plane-1 bytes of the tile's 256 rows from the 16-byte
-        // boundary at or before them (rows past N and bytes past the row's
-        // end arrive as zeros)
-        const int x = SG == 8 ? C::kStageBytes * s : C::kStageBytes * s - 8 * (s & 1);
-        asm volatile(
-            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-                smem_u32(dyn + C::p1_off((int)buf))),
-            "l"(maps), "r"(x), "r"(n0), "r"(smem_u32(full))
-            : "memory");
-#pragma unroll
-        for (int sl = 0; sl < kNSl; ++sl)
-          bulk_g2s(dyn + kA2 + C::kOffB + ((int)buf * 2 + sl) * C::kSlice,
-                   ws_b(P) + ((int64_t)s * 2 + sl) * C::kSliceG, C::kSliceG, full);
-        bulk_g2s(dyn + C::kOffCS + (int)buf * kCSStage, ws_cs(P, MB) + (int64_t)s * kCSStage, kCSStage, full);
-        if (so_map) {
-          asm volatile(
-              "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-                  smem_u32(so)),
-              "l"(maps + 128), "r"(8 * g8), "r"(n0), "r"(smem_u32(full))
-              : "memory");
-          asm volatile(
-              "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-                  smem_u32(so + C::kSOHalf)),
-              "l"(maps + 256), "r"(8 * g8), "r"(n0), "r"(smem_u32(full))
-              : "memory");
-        }
-      }
-      __syncwarp();
-      const int col0 = SG == 8 ? 0 : 4 * (s & 1);  // the stage's first column in the 8-group slot rows
-      if (!so_map && G % 4 == 0 && ((((uintptr_t)P.s1) | ((uintptr_t)P.off)) & 7u) == 0) {
-        // rows of scales in whole 8-byte units (G a multiple of 4): 8-byte
-        // asynchronous copies of each 4-group half of the stage (zero-filled
-        // past G or N); each lane's arrival waits for its own copies
-        const int rows = min(kRows, P.N - n0);
-        for (int r = lane; r < kRows; r += 32) {
-#pragma unroll
-          for (int hh = 0; hh < SG / 4; ++hh) {
-            const int gi = SG * s + 4 * hh;
-            const bool real = r < rows && gi < G;
-            const int64_t o = real ? (int64_t)(n0 + r) * G + gi : 0;
-            const uint32_t dst = smem_u32(so + r * 16 + 2 * (col0 + 4 * hh));
-            asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(P.s1 + o), "r"(real ? 8 : 0)
-                         : "memory");
-            asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst + C::kSOHalf), "l"(P.off + o),
-                         "r"(real ? 8 : 0)
-                         : "memory");
-          }
-        }
-        cp_async_mbar_arrive_noinc(full);  // the lane's arrival, once its copies have landed
-      } else {
-        if (!so_map) {
-          // other shapes: the stage's groups of s1 and off one by one (zeros
-          // past G or N) at their place in each row's 8-group slot
-          const int rows = min(kRows, P.N - n0);
-          __half *d1 = reinterpret_cast<__half *>(so), *d2 = reinterpret_cast<__half *>(so + C::kSOHalf);
-          for (int r = lane; r < rows; r += 32) {
-            const int64_t o = (int64_t)(n0 + r) * G;
-#pragma unroll
-            for (int gg = 0; gg < SG; ++gg) {
-              const int gi = SG * s + gg;
-              d1[r * 8 + col0 + gg] = gi < G ? P.s1[o + gi] : __float2half_rn(0.f);
-              d2[r * 8 + col0 + gg] = gi < G ? P.off[o + gi] : __float2half_rn(0.f);
-            }
-          }
-        }
-        mbar_arrive(full);  // the lanes' arrivals (the barrier counts 1 + 32)
-      }
+      produce_stage<MB, SG>(dyn, bars, (int)buf, w.P(), w.pi, map_pi, w.s, w.n0(), lane);
       if (++buf == (uint32_t)kNS) buf = 0, phase ^= 1u;
     }
     // drain: every issued copy lands before the CTA exits (waited on even
     // after an abort; bounded by the wall-time limit)
+    mm::cp_async_wait<0>();
+    if (lane == 0) {
+      for (uint32_t k = (q > (uint32_t)kNS ? q - kNS : 0); k < q; ++k) mbar_wait(&bars->full[k % kNS], (k / kNS) & 1u);
+    }
+  }
+  __syncthreads();
+}
+
+// ------------------------------------------------------------ sequence
+// Dependency-ordered sequence of problems (one token): problem p + 1 starts
+// only after every CTA has finished problem p, as the layers of a model need
+// (q/k/v, then o, then gate/up, then down, layer after layer; the attention,
+// norms and activation between them are outside this library).  One
+// persistent launch: for each problem every CTA takes its share of the
+// second-plane tiles and then of the 256-row tiles' stage units (tiles cut so
+// that the problem's units cover the CTAs), adding everything into y2 (fp32
+// atomics, zeroed by the prep kernel); a grid-wide barrier (a counter in the
+// workspace, bounded by the wall-time limit) ends the problem, after which
+// every CTA converts its slice of y2 into y.  The producer warp streams the
+// stages without waiting at the barriers (weights do not depend on earlier
+// problems).  barrier_extra > 0 makes every barrier wait for CTAs that do not
+// exist, so that its bounded wait runs out (the failure-path self-test).
+struct SeqWalk {
+  const BatchParams *bp;
+  int cta, ctas, p, unit, u_end, u, nst, tile, s, s_end;
+  __device__ void enter() {
+    const Problem &P = bp->prob[p];
+    const int G = P.K / kGroup, tiles = (P.N + kRows - 1) / kRows;
+    const int64_t share = ((int64_t)tiles * G + ctas - 1) / ctas;
+    const int split = share >= G ? 0 : (int)(share < 1 ? 1 : share);
+    u = unit_parts(P.K, 8, split);
+    nst = nstages(P.K, 8);
+    const int64_t U = (int64_t)tiles * u;
+    unit = (int)(U * cta / ctas);
+    u_end = (int)(U * (cta + 1) / ctas);
+    if (unit < u_end) locate();
+  }
+  __device__ void locate() {
+    tile = unit / u;
+    const int k = unit - tile * u;
+    s = k * nst / u;
+    s_end = (k + 1) * nst / u;
+  }
+  __device__ SeqWalk(const BatchParams *b, int c, int n) : bp(b), cta(c), ctas(n), p(0), unit(0), u_end(0) { enter(); }
+  __device__ const Problem &P() const { return bp->prob[p]; }
+  __device__ bool has_stage() const { return unit < u_end; }
+  __device__ bool unit_end() const { return s + 1 == s_end; }
+  __device__ int n0() const { return tile * kRows; }
+  __device__ void next_stage() {
+    if (++s < s_end) return;
+    if (++unit < u_end) locate();
+  }
+  __device__ bool next_problem() {
+    if (++p >= bp->count) return false;
+    enter();
+    return true;
+  }
+};
+
+__device__ __forceinline__ int ld_acquire(const int32_t *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// A decode warp's share of problem P's second-plane tiles (one token): the
+// CTA's contiguous share of the index's 16-entry tiles, cut among the WD
+// decode warps; runs of tiles of one group go through mm::p2_tiles with the
+// group's activation fragment of the per-group layout.
+template <int WD>
+__device__ __forceinline__ void second_plane_share(const Problem &P, int cta, int ctas, int warp, int lane,
+                                                   uint32_t tag) {
+  const int G = P.K / kGroup, c = lane & 3;
+  const int T2 = __ldg(P.p2idx + G) >> 4;  // tiles (group starts are multiples of 16 entries)
+  const int lo = (int)((int64_t)T2 * cta / ctas), hi = (int)((int64_t)T2 * (cta + 1) / ctas);
+  const int wlo = lo + (hi - lo) * warp / WD, whi = lo + (hi - lo) * (warp + 1) / WD;
+  for (int t = wlo; t < whi;) {
+    // the tile's group: the last g with colptr[g] <= 16 t
+    int g = 0;
+    for (int step = 1 << (31 - __clz(G)); step >= 1; step >>= 1)
+      if (g + step < G && __ldg(P.p2idx + g + step) <= 16 * t) g += step;
+    const int64_t e0 = __ldg(P.p2idx + g);
+    const int n = min(whi, __ldg(P.p2idx + g + 1) >> 4) - t;
+    if (n <= 0) break;  // malformed index: stop rather than loop
+    const unsigned char *Bg = P.wsB + (int64_t)g * mm::kBTok + c * mm::kBLane;
+    uint32_t b[20];
+#pragma unroll
+    for (int cp = 0; cp < mm::kCP; ++cp) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(Bg + cp * 4 * mm::kBLane));
+      b[4 * cp] = v.x, b[4 * cp + 1] = v.y, b[4 * cp + 2] = v.z, b[4 * cp + 3] = v.w;
+    }
+    const float2 Cv = __ldg(reinterpret_cast<const float2 *>(P.wsCS + (int64_t)g * (mm::kCSGroup / 4)));
+    mm::p2_tiles<true, false>(P, 1, g % mm::kStageG, e0, t - (int)(e0 >> 4), n, b, b, Cv, Cv, lane, tag);
+    t += n;
+  }
+}
+
+template <bool F32>
+__global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
+    gemv_seq_kernel(const __grid_constant__ BatchParams bp, int32_t barrier_extra) {
+  constexpr int SG = 8, MB = 1, WD = kWD1, TL = kTL1;
+  using C = Cfg<SG>;
+  constexpr int kNS = C::kNS;
+  extern __shared__ __align__(1024) unsigned char dyn[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (smem_u32(dyn) != kDynShared) {
+    if (tid == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  Bars *bars = reinterpret_cast<Bars *>(dyn + C::kOffBars);
+  volatile int32_t *abort_ = &bars->abort_;
+  setup_cta<SG, WD>(dyn, tid, (WD + 1) * 32);
+  __syncthreads();
+  grid_dep_wait();  // the prep kernel's operands, maps, zeroed y2 and counter
+  int32_t *counter = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(bp.prob[0].map()) + 448);
+
+  if (warp < WD) {
+    // ============================================================ decode
+    const int g = lane >> 2, c = lane & 3;
+    const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
+    const int wb = 52 * c, rA = 16 * TL * warp + g;
+    const bool realB = (g >> 1) == c;
+    float y[TL][2][MB];
+#pragma unroll
+    for (int t = 0; t < TL; ++t) y[t][0][0] = y[t][1][0] = 0.f;
+    uint32_t buf = 0, phase = 0;
+    SeqWalk w(&bp, blockIdx.x, gridDim.x);
+    for (bool more = true; more; more = w.next_problem()) {
+      const Problem &P = w.P();
+      if (P.nnz > 0) second_plane_share<WD>(P, blockIdx.x, gridDim.x, warp, lane, tag);
+      bool ok = true;
+      for (; w.has_stage(); w.next_stage()) {
+        ok = __all_sync(0xffffffffu, mm::wait_or_abort(&bars->full[buf], phase, abort_));
+        if (!ok) break;
+        decode_stage<MB, SG, TL>(dyn, (int)buf, w.s, rA, wb, c, g, realB, tag, y);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->empty[buf]);
+        if (w.unit_end()) {
+          quad_sum<MB, TL>(y);
+#pragma unroll
+          for (int t = 0; t < TL; ++t)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int n = w.n0() + rA + 16 * t + 8 * h;
+              if (((2 * t + h) & 3) == c && n < P.N) atomicAdd(P.y2() + n, y[t][h][0]);
+              y[t][h][0] = 0.f;
+            }
+        }
+        if (++buf == (uint32_t)kNS) buf = 0, phase ^= 1u;
+      }
+      // the problem's barrier: every CTA's additions into y2 are done
+      named_bar(1, WD * 32);
+      if (warp == 0 && lane == 0 && ok && !*abort_) {
+        __threadfence();
+        atomicAdd(counter, 1);
+        const int target = (w.p + 1) * ((int)gridDim.x + barrier_extra);
+        const uint64_t t0 = global_ns();
+        while (ld_acquire(counter) < target) {
+          if (*abort_) break;
+          if (global_ns() - t0 > kWaitLimitNs) {
+            atomicOr(&g_tq_device_status, kStatusTimeout);
+            *abort_ = 1;
+            break;
+          }
+          __nanosleep(128);
+        }
+        __threadfence();
+      }
+      // stop together: the flag may be raised (by the producer) while
+      // the warps read it, so they decide by one reduction over the barrier
+      if (named_bar_any(1, WD * 32, *abort_ != 0)) break;
+      // this CTA's slice of the problem's output
+      const int r0 = (int)((int64_t)P.N * blockIdx.x / gridDim.x), r1 = (int)((int64_t)P.N * (blockIdx.x + 1) / gridDim.x);
+      for (int n = r0 + warp * 32 + lane; n < r1; n += WD * 32) {
+        const float v = __ldcg(P.y2() + n);
+        if (F32)
+          static_cast<float *>(P.y)[n] = v;
+        else
+          static_cast<__half *>(P.y)[n] = __float2half_rn(v);
+      }
+    }
+  } else if (warp == WD) {
+    // ========================================================== producer
+    uint32_t buf = 0, phase = 0, q = 0;
+    int map_pi = -1;
+    SeqWalk w(&bp, blockIdx.x, gridDim.x);
+    bool ok = true;
+    for (bool more = true; more && ok; more = w.next_problem()) {
+      for (; w.has_stage(); w.next_stage(), ++q) {
+        int r = 1;
+        if (lane == 0) r = mm::wait_or_abort(&bars->empty[buf], phase ^ 1u, abort_) ? 1 : 0;
+        if (!__shfl_sync(0xffffffffu, r, 0)) {
+          ok = false;
+          break;
+        }
+        produce_stage<MB, SG>(dyn, bars, (int)buf, w.P(), w.p, map_pi, w.s, w.n0(), lane);
+        if (++buf == (uint32_t)kNS) buf = 0, phase ^= 1u;
+      }
+    }
     mm::cp_async_wait<0>();
     if (lane == 0) {
       for (uint32_t k = (q > (uint32_t)kNS ? q - kNS : 0); k < q; ++k) mbar_wait(&bars->full[k % kNS], (k / kNS) & 1u);
@@ -568,6 +798,27 @@ cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, bp, sc);
+}
+
+// The dependency-ordered sequence kernel (one token), launched
+// programmatically after its prep kernel.
+cudaError_t launch_gemv_seq(const BatchParams &bp, int num_sms, int barrier_extra, cudaStream_t s) {
+  if (bp.M != 1 || bp.count < 1) return cudaErrorInvalidValue;
+  const int ctas = std::min(num_sms, 256);
+  auto kern = bp.out_f32 ? g4::gemv_seq_kernel<true> : g4::gemv_seq_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, g4::kDynBytes);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(ctas);
+  cfg.blockDim = dim3((g4::kWD1 + 1) * 32);
+  cfg.dynamicSmemBytes = g4::kDynBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, bp, (int32_t)barrier_extra);
 }
 
 }  // namespace tq

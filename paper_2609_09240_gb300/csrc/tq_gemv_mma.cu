@@ -62,19 +62,13 @@
 
 #include "tq_common.cuh"
 #include "tq_decode_ops.cuh"
+#include "tq_p2_tile.cuh"
 #include "tq_sm100.cuh"
 
 namespace tq {
 namespace mm {
 
 constexpr int kRows = 128;        // tile rows (8 m16 tiles)
-constexpr int kStageG = 8;        // groups per stage
-constexpr int kStageBytes = 208;  // plane-1 bytes per row per stage (13 x 16)
-constexpr int kChunks = 10;       // k16 chunks per group (160 K slots)
-constexpr int kCP = 5;            // chunk pairs
-constexpr int kBLane = 16;        // B bytes per (chunk pair, token, lane position)
-constexpr int kBTok = kCP * 4 * kBLane;  // 320 B of B per group and token
-constexpr int kCSGroup = 64;             // C[8], S[8] floats per group and 8-token tile
 constexpr int kWarpsP1 = 8, kWarpProd = 8;
 constexpr int kThreads = 9 * 32;
 constexpr int kBytesSlot = kRows * kStageBytes;           // 26624
@@ -116,42 +110,7 @@ struct Sched {
   int32_t cta_tile[257];
 };
 
-// Window of a group: the aligned words of the stage row that cover its 26
-// bytes, words wstart .. wstart + 6 with wstart = 26 GL / 4 (GL = the
-// group's index in its stage); the group starts o = 26 GL % 4 bytes into
-// the first.  Lane c of a row owns the window words whose stage-row index
-// is c mod 4 (two words: the first at or after wstart, and the one four
-// words later; bytes outside the group get zero activations).
-__host__ __device__ constexpr int win_start(int GL) { return (26 * GL) / 4; }
-// Stage-row word index of lane c's first window word.
-__host__ __device__ constexpr int first_word(int GL, int c) {
-  return win_start(GL) + ((c - win_start(GL)) % 4 + 4) % 4;
-}
 
-// The 20 A words of one row and group from the lane's two window words
-// (lane-replicated table; `tag` = table base | lane * 4, so that one PRMT
-// yields the entry's address): W, W' of bytes 0..3 of the first word, then
-// of the second, then the four V words, each made by one PRMT of a word's
-// byte pair with the fifth slot's exponent byte 0x44.
-__device__ __forceinline__ void decode_words(uint32_t w0, uint32_t w1, uint32_t tag, uint32_t *a) {
-  uint32_t r[8];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    r[k] = prmt(w0, tag, 0x7604u | (k << 4));
-    r[4 + k] = prmt(w1, tag, 0x7604u | (k << 4));
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t w = lut_load(r[i]);
-    a[2 * i] = w;
-    a[2 * i + 1] = w_prime(w);
-  }
-  const uint32_t e44 = 0x44444444u;
-  a[16] = prmt(w0, e44, 0x4140u);
-  a[17] = prmt(w0, e44, 0x4342u);
-  a[18] = prmt(w1, e44, 0x4140u);
-  a[19] = prmt(w1, e44, 0x4342u);
-}
 
 // The same from a compact (not replicated) 256-word table at `lut`.
 __device__ __forceinline__ void decode_words_compact(uint32_t w0, uint32_t w1, const uint32_t *lut, uint32_t *a) {
@@ -171,14 +130,6 @@ __device__ __forceinline__ void decode_words_compact(uint32_t w0, uint32_t w1, c
   for (int i = 0; i < 4; ++i) a[16 + i] = 0x44004400u | v[2 * i] | (v[2 * i + 1] << 16);
 }
 
-// The MMAs of one group: rows g (aL) and g + 8 (aH), B words of this lane
-// (b[2j], b[2j+1] for chunk j), one accumulation chain (measured faster than
-// two or four chains summed at the end: the adds cost more than the latency).
-__device__ __forceinline__ void group_mma(const uint32_t *aL, const uint32_t *aH, const uint32_t *b, float *d) {
-  mma16816_z(d, aL[0], aH[0], aL[1], aH[1], b[0], b[1]);
-#pragma unroll
-  for (int j = 1; j < kChunks; ++j) mma16816(d, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
-}
 
 // Iterates (tile, stage) in the CTA's order.
 struct Walk {
@@ -228,7 +179,9 @@ static_assert(sizeof(CUtensorMap) == 8 * sizeof(uint4), "tensor map size");
 // indexed second-plane kernel's unit counter.
 constexpr int kMapSlotBytes = 512;
 constexpr int kMapS1 = 128, kMapOff = 256, kCounterOff = 384;
-static_assert(kCounterOff + 4 <= kMapSlotBytes, "map slot");
+// problem 0's slot also holds the sequence kernel's problem barrier counter
+constexpr int kSeqCounterOff = 448;
+static_assert(kSeqCounterOff + 4 <= kMapSlotBytes, "map slot");
 
 // ------------------------------------------------------------------ prep
 // Activation slots of one group for the one-group-per-lane kernel (M <= 2,
@@ -283,12 +236,17 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   // the next kernel (second plane or main) may start its own set-up now
   grid_dep_launch_next();
   const bool g4_shared = bp.M <= 2 && bp.g4_split > 0;  // split tiles add their partial sums into y2
-  if (P.nnz > 0 || g4_shared) {
+  // (the sequence kernel, g4_split < 0, adds every partial sum into y2)
+  if (P.nnz > 0 || g4_shared || bp.g4_split < 0) {
     // y2 starts at zero (the indexed second-plane kernel adds into it)
     float *y2 = P.y2();
     const int64_t n = (int64_t)P.N * bp.M;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
       y2[i] = 0.f;
+  }
+  if (bp.g4_split < 0 && p == 0 && blockIdx.x == 0 && threadIdx.x == 0) {
+    // the sequence kernel's problem barrier counter starts at zero
+    *reinterpret_cast<int32_t *>(static_cast<unsigned char *>(P.map()) + kSeqCounterOff) = 0;
   }
   if (g4_shared) {
     // the arrival counters of split tiles start at zero
@@ -979,7 +937,6 @@ __global__ void __launch_bounds__(kQThreads, 1)
 // threads per CTA: 1024 (64 registers) for up to 8 tokens, 768 for the
 // second token tile's extra fragment registers
 __host__ __device__ constexpr int c_threads(bool two) { return two ? 768 : 1024; }
-constexpr int kCDepth = 2;                        // tiles in flight per warp (in registers)
 constexpr int kCDynBytes2 = kArena1 + kLutBytes;  // the table of codes at its fixed address
 constexpr int kCUnitTiles = 32;                   // target tiles per unit
 
@@ -990,10 +947,6 @@ struct CBase {
   int32_t base[TQ_MAX_BATCH + 1];  // first unit of problem p (base[count]: all units)
 };
 
-__device__ __forceinline__ int64_t c_capacity(int K, int64_t nnz) {
-  return (nnz + 15 * (int64_t)(K / kGroup) + 15) & ~(int64_t)15;
-}
-__device__ __forceinline__ int64_t c_slot_off(int K) { return ((int64_t)(K / kGroup + 1) * 4 + 127) & ~(int64_t)127; }
 // Units per group: the mean tiles per group over kCUnitTiles, rounded up, 1 .. 32.
 __host__ __device__ __forceinline__ int c_parts(int K, int64_t nnz) {
   const int64_t per = (int64_t)(K / kGroup) * 16 * kCUnitTiles;
@@ -1061,70 +1014,7 @@ __global__ void __launch_bounds__(c_threads(TWO), 1)
       }
       Cv2 = __ldg(reinterpret_cast<const float2 *>(csg + 16 + 2 * c));
     }
-    // lane c's window words jw and jw + 4 are slot words 2 jw, 2 jw + 1; the row is the second
-    // word of the lane with jw = 3, s2 a half of the first word of jw = 0 (record at byte 2)
-    // or of the second word of jw = 2 (record at byte 0)
-    const int ws = win_start(GL), jw = (c - ws) & 3, odd = GL & 1;
-    const int c_row = quad + ((3 + ws) & 3), c_s2 = quad + (((odd ? 0 : 2) + ws) & 3);
-    const unsigned char *src = reinterpret_cast<const unsigned char *>(P.p2idx) + c_slot_off(P.K) +
-                               (e0 + 16 * (int64_t)t0 + g16) * 32 + jw * 8;
-    float *y2 = P.y2();
-    uint2 pre[kCDepth][2];
-#pragma unroll
-    for (int k = 0; k < kCDepth; ++k) {
-      pre[k][0] = pre[k][1] = make_uint2(0u, 0u);
-      if (k < n) {
-        pre[k][0] = __ldg(reinterpret_cast<const uint2 *>(src + k * 512));
-        pre[k][1] = __ldg(reinterpret_cast<const uint2 *>(src + k * 512 + 256));
-      }
-    }
-    for (int t = 0; t < n; t += kCDepth) {
-#pragma unroll
-      for (int k = 0; k < kCDepth; ++k) {
-        if (t + k < n) {
-          const uint2 r0 = pre[k][0], r1 = pre[k][1];
-          if (t + k + kCDepth < n) {
-            const unsigned char *p = src + (int64_t)(t + k + kCDepth) * 512;
-            pre[k][0] = __ldg(reinterpret_cast<const uint2 *>(p));
-            pre[k][1] = __ldg(reinterpret_cast<const uint2 *>(p + 256));
-          }
-          uint32_t aL[20], aH[20];
-          decode_words(r0.x, r0.y, tag, aL);
-          decode_words(r1.x, r1.y, tag, aH);
-          float d[4], d2[4] = {0.f, 0.f, 0.f, 0.f};
-          group_mma(aL, aH, b, d);
-          if (TWO) group_mma(aL, aH, b2, d2);
-          const uint32_t sw0 = __shfl_sync(0xffffffffu, odd ? r0.x : r0.y, c_s2);
-          const uint32_t sw1 = __shfl_sync(0xffffffffu, odd ? r1.x : r1.y, c_s2);
-          const float s2v0 = odd ? half_of<false>(sw0) : half_of<true>(sw0);
-          const float s2v1 = odd ? half_of<false>(sw1) : half_of<true>(sw1);
-          if (ONE) {
-            // every column of D is token 0: the lane holding the rows adds
-            if (lane == c_row) {
-              const int n0 = (int)r0.y, n1 = (int)r1.y;
-              if (n0 >= 0 && n0 < P.N) atomicAdd(&y2[n0], s2v0 * (d[0] - Cv.x));
-              if (n1 >= 0 && n1 < P.N) atomicAdd(&y2[n1], s2v1 * (d[2] - Cv.x));
-            }
-          } else {
-            const int rows[2] = {__shfl_sync(0xffffffffu, (int)r0.y, c_row),
-                                 __shfl_sync(0xffffffffu, (int)r1.y, c_row)};
-            const float s2v[2] = {s2v0, s2v1};
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int nr = rows[h];
-              if (nr < 0 || nr >= P.N) continue;
-#pragma unroll
-              for (int ii = 0; ii < 2; ++ii) {
-                const int m = 2 * c + ii;
-                if (m < MB) atomicAdd(&y2[(int64_t)nr * MB + m], s2v[h] * (d[2 * h + ii] - (ii ? Cv.y : Cv.x)));
-                if (TWO && 8 + m < MB)
-                  atomicAdd(&y2[(int64_t)nr * MB + 8 + m], s2v[h] * (d2[2 * h + ii] - (ii ? Cv2.y : Cv2.x)));
-              }
-            }
-          }
-        }
-      }
-    }
+    p2_tiles<ONE, TWO>(P, MB, GL, e0, t0, n, b, b2, Cv, Cv2, lane, tag);
   }
 }
 
@@ -1434,6 +1324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // -------------------------------------------------------------- launcher
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s);
 int g4_split_for(const BatchParams &bp, int num_sms);
+cudaError_t launch_gemv_seq(const BatchParams &bp, int num_sms, int barrier_extra, cudaStream_t s);
 
 static int num_sms_mm() {
   static int n = 0;
@@ -1534,6 +1425,40 @@ static int distinct_row_lengths(const BatchParams &bp, int first, int last, int 
   return n;
 }
 
+// The tensor-map templates of a batch (one per distinct kind and size) and
+// each problem's template indices.  g4path: the one-group-per-lane layouts
+// (kinds 2/4 and 3) instead of the general kernel's (0 and 1).
+static cudaError_t build_templates(const BatchParams &bp, bool g4path, mm::MapTemplates &mt) {
+  int64_t keys[mm::kMaxMapTemplates] = {};
+  int nt = 0;
+  auto slot = [&](int kind, int64_t len, const void *addr, int N) -> int {
+    const int64_t key = ((int64_t)N << 32) | (len << 3) | kind;
+    int k = 0;
+    while (k < nt && keys[k] != key) ++k;
+    if (k == nt) {
+      if (nt == mm::kMaxMapTemplates) return -1;  // launch_mm splits such batches
+      CUtensorMap enc;
+      if (!map_template(kind, len, addr, N, &enc)) return -2;
+      std::memcpy(&mt.t[nt][0], &enc, sizeof(enc));
+      keys[nt++] = key;
+    }
+    return k;
+  };
+  for (int i = 0; i < bp.count; ++i) {
+    const Problem &P = bp.prob[i];
+    const int k1 = slot(g4path ? (bp.M == 1 ? 4 : 2) : 0, row_bytes_of(P.K), P.plane1, P.N);
+    if (k1 < 0) return k1 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
+    mt.idx[i] = (uint8_t)k1;
+    mt.idx_so[i] = mm::kNoMap;
+    if (scales_by_map(P)) {
+      const int k2 = slot(g4path ? 3 : 1, P.K / kGroup, P.s1, P.N);
+      if (k2 < 0) return k2 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
+      mt.idx_so[i] = (uint8_t)k2;
+    }
+  }
+  return cudaSuccess;
+}
+
 template <bool F32>
 static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s);
 
@@ -1601,35 +1526,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   // one or two tokens: the one-group-per-lane kernel (tq_gemv_g4.cu)
   const bool g4path = bp.M <= 2;
   thread_local mm::MapTemplates mt;
-  {
-    int64_t keys[mm::kMaxMapTemplates] = {};
-    int nt = 0;
-    auto slot = [&](int kind, int64_t len, const void *addr, int N) -> int {
-      const int64_t key = ((int64_t)N << 32) | (len << 3) | kind;
-      int k = 0;
-      while (k < nt && keys[k] != key) ++k;
-      if (k == nt) {
-        if (nt == mm::kMaxMapTemplates) return -1;  // launch_mm splits such batches
-        CUtensorMap enc;
-        if (!map_template(kind, len, addr, N, &enc)) return -2;
-        std::memcpy(&mt.t[nt][0], &enc, sizeof(enc));
-        keys[nt++] = key;
-      }
-      return k;
-    };
-    for (int i = 0; i < bp.count; ++i) {
-      const Problem &P = bp.prob[i];
-      const int k1 = slot(g4path ? (bp.M == 1 ? 4 : 2) : 0, row_bytes_of(P.K), P.plane1, P.N);
-      if (k1 < 0) return k1 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
-      mt.idx[i] = (uint8_t)k1;
-      mt.idx_so[i] = mm::kNoMap;
-      if (scales_by_map(P)) {
-        const int k2 = slot(g4path ? 3 : 1, P.K / kGroup, P.s1, P.N);
-        if (k2 < 0) return k2 == -1 ? cudaErrorNotSupported : cudaErrorInvalidValue;
-        mt.idx_so[i] = (uint8_t)k2;
-      }
-    }
-  }
+  if (cudaError_t e = build_templates(bp, g4path, mt)) return e;
   // second plane: the indexed kernel when every weight with a second plane
   // has its index, else the span kernel (or, for rows of more than
   // kQMaxW salience words, the per-tile one)
@@ -1694,6 +1591,30 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   main_kern<<<ctas, mm::kThreads, mm::kDynBytes, s>>>(bp, sc);
   return cudaGetLastError();
+}
+
+// The dependency-ordered sequence (one token): prep (operands of every
+// problem, maps, zeroed y2 and barrier counter), then the persistent
+// sequence kernel (tq_gemv_g4.cu).  Every problem with a second plane must
+// carry its index.  A sequence's problems must fit one set of tensor-map
+// templates (cudaErrorNotSupported otherwise).
+cudaError_t launch_gemv_sequence(const BatchParams &bp_in, int barrier_extra, cudaStream_t s) {
+  if (bp_in.M != 1) return cudaErrorInvalidValue;
+  thread_local BatchParams bp;
+  bp = bp_in;
+  bp.g4_split = -1;  // sequence mode: y2 and the barrier counter zeroed by prep
+  int gmax = 0;
+  for (int i = 0; i < bp.count; ++i) {
+    gmax = max(gmax, bp.prob[i].K / kGroup);
+    if (bp.prob[i].nnz > 0 && !bp.prob[i].p2idx) return cudaErrorInvalidValue;
+  }
+  thread_local mm::MapTemplates mt;
+  if (cudaError_t e = build_templates(bp, true, mt)) return e;
+  const int gtasks = g4::stage_groups(1) * ((gmax + g4::stage_groups(1) - 1) / g4::stage_groups(1));
+  mm::gemv_mma_prep_kernel<<<dim3((gtasks + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, nullptr);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_gemv_seq(bp, num_sms_mm(), barrier_extra, s);
 }
 
 cudaError_t launch_gemv_mma(const BatchParams &bp, cudaStream_t s) {

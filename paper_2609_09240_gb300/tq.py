@@ -102,6 +102,10 @@ def lib():
             L.tq_linear_static.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp]
             L.tq_linear_batched.restype = ctypes.c_int
             L.tq_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
+            L.tq_linear_sequence.restype = ctypes.c_int
+            L.tq_linear_sequence.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
+            L.tq_sequence_selftest.restype = ctypes.c_int
+            L.tq_sequence_selftest.argtypes = [i32, ctypes.POINTER(tq_problem), vp, sz, vp]
             L.tq_ternarize_workspace_bytes.restype = sz
             L.tq_ternarize_workspace_bytes.argtypes = [i32, i32]
             L.tq_ternarize.restype = ctypes.c_int
@@ -540,3 +544,17 @@ class Batch:
 def tq_linear_batched(batch: Batch, stream=None):
     _check(lib().tq_linear_batched(batch.M, len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(),
                                    _stream(stream)), "tq_linear_batched")
+
+
+def tq_linear_sequence(batch: Batch, stream=None):
+    """The batch's problems in order, each complete before the next starts
+    (one persistent launch; M must be 1)."""
+    _check(lib().tq_linear_sequence(batch.M, len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(),
+                                    _stream(stream)), "tq_linear_sequence")
+
+
+def tq_sequence_selftest(batch: Batch, stream=None):
+    """Runs the sequence kernel with a problem barrier that cannot complete
+    (its bounded wait runs out; the device status then reports the timeout)."""
+    _check(lib().tq_sequence_selftest(len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(), _stream(stream)),
+           "tq_sequence_selftest")

@@ -32,3 +32,32 @@ def test_bounded_wait_runs_out_and_reports():
     H.device_status_ok()
     y_ref, a_ref = H.oracle_ref(w, x)
     H.assert_close(y.cpu().numpy(), y_ref, a_ref)
+
+
+def test_sequence_barrier_wait_runs_out_and_reports():
+    """The dependency-ordered sequence kernel's problem barrier, made to wait
+    for one CTA more than were launched: its bounded wait runs out (no
+    fault), the status word reports the timeout, every CTA leaves, and a
+    normal sequence afterwards matches the oracle."""
+    import gpu_helpers as H
+    from paper_2609_09240_gb300 import tq
+    shapes = [(512, 1024), (300, 2560)]
+    items, refs = [], []
+    for i, (N, K) in enumerate(shapes):
+        w = wl.gen_weights(N, K, 0.1, config=11, proj=i)
+        xb = wl.gen_x(1, K, config=11, proj=i)
+        refs.append(H.oracle_ref(w, xb))
+        items.append((H.pack_on_gpu(w), H.dev(xb), torch.empty((1, N), dtype=torch.float16, device="cuda")))
+    batch = tq.Batch(1, items)
+    tq.tq_get_device_status(clear=True)
+    torch.cuda.synchronize()
+    t0 = time.time()
+    tq.tq_sequence_selftest(batch)
+    torch.cuda.synchronize()
+    dt = time.time() - t0
+    assert tq.tq_get_device_status(clear=True) & 1
+    assert 1.5 < dt < 60, dt
+    tq.tq_linear_sequence(batch)
+    H.device_status_ok()
+    for (_, _, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
