@@ -214,3 +214,43 @@ def gen_x_torch(M: int, K: int, device, seed: int):
     g = torch.Generator(device=device)
     g.manual_seed(seed)
     return torch.randn((M, K), generator=g, device=device).half()
+
+
+# ------------------------------------------------------ element-wise masks
+# The paper's recorded projection: four disjoint salience masks with orders
+# [2, 2, 1, 1] covering 0.5 %, 3.1 %, 10.0 % and 86.5 % of the weights (the
+# printed coverages add to 100.1 %; the largest is taken as the rest).
+EW_ORDERS = (2, 2, 1, 1)
+EW_COVERAGE = (0.005, 0.031, 0.100)
+TENSOR_MASK, TENSOR_MU, TENSOR_A0, TENSOR_A1 = range(8, 12)
+
+
+@dataclass
+class EwWeights:
+    """Inputs of one projection in the element-wise four-mask form (host numpy)."""
+    N: int
+    K: int
+    T0: np.ndarray    # int8 [N][K]
+    T1: np.ndarray    # int8 [N][K], 0 wherever the element's mask has order 1
+    mask: np.ndarray  # uint8 [N][K], mask id 0..3 of every element
+    mu: np.ndarray    # uint16 fp16 bits [N][4]
+    a0: np.ndarray    # uint16 fp16 bits [N][4]
+    a1: np.ndarray    # uint16 fp16 bits [N][2] (masks 0 and 1)
+
+
+def gen_ew_weights(N: int, K: int, config: int = 0, layer: int = 0, proj: int = 0, seed: int = 0,
+                   coverage=EW_COVERAGE) -> EwWeights:
+    """Mask ids i.i.d. per element with the recorded coverages (mask 3 the
+    rest); T0, T1 i.i.d. {-1, 0, +1} at 0.3 / 0.4 / 0.3, T1 zero outside the
+    order-2 masks; mu ~ Normal(0, 1e-3), alpha0 and alpha1 ~ lognormal(-4,
+    0.5), all rounded to fp16."""
+    u = _rng(seed, config, layer, proj, TENSOR_MASK).random((N, K))
+    c = np.cumsum(coverage)
+    mask = (u >= c[0]).astype(np.uint8) + (u >= c[1]).astype(np.uint8) + (u >= c[2]).astype(np.uint8)
+    T0 = _trits(_rng(seed, config, layer, proj, TENSOR_T1), (N, K))
+    T1 = _trits(_rng(seed, config, layer, proj, TENSOR_T2), (N, K))
+    T1 *= (mask <= 1).astype(np.int8)
+    mu = _fp16_bits(_rng(seed, config, layer, proj, TENSOR_MU).normal(0.0, 1e-3, (N, 4)))
+    a0 = _fp16_bits(_rng(seed, config, layer, proj, TENSOR_A0).lognormal(-4.0, 0.5, (N, 4)))
+    a1 = _fp16_bits(_rng(seed, config, layer, proj, TENSOR_A1).lognormal(-4.0, 0.5, (N, 2)))
+    return EwWeights(N, K, T0, T1, mask, mu, a0, a1)
