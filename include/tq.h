@@ -356,6 +356,67 @@ TQ_API tq_status tq_sequence_selftest(int32_t count, const tq_problem *problems,
                                       size_t workspace_bytes, void *stream);
 
 /* ---------------------------------------------------------------------
+ * Element-wise four-mask representation (paper "Model and Representation":
+ * four disjoint salience masks, num_mask = 4, orders = [2, 2, 1, 1], and
+ * W-hat = (mu + alpha0 T0 + alpha1 T1) (.) M).  Every element (n, k) has a
+ * mask id m in 0..3; its weight is
+ *   mu[n][m] + alpha0[n][m] T0[n][k] + alpha1[n][m] T1[n][k],
+ * with alpha1 and T1 only for the order-2 masks 0 and 1 (T1 = 0 on the
+ * elements of masks 2 and 3).  The paper gives no storage layout; this
+ * library's:
+ *   mask: uint32 [N][K/16], element k's id in bits 2 (k mod 16) and
+ *         2 (k mod 16) + 1 of word k / 16;
+ *   plane1: T0 of every element in tq_weight's plane-1 layout;
+ *   plane2: per row, the T1 trits of the row's order-2 elements in increasing
+ *         k, five per byte (base 3 as plane 1, the row's last byte padded
+ *         with digit 1), row n's bytes from byte p2rowptr[n];
+ *   mu, alpha0: fp16 [N][4]; alpha1: fp16 [N][2].
+ * All device memory owned by the caller; K a multiple of 128. */
+typedef struct {
+  int32_t N, K;
+  const uint32_t *mask;
+  const uint8_t *plane1;    /* 16-byte aligned */
+  const int32_t *p2rowptr;  /* [N + 1] */
+  const uint8_t *plane2;    /* [p2rowptr[N]] bytes; may be NULL when that is 0 */
+  const uint16_t *mu;
+  const uint16_t *alpha0;
+  const uint16_t *alpha1;
+} tq_ew_weight;
+
+/* p2rowptr[N + 1] from the mask ids (uint8 [N][K], 0..3): bytes per row =
+ * ceil(order-2 elements / 5), prefix-summed.  Ids above 3 set
+ * TQ_DATA_BAD_CODE in *d_status.  The caller reads p2rowptr[N] to size
+ * plane 2. */
+TQ_API tq_status tq_ew_rowptr(int32_t N, int32_t K, const uint8_t *mask_ids, int32_t *p2rowptr, uint32_t *d_status,
+                              void *stream);
+/* int8 T0, T1 [N][K] and mask ids -> mask plane, plane 1, plane 2 (with
+ * p2rowptr from tq_ew_rowptr).  Data errors in *d_status: TQ_DATA_BAD_CODE
+ * (a code outside {-1, 0, 1} or an id above 3), TQ_DATA_T2_OUTSIDE (T1
+ * nonzero on an order-1 element), TQ_DATA_BAD_ROWPTR (p2rowptr does not
+ * match the mask ids). */
+TQ_API tq_status tq_ew_pack(int32_t N, int32_t K, const int8_t *T0, const int8_t *T1, const uint8_t *mask_ids,
+                            const int32_t *p2rowptr, uint32_t *mask, uint8_t *plane1, uint8_t *plane2,
+                            uint32_t *d_status, void *stream);
+/* The inverse: T0, T1 (int8 [N][K]) and mask ids (uint8 [N][K]); bytes
+ * above 242, pad digits other than 1 and pad bytes other than 0 are
+ * reported as in tq_unpack. */
+TQ_API tq_status tq_ew_unpack(int32_t N, int32_t K, const uint32_t *mask, const uint8_t *plane1,
+                              const int32_t *p2rowptr, const uint8_t *plane2, int8_t *T0, int8_t *T1,
+                              uint8_t *mask_ids, uint32_t *d_status, void *stream);
+/* Workspace of tq_ew_linear (per-call views of alpha0 / mu of mask 3 for
+ * the plane-1 pass, its fp32 result and the decode path's workspace). */
+TQ_API size_t tq_ew_workspace_bytes(int32_t M, int32_t N, int32_t K);
+/* y = x W-hat^T for the element-wise form, x fp16 [M][K] (16-byte aligned),
+ * y fp16 [M][N] (tq_ew_linear_f32out: fp32).  Plane 1 with mask 3's
+ * parameters runs through tq_linear's kernels; a second kernel adds, per
+ * row, the elements of masks 0..2 and writes y.  The fp32 sums are added in
+ * a fixed order. */
+TQ_API tq_status tq_ew_linear(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, uint16_t *y,
+                              void *workspace, size_t workspace_bytes, void *stream);
+TQ_API tq_status tq_ew_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x,
+                                     float *y, void *workspace, size_t workspace_bytes, void *stream);
+
+/* ---------------------------------------------------------------------
  * Allocation-free variant (no counterpart in the paper; an integration aid).
  *
  * tq_linear_static is tq_linear with its workspace taken from a scratch

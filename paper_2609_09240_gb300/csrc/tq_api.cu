@@ -22,6 +22,17 @@ cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *pl
                           uint32_t *status, cudaStream_t s);
 cudaError_t launch_gemv_mma(const BatchParams &p, cudaStream_t s);
 cudaError_t launch_gemv_sequence(const BatchParams &bp, int barrier_extra, cudaStream_t s);
+cudaError_t launch_ew_rowptr(int N, int K, const uint8_t *mask, int32_t *rowptr, uint32_t *status, cudaStream_t s);
+cudaError_t launch_ew_pack(int N, int K, const int8_t *T0, const int8_t *T1, const uint8_t *mask,
+                           const int32_t *rowptr, uint32_t *mplane, uint8_t *plane1, uint8_t *plane2,
+                           uint32_t *status, cudaStream_t s);
+cudaError_t launch_ew_unpack(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
+                             const uint8_t *plane2, int8_t *T0, int8_t *T1, uint8_t *mask, uint32_t *status,
+                             cudaStream_t s);
+cudaError_t launch_ew_views(int N, int K, const uint16_t *mu, const uint16_t *a0, uint16_t *s1v, uint16_t *offv,
+                            uint32_t *salv, int32_t *rpv, cudaStream_t s);
+cudaError_t launch_ew_correct(int M, int N, int K, const tq_ew_weight *w, const uint16_t *x, const float *ydense,
+                              void *y, bool f32, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
@@ -405,6 +416,108 @@ tq_status tq_linear_sequence(int32_t M, int32_t count, const tq_problem *problem
 tq_status tq_sequence_selftest(int32_t count, const tq_problem *problems, void *workspace, size_t workspace_bytes,
                                void *stream) {
   return run_sequence(1, count, problems, workspace, workspace_bytes, 1, (cudaStream_t)stream);
+}
+
+}  // extern "C"
+
+namespace {
+// Workspace parts of tq_ew_linear, each 256-byte padded: the s1 and off
+// views [N][G] fp16, the views' zero salience words and rowptr, the fp32
+// result of the plane-1 pass [M][N], the decode path's workspace.
+struct EwParts {
+  size_t s1v, offv, salv, rpv, yd, dec, total;
+};
+EwParts ew_parts(int32_t M, int32_t N, int32_t K) {
+  EwParts p;
+  const size_t G = (size_t)(K / TQ_GROUP), W = (size_t)sal_words_of(K);
+  p.s1v = 0;
+  p.offv = p.s1v + pad256((size_t)N * G * 2);
+  p.salv = p.offv + pad256((size_t)N * G * 2);
+  p.rpv = p.salv + pad256((size_t)N * W * 4);
+  p.yd = p.rpv + pad256(((size_t)N + 1) * 4);
+  p.dec = p.yd + pad256((size_t)M * N * 4);
+  p.total = p.dec + call_ws_bytes(M, N, K);
+  return p;
+}
+
+tq_status ew_linear_impl(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, void *y,
+                         bool f32, void *ws, size_t ws_bytes, cudaStream_t s) {
+  if (M < 1) return TQ_ERR_SHAPE;
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!w || !x || !y || !ws) return TQ_ERR_NULL;
+  if (w->N != N || w->K != K) return TQ_ERR_SHAPE;
+  if (!w->mask || !w->plane1 || !w->p2rowptr || !w->mu || !w->alpha0 || !w->alpha1) return TQ_ERR_NULL;
+  if (!aligned16(w->plane1) || !aligned16(x) || ((uintptr_t)ws & 255u) || ((uintptr_t)w->mask & 3u) ||
+      ((uintptr_t)w->p2rowptr & 3u) || !aligned2(w->mu) || !aligned2(w->alpha0) || !aligned2(w->alpha1))
+    return TQ_ERR_ALIGN;
+  if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
+  const EwParts p = ew_parts(M, N, K);
+  if (ws_bytes < p.total) return TQ_ERR_SHAPE;
+  unsigned char *b = static_cast<unsigned char *>(ws);
+  uint16_t *s1v = reinterpret_cast<uint16_t *>(b + p.s1v), *offv = reinterpret_cast<uint16_t *>(b + p.offv);
+  uint32_t *salv = reinterpret_cast<uint32_t *>(b + p.salv);
+  int32_t *rpv = reinterpret_cast<int32_t *>(b + p.rpv);
+  float *yd = reinterpret_cast<float *>(b + p.yd);
+  if (tq_status st = from_cuda(launch_ew_views(N, K, w->mu, w->alpha0, s1v, offv, salv, rpv, s))) return st;
+  // plane 1 with mask 3's parameters in every group, no second plane
+  tq_weight tw;
+  memset(&tw, 0, sizeof(tw));
+  tw.N = N;
+  tw.K = K;
+  tw.group = TQ_GROUP;
+  tw.plane1 = w->plane1;
+  tw.salience = salv;
+  tw.rowptr = rpv;
+  tw.scale1 = s1v;
+  tw.offset = offv;
+  tw.nnz = 0;
+  if (tq_status st = linear_impl(M, N, K, &tw, x, yd, true, b + p.dec, p.total - p.dec, s)) return st;
+  return from_cuda(launch_ew_correct(M, N, K, w, x, yd, y, f32, s));
+}
+}  // namespace
+
+extern "C" {
+
+tq_status tq_ew_rowptr(int32_t N, int32_t K, const uint8_t *mask_ids, int32_t *p2rowptr, uint32_t *d_status,
+                       void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!mask_ids || !p2rowptr || !d_status) return TQ_ERR_NULL;
+  return from_cuda(launch_ew_rowptr(N, K, mask_ids, p2rowptr, d_status, (cudaStream_t)stream));
+}
+
+tq_status tq_ew_pack(int32_t N, int32_t K, const int8_t *T0, const int8_t *T1, const uint8_t *mask_ids,
+                     const int32_t *p2rowptr, uint32_t *mask, uint8_t *plane1, uint8_t *plane2, uint32_t *d_status,
+                     void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!T0 || !T1 || !mask_ids || !p2rowptr || !mask || !plane1 || !d_status) return TQ_ERR_NULL;
+  if (((uintptr_t)mask & 3u) || ((uintptr_t)p2rowptr & 3u)) return TQ_ERR_ALIGN;
+  return from_cuda(launch_ew_pack(N, K, T0, T1, mask_ids, p2rowptr, mask, plane1, plane2, d_status,
+                                  (cudaStream_t)stream));
+}
+
+tq_status tq_ew_unpack(int32_t N, int32_t K, const uint32_t *mask, const uint8_t *plane1, const int32_t *p2rowptr,
+                       const uint8_t *plane2, int8_t *T0, int8_t *T1, uint8_t *mask_ids, uint32_t *d_status,
+                       void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if (!mask || !plane1 || !p2rowptr || !T0 || !T1 || !mask_ids || !d_status) return TQ_ERR_NULL;
+  if (((uintptr_t)mask & 3u) || ((uintptr_t)p2rowptr & 3u)) return TQ_ERR_ALIGN;
+  return from_cuda(launch_ew_unpack(N, K, mask, plane1, p2rowptr, plane2, T0, T1, mask_ids, d_status,
+                                    (cudaStream_t)stream));
+}
+
+size_t tq_ew_workspace_bytes(int32_t M, int32_t N, int32_t K) {
+  if (M < 1 || check_shape(N, K) != TQ_OK) return 0;
+  return ew_parts(M, N, K).total;
+}
+
+tq_status tq_ew_linear(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, uint16_t *y,
+                       void *workspace, size_t workspace_bytes, void *stream) {
+  return ew_linear_impl(M, N, K, w, x, y, false, workspace, workspace_bytes, (cudaStream_t)stream);
+}
+
+tq_status tq_ew_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, float *y,
+                              void *workspace, size_t workspace_bytes, void *stream) {
+  return ew_linear_impl(M, N, K, w, x, y, true, workspace, workspace_bytes, (cudaStream_t)stream);
 }
 
 tq_status tq_get_device_status(uint32_t *status_host, int clear) {

@@ -379,4 +379,249 @@ cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t
   return cudaGetLastError();
 }
 
+// ------------------------------------------ element-wise four-mask format
+// The paper's representation with four disjoint masks of orders [2, 2, 1, 1]
+// ("Model and Representation"), stored as: a 2-bit mask-id plane (element k
+// of row n in bits 2 (k mod 16) of word [n][k / 16]); T0 of every element in
+// plane 1's group layout (the codec above); per row, the T1 trits of its
+// order-2 elements (masks 0 and 1) in increasing k, five per byte, the last
+// byte padded with digit 1, row n's bytes from byte rowptr[n].
+constexpr int kEwRowWarps = 4;  // rows (warps) per block of the per-row kernels
+
+__device__ __forceinline__ uint32_t lanemask_lt() {
+  uint32_t m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Warp per row: plane-2 bytes of the row (ceil(order-2 elements / 5)) into
+// rowptr[n + 1]; mask ids above 3 set BAD_CODE.
+__global__ void __launch_bounds__(32 * kEwRowWarps) ew_count_kernel(int N, int K, const uint8_t *mask,
+                                                                   int32_t *rowptr, uint32_t *status) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kEwRowWarps + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const uint8_t *row = mask + (int64_t)n * K;
+  int c = 0;
+  uint32_t st = 0;
+  for (int k = lane; k < K; k += 32) {
+    const uint8_t m = row[k];
+    c += m <= 1;
+    if (m > 3) st |= TQ_DATA_BAD_CODE;
+  }
+  for (int o = 16; o; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) {
+    rowptr[n + 1] = (c + 4) / 5;
+    if (n == 0) rowptr[0] = 0;
+    if (st) atomicOr(status, st);
+  }
+}
+
+// One block: rowptr[1..N] (bytes per row) into offsets, in place.
+__global__ void __launch_bounds__(1024) ew_scan_kernel(int N, int32_t *rowptr) {
+  __shared__ int32_t part[1024];
+  const int t = threadIdx.x;
+  const int r0 = (int)((int64_t)N * t / 1024), r1 = (int)((int64_t)N * (t + 1) / 1024);
+  int32_t sum = 0;
+  for (int n = r0; n < r1; ++n) sum += rowptr[n + 1];
+  part[t] = sum;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    const int32_t v = t >= o ? part[t - o] : 0;
+    __syncthreads();
+    part[t] += v;
+    __syncthreads();
+  }
+  int32_t run = part[t] - sum;  // exclusive prefix of this thread's rows
+  for (int n = r0; n < r1; ++n) {
+    run += rowptr[n + 1];
+    rowptr[n + 1] = run;
+  }
+}
+
+// Thread per mask word.
+__global__ void ew_mask_pack_kernel(int N, int K, const uint8_t *mask, uint32_t *plane, uint32_t *status) {
+  const int64_t total = (int64_t)N * (K / 16);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint8_t *src = mask + i * 16;
+    uint32_t w = 0, st = 0;
+    for (int j = 0; j < 16; ++j) {
+      uint32_t m = src[j];
+      if (m > 3) st |= TQ_DATA_BAD_CODE, m = 3;
+      w |= m << (2 * j);
+    }
+    plane[i] = w;
+    if (st) atomicOr(status, st);
+  }
+}
+
+// Thread per plane-1 byte: T0 of every element (the group layout).
+__global__ void ew_plane1_pack_kernel(int N, int K, const int8_t *T0, uint8_t *plane1, uint32_t *status) {
+  const int G = K / kGroup;
+  const int64_t RB = row_bytes_of(K), total = (int64_t)N * RB;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int n = (int)(idx / RB), b = (int)(idx - (int64_t)n * RB);
+    if (b >= G * kGroupBytes) {
+      plane1[idx] = 0;
+      continue;
+    }
+    uint32_t st = 0;
+    const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+    plane1[idx] = encode_codes(T0 + (int64_t)n * K + (int64_t)g * kGroup + 5 * pos, pos < kFullBytes ? 5 : kTailTrits, &st);
+    if (st) atomicOr(status, st);
+  }
+}
+
+// Warp per row: the row's order-2 T1 trits in order, five per byte.  Each
+// 32-element chunk ranks its order-2 elements by ballot; their digits join
+// the (fewer than 5) left over from earlier chunks in a per-warp ring, whole
+// bytes are written, the rest carried on.
+__global__ void __launch_bounds__(32 * kEwRowWarps) ew_plane2_pack_kernel(int N, int K, const int8_t *T1,
+                                                                         const uint8_t *mask, const int32_t *rowptr,
+                                                                         uint8_t *plane2, uint32_t *status) {
+  __shared__ uint8_t dig[kEwRowWarps][40];
+  const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
+  const int n = blockIdx.x * kEwRowWarps + wi;
+  if (n >= N) return;
+  uint8_t *d = dig[wi];
+  const int8_t *t1 = T1 + (int64_t)n * K;
+  const uint8_t *mk = mask + (int64_t)n * K;
+  const int64_t b0 = rowptr[n], nb = (int64_t)rowptr[n + 1] - rowptr[n];
+  int pend = 0;   // digits carried into this chunk
+  int64_t out = 0;  // bytes written
+  uint32_t st = 0;
+  for (int k0 = 0; k0 < K; k0 += 32) {
+    const int k = k0 + lane;
+    const bool in = k < K;
+    const bool o2 = in && mk[k] <= 1;
+    int c = in ? t1[k] : 0;
+    if (c < -1 || c > 1) st |= TQ_DATA_BAD_CODE, c = c < -1 ? -1 : 1;
+    if (in && !o2 && c != 0) st |= TQ_DATA_T2_OUTSIDE;
+    const uint32_t bal = __ballot_sync(0xffffffffu, o2);
+    if (o2) d[pend + __popc(bal & lanemask_lt())] = (uint8_t)(c + 1);
+    __syncwarp();
+    const int tot = pend + __popc(bal), full = tot / 5, rem = tot - 5 * full;
+    if (lane < full) {
+      const uint8_t *q = d + 5 * lane;
+      const int v = q[0] + 3 * q[1] + 9 * q[2] + 27 * q[3] + 81 * q[4];
+      if (out + lane < nb) plane2[b0 + out + lane] = (uint8_t)v;
+    }
+    const uint8_t carry = lane < rem ? d[5 * full + lane] : 0;
+    __syncwarp();
+    if (lane < rem) d[lane] = carry;
+    __syncwarp();
+    out += full;
+    pend = rem;
+  }
+  if (pend > 0 && lane == 0) {
+    int v = 0, p = 1;
+    for (int i = 0; i < 5; ++i, p *= 3) v += (i < pend ? d[i] : 1) * p;
+    if (out < nb) plane2[b0 + out] = (uint8_t)v;
+    ++out;
+  }
+  if (lane == 0 && out != nb) st |= TQ_DATA_BAD_ROWPTR;
+  if (st) atomicOr(status, st);
+}
+
+// Thread per mask word: mask ids back.
+__global__ void ew_mask_unpack_kernel(int N, int K, const uint32_t *plane, uint8_t *mask) {
+  const int64_t total = (int64_t)N * (K / 16);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t w = plane[i];
+    for (int j = 0; j < 16; ++j) mask[i * 16 + j] = (uint8_t)((w >> (2 * j)) & 3u);
+  }
+}
+
+// Thread per plane-1 byte: T0 back (pad bytes must be 0).
+__global__ void ew_plane1_unpack_kernel(int N, int K, const uint8_t *plane1, int8_t *T0, uint32_t *status) {
+  const int G = K / kGroup;
+  const int64_t RB = row_bytes_of(K), total = (int64_t)N * RB;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int n = (int)(idx / RB), b = (int)(idx - (int64_t)n * RB);
+    const uint8_t v = plane1[idx];
+    if (b >= G * kGroupBytes) {
+      if (v != 0) atomicOr(status, TQ_DATA_BAD_PAD);
+      continue;
+    }
+    uint32_t st = 0;
+    const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+    decode_to(v, pos < kFullBytes ? 5 : kTailTrits, T0 + (int64_t)n * K + (int64_t)g * kGroup + 5 * pos, &st);
+    if (st) atomicOr(status, st);
+  }
+}
+
+// Warp per row: T1 back from plane 2 (zeros on order-1 elements); bytes
+// above 242 and pad digits other than 1 in the row's last byte are flagged.
+__global__ void __launch_bounds__(32 * kEwRowWarps) ew_plane2_unpack_kernel(int N, int K, const uint32_t *plane,
+                                                                           const int32_t *rowptr,
+                                                                           const uint8_t *plane2, int8_t *T1,
+                                                                           uint32_t *status) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kEwRowWarps + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const int64_t b0 = rowptr[n], nb = (int64_t)rowptr[n + 1] - rowptr[n];
+  const uint32_t *mw = plane + (int64_t)n * (K / 16);
+  int base = 0;
+  uint32_t st = 0;
+  for (int k0 = 0; k0 < K; k0 += 32) {
+    const int k = k0 + lane;
+    const bool in = k < K;
+    const bool o2 = in && ((mw[k >> 4] >> (2 * (k & 15))) & 3u) <= 1;
+    const uint32_t bal = __ballot_sync(0xffffffffu, o2);
+    int8_t t = 0;
+    if (o2) {
+      const int r = base + __popc(bal & lanemask_lt());
+      if (r / 5 < nb) {
+        int v = plane2[b0 + r / 5];
+        if (v > 242) st |= TQ_DATA_BAD_BYTE, v = 0;
+        for (int i = 0; i < r % 5; ++i) v /= 3;
+        t = (int8_t)(v % 3 - 1);
+      } else {
+        st |= TQ_DATA_BAD_ROWPTR;
+      }
+    }
+    if (in) T1[(int64_t)n * K + k] = t;
+    base += __popc(bal);
+  }
+  if (lane == 0) {
+    if ((base + 4) / 5 != nb) st |= TQ_DATA_BAD_ROWPTR;
+    if (base % 5 && nb > 0 && (base + 4) / 5 == nb) {
+      int v = plane2[b0 + nb - 1];
+      if (v <= 242) {
+        for (int i = 0; i < 5; ++i, v /= 3)
+          if (i >= base % 5 && v % 3 != 1) st |= TQ_DATA_BAD_PAD;
+      }
+    }
+  }
+  if (st) atomicOr(status, st);
+}
+
+cudaError_t launch_ew_rowptr(int N, int K, const uint8_t *mask, int32_t *rowptr, uint32_t *status, cudaStream_t s) {
+  ew_count_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, mask, rowptr, status);
+  ew_scan_kernel<<<1, 1024, 0, s>>>(N, rowptr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ew_pack(int N, int K, const int8_t *T0, const int8_t *T1, const uint8_t *mask,
+                           const int32_t *rowptr, uint32_t *mplane, uint8_t *plane1, uint8_t *plane2,
+                           uint32_t *status, cudaStream_t s) {
+  ew_mask_pack_kernel<<<grid_for((int64_t)N * (K / 16), 256), 256, 0, s>>>(N, K, mask, mplane, status);
+  ew_plane1_pack_kernel<<<grid_for((int64_t)N * row_bytes_of(K), 256), 256, 0, s>>>(N, K, T0, plane1, status);
+  ew_plane2_pack_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, T1, mask, rowptr,
+                                                                                        plane2, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ew_unpack(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
+                             const uint8_t *plane2, int8_t *T0, int8_t *T1, uint8_t *mask, uint32_t *status,
+                             cudaStream_t s) {
+  ew_mask_unpack_kernel<<<grid_for((int64_t)N * (K / 16), 256), 256, 0, s>>>(N, K, mplane, mask);
+  ew_plane1_unpack_kernel<<<grid_for((int64_t)N * row_bytes_of(K), 256), 256, 0, s>>>(N, K, plane1, T0, status);
+  ew_plane2_unpack_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, mplane, rowptr,
+                                                                                          plane2, T1, status);
+  return cudaGetLastError();
+}
+
 }  // namespace tq

@@ -49,6 +49,12 @@ class tq_problem(ctypes.Structure):
     _fields_ = [("w", tq_weight), ("x", ctypes.c_void_p), ("y", ctypes.c_void_p)]
 
 
+class tq_ew_weight(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int32), ("K", ctypes.c_int32), ("mask", ctypes.c_void_p), ("plane1", ctypes.c_void_p),
+                ("p2rowptr", ctypes.c_void_p), ("plane2", ctypes.c_void_p), ("mu", ctypes.c_void_p),
+                ("alpha0", ctypes.c_void_p), ("alpha1", ctypes.c_void_p)]
+
+
 class tq_host_weight(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("N", ctypes.c_int32), ("K", ctypes.c_int32), ("nnz", ctypes.c_int64),
                 ("plane1", ctypes.c_void_p), ("salience", ctypes.c_void_p), ("rowptr", ctypes.c_void_p),
@@ -102,6 +108,19 @@ def lib():
             L.tq_linear_static.argtypes = [i32, i32, i32, ctypes.POINTER(tq_weight), vp, vp, vp]
             L.tq_linear_batched.restype = ctypes.c_int
             L.tq_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
+            EW = ctypes.POINTER(tq_ew_weight)
+            L.tq_ew_rowptr.restype = ctypes.c_int
+            L.tq_ew_rowptr.argtypes = [i32, i32, vp, vp, vp, vp]
+            L.tq_ew_pack.restype = ctypes.c_int
+            L.tq_ew_pack.argtypes = [i32, i32] + [vp] * 8 + [vp]
+            L.tq_ew_unpack.restype = ctypes.c_int
+            L.tq_ew_unpack.argtypes = [i32, i32] + [vp] * 8 + [vp]
+            L.tq_ew_workspace_bytes.restype = sz
+            L.tq_ew_workspace_bytes.argtypes = [i32, i32, i32]
+            L.tq_ew_linear.restype = ctypes.c_int
+            L.tq_ew_linear.argtypes = [i32, i32, i32, EW, vp, vp, vp, sz, vp]
+            L.tq_ew_linear_f32out.restype = ctypes.c_int
+            L.tq_ew_linear_f32out.argtypes = [i32, i32, i32, EW, vp, vp, vp, sz, vp]
             L.tq_linear_sequence.restype = ctypes.c_int
             L.tq_linear_sequence.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
             L.tq_sequence_selftest.restype = ctypes.c_int
@@ -558,3 +577,79 @@ def tq_sequence_selftest(batch: Batch, stream=None):
     (its bounded wait runs out; the device status then reports the timeout)."""
     _check(lib().tq_sequence_selftest(len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(), _stream(stream)),
            "tq_sequence_selftest")
+
+
+# ------------------------------------------------ element-wise four masks
+@dataclass
+class EwWeight:
+    """Device tensors of one projection in the element-wise four-mask form
+    (the fields of tq_ew_weight)."""
+    N: int
+    K: int
+    mask: torch.Tensor      # int32 (uint32 bits) [N][K/16]
+    plane1: torch.Tensor    # uint8 [N][row_bytes]
+    p2rowptr: torch.Tensor  # int32 [N+1]
+    plane2: torch.Tensor    # uint8 [max(p2rowptr[N], 1)]
+    mu: torch.Tensor        # fp16 [N][4]
+    alpha0: torch.Tensor    # fp16 [N][4]
+    alpha1: torch.Tensor    # fp16 [N][2]
+
+    def struct(self) -> tq_ew_weight:
+        w = tq_ew_weight()
+        w.N, w.K = self.N, self.K
+        w.mask, w.plane1, w.p2rowptr = self.mask.data_ptr(), self.plane1.data_ptr(), self.p2rowptr.data_ptr()
+        w.plane2 = self.plane2.data_ptr()
+        w.mu, w.alpha0, w.alpha1 = self.mu.data_ptr(), self.alpha0.data_ptr(), self.alpha1.data_ptr()
+        return w
+
+    def packed_bytes(self) -> int:
+        t = [self.mask, self.plane1, self.p2rowptr, self.mu, self.alpha0, self.alpha1]
+        return sum(x.numel() * x.element_size() for x in t) + int(self.p2rowptr[-1].item())
+
+
+def pack_ew_weight(T0, T1, mask_ids, mu, a0, a1, stream=None, check=True) -> EwWeight:
+    """Pack device int8 T0, T1 [N][K] and uint8 mask ids with tq_ew_rowptr +
+    tq_ew_pack (one synchronization, to size plane 2)."""
+    N, K = T0.shape
+    dev = T0.device
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    rp = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    _check(lib().tq_ew_rowptr(N, K, _p(mask_ids), _p(rp), _p(status), _stream(stream)), "tq_ew_rowptr")
+    nb = int(rp[N].item())
+    mplane = torch.empty((N, K // 16), dtype=torch.int32, device=dev)
+    plane1 = torch.empty((N, tq_row_bytes(K)), dtype=torch.uint8, device=dev)
+    plane2 = torch.empty(max(nb, 1), dtype=torch.uint8, device=dev)
+    _check(lib().tq_ew_pack(N, K, _p(T0), _p(T1), _p(mask_ids), _p(rp), _p(mplane), _p(plane1), _p(plane2),
+                            _p(status), _stream(stream)), "tq_ew_pack")
+    if check:
+        st = int(status.item())
+        if st:
+            raise TQError(-4, f"tq_ew_pack data status {st:#x}")
+    return EwWeight(N, K, mplane, plane1, rp, plane2, mu, a0, a1)
+
+
+def tq_ew_unpack(w: EwWeight, status=None, stream=None):
+    """-> (T0, T1, mask ids) on the device."""
+    dev = w.plane1.device
+    if status is None:
+        status = torch.zeros(1, dtype=torch.int32, device=dev)
+    T0 = torch.empty((w.N, w.K), dtype=torch.int8, device=dev)
+    T1 = torch.empty((w.N, w.K), dtype=torch.int8, device=dev)
+    m = torch.empty((w.N, w.K), dtype=torch.uint8, device=dev)
+    _check(lib().tq_ew_unpack(w.N, w.K, _p(w.mask), _p(w.plane1), _p(w.p2rowptr), _p(w.plane2), _p(T0), _p(T1), _p(m),
+                              _p(status), _stream(stream)), "tq_ew_unpack")
+    return T0, T1, m
+
+
+def tq_ew_linear(x, w: EwWeight, y=None, ws=None, stream=None, f32=False):
+    """y = x W-hat^T for the element-wise form (fp16, or fp32 with f32=True)."""
+    M, K = x.shape
+    assert K == w.K and x.dtype == torch.float16
+    if y is None:
+        y = torch.empty((M, w.N), dtype=torch.float32 if f32 else torch.float16, device=x.device)
+    if ws is None:
+        ws = workspace(int(lib().tq_ew_workspace_bytes(M, w.N, K)), x.device)
+    s = w.struct()
+    fn = lib().tq_ew_linear_f32out if f32 else lib().tq_ew_linear
+    _check(fn(M, w.N, K, ctypes.byref(s), _p(x), _p(y), _p(ws), ws.numel(), _stream(stream)), "tq_ew_linear")
+    return y

@@ -1,0 +1,122 @@
+"""GPU parity of the element-wise four-mask representation (orders [2, 2, 1,
+1]) against the fp64 oracle (oracle/elementwise.py): tq_ew_rowptr / tq_ew_pack
+bytes equal the oracle's packing bit for bit and tq_ew_unpack inverts them;
+tq_ew_linear satisfies |y - y_ref| <= 2e-3 * sum_k |W x| per element on
+ragged shapes, 1..40 tokens (decode and prefill paths under the mask-3 pass)
+and Qwen3-8B projection shapes (sampled rows)."""
+import numpy as np
+import pytest
+import torch
+
+import workloads as wl
+from oracle import elementwise as ew
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def H():
+    import gpu_helpers
+    return gpu_helpers
+
+
+def _pack(H, w):
+    from paper_2609_09240_gb300 import tq
+    return tq.pack_ew_weight(H.dev(w.T0), H.dev(w.T1), H.dev(w.mask), H.dev(w.mu), H.dev(w.a0), H.dev(w.a1))
+
+
+def _np(t, dtype):
+    return np.ascontiguousarray(t.cpu().numpy()).view(dtype)
+
+
+@pytest.mark.parametrize("N,K", [(1, 128), (37, 256), (300, 1152), (129, 4096), (64, 12288)])
+def test_codec_bit_exact(H, N, K):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_ew_weights(N, K, config=12, proj=N)
+    mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+    assert st == 0
+    g = _pack(H, w)
+    torch.cuda.synchronize()
+    assert np.array_equal(_np(g.p2rowptr, np.int32), rp)
+    assert np.array_equal(_np(g.mask, np.uint32), mp)
+    assert np.array_equal(_np(g.plane1, np.uint8), p1)
+    assert np.array_equal(_np(g.plane2, np.uint8)[:rp[N]], p2)
+    T0, T1, m = tq.tq_ew_unpack(g)
+    torch.cuda.synchronize()
+    assert np.array_equal(T0.cpu().numpy(), w.T0) and np.array_equal(T1.cpu().numpy(), w.T1)
+    assert np.array_equal(m.cpu().numpy(), w.mask)
+
+
+def test_codec_coverage_extremes(H):
+    """Rows with no order-2 element, rows entirely of mask 0, and order-2
+    counts of every residue mod 5."""
+    N, K = 10, 256
+    w = wl.gen_ew_weights(N, K, config=13)
+    mask = np.full((N, K), 3, np.uint8)
+    mask[1] = 0
+    for r in range(2, 7):
+        mask[r, : (r - 2) + 5 * r] = 1
+    mask[7, ::2] = 2
+    T1 = (w.T1 * 0 + wl._trits(np.random.default_rng(3), (N, K))) * (mask <= 1)
+    T1 = T1.astype(np.int8)
+    mp, p1, rp, p2, st = ew.pack(w.T0, T1, mask)
+    assert st == 0
+    w2 = wl.EwWeights(N, K, w.T0, T1, mask, w.mu, w.a0, w.a1)
+    g = _pack(H, w2)
+    torch.cuda.synchronize()
+    assert np.array_equal(_np(g.p2rowptr, np.int32), rp)
+    assert np.array_equal(_np(g.plane2, np.uint8)[:rp[N]], p2)
+
+
+def test_codec_flags_bad_data(H):
+    from paper_2609_09240_gb300 import tq
+    N, K = 4, 256
+    w = wl.gen_ew_weights(N, K, config=14)
+    dev = lambda a: H.dev(a)
+    # T1 nonzero on an order-1 element
+    T1 = w.T1.copy()
+    k = int(np.argwhere(w.mask[0] >= 2)[0][0])
+    T1[0, k] = -1
+    with pytest.raises(tq.TQError):
+        tq.pack_ew_weight(dev(w.T0), dev(T1), dev(w.mask), dev(w.mu), dev(w.a0), dev(w.a1))
+    # a mask id above 3
+    mask = w.mask.copy()
+    mask[2, 5] = 7
+    with pytest.raises(tq.TQError):
+        tq.pack_ew_weight(dev(w.T0), dev(w.T1), dev(mask), dev(w.mu), dev(w.a0), dev(w.a1))
+    # a plane-2 byte above 242 is reported by unpack
+    g = _pack(H, w)
+    g.plane2[0] = 250
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    tq.tq_ew_unpack(g, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & 4
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 512, 1024), (2, 300, 2560), (5, 129, 4224), (16, 1000, 640), (40, 256, 1152),
+                                   (1, 1, 128)])
+@pytest.mark.parametrize("f32", [False, True])
+def test_linear_parity(H, M, N, K, f32):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_ew_weights(N, K, config=15, proj=M + N)
+    xb = wl.gen_x(M, K, config=15, proj=M + N)
+    mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+    assert st == 0
+    y_ref, a_ref = ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1)
+    y = tq.tq_ew_linear(H.dev(xb), _pack(H, w), f32=f32)
+    H.device_status_ok()
+    H.assert_close(y.float().cpu().numpy().astype(np.float64), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("N,K", [(4096, 4096), (12288, 4096), (4096, 12288)])
+def test_linear_qwen3_8b_shapes_sampled_rows(H, N, K):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_ew_weights(N, K, config=16, proj=N // 1024)
+    xb = wl.gen_x(1, K, config=16, proj=N // 1024)
+    mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+    assert st == 0
+    rows = np.sort(np.random.default_rng(N).choice(N, size=64, replace=False))
+    y_ref, a_ref = ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1, rows=rows)
+    y = tq.tq_ew_linear(H.dev(xb), _pack(H, w))
+    H.device_status_ok()
+    H.assert_close(y.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
