@@ -792,6 +792,56 @@ def sub_sequence(dev, peak, steps=30):
             "gpu_launches_per_step": 2, "device_status": st, "steps": steps}
 
 
+def sub_elementwise(dev, peak):
+    """The element-wise four-mask form (orders [2, 2, 1, 1], the paper's
+    recorded coverages) of one Qwen3-8B layer at M = 1: seven tq_ew_linear
+    calls per layer over rotated copies (more than 4 x L2 of packed bytes),
+    replayed as a CUDA graph."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    base, layer_bytes = [], 0
+    for p in wl.config_projections(4):
+        g = torch.Generator(device=dev)
+        g.manual_seed(900 + p.proj)
+        N, K = p.N, p.K
+        u = torch.rand((N, K), generator=g, device=dev)
+        mask = ((u >= 0.005).to(torch.uint8) + (u >= 0.036).to(torch.uint8) + (u >= 0.136).to(torch.uint8))
+        u0 = torch.rand((N, K), generator=g, device=dev)
+        T0 = ((u0 >= 0.3).to(torch.int8) + (u0 >= 0.7).to(torch.int8) - 1)
+        u1 = torch.rand((N, K), generator=g, device=dev)
+        T1 = ((u1 >= 0.3).to(torch.int8) + (u1 >= 0.7).to(torch.int8) - 1) * (mask <= 1).to(torch.int8)
+        mu = (torch.randn((N, 4), generator=g, device=dev) * 1e-3).half()
+        a0 = torch.empty((N, 4), device=dev).log_normal_(-4.0, 0.5, generator=g).half()
+        a1 = torch.empty((N, 2), device=dev).log_normal_(-4.0, 0.5, generator=g).half()
+        w = tq.pack_ew_weight(T0, T1, mask, mu, a0, a1)
+        del u, u0, u1, T0, T1, mask
+        base.append(w)
+        layer_bytes += w.packed_bytes()
+    R = -(-4 * L2_BYTES // layer_bytes)
+    clone = lambda w: tq.EwWeight(w.N, w.K, w.mask.clone(), w.plane1.clone(), w.p2rowptr.clone(), w.plane2.clone(),
+                                  w.mu.clone(), w.alpha0.clone(), w.alpha1.clone())
+    layers = [[(w if r == 0 else clone(w), wl.gen_x_torch(1, w.K, dev, 950 + 8 * r + i),
+                torch.empty((1, w.N), dtype=torch.float16, device=dev)) for i, w in enumerate(base)] for r in range(R)]
+    wss = [tq.workspace(int(tq.lib().tq_ew_workspace_bytes(1, w.N, w.K)), dev) for w in base]
+
+    def calls():
+        for items in layers:
+            for (w, x, y), wsb in zip(items, wss):
+                tq.tq_ew_linear(x, w, y=y, ws=wsb)
+
+    ms = graph_ms(calls, reps=5) / R
+    gbs = layer_bytes / (ms * 1e-3) / 1e9
+    n_w = sum(w.N * w.K for w in base)
+    return {"workload": "qwen3-8b one layer in the element-wise four-mask form (coverages 0.5/3.1/10/86.4 %), M=1",
+            "us_per_layer": ms * 1e3, "packed_bytes": layer_bytes, "bits_per_weight": 8 * layer_bytes / n_w,
+            "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
+            "timing": f"{R} rotated copies of the layer ({R * layer_bytes / 2 ** 20:.0f} MiB > 4 x L2); seven "
+                      "tq_ew_linear calls per layer (4 launches each), replayed as a CUDA graph"}
+
+
 def cpu_baseline_single(budget_s):
     """The oracle on one host core over a prefix of layer 0's rows."""
     L = OracleLayer()
@@ -985,6 +1035,7 @@ def main():
                    "unbatched_calls": sub_unbatched_8b(items, dev, ms_per_step)}
             cfg["config4"] = sub_prefill(dev)
             cfg["dependency_ordered"] = sub_sequence(dev, peak)
+            cfg["elementwise"] = sub_elementwise(dev, peak)
             clk2.mark()
         cfg["clocks"] = clk2.summary()
         out["configs"] = cfg
