@@ -137,6 +137,47 @@ def unpack(N: int, K: int, mplane: np.ndarray, p1: np.ndarray, rp: np.ndarray, p
     return T0, T1, mask, st
 
 
+# ------------------------------------------------------- correction index
+# A structure derived from a packed weight (this library's, no counterpart
+# in the paper), like the group format's second-plane index: the elements of
+# masks 0..2 of every row, block by block of IDX_BLOCK elements along K, in
+# increasing k, each as one uint16 entry
+#     (k mod IDX_BLOCK) | code << 10,  code = 9 q + 3 (T0 + 1) + (T1 + 1),
+# with int32 offsets[n * nb + b] of row n's block b (nb = ceil(K / IDX_BLOCK),
+# offsets[N nb] = all entries).  Everything the masks 0..2 add to the
+# mask-3 form of a row is in its entries.
+IDX_BLOCK = 1024
+
+
+def correction_index(T0: np.ndarray, T1: np.ndarray, mask: np.ndarray):
+    """-> (offsets int32 [N nb + 1], entries uint16)."""
+    N, K = mask.shape
+    nb = (K + IDX_BLOCK - 1) // IDX_BLOCK
+    rows, cols = np.nonzero(mask != 3)  # row-major: increasing k within a row
+    counts = np.bincount(rows * nb + cols // IDX_BLOCK, minlength=N * nb)
+    offsets = np.zeros(N * nb + 1, np.int64)
+    offsets[1:] = np.cumsum(counts)
+    q = mask[rows, cols].astype(np.int64)
+    code = 9 * q + 3 * (T0[rows, cols].astype(np.int64) + 1) + (T1[rows, cols].astype(np.int64) + 1)
+    entries = (cols % IDX_BLOCK) | (code << 10)
+    return offsets.astype(np.int32), entries.astype(np.uint16)
+
+
+def decode_index(N: int, K: int, offsets, entries):
+    """-> (mask, T0, T1) with mask 3 and zero codes wherever no entry is."""
+    nb = (K + IDX_BLOCK - 1) // IDX_BLOCK
+    mask = np.full((N, K), 3, np.uint8)
+    T0 = np.zeros((N, K), np.int8)
+    T1 = np.zeros((N, K), np.int8)
+    e = entries.astype(np.int64)
+    for n in range(N):
+        for b in range(nb):
+            for v in e[offsets[n * nb + b]:offsets[n * nb + b + 1]]:
+                k, code = b * IDX_BLOCK + (v & 1023), v >> 10
+                mask[n, k], T0[n, k], T1[n, k] = code // 9, (code // 3) % 3 - 1, code % 3 - 1
+    return mask, T0, T1
+
+
 # -------------------------------------------------------------------- linear
 def dense_rows(K: int, mplane, p1, rp, p2, mu, a0, a1, rows):
     """fp64 W rows decoded from the packed bytes (the paper's compact form)."""
