@@ -416,6 +416,24 @@ TQ_API tq_status tq_ew_linear(int32_t M, int32_t N, int32_t K, const tq_ew_weigh
 TQ_API tq_status tq_ew_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x,
                                      float *y, void *workspace, size_t workspace_bytes, void *stream);
 
+/* Many independent element-wise projections sharing M (<= TQ_MAX_SKINNY_M)
+ * in three launches plus the decode path's (one decode step's projections
+ * of a layer, say): the views of every problem in one launch, every
+ * problem's plane-1 pass in one tq_linear_batched-style call, the
+ * corrections of every problem in one launch per 8 tokens.  `problems` is a
+ * HOST array read during the call (at most TQ_MAX_BATCH entries); y is fp16
+ * [M][w.N].  Per-problem results equal tq_ew_linear's up to the order of
+ * fp32 additions in split tiles. */
+typedef struct {
+  tq_ew_weight w;
+  const uint16_t *x; /* fp16 [M][w.K], 16-byte aligned */
+  uint16_t *y;       /* fp16 [M][w.N] */
+} tq_ew_problem;
+/* Workspace bytes of a batched element-wise call (0 for invalid arguments). */
+TQ_API size_t tq_ew_batched_workspace_bytes(int32_t M, int32_t count, const tq_ew_problem *problems);
+TQ_API tq_status tq_ew_linear_batched(int32_t M, int32_t count, const tq_ew_problem *problems, void *workspace,
+                                      size_t workspace_bytes, void *stream);
+
 /* ---------------------------------------------------------------------
  * Allocation-free variant (no counterpart in the paper; an integration aid).
  *

@@ -29,10 +29,8 @@ cudaError_t launch_ew_pack(int N, int K, const int8_t *T0, const int8_t *T1, con
 cudaError_t launch_ew_unpack(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
                              const uint8_t *plane2, int8_t *T0, int8_t *T1, uint8_t *mask, uint32_t *status,
                              cudaStream_t s);
-cudaError_t launch_ew_views(int N, int K, const uint16_t *mu, const uint16_t *a0, uint16_t *s1v, uint16_t *offv,
-                            uint32_t *salv, int32_t *rpv, cudaStream_t s);
-cudaError_t launch_ew_correct(int M, int N, int K, const tq_ew_weight *w, const uint16_t *x, const float *ydense,
-                              void *y, bool f32, cudaStream_t s);
+cudaError_t launch_ew_views(const EwCall *calls, int count, cudaStream_t s);
+cudaError_t launch_ew_correct(int M, const EwCall *calls, int count, bool f32, cudaStream_t s);
 int mma_rows_per_tile();
 void mma_workspace_parts(int M, int N, int K, size_t *b, size_t *cs, size_t *y2);
 cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
@@ -156,24 +154,7 @@ tq_status place(BatchParams &bp, unsigned char *ws, size_t ws_bytes) {
 // tokens in one pass (warp-level MMA kernels).  Returns TQ_ERR_SHAPE when the
 // workspace is too small.
 tq_status run_pass(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStream_t s) {
-  const int rows = mma_rows_per_tile();
-  int tiles = 0;
-  size_t off = 0;
-  for (int i = 0; i < bp.count; ++i) {
-    Problem &P = bp.prob[i];
-    P.tile_begin = tiles;
-    tiles += (P.N + rows - 1) / rows;
-    const size_t tot = problem_ws_bytes(bp.M, P.N, P.K);
-    if (off + tot > ws_bytes) return TQ_ERR_SHAPE;
-    size_t b, cs, y2;
-    mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
-    P.wsB = ws + off;
-    P.wsCS = reinterpret_cast<float *>(ws + off + pad256(b));
-    P.y2_off = (int32_t)(pad256(b) + pad256(cs));
-    P.map_off = (int32_t)(pad256(b) + pad256(cs) + pad256(y2));
-    off += tot;
-  }
-  bp.total_tiles = tiles;
+  if (tq_status st = place(bp, ws, ws_bytes)) return st;
   return from_cuda(launch_gemv_mma(bp, s));
 }
 
@@ -421,11 +402,12 @@ tq_status tq_sequence_selftest(int32_t count, const tq_problem *problems, void *
 }  // extern "C"
 
 namespace {
-// Workspace parts of tq_ew_linear, each 256-byte padded: the s1 and off
-// views [N][G] fp16, the views' zero salience words and rowptr, the fp32
-// result of the plane-1 pass [M][N], the decode path's workspace.
+// Per-problem workspace parts of the element-wise linear, each 256-byte
+// padded: the s1 and off views [N][G] fp16, the views' zero salience words
+// and rowptr, the fp32 result of the plane-1 pass [M][N].  The decode
+// path's workspace follows (after every problem's parts in a batched call).
 struct EwParts {
-  size_t s1v, offv, salv, rpv, yd, dec, total;
+  size_t s1v, offv, salv, rpv, yd, total;
 };
 EwParts ew_parts(int32_t M, int32_t N, int32_t K) {
   EwParts p;
@@ -435,44 +417,90 @@ EwParts ew_parts(int32_t M, int32_t N, int32_t K) {
   p.salv = p.offv + pad256((size_t)N * G * 2);
   p.rpv = p.salv + pad256((size_t)N * W * 4);
   p.yd = p.rpv + pad256(((size_t)N + 1) * 4);
-  p.dec = p.yd + pad256((size_t)M * N * 4);
-  p.total = p.dec + call_ws_bytes(M, N, K);
+  p.total = p.yd + pad256((size_t)M * N * 4);
   return p;
+}
+
+tq_status check_ew(int32_t M, const tq_ew_weight *w, const uint16_t *x, const void *y, bool f32) {
+  if (!w || !x || !y) return TQ_ERR_NULL;
+  if (tq_status st = check_shape(w->N, w->K)) return st;
+  if (!w->mask || !w->plane1 || !w->p2rowptr || !w->mu || !w->alpha0 || !w->alpha1) return TQ_ERR_NULL;
+  if (!aligned16(w->plane1) || !aligned16(x) || ((uintptr_t)w->mask & 3u) || ((uintptr_t)w->p2rowptr & 3u) ||
+      !aligned2(w->mu) || !aligned2(w->alpha0) || !aligned2(w->alpha1))
+    return TQ_ERR_ALIGN;
+  if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
+  (void)M;
+  return TQ_OK;
+}
+
+// count problems sharing M: every problem's views and plane-1 result, then
+// the plane-1 pass (one batched decode-path call; M > 16, a single problem
+// only, the prefill path), then the correction of every problem.
+tq_status ew_run(int32_t M, int32_t count, const tq_ew_weight *const *wts, const uint16_t *const *xs, void *const *ys,
+                 bool f32, void *ws, size_t ws_bytes, cudaStream_t s) {
+  thread_local EwCall calls[TQ_MAX_BATCH];
+  unsigned char *b = static_cast<unsigned char *>(ws);
+  size_t off = 0;
+  for (int i = 0; i < count; ++i) {
+    const tq_ew_weight *w = wts[i];
+    const EwParts p = ew_parts(M, w->N, w->K);
+    if (off + p.total > ws_bytes) return TQ_ERR_SHAPE;
+    EwCall &c = calls[i];
+    c.w = w;
+    c.x = xs[i];
+    c.y = ys[i];
+    c.s1v = reinterpret_cast<uint16_t *>(b + off + p.s1v);
+    c.offv = reinterpret_cast<uint16_t *>(b + off + p.offv);
+    c.salv = reinterpret_cast<uint32_t *>(b + off + p.salv);
+    c.rpv = reinterpret_cast<int32_t *>(b + off + p.rpv);
+    c.ydense = reinterpret_cast<float *>(b + off + p.yd);
+    off += p.total;
+  }
+  if (tq_status st = from_cuda(launch_ew_views(calls, count, s))) return st;
+  // plane 1 with mask 3's parameters in every group, no second plane
+  auto view_weight = [](const EwCall &c) {
+    tq_weight tw;
+    memset(&tw, 0, sizeof(tw));
+    tw.N = c.w->N;
+    tw.K = c.w->K;
+    tw.group = TQ_GROUP;
+    tw.plane1 = c.w->plane1;
+    tw.salience = c.salv;
+    tw.rowptr = c.rpv;
+    tw.scale1 = c.s1v;
+    tw.offset = c.offv;
+    tw.nnz = 0;
+    return tw;
+  };
+  if (M > TQ_MAX_SKINNY_M) {
+    if (count != 1) return TQ_ERR_SHAPE;
+    const tq_weight tw = view_weight(calls[0]);
+    if (tq_status st = linear_impl(M, tw.N, tw.K, &tw, calls[0].x, calls[0].ydense, true, b + off, ws_bytes - off, s))
+      return st;
+  } else {
+    thread_local BatchParams bp;
+    bp.count = count;
+    bp.M = M;
+    bp.out_f32 = 1;
+    for (int i = 0; i < count; ++i) {
+      const tq_weight tw = view_weight(calls[i]);
+      bp.prob[i] = to_problem(&tw, calls[i].x, calls[i].ydense);
+    }
+    if (tq_status st = run_batch(bp, b + off, ws_bytes - off, s)) return st;
+  }
+  return from_cuda(launch_ew_correct(M, calls, count, f32, s));
 }
 
 tq_status ew_linear_impl(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, void *y,
                          bool f32, void *ws, size_t ws_bytes, cudaStream_t s) {
   if (M < 1) return TQ_ERR_SHAPE;
-  if (tq_status st = check_shape(N, K)) return st;
-  if (!w || !x || !y || !ws) return TQ_ERR_NULL;
+  if (tq_status st = check_ew(M, w, x, y, f32)) return st;
   if (w->N != N || w->K != K) return TQ_ERR_SHAPE;
-  if (!w->mask || !w->plane1 || !w->p2rowptr || !w->mu || !w->alpha0 || !w->alpha1) return TQ_ERR_NULL;
-  if (!aligned16(w->plane1) || !aligned16(x) || ((uintptr_t)ws & 255u) || ((uintptr_t)w->mask & 3u) ||
-      ((uintptr_t)w->p2rowptr & 3u) || !aligned2(w->mu) || !aligned2(w->alpha0) || !aligned2(w->alpha1))
-    return TQ_ERR_ALIGN;
-  if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
-  const EwParts p = ew_parts(M, N, K);
-  if (ws_bytes < p.total) return TQ_ERR_SHAPE;
-  unsigned char *b = static_cast<unsigned char *>(ws);
-  uint16_t *s1v = reinterpret_cast<uint16_t *>(b + p.s1v), *offv = reinterpret_cast<uint16_t *>(b + p.offv);
-  uint32_t *salv = reinterpret_cast<uint32_t *>(b + p.salv);
-  int32_t *rpv = reinterpret_cast<int32_t *>(b + p.rpv);
-  float *yd = reinterpret_cast<float *>(b + p.yd);
-  if (tq_status st = from_cuda(launch_ew_views(N, K, w->mu, w->alpha0, s1v, offv, salv, rpv, s))) return st;
-  // plane 1 with mask 3's parameters in every group, no second plane
-  tq_weight tw;
-  memset(&tw, 0, sizeof(tw));
-  tw.N = N;
-  tw.K = K;
-  tw.group = TQ_GROUP;
-  tw.plane1 = w->plane1;
-  tw.salience = salv;
-  tw.rowptr = rpv;
-  tw.scale1 = s1v;
-  tw.offset = offv;
-  tw.nnz = 0;
-  if (tq_status st = linear_impl(M, N, K, &tw, x, yd, true, b + p.dec, p.total - p.dec, s)) return st;
-  return from_cuda(launch_ew_correct(M, N, K, w, x, yd, y, f32, s));
+  if (!ws) return TQ_ERR_NULL;
+  if ((uintptr_t)ws & 255u) return TQ_ERR_ALIGN;
+  if (ws_bytes < ew_parts(M, N, K).total + call_ws_bytes(M, N, K)) return TQ_ERR_SHAPE;
+  void *yv = y;
+  return ew_run(M, 1, &w, &x, &yv, f32, ws, ws_bytes, s);
 }
 }  // namespace
 
@@ -507,7 +535,37 @@ tq_status tq_ew_unpack(int32_t N, int32_t K, const uint32_t *mask, const uint8_t
 
 size_t tq_ew_workspace_bytes(int32_t M, int32_t N, int32_t K) {
   if (M < 1 || check_shape(N, K) != TQ_OK) return 0;
-  return ew_parts(M, N, K).total;
+  return ew_parts(M, N, K).total + call_ws_bytes(M, N, K);
+}
+
+size_t tq_ew_batched_workspace_bytes(int32_t M, int32_t count, const tq_ew_problem *problems) {
+  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH || !problems) return 0;
+  size_t tot = 0;
+  for (int i = 0; i < count; ++i) {
+    const tq_ew_weight &w = problems[i].w;
+    if (check_shape(w.N, w.K) != TQ_OK) return 0;
+    tot += ew_parts(M, w.N, w.K).total + problem_ws_bytes(M, w.N, w.K);
+  }
+  return tot;
+}
+
+tq_status tq_ew_linear_batched(int32_t M, int32_t count, const tq_ew_problem *problems, void *workspace,
+                               size_t workspace_bytes, void *stream) {
+  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
+  if (!problems || !workspace) return TQ_ERR_NULL;
+  if ((uintptr_t)workspace & 255u) return TQ_ERR_ALIGN;
+  thread_local const tq_ew_weight *wp[TQ_MAX_BATCH];
+  thread_local const uint16_t *xp[TQ_MAX_BATCH];
+  thread_local void *yp[TQ_MAX_BATCH];
+  for (int i = 0; i < count; ++i) {
+    const tq_ew_problem &q = problems[i];
+    if (tq_status st = check_ew(M, &q.w, q.x, q.y, false)) return st;
+    wp[i] = &q.w;
+    xp[i] = q.x;
+    yp[i] = q.y;
+  }
+  if (workspace_bytes < tq_ew_batched_workspace_bytes(M, count, problems)) return TQ_ERR_SHAPE;
+  return ew_run(M, count, wp, xp, yp, false, workspace, workspace_bytes, (cudaStream_t)stream);
 }
 
 tq_status tq_ew_linear(int32_t M, int32_t N, int32_t K, const tq_ew_weight *w, const uint16_t *x, uint16_t *y,

@@ -58,4 +58,17 @@ struct BatchParams {
   Problem prob[TQ_MAX_BATCH];
 };
 
+// One problem of an element-wise call as the API hands it to the kernels
+// (tq_ew.cu): the weight, x, the fp32 plane-1 result, y and the views of
+// the plane-1 pass in the workspace.
+struct EwCall {
+  const tq_ew_weight *w;
+  const uint16_t *x;
+  float *ydense;
+  void *y;
+  uint16_t *s1v, *offv;
+  uint32_t *salv;
+  int32_t *rpv;
+};
+
 }  // namespace tq

@@ -55,6 +55,16 @@ __host__ __device__ __forceinline__ uint32_t lut_word(int v) {
   return w;
 }
 
+// Fills the lane-replicated table: entry v in words 64 v .. 64 v + 31 (the
+// copy of lane l at word 64 v + l), written as 16-byte stores, each thread
+// computing an entry once per four copies.
+__device__ __forceinline__ void lut_fill_replicated(uint32_t *lut, int tid, int nthreads) {
+  for (int i = tid; i < 256 * 8; i += nthreads) {
+    const uint32_t w = lut_word(i >> 3);
+    reinterpret_cast<uint4 *>(lut + (i >> 3) * 64)[i & 7] = make_uint4(w, w, w, w);
+  }
+}
+
 // The low (hi = false) or high fp16 of a word, as float.
 template <bool HI>
 __device__ __forceinline__ float half_of(uint32_t w) {

@@ -193,7 +193,7 @@ __device__ __forceinline__ void setup_cta(unsigned char *dyn, int tid, int nthre
   using C = Cfg<SG>;
   Bars *bars = reinterpret_cast<Bars *>(dyn + C::kOffBars);
   uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
-  for (int i = tid; i < 256 * 32; i += nthreads) lut[(i >> 5) * 64 + (i & 31)] = mm::lut_word(i >> 5);
+  mm::lut_fill_replicated(lut, tid, nthreads);
   for (int i = tid; i < C::kZeroBytes / 16; i += nthreads)
     reinterpret_cast<uint4 *>(dyn + C::kOffZero)[i] = make_uint4(0u, 0u, 0u, 0u);
   if (tid == 0) {
@@ -409,6 +409,9 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
   __syncthreads();
   // everything below reads what the prep and second-plane kernels wrote
   grid_dep_wait();
+  // a programmatically launched successor (the next call's prep kernel)
+  // may be scheduled now; it waits for this grid before touching memory
+  grid_dep_launch_next();
   const int t_begin = sc.cta_unit[blockIdx.x], t_end = sc.cta_unit[blockIdx.x + 1];
 
   if (warp < WD) {

@@ -184,49 +184,7 @@ constexpr int kSeqCounterOff = 448;
 static_assert(kSeqCounterOff + 4 <= kMapSlotBytes, "map slot");
 
 // ------------------------------------------------------------------ prep
-// Activation slots of one group for the one-group-per-lane kernel (M <= 2,
-// tq_gemv_g4.cu), in the slice of the lane that owns it: MMA j = 5 i + m of
-// the lane's window words takes W, W' of window byte 4 i + m (m < 4) or the
-// fifth-slot words of window bytes 4 i .. 4 i + 3 (m = 4).  Window byte beta
-// is group byte beta - OFFS (OFFS = 2 for the odd groups of a 4-group stage,
-// whose window starts two bytes before the group; 26 for the second group
-// of a lane in an 8-group stage); bytes outside the group get zero
-// activations.  dst: the slice's chunk of this lane position, chunks 64 B
-// apart.
-template <int SG, int OFFS>
-__device__ __forceinline__ void g4_write_slots(unsigned char *dst, const __half *ya, const __half *yb,
-                                               const __half *yc, const __half *yd, const __half *ye) {
-  auto pk = [](__half lo, __half hi) -> uint32_t {
-    __half2 v = __halves2half2(lo, hi);
-    return *reinterpret_cast<uint32_t *>(&v);
-  };
-  const __half z = __float2half_rn(0.f);
-  auto yev = [&](int b) -> __half { return (b >= 0 && b < 26) ? ye[b] : z; };
-#pragma unroll
-  for (int jp = 0; jp < g4::pairs(SG); ++jp) {
-    uint32_t w[4];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int j = 2 * jp + h, i = j / 5, m = j % 5;
-      uint32_t b0 = 0u, b1 = 0u;
-      if (j < 5 * g4::words(SG)) {
-        if (m < 4) {
-          const int b = 4 * i + m - OFFS;
-          if (b >= 0 && b < 26) {
-            b0 = pk(ya[b], yb[b]);
-            b1 = pk(yc[b], yd[b]);
-          }
-        } else {
-          b0 = pk(yev(4 * i - OFFS), yev(4 * i + 1 - OFFS));
-          b1 = pk(yev(4 * i + 2 - OFFS), yev(4 * i + 3 - OFFS));
-        }
-      }
-      w[2 * h] = b0;
-      w[2 * h + 1] = b1;
-    }
-    *reinterpret_cast<uint4 *>(dst + jp * 64) = make_uint4(w[0], w[1], w[2], w[3]);
-  }
-}
+constexpr int kPrepTasks = 16;  // (group, token) tasks per 128-thread prep block
 
 __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, const __grid_constant__ MapTemplates mt,
                                      int32_t *unit_counter) {
@@ -235,6 +193,10 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   const Problem &P = bp.prob[p];
   // the next kernel (second plane or main) may start its own set-up now
   grid_dep_launch_next();
+  // launched programmatically: the stream's previous kernel (often the
+  // last call's decode kernel, whose workspace this may be) has finished
+  // and its writes are visible past this point
+  grid_dep_wait();
   const bool g4_shared = bp.M <= 2 && bp.g4_split > 0;  // split tiles add their partial sums into y2
   // (the sequence kernel, g4_split < 0, adds every partial sum into y2)
   if (P.nnz > 0 || g4_shared || bp.g4_split < 0) {
@@ -282,113 +244,154 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   }
   const int MB = bp.M;
   const int G = P.K / kGroup;
-  const int task = blockIdx.x * blockDim.x + threadIdx.x;
+  // eight threads per (group, token) task: thread `sub` forms the slots of
+  // group bytes 4 sub .. 4 sub + 3 (bytes past 25 are none), the task's
+  // threads exchange them through shared memory and each writes a share of
+  // the task's outputs; C and S are summed over the eight.
+  __shared__ __half sv[kPrepTasks][26][5];
+  const int tib = threadIdx.x >> 3, sub = threadIdx.x & 7;
+  const int task = blockIdx.x * kPrepTasks + tib;
   // with M <= 2 the one-group-per-lane kernel runs; its operands cover whole
   // stages of SG groups (groups past G get zero activations and C/S)
   const int SG = g4::stage_groups(MB);
   const int Gx = MB <= 2 ? SG * g4::nstages(P.K, SG) : G;
-  if (task >= Gx * MB) return;
-  const int g = task / MB, m = task % MB;
+  const bool live = task < Gx * MB;
+  const int g = live ? task / MB : 0, m = live ? task % MB : 0;
+  const bool real = live && g < G;
+  float C = 0.f, S = 0.f;
+  if (real) {
+    const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
+    // this thread's activations: trits 20 sub .. min(20 sub + 19, 127)
+    // (group rows are 16-byte aligned, so the 40-byte runs are 8-byte
+    // aligned)
+    const int nb = sub < 6 ? 4 : sub == 6 ? 2 : 0;
+    uint2 xv[5];
+#pragma unroll
+    for (int i = 0; i < 5; ++i)
+      xv[i] = (4 * i < kGroup - 20 * sub) ? __ldg(reinterpret_cast<const uint2 *>(xr + 20 * sub) + i) : make_uint2(0u, 0u);
+    auto xg = [&](int j) -> float {  // activation 20 sub + j (0 past the group)
+      const uint2 &v = xv[j >> 2];
+      const uint32_t w = (j & 2) ? v.y : v.x;
+      return __half2float(__ushort_as_half((unsigned short)((j & 1) ? (w >> 16) : (w & 0xffffu))));
+    };
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (q >= nb) break;
+      const int b = 4 * sub + q;
+      const int ntr = b < 25 ? 5 : 3;
+      float x[5];
+#pragma unroll
+      for (int i = 0; i < 5; ++i) x[i] = i < ntr ? xg(5 * q + i) : 0.f;
+      const float z0 = x[0] - x[4] * (1.f / 81.f), z1 = x[1] - x[4] * (3.f / 81.f);
+      const float z2 = x[2] - x[4] * (9.f / 81.f), z3 = x[3] - x[4] * (27.f / 81.f);
+      const __half ha = __float2half_rn(z0), hb = __float2half_rn(z1);
+      const float fa = __half2float(ha), fb = __half2float(hb);
+      const __half hc = __float2half_rn(z2 - 0.25f * fa), hd = __float2half_rn(z3 - 0.25f * fb);
+      const __half he = __float2half_rn(x[4] * (256.f / 81.f));
+      sv[tib][b][0] = ha, sv[tib][b][1] = hb, sv[tib][b][2] = hc, sv[tib][b][3] = hd, sv[tib][b][4] = he;
+      // all digits 1: slots 4 + 1 + 1/4, 16 + 1, 4 + 121/256
+      C += 5.25f * (fa + fb) + 17.f * (__half2float(hc) + __half2float(hd)) + (4.f + 121.f / 256.f) * __half2float(he);
+      S += x[0] + x[1] + x[2] + x[3] + x[4];
+    }
+  }
+#pragma unroll
+  for (int o = 1; o < 8; o <<= 1) {
+    C += __shfl_xor_sync(0xffffffffu, C, o);
+    S += __shfl_xor_sync(0xffffffffu, S, o);
+  }
+  __syncwarp();
+  if (!live) return;
+  const __half z = __float2half_rn(0.f);
+  // slot k (0..4) of group byte b, zero outside the group
+  auto slot = [&](int b, int k) -> __half { return (b >= 0 && b < 26) ? sv[tib][b][k] : z; };
+  auto pk = [](__half lo, __half hi) -> uint32_t {
+    __half2 v = __halves2half2(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+  };
   // the group's lane position and slice: 4-group stages, group g % 4 and
   // token m; 8-group stages, lane (g % 8) / 2 and the lane's group g % 2
   const int gs = g / SG, gp = g % SG;
   const int g4c = SG == 8 ? gp >> 1 : gp, g4sl = SG == 8 ? gp & 1 : m;
-  unsigned char *g4b = P.wsB + P.map_off + kMapSlotBytes;
-  float *g4cs = reinterpret_cast<float *>(g4b + g4::pad256(g4::b_bytes(MB, P.K)));
-  unsigned char *g4dst = g4b + (int64_t)(gs * 2 + g4sl) * g4::slice_bytes(SG) + g4c * 16;
-  float *g4q = g4cs + (gs * 4 + g4c) * 4;  // (C_a, C_b, S_a, S_b) of the lane position
-  if (MB <= 2 && g >= G) {
-    for (int jp = 0; jp < g4::pairs(SG); ++jp) *reinterpret_cast<uint4 *>(g4dst + jp * 64) = make_uint4(0u, 0u, 0u, 0u);
-    g4q[g4sl] = g4q[2 + g4sl] = 0.f;
-    return;
-  }
-  const __half *xr = P.x + (int64_t)m * P.K + (int64_t)g * kGroup;
-  // the group's 128 activations, all loads issued at once (x rows are
-  // 16-byte aligned and groups are 256 bytes)
-  uint4 xv[kGroup / 8];
-#pragma unroll
-  for (int i = 0; i < kGroup / 8; ++i) xv[i] = __ldg(reinterpret_cast<const uint4 *>(xr) + i);
-  // activation j of the group (j known at compile time once unrolled)
-  auto xg = [&](int j) -> float {
-    const uint4 &v = xv[j >> 3];
-    const uint32_t w = (j & 6) == 0 ? v.x : (j & 6) == 2 ? v.y : (j & 6) == 4 ? v.z : v.w;
-    return __half2float(__ushort_as_half((unsigned short)((j & 1) ? (w >> 16) : (w & 0xffffu))));
-  };
-  // activation slots of the 26 bytes, rounded to fp16
-  __half ya[26], yb[26], yc[26], yd[26], ye[26];
-  float C = 0.f, S = 0.f;
-#pragma unroll
-  for (int b = 0; b < 26; ++b) {
-    const int ntr = b < 25 ? 5 : 3;
-    float x[5];
-#pragma unroll
-    for (int i = 0; i < 5; ++i) x[i] = i < ntr ? xg(5 * b + i) : 0.f;
-    const float z0 = x[0] - x[4] * (1.f / 81.f), z1 = x[1] - x[4] * (3.f / 81.f);
-    const float z2 = x[2] - x[4] * (9.f / 81.f), z3 = x[3] - x[4] * (27.f / 81.f);
-    ya[b] = __float2half_rn(z0);
-    yb[b] = __float2half_rn(z1);
-    const float fa = __half2float(ya[b]), fb = __half2float(yb[b]);
-    yc[b] = __float2half_rn(z2 - 0.25f * fa);
-    yd[b] = __float2half_rn(z3 - 0.25f * fb);
-    ye[b] = __float2half_rn(x[4] * (256.f / 81.f));
-    // all digits 1: slots 4 + 1 + 1/4, 16 + 1, 4 + 121/256
-    C += 5.25f * (fa + fb) + 17.f * (__half2float(yc[b]) + __half2float(yd[b])) +
-         (4.f + 121.f / 256.f) * __half2float(ye[b]);
-    S += x[0] + x[1] + x[2] + x[3] + x[4];
-  }
-  if (MB == 1) {
-    if (g4sl)
-      g4_write_slots<8, 26>(g4dst, ya, yb, yc, yd, ye);
-    else
-      g4_write_slots<8, 0>(g4dst, ya, yb, yc, yd, ye);
-  } else if (MB == 2) {
-    if (g & 1)
-      g4_write_slots<4, 2>(g4dst, ya, yb, yc, yd, ye);
-    else
-      g4_write_slots<4, 0>(g4dst, ya, yb, yc, yd, ye);
-  }
   if (MB <= 2) {
-    g4q[g4sl] = C;
-    g4q[2 + g4sl] = S;
+    unsigned char *g4b = P.wsB + P.map_off + kMapSlotBytes;
+    float *g4cs = reinterpret_cast<float *>(g4b + g4::pad256(g4::b_bytes(MB, P.K)));
+    unsigned char *g4dst = g4b + (int64_t)(gs * 2 + g4sl) * g4::slice_bytes(SG) + g4c * 16;
+    // activation slots for the one-group-per-lane kernel: MMA j = 5 i + r
+    // of the lane's window words takes W, W' of window byte 4 i + r (r < 4)
+    // or the fifth-slot words of window bytes 4 i .. 4 i + 3 (r = 4);
+    // window byte beta is group byte beta - offs (offs = 26 for the second
+    // group of a lane in an 8-group stage, 2 for the odd groups of a
+    // 4-group stage)
+    const int offs = SG == 8 ? (g4sl ? 26 : 0) : (g & 1 ? 2 : 0);
+    const int nj = 5 * g4::words(SG);
+    for (int jp = sub; jp < g4::pairs(SG); jp += 8) {
+      uint32_t w[4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int j = 2 * jp + h, i = j / 5, r5 = j % 5;
+        uint32_t b0 = 0u, b1 = 0u;
+        if (real && j < nj) {
+          if (r5 < 4) {
+            const int b = 4 * i + r5 - offs;
+            if (b >= 0 && b < 26) {
+              b0 = pk(sv[tib][b][0], sv[tib][b][1]);
+              b1 = pk(sv[tib][b][2], sv[tib][b][3]);
+            }
+          } else {
+            b0 = pk(slot(4 * i - offs, 4), slot(4 * i + 1 - offs, 4));
+            b1 = pk(slot(4 * i + 2 - offs, 4), slot(4 * i + 3 - offs, 4));
+          }
+        }
+        w[2 * h] = b0;
+        w[2 * h + 1] = b1;
+      }
+      *reinterpret_cast<uint4 *>(g4dst + jp * 64) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    if (sub == 0) {
+      float *g4q = g4cs + (gs * 4 + g4c) * 4;  // (C_a, C_b, S_a, S_b) of the lane position
+      g4q[g4sl] = C;
+      g4q[2 + g4sl] = S;
+    }
   }
+  if (!real) return;
+  // the general decode kernels' per-group layout: lane position c's two
+  // window words give W, W' of their bytes (words 0..15) and the four
+  // fifth-slot words (16..19), as chunk pairs of 16 bytes
   const int GL = g % kStageG;  // the group's index in its stage fixes its window
   unsigned char *Bg = P.wsB + (int64_t)g * kBTok * MB;
-  const __half z = __float2half_rn(0.f);
-  for (int c = 0; c < 4; ++c) {
+  for (int it = sub; it < 4 * kCP; it += 8) {
+    const int c = it / kCP, cp = it % kCP;
     // group byte of byte k of lane c's word i (0: first, 1: second), or -1
     auto byte_of = [&](int i, int k) -> int {
       const int b = 4 * (first_word(GL, c) + 4 * i) + k - 26 * GL;
       return (b >= 0 && b < 26) ? b : -1;
     };
-    uint32_t words[20];
-    for (int i = 0; i < 2; ++i) {
-      for (int k = 0; k < 4; ++k) {
-        const int b = byte_of(i, k);
-        __half2 w0 = __halves2half2(z, z), w1 = __halves2half2(z, z);
-        if (b >= 0) {
-          w0 = __halves2half2(ya[b], yb[b]);
-          w1 = __halves2half2(yc[b], yd[b]);
-        }
-        words[2 * (4 * i + k)] = *reinterpret_cast<uint32_t *>(&w0);
-        words[2 * (4 * i + k) + 1] = *reinterpret_cast<uint32_t *>(&w1);
+    uint32_t w[4];
+    if (cp < 4) {
+      // words 4 cp .. 4 cp + 3: W, W' of bytes k = 2 cp and 2 cp + 1 of the words (i = cp / 2)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int bi = 2 * cp + e, b = byte_of(bi >> 2, bi & 3);
+        w[2 * e] = b >= 0 ? pk(sv[tib][b][0], sv[tib][b][1]) : 0u;
+        w[2 * e + 1] = b >= 0 ? pk(sv[tib][b][2], sv[tib][b][3]) : 0u;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int b0 = byte_of(i >> 1, 2 * (i & 1)), b1 = byte_of(i >> 1, 2 * (i & 1) + 1);
+        w[i] = pk(b0 >= 0 ? sv[tib][b0][4] : z, b1 >= 0 ? sv[tib][b1][4] : z);
       }
     }
-    for (int i = 0; i < 4; ++i) {
-      const int b0 = byte_of(i >> 1, 2 * (i & 1)), b1 = byte_of(i >> 1, 2 * (i & 1) + 1);
-      __half2 v = __halves2half2(b0 >= 0 ? ye[b0] : z, b1 >= 0 ? ye[b1] : z);
-      words[16 + i] = *reinterpret_cast<uint32_t *>(&v);
-    }
-    for (int cp = 0; cp < kCP; ++cp) {
-      uint4 q = make_uint4(words[4 * cp], words[4 * cp + 1], words[4 * cp + 2], words[4 * cp + 3]);
-      *reinterpret_cast<uint4 *>(Bg + ((m * kCP + cp) * 4 + c) * kBLane) = q;
-    }
+    *reinterpret_cast<uint4 *>(Bg + ((m * kCP + cp) * 4 + c) * kBLane) = make_uint4(w[0], w[1], w[2], w[3]);
   }
-  // C, S of token m in its 8-token tile's block; unused tokens' entries zero
-  float *cs = P.wsCS + (int64_t)g * (cs_group_bytes(MB) / 4);
-  cs[(m >> 3) * 16 + (m & 7)] = C;
-  cs[(m >> 3) * 16 + 8 + (m & 7)] = S;
-  if (m == 0)
-    for (int mm = MB; mm < (MB > 8 ? 16 : 8); ++mm) cs[(mm >> 3) * 16 + (mm & 7)] = cs[(mm >> 3) * 16 + 8 + (mm & 7)] = 0.f;
+  if (sub == 0) {
+    // C, S of token m in its 8-token tile's block; unused tokens' entries zero
+    float *cs = P.wsCS + (int64_t)g * (cs_group_bytes(MB) / 4);
+    cs[(m >> 3) * 16 + (m & 7)] = C;
+    cs[(m >> 3) * 16 + 8 + (m & 7)] = S;
+    if (m == 0)
+      for (int q = MB; q < (MB > 8 ? 16 : 8); ++q) cs[(q >> 3) * 16 + (q & 7)] = cs[(q >> 3) * 16 + 8 + (q & 7)] = 0.f;
+  }
 }
 
 // ------------------------------------------------------------ plane 2
@@ -751,7 +754,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
   unsigned char *recbuf = dynq + kQRecOff;
   {
     uint32_t *lut = reinterpret_cast<uint32_t *>(dynq + kArena1);
-    for (int i = tid; i < 256 * 32; i += kQThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+    lut_fill_replicated(lut, tid, kQThreads);
     for (int i = tid; i < kQMaxSpanRows * 8; i += kQThreads) acc[i] = 0.f;
     for (int i = tid; i < kQMaxG; i += kQThreads) gcnt[i] = 0;
   }
@@ -965,7 +968,7 @@ __global__ void __launch_bounds__(c_threads(TWO), 1)
   }
   {
     uint32_t *lut = reinterpret_cast<uint32_t *>(dync + kArena1);
-    for (int i = tid; i < 256 * 32; i += c_threads(TWO)) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+    lut_fill_replicated(lut, tid, c_threads(TWO));
   }
   __syncthreads();
   // the work below reads the prep kernel's output (launched programmatically
@@ -1043,7 +1046,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ---- one-time set-up: the lane-replicated table, barriers
   {
     uint32_t *lut = reinterpret_cast<uint32_t *>(dyn + kArena1);
-    for (int i = tid; i < 256 * 32; i += kThreads) lut[(i >> 5) * 64 + (i & 31)] = lut_word(i >> 5);
+    lut_fill_replicated(lut, tid, kThreads);
   }
   if (tid == 0) {
     for (int i = 0; i < NS; ++i) {
@@ -1459,6 +1462,23 @@ static cudaError_t build_templates(const BatchParams &bp, bool g4path, mm::MapTe
   return cudaSuccess;
 }
 
+// The prep kernel, launched programmatically after the stream's previous
+// kernel (it waits for that kernel before touching memory), so that its
+// launch overlaps the previous kernel's tail.
+static cudaError_t launch_prep(const BatchParams &bp, const mm::MapTemplates &mt, int32_t *counter, int gtasks,
+                               cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((gtasks + mm::kPrepTasks - 1) / mm::kPrepTasks, bp.count);
+  cfg.blockDim = dim3(128);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, mm::gemv_mma_prep_kernel, bp, mt, counter);
+}
+
 template <bool F32>
 static cudaError_t launch_mm_one(const BatchParams &bp, cudaStream_t s);
 
@@ -1547,8 +1567,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   }
   const int sg = g4::stage_groups(bp.M);
   const int gtasks = (g4path ? sg * ((gmax + sg - 1) / sg) : gmax) * bp.M;
-  mm::gemv_mma_prep_kernel<<<dim3((gtasks + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, counter);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_prep(bp, mt, counter, gtasks, s);
   if (e != cudaSuccess) return e;
   // more than 8 tokens in one pass needs every second plane indexed (the
   // other plane-2 kernels take 8 tokens at most)
@@ -1611,8 +1630,7 @@ cudaError_t launch_gemv_sequence(const BatchParams &bp_in, int barrier_extra, cu
   thread_local mm::MapTemplates mt;
   if (cudaError_t e = build_templates(bp, true, mt)) return e;
   const int gtasks = g4::stage_groups(1) * ((gmax + g4::stage_groups(1) - 1) / g4::stage_groups(1));
-  mm::gemv_mma_prep_kernel<<<dim3((gtasks + 127) / 128, bp.count), 128, 0, s>>>(bp, mt, nullptr);
-  cudaError_t e = cudaGetLastError();
+  const cudaError_t e = launch_prep(bp, mt, nullptr, gtasks, s);
   if (e != cudaSuccess) return e;
   return launch_gemv_seq(bp, num_sms_mm(), barrier_extra, s);
 }

@@ -55,6 +55,10 @@ class tq_ew_weight(ctypes.Structure):
                 ("alpha0", ctypes.c_void_p), ("alpha1", ctypes.c_void_p)]
 
 
+class tq_ew_problem(ctypes.Structure):
+    _fields_ = [("w", tq_ew_weight), ("x", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
 class tq_host_weight(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("N", ctypes.c_int32), ("K", ctypes.c_int32), ("nnz", ctypes.c_int64),
                 ("plane1", ctypes.c_void_p), ("salience", ctypes.c_void_p), ("rowptr", ctypes.c_void_p),
@@ -121,6 +125,10 @@ def lib():
             L.tq_ew_linear.argtypes = [i32, i32, i32, EW, vp, vp, vp, sz, vp]
             L.tq_ew_linear_f32out.restype = ctypes.c_int
             L.tq_ew_linear_f32out.argtypes = [i32, i32, i32, EW, vp, vp, vp, sz, vp]
+            L.tq_ew_batched_workspace_bytes.restype = sz
+            L.tq_ew_batched_workspace_bytes.argtypes = [i32, i32, ctypes.POINTER(tq_ew_problem)]
+            L.tq_ew_linear_batched.restype = ctypes.c_int
+            L.tq_ew_linear_batched.argtypes = [i32, i32, ctypes.POINTER(tq_ew_problem), vp, sz, vp]
             L.tq_linear_sequence.restype = ctypes.c_int
             L.tq_linear_sequence.argtypes = [i32, i32, ctypes.POINTER(tq_problem), vp, sz, vp]
             L.tq_sequence_selftest.restype = ctypes.c_int
@@ -653,3 +661,26 @@ def tq_ew_linear(x, w: EwWeight, y=None, ws=None, stream=None, f32=False):
     fn = lib().tq_ew_linear_f32out if f32 else lib().tq_ew_linear
     _check(fn(M, w.N, K, ctypes.byref(s), _p(x), _p(y), _p(ws), ws.numel(), _stream(stream)), "tq_ew_linear")
     return y
+
+
+class EwBatch:
+    """A prepared tq_ew_problem array (host memory) and its device workspace."""
+
+    def __init__(self, M, items, device=None):
+        self.M = M
+        self.items = list(items)  # (EwWeight, x, y); keeps tensors alive
+        self.arr = (tq_ew_problem * len(self.items))()
+        for i, (w, x, y) in enumerate(self.items):
+            self.arr[i].w = w.struct()
+            self.arr[i].x = x.data_ptr()
+            self.arr[i].y = y.data_ptr()
+        nbytes = int(lib().tq_ew_batched_workspace_bytes(M, len(self.items), self.arr))
+        if nbytes == 0:
+            raise TQError(-2, "tq_ew_batched_workspace_bytes")
+        dev = device if device is not None else self.items[0][1].device
+        self.ws = workspace(nbytes, dev)
+
+
+def tq_ew_linear_batched(batch: EwBatch, stream=None):
+    _check(lib().tq_ew_linear_batched(batch.M, len(batch.items), batch.arr, _p(batch.ws), batch.ws.numel(),
+                                      _stream(stream)), "tq_ew_linear_batched")

@@ -93,6 +93,34 @@ def test_host_side_argument_errors_without_gpu():
     assert tq.tq_workspace_bytes(1, 0, 4096) == 0
 
 
+def test_elementwise_workspace_formulas():
+    """tq_ew_workspace_bytes = the views of the plane-1 pass (s1 and off
+    [N][G] fp16, zero salience words, zero rowptr) and its fp32 result, each
+    256-padded, plus the decode path's workspace; the batched form sums the
+    views and results of every problem and then every problem's decode-path
+    workspace, and refuses M > 16."""
+    from paper_2609_09240_gb300 import tq
+    L = tq.lib()
+    pad = lambda b: (b + 255) // 256 * 256
+
+    def parts(M, N, K):
+        G, W = K // 128, (K // 128 + 31) // 32
+        return 2 * pad(N * G * 2) + pad(N * W * 4) + pad((N + 1) * 4) + pad(M * N * 4)
+    for M, N, K in ((1, 4096, 4096), (2, 300, 1152), (5, 129, 4224), (40, 256, 1152)):
+        assert L.tq_ew_workspace_bytes(M, N, K) == parts(M, N, K) + tq.tq_workspace_bytes(M, N, K)
+    assert L.tq_ew_workspace_bytes(1, 4096, 100) == 0 and L.tq_ew_workspace_bytes(0, 64, 128) == 0
+    shapes = [(4096, 4096), (1024, 4096), (4096, 12288)]
+    arr = (tq.tq_ew_problem * 3)()
+    for i, (N, K) in enumerate(shapes):
+        arr[i].w.N, arr[i].w.K = N, K
+    for M in (1, 2, 16):
+        want = sum(parts(M, N, K) + tq.tq_workspace_bytes(M, N, K) for N, K in shapes)
+        assert L.tq_ew_batched_workspace_bytes(M, 3, arr) == want
+    assert L.tq_ew_batched_workspace_bytes(17, 3, arr) == 0
+    arr[1].w.K = 100
+    assert L.tq_ew_batched_workspace_bytes(1, 3, arr) == 0
+
+
 def test_binding_argument_counts_match_the_header():
     """Every function the ctypes binding declares takes as many arguments as
     its prototype in include/tq.h."""

@@ -3,7 +3,9 @@
 bytes equal the oracle's packing bit for bit and tq_ew_unpack inverts them;
 tq_ew_linear satisfies |y - y_ref| <= 2e-3 * sum_k |W x| per element on
 ragged shapes, 1..40 tokens (decode and prefill paths under the mask-3 pass)
-and Qwen3-8B projection shapes (sampled rows)."""
+and Qwen3-8B projection shapes (sampled rows); tq_ew_linear_batched meets
+the same bound on mixed batches and on a Qwen3-8B layer's seven
+projections."""
 import numpy as np
 import pytest
 import torch
@@ -120,3 +122,59 @@ def test_linear_qwen3_8b_shapes_sampled_rows(H, N, K):
     y = tq.tq_ew_linear(H.dev(xb), _pack(H, w))
     H.device_status_ok()
     H.assert_close(y.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M", [1, 2, 5, 16])
+def test_batched_parity_mixed_shapes(H, M):
+    from paper_2609_09240_gb300 import tq
+    shapes = [(512, 1024), (37, 256), (300, 2560), (129, 4224), (1, 128)]
+    items, refs = [], []
+    for i, (N, K) in enumerate(shapes):
+        w = wl.gen_ew_weights(N, K, config=17, proj=i)
+        xb = wl.gen_x(M, K, config=17, proj=i)
+        mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+        assert st == 0
+        refs.append(ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1))
+        items.append((_pack(H, w), H.dev(xb), torch.empty((M, N), dtype=torch.float16, device="cuda")))
+    b = tq.EwBatch(M, items)
+    tq.tq_ew_linear_batched(b)
+    H.device_status_ok()
+    for (_, _, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy().astype(np.float64), y_ref, a_ref)
+
+
+def test_batched_qwen3_8b_layer_sampled_rows(H):
+    """The seven projections of a Qwen3-8B layer in one batched call, M = 1,
+    64 sampled rows of each against the oracle; the same problems through
+    tq_ew_linear one by one agree within the bound as well."""
+    from paper_2609_09240_gb300 import tq
+    items, refs, singles = [], [], []
+    for p in wl.config_projections(4):
+        w = wl.gen_ew_weights(p.N, p.K, config=18, proj=p.proj)
+        xb = wl.gen_x(1, p.K, config=18, proj=p.proj)
+        mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+        assert st == 0
+        rows = np.sort(np.random.default_rng(p.proj).choice(p.N, size=64, replace=False))
+        refs.append((rows, ew.linear(xb, p.K, mp, p1, rp, p2, w.mu, w.a0, w.a1, rows=rows)))
+        g = _pack(H, w)
+        x = H.dev(xb)
+        items.append((g, x, torch.empty((1, p.N), dtype=torch.float16, device="cuda")))
+        singles.append(tq.tq_ew_linear(x, g))
+    tq.tq_ew_linear_batched(tq.EwBatch(1, items))
+    H.device_status_ok()
+    for (_, _, y), ys, (rows, (y_ref, a_ref)) in zip(items, singles, refs):
+        H.assert_close(y.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
+        H.assert_close(ys.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
+
+
+def test_batched_rejects_bad_arguments(H):
+    from paper_2609_09240_gb300 import tq
+    w = _pack(H, wl.gen_ew_weights(64, 256, config=19))
+    x = torch.zeros((17, 256), dtype=torch.float16, device="cuda")
+    y = torch.empty((17, 64), dtype=torch.float16, device="cuda")
+    with pytest.raises(tq.TQError):
+        tq.EwBatch(17, [(w, x, y)])  # M > 16: no batched workspace
+    b = tq.EwBatch(1, [(w, x[:1], y[:1])])
+    b.arr[0].x = b.arr[0].x + 2  # misaligned activations
+    with pytest.raises(tq.TQError):
+        tq.tq_ew_linear_batched(b)
