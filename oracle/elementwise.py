@@ -142,11 +142,13 @@ def unpack(N: int, K: int, mplane: np.ndarray, p1: np.ndarray, rp: np.ndarray, p
 # in the paper), like the group format's second-plane index: the elements of
 # masks 0..2 of every row, block by block of IDX_BLOCK elements along K, in
 # increasing k, each as one uint16 entry
-#     (k mod IDX_BLOCK) | code << 10,  code = 9 q + 3 (T0 + 1) + (T1 + 1),
+#     (k mod IDX_BLOCK) | code << 11,  code = 9 q + 3 (T0 + 1) + (T1 + 1),
 # with int32 offsets[n * nb + b] of row n's block b (nb = ceil(K / IDX_BLOCK),
 # offsets[N nb] = all entries).  Everything the masks 0..2 add to the
-# mask-3 form of a row is in its entries.
-IDX_BLOCK = 1024
+# mask-3 form of a row is in its entries.  A block of 2048 elements makes an
+# entry's 11 offset bits and 5 code bits (27 codes) fill its 16 bits.
+IDX_BLOCK = 2048
+IDX_SHIFT = 11
 
 
 def correction_index(T0: np.ndarray, T1: np.ndarray, mask: np.ndarray):
@@ -159,7 +161,7 @@ def correction_index(T0: np.ndarray, T1: np.ndarray, mask: np.ndarray):
     offsets[1:] = np.cumsum(counts)
     q = mask[rows, cols].astype(np.int64)
     code = 9 * q + 3 * (T0[rows, cols].astype(np.int64) + 1) + (T1[rows, cols].astype(np.int64) + 1)
-    entries = (cols % IDX_BLOCK) | (code << 10)
+    entries = (cols % IDX_BLOCK) | (code << IDX_SHIFT)
     return offsets.astype(np.int32), entries.astype(np.uint16)
 
 
@@ -173,7 +175,7 @@ def decode_index(N: int, K: int, offsets, entries):
     for n in range(N):
         for b in range(nb):
             for v in e[offsets[n * nb + b]:offsets[n * nb + b + 1]]:
-                k, code = b * IDX_BLOCK + (v & 1023), v >> 10
+                k, code = b * IDX_BLOCK + (v & (IDX_BLOCK - 1)), v >> IDX_SHIFT
                 mask[n, k], T0[n, k], T1[n, k] = code // 9, (code // 3) % 3 - 1, code % 3 - 1
     return mask, T0, T1
 

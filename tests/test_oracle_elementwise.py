@@ -179,26 +179,26 @@ def test_order1_masks_ignore_alpha1_and_mu_is_per_mask():
 
 
 def test_index_entries_by_hand():
-    # row 0: k = 3 mask 0 (T0 = 1, T1 = -1), k = 1030 mask 2 (T0 = -1); row 1: k = 5 mask 1 (T0 = 0, T1 = 1)
-    N, K = 2, 1152
+    # row 0: k = 3 mask 0 (T0 = 1, T1 = -1), k = 2060 mask 2 (T0 = -1); row 1: k = 5 mask 1 (T0 = 0, T1 = 1)
+    N, K = 2, 2176
     mask = np.full((N, K), 3, np.uint8)
     T0 = np.zeros((N, K), np.int8)
     T1 = np.zeros((N, K), np.int8)
     mask[0, 3], T0[0, 3], T1[0, 3] = 0, 1, -1
-    mask[0, 1030], T0[0, 1030] = 2, -1
+    mask[0, 2060], T0[0, 2060] = 2, -1
     mask[1, 5], T1[1, 5] = 1, 1
     off, ent = ew.correction_index(T0, T1, mask)
-    # nb = 2 blocks per row; code = 9 q + 3 (T0 + 1) + (T1 + 1)
+    # nb = 2 blocks of 2048 per row; code = 9 q + 3 (T0 + 1) + (T1 + 1) in bits 11..15
     assert off.tolist() == [0, 1, 2, 3, 3]
-    assert ent.tolist() == [3 | (0 + 6 + 0) << 10, 6 | (18 + 0 + 1) << 10, 5 | (9 + 3 + 2) << 10]
+    assert ent.tolist() == [3 | (0 + 6 + 0) << 11, 12 | (18 + 0 + 1) << 11, 5 | (9 + 3 + 2) << 11]
 
 
-@pytest.mark.parametrize("N,K", [(1, 128), (7, 1024), (33, 1152), (16, 4224)])
+@pytest.mark.parametrize("N,K", [(1, 128), (7, 2048), (33, 1152), (16, 4224)])
 def test_index_offsets_and_decoding(N, K):
     w = wl.gen_ew_weights(N, K, config=6, proj=N)
     off, ent = ew.correction_index(w.T0, w.T1, w.mask)
-    nb = (K + 1023) // 1024
-    want = [int((w.mask[n, b * 1024:(b + 1) * 1024] != 3).sum()) for n in range(N) for b in range(nb)]
+    nb = (K + 2047) // 2048
+    want = [int((w.mask[n, b * 2048:(b + 1) * 2048] != 3).sum()) for n in range(N) for b in range(nb)]
     assert np.array_equal(np.diff(off), want) and off[0] == 0
     m, T0, T1 = ew.decode_index(N, K, off, ent)
     sel = w.mask != 3
@@ -212,7 +212,7 @@ def test_index_correction_plus_mask3_form_is_exact():
     (mu_q - mu_3) + (alpha0_q - alpha0_3) T0 + alpha1_q T1 times x equals the
     oracle's linear exactly."""
     rng = np.random.default_rng(11)
-    N, K = 4, 2048 + 128
+    N, K = 4, 4096 + 128
     mask = rng.choice(4, size=(N, K), p=[0.05, 0.1, 0.15, 0.7]).astype(np.uint8)
     T0 = rng.integers(-1, 2, (N, K)).astype(np.int8)
     T1 = (rng.integers(-1, 2, (N, K)) * (mask <= 1)).astype(np.int8)
@@ -224,14 +224,14 @@ def test_index_correction_plus_mask3_form_is_exact():
     assert st == 0
     y, _ = ew.linear(_bits(x), K, mp, p1, rp, p2, _bits(mu), _bits(a0), _bits(a1))
     off, ent = ew.correction_index(T0, T1, mask)
-    nb = (K + 1023) // 1024
+    nb = (K + 2047) // 2048
     a1x = np.concatenate([a1, np.zeros((N, 2))], axis=1)
     for n in range(N):
         base = (mu[n, 3] + a0[n, 3] * T0[n].astype(np.float64)) @ x.T
         corr = np.zeros(2)
         for b in range(nb):
             for v in ent[off[n * nb + b]:off[n * nb + b + 1]].astype(np.int64):
-                k, code = b * 1024 + (v & 1023), v >> 10
+                k, code = b * 2048 + (v & 2047), v >> 11
                 q, t0, t1 = code // 9, (code // 3) % 3 - 1, code % 3 - 1
                 corr += ((mu[n, q] - mu[n, 3]) + (a0[n, q] - a0[n, 3]) * t0 + a1x[n, q] * t1) * x[:, k]
         assert np.array_equal(base + corr, y[:, n])
