@@ -19,6 +19,7 @@ context.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import subprocess
@@ -802,7 +803,7 @@ def sub_elementwise(dev, peak):
     import workloads as wl
     from paper_2609_09240_gb300 import tq
 
-    base, layer_bytes = [], 0
+    base, layer_bytes, index_bytes = [], 0, 0
     for p in wl.config_projections(4):
         g = torch.Generator(device=dev)
         g.manual_seed(900 + p.proj)
@@ -816,20 +817,27 @@ def sub_elementwise(dev, peak):
         mu = (torch.randn((N, 4), generator=g, device=dev) * 1e-3).half()
         a0 = torch.empty((N, 4), device=dev).log_normal_(-4.0, 0.5, generator=g).half()
         a1 = torch.empty((N, 2), device=dev).log_normal_(-4.0, 0.5, generator=g).half()
-        w = tq.pack_ew_weight(T0, T1, mask, mu, a0, a1)
+        w = tq.ew_index(tq.pack_ew_weight(T0, T1, mask, mu, a0, a1))
         del u, u0, u1, T0, T1, mask
         base.append(w)
         layer_bytes += w.packed_bytes()
+        index_bytes += w.index_bytes()
     R = -(-4 * L2_BYTES // layer_bytes)
     clone = lambda w: tq.EwWeight(w.N, w.K, w.mask.clone(), w.plane1.clone(), w.p2rowptr.clone(), w.plane2.clone(),
-                                  w.mu.clone(), w.alpha0.clone(), w.alpha1.clone())
+                                  w.mu.clone(), w.alpha0.clone(), w.alpha1.clone(), w.idx_off.clone(), w.idx.clone())
     layers = [[(w if r == 0 else clone(w), wl.gen_x_torch(1, w.K, dev, 950 + 8 * r + i),
                 torch.empty((1, w.N), dtype=torch.float16, device=dev)) for i, w in enumerate(base)] for r in range(R)]
     wss = [tq.workspace(int(tq.lib().tq_ew_workspace_bytes(1, w.N, w.K)), dev) for w in base]
     batches = [tq.EwBatch(1, items) for items in layers]
+    plain = [tq.EwBatch(1, [(dataclasses.replace(w, idx_off=None, idx=None), x, y) for w, x, y in items])
+             for items in layers]
 
     def batched():
         for b in batches:
+            tq.tq_ew_linear_batched(b)
+
+    def batched_plain():
+        for b in plain:
             tq.tq_ew_linear_batched(b)
 
     def calls():
@@ -838,15 +846,18 @@ def sub_elementwise(dev, peak):
                 tq.tq_ew_linear(x, w, y=y, ws=wsb)
 
     ms = graph_ms(batched, reps=5) / R
+    ms_plain = graph_ms(batched_plain, reps=5) / R
     ms_unb = graph_ms(calls, reps=5) / R
     gbs = layer_bytes / (ms * 1e-3) / 1e9
     n_w = sum(w.N * w.K for w in base)
     return {"workload": "qwen3-8b one layer in the element-wise four-mask form (coverages 0.5/3.1/10/86.4 %), M=1",
-            "us_per_layer": ms * 1e3, "us_per_layer_unbatched": ms_unb * 1e3, "packed_bytes": layer_bytes,
+            "us_per_layer": ms * 1e3, "us_per_layer_without_index": ms_plain * 1e3,
+            "us_per_layer_unbatched": ms_unb * 1e3, "packed_bytes": layer_bytes, "index_bytes": index_bytes,
             "bits_per_weight": 8 * layer_bytes / n_w, "packed_gbs": gbs, "frac_of_hbm_peak": gbs / peak,
             "timing": f"{R} rotated copies of the layer ({R * layer_bytes / 2 ** 20:.0f} MiB > 4 x L2); one "
-                      "tq_ew_linear_batched call per layer (views, prep, plane 1, correction: 4 launches), and "
-                      "(unbatched) seven tq_ew_linear calls per layer; each replayed as a CUDA graph"}
+                      "tq_ew_linear_batched call per layer (views, prep, plane 1, correction: 4 launches) with the "
+                      "correction index, the same without it (mask-plane correction), and (unbatched) seven "
+                      "tq_ew_linear calls per layer with the index; each replayed as a CUDA graph"}
 
 
 def cpu_baseline_single(budget_s):

@@ -381,6 +381,11 @@ typedef struct {
   const uint16_t *mu;
   const uint16_t *alpha0;
   const uint16_t *alpha1;
+  /* Optional correction index (tq_ew_index_offsets / tq_ew_index_fill), or
+   * both NULL: with it the linear reads the index instead of the mask plane
+   * and planes for the elements of masks 0..2. */
+  const int32_t *idx_off;
+  const uint16_t *idx;
 } tq_ew_weight;
 
 /* p2rowptr[N + 1] from the mask ids (uint8 [N][K], 0..3): bytes per row =
@@ -403,6 +408,22 @@ TQ_API tq_status tq_ew_pack(int32_t N, int32_t K, const int8_t *T0, const int8_t
 TQ_API tq_status tq_ew_unpack(int32_t N, int32_t K, const uint32_t *mask, const uint8_t *plane1,
                               const int32_t *p2rowptr, const uint8_t *plane2, int8_t *T0, int8_t *T1,
                               uint8_t *mask_ids, uint32_t *d_status, void *stream);
+/* Correction index (this library's, no counterpart in the paper; derived
+ * from a packed weight once, like tq_plane2_index for the group format):
+ * for every row n and block b of 2048 elements along K, the elements of
+ * masks 0..2 in increasing k as uint16 entries
+ *   (k mod 2048) | code << 11,  code = 9 q + 3 (T0 + 1) + (T1 + 1),
+ * from entry idx_off[n nb + b] on (nb = ceil(K / 2048); idx_off[N nb] =
+ * all entries, 2 bytes each).  tq_ew_index_offsets writes idx_off
+ * (int32 [N nb + 1]) from the mask plane; the caller reads idx_off[N nb] to
+ * size the entries; tq_ew_index_fill writes them from the weight's mask
+ * plane, plane 1, p2rowptr and plane 2 (w's index fields are ignored).
+ * Rows whose offsets or p2rowptr do not match the mask plane are skipped
+ * and reported as TQ_DATA_BAD_ROWPTR, bytes above 242 as TQ_DATA_BAD_BYTE
+ * (in *d_status).  N K must stay below 2^31. */
+TQ_API tq_status tq_ew_index_offsets(int32_t N, int32_t K, const uint32_t *mask, int32_t *idx_off, void *stream);
+TQ_API tq_status tq_ew_index_fill(int32_t N, int32_t K, const tq_ew_weight *w, const int32_t *idx_off, uint16_t *idx,
+                                  uint32_t *d_status, void *stream);
 /* Workspace of tq_ew_linear (per-call views of alpha0 / mu of mask 3 for
  * the plane-1 pass, its fp32 result and the decode path's workspace). */
 TQ_API size_t tq_ew_workspace_bytes(int32_t M, int32_t N, int32_t K);

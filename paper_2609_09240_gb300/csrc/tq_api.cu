@@ -29,6 +29,10 @@ cudaError_t launch_ew_pack(int N, int K, const int8_t *T0, const int8_t *T1, con
 cudaError_t launch_ew_unpack(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
                              const uint8_t *plane2, int8_t *T0, int8_t *T1, uint8_t *mask, uint32_t *status,
                              cudaStream_t s);
+cudaError_t launch_ew_index_offsets(int N, int K, const uint32_t *mplane, int32_t *off, cudaStream_t s);
+cudaError_t launch_ew_index_fill(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
+                                 const uint8_t *plane2, const int32_t *off, uint16_t *idx, uint32_t *status,
+                                 cudaStream_t s);
 cudaError_t launch_ew_views(const EwCall *calls, int count, cudaStream_t s);
 cudaError_t launch_ew_correct(int M, const EwCall *calls, int count, bool f32, cudaStream_t s);
 int mma_rows_per_tile();
@@ -428,6 +432,8 @@ tq_status check_ew(int32_t M, const tq_ew_weight *w, const uint16_t *x, const vo
   if (!aligned16(w->plane1) || !aligned16(x) || ((uintptr_t)w->mask & 3u) || ((uintptr_t)w->p2rowptr & 3u) ||
       !aligned2(w->mu) || !aligned2(w->alpha0) || !aligned2(w->alpha1))
     return TQ_ERR_ALIGN;
+  if ((w->idx_off == nullptr) != (w->idx == nullptr)) return TQ_ERR_NULL;  // an index has both parts
+  if (w->idx_off && (((uintptr_t)w->idx_off & 3u) || !aligned2(w->idx))) return TQ_ERR_ALIGN;
   if (f32 ? ((uintptr_t)y & 3u) : !aligned2(y)) return TQ_ERR_ALIGN;
   (void)M;
   return TQ_OK;
@@ -531,6 +537,27 @@ tq_status tq_ew_unpack(int32_t N, int32_t K, const uint32_t *mask, const uint8_t
   if (((uintptr_t)mask & 3u) || ((uintptr_t)p2rowptr & 3u)) return TQ_ERR_ALIGN;
   return from_cuda(launch_ew_unpack(N, K, mask, plane1, p2rowptr, plane2, T0, T1, mask_ids, d_status,
                                     (cudaStream_t)stream));
+}
+
+tq_status tq_ew_index_offsets(int32_t N, int32_t K, const uint32_t *mask, int32_t *idx_off, void *stream) {
+  if (tq_status st = check_shape(N, K)) return st;
+  if ((int64_t)N * K >= (int64_t)1 << 31) return TQ_ERR_SHAPE;
+  if (!mask || !idx_off) return TQ_ERR_NULL;
+  if (((uintptr_t)mask & 3u) || ((uintptr_t)idx_off & 3u)) return TQ_ERR_ALIGN;
+  return from_cuda(launch_ew_index_offsets(N, K, mask, idx_off, (cudaStream_t)stream));
+}
+
+tq_status tq_ew_index_fill(int32_t N, int32_t K, const tq_ew_weight *w, const int32_t *idx_off, uint16_t *idx,
+                           uint32_t *d_status, void *stream) {
+  if (!w || !idx_off || !idx || !d_status) return TQ_ERR_NULL;
+  if (w->N != N || w->K != K) return TQ_ERR_SHAPE;
+  if (tq_status st = check_shape(N, K)) return st;
+  if ((int64_t)N * K >= (int64_t)1 << 31) return TQ_ERR_SHAPE;
+  if (!w->mask || !w->plane1 || !w->p2rowptr) return TQ_ERR_NULL;
+  if (((uintptr_t)w->mask & 3u) || ((uintptr_t)w->p2rowptr & 3u) || ((uintptr_t)idx_off & 3u) || !aligned2(idx))
+    return TQ_ERR_ALIGN;
+  return from_cuda(launch_ew_index_fill(N, K, w->mask, w->plane1, w->p2rowptr, w->plane2, idx_off, idx, d_status,
+                                        (cudaStream_t)stream));
 }
 
 size_t tq_ew_workspace_bytes(int32_t M, int32_t N, int32_t K) {

@@ -598,6 +598,117 @@ __global__ void __launch_bounds__(32 * kEwRowWarps) ew_plane2_unpack_kernel(int 
   if (st) atomicOr(status, st);
 }
 
+// ----------------------------------------------- element-wise correction index
+// Entries of masks 0..2 per row and 2048-element block (uint16
+// (k mod 2048) | code << 11, code = 9 q + 3 (T0 + 1) + (T1 + 1)), with int32
+// offsets[n nb + b] (nb = ceil(K / 2048)).
+constexpr int kIdxBlock = 2048, kIdxShift = 11;
+
+// Warp per row: the count of each block's mask-0..2 elements into
+// off[n nb + b + 1] (off[0] = 0); ew_scan_kernel turns them into offsets.
+__global__ void __launch_bounds__(32 * kEwRowWarps) ew_index_count_kernel(int N, int K, const uint32_t *plane,
+                                                                          int32_t *off) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kEwRowWarps + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const int WK = K / 16, nb = (K + kIdxBlock - 1) / kIdxBlock;
+  const uint32_t *mw = plane + (int64_t)n * WK;
+  for (int b = 0; b < nb; ++b) {
+    int c = 0;
+    for (int wi = b * (kIdxBlock / 16) + lane; wi < min(WK, (b + 1) * (kIdxBlock / 16)); wi += 32) {
+      const uint32_t m = mw[wi];
+      c += __popc(~(m & (m >> 1)) & 0x55555555u);
+    }
+    for (int o = 16; o; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+    if (lane == 0) off[(int64_t)n * nb + b + 1] = c;
+  }
+  if (n == 0 && lane == 0) off[0] = 0;
+}
+
+__device__ __forceinline__ int base3_digit(int v, int i) {
+  for (int j = 0; j < i; ++j) v /= 3;
+  return v % 3;
+}
+
+// Warp per row, 32 elements per step (lane = element): each mask-0..2
+// element's entry at its rank in the row; T0 from plane 1, T1 from plane 2
+// at the element's rank among the row's order-2 elements.  A row whose
+// offsets or plane-2 rowptr do not match its mask plane is skipped and
+// reported (TQ_DATA_BAD_ROWPTR), so nothing is written outside its range.
+__global__ void __launch_bounds__(32 * kEwRowWarps) ew_index_fill_kernel(int N, int K, const uint32_t *plane,
+                                                                         const uint8_t *plane1,
+                                                                         const int32_t *rowptr,
+                                                                         const uint8_t *plane2, const int32_t *off,
+                                                                         uint16_t *idx, uint32_t *status) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kEwRowWarps + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const int WK = K / 16, nb = (K + kIdxBlock - 1) / kIdxBlock;
+  const uint32_t *mw = plane + (int64_t)n * WK;
+  const int64_t e0 = off[(int64_t)n * nb];
+  int c3 = 0, c2 = 0;
+  for (int wi = lane; wi < WK; wi += 32) {
+    const uint32_t m = mw[wi];
+    c3 += __popc(~(m & (m >> 1)) & 0x55555555u);
+    c2 += __popc(~m & 0xaaaaaaaau);
+  }
+  for (int o = 16; o; o >>= 1) {
+    c3 += __shfl_xor_sync(0xffffffffu, c3, o);
+    c2 += __shfl_xor_sync(0xffffffffu, c2, o);
+  }
+  const int64_t b2 = rowptr[n], nb2 = (int64_t)rowptr[n + 1] - rowptr[n];
+  if ((int64_t)off[(int64_t)n * nb + nb] - e0 != c3 || (c2 + 4) / 5 != nb2) {
+    if (lane == 0) atomicOr(status, TQ_DATA_BAD_ROWPTR);
+    return;
+  }
+  const uint8_t *p1 = plane1 + (int64_t)n * row_bytes_of(K);
+  uint32_t st = 0;
+  int run = 0, r2 = 0;
+  for (int k0 = 0; k0 < K; k0 += 32) {
+    if (k0 % kIdxBlock == 0 && run != (int)(off[(int64_t)n * nb + k0 / kIdxBlock] - e0)) {
+      st |= TQ_DATA_BAD_ROWPTR;  // per-block offsets that do not match the mask plane
+      break;
+    }
+    const int k = k0 + lane;
+    const uint32_t q = k < K ? (mw[k >> 4] >> (2 * (k & 15))) & 3u : 3u;
+    const uint32_t bal3 = __ballot_sync(0xffffffffu, q != 3u), bal2 = __ballot_sync(0xffffffffu, q <= 1u);
+    if (q != 3u) {
+      const int kg = k % kGroup;
+      int v = p1[(int64_t)(k / kGroup) * kGroupBytes + kg / 5];
+      if (v > 242) st |= TQ_DATA_BAD_BYTE, v = 242;
+      const int d0 = base3_digit(v, kg % 5);
+      int d1 = 1;
+      if (q <= 1u) {
+        const int r = r2 + __popc(bal2 & lanemask_lt());
+        int u = plane2[b2 + r / 5];
+        if (u > 242) st |= TQ_DATA_BAD_BYTE, u = 242;
+        d1 = base3_digit(u, r % 5);
+      }
+      const uint32_t code = 9u * q + 3u * (uint32_t)d0 + (uint32_t)d1;
+      idx[e0 + run + __popc(bal3 & lanemask_lt())] = (uint16_t)((uint32_t)(k % kIdxBlock) | (code << kIdxShift));
+    }
+    run += __popc(bal3);
+    r2 += __popc(bal2);
+  }
+  for (int o = 16; o; o >>= 1) st |= __shfl_xor_sync(0xffffffffu, st, o);
+  if (lane == 0 && st) atomicOr(status, st);
+}
+
+cudaError_t launch_ew_index_offsets(int N, int K, const uint32_t *mplane, int32_t *off, cudaStream_t s) {
+  const int nb = (K + kIdxBlock - 1) / kIdxBlock;
+  ew_index_count_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, mplane, off);
+  ew_scan_kernel<<<1, 1024, 0, s>>>(N * nb, off);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ew_index_fill(int N, int K, const uint32_t *mplane, const uint8_t *plane1, const int32_t *rowptr,
+                                 const uint8_t *plane2, const int32_t *off, uint16_t *idx, uint32_t *status,
+                                 cudaStream_t s) {
+  ew_index_fill_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, mplane, plane1, rowptr,
+                                                                                       plane2, off, idx, status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_ew_rowptr(int N, int K, const uint8_t *mask, int32_t *rowptr, uint32_t *status, cudaStream_t s) {
   ew_count_kernel<<<(N + kEwRowWarps - 1) / kEwRowWarps, 32 * kEwRowWarps, 0, s>>>(N, K, mask, rowptr, status);
   ew_scan_kernel<<<1, 1024, 0, s>>>(N, rowptr);

@@ -37,10 +37,13 @@ struct Prob {
   const int32_t *p2rowptr;  // [N+1]
   const uint8_t *plane2;
   const __half *mu, *a0, *a1;  // [N][4], [N][4], [N][2]
+  const int32_t *idx_off;      // correction index (or null): offsets [N nb + 1]
+  const uint16_t *idx;         //   and entries
   const __half *x;             // [M][K]
   const float *ydense;         // [M][N]
   void *y;                     // [M][N], fp16 or fp32
-  int32_t N, K, S, blocks;
+  int32_t N, K, S, blocks;     // blocks = 0: the problem is the other kernel's
+  int32_t row_begin;           // first row of the problem among the index kernel's rows
 };
 template <typename T>
 struct Batch {
@@ -49,21 +52,33 @@ struct Batch {
 };
 static_assert(sizeof(Batch<Prob>) <= 32764 && sizeof(Batch<ViewProb>) <= 32764, "launch parameters");
 
-// Block row blockIdx.y = problem; thread per (row, group): s1 view = alpha0
-// of mask 3, off view = mu of mask 3; the views' salience words and rowptr
-// are zero (no second plane).
+// Block row blockIdx.y = problem: s1 view = alpha0 of mask 3, off view =
+// mu of mask 3 in every group of the row (eight groups per 16-byte store
+// when a row's views are whole 16-byte units); the views' salience words
+// and rowptr are zero (no second plane).
 __global__ void views_kernel(const __grid_constant__ Batch<ViewProb> bt) {
   const ViewProb &P = bt.prob[blockIdx.y];
   const int N = P.N, G = P.K / kGroup, W = sal_words_of(P.K);
-  const int64_t total = (int64_t)N * G;
-  const int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, step = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t i = i0; i < total; i += step) {
-    const int64_t n = i / G;
-    P.s1v[i] = P.a0[n * 4 + 3];
-    P.offv[i] = P.mu[n * 4 + 3];
+  const int i0 = blockIdx.x * blockDim.x + threadIdx.x, step = gridDim.x * blockDim.x;
+  const __half *mu = P.mu, *a0 = P.a0;
+  if (G % 8 == 0) {
+    const int G8 = G / 8;
+    uint4 *s1 = reinterpret_cast<uint4 *>(P.s1v), *of = reinterpret_cast<uint4 *>(P.offv);
+    for (int i = i0; i < N * G8; i += step) {
+      const int n = i / G8;
+      const uint32_t a = __half_as_ushort(a0[n * 4 + 3]) * 0x10001u, m = __half_as_ushort(mu[n * 4 + 3]) * 0x10001u;
+      s1[i] = make_uint4(a, a, a, a);
+      of[i] = make_uint4(m, m, m, m);
+    }
+  } else {
+    for (int i = i0; i < N * G; i += step) {
+      const int n = i / G;
+      P.s1v[i] = a0[n * 4 + 3];
+      P.offv[i] = mu[n * 4 + 3];
+    }
   }
-  for (int64_t i = i0; i < (int64_t)N * W; i += step) P.salv[i] = 0u;
-  for (int64_t i = i0; i <= N; i += step) P.rpv[i] = 0;
+  for (int i = i0; i < N * W; i += step) P.salv[i] = 0u;
+  for (int i = i0; i <= N; i += step) P.rpv[i] = 0;
 }
 
 // The five base-3 digits of a byte (values above 242 read as 242), two bits
@@ -244,6 +259,87 @@ __global__ void __launch_bounds__(32 * kWarps) correct_kernel(const __grid_const
   }
 }
 
+constexpr int kIdxBlock = 2048, kIdxShift = 11;  // the correction index's blocks and code position
+constexpr uint32_t kIdxNone = 31u << kIdxShift;  // a code that weighs nothing (pads a step)
+
+// The same correction from the correction index: warp per row, the warps
+// striding over the rows of every indexed problem of the call; the lanes
+// take a block's entries two at a time per step.  An entry names its element
+// k (within its block) and code = 9 q + 3 d0 + d1 (digits d = trit + 1),
+// whose weight (mu_q - mu_3) + (alpha0_q - alpha0_3) T0 + alpha1_q T1 is read
+// from the row's 27-entry table.  Only the entries and x are read: no mask
+// plane, plane-1 or plane-2 bytes.
+template <bool F32, int MT>
+__global__ void __launch_bounds__(32 * kWarps) correct_idx_kernel(const __grid_constant__ Batch<Prob> bt,
+                                                                  int total_rows, int m0, int mt) {
+  __shared__ float tab[kWarps][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int top = 1 << (31 - __clz(max(bt.count, 1)));
+  for (int r = blockIdx.x * kWarps + warp; r < total_rows; r += gridDim.x * kWarps) {
+    // the problem of row r: the last with row_begin <= r (problems without
+    // an index have no rows: their row_begin equals the next one's)
+    int p = 0;
+    for (int step = top; step >= 1; step >>= 1)
+      if (p + step < bt.count && bt.prob[p + step].row_begin <= r) p += step;
+    const Prob &w = bt.prob[p];
+    const int n = r - w.row_begin, N = w.N, K = w.K;
+    {
+      // codes 27..31 (none in a valid index but the step padding) weigh nothing
+      const int q = lane / 9, d0 = (lane / 3) % 3, d1 = lane % 3;
+      float v = 0.f;
+      if (lane < 27) {
+        const __half *mu = w.mu + (int64_t)n * 4, *a0 = w.a0 + (int64_t)n * 4;
+        v = (__half2float(mu[q]) - __half2float(mu[3])) + (__half2float(a0[q]) - __half2float(a0[3])) * (float)(d0 - 1);
+        if (q < 2) v += __half2float(w.a1[(int64_t)n * 2 + q]) * (float)(d1 - 1);
+      }
+      tab[warp][lane] = v;
+    }
+    __syncwarp();
+    const float *tw = tab[warp];
+    const uint16_t *idx = w.idx;
+    const unsigned short *xm = reinterpret_cast<const unsigned short *>(w.x) + (int64_t)m0 * K;
+    const int nb = (K + kIdxBlock - 1) / kIdxBlock;
+    const int32_t *offr = w.idx_off + (int64_t)n * nb;
+    float acc[MT];
+#pragma unroll
+    for (int t = 0; t < MT; ++t) acc[t] = 0.f;
+    int e = __ldg(offr);
+    for (int b = 0; b < nb; ++b) {
+      const int e1 = __ldg(offr + b + 1);
+      const int kb = b * kIdxBlock, kmax = K - 1 - kb;
+      for (int e0 = e + lane; e0 < e1; e0 += 64) {
+        const uint32_t v0 = __ldg(idx + e0);
+        const uint32_t v1 = e0 + 32 < e1 ? __ldg(idx + e0 + 32) : kIdxNone;
+        const int k0 = kb + min((int)(v0 & (kIdxBlock - 1)), kmax), k1 = kb + min((int)(v1 & (kIdxBlock - 1)), kmax);
+        const float w0 = tw[v0 >> kIdxShift], w1 = tw[v1 >> kIdxShift];
+#pragma unroll
+        for (int t = 0; t < MT; ++t)
+          if (t < mt) {
+            const float x0 = __half2float(__ushort_as_half(__ldg(xm + t * K + k0)));
+            const float x1 = __half2float(__ushort_as_half(__ldg(xm + t * K + k1)));
+            acc[t] = fmaf(w0, x0, fmaf(w1, x1, acc[t]));
+          }
+      }
+      e = e1;
+    }
+#pragma unroll
+    for (int t = 0; t < MT; ++t) {
+      float v = acc[t];
+#pragma unroll
+      for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == t && t < mt) {
+        const int64_t i = (int64_t)(m0 + t) * N + n;
+        v += w.ydense[i];
+        if (F32)
+          static_cast<float *>(w.y)[i] = v;
+        else
+          static_cast<__half *>(w.y)[i] = __float2half_rn(v);
+      }
+    }
+    __syncwarp();  // the table is rewritten for the next row
+  }
+}
+
 // Warps per row: the largest power of two up to 8 that leaves each warp at
 // least three chunks, raised (up to one chunk per warp) while the grid holds
 // fewer than four blocks per SM.
@@ -255,14 +351,26 @@ int warps_per_row(int N, int K, int num_sms) {
   return S;
 }
 
+// indexed: grid blocks striding over `rows` rows; else grid x count.
 template <bool F32, int MT>
-cudaError_t launch_correct(int M, const Batch<Prob> &bt, int max_blocks, cudaStream_t s) {
+cudaError_t launch_correct(int M, const Batch<Prob> &bt, int grid, int rows, bool indexed, cudaStream_t s) {
   for (int m0 = 0; m0 < M; m0 += MT) {
-    correct_kernel<F32, MT><<<dim3(max_blocks, bt.count), 32 * kWarps, 0, s>>>(bt, m0, std::min(MT, M - m0));
+    if (indexed)
+      correct_idx_kernel<F32, MT><<<grid, 32 * kWarps, 0, s>>>(bt, rows, m0, std::min(MT, M - m0));
+    else
+      correct_kernel<F32, MT><<<dim3(grid, bt.count), 32 * kWarps, 0, s>>>(bt, m0, std::min(MT, M - m0));
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+template <bool F32>
+cudaError_t launch_correct_mt(int M, const Batch<Prob> &bt, int grid, int rows, bool indexed, cudaStream_t s) {
+  if (M == 1) return launch_correct<F32, 1>(M, bt, grid, rows, indexed, s);
+  if (M == 2) return launch_correct<F32, 2>(M, bt, grid, rows, indexed, s);
+  if (M <= 4) return launch_correct<F32, 4>(M, bt, grid, rows, indexed, s);
+  return launch_correct<F32, 8>(M, bt, grid, rows, indexed, s);
 }
 
 }  // namespace ew
@@ -290,39 +398,51 @@ cudaError_t launch_ew_views(const EwCall *calls, int count, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-// Masks 0..2 of every problem added to its plane-1 result, y written (one
-// launch per pass of up to 8 tokens).
+// Masks 0..2 of every problem added to its plane-1 result, y written: the
+// problems with a correction index through correct_idx_kernel, the others
+// through correct_kernel (one launch of each kind present per pass of up
+// to 8 tokens).
 cudaError_t launch_ew_correct(int M, const EwCall *calls, int count, bool f32, cudaStream_t s) {
   thread_local ew::Batch<ew::Prob> bt;
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   bt.count = count;
-  int most = 1;
-  for (int i = 0; i < count; ++i) {
-    const EwCall &c = calls[i];
-    ew::Prob &P = bt.prob[i];
-    P.mask = c.w->mask;
-    P.plane1 = c.w->plane1;
-    P.p2rowptr = c.w->p2rowptr;
-    P.plane2 = c.w->plane2;
-    P.mu = reinterpret_cast<const __half *>(c.w->mu);
-    P.a0 = reinterpret_cast<const __half *>(c.w->alpha0);
-    P.a1 = reinterpret_cast<const __half *>(c.w->alpha1);
-    P.x = reinterpret_cast<const __half *>(c.x);
-    P.ydense = c.ydense;
-    P.y = c.y;
-    P.N = c.w->N;
-    P.K = c.w->K;
-    P.S = ew::warps_per_row(P.N, P.K, sms);
-    const int rows = ew::kWarps / P.S;
-    P.blocks = (P.N + rows - 1) / rows;
-    most = std::max(most, P.blocks);
+  for (int pass = 0; pass < 2; ++pass) {
+    const bool indexed = pass == 1;
+    int most = 0, total = 0;
+    for (int i = 0; i < count; ++i) {
+      const EwCall &c = calls[i];
+      ew::Prob &P = bt.prob[i];
+      P.mask = c.w->mask;
+      P.plane1 = c.w->plane1;
+      P.p2rowptr = c.w->p2rowptr;
+      P.plane2 = c.w->plane2;
+      P.mu = reinterpret_cast<const __half *>(c.w->mu);
+      P.a0 = reinterpret_cast<const __half *>(c.w->alpha0);
+      P.a1 = reinterpret_cast<const __half *>(c.w->alpha1);
+      P.idx_off = c.w->idx_off;
+      P.idx = c.w->idx;
+      P.x = reinterpret_cast<const __half *>(c.x);
+      P.ydense = c.ydense;
+      P.y = c.y;
+      P.N = c.w->N;
+      P.K = c.w->K;
+      const bool mine = (c.w->idx_off && c.w->idx) == indexed;
+      P.S = ew::warps_per_row(P.N, P.K, sms);
+      const int rows = ew::kWarps / P.S;
+      P.blocks = mine && !indexed ? (P.N + rows - 1) / rows : 0;
+      P.row_begin = total;
+      if (mine && indexed) total += P.N;
+      most = std::max(most, P.blocks);
+    }
+    if (indexed ? total == 0 : most == 0) continue;
+    const int grid = indexed ? std::min((total + ew::kWarps - 1) / ew::kWarps, 8 * sms) : most;
+    const cudaError_t e = f32 ? ew::launch_correct_mt<true>(M, bt, grid, total, indexed, s)
+                              : ew::launch_correct_mt<false>(M, bt, grid, total, indexed, s);
+    if (e != cudaSuccess) return e;
   }
-  if (M == 1) return f32 ? ew::launch_correct<true, 1>(M, bt, most, s) : ew::launch_correct<false, 1>(M, bt, most, s);
-  if (M == 2) return f32 ? ew::launch_correct<true, 2>(M, bt, most, s) : ew::launch_correct<false, 2>(M, bt, most, s);
-  if (M <= 4) return f32 ? ew::launch_correct<true, 4>(M, bt, most, s) : ew::launch_correct<false, 4>(M, bt, most, s);
-  return f32 ? ew::launch_correct<true, 8>(M, bt, most, s) : ew::launch_correct<false, 8>(M, bt, most, s);
+  return cudaSuccess;
 }
 
 }  // namespace tq

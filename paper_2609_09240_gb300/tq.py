@@ -52,7 +52,8 @@ class tq_problem(ctypes.Structure):
 class tq_ew_weight(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int32), ("K", ctypes.c_int32), ("mask", ctypes.c_void_p), ("plane1", ctypes.c_void_p),
                 ("p2rowptr", ctypes.c_void_p), ("plane2", ctypes.c_void_p), ("mu", ctypes.c_void_p),
-                ("alpha0", ctypes.c_void_p), ("alpha1", ctypes.c_void_p)]
+                ("alpha0", ctypes.c_void_p), ("alpha1", ctypes.c_void_p), ("idx_off", ctypes.c_void_p),
+                ("idx", ctypes.c_void_p)]
 
 
 class tq_ew_problem(ctypes.Structure):
@@ -119,6 +120,10 @@ def lib():
             L.tq_ew_pack.argtypes = [i32, i32] + [vp] * 8 + [vp]
             L.tq_ew_unpack.restype = ctypes.c_int
             L.tq_ew_unpack.argtypes = [i32, i32] + [vp] * 8 + [vp]
+            L.tq_ew_index_offsets.restype = ctypes.c_int
+            L.tq_ew_index_offsets.argtypes = [i32, i32, vp, vp, vp]
+            L.tq_ew_index_fill.restype = ctypes.c_int
+            L.tq_ew_index_fill.argtypes = [i32, i32, EW, vp, vp, vp, vp]
             L.tq_ew_workspace_bytes.restype = sz
             L.tq_ew_workspace_bytes.argtypes = [i32, i32, i32]
             L.tq_ew_linear.restype = ctypes.c_int
@@ -601,6 +606,8 @@ class EwWeight:
     mu: torch.Tensor        # fp16 [N][4]
     alpha0: torch.Tensor    # fp16 [N][4]
     alpha1: torch.Tensor    # fp16 [N][2]
+    idx_off: torch.Tensor | None = None  # int32 [N nb + 1] (nb = ceil(K / 2048)), correction index (ew_index)
+    idx: torch.Tensor | None = None      # int16 (uint16 bits) entries
 
     def struct(self) -> tq_ew_weight:
         w = tq_ew_weight()
@@ -608,7 +615,15 @@ class EwWeight:
         w.mask, w.plane1, w.p2rowptr = self.mask.data_ptr(), self.plane1.data_ptr(), self.p2rowptr.data_ptr()
         w.plane2 = self.plane2.data_ptr()
         w.mu, w.alpha0, w.alpha1 = self.mu.data_ptr(), self.alpha0.data_ptr(), self.alpha1.data_ptr()
+        if self.idx_off is not None:
+            w.idx_off, w.idx = self.idx_off.data_ptr(), self.idx.data_ptr()
         return w
+
+    def index_bytes(self) -> int:
+        """Bytes of the correction index (0 without one)."""
+        if self.idx_off is None:
+            return 0
+        return self.idx_off.numel() * 4 + int(self.idx_off[-1].item()) * 2
 
     def packed_bytes(self) -> int:
         t = [self.mask, self.plane1, self.p2rowptr, self.mu, self.alpha0, self.alpha1]
@@ -634,6 +649,27 @@ def pack_ew_weight(T0, T1, mask_ids, mu, a0, a1, stream=None, check=True) -> EwW
         if st:
             raise TQError(-4, f"tq_ew_pack data status {st:#x}")
     return EwWeight(N, K, mplane, plane1, rp, plane2, mu, a0, a1)
+
+
+def ew_index(w: EwWeight, stream=None, check=True) -> EwWeight:
+    """The weight with its correction index built (tq_ew_index_offsets +
+    tq_ew_index_fill; one synchronization, to size the entries)."""
+    import dataclasses
+    dev = w.plane1.device
+    nb = (w.K + 2047) // 2048
+    off = torch.empty(w.N * nb + 1, dtype=torch.int32, device=dev)
+    _check(lib().tq_ew_index_offsets(w.N, w.K, _p(w.mask), _p(off), _stream(stream)), "tq_ew_index_offsets")
+    ne = int(off[-1].item())
+    idx = torch.empty(max(ne, 1), dtype=torch.int16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    s = w.struct()
+    _check(lib().tq_ew_index_fill(w.N, w.K, ctypes.byref(s), _p(off), _p(idx), _p(status), _stream(stream)),
+           "tq_ew_index_fill")
+    if check:
+        st = int(status.item())
+        if st:
+            raise TQError(-4, f"tq_ew_index_fill data status {st:#x}")
+    return dataclasses.replace(w, idx_off=off, idx=idx)
 
 
 def tq_ew_unpack(w: EwWeight, status=None, stream=None):

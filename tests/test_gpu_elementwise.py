@@ -5,7 +5,12 @@ tq_ew_linear satisfies |y - y_ref| <= 2e-3 * sum_k |W x| per element on
 ragged shapes, 1..40 tokens (decode and prefill paths under the mask-3 pass)
 and Qwen3-8B projection shapes (sampled rows); tq_ew_linear_batched meets
 the same bound on mixed batches and on a Qwen3-8B layer's seven
-projections."""
+projections; the correction index equals the oracle's bit for bit, reports
+offsets that do not match the mask plane, and the linear through it meets
+the bound on every path above, alone and mixed with index-less weights in
+one batched call."""
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -178,3 +183,80 @@ def test_batched_rejects_bad_arguments(H):
     b.arr[0].x = b.arr[0].x + 2  # misaligned activations
     with pytest.raises(tq.TQError):
         tq.tq_ew_linear_batched(b)
+
+
+def _indexed(H, w):
+    from paper_2609_09240_gb300 import tq
+    return tq.ew_index(_pack(H, w))
+
+
+@pytest.mark.parametrize("N,K", [(1, 128), (37, 1024), (300, 1152), (129, 4224), (64, 12288)])
+def test_index_bit_exact(H, N, K):
+    w = wl.gen_ew_weights(N, K, config=20, proj=N)
+    off, ent = ew.correction_index(w.T0, w.T1, w.mask)
+    g = _indexed(H, w)
+    torch.cuda.synchronize()
+    assert np.array_equal(_np(g.idx_off, np.int32), off)
+    assert np.array_equal(_np(g.idx, np.uint16)[:off[-1]], ent)
+
+
+def test_index_reports_offsets_that_do_not_match(H):
+    from paper_2609_09240_gb300 import tq
+    N, K = 16, 2048
+    a = _indexed(H, wl.gen_ew_weights(N, K, config=21, proj=0))
+    b = _pack(H, wl.gen_ew_weights(N, K, config=21, proj=1))
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    idx = torch.zeros_like(a.idx)
+    s_ = b.struct()
+    assert tq.lib().tq_ew_index_fill(N, K, ctypes.byref(s_), a.idx_off.data_ptr(), idx.data_ptr(), st.data_ptr(),
+                                     None) == 0
+    torch.cuda.synchronize()
+    assert int(st.item()) & 0x10  # TQ_DATA_BAD_ROWPTR
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 512, 1024), (2, 300, 2560), (5, 129, 4224), (16, 1000, 640), (40, 256, 1152),
+                                   (1, 1, 128)])
+@pytest.mark.parametrize("f32", [False, True])
+def test_linear_parity_indexed(H, M, N, K, f32):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_ew_weights(N, K, config=22, proj=M + N)
+    xb = wl.gen_x(M, K, config=22, proj=M + N)
+    mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+    y_ref, a_ref = ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1)
+    y = tq.tq_ew_linear(H.dev(xb), _indexed(H, w), f32=f32)
+    H.device_status_ok()
+    H.assert_close(y.float().cpu().numpy().astype(np.float64), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M", [1, 3])
+def test_batched_mixed_indexed_and_plain(H, M):
+    """Problems with and without a correction index in one batched call (the
+    two correction kernels share the call)."""
+    from paper_2609_09240_gb300 import tq
+    shapes = [(512, 4096), (300, 1152), (1024, 12288), (37, 256)]
+    items, refs = [], []
+    for i, (N, K) in enumerate(shapes):
+        w = wl.gen_ew_weights(N, K, config=23, proj=i)
+        xb = wl.gen_x(M, K, config=23, proj=i)
+        mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+        rows = np.arange(N) if N <= 512 else np.sort(np.random.default_rng(i).choice(N, 64, replace=False))
+        refs.append((rows, ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1, rows=rows)))
+        g = _indexed(H, w) if i % 2 == 0 else _pack(H, w)
+        items.append((g, H.dev(xb), torch.empty((M, N), dtype=torch.float16, device="cuda")))
+    tq.tq_ew_linear_batched(tq.EwBatch(M, items))
+    H.device_status_ok()
+    for (_, _, y), (rows, (y_ref, a_ref)) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
+
+
+@pytest.mark.parametrize("N,K", [(4096, 4096), (12288, 4096), (4096, 12288)])
+def test_linear_indexed_qwen3_8b_shapes_sampled_rows(H, N, K):
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_ew_weights(N, K, config=24, proj=N // 1024)
+    xb = wl.gen_x(1, K, config=24, proj=N // 1024)
+    mp, p1, rp, p2, st = ew.pack(w.T0, w.T1, w.mask)
+    rows = np.sort(np.random.default_rng(N + 1).choice(N, size=64, replace=False))
+    y_ref, a_ref = ew.linear(xb, K, mp, p1, rp, p2, w.mu, w.a0, w.a1, rows=rows)
+    y = tq.tq_ew_linear(H.dev(xb), _indexed(H, w))
+    H.device_status_ok()
+    H.assert_close(y.float().cpu().numpy()[:, rows].astype(np.float64), y_ref, a_ref)
