@@ -724,6 +724,174 @@ __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
   __syncthreads();
 }
 
+// ------------------------------------------------- second plane, one token
+// The second plane of one token with the group-ordered index, in the first
+// plane's one-group-per-lane layout: an m16 tile takes, for each of the 8
+// groups of one stage, 16 consecutive entries of that group (group 2c + h
+// of the stage in MMA column 2c + h).  Lane (r, c) loads the slots of
+// entries r and r + 8 of the stage's groups 2c (record at slot byte 0) and
+// 2c + 1 (record at byte 2): the even record's words 0..5, one PRMT of its
+// word 6 with the odd record's word 0, then the odd record's words 1..6 are
+// the 13 window words of an 8-group stage row, so the decode and the B
+// operands (the stage's activation slices, copied per unit into the warp's
+// shared-memory slot) are the first plane's.  The accumulator fragment of lane (r, c) then holds the
+// dot products of exactly its own four records, each added as s2 (D - C)
+// to y2 of the record's row (fp32 atomics; the prep kernel zeroes y2).
+// Warps take units (problem, stage, share of the stage's tiles) from a
+// counter in the workspace.
+// Shared memory per warp: its unit's two activation slices; the first
+// kP2rLow warps use the space below the table, the others the space above it.
+constexpr int kP2rWarps = 20;
+constexpr int kP2rTiles = 8;  // target m16 tiles (128 entries) per unit
+constexpr int kP2rSlices = 2 * Cfg<8>::kSlice;
+constexpr int kP2rLow = kArena1 / kP2rSlices;
+constexpr int kP2rDyn = kArena1 + kLutBytes + (kP2rWarps - kP2rLow) * kP2rSlices;
+static_assert(kP2rDyn <= kDynBytes && kP2rLow < kP2rWarps, "p2r shared memory");
+
+struct P2rBase {
+  int32_t count;
+  int32_t base[TQ_MAX_BATCH + 1];  // first unit of problem p (base[count]: all units)
+};
+
+// Units per stage of a problem: the expected tiles of a stage over
+// kP2rTiles, rounded up, 1 .. 64.
+__host__ __device__ inline int p2r_parts(int K, int64_t nnz) {
+  const int64_t per = (int64_t)nstages(K, 8) * 8 * 16 * kP2rTiles;
+  const int64_t q = (nnz + per - 1) / per;
+  return (int)(q < 1 ? 1 : q > 64 ? 64 : q);
+}
+
+__global__ void __launch_bounds__(kP2rWarps * 32, 1)
+    gemv_p2r_kernel(const __grid_constant__ P2rBase pb, const __grid_constant__ BatchParams bp, int32_t *counter) {
+  extern __shared__ __align__(1024) unsigned char dynr[];
+  const int tid = threadIdx.x, lane = tid & 31;
+  if (smem_u32(dynr) != kDynShared) {
+    if (tid == 0) atomicOr(&g_tq_device_status, 2u);
+    return;
+  }
+  mm::lut_fill_replicated(reinterpret_cast<uint32_t *>(dynr + kArena1), tid, kP2rWarps * 32);
+  __syncthreads();
+  // the work below reads the prep kernel's output (launched programmatically
+  // after it); the first-plane kernel may start its set-up meanwhile
+  grid_dep_wait();
+  grid_dep_launch_next();
+  const int g16 = lane >> 2, c = lane & 3, warp = tid >> 5;
+  const uint32_t tag = kLutShared | ((uint32_t)lane << 2);
+  const bool realB = (g16 >> 1) == c;
+  unsigned char *bw = warp < kP2rLow ? dynr + warp * kP2rSlices
+                                     : dynr + kArena1 + kLutBytes + (warp - kP2rLow) * kP2rSlices;
+  const int count = pb.count, total = pb.base[count];
+  const int top = 1 << (31 - __clz(max(count, 1)));
+  for (;;) {
+    int u = 0;
+    if (lane == 0) u = atomicAdd(counter, 1);
+    u = __shfl_sync(0xffffffffu, u, 0);
+    if (u >= total) break;
+    int pi = 0;  // the unit's problem: the last with base <= u
+    for (int step = top; step >= 1; step >>= 1)
+      if (pi + step < count && pb.base[pi + step] <= u) pi += step;
+    const Problem &P = bp.prob[pi];
+    const int G = P.K / kGroup, S = p2r_parts(P.K, P.nnz), local = u - pb.base[pi];
+    const int s = local / S, part = local - s * S;
+    // the stage's groups' entry ranges (16-entry multiples, clamped into the
+    // index): lane q < 8 reads group 8 s + q; the tiles are the longest's
+    const int64_t cap = mm::c_capacity(P.K, P.nnz);
+    int64_t gb = 0;
+    int gn = 0;
+    if (lane < 8 && 8 * s + lane < G) {
+      const int g = 8 * s + lane;
+      gb = min(max((int64_t)__ldg(P.p2idx + g), (int64_t)0), cap) & ~(int64_t)15;
+      const int64_t ge = min(max((int64_t)__ldg(P.p2idx + g + 1), gb), cap) & ~(int64_t)15;
+      gn = (int)((ge - gb) >> 4);
+    }
+    int T = gn;
+#pragma unroll
+    for (int o = 4; o; o >>= 1) T = max(T, __shfl_xor_sync(0xffffffffu, T, o));
+    T = __shfl_sync(0xffffffffu, T, 0);
+    const int t0 = (int)((int64_t)T * part / S), t1 = (int)((int64_t)T * (part + 1) / S);
+    if (t0 >= t1) continue;
+    // this lane's two groups (stage columns 2c, 2c + 1)
+    const int64_t gbE = __shfl_sync(0xffffffffu, gb, 2 * c), gbO = __shfl_sync(0xffffffffu, gb, 2 * c + 1);
+    const int gnE = __shfl_sync(0xffffffffu, gn, 2 * c), gnO = __shfl_sync(0xffffffffu, gn, 2 * c + 1);
+    const unsigned char *slots = reinterpret_cast<const unsigned char *>(P.p2idx) + mm::c_slot_off(P.K);
+    {
+      // the stage's two slices (contiguous in the workspace) into the warp's slot
+      const uint4 *src = reinterpret_cast<const uint4 *>(ws_b(P) + (int64_t)s * 2 * slice_bytes(8));
+      __syncwarp();  // the previous unit's reads are done
+      for (int i = lane; i < 2 * slice_bytes(8) / 16; i += 32) {
+        const int sl = i / (slice_bytes(8) / 16), k = i - sl * (slice_bytes(8) / 16);
+        reinterpret_cast<uint4 *>(bw + sl * Cfg<8>::kSlice)[k] = __ldg(src + i);
+      }
+      __syncwarp();
+    }
+    const unsigned char *bq = bw + (g16 & 1) * Cfg<8>::kSlice + c * 16;
+    const float4 cs = __ldg(reinterpret_cast<const float4 *>(ws_cs(P, 1) + s * kCSStage + c * 16));
+    float *y2 = P.y2();
+    for (int t = t0; t < t1; ++t) {
+      // slots of entries r, r + 8 of tile t: words in slot order (0, 4, 1, 5 | 2, 6, 3, 7)
+      uint4 sl[2][2][2];  // [h: row r / r + 8][odd][half]
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int o = 0; o < 2; ++o) {
+          const int r = 16 * t + g16 + 8 * h;
+          const bool ok = r < 16 * (o ? gnO : gnE);
+          const uint4 *p = reinterpret_cast<const uint4 *>(slots + ((o ? gbO : gbE) + r) * 32);
+          sl[h][o][0] = ok ? __ldcs(p) : make_uint4(0u, 0u, 0u, 0u);
+          sl[h][o][1] = ok ? __ldcs(p + 1) : make_uint4(0u, 0u, 0u, 0u);
+        }
+      // window word i of row h
+      auto win = [&](int h, int i) -> uint32_t {
+        const uint4 &e0 = sl[h][0][0], &e1 = sl[h][0][1], &o0 = sl[h][1][0], &o1 = sl[h][1][1];
+        switch (i) {
+          case 0: return e0.x;
+          case 1: return e0.z;
+          case 2: return e1.x;
+          case 3: return e1.z;
+          case 4: return e0.y;
+          case 5: return e0.w;
+          case 6: return mm::prmt(e1.y, o0.x, 0x7610u);
+          case 7: return o0.z;
+          case 8: return o1.x;
+          case 9: return o1.z;
+          case 10: return o0.y;
+          case 11: return o0.w;
+          default: return o1.y;
+        }
+      };
+      float d[4];
+      d[0] = d[2] = -cs.x;
+      d[1] = d[3] = -cs.y;
+#pragma unroll
+      for (int i = 0; i < words(8); ++i) {
+        uint32_t a[2][10];
+        decode_word(win(0, i), tag, a[0]);
+        decode_word(win(1, i), tag, a[1]);
+#pragma unroll
+        for (int m = 0; m < 5; ++m) {
+          const int j = 5 * i + m;
+          uint32_t b0 = 0u, b1 = 0u;
+          if (realB) {
+            const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
+            b0 = (j & 1) ? q.z : q.x;
+            b1 = (j & 1) ? q.w : q.y;
+          }
+          mm::mma16816(d, a[0][2 * m], a[1][2 * m], a[0][2 * m + 1], a[1][2 * m + 1], b0, b1);
+        }
+      }
+      // d: (row r: even, odd), (row r + 8: even, odd); s2 beside each record
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int r = 16 * t + g16 + 8 * h;
+        const int nE = (int)sl[h][0][1].w, nO = (int)sl[h][1][1].w;
+        const float s2E = mm::half_of<true>(sl[h][0][1].y), s2O = mm::half_of<false>(sl[h][1][0].x);
+        if (r < 16 * gnE && nE >= 0 && nE < P.N) atomicAdd(&y2[nE], s2E * d[2 * h]);
+        if (r < 16 * gnO && nO >= 0 && nO < P.N) atomicAdd(&y2[nO], s2O * d[2 * h + 1]);
+      }
+    }
+  }
+}
+
 }  // namespace g4
 
 TQ_STATUS_ACCESSOR(read_status_gemv_g4)
@@ -801,6 +969,34 @@ cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, bp, sc);
+}
+
+// The second plane of one token through gemv_p2r_kernel (every problem
+// with a second plane has its index): units numbered problem by problem,
+// launched programmatically after the prep kernel, which zeroes y2 and the
+// unit counter.
+cudaError_t launch_gemv_p2r(const BatchParams &bp, int num_sms, int32_t *counter, cudaStream_t s) {
+  thread_local g4::P2rBase pb;
+  if (bp.M != 1) return cudaErrorInvalidValue;
+  pb.count = bp.count;
+  pb.base[0] = 0;
+  for (int p = 0; p < bp.count; ++p) {
+    const Problem &P = bp.prob[p];
+    pb.base[p + 1] = pb.base[p] + (P.nnz > 0 ? g4::nstages(P.K, 8) * g4::p2r_parts(P.K, P.nnz) : 0);
+  }
+  cudaError_t e = cudaFuncSetAttribute(g4::gemv_p2r_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, g4::kP2rDyn);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(std::min(num_sms, 256));
+  cfg.blockDim = dim3(g4::kP2rWarps * 32);
+  cfg.dynamicSmemBytes = g4::kP2rDyn;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, g4::gemv_p2r_kernel, pb, bp, counter);
 }
 
 // The dependency-ordered sequence kernel (one token), launched

@@ -1326,6 +1326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // -------------------------------------------------------------- launcher
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s);
+cudaError_t launch_gemv_p2r(const BatchParams &bp, int num_sms, int32_t *counter, cudaStream_t s);
 int g4_split_for(const BatchParams &bp, int num_sms);
 cudaError_t launch_gemv_seq(const BatchParams &bp, int num_sms, int barrier_extra, cudaStream_t s);
 
@@ -1572,7 +1573,11 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   // more than 8 tokens in one pass needs every second plane indexed (the
   // other plane-2 kernels take 8 tokens at most)
   if (bp.M > 8 && any2 && !all_idx) return cudaErrorInvalidValue;
-  if (any2 && all_idx) {
+  if (any2 && all_idx && g4path && bp.M == 1) {
+    // one token: the second plane in the first plane's layout (tq_gemv_g4.cu)
+    e = launch_gemv_p2r(bp, num_sms_mm(), counter, s);
+    if (e != cudaSuccess) return e;
+  } else if (any2 && all_idx) {
     auto kern = bp.M == 1 ? mm::gemv_mma_p2c_kernel<true, false>
                           : (bp.M > 8 ? mm::gemv_mma_p2c_kernel<false, true> : mm::gemv_mma_p2c_kernel<false, false>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mm::kCDynBytes2);
