@@ -63,10 +63,12 @@ using mm::kDynShared;
 using mm::kLutBytes;
 using mm::kLutShared;
 
-// decode warps and m16 tiles per decode warp (x 16 = 256 rows): one token
-// shares each activation load between two tiles; two tokens run more warps
-// (measured 0.558 vs 0.560 ms and 0.649 vs 0.671 ms per Qwen3-8B step)
-constexpr int kWD1 = 8, kTL1 = 2;
+// decode warps and m16 tiles per decode warp (x 16 = 256 rows): sixteen
+// warps of one tile each, with the activation loads of the lanes that hold
+// zero columns left out (measured 0.542 ms per Qwen3-8B step against 0.557
+// for eight warps of two tiles sharing each load, and 0.554 for sixteen
+// warps loading on every lane)
+constexpr int kWD1 = 16, kTL1 = 1;
 constexpr int kWD2 = 16, kTL2 = 1;
 constexpr int kA2 = kArena1 + kLutBytes;  // dynamic-smem offset of arena 2 (above the table)
 
@@ -235,7 +237,11 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
 #pragma unroll
     for (int m = 0; m < 5; ++m) {
       const int j = 5 * i + m;
-      const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
+      // one token: lanes of zero columns keep zero registers (no shared-
+      // memory traffic; measured slower for two tokens, whose lanes load
+      // the zero block)
+      uint4 q = make_uint4(0u, 0u, 0u, 0u);
+      if (MB == 2 || realB) q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
       const uint32_t b0 = (j & 1) ? q.z : q.x, b1 = (j & 1) ? q.w : q.y;
 #pragma unroll
       for (int t = 0; t < TL; ++t)
