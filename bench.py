@@ -221,7 +221,7 @@ def build_step(M, device, seed0=0, layers=None, on_codes=None):
 
 
 # the sources the decode-step kernels are compiled from
-DECODE_SOURCES = ("tq_common.cuh", "tq_decode_ops.cuh", "tq_gemv_g4.cu", "tq_gemv_mma.cu", "tq_sm100.cuh")
+DECODE_SOURCES = ("tq_common.cuh", "tq_decode_ops.cuh", "tq_gemv_g4.cu", "tq_gemv_mma.cu", "tq_p2_tile.cuh", "tq_sm100.cuh")
 
 
 def kernel_hash():
