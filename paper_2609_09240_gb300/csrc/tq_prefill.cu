@@ -7,10 +7,11 @@
 //   W[n][k] = s1[n,g] t1[n,k] + off[n,g] + sal[n,g] s2[j(n,g)] t2[n,k],  g = k / 128,
 // each W element rounded once to fp16 (x is fp16), fp32 accumulation.
 //
-// prefill2_kernel: a 256-row x 256-token output tile per CTA (or 128 rows
-// for narrow grids), weights as the MMA's M operand; x tiles and per-group
-// plane-1 windows arrive by tensor copies, 16 warps decode the weight tiles
-// into shared memory, one thread issues the MMAs (see its comment).
+// prefill2_kernel: a 128-row x 512-token output tile per CTA (or 256
+// tokens for narrow grids), weights as the MMA's M operand; x tiles and
+// per-group plane-1 windows arrive by tensor copies, 16 warps decode the
+// weight tiles into shared memory, one thread issues the MMAs (see its
+// comment).
 // Weight decode: a byte's five digits d (trit + 1) select among the row's
 // three fp16 values off - s1, off, off + s1 held in two registers; a
 // 243-entry table gives, per digit, the PRMT selector nibbles of its value,
@@ -75,13 +76,13 @@ __device__ __forceinline__ void realign(const uint32_t *r8, bool odd, uint32_t *
   for (int i = 0; i < 7; ++i) rw[i] = odd ? __funnelshift_r(r8[i], i < 6 ? r8[i + 1] : 0u, 16) : r8[i];
 }
 
-// 35 fp16x2 words from byte pairs P0 .. P0 + 6 of a 26-byte run (word i =
-// trits 10 P0 + 2i, + 1), as decode_weights does for all 13 pairs.
-template <int P0>
-__device__ __forceinline__ void decode_pairs7(const uint32_t *rw, uint32_t v01, uint32_t v22, const uint64_t *sel,
-                                              uint32_t *out) {
+// 5 NP fp16x2 words from byte pairs P0 .. P0 + NP - 1 of a 26-byte run
+// (word i = trits 10 P0 + 2i, + 1).
+template <int P0, int NP>
+__device__ __forceinline__ void decode_pairs(const uint32_t *rw, uint32_t v01, uint32_t v22, const uint64_t *sel,
+                                             uint32_t *out) {
 #pragma unroll
-  for (int q = 0; q < 7; ++q) {
+  for (int q = 0; q < NP; ++q) {
     const int p = P0 + q;
     const int ba = 2 * p, bb = 2 * p + 1;
     const uint32_t va = (rw[ba >> 2] >> (8 * (ba & 3))) & 0xffu;
@@ -97,23 +98,23 @@ __device__ __forceinline__ void decode_pairs7(const uint32_t *rw, uint32_t v01, 
   }
 }
 
-// Half H of a group's 128 weights of one row (32 words, K = 64 H .. 64 H +
-// 63): s1 t1 + off, plus s2 t2 when any row of the warp is salient.  Half 0
-// decodes pairs 0..6 (trits 0..69, keeps words 0..31), half 1 pairs 6..12
-// (trits 60..129, keeps words 2..33).
-template <int H>
-__device__ __forceinline__ void decode_row_half(const RowGroup &cur, const uint64_t *sel, uint32_t *wv) {
-  constexpr int P0 = H ? 6 : 0, W0 = H ? 2 : 0;
+// Quarter Q of a group's 128 weights of one row (16 words, K = 32 Q .. 32 Q
+// + 31): s1 t1 + off, plus s2 t2 when any row of the warp is salient.
+// Quarter Q decodes byte pairs 3 Q .. 3 Q + 3 (trits 30 Q .. 30 Q + 39) and
+// keeps words Q .. Q + 15.
+template <int Q>
+__device__ __forceinline__ void decode_row_quarter(const RowGroup &cur, const uint64_t *sel, uint32_t *wv) {
+  constexpr int P0 = 3 * Q, W0 = Q;
   const float s1 = __half2float(__ushort_as_half(cur.s1)), of = __half2float(__ushort_as_half(cur.of));
   uint32_t rw[7];
   realign(cur.r8, cur.odd, rw);
   const __half h0 = __float2half_rn(of - s1), h1 = __float2half_rn(of), h2 = __float2half_rn(of + s1);
   const uint32_t v01 = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
   const uint32_t v22 = (uint32_t)__half_as_ushort(h2) * 0x00010001u;
-  uint32_t w1[35];
-  decode_pairs7<P0>(rw, v01, v22, sel, w1);
+  uint32_t w1[20];
+  decode_pairs<P0, 4>(rw, v01, v22, sel, w1);
 #pragma unroll
-  for (int i = 0; i < 32; ++i) wv[i] = w1[W0 + i];
+  for (int i = 0; i < 16; ++i) wv[i] = w1[W0 + i];
   if (__any_sync(0xffffffffu, cur.salient)) {
     const float s2 = __half2float(__ushort_as_half(cur.s2));
     uint32_t rec[7];
@@ -121,10 +122,10 @@ __device__ __forceinline__ void decode_row_half(const RowGroup &cur, const uint6
     const __half q0 = __float2half_rn(-s2), q2 = __float2half_rn(s2);
     const uint32_t u01 = (uint32_t)__half_as_ushort(q0);  // (-s2, 0)
     const uint32_t u22 = (uint32_t)__half_as_ushort(q2) * 0x00010001u;
-    uint32_t w2[35];
-    decode_pairs7<P0>(rec, u01, u22, sel, w2);
+    uint32_t w2[20];
+    decode_pairs<P0, 4>(rec, u01, u22, sel, w2);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       const __half2 x = *reinterpret_cast<const __half2 *>(&wv[i]);
       const __half2 y = *reinterpret_cast<const __half2 *>(&w2[W0 + i]);
       const __half2 z = __hadd2(x, y);
@@ -138,41 +139,45 @@ __device__ __forceinline__ void decode_row_half(const RowGroup &cur, const uint6
 __device__ __forceinline__ int cm_off(int row, int e) { return ((row >> 3) * 16 + (e >> 3)) * 128 + (row & 7) * 16; }
 
 // ------------------------------------------------------------------------
-// prefill2_kernel: a 256-row x 256-token output tile per CTA, weights as the
-// MMA's M operand (two halves of 128 rows), tokens as N = 256.
-//  * warps 0..15 (thread r + 256 h = half h of weight row n0 + r): decode
-//    each group's 64 weights of their half row into a 2-slot ring of weight
-//    tiles (64 KiB, the no-swizzle K-major core-matrix layout, 16 core
-//    matrices along K), from the group's plane-1 window (a tensor copy of
-//    48 bytes per row by warp 16's lane 1, 2-slot ring);
-//  * warp 16 (lane 0): the x tiles, 256 tokens x 64 K (32 KiB) per stage,
-//    one 2-D tensor copy each with 128-byte swizzling (the K-major layout
-//    the MMA reads through a swizzled descriptor), into a 3-slot ring, two
-//    stages per group;
-//  * warp 17 (one thread): per stage 8 MMAs (M = 128 rows, N = 256 tokens,
-//    K = 16; rows 0..127 into tensor-memory columns 0..255, rows 128..255
-//    into 256..511);
+// prefill2_kernel: a 128-row x (256 TT)-token output tile per CTA, weights
+// as the MMA's M operand (M = 128), tokens as N = 256 per token half.
+//  * warps 0..15 (thread r + 128 q = quarter q of weight row n0 + r): decode
+//    each group's 32 weights of their quarter row into a 2-slot ring of
+//    weight tiles (32 KiB, the no-swizzle K-major core-matrix layout, 16
+//    core matrices along K), from the group's plane-1 window (a tensor copy
+//    of 48 bytes per row by warp 16's lane 1, 2-slot ring);
+//  * warp 16 (lane 0): the x tiles, 256 TT tokens x 64 K per stage (TT
+//    2-D tensor copies of 256 tokens with 128-byte swizzling, the K-major
+//    layout the MMA reads through a swizzled descriptor), into a 2-slot
+//    ring, two stages per group;
+//  * warp 17 (one thread): per stage 4 TT MMAs (M = 128 rows, N = 256
+//    tokens, K = 16; token half t into tensor-memory columns 256 t ..);
 //  * at the end warps 0..15 read the accumulators and write y.
-// A decoded weight tile serves 256 tokens and 16 MMAs.  Needs a tensor map
-// of x that the host encodes (x 16-byte aligned, K a multiple of 128).
-constexpr int BR2 = 256;                 // weight rows per CTA
-constexpr int BT2 = 256;                 // tokens per CTA (MMA N)
+// A decoded weight tile serves 256 TT tokens and 8 TT MMAs: with TT = 2
+// every weight is decoded once per 512 tokens.  Needs a tensor map of x
+// that the host encodes (x 16-byte aligned, K a multiple of 128).
+constexpr int BR2 = 128;                 // weight rows per CTA
+constexpr int BT2 = 256;                 // tokens per MMA (N) and per token half
 constexpr int XK2 = 64;                  // K per x stage
-constexpr int kXStage2 = BT2 * XK2 * 2;  // 32 KiB
-constexpr int kWTile2 = BR2 * BK * 2;    // 64 KiB
+constexpr int kXHalf2 = BT2 * XK2 * 2;   // 32 KiB: one token half of an x stage
+constexpr int kWTile2 = BR2 * BK * 2;    // 32 KiB
 constexpr int kPRow2 = 48;                 // plane-1 window per row: the 16-byte units covering a group
-constexpr int kPSlot2 = BR2 * kPRow2;      // 12 KiB
+constexpr int kPSlot2 = BR2 * kPRow2;      // 6 KiB
 constexpr int NW2 = 2, NX2 = 2, NP2 = 2;
-constexpr int oW2 = 0;
-constexpr int oX2 = NW2 * kWTile2;
-constexpr int oP2 = oX2 + NX2 * kXStage2;
-constexpr int oSel2 = oP2 + NP2 * kPSlot2;
-constexpr int oBar2 = oSel2 + 256 * 8;
-constexpr int kSmem2 = oBar2 + 256;
-static_assert(kSmem2 <= 232448, "prefill2 shared memory");
 constexpr int kDecWarps2 = 16, kWarpProd2 = 16, kWarpMma2 = 17;
 constexpr int kThreads2 = 18 * 32;
 constexpr uint32_t kTmemCols2 = 512;
+template <int TT>
+struct Lay2 {
+  static constexpr int kXStage = TT * kXHalf2;
+  static constexpr int oW = 0;
+  static constexpr int oX = NW2 * kWTile2;
+  static constexpr int oP = oX + NX2 * kXStage;
+  static constexpr int oSel = oP + NP2 * kPSlot2;
+  static constexpr int oBar = oSel + 256 * 8;
+  static constexpr int kSmem = oBar + 256;
+  static_assert(kSmem <= 232448, "prefill2 shared memory");
+};
 
 struct Bars2 {
   uint64_t xfull[NX2], xempty[NX2], wfull[NW2], wempty[NW2], pfull[NP2], pempty[NP2], done;
@@ -181,16 +186,17 @@ struct Bars2 {
 };
 static_assert(sizeof(Bars2) <= 256, "prefill2 barriers");
 
-template <bool F32, int NH>
+template <bool F32, int TT>
 __global__ void __launch_bounds__(kThreads2, 1)
     prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap,
                     const __grid_constant__ CUtensorMap pmap, int M) {
+  using L = Lay2<TT>;
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * BT2, n0 = blockIdx.y * (NH * 128);
+  const int m0 = blockIdx.x * (TT * BT2), n0 = blockIdx.y * BR2;
   const int N = P.N, G = P.K / kGroup;
-  uint64_t *sel = reinterpret_cast<uint64_t *>(smem + oSel2);
-  Bars2 *bars = reinterpret_cast<Bars2 *>(smem + oBar2);
+  uint64_t *sel = reinterpret_cast<uint64_t *>(smem + L::oSel);
+  Bars2 *bars = reinterpret_cast<Bars2 *>(smem + L::oBar);
   volatile int32_t *abort_ = &bars->abort_;
   for (int i = tid; i < 256; i += kThreads2) sel[i] = sel_entry(i);
   if (tid == 0) {
@@ -199,12 +205,12 @@ __global__ void __launch_bounds__(kThreads2, 1)
       mbar_init(&bars->xempty[i], 1);
     }
     for (int i = 0; i < NW2; ++i) {
-      mbar_init(&bars->wfull[i], NH * 256);
+      mbar_init(&bars->wfull[i], kDecWarps2 * 32);
       mbar_init(&bars->wempty[i], 1);
     }
     for (int i = 0; i < NP2; ++i) {
-      mbar_init(&bars->pfull[i], 1);          // the producer's expect-tx arrival
-      mbar_init(&bars->pempty[i], NH * 8);    // one arrival per decoder warp
+      mbar_init(&bars->pfull[i], 1);           // the producer's expect-tx arrival
+      mbar_init(&bars->pempty[i], kDecWarps2);  // one arrival per decoder warp
     }
     mbar_init(&bars->done, 1);
     bars->abort_ = 0;
@@ -216,14 +222,14 @@ __global__ void __launch_bounds__(kThreads2, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_slot;
 
-  if (warp < kDecWarps2 && (warp & 7) < NH * 4) {
+  if (warp < kDecWarps2) {
     // ======================================================= weight decode
-    // Thread r = row n0 + r.  The group's packed bytes come from the plane-1
-    // window ring (one tensor copy per group: 48 bytes of each row, from the
-    // 16-byte unit that holds the group's first byte); s1 / off (8 groups
-    // per load where rows allow), salience and the plane-2 record are
-    // loaded by the thread one group ahead.
-    const int r = tid & 255, hh = tid >> 8;  // half hh of row r (warp-uniform)
+    // Thread r + 128 q = quarter q of row n0 + r.  The group's packed bytes
+    // come from the plane-1 window ring (one tensor copy per group: 48 bytes
+    // of each row, from the 16-byte unit that holds the group's first byte);
+    // s1 / off (8 groups per load where rows allow), salience and the
+    // plane-2 record are loaded by the thread one group ahead.
+    const int r = tid & (BR2 - 1), qq = tid >> 7;  // quarter qq of row r (warp-uniform)
     const int n = n0 + r;
     const bool valid = n < N;
     const int W = sal_words_of(P.K);
@@ -278,7 +284,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
       RowGroup cur = nx;
       {
         // the row's 7 words of group g: the window's words from (26 g mod 16) / 4 on
-        const uint4 *pw = reinterpret_cast<const uint4 *>(smem + oP2 + ps * kPSlot2 + r * kPRow2);
+        const uint4 *pw = reinterpret_cast<const uint4 *>(smem + L::oP + ps * kPSlot2 + r * kPRow2);
         const uint4 a0 = pw[0], a1 = pw[1], a2 = pw[2];
         const uint32_t w[12] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w, a2.x, a2.y, a2.z, a2.w};
         const int q = ((kGroupBytes * g) & 15) >> 2;
@@ -290,15 +296,19 @@ __global__ void __launch_bounds__(kThreads2, 1)
         cur.odd = g & 1;  // the group starts 2 bytes into its first word
       }
       if (g + 1 < G) fetch(g + 1, nx);
-      uint32_t wv[32];
-      if (hh == 0)
-        decode_row_half<0>(cur, sel, wv);
+      uint32_t wv[16];
+      if (qq == 0)
+        decode_row_quarter<0>(cur, sel, wv);
+      else if (qq == 1)
+        decode_row_quarter<1>(cur, sel, wv);
+      else if (qq == 2)
+        decode_row_quarter<2>(cur, sel, wv);
       else
-        decode_row_half<1>(cur, sel, wv);
-      unsigned char *Wt = smem + oW2 + s * kWTile2;
+        decode_row_quarter<3>(cur, sel, wv);
+      unsigned char *Wt = smem + L::oW + s * kWTile2;
 #pragma unroll
-      for (int kc = 0; kc < 8; ++kc)
-        *reinterpret_cast<uint4 *>(Wt + cm_off(r, (8 * hh + kc) * 8)) =
+      for (int kc = 0; kc < 4; ++kc)
+        *reinterpret_cast<uint4 *>(Wt + cm_off(r, (4 * qq + kc) * 8)) =
             make_uint4(wv[4 * kc], wv[4 * kc + 1], wv[4 * kc + 2], wv[4 * kc + 3]);
       fence_proxy_async_smem();  // the MMA reads these stores through the async proxy
       mbar_arrive(&bars->wfull[s]);
@@ -315,11 +325,11 @@ __global__ void __launch_bounds__(kThreads2, 1)
       for (int g = 0; g < G; ++g) {
         const int sl = g % NP2;
         if (g >= NP2 && !wait_or_abort(&bars->pempty[sl], ((uint32_t)(g / NP2) & 1u) ^ 1u, abort_)) break;
-        mbar_arrive_expect_tx(&bars->pfull[sl], (uint32_t)(NH * 128 * kPRow2));
+        mbar_arrive_expect_tx(&bars->pfull[sl], (uint32_t)(BR2 * kPRow2));
         // bytes from the 16-byte unit holding the group's first byte; rows n0 ..
         asm volatile(
             "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-                smem_u32(smem + oP2 + sl * kPSlot2)),
+                smem_u32(smem + L::oP + sl * kPSlot2)),
             "l"(&pmap), "r"((kGroupBytes * g) & ~15), "r"(n0), "r"(smem_u32(&bars->pfull[sl]))
             : "memory");
         ++issued;
@@ -332,13 +342,15 @@ __global__ void __launch_bounds__(kThreads2, 1)
       for (int xs = 0; xs < 2 * G; ++xs) {
         const int sl = xs % NX2;
         if (xs >= NX2 && !wait_or_abort(&bars->xempty[sl], ((uint32_t)(xs / NX2) & 1u) ^ 1u, abort_)) break;
-        mbar_arrive_expect_tx(&bars->xfull[sl], (uint32_t)kXStage2);
-        // K = 64 xs .., tokens m0 .. (tokens past M arrive as zeros)
-        asm volatile(
-            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-                smem_u32(smem + oX2 + sl * kXStage2)),
-            "l"(&xmap), "r"(xs * XK2), "r"(m0), "r"(smem_u32(&bars->xfull[sl]))
-            : "memory");
+        mbar_arrive_expect_tx(&bars->xfull[sl], (uint32_t)L::kXStage);
+        // K = 64 xs .., tokens m0 + 256 t .. (tokens past M arrive as zeros)
+#pragma unroll
+        for (int t = 0; t < TT; ++t)
+          asm volatile(
+              "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+                  smem_u32(smem + L::oX + sl * L::kXStage + t * kXHalf2)),
+              "l"(&xmap), "r"(xs * XK2), "r"(m0 + t * BT2), "r"(smem_u32(&bars->xfull[sl]))
+              : "memory");
         ++issued;
       }
       // every issued copy lands before the CTA exits (bounded)
@@ -356,7 +368,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
         break;
       }
       tc_fence_after();
-      const uint32_t Wb = smem_u32(smem + oW2 + s * kWTile2);
+      const uint32_t Wb = smem_u32(smem + L::oW + s * kWTile2);
       for (int h = 0; h < 2; ++h) {
         const int xs = 2 * g + h, sl = xs % NX2;
         if (!wait_or_abort(&bars->xfull[sl], (uint32_t)(xs / NX2) & 1u, abort_)) {
@@ -364,15 +376,14 @@ __global__ void __launch_bounds__(kThreads2, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t Xb = smem_u32(smem + oX2 + sl * kXStage2);
+        const uint32_t Xb = smem_u32(smem + L::oX + sl * L::kXStage);
 #pragma unroll
         for (int kk = 0; kk < XK2 / 16; ++kk) {
-          const uint64_t bdesc = smem_desc_sw128(Xb + kk * 32);
+          const uint64_t adesc = smem_desc(Wb + (4 * h + kk) * 256, 128, 2048);
           const uint32_t acc = (g > 0 || h > 0 || kk > 0) ? 1u : 0u;
 #pragma unroll
-          for (int half = 0; half < NH; ++half)
-            mma_smemA(tmem + (uint32_t)(half * BT2), smem_desc(Wb + half * (kWTile2 / 2) + (4 * h + kk) * 256, 128, 2048),
-                      bdesc, idesc, acc);
+          for (int t = 0; t < TT; ++t)
+            mma_smemA(tmem + (uint32_t)(t * BT2), adesc, smem_desc_sw128(Xb + t * kXHalf2 + kk * 32), idesc, acc);
         }
         mma_commit(&bars->xempty[sl]);
       }
@@ -387,18 +398,15 @@ __global__ void __launch_bounds__(kThreads2, 1)
     const bool ok = __all_sync(0xffffffffu, wait_or_abort(&bars->done, 0u, abort_));
     tc_fence_after();
     if (ok) {
-      // tensor-memory lanes 32 q..; two row halves (all tokens each), or for
-      // 128-row tiles two token halves of the one accumulator
-      // 16 warps: lane quarter q, then row half (two accumulators) and token quarter or half
-      const int q = warp & 3, sel2 = warp >> 2;  // 0..3
-      const int half = NH == 2 ? (sel2 & 1) : 0;
-      const int parts = NH == 2 ? 2 : 4, part = NH == 2 ? (sel2 >> 1) : sel2;
-      const int cb = part * (BT2 / parts), ce = cb + BT2 / parts;
-      const int n = n0 + half * 128 + 32 * q + lane;
+      // 16 warps: tensor-memory lane quarter q (rows 32 q ..), then a
+      // quarter of the 256 TT token columns
+      const int q = warp & 3, part = warp >> 2;  // 0..3
+      const int cb = part * (TT * BT2 / 4), ce = cb + TT * BT2 / 4;
+      const int n = n0 + 32 * q + lane;
 #pragma unroll 1
       for (int c0 = cb; c0 < ce; c0 += 8) {
         uint32_t v[8];
-        tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * BT2 + c0), v);
+        tmem_ld8(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0, v);
         tmem_wait_ld();
         if (n < N) {
 #pragma unroll
@@ -472,16 +480,23 @@ static bool encode_p_map(const void *plane1, int N, int K, int rows, CUtensorMap
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
   cudaError_t e;
   CUtensorMap xmap, pmap;
-  const int mt = (M + pf::BT2 - 1) / pf::BT2;
-  const bool narrow = (int64_t)mt * ((P.N + pf::BR2 - 1) / pf::BR2) * 2 <= 152;
-  if (encode_x_map(P.x, M, P.K, &xmap) && encode_p_map(P.plane1, P.N, P.K, narrow ? 128 : 256, &pmap)) {
-    // 128-row tiles when 256-row tiles would leave more than half of the SMs idle
-    const dim3 grid(mt, narrow ? (P.N + 127) / 128 : (P.N + pf::BR2 - 1) / pf::BR2);
-    auto kern = narrow ? (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>)
-                       : (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>);
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, pf::kSmem2);
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // 512 tokens per CTA (each weight decoded once per 512 tokens), unless
+  // the tokens fit one 256-token tile or twice as many 256-token CTAs still
+  // fit in one wave
+  const int rows = (P.N + pf::BR2 - 1) / pf::BR2;
+  const int mt512 = (M + 2 * pf::BT2 - 1) / (2 * pf::BT2);
+  const bool wide = M > pf::BT2 && (int64_t)mt512 * rows * 2 > sms;
+  if (encode_x_map(P.x, M, P.K, &xmap) && encode_p_map(P.plane1, P.N, P.K, pf::BR2, &pmap)) {
+    const dim3 grid(wide ? mt512 : (M + pf::BT2 - 1) / pf::BT2, rows);
+    auto kern = wide ? (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>)
+                     : (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>);
+    const int smem = wide ? pf::Lay2<2>::kSmem : pf::Lay2<1>::kSmem;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, pf::kThreads2, pf::kSmem2, s>>>(P, xmap, pmap, M);
+    kern<<<grid, pf::kThreads2, smem, s>>>(P, xmap, pmap, M);
     return cudaGetLastError();
   }
   // the driver's tensor-map encoder is unavailable or refused the shapes

@@ -48,8 +48,8 @@ PROJ = {"q": 0, "k": 1, "v": 2, "o": 3, "gate": 4, "up": 5, "down": 6}
 def test_prefill_qwen3_8b_shape_sampled_rows(H, name, N, K, nrows):
     """M = 2048 tokens through one Qwen3-8B projection shape; the oracle
     checks a seeded sample of rows (every token) across all row tiles.  q
-    (as o: 4096 x 4096) and gate (as up: 12288 x 4096) run 256-row tiles
-    over more than one wave of SMs; k runs 128-row tiles."""
+    (as o: 4096 x 4096), gate (as up: 12288 x 4096, more than one wave of
+    SMs) and down run 512-token tiles; k runs 256-token tiles."""
     from paper_2609_09240_gb300 import tq
     M = 2048
     w = wl.gen_weights(N, K, 0.1, config=4, layer=0, proj=PROJ[name])
@@ -62,20 +62,23 @@ def test_prefill_qwen3_8b_shape_sampled_rows(H, name, N, K, nrows):
     H.assert_close(y[:, rows], y_ref, a_ref)
 
 
-@pytest.mark.parametrize("M,N,K,narrow", [(2048, 2560, 640, False), (2048, 1024, 640, True)])
-def test_prefill_tile_heights_sampled_rows(H, M, N, K, narrow):
-    """Both row-tile heights of the tensor-copy kernel at M = 2048: 256-row
-    tiles when they fill the GPU (2560 rows), 128-row tiles when 256-row
-    ones would leave most SMs idle (1024 rows); sampled rows of every tile."""
+@pytest.mark.parametrize("M,N,K,wide", [(2048, 2560, 640, True), (2048, 1024, 640, False), (300, 10240, 256, True),
+                                        (700, 19584, 384, True)])
+def test_prefill_tile_widths_sampled_rows(H, M, N, K, wide):
+    """Both token-tile widths of the tensor-copy kernel: 512 tokens per CTA
+    when 256-token tiles would need more than one wave of SMs (2560 rows at
+    M = 2048; 10240 rows at M = 300, whose second token half holds 44
+    tokens; 19584 rows at M = 700, a ragged second 512-token tile), 256
+    tokens when twice as many CTAs still fit one wave (1024 rows); sampled
+    rows of every 128-row tile."""
     from paper_2609_09240_gb300 import tq
     w = wl.gen_weights(N, K, 0.2, config=4, layer=1, proj=N % 89)
     xb = wl.gen_x(M, K, config=4, layer=1, proj=N % 89)
     pw = H.pack_on_gpu(w)
     y = tq.tq_linear(H.dev(xb), pw).float().cpu().numpy()
     H.device_status_ok()
-    tile = 128 if narrow else 256
     rng = np.random.default_rng(N)
-    rows = np.sort(np.concatenate([t * tile + rng.choice(tile, size=2, replace=False)
-                                   for t in range(N // tile)])).astype(np.int32)
+    rows = np.sort(np.concatenate([t * 128 + rng.choice(min(128, N - t * 128), size=min(2, N - t * 128), replace=False)
+                                   for t in range((N + 127) // 128)])).astype(np.int32)
     y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
     H.assert_close(y[:, rows], y_ref, a_ref)
