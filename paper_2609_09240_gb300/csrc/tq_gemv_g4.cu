@@ -748,7 +748,7 @@ __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
 // Shared memory per warp: its unit's two activation slices; the first
 // kP2rLow warps use the space below the table, the others the space above it.
 constexpr int kP2rWarps = 20;
-constexpr int kP2rTiles = 8;  // target m16 tiles (128 entries) per unit
+constexpr int kP2rTiles = 8;  // most m16 tiles (128 entries) per unit
 constexpr int kP2rSlices = 2 * Cfg<8>::kSlice;
 constexpr int kP2rLow = kArena1 / kP2rSlices;
 constexpr int kP2rDyn = kArena1 + kLutBytes + (kP2rWarps - kP2rLow) * kP2rSlices;
@@ -756,13 +756,14 @@ static_assert(kP2rDyn <= kDynBytes && kP2rLow < kP2rWarps, "p2r shared memory");
 
 struct P2rBase {
   int32_t count;
+  int32_t tiles;                   // target tiles per unit (1 .. kP2rTiles)
   int32_t base[TQ_MAX_BATCH + 1];  // first unit of problem p (base[count]: all units)
 };
 
-// Units per stage of a problem: the expected tiles of a stage over
-// kP2rTiles, rounded up, 1 .. 64.
-__host__ __device__ inline int p2r_parts(int K, int64_t nnz) {
-  const int64_t per = (int64_t)nstages(K, 8) * 8 * 16 * kP2rTiles;
+// Units per stage of a problem: the expected tiles of a stage over the
+// call's target tiles per unit, rounded up, 1 .. 64.
+__host__ __device__ inline int p2r_parts(int K, int64_t nnz, int tiles) {
+  const int64_t per = (int64_t)nstages(K, 8) * 8 * 16 * tiles;
   const int64_t q = (nnz + per - 1) / per;
   return (int)(q < 1 ? 1 : q > 64 ? 64 : q);
 }
@@ -797,7 +798,7 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
     for (int step = top; step >= 1; step >>= 1)
       if (pi + step < count && pb.base[pi + step] <= u) pi += step;
     const Problem &P = bp.prob[pi];
-    const int G = P.K / kGroup, S = p2r_parts(P.K, P.nnz), local = u - pb.base[pi];
+    const int G = P.K / kGroup, S = p2r_parts(P.K, P.nnz, pb.tiles), local = u - pb.base[pi];
     const int s = local / S, part = local - s * S;
     // the stage's groups' entry ranges (16-entry multiples, clamped into the
     // index): lane q < 8 reads group 8 s + q; the tiles are the longest's
@@ -985,15 +986,22 @@ cudaError_t launch_gemv_p2r(const BatchParams &bp, int num_sms, int32_t *counter
   thread_local g4::P2rBase pb;
   if (bp.M != 1) return cudaErrorInvalidValue;
   pb.count = bp.count;
+  // tiles per unit: about one and a half units per warp of the grid, at
+  // most kP2rTiles (measured best for the Qwen3-8B step; small calls get
+  // one tile per unit)
+  const int ctas = std::min(num_sms, 256);
+  int64_t tiles = 0;
+  for (int p = 0; p < bp.count; ++p) tiles += (bp.prob[p].nnz + 127) / 128;
+  pb.tiles = (int)std::max<int64_t>(1, std::min<int64_t>(g4::kP2rTiles, 2 * tiles / (3LL * ctas * g4::kP2rWarps)));
   pb.base[0] = 0;
   for (int p = 0; p < bp.count; ++p) {
     const Problem &P = bp.prob[p];
-    pb.base[p + 1] = pb.base[p] + (P.nnz > 0 ? g4::nstages(P.K, 8) * g4::p2r_parts(P.K, P.nnz) : 0);
+    pb.base[p + 1] = pb.base[p] + (P.nnz > 0 ? g4::nstages(P.K, 8) * g4::p2r_parts(P.K, P.nnz, pb.tiles) : 0);
   }
   cudaError_t e = cudaFuncSetAttribute(g4::gemv_p2r_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, g4::kP2rDyn);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(std::min(num_sms, 256));
+  cfg.gridDim = dim3(ctas);
   cfg.blockDim = dim3(g4::kP2rWarps * 32);
   cfg.dynamicSmemBytes = g4::kP2rDyn;
   cfg.stream = s;
