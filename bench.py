@@ -307,8 +307,9 @@ def cpu_baseline(budget_s):
 # ------------------------------------------------------------------- prefill
 def run_prefill(args, ws, rank, local):
     """One Qwen3-8B layer (its seven projections) at M = 2048 tokens through
-    the prefill tile path, one tq_linear per projection; dense fp16 cuBLAS on
-    the same shapes is timed beside it as context."""
+    the prefill tile path, one tq_linear_batched call per layer (every
+    projection's tiles in one launch); dense fp16 cuBLAS on the same shapes
+    is timed beside it as context."""
     import torch
 
     import workloads as wl
@@ -329,10 +330,10 @@ def run_prefill(args, ws, rank, local):
         flops += 2 * M * p.N * p.K
         packed += pw.packed_bytes()
     stream = torch.cuda.current_stream()
+    batch = tq.Batch(M, [(pw, x, y) for pw, x, y, _ in items])
 
     def step():
-        for pw, x, y, wsb in items:
-            tq.tq_linear(x, pw, y=y, ws=wsb, stream=stream)
+        tq.tq_linear_batched(batch, stream=stream)
 
     steps = max(1, min(args.steps, 100))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -376,9 +377,9 @@ def run_prefill(args, ws, rank, local):
                    "l2": "no flush: 2048-token activations and outputs of a layer exceed L2 per step"},
         "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
                      "peak_kind": kind, "traffic": None,
-                     "kernel": "prefill tile kernel (one launch per projection, 7 per step)"},
+                     "kernel": "prefill tile kernel (one launch per step: every projection's tiles)"},
         "dense_fp16_cublas": {"ms_per_step": ms_dense, "tflops": flops / (ms_dense * 1e-3) / 1e12},
-        "gpu_launches": 7 * steps,
+        "gpu_launches": steps,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -710,8 +711,12 @@ def sub_prefill(dev, steps=20):
                       tq.workspace(tq.tq_workspace_bytes(M, p.N, p.K), dev)))
         flops += 2 * M * p.N * p.K
     stream = torch.cuda.current_stream()
+    batch = tq.Batch(M, [(pw, x, y) for pw, x, y, _ in items])
 
     def step():
+        tq.tq_linear_batched(batch, stream=stream)
+
+    def calls():
         for pw, x, y, wsb in items:
             tq.tq_linear(x, pw, y=y, ws=wsb, stream=stream)
 
@@ -733,16 +738,17 @@ def sub_prefill(dev, steps=20):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / steps
 
-    ms, ms_dense = timed(step), timed(dstep)
+    ms, ms_calls, ms_dense = timed(step), timed(calls), timed(dstep)
     peak, kind = measured_tensor_peak()
     tflops = flops / (ms * 1e-3) / 1e12
-    return {"workload": "qwen3-8b prefill: one layer's 7 projections at M=2048 tokens (config 4)",
-            "ms_per_layer": ms, "flops_per_layer": flops, "tflops": tflops,
+    return {"workload": "qwen3-8b prefill: one layer's 7 projections at M=2048 tokens (config 4), one "
+                        "tq_linear_batched call",
+            "ms_per_layer": ms, "ms_per_layer_seven_calls": ms_calls, "flops_per_layer": flops, "tflops": tflops,
             "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
                          "peak_kind": kind},
             "dense_fp16_cublas": {"ms_per_layer": ms_dense, "tflops": flops / (ms_dense * 1e-3) / 1e12},
             "l2": "no flush: a layer's 2048-token activations and outputs (~234 MB) exceed L2",
-            "gpu_launches_per_layer": 7, "steps": steps}
+            "gpu_launches_per_layer": 1, "steps": steps}
 
 
 def sub_sequence(dev, peak, steps=30):

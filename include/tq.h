@@ -309,10 +309,15 @@ TQ_API tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weig
                                   void *stream);
 
 /* Many independent projections in one launch (one decode step of a model:
- * every targeted projection of every layer).  Each problem has its own
- * weight, input and output; all share M (<= TQ_MAX_SKINNY_M).  `problems`
- * is a HOST array read during the call (validated, then passed to the kernel
- * by value in its launch parameters, at most TQ_MAX_BATCH entries). */
+ * every targeted projection of every layer; or one layer's projections at
+ * a prefill's M).  Each problem has its own weight, input and output; all
+ * share M.  `problems` is a HOST array read during the call (validated,
+ * then passed to the kernel by value in its launch parameters, at most
+ * TQ_MAX_BATCH entries).  M <= TQ_MAX_SKINNY_M runs the decode path, M >
+ * TQ_MAX_SKINNY_M the prefill tile path with every problem's output tiles
+ * in one launch per 16 problems (the longest K first), which fills the
+ * SMs' waves better than one launch per projection; it needs no workspace
+ * (tq_batched_workspace_bytes returns 256). */
 #define TQ_MAX_BATCH 256
 typedef struct {
   tq_weight w;

@@ -41,6 +41,7 @@ cudaError_t read_status_gemv_mma(uint32_t *out, bool clear);
 cudaError_t read_status_gemv_g4(uint32_t *out, bool clear);
 int64_t g4_workspace_bytes(int M, int N, int K);
 cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s);
+cudaError_t launch_prefill_batched(const Problem *probs, int count, int M, bool f32, cudaStream_t s);
 size_t ternarize_ws_bytes(int N, int K);
 cudaError_t launch_dequantize(int N, int K, const tq_weight *w, uint16_t *out, uint32_t *status, cudaStream_t s);
 cudaError_t launch_ternarize(int N, int K, const uint16_t *W, int64_t nnz, int sweeps, uint8_t *plane1,
@@ -318,7 +319,13 @@ size_t tq_workspace_bytes(int32_t M, int32_t N, int32_t K) {
 }
 
 size_t tq_batched_workspace_bytes(int32_t M, int32_t count, const tq_problem *problems) {
-  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH || !problems) return 0;
+  if (M < 1 || count < 1 || count > TQ_MAX_BATCH || !problems) return 0;
+  if (M > TQ_MAX_SKINNY_M) {
+    // the prefill tile path needs no workspace (256 bytes keep the argument uniform)
+    for (int i = 0; i < count; ++i)
+      if (check_shape(problems[i].w.N, problems[i].w.K) != TQ_OK) return 0;
+    return 256;
+  }
   size_t tot = 0;
   for (int i = 0; i < count; ++i) {
     if (check_shape(problems[i].w.N, problems[i].w.K) != TQ_OK) return 0;
@@ -340,9 +347,21 @@ tq_status tq_linear_f32out(int32_t M, int32_t N, int32_t K, const tq_weight *w,
 
 tq_status tq_linear_batched(int32_t M, int32_t count, const tq_problem *problems, void *workspace,
                             size_t workspace_bytes, void *stream) {
-  if (M < 1 || M > TQ_MAX_SKINNY_M || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
+  if (M < 1 || count < 1 || count > TQ_MAX_BATCH) return TQ_ERR_SHAPE;
   if (!problems || !workspace) return TQ_ERR_NULL;
   if ((uintptr_t)workspace & 255u) return TQ_ERR_ALIGN;
+  if (M > TQ_MAX_SKINNY_M) {
+    // prefill: every problem's tiles in one launch (per 16 problems)
+    thread_local Problem probs[TQ_MAX_BATCH];
+    for (int i = 0; i < count; ++i) {
+      const tq_problem &q = problems[i];
+      if (tq_status st = check_weight(&q.w, q.w.N, q.w.K)) return st;
+      if (!q.x || !q.y) return TQ_ERR_NULL;
+      if (!aligned16(q.x) || !aligned2(q.y)) return TQ_ERR_ALIGN;
+      probs[i] = to_problem(&q.w, q.x, q.y);
+    }
+    return from_cuda(launch_prefill_batched(probs, count, M, false, (cudaStream_t)stream));
+  }
   thread_local BatchParams bp;  // per host thread, as in linear_impl
   bp.count = count;
   bp.M = M;

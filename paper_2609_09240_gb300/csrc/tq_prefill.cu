@@ -17,6 +17,8 @@
 // 243-entry table gives, per digit, the PRMT selector nibbles of its value,
 // so two weights cost one PRMT.  Every wait is bounded.
 #include <cuda.h>
+
+#include <algorithm>
 #include <cudaTypedefs.h>
 
 #include "tq_common.cuh"
@@ -179,6 +181,21 @@ struct Lay2 {
   static_assert(kSmem <= 232448, "prefill2 shared memory");
 };
 
+// The problems of one launch (one projection, or a batch of them sharing
+// M): each problem's tensor maps of x and plane 1 and its first tile in the
+// launch's 1-D grid (tiles problem by problem, row tile major, token tile
+// minor; the host puts the problems with the longest K first, so that the
+// block scheduler starts the longest tiles first and back-fills the waves).
+constexpr int kPfMaxBatch = 16;
+struct PfBatch {
+  CUtensorMap xmap[kPfMaxBatch];
+  CUtensorMap pmap[kPfMaxBatch];
+  Problem prob[kPfMaxBatch];
+  int32_t tile_begin[kPfMaxBatch + 1];
+  int32_t count, mtiles;  // problems; token tiles per problem
+};
+static_assert(sizeof(PfBatch) <= 32764, "prefill launch parameters");
+
 struct Bars2 {
   uint64_t xfull[NX2], xempty[NX2], wfull[NW2], wempty[NW2], pfull[NP2], pempty[NP2], done;
   uint32_t tmem_slot;
@@ -188,12 +205,17 @@ static_assert(sizeof(Bars2) <= 256, "prefill2 barriers");
 
 template <bool F32, int TT>
 __global__ void __launch_bounds__(kThreads2, 1)
-    prefill2_kernel(const __grid_constant__ Problem P, const __grid_constant__ CUtensorMap xmap,
-                    const __grid_constant__ CUtensorMap pmap, int M) {
+    prefill2_kernel(const __grid_constant__ PfBatch B, int M) {
   using L = Lay2<TT>;
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * (TT * BT2), n0 = blockIdx.y * BR2;
+  // this CTA's problem and tile
+  int pi = 0;
+  while (pi + 1 < B.count && B.tile_begin[pi + 1] <= (int)blockIdx.x) ++pi;
+  const Problem &P = B.prob[pi];
+  const CUtensorMap *xmap = &B.xmap[pi], *pmap = &B.pmap[pi];
+  const int local = (int)blockIdx.x - B.tile_begin[pi];
+  const int m0 = (local % B.mtiles) * (TT * BT2), n0 = (local / B.mtiles) * BR2;
   const int N = P.N, G = P.K / kGroup;
   uint64_t *sel = reinterpret_cast<uint64_t *>(smem + L::oSel);
   Bars2 *bars = reinterpret_cast<Bars2 *>(smem + L::oBar);
@@ -330,7 +352,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
         asm volatile(
             "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
                 smem_u32(smem + L::oP + sl * kPSlot2)),
-            "l"(&pmap), "r"((kGroupBytes * g) & ~15), "r"(n0), "r"(smem_u32(&bars->pfull[sl]))
+            "l"(pmap), "r"((kGroupBytes * g) & ~15), "r"(n0), "r"(smem_u32(&bars->pfull[sl]))
             : "memory");
         ++issued;
       }
@@ -349,7 +371,7 @@ __global__ void __launch_bounds__(kThreads2, 1)
           asm volatile(
               "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
                   smem_u32(smem + L::oX + sl * L::kXStage + t * kXHalf2)),
-              "l"(&xmap), "r"(xs * XK2), "r"(m0 + t * BT2), "r"(smem_u32(&bars->xfull[sl]))
+              "l"(xmap), "r"(xs * XK2), "r"(m0 + t * BT2), "r"(smem_u32(&bars->xfull[sl]))
               : "memory");
         ++issued;
       }
@@ -477,30 +499,52 @@ static bool encode_p_map(const void *plane1, int N, int K, int rows, CUtensorMap
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
-  cudaError_t e;
-  CUtensorMap xmap, pmap;
+// One launch over `count` (<= kPfMaxBatch) problems sharing M: 512-token
+// tiles (each weight decoded once per 512 tokens) unless the tokens fit one
+// 256-token tile or twice as many 256-token CTAs still fit in one wave.
+static cudaError_t launch_prefill_group(const Problem *probs, int count, int M, bool f32, cudaStream_t s) {
+  thread_local pf::PfBatch B;  // large: kept off the stack
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // 512 tokens per CTA (each weight decoded once per 512 tokens), unless
-  // the tokens fit one 256-token tile or twice as many 256-token CTAs still
-  // fit in one wave
-  const int rows = (P.N + pf::BR2 - 1) / pf::BR2;
+  int64_t rows = 0;
+  for (int i = 0; i < count; ++i) rows += (probs[i].N + pf::BR2 - 1) / pf::BR2;
   const int mt512 = (M + 2 * pf::BT2 - 1) / (2 * pf::BT2);
   const bool wide = M > pf::BT2 && (int64_t)mt512 * rows * 2 > sms;
-  if (encode_x_map(P.x, M, P.K, &xmap) && encode_p_map(P.plane1, P.N, P.K, pf::BR2, &pmap)) {
-    const dim3 grid(wide ? mt512 : (M + pf::BT2 - 1) / pf::BT2, rows);
-    auto kern = wide ? (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>)
-                     : (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>);
-    const int smem = wide ? pf::Lay2<2>::kSmem : pf::Lay2<1>::kSmem;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    kern<<<grid, pf::kThreads2, smem, s>>>(P, xmap, pmap, M);
-    return cudaGetLastError();
+  B.mtiles = wide ? mt512 : (M + pf::BT2 - 1) / pf::BT2;
+  // problems with the longest K first (their tiles take the longest)
+  int order[pf::kPfMaxBatch];
+  for (int i = 0; i < count; ++i) order[i] = i;
+  std::stable_sort(order, order + count, [&](int a, int b) { return probs[a].K > probs[b].K; });
+  B.count = count;
+  B.tile_begin[0] = 0;
+  for (int k = 0; k < count; ++k) {
+    const Problem &P = probs[order[k]];
+    if (!encode_x_map(P.x, M, P.K, &B.xmap[k]) || !encode_p_map(P.plane1, P.N, P.K, pf::BR2, &B.pmap[k]))
+      return cudaErrorNotSupported;  // the driver's tensor-map encoder is unavailable or refused the shapes
+    B.prob[k] = P;
+    B.tile_begin[k + 1] = B.tile_begin[k] + (P.N + pf::BR2 - 1) / pf::BR2 * B.mtiles;
   }
-  // the driver's tensor-map encoder is unavailable or refused the shapes
-  return cudaErrorNotSupported;
+  auto kern = wide ? (f32 ? pf::prefill2_kernel<true, 2> : pf::prefill2_kernel<false, 2>)
+                   : (f32 ? pf::prefill2_kernel<true, 1> : pf::prefill2_kernel<false, 1>);
+  const int smem = wide ? pf::Lay2<2>::kSmem : pf::Lay2<1>::kSmem;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  kern<<<B.tile_begin[count], pf::kThreads2, smem, s>>>(B, M);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill(const Problem &P, int M, bool f32, cudaStream_t s) {
+  return launch_prefill_group(&P, 1, M, f32, s);
+}
+
+// A batch of problems sharing M > 16, kPfMaxBatch per launch.
+cudaError_t launch_prefill_batched(const Problem *probs, int count, int M, bool f32, cudaStream_t s) {
+  for (int i = 0; i < count; i += pf::kPfMaxBatch) {
+    const cudaError_t e = launch_prefill_group(probs + i, std::min(pf::kPfMaxBatch, count - i), M, f32, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace tq

@@ -45,7 +45,8 @@ def test_host_side_argument_errors_without_gpu():
     assert L.tq_pack(4, 128, None, None, None, None, None, None, None, None) == -1
     assert L.tq_unpack(4, 130, None, None, None, None, None, None, None, None) == -2
     assert L.tq_linear(1, 4, 128, None, None, None, None, 0, None) == -1
-    assert L.tq_linear_batched(17, 1, None, None, 0, None) == -2
+    assert L.tq_linear_batched(0, 1, None, None, 0, None) == -2
+    assert L.tq_linear_batched(17, 1, None, None, 0, None) == -1  # M > 16: the prefill path, null problems
     assert L.tq_linear_batched(1, 0, None, None, 0, None) == -2
     # ternarizer: shape, count and null checks come before anything touches the device
     assert L.tq_ternarize(0, 128, None, 0, 4, *[None] * 8, 0, None, None) == -2

@@ -82,3 +82,57 @@ def test_prefill_tile_widths_sampled_rows(H, M, N, K, wide):
                                    for t in range((N + 127) // 128)])).astype(np.int32)
     y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
     H.assert_close(y[:, rows], y_ref, a_ref)
+
+
+@pytest.mark.parametrize("M", [40, 300])
+def test_prefill_batched_mixed_shapes(H, M):
+    """tq_linear_batched at a prefill M: problems of different N and K in one
+    launch (the longest K first), every row against the oracle."""
+    from paper_2609_09240_gb300 import tq
+    shapes = [(300, 1152), (129, 4224), (512, 640), (64, 128), (1000, 256)]
+    items, refs = [], []
+    for i, (N, K) in enumerate(shapes):
+        w = wl.gen_weights(N, K, 0.2, config=4, layer=2, proj=i)
+        xb = wl.gen_x(M, K, config=4, layer=2, proj=i)
+        refs.append(H.oracle_ref(w, xb))
+        items.append((H.pack_on_gpu(w), H.dev(xb), torch.empty((M, N), dtype=torch.float16, device="cuda")))
+    tq.tq_linear_batched(tq.Batch(M, items))
+    H.device_status_ok()
+    for (_, _, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+
+
+def test_prefill_batched_more_than_one_launch(H):
+    """18 problems: two launches of at most 16 problems each."""
+    from paper_2609_09240_gb300 import tq
+    M = 64
+    items, refs = [], []
+    for i in range(18):
+        N, K = 32 + 8 * i, 128 * (1 + i % 3)
+        w = wl.gen_weights(N, K, 0.1, config=4, layer=3, proj=i)
+        xb = wl.gen_x(M, K, config=4, layer=3, proj=i)
+        refs.append(H.oracle_ref(w, xb))
+        items.append((H.pack_on_gpu(w), H.dev(xb), torch.empty((M, N), dtype=torch.float16, device="cuda")))
+    tq.tq_linear_batched(tq.Batch(M, items))
+    H.device_status_ok()
+    for (_, _, y), (y_ref, a_ref) in zip(items, refs):
+        H.assert_close(y.float().cpu().numpy(), y_ref, a_ref)
+
+
+def test_prefill_batched_qwen3_8b_layer_sampled_rows(H):
+    """One Qwen3-8B layer's seven projections at M = 2048 in one batched
+    call; 16 seeded rows of each against the oracle (every token)."""
+    from paper_2609_09240_gb300 import tq
+    M = 2048
+    items, checks = [], []
+    for p in wl.config_projections(4):
+        w = wl.gen_weights(p.N, p.K, 0.1, config=4, layer=0, proj=p.proj)
+        xb = wl.gen_x(M, p.K, config=4, layer=0, proj=p.proj)
+        rows = np.sort(np.random.default_rng(p.proj).choice(p.N, size=16, replace=False)).astype(np.int32)
+        checks.append((w, xb, rows))
+        items.append((H.pack_on_gpu(w), H.dev(xb), torch.empty((M, p.N), dtype=torch.float16, device="cuda")))
+    tq.tq_linear_batched(tq.Batch(M, items))
+    H.device_status_ok()
+    for (_, _, y), (w, xb, rows) in zip(items, checks):
+        y_ref, a_ref = H.oracle_ref(w, xb, rows=rows)
+        H.assert_close(y.float().cpu().numpy()[:, rows], y_ref, a_ref)
