@@ -799,6 +799,76 @@ def sub_sequence(dev, peak, steps=30):
             "gpu_launches_per_step": 2, "device_status": st, "steps": steps}
 
 
+def sub_codec(dev, peak, reps=5):
+    """The codec and conversion kernels over one Qwen3-8B layer's seven
+    projections (HBM-bound): tq_pack (int8 codes -> planes), tq_unpack
+    (planes -> int8 codes), tq_plane2_index (the group-ordered second-plane
+    index) and tq_dequantize (packed -> dense fp16 W-hat).  Algorithmic bytes
+    = what each must read and write once; GB/s against the measured copy
+    bandwidth."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_09240_gb300 import tq
+
+    L = tq.lib()
+    items = []
+    bytes_ = {"pack": 0, "unpack": 0, "plane2_index": 0, "dequantize": 0}
+    for p in wl.config_projections(4):
+        g = wl.gen_weights_torch(p.N, p.K, 0.1, dev, 700 + p.proj)
+        pw = tq.pack_weight(g["T1"], g["T2"], g["sal"], g["s1"], g["off"], g["s2"])
+        N, K, nnz = p.N, p.K, pw.nnz
+        T1o = torch.empty_like(g["T1"])
+        T2o = torch.empty_like(g["T2"])
+        Wd = torch.empty((N, K), dtype=torch.float16, device=dev)
+        idx = torch.empty(int(L.tq_plane2_index_bytes(N, K, nnz)) // 4, dtype=torch.int32, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        items.append((pw, g["T1"], g["T2"], T1o, T2o, Wd, idx, st))
+        side = pw.salience.numel() * 4 + pw.rowptr.numel() * 4
+        planes = pw.plane1.numel() + nnz * 26
+        bytes_["pack"] += N * K + nnz * 128 + side + planes
+        bytes_["unpack"] += planes + side + 2 * N * K
+        bytes_["plane2_index"] += nnz * 26 + nnz * 2 + side + idx.numel() * 4
+        bytes_["dequantize"] += pw.packed_bytes() + 2 * N * K
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+
+    def run(kind):
+        for pw, T1, T2, T1o, T2o, Wd, idx, st in items:
+            if kind == "pack":
+                tq.tq_pack(pw.N, pw.K, T1, T2, pw.salience, pw.rowptr, pw.plane1, pw.plane2, st, stream)
+            elif kind == "unpack":
+                tq.tq_unpack(pw.N, pw.K, pw.plane1, pw.plane2, pw.salience, pw.rowptr, T1o, T2o, st, stream)
+            elif kind == "plane2_index":
+                L.tq_plane2_index(pw.N, pw.K, pw.salience.data_ptr(), pw.rowptr.data_ptr(), pw.nnz,
+                                  pw.plane2.data_ptr(), pw.scale2.data_ptr(), idx.data_ptr(), sp)
+            else:
+                tq.tq_dequantize(pw, out=Wd, d_status=st, stream=stream)
+
+    out = {}
+    for kind in bytes_:
+        for _ in range(2):
+            run(kind)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            run(kind)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        gbs = bytes_[kind] / (ms * 1e-3) / 1e9
+        out[kind] = {"ms_per_layer": ms, "bytes_per_layer": bytes_[kind], "gbs": gbs, "frac_of_hbm_peak": gbs / peak}
+    status = sum(int(it[-1].item()) for it in items)
+    return {"workload": "qwen3-8b one layer's 7 projections (193 M weights, 10 % salient groups)",
+            "kernels": out, "data_status": status,
+            "bytes": "algorithmic: pack reads the int8 T1 codes, T2 of the salient groups, salience and rowptr and "
+                     "writes plane 1 and plane 2; unpack the reverse with full int8 T1 and T2; the index reads "
+                     "plane 2, s2, salience and rowptr and writes the index; dequantize reads the packed weight "
+                     "and writes fp16 W-hat",
+            "l2": "no flush: a layer's int8 codes (386 MB) and fp16 W-hat (386 MB) exceed L2"}
+
+
 def sub_elementwise(dev, peak):
     """The element-wise four-mask form (orders [2, 2, 1, 1], the paper's
     recorded coverages) of one Qwen3-8B layer at M = 1: seven tq_ew_linear
@@ -1060,6 +1130,7 @@ def main():
             cfg["config4"] = sub_prefill(dev)
             cfg["dependency_ordered"] = sub_sequence(dev, peak)
             cfg["elementwise"] = sub_elementwise(dev, peak)
+            cfg["codec"] = sub_codec(dev, peak)
             clk2.mark()
         cfg["clocks"] = clk2.summary()
         out["configs"] = cfg

@@ -121,18 +121,17 @@ __device__ __forceinline__ uint8_t encode_codes(const int8_t *t, int ntr, uint32
   return (uint8_t)v;
 }
 
-// Thread per plane-1 byte (n, b).
+// Thread per plane-1 byte (n, b): blocks stride over rows, threads over a
+// row's bytes.
 __global__ void pack_kernel(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                             const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2,
                             uint32_t *status) {
   const int G = K / kGroup, W = sal_words_of(K);
-  const int64_t RB = row_bytes_of(K);
-  const int64_t total = (int64_t)N * RB;
+  const int RB = (int)row_bytes_of(K);
   const int32_t nnz = rowptr[N];
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    const int n = (int)(idx / RB);
-    const int b = (int)(idx - (int64_t)n * RB);
+  for (int n = blockIdx.x; n < N; n += gridDim.x)
+  for (int b = threadIdx.x; b < RB; b += blockDim.x) {
+    const int64_t idx = (int64_t)n * RB + b;
     uint32_t st = 0;
     if (b >= G * kGroupBytes) {
       plane1[idx] = 0;
@@ -179,17 +178,17 @@ __device__ __forceinline__ void decode_to(uint8_t v, int ntr, int8_t *t, uint32_
   }
 }
 
+// Thread per plane-1 byte (n, b): blocks stride over rows, threads over a
+// row's bytes.
 __global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                               const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                               uint32_t *status) {
   const int G = K / kGroup, W = sal_words_of(K);
-  const int64_t RB = row_bytes_of(K);
-  const int64_t total = (int64_t)N * RB;
+  const int RB = (int)row_bytes_of(K);
   const int32_t nnz = rowptr[N];
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    const int n = (int)(idx / RB);
-    const int b = (int)(idx - (int64_t)n * RB);
+  for (int n = blockIdx.x; n < N; n += gridDim.x)
+  for (int b = threadIdx.x; b < RB; b += blockDim.x) {
+    const int64_t idx = (int64_t)n * RB + b;
     uint32_t st = 0;
     const uint8_t v = plane1[idx];
     if (b >= G * kGroupBytes) {
@@ -232,15 +231,37 @@ __host__ __device__ __forceinline__ int64_t p2index_slot_off(int K) {
   return ((int64_t)(K / kGroup + 1) * 4 + 127) & ~(int64_t)127;
 }
 
+// Rows are taken in chunks of kIdxChunk: block (g, c) handles group g's
+// rows [kIdxChunk c, kIdxChunk (c + 1)).
+constexpr int kIdxChunk = 1024;
+
+// Salient rows of group g in rows [r0, r1) (the block's threads together;
+// every thread gets the total).
+__device__ __forceinline__ int p2index_block_count(const uint32_t *sal, int W, int g, int r0, int r1, int *red) {
+  int c = 0;
+  for (int n = r0 + (int)threadIdx.x; n < r1; n += kIdxThreads) c += sal_bit(sal, W, n, g);
+  for (int o = 16; o; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = c;
+  __syncthreads();
+  int t = 0;
+  for (int w = 0; w < kIdxThreads / 32; ++w) t += red[w];
+  __syncthreads();
+  return t;
+}
+
+// colptr[g + 1] += salient rows of group g in the block's chunk (colptr
+// zeroed by p2index_zero_kernel).
 __global__ void __launch_bounds__(kIdxThreads) p2index_count_kernel(int N, int K, const uint32_t *sal,
                                                                      int32_t *colptr) {
-  const int g = blockIdx.x, W = sal_words_of(K);
-  int total = 0;
-  for (int n0 = 0; n0 < N; n0 += kIdxThreads) {
-    const int n = n0 + threadIdx.x;
-    total += __syncthreads_count(n < N && sal_bit(sal, W, n, g));
-  }
-  if (threadIdx.x == 0) colptr[g + 1] = total;
+  __shared__ int red[kIdxThreads / 32];
+  const int g = blockIdx.x, c = blockIdx.y, W = sal_words_of(K);
+  const int r0 = c * kIdxChunk, r1 = min(N, r0 + kIdxChunk);
+  const int t = p2index_block_count(sal, W, g, r0, r1, red);
+  if (threadIdx.x == 0 && t) atomicAdd(colptr + g + 1, t);
+}
+
+__global__ void p2index_zero_kernel(int G, int32_t *colptr) {
+  for (int i = threadIdx.x; i <= G; i += blockDim.x) colptr[i] = 0;
 }
 
 // colptr[g+1] = colptr[g] + count rounded up to 16, at most the capacity
@@ -288,35 +309,42 @@ __device__ __forceinline__ void p2index_fill_slot(uint8_t *slot, int g, int n, i
   p2index_store_slot(slot, L);
 }
 
-// Blocks 0 .. G-1 fill group g's entries; block G empties the slots from
+// Block (g, c) fills the entries of group g's salient rows of chunk c
+// (their place: colptr[g] plus the salient rows of the group's earlier
+// chunks, counted by the block itself); the group's last chunk empties the
+// slots after its last entry.  Block (G, 0) empties the slots from
 // colptr[G] to the capacity.
 __global__ void __launch_bounds__(kIdxThreads) p2index_fill_kernel(int N, int K, const uint32_t *sal,
                                                                     const int32_t *rowptr, int64_t nnz,
                                                                     const uint8_t *plane2, const uint16_t *scale2,
                                                                     int32_t *index) {
   __shared__ int warp_base[kIdxThreads / 32 + 1];
-  const int G = K / kGroup, g = blockIdx.x, W = sal_words_of(K);
+  __shared__ int red[kIdxThreads / 32];
+  const int G = K / kGroup, g = blockIdx.x, c = blockIdx.y, W = sal_words_of(K);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint8_t *slots = reinterpret_cast<uint8_t *>(index) + p2index_slot_off(K);
   if (g == G) {
+    if (c != 0) return;
     const int64_t cap = p2index_capacity(K, nnz);
     for (int64_t e = index[G] + threadIdx.x; e < cap; e += kIdxThreads) p2index_empty_slot(slots + 32 * e);
     return;
   }
+  const int r0 = c * kIdxChunk, r1 = min(N, r0 + kIdxChunk);
+  if (r0 >= N) return;
   const int64_t lim = index[g + 1];
-  int64_t base = index[g];
-  for (int n0 = 0; n0 < N; n0 += kIdxThreads) {
+  int64_t base = index[g] + p2index_block_count(sal, W, g, 0, r0, red);
+  for (int n0 = r0; n0 < r1; n0 += kIdxThreads) {
     const int n = n0 + threadIdx.x;
-    const bool bit = n < N && sal_bit(sal, W, n, g);
+    const bool bit = n < r1 && sal_bit(sal, W, n, g);
     const uint32_t m = __ballot_sync(0xffffffffu, bit);
     if (lane == 0) warp_base[warp] = __popc(m);
     __syncthreads();
     if (threadIdx.x == 0) {
       int run = 0;
       for (int w = 0; w < kIdxThreads / 32; ++w) {
-        const int c = warp_base[w];
+        const int cnt = warp_base[w];
         warp_base[w] = run;
-        run += c;
+        run += cnt;
       }
       warp_base[kIdxThreads / 32] = run;
     }
@@ -331,7 +359,8 @@ __global__ void __launch_bounds__(kIdxThreads) p2index_fill_kernel(int N, int K,
     base += warp_base[kIdxThreads / 32];
     __syncthreads();
   }
-  for (int64_t e = base + threadIdx.x; e < lim; e += kIdxThreads) p2index_empty_slot(slots + 32 * e);
+  if (r1 == N)
+    for (int64_t e = base + threadIdx.x; e < lim; e += kIdxThreads) p2index_empty_slot(slots + 32 * e);
 }
 
 // ------------------------------------------------------------- launchers
@@ -356,26 +385,25 @@ cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t
 cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                         const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
                         cudaStream_t s) {
-  int64_t total = (int64_t)N * row_bytes_of(K);
-  pack_kernel<<<grid_for(total, 256), 256, 0, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2, status);
+  pack_kernel<<<std::min(N, 152 * 16), 256, 0, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2, status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s) {
-  int64_t total = (int64_t)N * row_bytes_of(K);
-  unpack_kernel<<<grid_for(total, 256), 256, 0, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
+  unpack_kernel<<<std::min(N, 152 * 16), 256, 0, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
                                                      status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_plane2_index(int N, int K, const uint32_t *sal, const int32_t *rowptr, int64_t nnz,
                                 const uint8_t *plane2, const uint16_t *scale2, int32_t *index, cudaStream_t s) {
-  const int G = K / kGroup;
-  p2index_count_kernel<<<G, kIdxThreads, 0, s>>>(N, K, sal, index);
+  const int G = K / kGroup, C = (N + kIdxChunk - 1) / kIdxChunk;
+  p2index_zero_kernel<<<1, 256, 0, s>>>(G, index);
+  p2index_count_kernel<<<dim3(G, C), kIdxThreads, 0, s>>>(N, K, sal, index);
   p2index_scan_kernel<<<1, 32, 0, s>>>(G, p2index_capacity(K, nnz), index);
-  p2index_fill_kernel<<<G + 1, kIdxThreads, 0, s>>>(N, K, sal, rowptr, nnz, plane2, scale2, index);
+  p2index_fill_kernel<<<dim3(G + 1, C), kIdxThreads, 0, s>>>(N, K, sal, rowptr, nnz, plane2, scale2, index);
   return cudaGetLastError();
 }
 

@@ -187,6 +187,8 @@ __global__ void __launch_bounds__(128) dequantize_kernel(int N, int K, const uin
     const uint8_t *g1 = plane1 + n * RB + (int64_t)kGroupBytes * g;
     const uint8_t *g2 = rec >= 0 ? plane2 + rec * kGroupBytes : nullptr;
     uint4 *dst = reinterpret_cast<uint4 *>(out + b * kGroup);
+    // unrolled: every byte index and power of 3 below is a constant
+#pragma unroll
     for (int c = 0; c < kGroup / 8; ++c) {
       uint32_t wd[4];
 #pragma unroll
