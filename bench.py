@@ -395,8 +395,20 @@ def run_prefill(args, ws, rank, local):
 #   a salient block (support and moments 5, residual mean 5, second support
 #   and its moment 6).
 TERN_OPS_STATS, TERN_OPS_PLAIN, TERN_OPS_SALIENT = 15, 5, 16
-# fp32 lanes x SMs x maximum SM clock: the ALU peak for single fp32 operations
-ALU_PEAK_TOPS = 128 * 152 * 2.07e9 / 1e12
+# fp32 lanes per SM on sm_100-class parts; the ALU peak for single fp32
+# operations is lanes x the device's SM count x its maximum SM clock
+FP32_LANES_PER_SM = 128
+
+
+def alu_peak_tops(dev, sm_max_mhz=None):
+    """Single-fp32-operation peak of `dev` in Top/s: lanes x SMs x maximum clock.
+
+    The SM count is the device's own; the clock is the maximum that the clock
+    sampler read during the run, else 2070 MHz (the part's maximum SM clock).
+    """
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    mhz = sm_max_mhz if sm_max_mhz else 2070.0
+    return FP32_LANES_PER_SM * sms * mhz * 1e6 / 1e12, sms, mhz
 
 
 def run_ternarize(args, ws, rank, local):
@@ -482,6 +494,8 @@ def run_ternarize(args, ws, rank, local):
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / steps
     achieved = ops / (ms * 1e-3) / 1e12
+    clocks = clk.summary()
+    peak, sms, mhz = alu_peak_tops(torch.cuda.current_device(), clocks.get("sm_max_mhz"))
     out = {
         "metric": "Qwen3-8B E2M-ATQ ternarization into the packed format: weights/s", "value": n_weights / (ms * 1e-3) / 1e9,
         "unit": "Gweights/s", "n_gpus": 1, "steps": steps, "warmup": max(args.warmup, 3), "ms_per_step": ms,
@@ -489,15 +503,15 @@ def run_ternarize(args, ws, rank, local):
         "config": {"workload": "E2M-ATQ of one Qwen3-8B layer's 7 projections (fp16 in, packed out), "
                                "10% salient groups, 4 sweeps", "weights_per_step": n_weights,
                    "l2": "no flush: a layer's 386 MB of fp16 weights exceed L2 per step"},
-        "roofline": {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TOPS, "unit": "Top/s",
-                     "frac": achieved / ALU_PEAK_TOPS, "traffic": None,
-                     "peak_kind": "fp32 lanes x 152 SMs x 2.07 GHz (derived, not measured)",
+        "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "Top/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "peak_kind": f"{FP32_LANES_PER_SM} fp32 lanes x {sms} SMs x {mhz:.0f} MHz (derived, not measured)",
                      "kernel": "whole tq_ternarize call (nine launches per projection, 63 per step)",
                      "ops_per_step": ops},
         "e2e": {"value": n_weights / (e2e_ms * 1e-3) / 1e9, "unit": "Gweights/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": 9 * 7 * steps,
-        "clocks": clk.summary(),
+        "clocks": clocks,
     }
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = ternarize_cpu_baseline(10.0)
