@@ -234,9 +234,15 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
       dyn + (realB ? kA2 + C::kOffB + (buf * 2 + (g & 1)) * C::kSlice + c * 16 : C::kOffZero + 16 * ((g >> 1) + 2));
   const float4 cs = *reinterpret_cast<const float4 *>(dyn + C::kOffCS + buf * kCSStage + c * 16);
   // accumulators start at -C (slice 0 in columns 2c, slice 1 in 2c + 1)
-  float d[TL][4];
+  // two accumulator chains (even and odd words), so that consecutive MMAs
+  // do not wait for each other's results (0.513 ms per Qwen3-8B step
+  // against 0.517 with one)
+  float d2[TL][2][4];
 #pragma unroll
-  for (int t = 0; t < TL; ++t) d[t][0] = d[t][2] = -cs.x, d[t][1] = d[t][3] = -cs.y;
+  for (int t = 0; t < TL; ++t) {
+    d2[t][0][0] = d2[t][0][2] = -cs.x, d2[t][0][1] = d2[t][0][3] = -cs.y;
+    d2[t][1][0] = d2[t][1][1] = d2[t][1][2] = d2[t][1][3] = 0.f;
+  }
 #pragma unroll
   for (int i = 0; i < C::kWords; ++i) {
     uint32_t a[TL][2][10];
@@ -264,9 +270,14 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
       }
 #pragma unroll
       for (int t = 0; t < TL; ++t)
-        mm::mma16816(d[t], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
+        mm::mma16816(d2[t][i & 1], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
     }
   }
+  float d[TL][4];
+#pragma unroll
+  for (int t = 0; t < TL; ++t)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) d[t][e] = d2[t][0][e] + d2[t][1][e];
   // s1 / off of (row, the lane's groups): the slot holds 8 groups per row
   // (both halves of an 8-group stage; an odd 4-group stage's at 4)
   const unsigned char *so = dyn + kA2 + C::kOffSO + buf * C::kSOSlot;
@@ -810,6 +821,7 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
                                      : dynr + kArena1 + kLutBytes + (warp - kP2rLow) * kP2rSlices;
   const int count = pb.count, total = pb.base[count];
   const int top = 1 << (31 - __clz(max(count, 1)));
+  uint32_t bz[kBSets][4] = {};  // activation registers (zero-column lanes: zero throughout)
   for (;;) {
     int u = 0;
     if (lane == 0) u = atomicAdd(counter, 1);
@@ -898,12 +910,9 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
 #pragma unroll
         for (int m = 0; m < 5; ++m) {
           const int j = 5 * i + m;
-          uint32_t b0 = 0u, b1 = 0u;
-          if (realB) {
-            const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
-            b0 = (j & 1) ? q.z : q.x;
-            b1 = (j & 1) ? q.w : q.y;
-          }
+          uint32_t(&r)[4] = bz[(j >> 1) % kBSets];
+          if ((j & 1) == 0) ld_b_real(r, bq + (j >> 1) * 64, realB);
+          const uint32_t b0 = (j & 1) ? r[2] : r[0], b1 = (j & 1) ? r[3] : r[1];
           mm::mma16816(d, a[0][2 * m], a[1][2 * m], a[0][2 * m + 1], a[1][2 * m + 1], b0, b1);
         }
       }
