@@ -234,14 +234,17 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
       dyn + (realB ? kA2 + C::kOffB + (buf * 2 + (g & 1)) * C::kSlice + c * 16 : C::kOffZero + 16 * ((g >> 1) + 2));
   const float4 cs = *reinterpret_cast<const float4 *>(dyn + C::kOffCS + buf * kCSStage + c * 16);
   // accumulators start at -C (slice 0 in columns 2c, slice 1 in 2c + 1)
-  // two accumulator chains (even and odd words), so that consecutive MMAs
-  // do not wait for each other's results (0.513 ms per Qwen3-8B step
-  // against 0.517 with one)
-  float d2[TL][2][4];
+  // one accumulator chain per MMA position m of a word (five chains), so
+  // that an MMA waits for the result of the one five places earlier only
+  // (0.500 ms per Qwen3-8B step, against 0.513 with two chains by word and
+  // 0.517 with one; ten chains exceed the 96 registers a thread may hold
+  // with 17 warps, five of them on one scheduler)
+  float d2[TL][5][4];
 #pragma unroll
   for (int t = 0; t < TL; ++t) {
     d2[t][0][0] = d2[t][0][2] = -cs.x, d2[t][0][1] = d2[t][0][3] = -cs.y;
-    d2[t][1][0] = d2[t][1][1] = d2[t][1][2] = d2[t][1][3] = 0.f;
+#pragma unroll
+    for (int k = 1; k < 5; ++k) d2[t][k][0] = d2[t][k][1] = d2[t][k][2] = d2[t][k][3] = 0.f;
   }
 #pragma unroll
   for (int i = 0; i < C::kWords; ++i) {
@@ -270,14 +273,18 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
       }
 #pragma unroll
       for (int t = 0; t < TL; ++t)
-        mm::mma16816(d2[t][i & 1], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
+        mm::mma16816(d2[t][m], a[t][0][2 * m], a[t][1][2 * m], a[t][0][2 * m + 1], a[t][1][2 * m + 1], b0, b1);
     }
   }
   float d[TL][4];
 #pragma unroll
   for (int t = 0; t < TL; ++t)
 #pragma unroll
-    for (int e = 0; e < 4; ++e) d[t][e] = d2[t][0][e] + d2[t][1][e];
+    for (int e = 0; e < 4; ++e) {
+      d[t][e] = d2[t][0][e];
+#pragma unroll
+      for (int k = 1; k < 5; ++k) d[t][e] += d2[t][k][e];
+    }
   // s1 / off of (row, the lane's groups): the slot holds 8 groups per row
   // (both halves of an 8-group stage; an odd 4-group stage's at 4)
   const unsigned char *so = dyn + kA2 + C::kOffSO + buf * C::kSOSlot;
