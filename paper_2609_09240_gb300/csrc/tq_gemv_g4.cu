@@ -787,6 +787,12 @@ __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
 // Shared memory per warp: its unit's two activation slices; the first
 // kP2rLow warps use the space below the table, the others the space above it.
 constexpr int kP2rWarps = 20;
+// activation register sets and accumulator chains: two sets free the
+// registers for three chains within the 96 a thread may hold with 20 warps
+// (0.4995 ms per Qwen3-8B step against 0.5005 with four sets and one chain;
+// five chains spill)
+constexpr int kP2rBSets = 2;
+constexpr int kP2rChains = 3;
 constexpr int kP2rTiles = 8;  // most m16 tiles (128 entries) per unit
 constexpr int kP2rSlices = 2 * Cfg<8>::kSlice;
 constexpr int kP2rLow = kArena1 / kP2rSlices;
@@ -828,7 +834,7 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
                                      : dynr + kArena1 + kLutBytes + (warp - kP2rLow) * kP2rSlices;
   const int count = pb.count, total = pb.base[count];
   const int top = 1 << (31 - __clz(max(count, 1)));
-  uint32_t bz[kBSets][4] = {};  // activation registers (zero-column lanes: zero throughout)
+  uint32_t bz[kP2rBSets][4] = {};  // activation registers (zero-column lanes: zero throughout)
   for (;;) {
     int u = 0;
     if (lane == 0) u = atomicAdd(counter, 1);
@@ -906,9 +912,11 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
           default: return o1.y;
         }
       };
-      float d[4];
-      d[0] = d[2] = -cs.x;
-      d[1] = d[3] = -cs.y;
+      float dc[kP2rChains][4];
+      dc[0][0] = dc[0][2] = -cs.x;
+      dc[0][1] = dc[0][3] = -cs.y;
+#pragma unroll
+      for (int k = 1; k < kP2rChains; ++k) dc[k][0] = dc[k][1] = dc[k][2] = dc[k][3] = 0.f;
 #pragma unroll
       for (int i = 0; i < words(8); ++i) {
         uint32_t a[2][10];
@@ -917,11 +925,18 @@ __global__ void __launch_bounds__(kP2rWarps * 32, 1)
 #pragma unroll
         for (int m = 0; m < 5; ++m) {
           const int j = 5 * i + m;
-          uint32_t(&r)[4] = bz[(j >> 1) % kBSets];
+          uint32_t(&r)[4] = bz[(j >> 1) % kP2rBSets];
           if ((j & 1) == 0) ld_b_real(r, bq + (j >> 1) * 64, realB);
           const uint32_t b0 = (j & 1) ? r[2] : r[0], b1 = (j & 1) ? r[3] : r[1];
-          mm::mma16816(d, a[0][2 * m], a[1][2 * m], a[0][2 * m + 1], a[1][2 * m + 1], b0, b1);
+          mm::mma16816(dc[j % kP2rChains], a[0][2 * m], a[1][2 * m], a[0][2 * m + 1], a[1][2 * m + 1], b0, b1);
         }
+      }
+      float d[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        d[e] = dc[0][e];
+#pragma unroll
+        for (int k = 1; k < kP2rChains; ++k) d[e] += dc[k][e];
       }
       // d: (row r: even, odd), (row r + 8: even, odd); s2 beside each record
 #pragma unroll
