@@ -1164,8 +1164,14 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
             float d[4], d2[4] = {0.f, 0.f, 0.f, 0.f};
-            group_mma(aL, aH, b, d);
-            if (TWO) group_mma(aL, aH, b2, d2);
+            // one token tile: two chains; two tiles: one chain each (the
+            // tiles' MMAs are independent already, and the registers short)
+            if (TWO) {
+              group_mma(aL, aH, b, d);
+              group_mma(aL, aH, b2, d2);
+            } else {
+              group_mma2(aL, aH, b, d);
+            }
             if constexpr (GL >= 1) epilogue(std::integral_constant<int, GL - 1>{}, dp, dp2);
 #pragma unroll
             for (int i = 0; i < 4; ++i) dp[i] = d[i], dp2[i] = d2[i];

@@ -64,6 +64,19 @@ __device__ __forceinline__ void group_mma(const uint32_t *aL, const uint32_t *aH
 #pragma unroll
   for (int j = 1; j < kChunks; ++j) mma16816(d, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
 }
+// As group_mma, in two accumulator chains (even and odd chunks), so that an
+// MMA waits for the result of the one two places earlier only (for kernels
+// with the registers to spare).
+__device__ __forceinline__ void group_mma2(const uint32_t *aL, const uint32_t *aH, const uint32_t *b, float *d) {
+  float e[4];
+  mma16816_z(d, aL[0], aH[0], aL[1], aH[1], b[0], b[1]);
+  mma16816_z(e, aL[2], aH[2], aL[3], aH[3], b[2], b[3]);
+#pragma unroll
+  for (int j = 2; j < kChunks; ++j)
+    mma16816((j & 1) ? e : d, aL[2 * j], aH[2 * j], aL[2 * j + 1], aH[2 * j + 1], b[2 * j], b[2 * j + 1]);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) d[i] += e[i];
+}
 
 // The group-ordered second-plane index (tq_plane2_index): colptr [G + 1]
 // padded to 128 bytes, then 32-byte slots of at most c_capacity entries.
