@@ -216,6 +216,125 @@ __global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t
   }
 }
 
+// ------------------------------------------------ row-staged pack / unpack
+// The same byte layout and status bits as pack_kernel / unpack_kernel, with
+// one CTA per row at a time.  The row's codes move between global and
+// shared memory in 16-byte units (coalesced), and the per-byte encode or
+// decode works on shared memory; the salience rank of each group is formed
+// once per row.  Taken when the code arrays are 16-byte aligned and a row's
+// codes fit in shared memory.
+constexpr int kRowThreads = 256;
+constexpr int kRowMaxK = 49152;  // 2 x 48 KiB of codes per row
+
+__host__ __device__ inline int rows_smem_bytes(int K) { return 2 * K + 4 * (K / kGroup); }
+
+// rk[g]: rank of group g among row n's salient groups, -1 if not salient.
+__device__ __forceinline__ void row_ranks(const uint32_t *sal, int W, int G, int n, int32_t *rk) {
+  for (int g = threadIdx.x; g < G; g += blockDim.x) rk[g] = sal_bit(sal, W, n, g) ? sal_rank(sal, W, n, g) : -1;
+}
+
+__global__ void __launch_bounds__(kRowThreads) pack_rows_kernel(int N, int K, const int8_t *T1, const int8_t *T2,
+                                                               const uint32_t *sal, const int32_t *rowptr,
+                                                               uint8_t *plane1, uint8_t *plane2, uint32_t *status) {
+  extern __shared__ __align__(16) unsigned char smr[];
+  const int G = K / kGroup, W = sal_words_of(K);
+  const int RB = (int)row_bytes_of(K);
+  const int32_t nnz = rowptr[N];
+  int8_t *t1 = reinterpret_cast<int8_t *>(smr), *t2 = t1 + K;
+  int32_t *rk = reinterpret_cast<int32_t *>(smr + 2 * K);
+  uint32_t st = 0;
+  for (int n = blockIdx.x; n < N; n += gridDim.x) {
+    __syncthreads();  // the previous row's shared-memory reads are done
+    row_ranks(sal, W, G, n, rk);
+    const int4 *s1 = reinterpret_cast<const int4 *>(T1 + (int64_t)n * K);
+    for (int i = threadIdx.x; i < K / 16; i += blockDim.x) reinterpret_cast<int4 *>(t1)[i] = __ldcs(s1 + i);
+    if (T2) {
+      const int4 *s2 = reinterpret_cast<const int4 *>(T2 + (int64_t)n * K);
+      for (int i = threadIdx.x; i < K / 16; i += blockDim.x) {
+        const int4 v = __ldcs(s2 + i);
+        reinterpret_cast<int4 *>(t2)[i] = v;
+        // second-plane codes outside the salient groups must be zero
+        if ((v.x | v.y | v.z | v.w) != 0 && !sal_bit(sal, W, n, (16 * i) / kGroup)) st |= TQ_DATA_T2_OUTSIDE;
+      }
+    }
+    __syncthreads();
+    const int64_t p1 = (int64_t)n * RB;
+    const int32_t rp = rowptr[n];
+    for (int b = threadIdx.x; b < RB; b += blockDim.x) {
+      if (b >= G * kGroupBytes) {
+        plane1[p1 + b] = 0;
+        continue;
+      }
+      const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+      const int ntr = pos < kFullBytes ? 5 : kTailTrits;
+      const int k0 = g * kGroup + 5 * pos;
+      plane1[p1 + b] = encode_codes(t1 + k0, ntr, &st);
+      const int r = rk[g];
+      if (r >= 0) {
+        if (T2) {
+          const int64_t j = (int64_t)rp + r;
+          if (j >= 0 && j < nnz)
+            plane2[j * kGroupBytes + pos] = encode_codes(t2 + k0, ntr, &st);
+          else
+            st |= TQ_DATA_BAD_ROWPTR;
+        } else {
+          st |= TQ_DATA_T2_OUTSIDE;
+        }
+      }
+    }
+  }
+  if (st) atomicOr(status, st);
+}
+
+__global__ void __launch_bounds__(kRowThreads) unpack_rows_kernel(int N, int K, const uint8_t *plane1,
+                                                                 const uint8_t *plane2, const uint32_t *sal,
+                                                                 const int32_t *rowptr, int8_t *T1, int8_t *T2,
+                                                                 uint32_t *status) {
+  extern __shared__ __align__(16) unsigned char smr[];
+  const int G = K / kGroup, W = sal_words_of(K);
+  const int RB = (int)row_bytes_of(K);
+  const int32_t nnz = rowptr[N];
+  int8_t *t1 = reinterpret_cast<int8_t *>(smr), *t2 = t1 + K;
+  int32_t *rk = reinterpret_cast<int32_t *>(smr + 2 * K);
+  uint32_t st = 0;
+  for (int n = blockIdx.x; n < N; n += gridDim.x) {
+    __syncthreads();  // the previous row's stores have read shared memory
+    row_ranks(sal, W, G, n, rk);
+    __syncthreads();
+    const int64_t p1 = (int64_t)n * RB;
+    const int32_t rp = rowptr[n];
+    for (int b = threadIdx.x; b < RB; b += blockDim.x) {
+      const uint8_t v = __ldcs(plane1 + p1 + b);
+      if (b >= G * kGroupBytes) {
+        if (v != 0) st |= TQ_DATA_BAD_PAD;
+        continue;
+      }
+      const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
+      const int ntr = pos < kFullBytes ? 5 : kTailTrits;
+      const int k0 = g * kGroup + 5 * pos;
+      decode_to(v, ntr, t1 + k0, &st);
+      if (T2) {
+        const int r = rk[g];
+        const int64_t j = (int64_t)rp + r;
+        if (r >= 0 && plane2 && j >= 0 && j < nnz) {
+          decode_to(plane2[j * kGroupBytes + pos], ntr, t2 + k0, &st);
+        } else {
+          if (r >= 0) st |= TQ_DATA_BAD_ROWPTR;
+          for (int i = 0; i < ntr; ++i) t2[k0 + i] = 0;
+        }
+      }
+    }
+    __syncthreads();
+    int4 *d1 = reinterpret_cast<int4 *>(T1 + (int64_t)n * K);
+    for (int i = threadIdx.x; i < K / 16; i += blockDim.x) __stcs(d1 + i, reinterpret_cast<const int4 *>(t1)[i]);
+    if (T2) {
+      int4 *d2 = reinterpret_cast<int4 *>(T2 + (int64_t)n * K);
+      for (int i = threadIdx.x; i < K / 16; i += blockDim.x) __stcs(d2 + i, reinterpret_cast<const int4 *>(t2)[i]);
+    }
+  }
+  if (st) atomicOr(status, st);
+}
+
 // ------------------------------------------------------ second-plane index
 // One block per group g walks the rows in chunks of blockDim.x, in order;
 // a block-wide count (and, for the fill, an exclusive scan of the row bits)
@@ -385,6 +504,16 @@ cudaError_t launch_check_rowptr(int N, int K, const uint32_t *sal, const int32_t
 cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const uint32_t *sal,
                         const int32_t *rowptr, uint8_t *plane1, uint8_t *plane2, uint32_t *status,
                         cudaStream_t s) {
+  if (K <= kRowMaxK && ((((uintptr_t)T1) | ((uintptr_t)T2)) & 15u) == 0) {
+    const int sm = rows_smem_bytes(K);
+    if (sm > 48 * 1024) {
+      const cudaError_t e = cudaFuncSetAttribute(pack_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+      if (e != cudaSuccess) return e;
+    }
+    pack_rows_kernel<<<std::min(N, 152 * 8), kRowThreads, sm, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2,
+                                                                    status);
+    return cudaGetLastError();
+  }
   pack_kernel<<<std::min(N, 152 * 16), 256, 0, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2, status);
   return cudaGetLastError();
 }
@@ -392,6 +521,16 @@ cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const 
 cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *plane2,
                           const uint32_t *sal, const int32_t *rowptr, int8_t *T1, int8_t *T2,
                           uint32_t *status, cudaStream_t s) {
+  if (K <= kRowMaxK && ((((uintptr_t)T1) | ((uintptr_t)T2)) & 15u) == 0) {
+    const int sm = rows_smem_bytes(K);
+    if (sm > 48 * 1024) {
+      const cudaError_t e = cudaFuncSetAttribute(unpack_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+      if (e != cudaSuccess) return e;
+    }
+    unpack_rows_kernel<<<std::min(N, 152 * 8), kRowThreads, sm, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
+                                                                      status);
+    return cudaGetLastError();
+  }
   unpack_kernel<<<std::min(N, 152 * 16), 256, 0, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
                                                      status);
   return cudaGetLastError();

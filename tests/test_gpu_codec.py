@@ -45,6 +45,41 @@ def test_pack_unpack_bit_exact(H, N, K, frac):
     assert np.array_equal(T2.cpu().numpy(), w.T2)
 
 
+@pytest.mark.parametrize("N,K,offset", [(37, 1024, 1), (9, 4224, 3), (3, 49280, 0)])
+def test_pack_unpack_unstaged_paths(H, N, K, offset):
+    """Code arrays that are not 16-byte aligned (offset into a larger buffer),
+    or rows longer than the row-staged kernels take (K > 49152), go through
+    the per-byte kernels; both must match the oracle bit for bit."""
+    from paper_2609_09240_gb300 import tq
+    w = wl.gen_weights(N, K, 0.2, config=7, proj=N + 3 * K)
+    rp, st = oracle.rowptr(N, K, w.sal)
+    p1_o, p2_o, st = oracle.pack(N, K, w.T1, w.T2, w.sal, rp)
+    assert st == 0
+
+    def codes(a):
+        # a copy of a at `offset` bytes into a device buffer
+        buf = torch.zeros(a.size + 16, dtype=torch.int8, device="cuda")
+        v = buf[offset:offset + a.size]
+        v.copy_(torch.from_numpy(np.ascontiguousarray(a).reshape(-1)))
+        return v
+
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    p1 = torch.empty((N, tq.tq_row_bytes(K)), dtype=torch.uint8, device="cuda")
+    p2 = torch.empty((max(int(rp[N]), 1), 26), dtype=torch.uint8, device="cuda")
+    tq.tq_pack(N, K, codes(w.T1), codes(w.T2), H.dev(w.sal), H.dev(rp), p1, p2, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert np.array_equal(p1.cpu().numpy(), p1_o)
+    assert np.array_equal(p2.cpu().numpy()[:int(rp[N])], p2_o)
+    T1 = codes(np.full(N * K, 7, np.int8))
+    T2 = codes(np.full(N * K, 7, np.int8))
+    tq.tq_unpack(N, K, p1, p2, H.dev(w.sal), H.dev(rp), T1, T2, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert np.array_equal(T1.cpu().numpy().reshape(N, K), w.T1)
+    assert np.array_equal(T2.cpu().numpy().reshape(N, K), w.T2)
+
+
 def test_unpack_reports_corruption_like_oracle(H):
     from paper_2609_09240_gb300 import tq
     N, K = 9, 512
