@@ -223,8 +223,26 @@ __global__ void unpack_kernel(int N, int K, const uint8_t *plane1, const uint8_t
 // decode works on shared memory; the salience rank of each group is formed
 // once per row.  Taken when the code arrays are 16-byte aligned and a row's
 // codes fit in shared memory.
-constexpr int kRowThreads = 256;
+constexpr int kPackThreads = 128;    // pack: up to 16 CTAs (rows in flight) per SM
+constexpr int kUnpackThreads = 256;
 constexpr int kRowMaxK = 49152;  // 2 x 48 KiB of codes per row
+
+// The byte of the five codes row[k0 .. k0 + 4] (a full byte): two 32-bit
+// shared-memory loads and a funnel shift give the codes, their digits
+// (code + 1) come bytewise without carries between bytes, and one dp4a
+// forms sum d_i 3^i.  A code outside {-1, 0, 1} goes through encode_codes,
+// which clamps it and flags the status.
+__device__ __forceinline__ uint8_t encode5(const int8_t *row, int k0, uint32_t *st) {
+  const uint32_t *w = reinterpret_cast<const uint32_t *>(row) + (k0 >> 2);
+  const uint32_t sh = 8u * (uint32_t)(k0 & 3);
+  const uint32_t lo = w[0], hi = w[1];
+  const uint32_t c4 = __funnelshift_r(lo, hi, sh), c5 = (hi >> sh) & 0xFFu;
+  const uint32_t d4 = ((c4 & 0x7F7F7F7Fu) + 0x01010101u) ^ (c4 & 0x80808080u);
+  const uint32_t d5 = ((c5 & 0x7Fu) + 1u) ^ (c5 & 0x80u);
+  if ((((d4 | d5) & 0xFCFCFCFCu) | (d4 & (d4 >> 1) & 0x01010101u) | (d5 & (d5 >> 1) & 1u)) != 0)
+    return encode_codes(row + k0, 5, st);
+  return (uint8_t)__dp4a(d4, 0x1B090301u, 81u * d5);
+}
 
 __host__ __device__ inline int rows_smem_bytes(int K) { return 2 * K + 4 * (K / kGroup); }
 
@@ -233,7 +251,7 @@ __device__ __forceinline__ void row_ranks(const uint32_t *sal, int W, int G, int
   for (int g = threadIdx.x; g < G; g += blockDim.x) rk[g] = sal_bit(sal, W, n, g) ? sal_rank(sal, W, n, g) : -1;
 }
 
-__global__ void __launch_bounds__(kRowThreads) pack_rows_kernel(int N, int K, const int8_t *T1, const int8_t *T2,
+__global__ void __launch_bounds__(kPackThreads) pack_rows_kernel(int N, int K, const int8_t *T1, const int8_t *T2,
                                                                const uint32_t *sal, const int32_t *rowptr,
                                                                uint8_t *plane1, uint8_t *plane2, uint32_t *status) {
   extern __shared__ __align__(16) unsigned char smr[];
@@ -268,13 +286,13 @@ __global__ void __launch_bounds__(kRowThreads) pack_rows_kernel(int N, int K, co
       const int g = b / kGroupBytes, pos = b - g * kGroupBytes;
       const int ntr = pos < kFullBytes ? 5 : kTailTrits;
       const int k0 = g * kGroup + 5 * pos;
-      plane1[p1 + b] = encode_codes(t1 + k0, ntr, &st);
+      plane1[p1 + b] = ntr == 5 ? encode5(t1, k0, &st) : encode_codes(t1 + k0, ntr, &st);
       const int r = rk[g];
       if (r >= 0) {
         if (T2) {
           const int64_t j = (int64_t)rp + r;
           if (j >= 0 && j < nnz)
-            plane2[j * kGroupBytes + pos] = encode_codes(t2 + k0, ntr, &st);
+            plane2[j * kGroupBytes + pos] = ntr == 5 ? encode5(t2, k0, &st) : encode_codes(t2 + k0, ntr, &st);
           else
             st |= TQ_DATA_BAD_ROWPTR;
         } else {
@@ -286,7 +304,7 @@ __global__ void __launch_bounds__(kRowThreads) pack_rows_kernel(int N, int K, co
   if (st) atomicOr(status, st);
 }
 
-__global__ void __launch_bounds__(kRowThreads) unpack_rows_kernel(int N, int K, const uint8_t *plane1,
+__global__ void __launch_bounds__(kUnpackThreads) unpack_rows_kernel(int N, int K, const uint8_t *plane1,
                                                                  const uint8_t *plane2, const uint32_t *sal,
                                                                  const int32_t *rowptr, int8_t *T1, int8_t *T2,
                                                                  uint32_t *status) {
@@ -510,7 +528,7 @@ cudaError_t launch_pack(int N, int K, const int8_t *T1, const int8_t *T2, const 
       const cudaError_t e = cudaFuncSetAttribute(pack_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
       if (e != cudaSuccess) return e;
     }
-    pack_rows_kernel<<<std::min(N, 152 * 8), kRowThreads, sm, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2,
+    pack_rows_kernel<<<std::min(N, 152 * 16), kPackThreads, sm, s>>>(N, K, T1, T2, sal, rowptr, plane1, plane2,
                                                                     status);
     return cudaGetLastError();
   }
@@ -527,7 +545,7 @@ cudaError_t launch_unpack(int N, int K, const uint8_t *plane1, const uint8_t *pl
       const cudaError_t e = cudaFuncSetAttribute(unpack_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
       if (e != cudaSuccess) return e;
     }
-    unpack_rows_kernel<<<std::min(N, 152 * 8), kRowThreads, sm, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
+    unpack_rows_kernel<<<std::min(N, 152 * 8), kUnpackThreads, sm, s>>>(N, K, plane1, plane2, sal, rowptr, T1, T2,
                                                                       status);
     return cudaGetLastError();
   }
