@@ -840,7 +840,7 @@ def sub_codec(dev, peak, reps=5):
         items.append((pw, g["T1"], g["T2"], T1o, T2o, Wd, idx, st))
         side = pw.salience.numel() * 4 + pw.rowptr.numel() * 4
         planes = pw.plane1.numel() + nnz * 26
-        bytes_["pack"] += N * K + nnz * 128 + side + planes
+        bytes_["pack"] += 2 * N * K + side + planes
         bytes_["unpack"] += planes + side + 2 * N * K
         bytes_["plane2_index"] += nnz * 26 + nnz * 2 + side + idx.numel() * 4
         bytes_["dequantize"] += pw.packed_bytes() + 2 * N * K
@@ -876,8 +876,9 @@ def sub_codec(dev, peak, reps=5):
     status = sum(int(it[-1].item()) for it in items)
     return {"workload": "qwen3-8b one layer's 7 projections (193 M weights, 10 % salient groups)",
             "kernels": out, "data_status": status,
-            "bytes": "algorithmic: pack reads the int8 T1 codes, T2 of the salient groups, salience and rowptr and "
-                     "writes plane 1 and plane 2; unpack the reverse with full int8 T1 and T2; the index reads "
+            "bytes": "algorithmic: pack reads the int8 T1 and T2 codes (all of T2: codes outside the salient groups "
+                     "must be checked to be zero), salience and rowptr and writes plane 1 and plane 2; unpack the "
+                     "reverse with full int8 T1 and T2; the index reads "
                      "plane 2, s2, salience and rowptr and writes the index; dequantize reads the packed weight "
                      "and writes fp16 W-hat",
             "l2": "no flush: a layer's int8 codes (386 MB) and fp16 W-hat (386 MB) exceed L2"}
