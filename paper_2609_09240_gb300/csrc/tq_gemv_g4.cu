@@ -257,16 +257,13 @@ __device__ __forceinline__ void decode_stage(const unsigned char *dyn, int buf, 
 #pragma unroll
     for (int m = 0; m < 5; ++m) {
       const int j = 5 * i + m;
-      // one token: lanes of zero columns keep zero registers (no shared-
-      // memory traffic; measured slower for two tokens, whose lanes load
-      // the zero block); the registers are never cleared, as a predicated
-      // load into a fresh value would cost a clearing move per MMA
-      // (measured 0.518 ms per Qwen3-8B step against 0.541)
+      // lanes of zero columns keep zero registers (no shared-memory
+      // traffic); the registers are never cleared, as a predicated load into
+      // a fresh value would cost a clearing move per MMA (one token: 0.518
+      // ms per Qwen3-8B step against 0.541; two tokens: 0.626 against 0.640
+      // with the zero lanes loading a zero block)
       uint32_t b0, b1;
-      if (MB == 2) {
-        const uint4 q = *reinterpret_cast<const uint4 *>(bq + (j >> 1) * 64);
-        b0 = (j & 1) ? q.z : q.x, b1 = (j & 1) ? q.w : q.y;
-      } else {
+      {
         uint32_t(&r)[4] = bz[(j >> 1) % kBSets];
         if ((j & 1) == 0) ld_b_real(r, bq + (j >> 1) * 64, realB);
         b0 = (j & 1) ? r[2] : r[0], b1 = (j & 1) ? r[3] : r[1];
