@@ -110,12 +110,12 @@ size_t pad256(size_t b) { return (b + 255) / 256 * 256; }
 // Workspace bytes of one problem for a pass over M <= 16 tokens.  (A call
 // whose more than 8 tokens have to run as two passes of at most 8 places the
 // smaller 8-token layout in the same space.)
-size_t problem_ws_bytes(int M, int N, int K) {
+size_t problem_ws_bytes(int M, int N, int K, bool general = false) {
   size_t b, cs, y2;
   mma_workspace_parts(M, N, K, &b, &cs, &y2);
   // + the tensor maps of plane 1, s1, off; with M <= 2 the operands of the
   // one-group-per-lane kernel follow
-  const size_t g4 = M <= 2 ? (size_t)g4_workspace_bytes(M, N, K) : 0;
+  const size_t g4 = M <= 2 && !general ? (size_t)g4_workspace_bytes(M, N, K) : 0;
   return pad256(b) + pad256(cs) + pad256(y2) + 512 + g4;
 }
 
@@ -141,7 +141,7 @@ tq_status place(BatchParams &bp, unsigned char *ws, size_t ws_bytes) {
     Problem &P = bp.prob[i];
     P.tile_begin = tiles;
     tiles += (P.N + rows - 1) / rows;
-    const size_t tot = problem_ws_bytes(bp.M, P.N, P.K);
+    const size_t tot = problem_ws_bytes(bp.M, P.N, P.K, bp.general != 0);
     if (off + tot > ws_bytes) return TQ_ERR_SHAPE;
     size_t b, cs, y2;
     mma_workspace_parts(bp.M, P.N, P.K, &b, &cs, &y2);
@@ -176,6 +176,7 @@ tq_status run_batch(BatchParams &bp, unsigned char *ws, size_t ws_bytes, cudaStr
   thread_local BatchParams hi;  // large: kept off the stack
   hi = bp;
   hi.M = bp.M - 8;
+  hi.general = 1;  // the workspace holds the 8-token layout, not the one-group-per-lane operands
   for (int i = 0; i < hi.count; ++i) {
     Problem &P = hi.prob[i];
     P.x += (int64_t)8 * P.K;

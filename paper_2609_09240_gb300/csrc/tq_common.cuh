@@ -54,7 +54,8 @@ struct BatchParams {
   int32_t total_tiles;  // sum of tiles over problems
   int32_t out_f32;      // y is fp32 (else fp16)
   int32_t g4_split;     // M <= 2: target groups per work unit of a 256-row tile (0: whole tiles)
-  int32_t reserved_;
+  int32_t general;      // nonzero: the general decode kernels even for M <= 2 (the one-group-per-lane
+                        // kernel's operands are then not in the workspace)
   Problem prob[TQ_MAX_BATCH];
 };
 

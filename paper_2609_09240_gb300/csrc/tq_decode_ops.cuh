@@ -134,6 +134,7 @@ __device__ __forceinline__ void mma16816_z(float *d, uint32_t a0, uint32_t a1, u
 // slots of all stages come first, then the C/S blocks.
 namespace g4 {
 constexpr int kRows = 256;  // tile rows
+constexpr int kMaxM = 2;    // most tokens of the one-group-per-lane kernel
 __host__ __device__ constexpr int stage_groups(int M) { return M == 1 ? 8 : 4; }
 __host__ __device__ constexpr int words(int SG) { return SG == 8 ? 13 : 7; }  // window words per lane and row
 __host__ __device__ constexpr int pairs(int SG) { return (5 * words(SG) + 1) / 2; }  // 16-byte chunks per slice
@@ -145,6 +146,8 @@ __host__ __device__ inline int64_t b_bytes(int M, int K) {
   return (int64_t)nstages(K, stage_groups(M)) * 2 * slice_bytes(stage_groups(M));
 }
 __host__ __device__ inline int64_t cs_bytes(int M, int K) { return (int64_t)nstages(K, stage_groups(M)) * kCSStage; }
+// Whether a batch runs the one-group-per-lane kernel.
+__host__ __device__ inline bool takes(const BatchParams &bp) { return bp.M >= 1 && bp.M <= kMaxM && !bp.general; }
 // Split tiles (several CTAs per tile): one arrival counter per (tile,
 // decode warp), after the C/S blocks.
 constexpr int kMaxWarps = 16;

@@ -978,7 +978,7 @@ int g4_split_for(const BatchParams &bp, int num_sms) {
 // y2, tickets) and second plane have been launched on the same stream.
 cudaError_t launch_gemv_g4(const BatchParams &bp, int num_sms, cudaStream_t s) {
   thread_local g4::Sched sc;
-  if (bp.M < 1 || bp.M > 2 || bp.g4_split < 0) return cudaErrorInvalidValue;
+  if (!g4::takes(bp) || bp.g4_split < 0) return cudaErrorInvalidValue;
   const int ctas = min(num_sms, 256);
   const int SG = g4::stage_groups(bp.M);
   sc.split = bp.g4_split;

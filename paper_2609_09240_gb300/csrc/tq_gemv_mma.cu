@@ -197,7 +197,7 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   // last call's decode kernel, whose workspace this may be) has finished
   // and its writes are visible past this point
   grid_dep_wait();
-  const bool g4_shared = bp.M <= 2 && bp.g4_split > 0;  // split tiles add their partial sums into y2
+  const bool g4_shared = g4::takes(bp) && bp.g4_split > 0;  // split tiles add their partial sums into y2
   // (the sequence kernel, g4_split < 0, adds every partial sum into y2)
   if (P.nnz > 0 || g4_shared || bp.g4_split < 0) {
     // y2 starts at zero (the indexed second-plane kernel adds into it)
@@ -254,7 +254,8 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   // with M <= 2 the one-group-per-lane kernel runs; its operands cover whole
   // stages of SG groups (groups past G get zero activations and C/S)
   const int SG = g4::stage_groups(MB);
-  const int Gx = MB <= 2 ? SG * g4::nstages(P.K, SG) : G;
+  const bool g4ops = g4::takes(bp);
+  const int Gx = g4ops ? SG * g4::nstages(P.K, SG) : G;
   const bool live = task < Gx * MB;
   const int g = live ? task / MB : 0, m = live ? task % MB : 0;
   const bool real = live && g < G;
@@ -312,7 +313,7 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
   // token m; 8-group stages, lane (g % 8) / 2 and the lane's group g % 2
   const int gs = g / SG, gp = g % SG;
   const int g4c = SG == 8 ? gp >> 1 : gp, g4sl = SG == 8 ? gp & 1 : m;
-  if (MB <= 2) {
+  if (g4ops) {
     unsigned char *g4b = P.wsB + P.map_off + kMapSlotBytes;
     float *g4cs = reinterpret_cast<float *>(g4b + g4::pad256(g4::b_bytes(MB, P.K)));
     unsigned char *g4dst = g4b + (int64_t)(gs * 2 + g4sl) * g4::slice_bytes(SG) + g4c * 16;
@@ -1521,7 +1522,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   // the batch with the M <= 2 kernel's tile split filled in
   thread_local BatchParams bp;
   bp = bp_in;
-  bp.g4_split = bp.M <= 2 ? g4_split_for(bp, num_sms_mm()) : 1;
+  bp.g4_split = g4::takes(bp) ? g4_split_for(bp, num_sms_mm()) : 1;
   thread_local mm::Sched sc;
   if (bp.M < 1 || bp.M > 16 || mm::Layout(bp.M).used2 > mm::kArena2) return cudaErrorInvalidValue;
   const int ctas = min(num_sms_mm(), 256);
@@ -1551,7 +1552,7 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
     any2 = any2 || bp.prob[i].nnz > 0;
   }
   // one or two tokens: the one-group-per-lane kernel (tq_gemv_g4.cu)
-  const bool g4path = bp.M <= 2;
+  const bool g4path = g4::takes(bp);
   thread_local mm::MapTemplates mt;
   if (cudaError_t e = build_templates(bp, g4path, mt)) return e;
   // second plane: the indexed kernel when every weight with a second plane

@@ -160,11 +160,13 @@ def test_batched_max_problems(H, M, index):
 
 
 @pytest.mark.parametrize("N,K,frac", [(1, 128, 1.0), (129, 256, 0.5), (300, 9728, 0.1), (700, 4096, 0.3)])
-@pytest.mark.parametrize("M", [1, 3, 8, 12])
+@pytest.mark.parametrize("M", [1, 3, 8, 9, 10, 12])
 def test_second_plane_without_index(H, N, K, frac, M):
     """Weights packed without the second-plane index: the span kernel groups
     the records itself (more than 8 tokens then run as two passes of at most
-    8, the indexed path takes up to 16 in one pass)."""
+    8, the indexed path takes up to 16 in one pass; a second pass of one or
+    two tokens stays on the general kernels, whose layout the workspace
+    holds)."""
     run_case(H, N, K, frac, M, f32=True, proj=40 + N, index=False)
 
 
