@@ -655,6 +655,20 @@ __device__ __forceinline__ void second_plane_share(const Problem &P, int cta, in
   }
 }
 
+// The CTA's share of problem P's second-plane records (the tiles that
+// second_plane_share gives it) into L2, one bulk prefetch: they are weights,
+// so they can be fetched while the problem before P still runs.
+__device__ __forceinline__ void prefetch_second_plane(const Problem &P, int cta, int ctas) {
+  const int G = P.K / kGroup;
+  const int T2 = __ldg(P.p2idx + G) >> 4;
+  const int lo = (int)((int64_t)T2 * cta / ctas), hi = (int)((int64_t)T2 * (cta + 1) / ctas);
+  if (hi <= lo) return;
+  const unsigned char *slots = reinterpret_cast<const unsigned char *>(P.p2idx) + mm::c_slot_off(P.K);
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(slots + (int64_t)lo * 512),
+               "r"((uint32_t)(hi - lo) * 512u)
+               : "memory");
+}
+
 template <bool F32>
 __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
     gemv_seq_kernel(const __grid_constant__ BatchParams bp, int32_t barrier_extra) {
@@ -688,6 +702,8 @@ __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
     SeqWalk w(&bp, blockIdx.x, gridDim.x);
     for (bool more = true; more; more = w.next_problem()) {
       const Problem &P = w.P();
+      if (warp == 0 && lane == 0 && w.p + 1 < bp.count && bp.prob[w.p + 1].nnz > 0)
+        prefetch_second_plane(bp.prob[w.p + 1], blockIdx.x, gridDim.x);
       if (P.nnz > 0) second_plane_share<WD>(P, blockIdx.x, gridDim.x, warp, lane, tag);
       bool ok = true;
       for (; w.has_stage(); w.next_stage()) {
