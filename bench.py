@@ -225,12 +225,17 @@ DECODE_SOURCES = ("tq_common.cuh", "tq_decode_ops.cuh", "tq_gemv_g4.cu", "tq_gem
 
 
 def kernel_hash():
+    """sha256 (16 hex digits) of the decode kernels' sources without their
+    // comments and blank lines, so that a comment edit keeps the counters"""
     import hashlib
 
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_09240_gb300", "csrc")
     for f in DECODE_SOURCES:
-        h.update(open(os.path.join(csrc, f), "rb").read())
+        for line in open(os.path.join(csrc, f), encoding="utf-8"):
+            code = line.split("//", 1)[0].rstrip()
+            if code:
+                h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
 
 
