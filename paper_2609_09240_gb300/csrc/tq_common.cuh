@@ -56,6 +56,8 @@ struct BatchParams {
   int32_t g4_split;     // M <= 2: target groups per work unit of a 256-row tile (0: whole tiles)
   int32_t general;      // nonzero: the general decode kernels even for M <= 2 (the one-group-per-lane
                         // kernel's operands are then not in the workspace)
+  int32_t g4_only;      // nonzero: only the one-group-per-lane kernels read the activation operands
+                        // (the prep kernel writes no general-layout fragments or C/S)
   Problem prob[TQ_MAX_BATCH];
 };
 

@@ -354,7 +354,7 @@ __global__ void gemv_mma_prep_kernel(const __grid_constant__ BatchParams bp, con
       g4q[2 + g4sl] = S;
     }
   }
-  if (!real) return;
+  if (!real || bp.g4_only) return;
   // the general decode kernels' per-group layout: lane position c's two
   // window words give W, W' of their bytes (words 0..15) and the four
   // fifth-slot words (16..19), as chunk pairs of 16 bytes
@@ -1575,6 +1575,9 @@ static cudaError_t launch_mm_one(const BatchParams &bp_in, cudaStream_t s) {
   }
   const int sg = g4::stage_groups(bp.M);
   const int gtasks = (g4path ? sg * ((gmax + sg - 1) / sg) : gmax) * bp.M;
+  // the general layout is read by the general decode kernels and by the
+  // second-plane kernels other than the one-token indexed one
+  bp.g4_only = g4path && (!any2 || (all_idx && bp.M == 1)) ? 1 : 0;
   cudaError_t e = launch_prep(bp, mt, counter, gtasks, s);
   if (e != cudaSuccess) return e;
   // more than 8 tokens in one pass needs every second plane indexed (the
