@@ -180,16 +180,16 @@ __device__ __forceinline__ void decode_word(uint32_t x, uint32_t tag, uint32_t *
   a[9] = mm::prmt(x, 0x44444444u, 0x4342u);
 }
 
-// One token's activation registers of an MMA pair: a 16-byte shared-memory
-// load by the lanes that hold real slots; the other lanes leave r as it is
-// (zero from the start of the kernel), so no register needs clearing.
+// The activation registers of an MMA pair: a 16-byte shared-memory load by
+// the lanes that hold real slots; the other lanes leave r as it is (zero
+// from the start of the kernel), so no register needs clearing.
 __device__ __forceinline__ void ld_b_real(uint32_t (&r)[4], const unsigned char *addr, bool real) {
   asm volatile(
       "{\n.reg .pred p;\nsetp.ne.b32 p, %5, 0;\n@p ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];\n}"
       : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3])
       : "r"(smem_u32(addr)), "r"((uint32_t)real));
 }
-constexpr int kBSets = 4;  // one-token activation register sets (pairs p, p + 1, ... in rotation)
+constexpr int kBSets = 4;  // activation register sets (pairs p, p + 1, ... in rotation)
 
 // Workspace addresses of a problem's activation slots and C/S (after the
 // general decode path's 512-byte map slot).
@@ -475,7 +475,7 @@ __global__ void __launch_bounds__((WD + 1) * 32, 1)
       for (int h = 0; h < 2; ++h)
 #pragma unroll
         for (int k = 0; k < MB; ++k) y[t][h][k] = 0.f;
-    uint32_t bz[kBSets][4] = {};  // one token's activation registers (zero-column lanes: zero throughout)
+    uint32_t bz[kBSets][4] = {};  // activation registers (zero-column lanes: zero throughout)
     uint32_t buf = 0, phase = 0;
     for (Walk<SG> w(&bp, sc.split, t_begin, t_end); w.valid(); w.next()) {
       const bool ok = __all_sync(0xffffffffu, mm::wait_or_abort(&bars->full[buf], phase, abort_));
