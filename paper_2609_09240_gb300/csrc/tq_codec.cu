@@ -318,6 +318,10 @@ __global__ void __launch_bounds__(kUnpackThreads) unpack_rows_kernel(int N, int 
   for (int n = blockIdx.x; n < N; n += gridDim.x) {
     __syncthreads();  // the previous row's stores have read shared memory
     row_ranks(sal, W, G, n, rk);
+    // second-plane codes are zero outside the salient groups: the row starts
+    // zeroed by 16-byte stores, and only salient groups are decoded into it
+    if (T2)
+      for (int i = threadIdx.x; i < K / 16; i += blockDim.x) reinterpret_cast<int4 *>(t2)[i] = make_int4(0, 0, 0, 0);
     __syncthreads();
     const int64_t p1 = (int64_t)n * RB;
     const int32_t rp = rowptr[n];
@@ -334,12 +338,10 @@ __global__ void __launch_bounds__(kUnpackThreads) unpack_rows_kernel(int N, int 
       if (T2) {
         const int r = rk[g];
         const int64_t j = (int64_t)rp + r;
-        if (r >= 0 && plane2 && j >= 0 && j < nnz) {
+        if (r >= 0 && plane2 && j >= 0 && j < nnz)
           decode_to(plane2[j * kGroupBytes + pos], ntr, t2 + k0, &st);
-        } else {
-          if (r >= 0) st |= TQ_DATA_BAD_ROWPTR;
-          for (int i = 0; i < ntr; ++i) t2[k0 + i] = 0;
-        }
+        else if (r >= 0)
+          st |= TQ_DATA_BAD_ROWPTR;
       }
     }
     __syncthreads();
