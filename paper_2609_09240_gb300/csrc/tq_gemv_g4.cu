@@ -741,7 +741,7 @@ __global__ void __launch_bounds__((kWD1 + 1) * 32, 1)
             *abort_ = 1;
             break;
           }
-          __nanosleep(128);
+          __nanosleep(32);  // 1.603 ms per Qwen3-8B step against 1.610 with 128 ns (spinning: 1.611)
         }
         __threadfence();
       }
