@@ -34,3 +34,24 @@ def test_single_process_passthrough():
 
     assert bench.max_over_ranks(3.25, None, "cpu") == 3.25
     assert bench.whole_job_rate(1.79e9, 1, 0.73) == pytest.approx(1.79e9 / 0.73e-3 / 1e9)
+
+
+def test_kernel_hash_ignores_comments(tmp_path, monkeypatch):
+    """The key of the committed traffic summary: a // comment or blank line
+    added to a decode source keeps it, a changed line of code does not."""
+    import shutil
+
+    import bench
+
+    csrc = tmp_path / "paper_2609_09240_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for f in bench.DECODE_SOURCES:
+        shutil.copy(os.path.join(bench.ROOT, "paper_2609_09240_gb300", "csrc", f), csrc / f)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.kernel_hash()
+    src = csrc / "tq_gemv_g4.cu"
+    text = src.read_text()
+    src.write_text("// a note\n\n" + text.replace("\n", "  // trailing\n", 1))
+    assert bench.kernel_hash() == h0
+    src.write_text(text.replace("kP2rTiles = 8;", "kP2rTiles = 9;", 1))
+    assert "kP2rTiles = 9;" in src.read_text() and bench.kernel_hash() != h0
